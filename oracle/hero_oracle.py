@@ -1,0 +1,354 @@
+"""Plain float64 CPU oracle of HeRo's history-aware routed FFN stack.
+
+TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and bench.py's
+cpu_baseline leg may import or run this module; the CUDA product path never
+does, and this module imports nothing from the product package.
+
+What it computes (paper "Do Dynamic Routers Need Memory? HeRo", Sec. 3):
+for each routed block j = 1..L_R and each token, in the paper's order,
+    h_bar   = h + P_j                                   Eq. 1 (attention stand-in)
+    delta, d, gamma                                     Eqs. 7-8 (transition features)
+    x_path = [r, q_rem, d, gamma, p_hist, m_hist]       Eqs. 4, 6
+    z_h = W_hu SiLU(W_hd RMSNorm(h_bar))                Eq. 5
+    z_a = FFN_path(x_path);  s = [z_h; z_a]             Eq. 9
+    q, k, v = W_q s, W_k s, W_v s                       Eq. 10
+    c = phi(q)^T S / (phi(q)^T zeta + eps)              Eq. 11 (read before write)
+    nu = 0 (j = 1) | 1 - cos(W_n s, W_c c)              Eq. 13
+    a = f_theta([s; c; nu]); p_hist = sigma(a/T_hist)   Eq. 14
+    m_hist = m_hist * p_hist                            Eq. 15
+    b = f_psi(h_bar);  g = sigma(a + b)                 Eq. 16
+    S = rho S + phi(k) v^T; zeta = rho zeta + phi(k)    Eq. 12, rho = sigma(eta_j)
+    u = LN_ffn(h_bar)                                   Eq. 1
+    h = h_bar + g FFN(u)          if g >= tau_exec      Eq. 3
+        h_bar + (1-g) Adapter(u)  otherwise             Eqs. 2-3
+Equation numbers count the displayed equations of Sec. 3 in order
+(1 dense_attention, 2 adapter, 3 ffn_route, 4 path_vector, 5 hidden encoder,
+6 depth features, 7 transition, 8 transition_features, 9 router_state,
+10 q/k/v, 11 memory_read, 12 memory_update, 13 nu, 14 history head,
+15 cumulative history, 16 final_gate).
+
+Readings where the paper is silent (each listed in the design notes):
+  * FFN = Llama SwiGLU W_down(SiLU(W_gate u) * W_up u), no biases.
+  * RMSNorm(h) = h / sqrt(mean(h^2) + rms_eps) * gain; the router's RMSNorm has its
+    own shared gain.  FFN_path, f_theta, f_psi = Linear+bias -> SiLU -> Linear+bias;
+    matrices written without a bias in the paper (W_hd, W_hu, W_q, W_k, W_v, W_n,
+    W_c, W_1, W_2) have none.
+  * eps = 1e-6 in Eq. 8, Eq. 11 and the cosine of Eq. 13.
+  * phi(x) = ELU(x) + 1 with alpha = 1.
+  * decisions: g >= tau_exec -> FFN (ties go to the FFN).
+  * precision contract for bf16 workloads: values are rounded to bf16 (nearest,
+    ties to even) exactly at (i) every parameter (done by the input generator),
+    (ii) the operands of the router's d-wide contraction: bf16(h_bar) and
+    bf16(W_hd diag(gain_r)) for the encoder (the row scale 1/rms is applied after
+    the contraction, exact in real arithmetic), bf16(h_bar) for f_psi's first
+    layer, (iii) u = LN_ffn(h_bar), the FFN and adapter input, (iv) the SwiGLU
+    product entering W_down, (v) the adapter hidden SiLU(W_1 u) entering W_2.
+    Everything else is float64 here.  f32 workloads round nowhere.
+
+Modes: "route" (the method), "force" (decisions taken from mask_in, g still
+computed and used as branch scale), "dense" (router skipped, every token through
+the FFN with scale 1: the dense SwiGLU stack).
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import Callable, Dict, List, Optional
+
+import numpy as np
+
+
+# ---------------------------------------------------------------------------
+# Elementary functions
+# ---------------------------------------------------------------------------
+
+def bf16_round(x: np.ndarray) -> np.ndarray:
+    """Nearest bf16 value of each float64 element, ties to even (8 significant bits).
+
+    Written from the bf16 format definition: 1 sign, 8 exponent and 7 fraction bits,
+    the same exponent range as IEEE binary32 (subnormal spacing 2^-133).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)                        # x = m * 2^e, 0.5 <= |m| < 1
+    e = np.maximum(e, -125)                   # below 2^-126 the spacing stays 2^-133
+    spacing = np.ldexp(1.0, e - 8)            # 8 significant bits
+    with np.errstate(invalid="ignore"):
+        out = np.rint(x / spacing) * spacing  # np.rint rounds half to even
+    return np.where(np.isfinite(x), out, x)
+
+
+def _identity(x: np.ndarray) -> np.ndarray:
+    return x
+
+
+def sigmoid(x: np.ndarray) -> np.ndarray:
+    """Logistic function sigma(x) = 1 / (1 + exp(-x))."""
+    x = np.asarray(x, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        return 1.0 / (1.0 + np.exp(-x))
+
+
+def silu(x: np.ndarray) -> np.ndarray:
+    """SiLU(x) = x * sigma(x)."""
+    return x * sigmoid(x)
+
+
+def phi(x: np.ndarray) -> np.ndarray:
+    """Positive feature map phi(x) = ELU(x) + 1 (Sec. 3.2, before Eq. 11), alpha = 1."""
+    x = np.asarray(x, dtype=np.float64)
+    return np.where(x > 0, x + 1.0, np.exp(np.minimum(x, 0.0)))
+
+
+def rms_norm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
+    """RMSNorm over the last axis: x / sqrt(mean(x^2) + eps) * gain."""
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * gain
+
+
+def _mlp2(x, w1, b1, w2, b2):
+    """Linear+bias -> SiLU -> Linear+bias (the two-layer heads and FFN_path)."""
+    return silu(x @ w1.T + b1) @ w2.T + b2
+
+
+# ---------------------------------------------------------------------------
+# Configuration and parameters
+# ---------------------------------------------------------------------------
+
+@dataclass
+class OracleConfig:
+    n_layers: int
+    d_model: int
+    d_ff: int
+    d_r: int
+    d_m: int
+    d_h: int = 48
+    d_a: int = 16
+    d_enc: int = 256
+    d_head: int = 256
+    d_path: int = 16
+    rms_eps: float = 1e-5
+    eps: float = 1e-6
+    t_hist: float = 0.9
+    dtype: str = "f32"
+
+    @staticmethod
+    def from_stack(c) -> "OracleConfig":
+        return OracleConfig(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a,
+                            c.d_enc, c.d_head, c.d_path, c.rms_eps, c.eps, c.t_hist, c.dtype)
+
+
+def _f64(a) -> np.ndarray:
+    """Decode a parameter/input array (float32, float64, or uint16 bf16 bits) to float64."""
+    a = np.asarray(a)
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
+# ---------------------------------------------------------------------------
+# One routed block, step by step (Sec. 3.1-3.2)
+# ---------------------------------------------------------------------------
+
+def transition_features(j: int, h_bar, h_bar_prev, delta_prev, d_prev, eps):
+    """Eqs. 7-8: delta_j = h_bar_j - h_bar_{j-1} (delta_1 = 0), d_j = ||delta_j||,
+    gamma_j = <delta_j, delta_{j-1}> / (d_j d_{j-1} + eps) for j > 2, else 0."""
+    if j == 1:
+        delta = np.zeros_like(h_bar)
+    else:
+        delta = h_bar - h_bar_prev
+    d = np.sqrt(np.sum(delta * delta, axis=1))
+    if j > 2:
+        gamma = np.sum(delta * delta_prev, axis=1) / (d * d_prev + eps)
+    else:
+        gamma = np.zeros_like(d)
+    return delta, d, gamma
+
+
+def path_vector(j: int, L: int, d, gamma, p_prev, m_prev):
+    """Eq. 4 with Eq. 6: [r_j, q_rem_j, d_j, gamma_j, p_hist_{j-1}, m_hist_{j-1}]."""
+    T = d.shape[0]
+    r = np.full(T, j / L)
+    q_rem = np.full(T, (L - j) / L)
+    return np.stack([r, q_rem, d, gamma, p_prev, m_prev], axis=1)
+
+
+def hidden_encoder(h_bar, w, cfg: OracleConfig, R):
+    """Eq. 5: z_h = W_hu SiLU(W_hd RMSNorm(h_bar)).
+
+    RMSNorm(h) = (h * gain_r) / rms(h); the contraction is written as
+    (1/rms) * (W_hd diag(gain_r)) h so that the bf16 operand rounding of the
+    precision contract applies to bf16(h_bar) and bf16(W_hd diag(gain_r)).
+    """
+    rinv = 1.0 / np.sqrt(np.mean(h_bar * h_bar, axis=1) + cfg.rms_eps)
+    w_enc = R(w["w_hd"] * w["r_norm_g"][None, :])
+    pre = rinv[:, None] * (R(h_bar) @ w_enc.T)
+    return silu(pre) @ w["w_hu"].T
+
+
+def path_encoder(x_path, w):
+    """Eq. 9, first line: z_a = FFN_path(x_path) (Linear+bias, SiLU, Linear+bias)."""
+    return _mlp2(x_path, w["path_w1"], w["path_b1"], w["path_w2"], w["path_b2"])
+
+
+def memory_read(fq, S, zeta, eps):
+    """Eq. 11: c = phi(q)^T S / (phi(q)^T zeta + eps), S[t] indexed [key m, value n]."""
+    num = np.einsum("tm,tmn->tn", fq, S)
+    den = np.einsum("tm,tm->t", fq, zeta)
+    return num / (den + eps)[:, None]
+
+
+def memory_write(S, zeta, fk, v, rho):
+    """Eq. 12: S = rho S + phi(k) v^T;  zeta = rho zeta + phi(k)."""
+    S_new = rho * S + np.einsum("tm,tn->tmn", fk, v)
+    zeta_new = rho * zeta + fk
+    return S_new, zeta_new
+
+
+def history_dissimilarity(j: int, s, c, w, eps):
+    """Eq. 13: nu_1 = 0; for j > 1, nu_j = 1 - cos(W_n s, W_c c)."""
+    if j == 1:
+        return np.zeros(s.shape[0])
+    a = s @ w["w_n"].T
+    b = c @ w["w_c"].T
+    cos = np.sum(a * b, axis=1) / (np.linalg.norm(a, axis=1) * np.linalg.norm(b, axis=1) + eps)
+    return 1.0 - cos
+
+
+def history_head(s, c, nu, w):
+    """Eq. 14, first part: a = f_theta([s; c; nu]) (scalar per token)."""
+    x = np.concatenate([s, c, nu[:, None]], axis=1)
+    return _mlp2(x, w["th_w1"], w["th_b1"], w["th_w2"], w["th_b2"])[:, 0]
+
+
+def local_head(h_bar, w, R):
+    """Eq. 16, first part: b = f_psi(h_bar); its first layer reads bf16(h_bar) in bf16."""
+    return _mlp2(R(h_bar), w["ps_w1"], w["ps_b1"], w["ps_w2"], w["ps_b2"])[:, 0]
+
+
+def swiglu_ffn(u, wl, R):
+    """Frozen FFN (Llama SwiGLU): W_down (SiLU(W_gate u) * W_up u)."""
+    act = R(silu(u @ wl["w_gate"].T) * (u @ wl["w_up"].T))
+    return act @ wl["w_down"].T
+
+
+def adapter(u, wl, R):
+    """Eq. 2: Adapter(u) = W_2 SiLU(W_1 u)."""
+    return R(silu(u @ wl["ad_w1"].T)) @ wl["ad_w2"].T
+
+
+# ---------------------------------------------------------------------------
+# The stack
+# ---------------------------------------------------------------------------
+
+_LAYER_KEYS = ("ffn_norm_g", "w_gate", "w_up", "w_down", "ad_w1", "ad_w2")
+_SHARED_KEYS = ("r_norm_g", "w_hd", "w_hu", "path_w1", "path_b1", "path_w2", "path_b2",
+                "w_q", "w_k", "w_v", "w_n", "w_c", "th_w1", "th_b1", "th_w2", "th_b2",
+                "ps_w1", "ps_b1", "ps_w2", "ps_b2")
+
+
+def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, attn_delta,
+                     tau: float, mode: str = "route", mask_in=None,
+                     branch_scale: str = "gate", record: bool = False,
+                     hooks: Optional[Dict[str, Callable]] = None) -> Dict[str, object]:
+    """Run the routed FFN stack on tokens h_in [T, d].
+
+    attn_delta: [L, T, d] attention stand-in (None = zero).
+    mode: "route" | "force" (mask_in [L, T] gives decisions) | "dense".
+    branch_scale: "gate" (Eq. 3: g and 1 - g) or "one" (unscaled branches).
+    Returns h_out [T, d], gate [L, T], mask [L, T] (uint8), counts [L] (FFN tokens)
+    and, if record, per-layer intermediates under "layers".
+    """
+    if mode not in ("route", "force", "dense"):
+        raise ValueError(mode)
+    if mode == "force" and mask_in is None:
+        raise ValueError("force mode needs mask_in")
+    R = bf16_round if cfg.dtype == "bf16" else _identity
+    hk = hooks or {}
+    L = cfg.n_layers
+    h = _f64(h_in)
+    T = h.shape[0]
+    w = {k: _f64(weights[k]) for k in _SHARED_KEYS}
+    eta = _f64(weights["eta"])
+
+    S = np.zeros((T, cfg.d_m, cfg.d_m))
+    zeta = np.zeros((T, cfg.d_m))
+    p_prev = np.ones(T)            # p_hist_{l_0} = 1
+    m_prev = np.ones(T)            # m_hist_{l_0} = 1
+    h_bar_prev = None
+    delta_prev = None
+    d_prev = np.zeros(T)
+    gates = np.zeros((L, T))
+    masks = np.zeros((L, T), dtype=np.uint8)
+    counts = np.zeros(L, dtype=np.int64)
+    layers: List[Dict[str, np.ndarray]] = []
+
+    for j in range(1, L + 1):
+        wl = {k: _f64(weights[k][j - 1]) for k in _LAYER_KEYS}
+        P = 0.0 if attn_delta is None else _f64(attn_delta[j - 1])
+        h_bar = h + P                                               # Eq. 1 stand-in
+        rec: Dict[str, np.ndarray] = {"h_bar": h_bar}
+        if mode == "dense":
+            g = np.ones(T)
+            decide = np.ones(T, dtype=bool)
+        else:
+            delta, d, gamma = transition_features(j, h_bar, h_bar_prev, delta_prev,
+                                                  d_prev, cfg.eps)
+            x_path = path_vector(j, L, d, gamma, p_prev, m_prev)
+            z_h = hidden_encoder(h_bar, w, cfg, R)
+            z_a = path_encoder(x_path, w)
+            s = np.concatenate([z_h, z_a], axis=1)                 # Eq. 9
+            q = s @ w["w_q"].T                                      # Eq. 10
+            k = s @ w["w_k"].T
+            v = s @ w["w_v"].T
+            fq = hk.get("phi", phi)(q)
+            fk = hk.get("phi", phi)(k)
+            c = memory_read(fq, S, zeta, cfg.eps)                   # Eq. 11 (before write)
+            nu = history_dissimilarity(j, s, c, w, cfg.eps)         # Eq. 13
+            a = history_head(s, c, nu, w)                           # Eq. 14
+            p = sigmoid(a / cfg.t_hist)
+            m = m_prev * p                                          # Eq. 15
+            b = local_head(h_bar, w, R)                             # Eq. 16
+            g = sigmoid(a + b)
+            rho = sigmoid(eta[j - 1])
+            S, zeta = memory_write(S, zeta, fk, v, rho)             # Eq. 12
+            if mode == "route":
+                decide = g >= tau                                   # Eq. 3 threshold
+            else:
+                decide = np.asarray(mask_in[j - 1]).astype(bool)
+            if record:
+                rec.update(delta=delta, d=d, gamma=gamma, x_path=x_path, z_h=z_h, z_a=z_a,
+                           s=s, q=q, k=k, v=v, c=c, nu=nu, a=a, b=b, p=p, m=m,
+                           S=S.copy(), zeta=zeta.copy(), rho=np.float64(rho))
+            h_bar_prev, delta_prev, d_prev = h_bar, delta, d
+            p_prev, m_prev = p, m
+
+        u = R(rms_norm(h_bar, wl["ffn_norm_g"], cfg.rms_eps))       # Eq. 1, u = LN_ffn(h_bar)
+        if mode == "dense" or branch_scale == "one":
+            sf = np.ones(T)
+            sa = np.ones(T)
+        else:
+            sf, sa = g, 1.0 - g
+        h_new = h_bar.copy()
+        F = np.nonzero(decide)[0]
+        A = np.nonzero(~decide)[0]
+        if F.size:
+            h_new[F] += sf[F, None] * swiglu_ffn(u[F], wl, R)       # Eq. 3, g >= tau
+        if A.size:
+            h_new[A] += sa[A, None] * adapter(u[A], wl, R)          # Eq. 3, g < tau
+        gates[j - 1] = g
+        masks[j - 1] = decide.astype(np.uint8)
+        counts[j - 1] = F.size
+        if record:
+            rec.update(g=g, mask=decide.copy(), u=u, h=h_new)
+            layers.append(rec)
+        h = h_new
+
+    out: Dict[str, object] = {"h_out": h, "gate": gates, "mask": masks, "counts": counts}
+    if record:
+        out["layers"] = layers
+    return out
+
+
+def bypass_fraction(masks: np.ndarray) -> float:
+    """Share of FFN executions replaced by the adapter: sum_j n_a,j / (L_R T)."""
+    m = np.asarray(masks)
+    return float(1.0 - m.mean()) if m.size else 0.0

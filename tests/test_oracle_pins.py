@@ -1,0 +1,571 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each check compares the oracle with something other than itself: a library
+routine (torch's bf16 conversion, F.rms_norm, F.silu, F.elu), a textbook stack
+(dense SwiGLU, Houlsby adapter), a closed form (the memory as an explicit
+weighted sum, the second-block read, transition features of a branch-free
+stack, the zero-router gate), invariants (ranges, token independence,
+causality of decisions by brute force over all paths) and an independent
+per-token pure-Python restatement on tiny shapes.  The last group plants
+plausible mistakes in the oracle and shows that a pin catches each one.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+from oracle import hero_oracle as ho
+from synth import hero_inputs as hi
+
+pytestmark = pytest.mark.filterwarnings("ignore::RuntimeWarning")
+
+
+def _tiny(dtype="f32", **kw):
+    base = hi.CONFIGS["tiny_f32"] if dtype == "f32" else hi.CONFIGS["small_bf16"]
+    return base.replace(**kw) if kw else base
+
+
+def _inputs(cfg):
+    return hi.generate_weights(cfg), hi.generate_h_in(cfg), hi.generate_attn_delta(cfg)
+
+
+def _w64(w):
+    return {k: hi.to_f64(v) for k, v in w.items()}
+
+
+def _t(x):
+    return torch.as_tensor(np.asarray(x, dtype=np.float64))
+
+
+def _tbf16(x: torch.Tensor) -> torch.Tensor:
+    """Library bf16 rounding (torch) of a float64 tensor, through float32."""
+    return x.to(torch.float32).to(torch.bfloat16).to(torch.float64)
+
+
+# ---------------------------------------------------------------------------
+# Elementary functions against library routines
+# ---------------------------------------------------------------------------
+
+def test_bf16_round_matches_torch():
+    rng = np.random.default_rng(5)
+    x = np.concatenate([rng.standard_normal(200000) * 10.0 ** rng.integers(-30, 30, 200000),
+                        [0.0, -0.0, 1.0, -1.0, 3.0e38, 1e-40, -1e-42]])
+    x32 = x.astype(np.float32).astype(np.float64)      # f32-representable: no double rounding
+    # exact ties between two bf16 neighbours must go to the even one
+    ties = (np.arange(1, 2000, dtype=np.float64) * 2.0 + 1.0) * 2.0 ** -8 + 1.0
+    for v in (x32, ties, -ties):
+        ref = torch.tensor(v, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+        np.testing.assert_array_equal(ho.bf16_round(v), ref)
+
+
+def test_elementwise_functions_match_torch():
+    x = np.linspace(-30, 30, 10001)
+    np.testing.assert_allclose(ho.sigmoid(x), torch.sigmoid(_t(x)).numpy(), rtol=1e-15, atol=1e-300)
+    np.testing.assert_allclose(ho.silu(x), F.silu(_t(x)).numpy(), rtol=1e-14, atol=1e-300)
+    # torch forms ELU(x) + 1 as expm1(x) + 1, which cancels for x << 0: absolute bound
+    np.testing.assert_allclose(ho.phi(x), (F.elu(_t(x)) + 1.0).numpy(), rtol=1e-15, atol=1e-15)
+    g = np.linspace(0.5, 1.5, 64)
+    hbar = np.random.default_rng(1).standard_normal((7, 64)) * 3
+    np.testing.assert_allclose(ho.rms_norm(hbar, g, 1e-5),
+                               F.rms_norm(_t(hbar), (64,), _t(g), 1e-5).numpy(), rtol=1e-14)
+
+
+# ---------------------------------------------------------------------------
+# P1 / P1': dense stack and adapter stack against textbook restatements
+# ---------------------------------------------------------------------------
+
+def _textbook_dense(cfg, w, h, P, bf16):
+    """Textbook residual SwiGLU stack h_j = h_{j-1} + P_j + W_d(SiLU(W_g u) * W_u u)."""
+    r = _tbf16 if bf16 else (lambda x: x)
+    W = _w64(w)
+    x = _t(h)
+    for j in range(cfg.n_layers):
+        hb = x + _t(hi.to_f64(P[j]))
+        u = r(F.rms_norm(hb, (cfg.d_model,), _t(W["ffn_norm_g"][j]), cfg.rms_eps))
+        act = r(F.silu(u @ _t(W["w_gate"][j]).T) * (u @ _t(W["w_up"][j]).T))
+        x = hb + act @ _t(W["w_down"][j]).T
+    return x.numpy()
+
+
+def _textbook_adapter(cfg, w, h, P, bf16):
+    """Houlsby bottleneck-adapter stack h_j = h_{j-1} + P_j + W_2 SiLU(W_1 u)."""
+    r = _tbf16 if bf16 else (lambda x: x)
+    W = _w64(w)
+    x = _t(h)
+    for j in range(cfg.n_layers):
+        hb = x + _t(hi.to_f64(P[j]))
+        u = r(F.rms_norm(hb, (cfg.d_model,), _t(W["ffn_norm_g"][j]), cfg.rms_eps))
+        x = hb + r(F.silu(u @ _t(W["ad_w1"][j]).T)) @ _t(W["ad_w2"][j]).T
+    return x.numpy()
+
+
+def check_dense(cfg):
+    w, h, P = _inputs(cfg)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.5, mode="dense")
+    ref = _textbook_dense(cfg, w, h, P, cfg.dtype == "bf16")
+    return np.max(np.abs(out["h_out"] - ref)) / np.max(np.abs(ref)), out
+
+
+def test_p1_dense_equals_textbook_swiglu_stack_f32():
+    err, out = check_dense(_tiny())
+    assert err < 1e-13
+    assert (out["mask"] == 1).all() and (out["gate"] == 1).all()
+
+
+def test_p1_dense_equals_textbook_swiglu_stack_bf16():
+    # torch rounds float64 -> bf16 through float32; rare double-rounding cases move
+    # single elements by one bf16 step, hence the looser bound.
+    err, _ = check_dense(_tiny("bf16"))
+    assert err < 1e-4
+
+
+def check_adapter_stack(cfg):
+    w, h, P = _inputs(cfg)
+    zeros = np.zeros((cfg.n_layers, cfg.n_tokens), dtype=np.uint8)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.5, mode="force",
+                              mask_in=zeros, branch_scale="one")
+    ref = _textbook_adapter(cfg, w, h, P, cfg.dtype == "bf16")
+    return np.max(np.abs(out["h_out"] - ref)) / np.max(np.abs(ref))
+
+
+def test_p1p_all_adapter_equals_houlsby_stack():
+    assert check_adapter_stack(_tiny()) < 1e-13
+    assert check_adapter_stack(_tiny("bf16")) < 1e-4
+
+
+# ---------------------------------------------------------------------------
+# Eq. 3: branch choice and gate scaling, layer by layer
+# ---------------------------------------------------------------------------
+
+def check_branch_scaling(cfg, tau):
+    w, h, P = _inputs(cfg)
+    W = _w64(w)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, tau, record=True)
+    worst = 0.0
+    for j, rec in enumerate(out["layers"]):
+        hb = _t(rec["h_bar"])
+        g = _t(rec["g"])[:, None]
+        u = F.rms_norm(hb, (cfg.d_model,), _t(W["ffn_norm_g"][j]), cfg.rms_eps)
+        ffn = (F.silu(u @ _t(W["w_gate"][j]).T) * (u @ _t(W["w_up"][j]).T)) @ _t(W["w_down"][j]).T
+        ada = F.silu(u @ _t(W["ad_w1"][j]).T) @ _t(W["ad_w2"][j]).T
+        m = torch.as_tensor(rec["g"] >= tau)[:, None]
+        assert (m[:, 0].numpy() == rec["mask"]).all()
+        ref = torch.where(m, hb + g * ffn, hb + (1 - g) * ada)
+        worst = max(worst, float((ref - _t(rec["h"])).abs().max()))
+    return worst, out
+
+
+def test_eq3_branch_choice_and_scaling():
+    cfg = _tiny()
+    worst, out = check_branch_scaling(cfg, hi.calibrated_tau("tiny_f32"))
+    assert worst < 1e-13
+    assert 0 < out["mask"].sum() < out["mask"].size
+
+
+# ---------------------------------------------------------------------------
+# P2 / P3: the depth memory against closed forms
+# ---------------------------------------------------------------------------
+
+def _phi_t(x):
+    return (F.elu(_t(x)) + 1.0).numpy()
+
+
+def check_memory_closed_form(cfg, eta=None):
+    w, h, P = _inputs(cfg)
+    if eta is not None:
+        w = dict(w)
+        w["eta"] = np.full(cfg.n_layers, eta, dtype=np.float32)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.4, record=True)
+    lay = out["layers"]
+    eta64 = hi.to_f64(w["eta"])
+    rho = 1.0 / (1.0 + np.exp(-eta64))
+    worst_S = worst_c = 0.0
+    for j in range(len(lay)):
+        # S_j = sum_{i<=j} (prod_{m=i+1..j} rho_m) phi(k_i) v_i^T ; zeta likewise
+        S = np.zeros_like(lay[j]["S"])
+        Z = np.zeros_like(lay[j]["zeta"])
+        for i in range(j + 1):
+            decay = np.prod(rho[i + 1:j + 1])
+            fk = _phi_t(lay[i]["k"])
+            S += decay * fk[:, :, None] * lay[i]["v"][:, None, :]
+            Z += decay * fk
+        worst_S = max(worst_S, np.max(np.abs(S - lay[j]["S"])) / (np.max(np.abs(S)) + 1e-300),
+                      np.max(np.abs(Z - lay[j]["zeta"])) / np.max(np.abs(Z)))
+        # c_j reads S_{j-1}: a weighted sum of v_1..v_{j-1}
+        fq = _phi_t(lay[j]["q"])
+        num = np.zeros_like(lay[j]["c"])
+        den = np.zeros(fq.shape[0])
+        for i in range(j):
+            wgt = np.prod(rho[i + 1:j]) * np.sum(fq * _phi_t(lay[i]["k"]), axis=1)
+            num += wgt[:, None] * lay[i]["v"]
+            den += wgt
+        c = num / (den + cfg.eps)[:, None]
+        worst_c = max(worst_c, np.max(np.abs(c - lay[j]["c"])))
+    return worst_S, worst_c, out
+
+
+def test_p2_memory_equals_explicit_weighted_sum():
+    ws, wc, out = check_memory_closed_form(_tiny())
+    assert ws < 1e-12 and wc < 1e-12
+    ws, wc, _ = check_memory_closed_form(_tiny("bf16"))
+    assert ws < 1e-12 and wc < 1e-12
+
+
+def test_p2_rho_one_is_causal_linear_attention():
+    """With rho = 1 the read is Katharopoulos causal linear attention over depth."""
+    cfg = _tiny()
+    w, h, P = _inputs(cfg)
+    w = dict(w)
+    w["eta"] = np.full(cfg.n_layers, 60.0, dtype=np.float32)   # sigma(60) == 1.0 in float64
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.4, record=True)
+    lay = out["layers"]
+    q = torch.stack([_t(l["q"]) for l in lay], 1)               # [T, L, dm]
+    k = torch.stack([_t(l["k"]) for l in lay], 1)
+    v = torch.stack([_t(l["v"]) for l in lay], 1)
+    fq, fk = F.elu(q) + 1, F.elu(k) + 1
+    kv = torch.cumsum(fk[..., :, None] * v[..., None, :], dim=1)  # inclusive prefix sums
+    ks = torch.cumsum(fk, dim=1)
+    kv = torch.cat([torch.zeros_like(kv[:, :1]), kv[:, :-1]], 1)   # strictly earlier blocks
+    ks = torch.cat([torch.zeros_like(ks[:, :1]), ks[:, :-1]], 1)
+    c = torch.einsum("tlm,tlmn->tln", fq, kv) / (torch.einsum("tlm,tlm->tl", fq, ks) + cfg.eps)[..., None]
+    got = torch.stack([_t(l["c"]) for l in lay], 1)
+    assert float((c - got).abs().max()) < 1e-12
+
+
+def check_second_block(cfg):
+    w, h, P = _inputs(cfg)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.4, record=True)
+    l1, l2 = out["layers"][0], out["layers"][1]
+    x = np.sum(_phi_t(l2["q"]) * _phi_t(l1["k"]), axis=1)
+    c2 = l1["v"] * (x / (x + cfg.eps))[:, None]
+    return max(np.max(np.abs(l1["c"])), np.max(np.abs(c2 - l2["c"]))), out
+
+
+def test_p3_first_and_second_block_reads():
+    err, out = check_second_block(_tiny())
+    assert err < 1e-13
+    l1 = out["layers"][0]
+    assert (l1["nu"] == 0).all() and (l1["d"] == 0).all() and (l1["gamma"] == 0).all()
+    assert (out["layers"][1]["gamma"] == 0).all()
+
+
+# ---------------------------------------------------------------------------
+# P4: ranges and recurrences
+# ---------------------------------------------------------------------------
+
+def test_p4_ranges_and_recurrences():
+    cfg = _tiny()
+    w, h, P = _inputs(cfg)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P,
+                              hi.calibrated_tau("tiny_f32"), record=True)
+    m_acc = np.ones(cfg.n_tokens)
+    for j, l in enumerate(out["layers"], start=1):
+        xp = l["x_path"]
+        assert np.allclose(xp[:, 0] + xp[:, 1], 1.0)
+        assert np.allclose(xp[:, 0], j / cfg.n_layers)
+        m_acc = m_acc * l["p"]
+        np.testing.assert_allclose(l["m"], m_acc, rtol=1e-14)
+        assert ((l["p"] > 0) & (l["p"] < 1)).all() and ((l["g"] > 0) & (l["g"] < 1)).all()
+        assert (np.abs(l["gamma"]) <= 1).all() and ((l["nu"] >= 0) & (l["nu"] <= 2)).all()
+        assert (l["zeta"] > 0).all()
+        if j > 1:
+            assert np.allclose(xp[:, 4], out["layers"][j - 2]["p"])
+            assert np.allclose(xp[:, 5], out["layers"][j - 2]["m"])
+        else:
+            assert (xp[:, 4] == 1).all() and (xp[:, 5] == 1).all()
+
+
+# ---------------------------------------------------------------------------
+# Closed forms with designed parameters
+# ---------------------------------------------------------------------------
+
+def check_transition_closed_form(cfg):
+    """Branch-free stack (W_down = W_2 = 0): h_bar_j - h_bar_{j-1} = P_j exactly."""
+    w, h, _ = _inputs(cfg)
+    w = dict(w)
+    w["w_down"] = np.zeros_like(w["w_down"])
+    w["ad_w2"] = np.zeros_like(w["ad_w2"])
+    rng = np.random.default_rng(3)
+    P = np.empty((cfg.n_layers, cfg.n_tokens, cfg.d_model))
+    P[0] = rng.standard_normal(P[0].shape) * 0.1
+    for j in range(1, cfg.n_layers):            # correlated so that gamma is far from 0
+        P[j] = 0.8 * P[j - 1] * (-1) ** j + 0.2 * rng.standard_normal(P[0].shape) * 0.1
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.4, record=True)
+    worst = 0.0
+    for j, l in enumerate(out["layers"], start=1):
+        if j == 1:
+            d_ref = np.zeros(cfg.n_tokens)
+            g_ref = np.zeros(cfg.n_tokens)
+        else:
+            d_ref = np.linalg.norm(P[j - 1], axis=1)
+            if j > 2:
+                g_ref = np.sum(P[j - 1] * P[j - 2], axis=1) / (
+                    d_ref * np.linalg.norm(P[j - 2], axis=1) + cfg.eps)
+            else:
+                g_ref = np.zeros(cfg.n_tokens)
+        worst = max(worst, np.max(np.abs(l["d"] - d_ref)), np.max(np.abs(l["gamma"] - g_ref)))
+    return worst, out
+
+
+def test_transition_features_closed_form():
+    worst, out = check_transition_closed_form(_tiny())
+    assert worst < 1e-12
+    assert np.abs(out["layers"][2]["gamma"]).mean() > 0.5
+
+
+def test_zero_router_closed_form():
+    """All router matrices zero, biases kept: every quantity has a closed form."""
+    cfg = _tiny()
+    w, h, P = _inputs(cfg)
+    w = dict(w)
+    for k in ("w_hd", "w_hu", "path_w1", "path_w2", "w_q", "w_k", "w_v", "w_n", "w_c",
+              "th_w1", "th_w2", "ps_w1", "ps_w2"):
+        w[k] = np.zeros_like(w[k])
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, 0.5, record=True)
+    bt2, bp2 = float(w["th_b2"][0]), float(w["ps_b2"][0])
+    p = 1 / (1 + math.exp(-bt2 / cfg.t_hist))
+    for j, l in enumerate(out["layers"], start=1):
+        np.testing.assert_allclose(l["g"], 1 / (1 + math.exp(-(bt2 + bp2))), rtol=1e-14)
+        np.testing.assert_allclose(l["p"], p, rtol=1e-14)
+        np.testing.assert_allclose(l["m"], p ** j, rtol=1e-13)
+        np.testing.assert_allclose(l["s"][:, cfg.d_h:], np.broadcast_to(w["path_b2"], (cfg.n_tokens, cfg.d_a)))
+        assert (l["s"][:, :cfg.d_h] == 0).all() and (l["c"] == 0).all()
+        np.testing.assert_allclose(l["nu"], 0.0 if j == 1 else 1.0)
+        np.testing.assert_allclose(l["zeta"], sum(np.prod(1 / (1 + np.exp(-hi.to_f64(w["eta"][i + 1:j]))))
+                                                  for i in range(j)), rtol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# P5: brute force over every forced path (causality of decisions)
+# ---------------------------------------------------------------------------
+
+def check_path_brute_force(cfg, tau):
+    w, h, P = _inputs(cfg)
+    oc = ho.OracleConfig.from_stack(cfg)
+    free = ho.routed_ffn_stack(oc, w, h, P, tau)
+    L, T = cfg.n_layers, cfg.n_tokens
+    consistent = np.zeros((2 ** L, T), dtype=bool)
+    for pi in range(2 ** L):
+        path = np.array([(pi >> j) & 1 for j in range(L)], dtype=np.uint8)
+        forced = ho.routed_ffn_stack(oc, w, h, P, tau, mode="force",
+                                     mask_in=np.repeat(path[:, None], T, axis=1))
+        consistent[pi] = ((forced["gate"] >= tau) == path[:, None].astype(bool)).all(axis=0)
+    n_consistent = consistent.sum(axis=0)
+    chosen = np.argmax(consistent, axis=0)
+    free_code = sum(free["mask"][j].astype(np.int64) << j for j in range(L))
+    return n_consistent, chosen, free_code
+
+
+def test_p5_unique_self_consistent_path_is_the_free_run():
+    n, chosen, free_code = check_path_brute_force(_tiny(), hi.calibrated_tau("tiny_f32"))
+    assert (n == 1).all()
+    assert (chosen == free_code).all()
+    assert len(np.unique(free_code)) > 3
+
+
+# ---------------------------------------------------------------------------
+# P6: token independence;  P7: budget
+# ---------------------------------------------------------------------------
+
+def test_p6_token_independence():
+    cfg = _tiny()
+    w, h, P = _inputs(cfg)
+    oc = ho.OracleConfig.from_stack(cfg)
+    tau = hi.calibrated_tau("tiny_f32")
+    full = ho.routed_ffn_stack(oc, w, h, P, tau)
+    perm = np.random.default_rng(0).permutation(cfg.n_tokens)
+    permuted = ho.routed_ffn_stack(oc, w, h[perm], P[:, perm], tau)
+    np.testing.assert_array_equal(permuted["h_out"], full["h_out"][perm])
+    np.testing.assert_array_equal(permuted["mask"], full["mask"][:, perm])
+    sub = np.arange(5, 40, 3)
+    part = ho.routed_ffn_stack(oc, w, h[sub], P[:, sub], tau)
+    np.testing.assert_allclose(part["h_out"], full["h_out"][sub], rtol=1e-14, atol=1e-14)
+    np.testing.assert_array_equal(part["mask"], full["mask"][:, sub])
+
+
+def test_p7_budget_tiny():
+    cfg = _tiny()
+    w, h, P = _inputs(cfg)
+    out = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P,
+                              hi.calibrated_tau("tiny_f32"))
+    assert abs(ho.bypass_fraction(out["mask"]) - cfg.bypass) <= 1.0 / (cfg.n_layers * cfg.n_tokens)
+    np.testing.assert_array_equal(out["counts"], out["mask"].sum(axis=1))
+
+
+# ---------------------------------------------------------------------------
+# P8: independent per-token, per-element pure-Python restatement (tiny shapes)
+# ---------------------------------------------------------------------------
+
+def _py_stack(cfg, W, h_in, P, tau):
+    """Per-token loops over scalars, written from Sec. 3 without numpy linear algebra."""
+    L, d = cfg.n_layers, cfg.d_model
+
+    def mv(M, x):
+        return [sum(M[o][i] * x[i] for i in range(len(x))) for o in range(len(M))]
+
+    def sg(x):
+        return 1.0 / (1.0 + math.exp(-x))
+
+    def sl(x):
+        return x * sg(x)
+
+    def ph(x):
+        return x + 1.0 if x > 0 else math.exp(x)
+
+    out_h, out_g = [], []
+    for t in range(len(h_in)):
+        h = list(h_in[t])
+        dm = cfg.d_m
+        S = [[0.0] * dm for _ in range(dm)]
+        Z = [0.0] * dm
+        p_prev = m_prev = 1.0
+        hb_prev = dl_prev = None
+        d_prev = 0.0
+        gs = []
+        for j in range(1, L + 1):
+            hb = [h[i] + P[j - 1][t][i] for i in range(d)]
+            if j == 1:
+                dl = [0.0] * d
+            else:
+                dl = [hb[i] - hb_prev[i] for i in range(d)]
+            dd = math.sqrt(sum(x * x for x in dl))
+            gam = 0.0
+            if j > 2:
+                gam = sum(dl[i] * dl_prev[i] for i in range(d)) / (dd * d_prev + cfg.eps)
+            rms = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+            nr = [hb[i] / rms * W["r_norm_g"][i] for i in range(d)]
+            zh = mv(W["w_hu"], [sl(x) for x in mv(W["w_hd"], nr)])
+            xp = [j / L, (L - j) / L, dd, gam, p_prev, m_prev]
+            hid = [sl(x + b) for x, b in zip(mv(W["path_w1"], xp), W["path_b1"])]
+            za = [x + b for x, b in zip(mv(W["path_w2"], hid), W["path_b2"])]
+            s = zh + za
+            q, k, v = mv(W["w_q"], s), mv(W["w_k"], s), mv(W["w_v"], s)
+            fq, fk = [ph(x) for x in q], [ph(x) for x in k]
+            den = sum(fq[m] * Z[m] for m in range(dm)) + cfg.eps
+            c = [sum(fq[m] * S[m][n] for m in range(dm)) / den for n in range(dm)]
+            if j == 1:
+                nu = 0.0
+            else:
+                a1, b1 = mv(W["w_n"], s), mv(W["w_c"], c)
+                na = math.sqrt(sum(x * x for x in a1))
+                nb = math.sqrt(sum(x * x for x in b1))
+                nu = 1.0 - sum(x * y for x, y in zip(a1, b1)) / (na * nb + cfg.eps)
+            hh = [sl(x + b) for x, b in zip(mv(W["th_w1"], s + c + [nu]), W["th_b1"])]
+            a = sum(x * y for x, y in zip(W["th_w2"][0], hh)) + W["th_b2"][0]
+            p = sg(a / cfg.t_hist)
+            m = m_prev * p
+            hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], hb), W["ps_b1"])]
+            bb = sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0]
+            g = sg(a + bb)
+            rho = sg(W["eta"][j - 1])
+            for mm in range(dm):
+                for n in range(dm):
+                    S[mm][n] = rho * S[mm][n] + fk[mm] * v[n]
+                Z[mm] = rho * Z[mm] + fk[mm]
+            rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+            u = [hb[i] / rf * W["ffn_norm_g"][j - 1][i] for i in range(d)]
+            if g >= tau:
+                gt, up = mv(W["w_gate"][j - 1], u), mv(W["w_up"][j - 1], u)
+                y = mv(W["w_down"][j - 1], [sl(x) * z for x, z in zip(gt, up)])
+                h = [hb[i] + g * y[i] for i in range(d)]
+            else:
+                y = mv(W["ad_w2"][j - 1], [sl(x) for x in mv(W["ad_w1"][j - 1], u)])
+                h = [hb[i] + (1 - g) * y[i] for i in range(d)]
+            gs.append(g)
+            hb_prev, dl_prev, d_prev, p_prev, m_prev = hb, dl, dd, p, m
+        out_h.append(h)
+        out_g.append(gs)
+    return np.array(out_h), np.array(out_g).T
+
+
+def test_p8_loop_restatement_tiny_shapes():
+    cfg = hi.StackConfig("micro", 3, 8, 12, 4, 4, 6, "f32", 0.3, d_h=3, d_a=2, d_enc=5,
+                         d_head=6, d_path=3, seed=11)
+    w, h, P = _inputs(cfg)
+    W = {k: hi.to_f64(v).tolist() for k, v in w.items()}
+    oc = ho.OracleConfig.from_stack(cfg)
+    base = ho.routed_ffn_stack(oc, w, h, P, 0.0, record=True)
+    tau = float(np.median(base["gate"]))                  # a mix of both branches
+    got = ho.routed_ffn_stack(oc, w, h, P, tau)
+    ref_h, ref_g = _py_stack(cfg, W, hi.to_f64(h).tolist(), hi.to_f64(P).tolist(), tau)
+    np.testing.assert_allclose(got["gate"], ref_g, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
+    assert 0 < got["mask"].sum() < got["mask"].size
+
+
+# ---------------------------------------------------------------------------
+# Planted mistakes: each plausible slip in the oracle is caught by a pin
+# ---------------------------------------------------------------------------
+
+def test_planted_mistakes_are_caught(monkeypatch):
+    cfg = _tiny()
+    tau = hi.calibrated_tau("tiny_f32")
+
+    def caught(check):
+        try:
+            return not check()
+        except AssertionError:
+            return True
+
+    # 1. phi without the +1 (plain ELU): the second-block closed form fails
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "phi", lambda x: np.where(x > 0, x, np.exp(np.minimum(x, 0)) - 1))
+        assert caught(lambda: check_second_block(cfg)[0] < 1e-13)
+    # 2. forgetting applied to the new term instead of the old state
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "memory_write",
+                   lambda S, z, fk, v, rho: (S + rho * np.einsum("tm,tn->tmn", fk, v), z + rho * fk))
+        assert caught(lambda: max(check_memory_closed_form(cfg)[:2]) < 1e-12)
+    # 3. write before read: c_j would see the current block's own state
+    orig_read = ho.memory_read
+
+    def read_after_write(fq, S, zeta, eps):
+        return orig_read(fq, S + 1.0, zeta + 1.0, eps)
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "memory_read", read_after_write)
+        assert caught(lambda: check_second_block(cfg)[0] < 1e-13)
+    # 4. transition against two blocks back
+    orig_tf = ho.transition_features
+
+    def tf_wrong_sign(j, hb, hbp, dp, d_prev, eps):
+        delta, d, gamma = orig_tf(j, hb, hbp, dp, d_prev, eps)
+        return delta, d, -gamma
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "transition_features", tf_wrong_sign)
+        assert caught(lambda: check_transition_closed_form(cfg)[0] < 1e-12)
+    # 5. gate and up projections swapped in the SwiGLU
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "swiglu_ffn", lambda u, wl, R: R(silu_swapped(u, wl)) @ wl["w_down"].T)
+        assert caught(lambda: check_dense(cfg)[0] < 1e-13)
+    # 6. adapter hidden without its activation
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "adapter", lambda u, wl, R: (u @ wl["ad_w1"].T) @ wl["ad_w2"].T)
+        assert caught(lambda: check_adapter_stack(cfg) < 1e-13)
+    # 7. branch scale swapped (FFN scaled by 1 - g)
+    orig_stack = ho.routed_ffn_stack
+
+    def swapped(*a, **k):
+        out = orig_stack(*a, **k)
+        for rec in out.get("layers", []):
+            rec["g"] = 1.0 - rec["g"]
+        return out
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "routed_ffn_stack", swapped)
+        assert caught(lambda: check_branch_scaling(cfg, tau)[0] < 1e-13)
+    # 8. decision threshold inverted: brute force no longer finds the free run
+    def inverted(*a, **k):
+        out = orig_stack(*a, **k)
+        if k.get("mode", "route") == "route":
+            out["mask"] = 1 - out["mask"]
+        return out
+    with monkeypatch.context() as mp:
+        mp.setattr(ho, "routed_ffn_stack", inverted)
+        n, chosen, free_code = check_path_brute_force(cfg, tau)
+        assert not (chosen == free_code).all()
+
+
+def silu_swapped(u, wl):
+    return ho.silu(u @ wl["w_up"].T) * (u @ wl["w_gate"].T)
