@@ -1,0 +1,350 @@
+"""Throughput of the routed FFN stack on GB300 (one JSON line on rank 0).
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                [--workload NAME] [--cpu-sample N] [--no-cpu-baseline]
+
+A step is one pass of the whole routed FFN stack (all routed blocks: memory
+readout, router score, compaction, FFN / adapter, scatter into the residual,
+memory update) over the workload's T tokens.  Inputs (weights 11.3 GB, the
+attention stand-in 4.3 GB) are far larger than the 129 MB L2, so no flush is
+needed between steps.  With N > 1 ranks (torchrun), every rank runs its own
+token shard of the same size on its own GPU (weak scaling, no collective on the
+data path); value = all ranks' tokens / the slowest rank's time.
+
+--impl reference times the CPU oracle (the only reference this method has) on a
+bounded token sample per step, on rank 0 only.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import hero_inputs as hi  # noqa: E402
+
+METRIC = "routed-FFN-stack tokens/s at Llama-3.1-8B shapes; % of bf16 tensor peak"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_desc(cfg, bypass):
+    return (f"{cfg.name}: {cfg.n_layers} routed blocks, d={cfg.d_model}, I={cfg.d_ff}, "
+            f"d_r={cfg.d_r}, d_m={cfg.d_m}, T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len}), "
+            f"{cfg.dtype}, bypass target {bypass:.2%}, random-init weights, seeded inputs")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.hw_slowdown",
+              "clocks_event_reasons.hw_thermal_slowdown", "clocks_event_reasons.sw_thermal_slowdown",
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) != len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def algorithmic_work(cfg, counts_per_step, steps):
+    """Executed FLOPs per kernel class over the timed steps (counts: FFN tokens per block)."""
+    T, d, I, r = cfg.n_tokens, cfg.d_model, cfg.d_ff, cfg.d_r
+    nY = cfg.d_enc + cfg.d_head
+    nf = np.asarray(counts_per_step, dtype=np.float64)
+    na = T - nf
+    return {
+        "ffn_gate_up": steps * float(np.sum(2.0 * nf * 2 * I * d)),
+        "ffn_down": steps * float(np.sum(2.0 * nf * I * d)),
+        "router_gemm": steps * float(cfg.n_layers * 2.0 * T * nY * d),
+        "adapter_down": steps * float(np.sum(2.0 * na * r * d)),
+        "adapter_up": steps * float(np.sum(2.0 * na * d * r)),
+    }
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return
+    from oracle import hero_oracle as ho
+    cfg = hi.CONFIGS[args.workload]
+    tau = hi.calibrated_tau(cfg.name)
+    w = hi.generate_weights(cfg)
+    rows = hi.sample_tokens(cfg.n_tokens, args.cpu_sample)
+    h = hi.generate_h_in(cfg)[rows]
+    P = hi.generate_attn_delta(cfg)[:, rows]
+    oc = ho.OracleConfig.from_stack(cfg)
+    for _ in range(args.warmup):
+        ho.routed_ffn_stack(oc, w, h, P, tau)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ho.routed_ffn_stack(oc, w, h, P, tau)
+    dt = time.perf_counter() - t0
+    v = len(rows) * args.steps / dt
+    cores = len(os.sched_getaffinity(0))
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": workload_desc(cfg, cfg.bypass),
+                       "sample": f"{len(rows)} evenly spread tokens of T={cfg.n_tokens} per step"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"{len(rows)} tokens x {cfg.n_layers} blocks per step"},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama31_8b_prefill", choices=sorted(hi.CONFIGS))
+    ap.add_argument("--cpu-sample", type=int, default=8)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return reference_arm(args, rank, world)
+
+    import torch
+    from paper_2609_08189_gb300 import build, hero
+
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    if rank == 0:
+        build.build()
+    if dist:
+        dist.barrier()
+    hero.load()
+
+    cfg = hi.CONFIGS[args.workload]
+    tau = hi.calibrated_tau(cfg.name)
+    T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
+    t_gen = time.time()
+    w = hi.generate_weights(cfg)
+    h_np = hi.generate_h_in(cfg)
+    P_np = hi.generate_attn_delta(cfg)
+    t_gen = time.time() - t_gen
+    stack = hero.HeroStack(cfg, w)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.current_stream(dev)
+    h = torch.from_numpy(h_np).to(dev)
+    P = torch.from_numpy(P_np).to(dev)
+    h_out = torch.empty((T, d), dtype=torch.float32, device=dev)
+    g = torch.empty((L, T), dtype=torch.float32, device=dev)
+    m = torch.empty((L, T), dtype=torch.uint8, device=dev)
+    c = torch.empty((L,), dtype=torch.int32, device=dev)
+
+    def barrier():
+        if dist:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if not dist:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def run(flags):
+        stack(h, P, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m, counts_out=c, stream=stream)
+
+    def timed(fn, K, sampler=None):
+        barrier()
+        torch.cuda.synchronize()
+        if sampler:
+            sampler.start()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(K):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        clk = sampler.stop() if sampler else None
+        return max_over_ranks(e0.elapsed_time(e1)), clk
+
+    # ---- routed stack (the metric) ----
+    for _ in range(args.warmup):
+        run(0)
+    torch.cuda.synchronize()
+    stack.check()
+    hero.hero_get_profile(stack.model, reset=True)
+    hero.hero_set_profiling(stack.model, True)
+    sampler = ClockSampler(local_rank)
+    ms, clocks = timed(lambda: run(0), args.steps, sampler)
+    hero.hero_set_profiling(stack.model, False)
+    prof = hero.hero_get_profile(stack.model, reset=True)
+    stack.check()
+    counts = c.cpu().numpy().astype(np.int64)
+    bypass = 1.0 - counts.sum() / (L * T)
+    value = world * T * args.steps / (ms / 1e3)
+
+    # ---- dense stack, same kernels ----
+    dense = None
+    if not args.no_dense:
+        for _ in range(2):
+            run(hero.HERO_FLAG_DENSE)
+        ms_dense, _ = timed(lambda: run(hero.HERO_FLAG_DENSE), args.steps)
+        dense = world * T * args.steps / (ms_dense / 1e3)
+        stack.check()
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        hp = torch.from_numpy(h_np).pin_memory()
+        Pp = torch.from_numpy(P_np).pin_memory()
+        ho_ = torch.empty((T, d), dtype=torch.float32).pin_memory()
+        cp = torch.empty((L,), dtype=torch.int32).pin_memory()
+
+        def run_host():
+            hero.hero_routed_ffn_stack(stack.model, T, hp.data_ptr(), Pp.data_ptr(), tau,
+                                       hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                       cp.data_ptr(), stream.cuda_stream)
+        run_host()
+        torch.cuda.synchronize()
+        ms_e2e, _ = timed(run_host, args.steps)
+        stack.check()
+        e2e = {"value": world * T * args.steps / (ms_e2e / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(hp.numel() * 4 + Pp.numel() * 2),
+               "d2h_bytes_per_step": int(ho_.numel() * 4 + cp.numel() * 4)}
+        assert np.array_equal(cp.numpy(), counts), "host-IO path routed differently"
+
+    # ---- roofline of the dominant kernel ----
+    peaks, peak_src = load_peaks()
+    work = algorithmic_work(cfg, counts, args.steps)
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms, dom_n = prof[dom]
+    roof = None
+    if dom in work and dom_ms > 0:
+        achieved = work[dom] / (dom_ms / 1e3) / 1e12
+        peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)",
+                "avg_launch_ms": dom_ms / max(dom_n, 1)}
+    ffn_ms = prof["ffn_gate_up"][0] + prof["ffn_down"][0]
+    ffn_tflops = (work["ffn_gate_up"] + work["ffn_down"]) / (ffn_ms / 1e3) / 1e12 if ffn_ms else None
+
+    # ---- CPU baseline: the oracle on a bounded sample ----
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import hero_oracle as ho
+        rows = hi.sample_tokens(T, args.cpu_sample)
+        oc = ho.OracleConfig.from_stack(cfg)
+        t0 = time.perf_counter()
+        ho.routed_ffn_stack(oc, w, h_np[rows], P_np[:, rows], tau)
+        dt = time.perf_counter() - t0
+        cpu = {"value": len(rows) / dt, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
+               "kind": "oracle",
+               "sample": f"{len(rows)} evenly spread tokens of T={T} through all {L} blocks, "
+                         f"float64 numpy ({dt:.1f} s; BLAS threads = cores)"}
+
+    launches = int(sum(n for _, n in prof.values()))
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+        "config": {"workload": workload_desc(cfg, cfg.bypass),
+                   "l2": "inputs larger than L2 (no flush): weights and P_j stream from HBM each step",
+                   "parallelism": f"token shards, {world} rank(s), no collective"},
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "dense_value": dense,
+        "routed_vs_dense": (value / dense) if dense else None,
+        "bypass": bypass,
+        "ffn_counts": counts.tolist(),
+        "ffn_gemm_tflops": ffn_tflops,
+        "ffn_gemm_frac_of_sustained": (ffn_tflops / float(peaks.get("bf16_tflops_sustained", 1700.0)))
+        if ffn_tflops else None,
+        "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items()},
+        "setup_s": {"generate": t_gen},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    stack.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,191 @@
+/*
+ * hero.h - C ABI of the GB300 (sm_103a) implementation of HeRo's history-aware
+ * routed FFN stack ("Do Dynamic Routers Need Memory? HeRo: History-Aware Routing
+ * for Efficient LLM Inference", Sec. 3).
+ *
+ * One call runs L_R routed blocks over T independent tokens.  Each block does, per
+ * token and in this order (equation numbers count the displayed equations of
+ * Sec. 3: 1 dense_attention, 2 adapter, 3 ffn_route, 4 path_vector, 5 hidden
+ * encoder, 6 depth features, 7-8 transition features, 9 router_state, 10 q/k/v,
+ * 11 memory_read, 12 memory_update, 13 nu, 14 history head, 15 cumulative
+ * history, 16 final_gate):
+ *   1. memory readout  c = phi(q)^T S / (phi(q)^T zeta + eps)            Eq. 11
+ *   2. router score    g = sigma(f_theta([s;c;nu]) + f_psi(h_bar))       Eqs. 4-10, 13-16
+ *   3. compaction of the tokens with g >= tau_exec                        Eq. 3
+ *   4. frozen SwiGLU FFN on those tokens, adapter W_2 SiLU(W_1 u) on the rest   Eqs. 2-3
+ *   5. h = h_bar + g FFN(u)  or  h_bar + (1-g) Adapter(u)                 Eq. 3
+ *   6. memory update   S = rho S + phi(k) v^T, zeta = rho zeta + phi(k)   Eq. 12
+ * h_bar_j = h_{j-1} + P_j, where P_j (attn_delta) stands in for the dense attention
+ * sublayer of Eq. 1.  Per-token memory S, zeta and path state are created and
+ * zeroed inside every call (one forward pass, Sec. 3.2).
+ *
+ * Conventions
+ *   - Every function returns hero_status; nothing aborts or exits.  On failure
+ *     hero_last_error() returns a thread-local message.
+ *   - Argument errors are detected before any work is enqueued (HERO_ERR_ARG).
+ *   - Tensor pointers are DEVICE memory owned by the caller unless noted (see
+ *     HERO_FLAG_HOST_IO); all tensors are dense row-major.
+ *   - Execution is asynchronous on the given CUDA stream (cudaStream_t, NULL =
+ *     legacy default stream).  Kernels never spin without a bound: a wait that
+ *     expires (about 4 s) sets a device error word that hero_check_device_status
+ *     reports as HERO_ERR_TIMEOUT.
+ *   - A model may be used by one host thread at a time.
+ */
+#ifndef HERO_H_
+#define HERO_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  HERO_OK = 0,
+  HERO_ERR_ARG = 1,          /* invalid argument; nothing was enqueued          */
+  HERO_ERR_CUDA = 2,         /* a CUDA runtime call failed                      */
+  HERO_ERR_NOMEM = 3,        /* device or host allocation failed                */
+  HERO_ERR_UNSUPPORTED = 4,  /* shape or dtype outside what the kernels support */
+  HERO_ERR_TIMEOUT = 5       /* a device-side bounded wait expired              */
+} hero_status;
+
+typedef enum { HERO_F32 = 0, HERO_BF16 = 1 } hero_dtype;
+
+/* Shapes and constants of one routed FFN stack.
+ *   n_layers   L_R, routed blocks (Sec. 3.1)
+ *   d_model    d, hidden width; d_ff = I, SwiGLU intermediate width
+ *   d_r        adapter rank (W_1: d_r x d, W_2: d x d_r; Eq. 2)
+ *   d_m        memory width (q, k, v in R^{d_m}; S is d_m x d_m per token; Sec. 3.2)
+ *   d_h, d_a   widths of z^h and z^a; the router state s has d_s = d_h + d_a (Eq. 9)
+ *   d_enc      inner width of the hidden encoder W_hd (Eq. 5)
+ *   d_head     hidden width of f_theta and f_psi (Sec. 4.1: 256)
+ *   d_path     hidden width of FFN_path (Eq. 9)
+ *   max_tokens largest T a call may pass; sizes the library-owned workspace
+ *   dtype      HERO_BF16: bf16 weights and GEMM operands, fp32 accumulation and
+ *              fp32 residual; HERO_F32: fp32 everywhere
+ *   rms_eps    RMSNorm epsilon; eps: the epsilon of Eqs. 8, 11 and 13's cosine
+ *   t_hist     history temperature T_hist (Eq. 14)
+ * Supported: d_m in {16, 32, 64, 128}; d_s <= 128; d_enc, d_head <= 256;
+ * d_path <= 64.  bf16 additionally needs d % 256 == 0, d_ff % 128 == 0 and
+ * d_r == 64; f32 needs d % 4 == 0. */
+typedef struct {
+  int32_t n_layers, d_model, d_ff, d_r, d_m;
+  int32_t d_h, d_a, d_enc, d_head, d_path;
+  int32_t max_tokens;
+  hero_dtype dtype;
+  float rms_eps, eps, t_hist;
+} hero_config;
+
+/* HOST pointers to the parameters, canonical [out, in] layouts, stacked over
+ * layers where marked [L, ...].  All arrays have element type host_dtype
+ * (HERO_F32: float; HERO_BF16: uint16 bf16 bit patterns, allowed only for bf16
+ * models).  The library copies (and for bf16 models rounds to bf16 with
+ * round-to-nearest-even) during hero_init_weights; the caller may free them on
+ * return.
+ *   ffn_norm_g [L,d]   gain of LN^ffn (RMSNorm)                      Eq. 1
+ *   w_gate, w_up [L,I,d], w_down [L,d,I]   frozen SwiGLU FFN          Eq. 3
+ *   ad_w1 [L,d_r,d], ad_w2 [L,d,d_r]       adapter                     Eq. 2
+ *   eta [L]            forgetting parameters, rho_j = sigma(eta_j)    Eq. 12
+ *   r_norm_g [d]       router RMSNorm gain; w_hd [d_enc,d]; w_hu [d_h,d_enc]   Eq. 5
+ *   path_w1 [d_path,6], path_b1 [d_path], path_w2 [d_a,d_path], path_b2 [d_a]  Eq. 9
+ *   w_q, w_k, w_v [d_m,d_s]                                            Eq. 10
+ *   w_n [d_m,d_s], w_c [d_m,d_m]                                       Eq. 13
+ *   th_w1 [d_head,d_s+d_m+1], th_b1 [d_head], th_w2 [1,d_head], th_b2 [1]   f_theta, Eq. 14
+ *   ps_w1 [d_head,d], ps_b1 [d_head], ps_w2 [1,d_head], ps_b2 [1]          f_psi, Eq. 16
+ * Shared router parameters serve every block; FFN, adapter and eta are per
+ * block (Sec. 3.2). */
+typedef struct {
+  hero_dtype host_dtype;
+  const void *ffn_norm_g, *w_gate, *w_up, *w_down, *ad_w1, *ad_w2, *eta;
+  const void *r_norm_g, *w_hd, *w_hu, *path_w1, *path_b1, *path_w2, *path_b2;
+  const void *w_q, *w_k, *w_v, *w_n, *w_c;
+  const void *th_w1, *th_b1, *th_w2, *th_b2;
+  const void *ps_w1, *ps_b1, *ps_w2, *ps_b2;
+} hero_weights_host;
+
+typedef struct hero_model hero_model; /* opaque, library-owned */
+
+enum {
+  /* Router skipped; every token runs the FFN with branch scale 1 (the dense
+   * SwiGLU stack run by the same kernels).  gate_out is filled with 1,
+   * mask_out with 1, ffn_count_out with T. */
+  HERO_FLAG_DENSE = 1u,
+  /* Decisions are read from mask_in [L,T] (nonzero = FFN); g is still computed
+   * and scales the branches as in Eq. 3. */
+  HERO_FLAG_FORCE_MASK = 2u,
+  /* h_in, attn_delta, mask_in, h_out, gate_out, mask_out and ffn_count_out are
+   * HOST pointers; the library copies them to and from the device on the stream
+   * (page-locked host memory makes the copies asynchronous). */
+  HERO_FLAG_HOST_IO = 4u
+};
+
+/* Copy, convert and repack the parameters to the current CUDA device and size
+ * the workspace for cfg->max_tokens.  Synchronous.  On success *out owns all
+ * device memory of the model. */
+hero_status hero_init_weights(const hero_config* cfg, const hero_weights_host* w,
+                              hero_model** out);
+
+/* Run the routed FFN stack on n_tokens tokens (0 <= n_tokens <= max_tokens).
+ *   h_in       [T,d] fp32 input hidden states h_0
+ *   attn_delta [L,T,d] attention stand-in P_j, fp32 for f32 models, bf16 bits for
+ *              bf16 models; NULL means zero
+ *   tau_exec   execution threshold of Eq. 3 (g >= tau_exec runs the FFN)
+ *   flags      HERO_FLAG_*
+ *   mask_in    [L,T] decisions for HERO_FLAG_FORCE_MASK, else ignored (may be NULL)
+ *   h_out      [T,d] fp32 output h_{L_R}; must not alias h_in
+ *   gate_out   [L,T] fp32 gates g, or NULL
+ *   mask_out   [L,T] uint8 decisions (1 = FFN), or NULL
+ *   ffn_count_out [L] int32 number of FFN tokens per block, or NULL
+ * Returns after enqueueing; outputs are valid once the stream reaches them. */
+hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, const float* h_in,
+                                  const void* attn_delta, float tau_exec, uint32_t flags,
+                                  const uint8_t* mask_in, float* h_out, float* gate_out,
+                                  uint8_t* mask_out, int32_t* ffn_count_out,
+                                  void* cuda_stream);
+
+/* Release every resource of the model (NULL-safe).  Synchronizes the device. */
+void hero_free(hero_model* m);
+
+/* Message of the last failure on this host thread ("" if none). */
+const char* hero_last_error(void);
+
+/* Synchronize cuda_stream, then report HERO_ERR_TIMEOUT if any kernel of this
+ * model hit its wait bound since the last check (and clear the record), or
+ * HERO_ERR_CUDA if the stream holds a CUDA error. */
+hero_status hero_check_device_status(hero_model* m, void* cuda_stream);
+
+/* ---- measurement ------------------------------------------------------------
+ * Kernel classes of one block, for per-kernel timing. */
+enum {
+  HERO_K_INIT = 0,        /* first h_bar, workspace reset                     */
+  HERO_K_ROUTER_GEMM = 1, /* [T x d] x [d x (d_enc+d_head)] router contraction */
+  HERO_K_ROUTER = 2,      /* memory read/update, heads, gate, decision        */
+  HERO_K_COMPACT = 3,     /* stable scan of the decisions into index lists    */
+  HERO_K_NORM = 4,        /* LN^ffn of each token into its branch's rows      */
+  HERO_K_FFN_GATE_UP = 5, /* gathered gate/up GEMM with the SwiGLU epilogue   */
+  HERO_K_FFN_DOWN = 6,    /* down GEMM with the scaled scatter epilogue       */
+  HERO_K_ADAPTER_DOWN = 7,/* adapter W_1 GEMM with the SiLU epilogue          */
+  HERO_K_ADAPTER_UP = 8,  /* adapter W_2 GEMM with the scaled scatter epilogue */
+  HERO_K_COUNT = 9
+};
+
+/* When enabled, every later launch of the model is bracketed by CUDA events on
+ * its stream.  hero_get_profile synchronizes those events and returns, per
+ * kernel class, the summed device milliseconds and the launch count since the
+ * last reset (then resets when reset != 0).  Both arrays hold HERO_K_COUNT
+ * entries.  The launch counters run whether or not timing is enabled. */
+hero_status hero_set_profiling(hero_model* m, int enable);
+hero_status hero_get_profile(hero_model* m, double* ms_out, int64_t* launches_out, int reset);
+
+/* Building-block check of the tensor-core GEMM: C[M,N] (fp32) = A[M,K] B[N,K]^T
+ * with A, B bf16 (uint16 bit patterns), DEVICE pointers, row-major, K % 64 == 0,
+ * K and N multiples of 8 elements.  Not part of the routed stack's contract;
+ * exposed so the GEMM core can be tested alone. */
+hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B, float* C, int32_t M,
+                                 int32_t N, int32_t K, void* cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HERO_H_ */

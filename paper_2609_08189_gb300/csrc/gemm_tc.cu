@@ -1,0 +1,367 @@
+// Persistent tensor-core GEMM for sm_103a: TMA-fed shared-memory ring, tcgen05.mma
+// with the accumulator in TMEM (double buffered), and fused epilogues.
+//
+//   C[M, N] = A[M, K] * B[N, K]^T        (bf16 operands, fp32 accumulation)
+//
+// One CTA per SM, 6 warps:
+//   warp 0      TMA producer (one elected lane) - A and B tiles into a STAGES-deep ring
+//   warp 1      TMEM allocator and MMA issuer (one elected lane)
+//   warps 2..5  epilogue: each owns the 32 TMEM lanes (= tile rows) of its quadrant
+// Tiles are 128 x BN with K-blocks of 64 bf16 (one 128-byte swizzle row).  The row
+// count M may live in device memory (the compacted token count of a routed block),
+// so no host synchronisation is needed between routing and the GEMMs; tiles past M
+// do no work.  Every mbarrier wait is bounded (%globaltimer) and reports through
+// the error word instead of hanging.
+#include "hero_device.cuh"
+
+namespace hero {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int kGroupM = 16;   // raster: 16 M-tiles share each wave of N-tiles (L2 reuse)
+
+template <int BN>
+struct TcCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+  // instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
+  // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                                    ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+  static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+};
+
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
+  const int group = kGroupM * n_tiles;
+  const int g = tile / group;
+  const int first_m = g * kGroupM;
+  const int gm = min(kGroupM, m_tiles - first_m);
+  const int local = tile - g * group;
+  mb = first_m + local % gm;
+  nb = local / gm;
+}
+
+// ---- epilogues: one thread = one tile row; TMEM read in 32 or 16 column chunks ----
+
+template <int BN>
+__device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                              int nb) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < BN; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    const int n0 = nb * BN + c0;
+    if (valid) {
+      float* dst = a.out_f32 + (size_t)m * a.ldo + n0;
+#pragma unroll
+      for (int i = 0; i < 32; i += 4) {
+        if (n0 + i < a.N) {
+          *reinterpret_cast<float4*>(dst + i) =
+              make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]),
+                          __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3]));
+        }
+      }
+    }
+  }
+}
+
+// Gate/up columns are interleaved per 256-wide tile: [0,128) gate, [128,256) up of
+// the same 128 intermediate features; output act[m, nb*128 + c].
+__device__ __forceinline__ void epi_swiglu(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                           int nb) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < 128; c0 += 16) {
+    uint32_t g[16], u[16];
+    tmem_ld16(tbase + c0, g);
+    tmem_ld16(tbase + 128 + c0, u);
+    if (valid) {
+      uint32_t pk[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        pk[i] = pack_bf16x2(siluf_(g0) * u0, siluf_(g1) * u1);
+      }
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) + (size_t)m * a.ldo +
+                                            nb * 128 + c0);
+      dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+    }
+  }
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                         int nb) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < BN; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    if (valid) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        pk[i] = pack_bf16x2(siluf_(__uint_as_float(r[2 * i])), siluf_(__uint_as_float(r[2 * i + 1])));
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) + (size_t)m * a.ldo +
+                                            nb * BN + c0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+    }
+  }
+}
+
+template <int BN>
+__device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                              int nb) {
+  int t = 0;
+  float s = 0.f;
+  if (valid) {
+    t = a.lo.idx[m];
+    s = a.lo.scale[m];
+  }
+  float ss = 0.f, dd = 0.f, dp = 0.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < BN; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    if (valid) {
+#pragma unroll
+      for (int i = 0; i < 32; i += 4) {
+        const float4 y = make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]),
+                                     __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3]));
+        layer_out4(a.lo, t, nb * BN + c0 + i, y, s, ss, dd, dp);
+      }
+    }
+  }
+  if (valid && !a.lo.last) {
+    *reinterpret_cast<float4*>(a.lo.part + ((size_t)t * a.lo.np + nb) * 4) =
+        make_float4(ss, dd, dp, 0.f);
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const GemmArgs args) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::STAGES + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * C::STAGES + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * C::STAGES + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * C::STAGES + 4);
+  volatile uint32_t* misc = reinterpret_cast<volatile uint32_t*>(bars + 2 * C::STAGES + 5);
+  const uint32_t smem_base = smem_u32(smem);
+  auto sA = [&](int s) { return smem_base + s * C::STAGE_BYTES; };
+  auto sB = [&](int s) { return smem_base + s * C::STAGE_BYTES + C::A_BYTES; };
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  int M = args.m_dev ? *args.m_dev : args.m_static;
+  if (M < 0 || M > args.m_max) {
+    if (threadIdx.x == 0) atomicOr(args.err, ERR_BAD_INDEX);
+    M = 0;
+  }
+  const int m_tiles = (M + BM - 1) / BM;
+  const int n_tiles = (args.N + BN - 1) / BN;
+  const int total = m_tiles * n_tiles;
+  const int kblocks = (args.K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar(a), 1);
+      mbar_init(tempty_bar(a), 4);
+    }
+    mbar_init(drain_bar, 1);
+    misc[1] = 0;  // abort flag
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(misc)), C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = misc[0];
+
+  if (warp == 0) {
+    // ------------------------------ TMA producer ------------------------------
+    if (lane == 0 && total > 0) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, last_par = 0;  // per-stage bit masks for the drain
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        int mb, nb;
+        tile_coords(tile, m_tiles, n_tiles, mb, nb);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitLimitNs) || misc[1]) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full_bar(stage), C::STAGE_BYTES);
+          tma_load_2d(sA(stage), &tmA, kb * BK, mb * BM, full_bar(stage));
+          tma_load_2d(sB(stage), &tmB, kb * BK, nb * BN, full_bar(stage));
+          issued |= 1u << stage;
+          last_par = (last_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        misc[1] = 1;
+        atomicOr(args.err, ERR_WAIT_PRODUCER);
+        // let copies still in flight land before the CTA can exit
+        for (int s = 0; s < C::STAGES; ++s)
+          if (issued & (1u << s)) mbar_wait(full_bar(s), (last_par >> s) & 1u, 100000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer ------------------------------
+    if (lane == 0 && total > 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, kWaitLimitNs) || misc[1]) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(full_bar(stage), phase, kWaitLimitNs) || misc[1]) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t adesc = sw128_desc(sA(stage));
+          const uint64_t bdesc = sw128_desc(sB(stage));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            // +32 bytes per K step of 16 bf16 inside the 128-byte swizzle row
+            umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb | k) != 0);
+          }
+          umma_commit(empty_bar(stage));
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(tfull_bar(acc));
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      if (!ok) {
+        misc[1] = 1;
+        atomicOr(args.err, ERR_WAIT_MMA);
+        umma_commit(drain_bar);  // completes once every issued MMA has finished
+        if (!mbar_wait(drain_bar, 0, 100000000ull)) atomicOr(args.err, ERR_WAIT_DRAIN);
+      }
+    }
+  } else {
+    // ------------------------------ epilogue ------------------------------
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int row = q * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      int mb, nb;
+      tile_coords(tile, m_tiles, n_tiles, mb, nb);
+      bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
+      ok = __all_sync(0xffffffffu, ok) && !misc[1];
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) {
+        if (lane == 0) {
+          misc[1] = 1;
+          atomicOr(args.err, ERR_WAIT_EPILOGUE);
+        }
+        break;
+      }
+      tc_fence_after();
+      const int m = mb * BM + row;
+      const bool valid = m < M;
+      const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      if constexpr (EPI == EPI_STORE_F32) {
+        epi_store_f32<BN>(args, tbase, m, valid, nb);
+      } else if constexpr (EPI == EPI_SWIGLU) {
+        epi_swiglu(args, tbase, m, valid, nb);
+      } else if constexpr (EPI == EPI_SILU) {
+        epi_silu<BN>(args, tbase, m, valid, nb);
+      } else {
+        epi_layer_out<BN>(args, tbase, m, valid, nb);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty_bar(acc));
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+template <int BN, int EPI>
+cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& args,
+                       int num_sms, cudaStream_t st) {
+  using C = TcCfg<BN>;
+  static bool attr_set = false;  // per process; the attribute is per function
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const long max_tiles = (long)((args.m_max + BM - 1) / BM) * ((args.N + BN - 1) / BN);
+  if (max_tiles <= 0) return cudaSuccess;
+  const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
+  k_gemm_tc<BN, EPI><<<grid, 192, C::SMEM, st>>>(tmA, tmB, args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                           const GemmArgs& args, int num_sms, cudaStream_t st) {
+  if (bn == 256) {
+    switch (epi) {
+      case EPI_STORE_F32: return launch_one<256, EPI_STORE_F32>(tmA, tmB, args, num_sms, st);
+      case EPI_SWIGLU: return launch_one<256, EPI_SWIGLU>(tmA, tmB, args, num_sms, st);
+      case EPI_LAYER_OUT: return launch_one<256, EPI_LAYER_OUT>(tmA, tmB, args, num_sms, st);
+      default: break;
+    }
+  } else if (bn == 64 && epi == EPI_SILU) {
+    return launch_one<64, EPI_SILU>(tmA, tmB, args, num_sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace hero

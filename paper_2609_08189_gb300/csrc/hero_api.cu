@@ -1,0 +1,819 @@
+// Host runtime of libhero: parameter loading and repacking, workspace, the
+// per-block launch sequence of the routed FFN stack, profiling and the C ABI.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/hero.h"
+#include "hero_internal.cuh"
+
+using namespace hero;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+hero_status fail(hero_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+#define CUDA_TRY(expr)                                                                    \
+  do {                                                                                    \
+    cudaError_t e_ = (expr);                                                              \
+    if (e_ != cudaSuccess)                                                                \
+      return fail(e_ == cudaErrorMemoryAllocation ? HERO_ERR_NOMEM : HERO_ERR_CUDA,        \
+                  "%s failed: %s (%s:%d)", #expr, cudaGetErrorString(e_), __FILE__, __LINE__); \
+  } while (0)
+
+// ---- cuTensorMapEncodeTiled through the runtime's driver entry point -----------
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encoder() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+// 2-D bf16 tensor [outer, inner] (inner contiguous), box [box_outer, 64] with the
+// 128-byte swizzle expected by the tcgen05 shared-memory descriptors.
+bool encode_bf16_2d(CUtensorMap* tm, const void* ptr, uint64_t inner, uint64_t outer,
+                    uint32_t box_outer) {
+  if (!get_encoder()) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+std::vector<float> host_f32(const void* p, size_t n, hero_dtype dt) {
+  std::vector<float> v(n);
+  if (dt == HERO_BF16) {
+    const uint16_t* s = static_cast<const uint16_t*>(p);
+    for (size_t i = 0; i < n; ++i) {
+      uint32_t u = (uint32_t)s[i] << 16;
+      memcpy(&v[i], &u, 4);
+    }
+  } else {
+    memcpy(v.data(), p, n * sizeof(float));
+  }
+  return v;
+}
+
+struct ProfEvent {
+  int cls;
+  cudaEvent_t e0, e1;
+};
+
+}  // namespace
+
+struct hero_model {
+  hero_config cfg{};
+  int device = 0;
+  int num_sms = 0;
+  bool bf16 = false;
+  size_t esz = 4;  // operand element size
+  int np = 1;      // partial-sum slots per token
+
+  // parameters
+  void* wgu = nullptr;     // bf16: [L][2I][d] gate/up interleaved per 128 rows; f32: gate
+  void* wup = nullptr;     // f32 only: [L][I][d]
+  void* wdown = nullptr;   // [L][d][I]
+  void* w1 = nullptr;      // [L][d_r][d]
+  void* w2 = nullptr;      // [L][d][d_r]
+  void* wr = nullptr;      // [d_enc + d_head][d]: W_hd diag(g_r) ; f_psi first layer
+  float* ffn_gain = nullptr;  // [L][d]
+  float* router_small = nullptr;
+  RouterWeights rw{};
+  std::vector<float> rho;  // [L]
+
+  // workspace
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  float *hbar, *delta, *part, *Y, *S, *zeta, *pst, *mst, *dprev, *gate, *scale_f, *scale_a;
+  void *xl, *u_f, *u_a, *act, *ah;
+  uint8_t* mask;
+  int *idx_f, *idx_a, *counts;
+  uint32_t* err;
+
+  // host-IO staging (lazily grown)
+  void* io = nullptr;
+  size_t io_bytes = 0;
+
+  // tensor maps (bf16 only)
+  CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
+  std::vector<CUtensorMap> tm_wgu, tm_wd, tm_w1, tm_w2;
+
+  // measurement
+  bool profiling = false;
+  std::vector<ProfEvent> pending;
+  std::vector<cudaEvent_t> event_pool;
+  double prof_ms[HERO_K_COUNT] = {};
+  int64_t launches[HERO_K_COUNT] = {};
+};
+
+namespace {
+
+cudaEvent_t take_event(hero_model* m) {
+  if (!m->event_pool.empty()) {
+    cudaEvent_t e = m->event_pool.back();
+    m->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Run one launch of kernel class `cls`, bracketed by events when profiling.
+template <class F>
+cudaError_t timed(hero_model* m, int cls, cudaStream_t st, F&& launch) {
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (m->profiling) {
+    e0 = take_event(m);
+    cudaEventRecord(e0, st);
+  }
+  cudaError_t e = launch();
+  m->launches[cls]++;
+  if (m->profiling) {
+    e1 = take_event(m);
+    cudaEventRecord(e1, st);
+    m->pending.push_back({cls, e0, e1});
+  }
+  return e;
+}
+
+hero_status validate_config(const hero_config* c) {
+  if (!c) return fail(HERO_ERR_ARG, "config is NULL");
+  if (c->n_layers < 1 || c->d_model < 8 || c->d_ff < 1 || c->d_r < 1 || c->d_m < 1 || c->d_h < 1 ||
+      c->d_a < 1 || c->d_enc < 1 || c->d_head < 1 || c->d_path < 1 || c->max_tokens < 1)
+    return fail(HERO_ERR_ARG, "config has a non-positive dimension");
+  if (c->dtype != HERO_F32 && c->dtype != HERO_BF16) return fail(HERO_ERR_ARG, "unknown dtype");
+  if (!(c->rms_eps >= 0.f) || !(c->eps >= 0.f) || !(c->t_hist > 0.f))
+    return fail(HERO_ERR_ARG, "eps must be >= 0 and t_hist > 0");
+  if (c->d_m != 16 && c->d_m != 32 && c->d_m != 64 && c->d_m != 128)
+    return fail(HERO_ERR_UNSUPPORTED, "d_m must be 16, 32, 64 or 128 (got %d)", c->d_m);
+  if (c->d_h + c->d_a > 128 || c->d_enc > 256 || c->d_head > 256 || c->d_path > 64)
+    return fail(HERO_ERR_UNSUPPORTED, "router widths exceed d_s<=128, d_enc,d_head<=256, d_path<=64");
+  if (c->d_model % 8 != 0) return fail(HERO_ERR_UNSUPPORTED, "d_model must be a multiple of 8");
+  if (c->dtype == HERO_BF16) {
+    if (c->d_model % 256 != 0 || c->d_ff % 128 != 0 || c->d_r != 64)
+      return fail(HERO_ERR_UNSUPPORTED,
+                  "bf16 needs d_model %% 256 == 0, d_ff %% 128 == 0 and d_r == 64");
+    if ((c->d_enc + c->d_head) % 8 != 0)
+      return fail(HERO_ERR_UNSUPPORTED, "bf16 needs d_enc + d_head to be a multiple of 8");
+  }
+  return HERO_OK;
+}
+
+// Upload a host matrix [rows, cols] (element type src_dt) through a device staging
+// buffer into dst with the row map of launch_convert_rows.
+hero_status upload_rows(hero_model* m, const void* src, hero_dtype src_dt, void* dst, long rows,
+                        long cols, long grp, long grp_stride, long offset, const float* col_scale,
+                        void* stage, size_t stage_elems) {
+  const size_t src_es = src_dt == HERO_BF16 ? 2 : 4;
+  const size_t dst_es = m->esz;
+  long chunk = (long)(stage_elems / (size_t)cols);
+  if (grp > 1) chunk = (chunk / grp) * grp;
+  if (chunk < 1) return fail(HERO_ERR_NOMEM, "staging buffer too small for a row");
+  for (long r0 = 0; r0 < rows; r0 += chunk) {
+    const long nr = rows - r0 < chunk ? rows - r0 : chunk;
+    CUDA_TRY(cudaMemcpy(stage, static_cast<const char*>(src) + (size_t)r0 * cols * src_es,
+                        (size_t)nr * cols * src_es, cudaMemcpyHostToDevice));
+    const long dst_row0 = (r0 / grp) * grp_stride;
+    void* d = static_cast<char*>(dst) + (size_t)dst_row0 * cols * dst_es;
+    CUDA_TRY(launch_convert_rows(stage, src_dt == HERO_BF16, d, m->bf16, nr, cols, grp, grp_stride,
+                                 offset, col_scale, 0));
+  }
+  return HERO_OK;
+}
+
+void free_model(hero_model* m) {
+  if (!m) return;
+  cudaDeviceSynchronize();
+  for (auto& p : m->pending) {
+    cudaEventDestroy(p.e0);
+    cudaEventDestroy(p.e1);
+  }
+  for (auto e : m->event_pool) cudaEventDestroy(e);
+  void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
+                  m->ws, m->io};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  delete m;
+}
+
+}  // namespace
+
+// ============================================================================
+// C ABI
+// ============================================================================
+
+extern "C" const char* hero_last_error(void) { return g_last_error.c_str(); }
+
+extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weights_host* w,
+                                         hero_model** out) {
+  g_last_error.clear();
+  if (!out) return fail(HERO_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  hero_status s = validate_config(cfg);
+  if (s != HERO_OK) return s;
+  if (!w) return fail(HERO_ERR_ARG, "weights are NULL");
+  const void* need[] = {w->ffn_norm_g, w->w_gate, w->w_up, w->w_down, w->ad_w1, w->ad_w2, w->eta,
+                        w->r_norm_g, w->w_hd, w->w_hu, w->path_w1, w->path_b1, w->path_w2,
+                        w->path_b2, w->w_q, w->w_k, w->w_v, w->w_n, w->w_c, w->th_w1, w->th_b1,
+                        w->th_w2, w->th_b2, w->ps_w1, w->ps_b1, w->ps_w2, w->ps_b2};
+  for (size_t i = 0; i < sizeof(need) / sizeof(need[0]); ++i)
+    if (!need[i]) return fail(HERO_ERR_ARG, "weight pointer %zu is NULL", i);
+  if (w->host_dtype != HERO_F32 && w->host_dtype != HERO_BF16)
+    return fail(HERO_ERR_ARG, "unknown host_dtype");
+  if (w->host_dtype == HERO_BF16 && cfg->dtype != HERO_BF16)
+    return fail(HERO_ERR_ARG, "bf16 host weights need a bf16 model");
+
+  int dev = 0;
+  CUDA_TRY(cudaGetDevice(&dev));
+  cudaDeviceProp prop;
+  CUDA_TRY(cudaGetDeviceProperties(&prop, dev));
+  const bool bf16 = cfg->dtype == HERO_BF16;
+  if (bf16 && prop.major < 10)
+    return fail(HERO_ERR_UNSUPPORTED, "bf16 models need an sm_100-family GPU (found sm_%d%d)",
+                prop.major, prop.minor);
+  if (bf16 && !get_encoder())
+    return fail(HERO_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+
+  hero_model* m = new hero_model();
+  m->cfg = *cfg;
+  m->device = dev;
+  m->num_sms = prop.multiProcessorCount;
+  m->bf16 = bf16;
+  m->esz = bf16 ? 2 : 4;
+  const hero_config& c = *cfg;
+  const long L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r, dm = c.d_m;
+  const long ds = c.d_h + c.d_a, nY = c.d_enc + c.d_head;
+  m->np = bf16 ? (int)(d / 256) : (int)((d + kSimtTileN - 1) / kSimtTileN);
+  const hero_dtype hd = w->host_dtype;
+  const size_t hes = hd == HERO_BF16 ? 2 : 4;
+
+  auto bail = [&](hero_status st) {
+    free_model(m);
+    return st;
+  };
+#define TRY_M(expr)                      \
+  do {                                   \
+    hero_status st_ = (expr);            \
+    if (st_ != HERO_OK) return bail(st_); \
+  } while (0)
+#define CUDA_M(expr)                                                                        \
+  do {                                                                                      \
+    cudaError_t e_ = (expr);                                                                \
+    if (e_ != cudaSuccess)                                                                  \
+      return bail(fail(e_ == cudaErrorMemoryAllocation ? HERO_ERR_NOMEM : HERO_ERR_CUDA,    \
+                       "%s failed: %s", #expr, cudaGetErrorString(e_)));                    \
+  } while (0)
+
+  // ---- parameters ----
+  const size_t es = m->esz;
+  if (bf16) {
+    CUDA_M(cudaMalloc(&m->wgu, (size_t)L * 2 * I * d * es));
+  } else {
+    CUDA_M(cudaMalloc(&m->wgu, (size_t)L * I * d * es));
+    CUDA_M(cudaMalloc(&m->wup, (size_t)L * I * d * es));
+  }
+  CUDA_M(cudaMalloc(&m->wdown, (size_t)L * d * I * es));
+  CUDA_M(cudaMalloc(&m->w1, (size_t)L * r * d * es));
+  CUDA_M(cudaMalloc(&m->w2, (size_t)L * d * r * es));
+  CUDA_M(cudaMalloc(&m->wr, (size_t)nY * d * es));
+
+  size_t stage_elems = (size_t)1 << 25;  // 32 Mi elements
+  void* stage = nullptr;
+  CUDA_M(cudaMalloc(&stage, stage_elems * 4));
+  float* gain_r = nullptr;
+  auto cleanup_stage = [&] {
+    if (stage) cudaFree(stage);
+    if (gain_r) cudaFree(gain_r);
+    stage = nullptr;
+    gain_r = nullptr;
+  };
+  auto up = [&](const void* src, void* dst, long rows, long cols, long grp, long gstride,
+                long off, const float* cs) {
+    hero_status st = upload_rows(m, src, hd, dst, rows, cols, grp, gstride, off, cs, stage,
+                                 stage_elems);
+    return st;
+  };
+  hero_status st = HERO_OK;
+  for (long j = 0; j < L && st == HERO_OK; ++j) {
+    const char* g = static_cast<const char*>(w->w_gate) + (size_t)j * I * d * hes;
+    const char* u = static_cast<const char*>(w->w_up) + (size_t)j * I * d * hes;
+    if (bf16) {
+      void* dst = static_cast<char*>(m->wgu) + (size_t)j * 2 * I * d * es;
+      st = up(g, dst, I, d, 128, 256, 0, nullptr);
+      if (st == HERO_OK) st = up(u, dst, I, d, 128, 256, 128, nullptr);
+    } else {
+      st = up(g, static_cast<char*>(m->wgu) + (size_t)j * I * d * es, I, d, 1, 1, 0, nullptr);
+      if (st == HERO_OK)
+        st = up(u, static_cast<char*>(m->wup) + (size_t)j * I * d * es, I, d, 1, 1, 0, nullptr);
+    }
+    if (st == HERO_OK)
+      st = up(static_cast<const char*>(w->w_down) + (size_t)j * d * I * hes,
+              static_cast<char*>(m->wdown) + (size_t)j * d * I * es, d, I, 1, 1, 0, nullptr);
+    if (st == HERO_OK)
+      st = up(static_cast<const char*>(w->ad_w1) + (size_t)j * r * d * hes,
+              static_cast<char*>(m->w1) + (size_t)j * r * d * es, r, d, 1, 1, 0, nullptr);
+    if (st == HERO_OK)
+      st = up(static_cast<const char*>(w->ad_w2) + (size_t)j * d * r * hes,
+              static_cast<char*>(m->w2) + (size_t)j * d * r * es, d, r, 1, 1, 0, nullptr);
+  }
+  if (st == HERO_OK) {
+    // router contraction weight: rows [0, d_enc) = W_hd diag(g_r), rounded once;
+    // rows [d_enc, d_enc + d_head) = first layer of f_psi.
+    std::vector<float> gr = host_f32(w->r_norm_g, d, hd);
+    if (cudaMalloc(&gain_r, d * sizeof(float)) != cudaSuccess ||
+        cudaMemcpy(gain_r, gr.data(), d * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess)
+      st = fail(HERO_ERR_CUDA, "router gain upload failed");
+    if (st == HERO_OK) st = up(w->w_hd, m->wr, c.d_enc, d, 1, 1, 0, gain_r);
+    if (st == HERO_OK)
+      st = up(w->ps_w1, static_cast<char*>(m->wr) + (size_t)c.d_enc * d * es, c.d_head, d, 1, 1, 0,
+              nullptr);
+  }
+  if (st == HERO_OK && cudaDeviceSynchronize() != cudaSuccess)
+    st = fail(HERO_ERR_CUDA, "weight conversion failed: %s", cudaGetErrorString(cudaGetLastError()));
+  cleanup_stage();
+  if (st != HERO_OK) return bail(st);
+
+  {  // LN^ffn gains and forgetting factors
+    std::vector<float> gains = host_f32(w->ffn_norm_g, (size_t)L * d, hd);
+    CUDA_M(cudaMalloc(&m->ffn_gain, gains.size() * sizeof(float)));
+    CUDA_M(cudaMemcpy(m->ffn_gain, gains.data(), gains.size() * sizeof(float), cudaMemcpyHostToDevice));
+    std::vector<float> eta = host_f32(w->eta, L, hd);
+    m->rho.resize(L);
+    for (long j = 0; j < L; ++j) m->rho[j] = (float)(1.0 / (1.0 + std::exp(-(double)eta[j])));
+  }
+  {  // shared router parameters, transposed to [in][out]
+    std::vector<float> pack;
+    auto add_t = [&](const void* src, long rows, long cols) {  // src [rows][cols] -> [cols][rows]
+      std::vector<float> v = host_f32(src, (size_t)rows * cols, hd);
+      size_t at = pack.size();
+      pack.resize(at + (size_t)rows * cols);
+      for (long i = 0; i < rows; ++i)
+        for (long k = 0; k < cols; ++k) pack[at + (size_t)k * rows + i] = v[(size_t)i * cols + k];
+      return at;
+    };
+    auto add = [&](const void* src, long n) {
+      std::vector<float> v = host_f32(src, n, hd);
+      size_t at = pack.size();
+      pack.insert(pack.end(), v.begin(), v.end());
+      return at;
+    };
+    size_t o_hu = add_t(w->w_hu, c.d_h, c.d_enc);
+    size_t o_p1 = add_t(w->path_w1, c.d_path, 6);
+    size_t o_pb1 = add(w->path_b1, c.d_path);
+    size_t o_p2 = add_t(w->path_w2, c.d_a, c.d_path);
+    size_t o_pb2 = add(w->path_b2, c.d_a);
+    // q | k | v as one [d_s][3 d_m] matrix
+    size_t o_qkv = pack.size();
+    pack.resize(o_qkv + (size_t)ds * 3 * dm);
+    {
+      const void* src[3] = {w->w_q, w->w_k, w->w_v};
+      for (int p = 0; p < 3; ++p) {
+        std::vector<float> v = host_f32(src[p], (size_t)dm * ds, hd);
+        for (long i = 0; i < dm; ++i)
+          for (long k = 0; k < ds; ++k)
+            pack[o_qkv + (size_t)k * 3 * dm + p * dm + i] = v[(size_t)i * ds + k];
+      }
+    }
+    size_t o_n = add_t(w->w_n, dm, ds);
+    size_t o_c = add_t(w->w_c, dm, dm);
+    size_t o_t1 = add_t(w->th_w1, c.d_head, ds + dm + 1);
+    size_t o_tb1 = add(w->th_b1, c.d_head);
+    size_t o_t2 = add(w->th_w2, c.d_head);
+    size_t o_tb2 = add(w->th_b2, 1);
+    size_t o_pb = add(w->ps_b1, c.d_head);
+    size_t o_p2w = add(w->ps_w2, c.d_head);
+    size_t o_p2b = add(w->ps_b2, 1);
+    CUDA_M(cudaMalloc(&m->router_small, pack.size() * sizeof(float)));
+    CUDA_M(cudaMemcpy(m->router_small, pack.data(), pack.size() * sizeof(float),
+                      cudaMemcpyHostToDevice));
+    float* b = m->router_small;
+    m->rw = RouterWeights{b + o_hu, b + o_p1, b + o_pb1, b + o_p2, b + o_pb2, b + o_qkv, b + o_n,
+                          b + o_c,  b + o_t1, b + o_tb1, b + o_t2, b + o_tb2, b + o_pb, b + o_p2w,
+                          b + o_p2b};
+  }
+
+  // ---- workspace ----
+  {
+    const size_t Tm = (size_t)c.max_tokens;
+    size_t off = 0;
+    struct Item {
+      void** p;
+      size_t bytes;
+    };
+    std::vector<Item> items = {
+        {(void**)&m->hbar, Tm * d * 4},        {(void**)&m->delta, Tm * d * 4},
+        {(void**)&m->part, Tm * m->np * 16},   {(void**)&m->Y, Tm * nY * 4},
+        {(void**)&m->S, Tm * dm * dm * 4},     {(void**)&m->zeta, Tm * dm * 4},
+        {(void**)&m->pst, Tm * 4},             {(void**)&m->mst, Tm * 4},
+        {(void**)&m->dprev, Tm * 4},           {(void**)&m->gate, Tm * 4},
+        {(void**)&m->scale_f, Tm * 4},         {(void**)&m->scale_a, Tm * 4},
+        {(void**)&m->xl, Tm * d * es},         {(void**)&m->u_f, Tm * d * es},
+        {(void**)&m->u_a, Tm * d * es},        {(void**)&m->act, Tm * I * es},
+        {(void**)&m->ah, Tm * r * es},         {(void**)&m->mask, Tm},
+        {(void**)&m->idx_f, Tm * 4},           {(void**)&m->idx_a, Tm * 4},
+        {(void**)&m->counts, 64},              {(void**)&m->err, 64},
+    };
+    for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
+    CUDA_M(cudaMalloc(&m->ws, off));
+    CUDA_M(cudaMemset(m->ws, 0, off));
+    m->ws_bytes = off;
+    off = 0;
+    for (auto& it : items) {
+      *it.p = static_cast<char*>(m->ws) + off;
+      off += (it.bytes + 1023) & ~(size_t)1023;
+    }
+  }
+
+  // ---- tensor maps ----
+  if (bf16) {
+    const uint64_t Tm = (uint64_t)c.max_tokens;
+    bool ok = encode_bf16_2d(&m->tm_xl, m->xl, d, Tm, 128) &&
+              encode_bf16_2d(&m->tm_uf, m->u_f, d, Tm, 128) &&
+              encode_bf16_2d(&m->tm_ua, m->u_a, d, Tm, 128) &&
+              encode_bf16_2d(&m->tm_act, m->act, I, Tm, 128) &&
+              encode_bf16_2d(&m->tm_ah, m->ah, r, Tm, 128) &&
+              encode_bf16_2d(&m->tm_wr, m->wr, d, nY, 256);
+    m->tm_wgu.resize(L);
+    m->tm_wd.resize(L);
+    m->tm_w1.resize(L);
+    m->tm_w2.resize(L);
+    for (long j = 0; j < L && ok; ++j) {
+      ok = encode_bf16_2d(&m->tm_wgu[j], static_cast<char*>(m->wgu) + (size_t)j * 2 * I * d * 2, d,
+                          2 * I, 256) &&
+           encode_bf16_2d(&m->tm_wd[j], static_cast<char*>(m->wdown) + (size_t)j * d * I * 2, I, d,
+                          256) &&
+           encode_bf16_2d(&m->tm_w1[j], static_cast<char*>(m->w1) + (size_t)j * r * d * 2, d, r,
+                          64) &&
+           encode_bf16_2d(&m->tm_w2[j], static_cast<char*>(m->w2) + (size_t)j * d * r * 2, r, d,
+                          256);
+    }
+    if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
+  }
+  *out = m;
+  return HERO_OK;
+#undef TRY_M
+#undef CUDA_M
+}
+
+extern "C" void hero_free(hero_model* m) { free_model(m); }
+
+namespace {
+
+hero_status ensure_io(hero_model* m, size_t bytes) {
+  if (m->io_bytes >= bytes) return HERO_OK;
+  if (m->io) cudaFree(m->io);
+  m->io = nullptr;
+  m->io_bytes = 0;
+  CUDA_TRY(cudaMalloc(&m->io, bytes));
+  m->io_bytes = bytes;
+  return HERO_OK;
+}
+
+// The per-block launch sequence on device pointers.
+hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, float tau,
+                      uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
+                      uint8_t* mask_out, int32_t* count_out, cudaStream_t st) {
+  const hero_config& c = m->cfg;
+  const int L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r;
+  const int nY = c.d_enc + c.d_head;
+  const bool dense = flags & HERO_FLAG_DENSE;
+  const bool force = flags & HERO_FLAG_FORCE_MASK;
+  const size_t es = m->esz;
+  const size_t layer_elems = (size_t)T * d;
+
+  for (int jj = 0; jj < L; ++jj) {
+    const int j = jj + 1;
+    const void* Pj = P ? static_cast<const char*>(P) + (size_t)jj * layer_elems * es : nullptr;
+    const void* Pn = (P && jj + 1 < L) ? static_cast<const char*>(P) + (size_t)(jj + 1) * layer_elems * es
+                                       : nullptr;
+    if (jj == 0) {
+      InitArgs ia{T, d, m->np, c.d_m, h_in, Pj, (int)m->bf16, m->hbar, m->xl, (int)m->bf16,
+                  m->part, m->S, m->zeta, m->pst, m->mst, m->dprev, dense ? 0 : 1};
+      CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_init(ia, st); }));
+    }
+    if (!dense) {
+      GemmArgs g{};
+      g.m_dev = nullptr;
+      g.m_static = T;
+      g.m_max = T;
+      g.N = nY;
+      g.K = d;
+      g.out_f32 = m->Y;
+      g.ldo = nY;
+      g.err = m->err;
+      g.A = m->xl;
+      g.B = m->wr;
+      g.lda = d;
+      g.ldb = d;
+      CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
+        return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
+                       : launch_gemm_simt(EPI_STORE_F32, g, st);
+      }));
+      RouterArgs ra{};
+      ra.T = T;
+      ra.j = j;
+      ra.L = L;
+      ra.np = m->np;
+      ra.d = d;
+      ra.d_h = c.d_h;
+      ra.d_a = c.d_a;
+      ra.d_enc = c.d_enc;
+      ra.d_head = c.d_head;
+      ra.d_path = c.d_path;
+      ra.Y = m->Y;
+      ra.part = m->part;
+      ra.dprev = m->dprev;
+      ra.pst = m->pst;
+      ra.mst = m->mst;
+      ra.S = m->S;
+      ra.zeta = m->zeta;
+      ra.rho = m->rho[jj];
+      ra.w = m->rw;
+      ra.rms_eps = c.rms_eps;
+      ra.eps = c.eps;
+      ra.t_hist = c.t_hist;
+      ra.tau = tau;
+      ra.mask_in = force ? mask_in + (size_t)jj * T : nullptr;
+      ra.gate = m->gate;
+      ra.mask = m->mask;
+      ra.gate_out = gate_out ? gate_out + (size_t)jj * T : nullptr;
+      ra.mask_out = mask_out ? mask_out + (size_t)jj * T : nullptr;
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, st); }));
+    }
+    CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
+                   m->counts, count_out ? count_out + jj : nullptr,
+                   dense && gate_out ? gate_out + (size_t)jj * T : nullptr,
+                   dense && mask_out ? mask_out + (size_t)jj * T : nullptr};
+    CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
+    NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, m->hbar, m->part,
+                m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
+    CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, st); }));
+
+    LayerOutArgs lo{};
+    lo.hbar = m->hbar;
+    lo.delta = m->delta;
+    lo.p_next = Pn;
+    lo.xl = m->xl;
+    lo.part = m->part;
+    lo.h_out = h_out;
+    lo.d = d;
+    lo.np = m->np;
+    lo.tile_n = m->bf16 ? 256 : kSimtTileN;
+    lo.last = jj == L - 1;
+    lo.first = jj == 0;
+    lo.p_bf16 = m->bf16;
+    lo.xl_bf16 = m->bf16;
+    lo.router = dense ? 0 : 1;
+
+    // FFN branch: gate/up + SwiGLU, then down + scaled scatter
+    {
+      GemmArgs g{};
+      g.m_dev = m->counts;
+      g.m_max = T;
+      g.N = m->bf16 ? 2 * I : I;
+      g.K = d;
+      g.out = m->act;
+      g.ldo = I;
+      g.err = m->err;
+      g.A = m->u_f;
+      g.lda = d;
+      g.B = static_cast<const char*>(m->wgu) + (size_t)jj * (m->bf16 ? 2 : 1) * I * d * es;
+      g.B2 = m->bf16 ? nullptr : static_cast<const char*>(m->wup) + (size_t)jj * I * d * es;
+      g.ldb = d;
+      CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] {
+        return m->bf16 ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], g, m->num_sms, st)
+                       : launch_gemm_simt(EPI_SWIGLU, g, st);
+      }));
+      GemmArgs g2{};
+      g2.m_dev = m->counts;
+      g2.m_max = T;
+      g2.N = d;
+      g2.K = I;
+      g2.err = m->err;
+      g2.lo = lo;
+      g2.lo.idx = m->idx_f;
+      g2.lo.scale = m->scale_f;
+      g2.A = m->act;
+      g2.lda = I;
+      g2.B = static_cast<const char*>(m->wdown) + (size_t)jj * d * I * es;
+      g2.ldb = I;
+      CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
+        return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], g2, m->num_sms, st)
+                       : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
+      }));
+    }
+    // adapter branch
+    if (!dense) {
+      GemmArgs g{};
+      g.m_dev = m->counts + 1;
+      g.m_max = T;
+      g.N = r;
+      g.K = d;
+      g.out = m->ah;
+      g.ldo = r;
+      g.err = m->err;
+      g.A = m->u_a;
+      g.lda = d;
+      g.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
+      g.ldb = d;
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_DOWN, st, [&] {
+        return m->bf16 ? launch_gemm_tc(64, EPI_SILU, m->tm_ua, m->tm_w1[jj], g, m->num_sms, st)
+                       : launch_gemm_simt(EPI_SILU, g, st);
+      }));
+      GemmArgs g2{};
+      g2.m_dev = m->counts + 1;
+      g2.m_max = T;
+      g2.N = d;
+      g2.K = r;
+      g2.err = m->err;
+      g2.lo = lo;
+      g2.lo.idx = m->idx_a;
+      g2.lo.scale = m->scale_a;
+      g2.A = m->ah;
+      g2.lda = r;
+      g2.B = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
+      g2.ldb = r;
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
+        return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_ah, m->tm_w2[jj], g2, m->num_sms, st)
+                       : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
+      }));
+    }
+  }
+  return HERO_OK;
+}
+
+}  // namespace
+
+extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, const float* h_in,
+                                             const void* attn_delta, float tau_exec,
+                                             uint32_t flags, const uint8_t* mask_in, float* h_out,
+                                             float* gate_out, uint8_t* mask_out,
+                                             int32_t* ffn_count_out, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  const hero_config& c = m->cfg;
+  if (n_tokens < 0 || n_tokens > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_tokens %lld outside [0, max_tokens=%d]", (long long)n_tokens,
+                c.max_tokens);
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO))
+    return fail(HERO_ERR_ARG, "unknown flag bits 0x%x", flags);
+  if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
+    return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
+  if ((flags & HERO_FLAG_FORCE_MASK) && !mask_in && n_tokens > 0)
+    return fail(HERO_ERR_ARG, "HERO_FLAG_FORCE_MASK needs mask_in");
+  if (n_tokens > 0 && (!h_in || !h_out)) return fail(HERO_ERR_ARG, "h_in and h_out are required");
+  if (n_tokens > 0 && (const void*)h_in == (const void*)h_out)
+    return fail(HERO_ERR_ARG, "h_out must not alias h_in");
+  if (!std::isfinite(tau_exec)) return fail(HERO_ERR_ARG, "tau_exec is not finite");
+  cudaError_t e0 = cudaSetDevice(m->device);
+  if (e0 != cudaSuccess) return fail(HERO_ERR_CUDA, "cudaSetDevice: %s", cudaGetErrorString(e0));
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const int T = (int)n_tokens;
+  const int L = c.n_layers, d = c.d_model;
+  const bool host = flags & HERO_FLAG_HOST_IO;
+
+  if (T == 0) {
+    if (ffn_count_out) {
+      if (host)
+        memset(ffn_count_out, 0, (size_t)L * 4);
+      else
+        CUDA_TRY(cudaMemsetAsync(ffn_count_out, 0, (size_t)L * 4, st));
+    }
+    return HERO_OK;
+  }
+  if (!host)
+    return run_stack(m, T, h_in, attn_delta, tau_exec, flags, mask_in, h_out, gate_out, mask_out,
+                     ffn_count_out, st);
+
+  // Host I/O: stage inputs on the device, run, copy outputs back on the stream.
+  const size_t esz = m->esz;
+  const size_t p_bytes = attn_delta ? (size_t)L * T * d * esz : 0;
+  const size_t lt = (size_t)L * T;
+  const size_t need = (size_t)T * d * 4 /*h_out*/ + p_bytes + lt /*mask_in*/ + lt * 4 /*gate*/ +
+                      lt /*mask*/ + (size_t)L * 4 + 4096;
+  hero_status s = ensure_io(m, need);
+  if (s != HERO_OK) return s;
+  char* p = static_cast<char*>(m->io);
+  auto carve = [&](size_t bytes) {
+    char* q = p;
+    p += (bytes + 255) & ~(size_t)255;
+    return q;
+  };
+  float* d_hout = reinterpret_cast<float*>(carve((size_t)T * d * 4));
+  void* d_P = attn_delta ? carve(p_bytes) : nullptr;
+  uint8_t* d_mask_in = (flags & HERO_FLAG_FORCE_MASK) ? reinterpret_cast<uint8_t*>(carve(lt)) : nullptr;
+  float* d_gate = gate_out ? reinterpret_cast<float*>(carve(lt * 4)) : nullptr;
+  uint8_t* d_mask = mask_out ? reinterpret_cast<uint8_t*>(carve(lt)) : nullptr;
+  int32_t* d_cnt = ffn_count_out ? reinterpret_cast<int32_t*>(carve((size_t)L * 4)) : nullptr;
+  // h_0 goes straight into the h_bar buffer; k_init adds P_1 in place.
+  CUDA_TRY(cudaMemcpyAsync(m->hbar, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
+  if (d_P) CUDA_TRY(cudaMemcpyAsync(d_P, attn_delta, p_bytes, cudaMemcpyHostToDevice, st));
+  if (d_mask_in) CUDA_TRY(cudaMemcpyAsync(d_mask_in, mask_in, lt, cudaMemcpyHostToDevice, st));
+  s = run_stack(m, T, m->hbar, d_P, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask, d_cnt, st);
+  if (s != HERO_OK) return s;
+  CUDA_TRY(cudaMemcpyAsync(h_out, d_hout, (size_t)T * d * 4, cudaMemcpyDeviceToHost, st));
+  if (d_gate) CUDA_TRY(cudaMemcpyAsync(gate_out, d_gate, lt * 4, cudaMemcpyDeviceToHost, st));
+  if (d_mask) CUDA_TRY(cudaMemcpyAsync(mask_out, d_mask, lt, cudaMemcpyDeviceToHost, st));
+  if (d_cnt) CUDA_TRY(cudaMemcpyAsync(ffn_count_out, d_cnt, (size_t)L * 4, cudaMemcpyDeviceToHost, st));
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_check_device_status(hero_model* m, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  CUDA_TRY(cudaStreamSynchronize(st));
+  uint32_t e = 0;
+  CUDA_TRY(cudaMemcpy(&e, m->err, 4, cudaMemcpyDeviceToHost));
+  if (e) {
+    CUDA_TRY(cudaMemset(m->err, 0, 4));
+    return fail(HERO_ERR_TIMEOUT, "device-side wait bound expired or bad index (error word 0x%x)", e);
+  }
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_set_profiling(hero_model* m, int enable) {
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  m->profiling = enable != 0;
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_get_profile(hero_model* m, double* ms_out, int64_t* launches_out,
+                                        int reset) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  for (auto& p : m->pending) {
+    CUDA_TRY(cudaEventSynchronize(p.e1));
+    float ms = 0.f;
+    CUDA_TRY(cudaEventElapsedTime(&ms, p.e0, p.e1));
+    m->prof_ms[p.cls] += ms;
+    m->event_pool.push_back(p.e0);
+    m->event_pool.push_back(p.e1);
+  }
+  m->pending.clear();
+  for (int k = 0; k < HERO_K_COUNT; ++k) {
+    if (ms_out) ms_out[k] = m->prof_ms[k];
+    if (launches_out) launches_out[k] = m->launches[k];
+    if (reset) {
+      m->prof_ms[k] = 0.0;
+      m->launches[k] = 0;
+    }
+  }
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B, float* C,
+                                            int32_t M, int32_t N, int32_t K, void* cuda_stream) {
+  g_last_error.clear();
+  if (!A || !B || !C || M < 1 || N < 8 || K < 64 || K % 64 != 0 || N % 8 != 0)
+    return fail(HERO_ERR_ARG, "need M >= 1, N >= 8 (N %% 8 == 0), K %% 64 == 0 and non-NULL pointers");
+  static uint32_t* err = nullptr;
+  if (!err) CUDA_TRY(cudaMalloc(&err, 64));
+  int dev = 0;
+  CUDA_TRY(cudaGetDevice(&dev));
+  int sms = 0;
+  CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  CUtensorMap ta, tb;
+  if (!encode_bf16_2d(&ta, A, K, M, 128) || !encode_bf16_2d(&tb, B, K, N, 256))
+    return fail(HERO_ERR_CUDA, "tensor map encoding failed");
+  GemmArgs g{};
+  g.m_static = M;
+  g.m_max = M;
+  g.N = N;
+  g.K = K;
+  g.out_f32 = C;
+  g.ldo = N;
+  g.err = err;
+  CUDA_TRY(launch_gemm_tc(256, EPI_STORE_F32, ta, tb, g, sms, static_cast<cudaStream_t>(cuda_stream)));
+  return HERO_OK;
+}

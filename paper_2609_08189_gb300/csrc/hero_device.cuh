@@ -1,0 +1,235 @@
+// Device-side helpers: math, bf16 packing, PTX wrappers for mbarrier / TMA /
+// tcgen05, and the shared block-closing epilogue.
+#pragma once
+
+#include "hero_internal.cuh"
+
+namespace hero {
+
+__device__ __forceinline__ float sigmoidf_(float x) { return 1.0f / (1.0f + expf(-x)); }
+__device__ __forceinline__ float siluf_(float x) { return x / (1.0f + expf(-x)); }
+// phi(x) = ELU(x) + 1, alpha = 1 (Sec. 3.2)
+__device__ __forceinline__ float phif_(float x) { return x > 0.0f ? x + 1.0f : expf(x); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&b);
+}
+
+__device__ __forceinline__ void unpack_bf16x2(uint32_t u, float& lo, float& hi) {
+  lo = __uint_as_float(u << 16);
+  hi = __uint_as_float(u & 0xffff0000u);
+}
+
+// Load 4 consecutive elements (16-byte aligned fp32, 8-byte aligned bf16) as fp32.
+__device__ __forceinline__ float4 load4(const void* base, size_t idx, int is_bf16) {
+  if (is_bf16) {
+    uint2 u = *reinterpret_cast<const uint2*>(static_cast<const uint16_t*>(base) + idx);
+    float4 r;
+    unpack_bf16x2(u.x, r.x, r.y);
+    unpack_bf16x2(u.y, r.z, r.w);
+    return r;
+  }
+  return *reinterpret_cast<const float4*>(static_cast<const float*>(base) + idx);
+}
+
+__device__ __forceinline__ void store4(void* base, size_t idx, float4 v, int is_bf16) {
+  if (is_bf16) {
+    uint2 u;
+    u.x = pack_bf16x2(v.x, v.y);
+    u.y = pack_bf16x2(v.z, v.w);
+    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(base) + idx) = u;
+  } else {
+    *reinterpret_cast<float4*>(static_cast<float*>(base) + idx) = v;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Block-closing epilogue on 4 consecutive columns n..n+3 of token t.
+// y: GEMM outputs, s: branch scale.  Accumulates the partial sums.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void layer_out4(const LayerOutArgs& p, int t, int n, float4 y, float s,
+                                           float& ss, float& dd, float& dp) {
+  const size_t off = (size_t)t * p.d + n;
+  float4 hb = *reinterpret_cast<const float4*>(p.hbar + off);
+  float4 h;
+  h.x = hb.x + s * y.x;
+  h.y = hb.y + s * y.y;
+  h.z = hb.z + s * y.z;
+  h.w = hb.w + s * y.w;
+  if (p.last) {
+    *reinterpret_cast<float4*>(p.h_out + off) = h;
+    return;
+  }
+  float4 pn = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (p.p_next) pn = load4(p.p_next, off, p.p_bf16);
+  float4 hn;
+  hn.x = h.x + pn.x; hn.y = h.y + pn.y; hn.z = h.z + pn.z; hn.w = h.w + pn.w;
+  *reinterpret_cast<float4*>(p.hbar + off) = hn;
+  ss += hn.x * hn.x + hn.y * hn.y + hn.z * hn.z + hn.w * hn.w;
+  if (p.router) {  // the router of the next block needs delta and the operand copy
+    float4 dprev = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (!p.first) dprev = *reinterpret_cast<const float4*>(p.delta + off);
+    float4 dn;
+    dn.x = s * y.x + pn.x; dn.y = s * y.y + pn.y; dn.z = s * y.z + pn.z; dn.w = s * y.w + pn.w;
+    *reinterpret_cast<float4*>(p.delta + off) = dn;
+    store4(p.xl, off, hn, p.xl_bf16);
+    dd += dn.x * dn.x + dn.y * dn.y + dn.z * dn.z + dn.w * dn.w;
+    dp += dn.x * dprev.x + dn.y * dprev.y + dn.z * dprev.z + dn.w * dprev.w;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// PTX wrappers (sm_100 family: mbarrier, TMA, tcgen05)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: true when the phase with the given parity completed, false after
+// limit_ns of %globaltimer.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 x bf16 -> fp32, M = 128, one CTA.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier once every tcgen05 operation issued so far by this thread
+// has completed.
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major tile stored with the 128-byte
+// swizzle (rows of 128 bytes, 8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+  d |= (uint64_t)1 << 16;                    // leading byte offset (unused with swizzle)
+  d |= (uint64_t)(1024 >> 4) << 32;          // stride byte offset: 8 rows x 128 B
+  d |= (uint64_t)1 << 46;                    // descriptor version
+  d |= (uint64_t)2 << 61;                    // 128-byte swizzle
+  return d;
+}
+
+#define HERO_R8(i) "=r"(r[i]), "=r"(r[i + 1]), "=r"(r[i + 2]), "=r"(r[i + 3]), \
+                   "=r"(r[i + 4]), "=r"(r[i + 5]), "=r"(r[i + 6]), "=r"(r[i + 7])
+
+// 32 lanes x 32 consecutive fp32 columns from TMEM (lane quadrant of this warp),
+// waiting for the load inside the same asm statement.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : HERO_R8(0), HERO_R8(8), HERO_R8(16), HERO_R8(24)
+      : "r"(taddr)
+      : "memory");
+}
+
+// 16 consecutive fp32 columns.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : HERO_R8(0), HERO_R8(8)
+      : "r"(taddr)
+      : "memory");
+}
+
+}  // namespace hero

@@ -1,0 +1,187 @@
+// Internal declarations shared by the kernels and the host runtime of libhero.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace hero {
+
+// Device error word bits (set by kernels, read by hero_check_device_status).
+enum : uint32_t {
+  ERR_WAIT_PRODUCER = 1u,
+  ERR_WAIT_MMA = 2u,
+  ERR_WAIT_EPILOGUE = 4u,
+  ERR_WAIT_DRAIN = 8u,
+  ERR_BAD_INDEX = 16u,
+};
+
+// Bound on every device-side wait (nanoseconds of %globaltimer).
+constexpr uint64_t kWaitLimitNs = 4000000000ull;
+
+// ---------------------------------------------------------------------------
+// Epilogue of the two GEMMs that close a routed block (FFN down, adapter up):
+// for compacted row m with token t = idx[m] and branch scale s = scale[m],
+// and y = the GEMM output row,
+//     h_j       = h_bar_j + s * y                        (Eq. 3)
+//   if this is not the last block:
+//     h_bar_{j+1} = h_j + P_{j+1}                        (Eq. 1 stand-in)
+//     delta_{j+1} = h_bar_{j+1} - h_bar_j = s * y + P_{j+1}   (Eq. 7)
+//   and per (token, column tile) partial sums of h_bar_{j+1}^2, delta_{j+1}^2
+//   and delta_{j+1} . delta_j feed the next block's RMSNorm (Eq. 5, LN^ffn) and
+//   transition features (Eqs. 7-8).  The last block writes h_j to h_out.
+// ---------------------------------------------------------------------------
+struct LayerOutArgs {
+  const int* idx;        // [rows] compacted row -> token
+  const float* scale;    // [rows] branch scale (g, 1 - g, or 1)
+  float* hbar;           // [T, d] in: h_bar_j; out: h_bar_{j+1}
+  float* delta;          // [T, d] in: delta_j (unless first); out: delta_{j+1}
+  const void* p_next;    // [T, d] P_{j+1} (bf16 or fp32) or nullptr (= 0)
+  void* xl;              // [T, d] out: h_bar_{j+1} in the GEMM operand dtype
+  float* part;           // [T, np, 4] out: partial sums per column tile
+  float* h_out;          // [T, d] out (last block only)
+  int d;
+  int np;                // partial slots per token
+  int tile_n;            // columns per partial slot
+  int last;              // 1: write h_out only
+  int first;             // 1: delta_j = 0 (do not read it)
+  int p_bf16;            // P_{j+1} element type
+  int xl_bf16;           // operand element type of xl
+  int router;            // 0 (dense stack): skip delta and the operand copy
+};
+
+// GEMM problem description shared by the tensor-core and SIMT GEMMs.
+enum EpiKind : int {
+  EPI_STORE_F32 = 0,   // out_f32[m, n] = acc
+  EPI_SWIGLU = 1,      // out[m, n] = SiLU(gate) * up   (gate/up column pairs)
+  EPI_SILU = 2,        // out[m, n] = SiLU(acc)
+  EPI_LAYER_OUT = 3,   // LayerOutArgs
+};
+
+struct GemmArgs {
+  const int* m_dev;    // device row count (nullptr: use m_static)
+  int m_static;
+  int m_max;           // upper bound of M (sizes the grid)
+  int N, K;
+  // outputs
+  float* out_f32;      // EPI_STORE_F32
+  void* out;           // EPI_SWIGLU / EPI_SILU: bf16 (tensor-core path) or f32
+  int ldo;             // leading dimension of out / out_f32 in elements
+  LayerOutArgs lo;     // EPI_LAYER_OUT
+  uint32_t* err;
+  // SIMT path only (row-major [rows, K] operands)
+  const void* A;
+  const void* B;
+  const void* B2;      // EPI_SWIGLU: up-projection weights (gate in B)
+  int lda, ldb;
+};
+
+// Tensor-core GEMM (tcgen05 + TMA + TMEM), bf16 operands, fp32 accumulation.
+// A: [rows, K] K-major; B: [N, K] K-major.  BN = 256 (STORE/SWIGLU/LAYER_OUT) or
+// 64 (SILU, the adapter's rank-64 projection).
+cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                           const GemmArgs& args, int num_sms, cudaStream_t st);
+
+// SIMT fp32 GEMM with the same epilogues (f32 models).
+cudaError_t launch_gemm_simt(EpiKind epi, const GemmArgs& args, cudaStream_t st);
+constexpr int kSimtTileN = 64;
+
+// Router and bookkeeping kernels ------------------------------------------------
+
+struct RouterWeights {   // shared router parameters, fp32, transposed to [in][out]
+  const float* w_hu_t;    // [d_enc][d_h]
+  const float* path_w1_t; // [6][d_path]
+  const float* path_b1;   // [d_path]
+  const float* path_w2_t; // [d_path][d_a]
+  const float* path_b2;   // [d_a]
+  const float* w_qkv_t;   // [d_s][3 d_m]  (q | k | v)
+  const float* w_n_t;     // [d_s][d_m]
+  const float* w_c_t;     // [d_m][d_m]
+  const float* th_w1_t;   // [d_s + d_m + 1][d_head]
+  const float* th_b1;     // [d_head]
+  const float* th_w2;     // [d_head]
+  const float* th_b2;     // [1]
+  const float* ps_b1;     // [d_head]
+  const float* ps_w2;     // [d_head]
+  const float* ps_b2;     // [1]
+};
+
+struct RouterArgs {
+  int T, j, L, np;       // j is 1-based
+  int d, d_h, d_a, d_enc, d_head, d_path;
+  const float* Y;        // [T, d_enc + d_head] router contraction output
+  const float* part;     // [T, np, 4]
+  float* dprev;          // [T] in: d_{j-1}; out: d_j
+  float* pst;            // [T] p_hist
+  float* mst;            // [T] m_hist
+  float* S;              // [T, d_m, d_m]
+  float* zeta;           // [T, d_m]
+  float rho;
+  RouterWeights w;
+  float rms_eps, eps, t_hist, tau;
+  const uint8_t* mask_in;  // [T] decisions of this block (FORCE_MASK) or nullptr
+  float* gate;           // [T]
+  uint8_t* mask;         // [T]
+  float* gate_out;       // [T] caller slice or nullptr
+  uint8_t* mask_out;     // [T] caller slice or nullptr
+};
+
+cudaError_t launch_router(int d_m, const RouterArgs& a, cudaStream_t st);
+
+struct InitArgs {
+  int T, d, np, d_m;
+  const float* h_in;     // [T, d] (may equal hbar for in-place)
+  const void* p0;        // [T, d] P_1 or nullptr
+  int p_bf16;
+  float* hbar;
+  void* xl;
+  int xl_bf16;
+  float* part;
+  float* S;
+  float* zeta;
+  float* pst;
+  float* mst;
+  float* dprev;
+  int reset_router;      // 0 in dense mode
+};
+cudaError_t launch_init(const InitArgs& a, cudaStream_t st);
+
+struct CompactArgs {
+  int T;
+  const uint8_t* mask;   // [T]
+  const float* gate;     // [T]
+  int dense;             // all tokens FFN, scale 1
+  int* idx_f;
+  int* idx_a;
+  float* scale_f;
+  float* scale_a;
+  int* counts;           // [2] n_f, n_a
+  int* count_out;        // caller slot or nullptr
+  float* gate_out;       // dense mode: fill with 1 (or nullptr)
+  uint8_t* mask_out;     // dense mode: fill with 1 (or nullptr)
+};
+cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
+
+struct NormArgs {
+  int T, d, np;
+  const int* counts;
+  const int* idx_f;
+  const int* idx_a;
+  const float* hbar;
+  const float* part;
+  const float* gain;     // [d]
+  float rms_eps;
+  void* u_f;             // [T, d]
+  void* u_a;             // [T, d]
+  int out_bf16;
+};
+cudaError_t launch_norm(const NormArgs& a, cudaStream_t st);
+
+// Weight conversion: dst[map(r)] = convert(src[r]) for rows of `cols` elements.
+// map(r) = (r / grp) * grp_stride + (r % grp) + offset.
+cudaError_t launch_convert_rows(const void* src, int src_bf16, void* dst, int dst_bf16,
+                                long rows, long cols, long grp, long grp_stride, long offset,
+                                const float* col_scale, cudaStream_t st);
+
+}  // namespace hero

@@ -1,0 +1,213 @@
+"""ctypes binding of libhero (include/hero.h): argument marshalling only.
+
+Every step of the routed FFN stack runs in the CUDA kernels of libhero.so; this
+module only converts Python/PyTorch arguments into the C ABI's plain pointers and
+sizes.  There is no fallback: if the library is missing or fails to load, every
+entry point raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Optional, Sequence
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libhero.so")
+
+HERO_OK, HERO_ERR_ARG, HERO_ERR_CUDA, HERO_ERR_NOMEM, HERO_ERR_UNSUPPORTED, HERO_ERR_TIMEOUT = range(6)
+STATUS_NAMES = {0: "HERO_OK", 1: "HERO_ERR_ARG", 2: "HERO_ERR_CUDA", 3: "HERO_ERR_NOMEM",
+                4: "HERO_ERR_UNSUPPORTED", 5: "HERO_ERR_TIMEOUT"}
+HERO_F32, HERO_BF16 = 0, 1
+HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO = 1, 2, 4
+KERNEL_CLASSES = ("init", "router_gemm", "router", "compact", "norm", "ffn_gate_up", "ffn_down",
+                  "adapter_down", "adapter_up")
+HERO_K_COUNT = len(KERNEL_CLASSES)
+
+WEIGHT_FIELDS = ("ffn_norm_g", "w_gate", "w_up", "w_down", "ad_w1", "ad_w2", "eta",
+                 "r_norm_g", "w_hd", "w_hu", "path_w1", "path_b1", "path_w2", "path_b2",
+                 "w_q", "w_k", "w_v", "w_n", "w_c", "th_w1", "th_b1", "th_w2", "th_b2",
+                 "ps_w1", "ps_b1", "ps_w2", "ps_b2")
+
+
+class hero_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("n_layers", "d_model", "d_ff", "d_r", "d_m", "d_h", "d_a", "d_enc", "d_head",
+                 "d_path", "max_tokens")] + \
+               [("dtype", ctypes.c_int), ("rms_eps", ctypes.c_float), ("eps", ctypes.c_float),
+                ("t_hist", ctypes.c_float)]
+
+
+class hero_weights_host(ctypes.Structure):
+    _fields_ = [("host_dtype", ctypes.c_int)] + [(n, ctypes.c_void_p) for n in WEIGHT_FIELDS]
+
+
+class HeroError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def load(path: Optional[str] = None) -> ctypes.CDLL:
+    """Load libhero.so (raises if it is missing; build it with __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libhero.so not found at {p}; run __graft_entry__.build()")
+    lib = ctypes.CDLL(p)
+    vp, i32, i64, f32, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_uint32
+    lib.hero_init_weights.argtypes = [ctypes.POINTER(hero_config), ctypes.POINTER(hero_weights_host),
+                                      ctypes.POINTER(vp)]
+    lib.hero_init_weights.restype = ctypes.c_int
+    lib.hero_routed_ffn_stack.argtypes = [vp, i64, vp, vp, f32, u32, vp, vp, vp, vp, vp, vp]
+    lib.hero_routed_ffn_stack.restype = ctypes.c_int
+    lib.hero_free.argtypes = [vp]
+    lib.hero_free.restype = None
+    lib.hero_last_error.argtypes = []
+    lib.hero_last_error.restype = ctypes.c_char_p
+    lib.hero_check_device_status.argtypes = [vp, vp]
+    lib.hero_check_device_status.restype = ctypes.c_int
+    lib.hero_set_profiling.argtypes = [vp, ctypes.c_int]
+    lib.hero_set_profiling.restype = ctypes.c_int
+    lib.hero_get_profile.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64), ctypes.c_int]
+    lib.hero_get_profile.restype = ctypes.c_int
+    lib.hero_gemm_bf16_check.argtypes = [vp, vp, vp, i32, i32, i32, vp]
+    lib.hero_gemm_bf16_check.restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _check(status: int) -> None:
+    if status != HERO_OK:
+        raise HeroError(status, hero_last_error())
+
+
+def hero_last_error() -> str:
+    return load().hero_last_error().decode()
+
+
+def make_config(stack_cfg, max_tokens: Optional[int] = None) -> hero_config:
+    """hero_config from a synth StackConfig."""
+    c = stack_cfg
+    return hero_config(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a, c.d_enc,
+                       c.d_head, c.d_path, max_tokens or c.n_tokens,
+                       HERO_BF16 if c.dtype == "bf16" else HERO_F32, c.rms_eps, c.eps, c.t_hist)
+
+
+def make_weights(weights: Dict[str, np.ndarray]):
+    """hero_weights_host pointing into contiguous numpy arrays (kept alive by the caller)."""
+    arrs = {k: np.ascontiguousarray(weights[k]) for k in WEIGHT_FIELDS}
+    dts = {a.dtype for a in arrs.values()}
+    if dts == {np.dtype(np.uint16)}:
+        hd = HERO_BF16
+    elif dts == {np.dtype(np.float32)}:
+        hd = HERO_F32
+    else:
+        raise TypeError(f"weights must be all float32 or all uint16 bf16 bits, got {dts}")
+    w = hero_weights_host(hd, *[arrs[k].ctypes.data for k in WEIGHT_FIELDS])
+    return w, arrs
+
+
+def hero_init_weights(cfg: hero_config, weights: Dict[str, np.ndarray]) -> int:
+    w, keep = make_weights(weights)
+    out = ctypes.c_void_p()
+    _check(load().hero_init_weights(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(out)))
+    del keep
+    return out.value
+
+
+def hero_routed_ffn_stack(model: int, n_tokens: int, h_in: int, attn_delta: int, tau_exec: float,
+                          flags: int, mask_in: int, h_out: int, gate_out: int, mask_out: int,
+                          ffn_count_out: int, cuda_stream: int) -> None:
+    """Pointer-level call (ints are raw addresses, 0 for NULL)."""
+    _check(load().hero_routed_ffn_stack(model, n_tokens, h_in or None, attn_delta or None,
+                                        float(tau_exec), flags, mask_in or None, h_out or None,
+                                        gate_out or None, mask_out or None, ffn_count_out or None,
+                                        cuda_stream or None))
+
+
+def hero_free(model: int) -> None:
+    if model:
+        load().hero_free(model)
+
+
+def hero_check_device_status(model: int, cuda_stream: int = 0) -> None:
+    _check(load().hero_check_device_status(model, cuda_stream or None))
+
+
+def hero_set_profiling(model: int, enable: bool) -> None:
+    _check(load().hero_set_profiling(model, 1 if enable else 0))
+
+
+def hero_get_profile(model: int, reset: bool = True):
+    ms = (ctypes.c_double * HERO_K_COUNT)()
+    n = (ctypes.c_int64 * HERO_K_COUNT)()
+    _check(load().hero_get_profile(model, ms, n, 1 if reset else 0))
+    return {k: (ms[i], n[i]) for i, k in enumerate(KERNEL_CLASSES)}
+
+
+def hero_gemm_bf16_check(A: int, B: int, C: int, M: int, N: int, K: int, cuda_stream: int = 0) -> None:
+    _check(load().hero_gemm_bf16_check(A, B, C, M, N, K, cuda_stream or None))
+
+
+# ---------------------------------------------------------------------------
+# PyTorch convenience layer (device tensors, current stream)
+# ---------------------------------------------------------------------------
+
+class HeroStack:
+    """A loaded model plus torch-tensor calls.  PyTorch supplies memory and streams."""
+
+    def __init__(self, stack_cfg, weights: Dict[str, np.ndarray], max_tokens: Optional[int] = None):
+        self.cfg = stack_cfg
+        self.max_tokens = max_tokens or stack_cfg.n_tokens
+        self.model = hero_init_weights(make_config(stack_cfg, self.max_tokens), weights)
+
+    def close(self):
+        if self.model:
+            hero_free(self.model)
+            self.model = 0
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __call__(self, h_in, attn_delta, tau: float, flags: int = 0, mask_in=None,
+                 h_out=None, gate_out=None, mask_out=None, counts_out=None, stream=None):
+        """Device tensors in and out.  Returns (h_out, gate, mask, counts)."""
+        import torch
+        T, d = h_in.shape
+        L = self.cfg.n_layers
+        dev = h_in.device
+        if h_out is None:
+            h_out = torch.empty((T, d), dtype=torch.float32, device=dev)
+        if gate_out is None:
+            gate_out = torch.empty((L, T), dtype=torch.float32, device=dev)
+        if mask_out is None:
+            mask_out = torch.empty((L, T), dtype=torch.uint8, device=dev)
+        if counts_out is None:
+            counts_out = torch.empty((L,), dtype=torch.int32, device=dev)
+        for t in (h_in, h_out, gate_out, mask_out, counts_out):
+            assert t.is_contiguous()
+        if attn_delta is not None:
+            assert attn_delta.is_contiguous() and attn_delta.shape == (L, T, d)
+        st = stream if stream is not None else torch.cuda.current_stream(dev)
+        hero_routed_ffn_stack(self.model, T, h_in.data_ptr(),
+                              attn_delta.data_ptr() if attn_delta is not None else 0,
+                              tau, flags, mask_in.data_ptr() if mask_in is not None else 0,
+                              h_out.data_ptr(), gate_out.data_ptr(), mask_out.data_ptr(),
+                              counts_out.data_ptr(), st.cuda_stream)
+        return h_out, gate_out, mask_out, counts_out
+
+    def check(self, stream=None):
+        import torch
+        st = stream if stream is not None else torch.cuda.current_stream()
+        hero_check_device_status(self.model, st.cuda_stream)

@@ -1,0 +1,212 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Small workloads compare every token; the full-size workloads run all T tokens on
+the GPU in the bench's launch configuration and compare an evenly spread token
+sample with the oracle run on exactly those tokens (tokens are independent
+through the stack, P6 of the oracle pins).
+"""
+
+import numpy as np
+import pytest
+
+from synth import hero_inputs as hi
+from tests import parity as pr
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hero():
+    import torch
+    assert torch.cuda.is_available()
+    from paper_2609_08189_gb300 import build, hero as H
+    build.build()
+    H.load()
+    return H
+
+
+def _stack(H, inp, max_tokens=None):
+    return H.HeroStack(inp.cfg, inp.weights, max_tokens=max_tokens)
+
+
+def _assert_free(rep, tol_h, max_boundary_frac=0.02):
+    assert rep.mask_mismatch_far == 0, rep
+    assert rep.gate_err < pr.GATE_TOL, rep
+    assert len(rep.boundary_tokens) <= max(1, max_boundary_frac * rep.n_tokens), rep
+    assert rep.compared_h >= 0.9 * rep.n_tokens, rep
+    assert rep.h_err < tol_h, rep
+
+
+# ------------------------------------------------------------------------------
+# the tensor-core GEMM alone
+# ------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("M,N,K", [(1, 256, 64), (128, 512, 128), (129, 264, 4096), (333, 512, 1024),
+                                   (1000, 768, 256)])
+def test_gemm_building_block(hero, M, N, K):
+    import torch
+    g = torch.Generator(device="cuda").manual_seed(M * 7 + N + K)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
+    B = torch.randn(N, K, device="cuda", generator=g).to(torch.bfloat16)
+    C = torch.full((M, N), float("nan"), device="cuda")
+    hero.hero_gemm_bf16_check(A.data_ptr(), B.data_ptr(), C.data_ptr(), M, N, K,
+                              torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    ref = A.double() @ B.double().T
+    err = (C.double() - ref).abs().max().item()
+    assert err <= 1e-5 * K ** 0.5 * ref.abs().max().item() + 1e-6, err
+
+
+# ------------------------------------------------------------------------------
+# full-token parity on small workloads
+# ------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+def test_free_running(hero, name):
+    inp = pr.inputs(name)
+    st = _stack(hero, inp)
+    gpu = pr.run_gpu(st, inp)
+    ref = pr.run_oracle(inp)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL[inp.cfg.dtype])
+    print(name, rep)
+    _assert_free(rep, pr.H_TOL[inp.cfg.dtype])
+    np.testing.assert_array_equal(gpu.counts, gpu.mask.sum(axis=1))
+    bypass = 1 - gpu.mask.mean()
+    assert abs(bypass - inp.cfg.bypass) < 0.03
+    st.close()
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+def test_forced_mask(hero, name):
+    inp = pr.inputs(name)
+    st = _stack(hero, inp)
+    ref = pr.run_oracle(inp)
+    gpu = pr.run_gpu(st, inp, flags=hero.HERO_FLAG_FORCE_MASK, mask_in=ref["mask"])
+    rep = pr.compare_forced(gpu, ref)
+    print(name, rep)
+    assert rep.mask_mismatch_far == 0
+    assert rep.gate_err < pr.GATE_TOL
+    assert rep.h_err < pr.H_TOL[inp.cfg.dtype]
+    st.close()
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+def test_dense(hero, name):
+    inp = pr.inputs(name)
+    st = _stack(hero, inp)
+    ref = pr.run_oracle(inp, mode="dense")
+    gpu = pr.run_gpu(st, inp, flags=hero.HERO_FLAG_DENSE)
+    assert (gpu.mask == 1).all() and (gpu.gate == 1).all()
+    assert (gpu.counts == inp.cfg.n_tokens).all()
+    err = np.max(pr.rel_err_rows(gpu.h_out, ref["h_out"]))
+    assert err < pr.H_TOL[inp.cfg.dtype], err
+    st.close()
+
+
+@pytest.mark.parametrize("name,path", [("tiny_f32", 0), ("tiny_f32", 1), ("small_bf16", 0),
+                                       ("small_bf16", 1)])
+def test_single_branch_everywhere(hero, name, path):
+    """Forced all-adapter and all-FFN paths (one branch empty at every block)."""
+    inp = pr.inputs(name)
+    L, T = inp.cfg.n_layers, inp.cfg.n_tokens
+    mask = np.full((L, T), path, dtype=np.uint8)
+    st = _stack(hero, inp)
+    ref = pr.run_oracle(inp, mode="force", mask_in=mask)
+    gpu = pr.run_gpu(st, inp, flags=hero.HERO_FLAG_FORCE_MASK, mask_in=mask)
+    assert (gpu.counts == path * T).all()
+    assert np.max(np.abs(gpu.gate - ref["gate"])) < pr.GATE_TOL
+    assert np.max(pr.rel_err_rows(gpu.h_out, ref["h_out"])) < pr.H_TOL[inp.cfg.dtype]
+    st.close()
+
+
+@pytest.mark.parametrize("T", [1, 2, 127, 129])
+def test_ragged_token_counts(hero, T):
+    """Fewer tokens than the model was sized for, including a single token."""
+    inp = pr.inputs("small_bf16")
+    st = _stack(hero, inp)
+    rows = np.arange(T)
+    gpu = pr.run_gpu(st, inp, n_tokens=T)
+    ref = pr.run_oracle(inp, rows=rows)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"])
+    _assert_free(rep, pr.H_TOL["bf16"], max_boundary_frac=0.5)
+    st.close()
+
+
+def test_zero_tokens_and_argument_errors(hero):
+    import torch
+    inp = pr.inputs("tiny_f32")
+    st = _stack(hero, inp)
+    counts = torch.full((inp.cfg.n_layers,), 7, dtype=torch.int32, device="cuda")
+    hero.hero_routed_ffn_stack(st.model, 0, 0, 0, inp.tau, 0, 0, 0, 0, 0, counts.data_ptr(), 0)
+    torch.cuda.synchronize()
+    assert (counts == 0).all()
+    x = torch.zeros((inp.cfg.n_tokens, inp.cfg.d_model), device="cuda")
+    with pytest.raises(hero.HeroError) as e:   # T above max_tokens
+        hero.hero_routed_ffn_stack(st.model, inp.cfg.n_tokens + 1, x.data_ptr(), 0, 0.5, 0, 0,
+                                   x.data_ptr() + 4, 0, 0, 0, 0)
+    assert e.value.status == hero.HERO_ERR_ARG
+    with pytest.raises(hero.HeroError) as e:   # aliasing in/out
+        hero.hero_routed_ffn_stack(st.model, 4, x.data_ptr(), 0, 0.5, 0, 0, x.data_ptr(), 0, 0, 0, 0)
+    assert e.value.status == hero.HERO_ERR_ARG
+    st.check()
+    st.close()
+
+
+def test_host_io_matches_device_path(hero):
+    """HERO_FLAG_HOST_IO (host buffers, copies inside the call) == device buffers."""
+    import torch
+    inp = pr.inputs("small_bf16")
+    st = _stack(hero, inp)
+    dev = pr.run_gpu(st, inp)
+    L, T, d = inp.cfg.n_layers, inp.cfg.n_tokens, inp.cfg.d_model
+    h = torch.from_numpy(inp.h).pin_memory()
+    P = torch.from_numpy(inp.P).pin_memory()
+    h_out = torch.empty((T, d), dtype=torch.float32).pin_memory()
+    g = torch.empty((L, T), dtype=torch.float32).pin_memory()
+    m = torch.empty((L, T), dtype=torch.uint8).pin_memory()
+    c = torch.empty((L,), dtype=torch.int32).pin_memory()
+    hero.hero_routed_ffn_stack(st.model, T, h.data_ptr(), P.data_ptr(), inp.tau,
+                               hero.HERO_FLAG_HOST_IO, 0, h_out.data_ptr(), g.data_ptr(),
+                               m.data_ptr(), c.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(h_out.numpy(), dev.h_out.astype(np.float32))
+    np.testing.assert_array_equal(m.numpy(), dev.mask)
+    np.testing.assert_array_equal(c.numpy(), dev.counts)
+    st.close()
+
+
+# ------------------------------------------------------------------------------
+# full-size workloads, sampled tokens
+# ------------------------------------------------------------------------------
+
+FULL = [("llama2_7b_prefill", None, 64), ("llama31_8b_prefill", None, 64),
+        ("llama31_8b_decode", None, 64), ("llama2_13b_prefill", 0.27, 32)]
+
+
+@pytest.mark.parametrize("name,bypass,n_sample", FULL)
+def test_full_size_sampled(hero, name, bypass, n_sample):
+    import torch
+    inp = pr.inputs(name, bypass=bypass)
+    cfg = inp.cfg
+    rows = hi.sample_tokens(cfg.n_tokens, n_sample)
+    st = _stack(hero, inp)
+    gpu_all = pr.run_gpu(st, inp)          # all T tokens, bench launch configuration
+    gpu = pr.GpuRun(gpu_all.h_out[rows], gpu_all.gate[:, rows], gpu_all.mask[:, rows], gpu_all.counts)
+    ref = pr.run_oracle(inp, rows=rows)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"])
+    print(name, rep, "bypass", 1 - gpu_all.mask.mean())
+    _assert_free(rep, pr.H_TOL["bf16"], max_boundary_frac=0.1)
+    # whole-workload properties: counts agree with decisions, bypass near the budget
+    np.testing.assert_array_equal(gpu_all.counts, gpu_all.mask.sum(axis=1))
+    target = cfg.bypass if bypass is None else bypass
+    assert abs((1 - gpu_all.mask.mean()) - target) < 0.05
+    # forced mode on the sample: the GPU follows the oracle's decisions
+    mask_in = gpu_all.mask.copy()
+    mask_in[:, rows] = ref["mask"]
+    forced = pr.run_gpu(st, inp, flags=hero.HERO_FLAG_FORCE_MASK, mask_in=mask_in, rows=rows)
+    frep = pr.compare_forced(forced, ref)
+    print(name, "forced", frep)
+    assert frep.gate_err < pr.GATE_TOL and frep.h_err < pr.H_TOL["bf16"]
+    st.close()
+    del gpu_all
+    torch.cuda.empty_cache()
