@@ -169,6 +169,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    # overrides for profiling small cases (a line produced with them is not the workload's)
+    ap.add_argument("--tau", type=float, default=None)
+    ap.add_argument("--tokens", type=int, default=None)
+    ap.add_argument("--layers", type=int, default=None)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -193,7 +197,9 @@ def main():
     hero.load()
 
     cfg = hi.CONFIGS[args.workload]
-    tau = hi.calibrated_tau(cfg.name)
+    tau = hi.calibrated_tau(cfg.name) if args.tau is None else args.tau
+    if args.tokens or args.layers:
+        cfg = cfg.replace(n_tokens=args.tokens or cfg.n_tokens, n_layers=args.layers or cfg.n_layers)
     T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
     t_gen = time.time()
     w = hi.generate_weights(cfg)

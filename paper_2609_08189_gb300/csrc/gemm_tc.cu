@@ -32,7 +32,9 @@ struct TcCfg {
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                     ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-  static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+  // ring | barriers (256 B) | per-epilogue-warp staging tiles (4 x 32 x 32 fp32)
+  static constexpr uint32_t EPI_STAGE_OFF = STAGES * STAGE_BYTES + 256;
+  static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + 4 * 32 * 32 * 4 + 1024;
 };
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
@@ -47,25 +49,42 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
 
 // ---- epilogues: one thread = one tile row; TMEM read in 32 or 16 column chunks ----
 
+// Stage one warp's 32 rows x 32 fp32 columns through shared memory so that the
+// global accesses that follow are row-contiguous: lane l then owns float4 slot
+// (l & 7) of rows (l >> 3) + 4k, k = 0..7 (128 contiguous bytes per row per
+// instruction).  Float4 slots are XOR-swizzled by row to avoid bank conflicts.
+__device__ __forceinline__ void stage_rows(float4* st, const uint32_t (&r)[32], int lane) {
+#pragma unroll
+  for (int c4 = 0; c4 < 8; ++c4)
+    st[lane * 8 + (c4 ^ (lane & 7))] =
+        make_float4(__uint_as_float(r[4 * c4]), __uint_as_float(r[4 * c4 + 1]),
+                    __uint_as_float(r[4 * c4 + 2]), __uint_as_float(r[4 * c4 + 3]));
+}
+
+__device__ __forceinline__ float4 staged(const float4* st, int row, int slot) {
+  return st[row * 8 + (slot ^ (row & 7))];
+}
+
 template <int BN>
-__device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase, int m, bool valid,
-                                              int nb) {
+__device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase, int row0, int M,
+                                              int nb, float4* st) {
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> 3, slot = lane & 7;
 #pragma unroll 1
   for (int c0 = 0; c0 < BN; c0 += 32) {
     uint32_t r[32];
     tmem_ld32(tbase + c0, r);
-    const int n0 = nb * BN + c0;
-    if (valid) {
-      float* dst = a.out_f32 + (size_t)m * a.ldo + n0;
+    stage_rows(st, r, lane);
+    __syncwarp();
+    const int n = nb * BN + c0 + 4 * slot;
 #pragma unroll
-      for (int i = 0; i < 32; i += 4) {
-        if (n0 + i < a.N) {
-          *reinterpret_cast<float4*>(dst + i) =
-              make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]),
-                          __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3]));
-        }
-      }
+    for (int k = 0; k < 8; ++k) {
+      const int rr = sub + 4 * k;
+      const int m = row0 + rr;
+      if (m < M && n < a.N)
+        *reinterpret_cast<float4*>(a.out_f32 + (size_t)m * a.ldo + n) = staged(st, rr, slot);
     }
+    __syncwarp();
   }
 }
 
@@ -114,32 +133,61 @@ __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int 
   }
 }
 
+// Block-closing epilogue, row-contiguous through the staging tile.  Each lane
+// keeps the partial sums of its 8 rows and reduces them over the 8 lanes that
+// share a row at the end of the tile.
 template <int BN>
-__device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase, int m, bool valid,
-                                              int nb) {
-  int t = 0;
-  float s = 0.f;
-  if (valid) {
-    t = a.lo.idx[m];
-    s = a.lo.scale[m];
+__device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase, int row0, int M,
+                                              int nb, float4* st) {
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> 3, slot = lane & 7;
+  const LayerOutArgs& p = a.lo;
+  int tok[8];
+  float scl[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int m = row0 + sub + 4 * k;
+    tok[k] = m < M ? p.idx[m] : -1;
+    scl[k] = m < M ? p.scale[m] : 0.f;
   }
-  float ss = 0.f, dd = 0.f, dp = 0.f;
+  float ss[8], dd[8], dp[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) ss[k] = dd[k] = dp[k] = 0.f;
 #pragma unroll 1
   for (int c0 = 0; c0 < BN; c0 += 32) {
     uint32_t r[32];
     tmem_ld32(tbase + c0, r);
-    if (valid) {
+    stage_rows(st, r, lane);
+    __syncwarp();
+    const int n = nb * BN + c0 + 4 * slot;
+    // two groups of 4 rows: issue every load of a group before any store
 #pragma unroll
-      for (int i = 0; i < 32; i += 4) {
-        const float4 y = make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]),
-                                     __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3]));
-        layer_out4(a.lo, t, nb * BN + c0 + i, y, s, ss, dd, dp);
-      }
+    for (int k0 = 0; k0 < 8; k0 += 4) {
+      LayerOutIn in[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if (tok[k0 + k] >= 0) in[k] = layer_out_load(p, tok[k0 + k], n);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if (tok[k0 + k] >= 0)
+          layer_out_store(p, tok[k0 + k], n, in[k], staged(st, sub + 4 * (k0 + k), slot),
+                          scl[k0 + k], ss[k0 + k], dd[k0 + k], dp[k0 + k]);
     }
+    __syncwarp();
   }
-  if (valid && !a.lo.last) {
-    *reinterpret_cast<float4*>(a.lo.part + ((size_t)t * a.lo.np + nb) * 4) =
-        make_float4(ss, dd, dp, 0.f);
+  if (!p.last) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+#pragma unroll
+      for (int o = 1; o < 8; o <<= 1) {
+        ss[k] += __shfl_xor_sync(0xffffffffu, ss[k], o);
+        dd[k] += __shfl_xor_sync(0xffffffffu, dd[k], o);
+        dp[k] += __shfl_xor_sync(0xffffffffu, dp[k], o);
+      }
+      if (slot == 0 && tok[k] >= 0)
+        *reinterpret_cast<float4*>(p.part + ((size_t)tok[k] * p.np + nb) * 4) =
+            make_float4(ss[k], dd[k], dp[k], 0.f);
+    }
   }
 }
 
@@ -304,14 +352,15 @@ __global__ void __launch_bounds__(192, 1)
       const int m = mb * BM + row;
       const bool valid = m < M;
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + q * (32 * 8);
       if constexpr (EPI == EPI_STORE_F32) {
-        epi_store_f32<BN>(args, tbase, m, valid, nb);
+        epi_store_f32<BN>(args, tbase, mb * BM + q * 32, M, nb, stg);
       } else if constexpr (EPI == EPI_SWIGLU) {
         epi_swiglu(args, tbase, m, valid, nb);
       } else if constexpr (EPI == EPI_SILU) {
         epi_silu<BN>(args, tbase, m, valid, nb);
       } else {
-        epi_layer_out<BN>(args, tbase, m, valid, nb);
+        epi_layer_out<BN>(args, tbase, mb * BM + q * 32, M, nb, stg);
       }
       tc_fence_before();
       __syncwarp();

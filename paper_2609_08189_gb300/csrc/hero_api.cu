@@ -178,6 +178,8 @@ hero_status validate_config(const hero_config* c) {
     return fail(HERO_ERR_UNSUPPORTED, "d_m must be 16, 32, 64 or 128 (got %d)", c->d_m);
   if (c->d_h + c->d_a > 128 || c->d_enc > 256 || c->d_head > 256 || c->d_path > 64)
     return fail(HERO_ERR_UNSUPPORTED, "router widths exceed d_s<=128, d_enc,d_head<=256, d_path<=64");
+  if (c->d_h % 4 || c->d_a % 4 || c->d_enc % 4 || c->d_head % 4 || c->d_path % 4)
+    return fail(HERO_ERR_UNSUPPORTED, "router widths d_h, d_a, d_enc, d_head, d_path must be multiples of 4");
   if (c->d_model % 8 != 0) return fail(HERO_ERR_UNSUPPORTED, "d_model must be a multiple of 8");
   if (c->dtype == HERO_BF16) {
     if (c->d_model % 256 != 0 || c->d_ff % 128 != 0 || c->d_r != 64)
@@ -375,6 +377,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     std::vector<float> pack;
     auto add_t = [&](const void* src, long rows, long cols) {  // src [rows][cols] -> [cols][rows]
       std::vector<float> v = host_f32(src, (size_t)rows * cols, hd);
+      pack.resize((pack.size() + 3) & ~(size_t)3);  // 16-byte aligned sub-arrays
       size_t at = pack.size();
       pack.resize(at + (size_t)rows * cols);
       for (long i = 0; i < rows; ++i)
@@ -383,6 +386,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     };
     auto add = [&](const void* src, long n) {
       std::vector<float> v = host_f32(src, n, hd);
+      pack.resize((pack.size() + 3) & ~(size_t)3);
       size_t at = pack.size();
       pack.insert(pack.end(), v.begin(), v.end());
       return at;
@@ -393,6 +397,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     size_t o_p2 = add_t(w->path_w2, c.d_a, c.d_path);
     size_t o_pb2 = add(w->path_b2, c.d_a);
     // q | k | v as one [d_s][3 d_m] matrix
+    pack.resize((pack.size() + 3) & ~(size_t)3);
     size_t o_qkv = pack.size();
     pack.resize(o_qkv + (size_t)ds * 3 * dm);
     {

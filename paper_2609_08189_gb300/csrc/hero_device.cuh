@@ -85,6 +85,54 @@ __device__ __forceinline__ void layer_out4(const LayerOutArgs& p, int t, int n, 
   }
 }
 
+// The same epilogue split into a load phase and a compute/store phase so that a
+// caller can keep several rows' loads in flight.
+struct LayerOutIn {
+  float4 hb, pn, dprev;
+};
+
+__device__ __forceinline__ LayerOutIn layer_out_load(const LayerOutArgs& p, int t, int n) {
+  const size_t off = (size_t)t * p.d + n;
+  LayerOutIn in;
+  in.hb = *reinterpret_cast<const float4*>(p.hbar + off);
+  in.pn = make_float4(0.f, 0.f, 0.f, 0.f);
+  in.dprev = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (!p.last) {
+    if (p.p_next) in.pn = load4(p.p_next, off, p.p_bf16);
+    if (p.router && !p.first) in.dprev = *reinterpret_cast<const float4*>(p.delta + off);
+  }
+  return in;
+}
+
+__device__ __forceinline__ void layer_out_store(const LayerOutArgs& p, int t, int n,
+                                                const LayerOutIn& in, float4 y, float s,
+                                                float& ss, float& dd, float& dp) {
+  const size_t off = (size_t)t * p.d + n;
+  float4 h;
+  h.x = in.hb.x + s * y.x;
+  h.y = in.hb.y + s * y.y;
+  h.z = in.hb.z + s * y.z;
+  h.w = in.hb.w + s * y.w;
+  if (p.last) {
+    *reinterpret_cast<float4*>(p.h_out + off) = h;
+    return;
+  }
+  const float4 pn = in.pn;
+  float4 hn;
+  hn.x = h.x + pn.x; hn.y = h.y + pn.y; hn.z = h.z + pn.z; hn.w = h.w + pn.w;
+  *reinterpret_cast<float4*>(p.hbar + off) = hn;
+  ss += hn.x * hn.x + hn.y * hn.y + hn.z * hn.z + hn.w * hn.w;
+  if (p.router) {
+    float4 dn;
+    dn.x = s * y.x + pn.x; dn.y = s * y.y + pn.y; dn.z = s * y.z + pn.z; dn.w = s * y.w + pn.w;
+    *reinterpret_cast<float4*>(p.delta + off) = dn;
+    store4(p.xl, off, hn, p.xl_bf16);
+    const float4 dv = in.dprev;
+    dd += dn.x * dn.x + dn.y * dn.y + dn.z * dn.z + dn.w * dn.w;
+    dp += dn.x * dv.x + dn.y * dv.y + dn.z * dv.z + dn.w * dv.w;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // PTX wrappers (sm_100 family: mbarrier, TMA, tcgen05)
 // ---------------------------------------------------------------------------

@@ -55,71 +55,148 @@ __global__ void __launch_bounds__(256) k_init(const InitArgs a) {
 }
 
 // ------------------------------------------------------------------------------
-// Block-level small matmul: out[t][o] = act(sum_i in[t][i] * Wt[i][o] + bias[o])
-// for t < TB tokens held in shared memory.  Each work item owns one output column
-// for a group of TPG tokens so every weight is loaded once per group.
+// k_router: TB tokens per CTA.  Activations live in shared memory transposed,
+// [feature][TB], so a block matmul loads one float4 of weights (four outputs) and
+// one float4 of activations (four tokens) per 16 FMAs.
 // ------------------------------------------------------------------------------
 constexpr int TB = 16;        // tokens per CTA
 constexpr int NTHR = 256;
 
-template <int TPG>
-__device__ __forceinline__ void bmm_tpg(const float* in, int in_ld, int NI,
-                                        const float* __restrict__ Wt, int NO,
-                                        const float* __restrict__ bias, float* out, int out_ld,
-                                        bool silu_act) {
-  constexpr int G = TB / TPG;
-  for (int w = threadIdx.x; w < NO * G; w += NTHR) {
-    const int o = w % NO;
-    const int g = w / NO;
-    float acc[TPG];
-    const float b = bias ? __ldg(bias + o) : 0.f;
+// Shared-memory layout (floats), computed from the model's widths on host and
+// device alike.  Regions are reused once their contents are dead:
+//   big   [max(d_enc, d_head)][TB]: encoder input (steps 2-3), split-K scratch of
+//         W_n / W_c (step 6), f_theta hidden (steps 7-8)
+//   s     [d_s + d_m + 1][TB]: s | c | nu
+//   qkv   [TB][3 d_m] token-major
+//   aux   [max(3072, 2 d_m TB)]: split-K scratch of W_hu (step 3), W_n s | W_c c (step 6)
+struct RouterLayout {
+  int big, s, qkv, aux, x, ph, red, sc, ab, floats;
+  __host__ __device__ RouterLayout(int d_enc, int d_head, int ds, int dm, int d_path) {
+    const int nbig = (d_enc > d_head ? d_enc : d_head) * TB;
+    const int ns = ((ds + dm + 1 + 3) & ~3) * TB;
+    const int naux = (3072 > 2 * dm * TB ? 3072 : 2 * dm * TB);
+    big = 0;
+    s = big + nbig;
+    qkv = s + ns;
+    aux = qkv + TB * 3 * dm;
+    x = aux + naux;
+    ph = x + 8 * TB;
+    red = ph + d_path * TB;
+    sc = red + 2 * 16 * TB;
+    ab = sc + TB * 16;
+    floats = ab + 2 * TB;
+  }
+};
+
+// out[o][t] = sum_i Wt[i][o] in[i][t]  (+ bias[o], then optional SiLU), o < NO,
+// t < TB; `in` is [NI][TB]; `out` is [NO][TB] or, if out_tok_ld > 0, token-major
+// [TB][out_tok_ld].  Narrow outputs split K across threads; the partial sums go to
+// `scratch` ([ks][NO][TB], at most scratch_cap floats) and are added in a fixed
+// order, so results are bitwise reproducible.  NO must be a multiple of 4;
+// contains __syncthreads.
+__device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int NO,
+                     const float* __restrict__ bias, float* out, int out_tok_ld, bool silu_act,
+                     float* scratch = nullptr, int scratch_cap = 0) {
+  const int no4 = NO >> 2;
+  const int base = no4 * (TB / 4);
+  int ks = 1;
+  if (scratch)
+    while (base * ks * 2 <= NTHR && NI / (ks * 2) >= 16 && (ks * 2) * NO * TB <= scratch_cap) ks <<= 1;
+  const int kchunk = (NI + ks - 1) / ks;
+  auto oidx = [&](int o, int t) { return out_tok_ld > 0 ? t * out_tok_ld + o : o * TB + t; };
+  for (int w = threadIdx.x; w < base * ks; w += NTHR) {
+    const int o4 = (w % no4) * 4;
+    const int rest = w / no4;
+    const int t4 = (rest % (TB / 4)) * 4;
+    const int kk = rest / (TB / 4);
+    const int i0 = kk * kchunk;
+    const int i1 = min(NI, i0 + kchunk);
+    float acc[4][4];
 #pragma unroll
-    for (int t = 0; t < TPG; ++t) acc[t] = b;
-    const float* inb = in + g * TPG * in_ld;
-    for (int i = 0; i < NI; ++i) {
-      const float wv = __ldg(Wt + (size_t)i * NO + o);
+    for (int a = 0; a < 4; ++a)
 #pragma unroll
-      for (int t = 0; t < TPG; ++t) acc[t] = fmaf(inb[t * in_ld + i], wv, acc[t]);
+      for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+#pragma unroll 4
+    for (int i = i0; i < i1; ++i) {
+      const float4 wv = __ldg(reinterpret_cast<const float4*>(Wt + (size_t)i * NO + o4));
+      const float4 xv = *reinterpret_cast<const float4*>(in + i * TB + t4);
+      const float wa[4] = {wv.x, wv.y, wv.z, wv.w};
+      const float xb[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = fmaf(wa[a], xb[b], acc[a][b]);
     }
 #pragma unroll
-    for (int t = 0; t < TPG; ++t) out[(g * TPG + t) * out_ld + o] = silu_act ? siluf_(acc[t]) : acc[t];
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if (ks > 1) {
+          scratch[(kk * NO + o4 + a) * TB + t4 + b] = acc[a][b];
+        } else {
+          float v = acc[a][b] + (bias ? __ldg(bias + o4 + a) : 0.f);
+          out[oidx(o4 + a, t4 + b)] = silu_act ? siluf_(v) : v;
+        }
+      }
+  }
+  __syncthreads();
+  if (ks > 1) {
+    for (int e = threadIdx.x; e < NO * TB; e += NTHR) {
+      const int o = e / TB, t = e % TB;
+      float v = 0.f;
+      for (int kk = 0; kk < ks; ++kk) v += scratch[(kk * NO + o) * TB + t];
+      v += bias ? __ldg(bias + o) : 0.f;
+      out[oidx(o, t)] = silu_act ? siluf_(v) : v;
+    }
+    __syncthreads();
   }
 }
 
-__device__ __forceinline__ void bmm(const float* in, int in_ld, int NI, const float* Wt, int NO,
-                                    const float* bias, float* out, int out_ld, bool silu_act) {
-  if (NO >= 128)
-    bmm_tpg<16>(in, in_ld, NI, Wt, NO, bias, out, out_ld, silu_act);
-  else if (NO >= 32)
-    bmm_tpg<4>(in, in_ld, NI, Wt, NO, bias, out, out_ld, silu_act);
-  else
-    bmm_tpg<1>(in, in_ld, NI, Wt, NO, bias, out, out_ld, silu_act);
+// Sum the 16 per-thread partials of each token (thread t + 16 p holds partial p of
+// token t) in a fixed order; contains __syncthreads.
+__device__ __forceinline__ void reduce16(float* red, float v, float* out) {
+  red[threadIdx.x] = v;
+  __syncthreads();
+  if (threadIdx.x < TB) {
+    float s = 0.f;
+    for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + threadIdx.x];
+    out[threadIdx.x] = s;
+  }
+  __syncthreads();
 }
 
-// Shared-memory layout of k_router (floats).
-constexpr int LD_ENC = 256 + 1;   // encoder / psi hidden rows (<= 256 wide)
-constexpr int LD_S = 128 + 128 + 2;  // [s ; c ; nu] rows (d_s <= 128, d_m <= 128)
-constexpr int LD_QKV = 3 * 128 + 1;
-constexpr int LD_HID = 256 + 1;
-
 template <int DM>
-__global__ void __launch_bounds__(NTHR) k_router(const RouterArgs a) {
-  extern __shared__ float sm[];
-  float* enc = sm;                          // [TB][LD_ENC]  SiLU(W_hd RMSNorm(h_bar))
-  float* psi = enc + TB * LD_ENC;           // [TB][LD_ENC]  SiLU(f_psi first layer)
-  float* scn = psi + TB * LD_ENC;           // [TB][LD_S]    s | c | nu
-  float* qkv = scn + TB * LD_S;             // [TB][LD_QKV]  q | k | v
-  float* hid = qkv + TB * LD_QKV;           // [TB][LD_HID]  f_theta hidden / scratch
-  float* sc = hid + TB * LD_HID;            // [TB][16] per-token scalars
-  // sc: 0 rinv, 1 d_j, 2 gamma_j, 3 p_prev, 4 m_prev, 5 a, 6 b, 8.. path x (6)
-
+__global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
+  extern __shared__ __align__(16) float sm[];
   const int ds = a.d_h + a.d_a;
+  const RouterLayout lay(a.d_enc, a.d_head, ds, DM, a.d_path);
+  float* bigT = sm + lay.big;
+  float* sT = sm + lay.s;      // rows [0, d_s) s, [d_s, d_s + DM) c, d_s + DM nu
+  float* qkv = sm + lay.qkv;   // [TB][3 DM]
+  float* aux = sm + lay.aux;
+  float* xT = sm + lay.x;
+  float* phT = sm + lay.ph;
+  float* red = sm + lay.red;
+  float* sc = sm + lay.sc;     // per token: 0 rinv, 1 d_j, 4 m_prev
+  float* ab = sm + lay.ab;     // a[TB] | b[TB]
   const int t0 = blockIdx.x * TB;
   const int nY = a.d_enc + a.d_head;
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
+  const int nvalid = min(TB, a.T - t0);
 
-  // 1. per-token scalars from the partial sums of the previous block's epilogue
+  // 0. pull this CTA's memory block into L2 while the heads run (read in step 5)
+  if (tid == 0) {
+    const char* Sb = reinterpret_cast<const char*>(a.S + (size_t)t0 * DM * DM);
+    const uint32_t bytes = (uint32_t)(DM * DM * sizeof(float));
+    for (int i = 0; i < nvalid; ++i)
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(Sb + (size_t)i * bytes),
+                   "r"(bytes)
+                   : "memory");
+  }
+
+  // 1. per-token scalars from the partial sums of the previous block's epilogue;
+  //    transition features (Eqs. 7-8) and the path vector (Eqs. 4, 6)
   if (tid < TB) {
     const int t = t0 + tid;
     float ss = 0.f, dd = 0.f, dp = 0.f, dprev = 0.f, pp = 1.f, mp = 1.f;
@@ -137,57 +214,59 @@ __global__ void __launch_bounds__(NTHR) k_router(const RouterArgs a) {
     const float rinv = rsqrtf(ss / (float)a.d + a.rms_eps);
     const float dj = a.j == 1 ? 0.f : sqrtf(dd);                       // Eq. 7
     const float gam = a.j > 2 ? dp / (dj * dprev + a.eps) : 0.f;       // Eq. 8
-    float* s_ = sc + tid * 16;
-    s_[0] = rinv;
-    s_[1] = dj;
-    s_[2] = gam;
-    s_[3] = pp;
-    s_[4] = mp;
-    // path vector, Eq. 4 with Eq. 6
-    s_[8] = (float)a.j / (float)a.L;
-    s_[9] = (float)(a.L - a.j) / (float)a.L;
-    s_[10] = dj;
-    s_[11] = gam;
-    s_[12] = pp;
-    s_[13] = mp;
+    sc[tid * 16 + 0] = rinv;
+    sc[tid * 16 + 1] = dj;
+    sc[tid * 16 + 4] = mp;
+    xT[0 * TB + tid] = (float)a.j / (float)a.L;
+    xT[1 * TB + tid] = (float)(a.L - a.j) / (float)a.L;
+    xT[2 * TB + tid] = dj;
+    xT[3 * TB + tid] = gam;
+    xT[4 * TB + tid] = pp;
+    xT[5 * TB + tid] = mp;
   }
   __syncthreads();
 
-  // 2. encoder hidden SiLU(rinv * (W_hd diag(g_r)) h_bar) and f_psi hidden
-  for (int i = tid; i < TB * nY; i += NTHR) {
-    const int tl = i / nY, c = i % nY;
+  // 2. encoder hidden SiLU(rinv (W_hd diag(g_r)) h_bar), transposed; f_psi's
+  //    second layer reduced on the fly (b = w_ps2 . SiLU(W_ps1 h_bar + b_ps1), Eq. 16).
+  //    Thread tid always serves token tid % TB (the stride is a multiple of TB).
+  {
+    float bpart = 0.f;
+    const int tl = tid % TB;
     const int t = t0 + tl;
-    const float y = t < a.T ? a.Y[(size_t)t * nY + c] : 0.f;
-    if (c < a.d_enc)
-      enc[tl * LD_ENC + c] = siluf_(y * sc[tl * 16]);
-    else
-      psi[tl * LD_ENC + (c - a.d_enc)] = siluf_(y + a.w.ps_b1[c - a.d_enc]);
+    for (int i = tid; i < TB * nY; i += NTHR) {
+      const int c = i / TB;
+      const float y = t < a.T ? __ldg(a.Y + (size_t)t * nY + c) : 0.f;
+      if (c < a.d_enc) {
+        bigT[c * TB + tl] = siluf_(y * sc[tl * 16]);
+      } else {
+        const int e = c - a.d_enc;
+        bpart = fmaf(__ldg(a.w.ps_w2 + e), siluf_(y + __ldg(a.w.ps_b1 + e)), bpart);
+      }
+    }
+    reduce16(red, bpart, ab + TB);   // also orders step 2's writes before step 3
   }
-  __syncthreads();
 
-  // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h);  path encoder hidden -> hid
-  bmm(enc, LD_ENC, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, scn, LD_S, false);
-  bmm(sc + 8, 16, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, hid, LD_HID, true);
-  __syncthreads();
-  // z_a = W_a2 hid + b_a2 (Eq. 9) -> s[d_h, d_s)
-  bmm(hid, LD_HID, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, scn + a.d_h, LD_S, false);
-  __syncthreads();
+  // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s)
+  bmm4(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
+  bmm4(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
+  bmm4(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
 
-  // 4. q | k | v = W_{q,k,v} s (Eq. 10)
-  bmm(scn, LD_S, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, LD_QKV, false);
-  __syncthreads();
+  // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step
+  bmm4(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false);
 
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   //    Lane owns a 4-column group and every (32/LPR)-th row of S.
   {
     constexpr int LPR = DM / 4;          // lanes per S row
     constexpr int RPI = 32 / LPR;        // rows per iteration
+    constexpr int NIT = DM / RPI;        // S rows handled by this lane
+    constexpr int BATCH = NIT < 8 ? NIT : 8;  // loads kept in flight
     const int cq = lane % LPR;
     const int r0 = lane / LPR;
     for (int tl = warp; tl < TB; tl += NTHR / 32) {
       const int t = t0 + tl;
       if (t >= a.T) continue;
-      const float* q = qkv + tl * LD_QKV;
+      const float* q = qkv + tl * 3 * DM;
       const float* k = q + DM;
       const float* v = q + 2 * DM;
       float* S = a.S + (size_t)t * DM * DM;
@@ -200,16 +279,23 @@ __global__ void __launch_bounds__(NTHR) k_router(const RouterArgs a) {
       }
       den = warp_sum(den);
       float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
-      const float4 vv = make_float4(v[4 * cq], v[4 * cq + 1], v[4 * cq + 2], v[4 * cq + 3]);
-#pragma unroll 4
-      for (int r = r0; r < DM; r += RPI) {
-        float4* p = reinterpret_cast<float4*>(S + r * DM + 4 * cq);
-        const float4 so = *p;
-        const float fq = phif_(q[r]);
-        const float fk = phif_(k[r]);
-        c.x += fq * so.x; c.y += fq * so.y; c.z += fq * so.z; c.w += fq * so.w;
-        *p = make_float4(a.rho * so.x + fk * vv.x, a.rho * so.y + fk * vv.y,
-                         a.rho * so.z + fk * vv.z, a.rho * so.w + fk * vv.w);
+      const float4 vv = *reinterpret_cast<const float4*>(v + 4 * cq);
+#pragma unroll 1
+      for (int i0 = 0; i0 < NIT; i0 += BATCH) {
+        float4 so[BATCH];
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i)
+          so[i] = *reinterpret_cast<const float4*>(S + (r0 + (i0 + i) * RPI) * DM + 4 * cq);
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i) {
+          const int r = r0 + (i0 + i) * RPI;
+          const float fq = phif_(q[r]);
+          const float fk = phif_(k[r]);
+          c.x += fq * so[i].x; c.y += fq * so[i].y; c.z += fq * so[i].z; c.w += fq * so[i].w;
+          *reinterpret_cast<float4*>(S + r * DM + 4 * cq) =
+              make_float4(a.rho * so[i].x + fk * vv.x, a.rho * so[i].y + fk * vv.y,
+                          a.rho * so[i].z + fk * vv.z, a.rho * so[i].w + fk * vv.w);
+        }
       }
 #pragma unroll
       for (int o = LPR; o < 32; o <<= 1) {
@@ -220,69 +306,91 @@ __global__ void __launch_bounds__(NTHR) k_router(const RouterArgs a) {
       }
       if (r0 == 0) {
         const float inv = 1.0f / (den + a.eps);
-        float* cdst = scn + tl * LD_S + ds + 4 * cq;
-        cdst[0] = c.x * inv;
-        cdst[1] = c.y * inv;
-        cdst[2] = c.z * inv;
-        cdst[3] = c.w * inv;
+        float* cdst = sT + (ds + 4 * cq) * TB + tl;
+        cdst[0 * TB] = c.x * inv;
+        cdst[1 * TB] = c.y * inv;
+        cdst[2 * TB] = c.z * inv;
+        cdst[3 * TB] = c.w * inv;
       }
     }
   }
   __syncthreads();
 
   // 6. nu = 1 - cos(W_n s, W_c c) for j > 1 (Eq. 13); nu_1 = 0
+  float* nuT = sT + (ds + DM) * TB;
   if (a.j > 1) {
-    float* nv = hid;                 // [TB][LD_HID]: cols [0, DM) W_n s, [128, 128+DM) W_c c
-    bmm(scn, LD_S, ds, a.w.w_n_t, DM, nullptr, nv, LD_HID, false);
-    bmm(scn + ds, LD_S, DM, a.w.w_c_t, DM, nullptr, nv + 128, LD_HID, false);
+    const int cap = (a.d_enc > a.d_head ? a.d_enc : a.d_head) * TB;
+    float* nv = aux;               // [DM][TB]
+    float* cv = aux + DM * TB;     // [DM][TB]
+    bmm4(sT, ds, a.w.w_n_t, DM, nullptr, nv, 0, false, bigT, cap);
+    bmm4(sT + ds * TB, DM, a.w.w_c_t, DM, nullptr, cv, 0, false, bigT, cap);
+    // thread (part, t) sums DM/16 products; fixed-order reduction per token
+    const int tl = tid % TB, part = tid / TB;
+    float xy = 0.f, xx = 0.f, yy = 0.f;
+    for (int i = part; i < DM; i += NTHR / TB) {
+      const float u = nv[i * TB + tl], w = cv[i * TB + tl];
+      xy += u * w;
+      xx += u * u;
+      yy += w * w;
+    }
+    float* r3 = sc;  // reuse columns 8..10 of the scalar rows for the three sums
+    red[tid] = xy;
     __syncthreads();
-    for (int tl = warp; tl < TB; tl += NTHR / 32) {
-      const float* x = nv + tl * LD_HID;
-      float xy = 0.f, xx = 0.f, yy = 0.f;
-      for (int i = lane; i < DM; i += 32) {
-        const float u = x[i], w = x[128 + i];
-        xy += u * w;
-        xx += u * u;
-        yy += w * w;
-      }
-      xy = warp_sum(xy);
-      xx = warp_sum(xx);
-      yy = warp_sum(yy);
-      if (lane == 0) scn[tl * LD_S + ds + DM] = 1.f - xy / (sqrtf(xx) * sqrtf(yy) + a.eps);
+    if (tid < TB) {
+      float s = 0.f;
+      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
+      r3[tid * 16 + 8] = s;
+    }
+    __syncthreads();
+    red[tid] = xx;
+    __syncthreads();
+    if (tid < TB) {
+      float s = 0.f;
+      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
+      r3[tid * 16 + 9] = s;
+    }
+    __syncthreads();
+    red[tid] = yy;
+    __syncthreads();
+    if (tid < TB) {
+      float s = 0.f;
+      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
+      const float sxy = r3[tid * 16 + 8], sxx = r3[tid * 16 + 9];
+      nuT[tid] = 1.f - sxy / (sqrtf(sxx) * sqrtf(s) + a.eps);
     }
   } else {
-    if (tid < TB) scn[tid * LD_S + ds + DM] = 0.f;
+    if (tid < TB) nuT[tid] = 0.f;
   }
   __syncthreads();
 
-  // 7. f_theta hidden = SiLU(W_th1 [s; c; nu] + b)
-  bmm(scn, LD_S, ds + DM + 1, a.w.th_w1_t, a.d_head, a.w.th_b1, hid, LD_HID, true);
-  __syncthreads();
+  // 7. f_theta hidden = SiLU(W_th1 [s; c; nu] + b) -> big region
+  bmm4(sT, ds + DM + 1, a.w.th_w1_t, a.d_head, a.w.th_b1, bigT, 0, true);
 
-  // 8. a = w_th2 . hidden + b (Eq. 14), b = w_ps2 . psi + b (Eq. 16); gate and decision
-  for (int tl = warp; tl < TB; tl += NTHR / 32) {
-    float sa = 0.f, sb = 0.f;
-    for (int i = lane; i < a.d_head; i += 32) {
-      sa += a.w.th_w2[i] * hid[tl * LD_HID + i];
-      sb += a.w.ps_w2[i] * psi[tl * LD_ENC + i];
-    }
-    sa = warp_sum(sa);
-    sb = warp_sum(sb);
-    const int t = t0 + tl;
-    if (lane == 0 && t < a.T) {
-      const float av = sa + a.w.th_b2[0];
-      const float bv = sb + a.w.ps_b2[0];
-      const float p = sigmoidf_(av / a.t_hist);      // Eq. 14
-      const float m = sc[tl * 16 + 4] * p;          // Eq. 15
-      const float g = sigmoidf_(av + bv);            // Eq. 16
+  // 8. a = w_th2 . hidden + b (Eq. 14)
+  {
+    const int tl = tid % TB, part = tid / TB;
+    float sa = 0.f;
+    for (int i = part; i < a.d_head; i += NTHR / TB) sa = fmaf(__ldg(a.w.th_w2 + i), bigT[i * TB + tl], sa);
+    reduce16(red, sa, ab);
+  }
+
+  // 9. history score, cumulative score, gate and decision
+  if (tid < TB) {
+    const int t = t0 + tid;
+    if (t < a.T) {
+      const float av = ab[tid] + __ldg(a.w.th_b2);
+      const float bv = ab[TB + tid] + __ldg(a.w.ps_b2);
+      const float p = sigmoidf_(av / a.t_hist);     // Eq. 14
+      const float m = sc[tid * 16 + 4] * p;         // Eq. 15
+      const float g = sigmoidf_(av + bv);           // Eq. 16
       uint8_t dec;
       if (a.mask_in)
         dec = a.mask_in[t] ? 1 : 0;
       else
-        dec = g >= a.tau ? 1 : 0;                    // Eq. 3 (ties run the FFN)
+        dec = g >= a.tau ? 1 : 0;                   // Eq. 3 (ties run the FFN)
       a.pst[t] = p;
       a.mst[t] = m;
-      a.dprev[t] = sc[tl * 16 + 1];
+      a.dprev[t] = sc[tid * 16 + 1];
       a.gate[t] = g;
       a.mask[t] = dec;
       if (a.gate_out) a.gate_out[t] = g;
@@ -291,13 +399,10 @@ __global__ void __launch_bounds__(NTHR) k_router(const RouterArgs a) {
   }
 }
 
-constexpr size_t kRouterSmem =
-    sizeof(float) * (size_t)TB * (2 * LD_ENC + LD_S + LD_QKV + LD_HID + 16);
-
 // ------------------------------------------------------------------------------
-// k_compact: one CTA; stable exclusive scan of the decisions, chunks of 8192.
+// k_compact: one CTA; stable exclusive scan of the decisions, chunks of 16384.
 // ------------------------------------------------------------------------------
-constexpr int CT = 1024, CPT = 8;
+constexpr int CT = 1024, CPT = 16;
 
 __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
   __shared__ int wsum[CT / 32];
@@ -308,12 +413,21 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
   for (int base = 0; base < a.T; base += CT * CPT) {
     uint8_t f[CPT];
     int cnt = 0;
+    const int tb = base + tid * CPT;
+    if (!a.dense && tb + CPT <= a.T) {   // 16 flags in one 16-byte load (tb is 16-aligned)
+      const uint4 u = *reinterpret_cast<const uint4*>(a.mask + tb);
+      const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
-      const int t = base + tid * CPT + i;
-      f[i] = (t < a.T) ? (a.dense ? 1 : (a.mask[t] ? 1 : 0)) : 2;
-      cnt += f[i] == 1;
+      for (int i = 0; i < CPT; ++i) f[i] = ((w4[i >> 2] >> (8 * (i & 3))) & 0xffu) ? 1 : 0;
+    } else {
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) {
+        const int t = tb + i;
+        f[i] = (t < a.T) ? (a.dense ? 1 : (a.mask[t] ? 1 : 0)) : 2;
+      }
     }
+#pragma unroll
+    for (int i = 0; i < CPT; ++i) cnt += f[i] == 1;
     // inclusive warp scan of the per-thread counts
     int x = cnt;
 #pragma unroll
@@ -335,7 +449,7 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
     __syncthreads();
     const int carry = carry_s;
     int pos_f = carry + (warp ? wsum[warp - 1] : 0) + x - cnt;  // exclusive
-    int t = base + tid * CPT;
+    int t = tb;
     int pos_a = t - pos_f;  // tokens before t that went to the adapter
 #pragma unroll
     for (int i = 0; i < CPT; ++i, ++t) {
@@ -438,14 +552,16 @@ cudaError_t launch_init(const InitArgs& a, cudaStream_t st) {
 
 template <int DM>
 static cudaError_t launch_router_dm(const RouterArgs& a, cudaStream_t st) {
-  static bool attr = false;
-  if (!attr) {
+  const RouterLayout lay(a.d_enc, a.d_head, a.d_h + a.d_a, DM, a.d_path);
+  const size_t smem = sizeof(float) * (size_t)lay.floats;
+  static size_t attr = 0;
+  if (smem > attr) {
     cudaError_t e = cudaFuncSetAttribute(k_router<DM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kRouterSmem);
+                                         (int)smem);
     if (e != cudaSuccess) return e;
-    attr = true;
+    attr = smem;
   }
-  k_router<DM><<<(a.T + TB - 1) / TB, NTHR, kRouterSmem, st>>>(a);
+  k_router<DM><<<(a.T + TB - 1) / TB, NTHR, smem, st>>>(a);
   return cudaGetLastError();
 }
 
