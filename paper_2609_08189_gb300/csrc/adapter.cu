@@ -1,0 +1,153 @@
+// Adapter up-projection fused with the block-closing epilogue (Eqs. 2-3 for the
+// tokens routed to the adapter):
+//   y = W_2 SiLU(W_1 u)   (the SiLU(W_1 u) rows come from the adapter-down GEMM)
+//   h = h_bar + (1 - g) y, then the next block's h_bar, delta and partial sums.
+// The contraction has depth d_r (64), i.e. 2 d_r FLOP per output element against
+// 20 bytes of epilogue traffic, so this runs on the FMA pipes with many warps per
+// SM and row-contiguous global access rather than as a tensor-core GEMM.
+//
+// CTA: 32 adapter rows x 256 output columns, 256 threads.  Warp w owns rows
+// 4w..4w+3; lane x owns columns x + 32 j (j < 8), so every warp instruction of
+// the epilogue touches 128 contiguous bytes of one row.  The rows the epilogue
+// will update are bulk-prefetched into L2 at kernel start.
+#include "hero_device.cuh"
+
+namespace hero {
+namespace {
+
+constexpr int AU_ROWS = 32;
+constexpr int AU_COLS = 256;
+constexpr int AU_DR = 64;          // largest supported rank
+constexpr int AU_WLD = AU_DR + 2;  // row stride of the staged W_2 slice (conflict-free reads)
+
+template <typename WT>
+constexpr size_t au_smem() {
+  return sizeof(float) * AU_ROWS * AU_DR + sizeof(WT) * AU_COLS * AU_WLD;
+}
+
+__device__ __forceinline__ float to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
+__device__ __forceinline__ float to_f32(float v) { return v; }
+
+// WT: operand element type, uint16_t (bf16 bits) or float.  SLOT: columns per
+// partial-sum slot of the model (64 or 256).
+template <int SLOT, typename WT>
+__global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
+  extern __shared__ __align__(16) float smem_au[];
+  float* ahs = smem_au;                                         // [AU_ROWS][AU_DR] fp32
+  WT* w2s = reinterpret_cast<WT*>(smem_au + AU_ROWS * AU_DR);   // [AU_COLS][AU_WLD]
+  int M = *a.m_dev;
+  if (M < 0 || M > a.m_max) M = 0;
+  const int m0 = blockIdx.y * AU_ROWS;
+  if (m0 >= M) return;
+  const int n0 = blockIdx.x * AU_COLS;
+  const int dr = a.d_r;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const LayerOutArgs& p = a.lo;
+  const WT* ah = static_cast<const WT*>(a.ah);
+  const WT* w2 = static_cast<const WT*>(a.w2);
+
+  // Start pulling the epilogue's rows (h_bar, delta, P_{j+1} over this CTA's
+  // columns) into L2 while the contraction runs.
+  if (tid < AU_ROWS && m0 + tid < M) {
+    const int t = p.idx[m0 + tid];
+    const int cols = min(AU_COLS, a.d - n0);
+    const size_t off = (size_t)t * p.d + n0;
+    prefetch_l2(p.hbar + off, cols * 4);
+    if (!p.last) {
+      if (p.router && !p.first) prefetch_l2(p.delta + off, cols * 4);
+      const int pes = p.p_bf16 ? 2 : 4;
+      if (p.p_next) prefetch_l2(static_cast<const char*>(p.p_next) + off * pes, cols * pes);
+    }
+  }
+
+  for (int e = tid; e < AU_ROWS * dr; e += 256) {
+    const int r = e / dr, k = e % dr;
+    const int m = m0 + r;
+    ahs[r * AU_DR + k] = m < M ? to_f32(ah[(size_t)m * dr + k]) : 0.f;
+  }
+  for (int e = tid; e < AU_COLS * dr; e += 256) {
+    const int c = e / dr, k = e % dr;
+    const int n = n0 + c;
+    w2s[c * AU_WLD + k] = n < a.d ? w2[(size_t)n * dr + k] : WT(0);
+  }
+  __syncthreads();
+
+  float acc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  const float* arow = ahs + (warp * 4) * AU_DR;
+  for (int k = 0; k < dr; ++k) {
+    float x[4], w[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = arow[i * AU_DR + k];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = to_f32(w2s[(lane + 32 * j) * AU_WLD + k]);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(x[i], w[j], acc[i][j]);
+  }
+
+  constexpr int spt = AU_COLS / SLOT;   // partial slots per tile: 1 or 4
+#pragma unroll 1
+  for (int i = 0; i < 4; ++i) {
+    const int m = m0 + warp * 4 + i;
+    if (m >= M) break;                     // warp-uniform
+    const int t = p.idx[m];
+    const float s = p.scale[m];
+    LayerOutIn1 in[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int n = n0 + lane + 32 * j;
+      if (n < a.d) in[j] = layer_out_load1(p, t, n);
+    }
+    float ss[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f}, dp[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int n = n0 + lane + 32 * j;
+      const int sl = (32 * j) / SLOT;
+      if (n < a.d) layer_out_store1(p, t, n, in[j], acc[i][j], s, ss[sl], dd[sl], dp[sl]);
+    }
+    if (!p.last) {
+#pragma unroll
+      for (int sl = 0; sl < spt; ++sl) {
+        const float v0 = warp_sum(ss[sl]), v1 = warp_sum(dd[sl]), v2 = warp_sum(dp[sl]);
+        const int slot = n0 / SLOT + sl;
+        if (lane == 0 && slot * SLOT < a.d)
+          *reinterpret_cast<float4*>(p.part + ((size_t)t * p.np + slot) * 4) =
+              make_float4(v0, v1, v2, 0.f);
+      }
+    }
+  }
+}
+
+template <int SLOT, typename WT>
+cudaError_t launch_au(const AdapterUpArgs& a, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_adapter_up<SLOT, WT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)au_smem<WT>());
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((a.d + AU_COLS - 1) / AU_COLS, (a.m_max + AU_ROWS - 1) / AU_ROWS);
+  k_adapter_up<SLOT, WT><<<grid, 256, au_smem<WT>(), st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st) {
+  if (a.m_max <= 0) return cudaSuccess;
+  if (a.d_r > AU_DR) return cudaErrorInvalidValue;
+  if (a.bf16 && a.slot_cols == 256) return launch_au<256, uint16_t>(a, st);
+  if (!a.bf16 && a.slot_cols == 64) return launch_au<64, float>(a, st);
+  if (a.bf16 && a.slot_cols == 64) return launch_au<64, uint16_t>(a, st);
+  if (!a.bf16 && a.slot_cols == 256) return launch_au<256, float>(a, st);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace hero

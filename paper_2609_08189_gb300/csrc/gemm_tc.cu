@@ -338,6 +338,20 @@ __global__ void __launch_bounds__(192, 1)
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       int mb, nb;
       tile_coords(tile, m_tiles, n_tiles, mb, nb);
+      if constexpr (EPI == EPI_LAYER_OUT) {
+        // pull this row's h_bar / delta / P_{j+1} segment into L2 while the tile accumulates
+        const LayerOutArgs& p = args.lo;
+        const int mr = mb * BM + row;
+        if (mr < M) {
+          const size_t off = (size_t)p.idx[mr] * p.d + (size_t)nb * BN;
+          prefetch_l2(p.hbar + off, BN * 4);
+          if (!p.last) {
+            if (p.router && !p.first) prefetch_l2(p.delta + off, BN * 4);
+            const int pes = p.p_bf16 ? 2 : 4;
+            if (p.p_next) prefetch_l2(static_cast<const char*>(p.p_next) + off * pes, BN * pes);
+          }
+        }
+      }
       bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);

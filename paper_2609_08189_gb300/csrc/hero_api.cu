@@ -181,6 +181,7 @@ hero_status validate_config(const hero_config* c) {
   if (c->d_h % 4 || c->d_a % 4 || c->d_enc % 4 || c->d_head % 4 || c->d_path % 4)
     return fail(HERO_ERR_UNSUPPORTED, "router widths d_h, d_a, d_enc, d_head, d_path must be multiples of 4");
   if (c->d_model % 8 != 0) return fail(HERO_ERR_UNSUPPORTED, "d_model must be a multiple of 8");
+  if (c->d_r > 64) return fail(HERO_ERR_UNSUPPORTED, "d_r must be at most 64");
   if (c->dtype == HERO_BF16) {
     if (c->d_model % 256 != 0 || c->d_ff % 128 != 0 || c->d_r != 64)
       return fail(HERO_ERR_UNSUPPORTED,
@@ -235,6 +236,8 @@ void free_model(hero_model* m) {
 // ============================================================================
 
 extern "C" const char* hero_last_error(void) { return g_last_error.c_str(); }
+
+void hero::set_last_error(const char* msg) { g_last_error = msg; }
 
 extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weights_host* w,
                                          hero_model** out) {
@@ -655,23 +658,19 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
         return m->bf16 ? launch_gemm_tc(64, EPI_SILU, m->tm_ua, m->tm_w1[jj], g, m->num_sms, st)
                        : launch_gemm_simt(EPI_SILU, g, st);
       }));
-      GemmArgs g2{};
-      g2.m_dev = m->counts + 1;
-      g2.m_max = T;
-      g2.N = d;
-      g2.K = r;
-      g2.err = m->err;
-      g2.lo = lo;
-      g2.lo.idx = m->idx_a;
-      g2.lo.scale = m->scale_a;
-      g2.A = m->ah;
-      g2.lda = r;
-      g2.B = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
-      g2.ldb = r;
-      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
-        return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_ah, m->tm_w2[jj], g2, m->num_sms, st)
-                       : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
-      }));
+      AdapterUpArgs au{};
+      au.m_dev = m->counts + 1;
+      au.m_max = T;
+      au.d = d;
+      au.d_r = r;
+      au.ah = m->ah;
+      au.w2 = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
+      au.bf16 = m->bf16;
+      au.slot_cols = m->bf16 ? 256 : kSimtTileN;
+      au.lo = lo;
+      au.lo.idx = m->idx_a;
+      au.lo.scale = m->scale_a;
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] { return launch_adapter_up(au, st); }));
     }
   }
   return HERO_OK;

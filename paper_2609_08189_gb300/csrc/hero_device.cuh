@@ -133,6 +133,50 @@ __device__ __forceinline__ void layer_out_store(const LayerOutArgs& p, int t, in
   }
 }
 
+// Scalar form (one column n of token t).
+struct LayerOutIn1 {
+  float hb, pn, dprev;
+};
+
+__device__ __forceinline__ LayerOutIn1 layer_out_load1(const LayerOutArgs& p, int t, int n) {
+  const size_t off = (size_t)t * p.d + n;
+  LayerOutIn1 in;
+  in.hb = p.hbar[off];
+  in.pn = 0.f;
+  in.dprev = 0.f;
+  if (!p.last) {
+    if (p.p_next)
+      in.pn = p.p_bf16 ? __uint_as_float((uint32_t)static_cast<const uint16_t*>(p.p_next)[off] << 16)
+                       : static_cast<const float*>(p.p_next)[off];
+    if (p.router && !p.first) in.dprev = p.delta[off];
+  }
+  return in;
+}
+
+__device__ __forceinline__ void layer_out_store1(const LayerOutArgs& p, int t, int n,
+                                                 const LayerOutIn1& in, float y, float s,
+                                                 float& ss, float& dd, float& dp) {
+  const size_t off = (size_t)t * p.d + n;
+  const float h = in.hb + s * y;
+  if (p.last) {
+    p.h_out[off] = h;
+    return;
+  }
+  const float hn = h + in.pn;
+  p.hbar[off] = hn;
+  ss += hn * hn;
+  if (p.router) {
+    const float dn = s * y + in.pn;
+    p.delta[off] = dn;
+    if (p.xl_bf16)
+      static_cast<__nv_bfloat16*>(p.xl)[off] = __float2bfloat16_rn(hn);
+    else
+      static_cast<float*>(p.xl)[off] = hn;
+    dd += dn * dn;
+    dp += dn * in.dprev;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // PTX wrappers (sm_100 family: mbarrier, TMA, tcgen05)
 // ---------------------------------------------------------------------------
@@ -193,6 +237,11 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm,
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
       : "memory");
+}
+
+// Bulk prefetch of [p, p + bytes) into L2 (p 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void prefetch_l2(const void* p, int bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {

@@ -17,6 +17,9 @@ enum : uint32_t {
   ERR_BAD_INDEX = 16u,
 };
 
+// Record the message hero_last_error() returns on this host thread.
+void set_last_error(const char* msg);
+
 // Bound on every device-side wait (nanoseconds of %globaltimer).
 constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
@@ -177,6 +180,22 @@ struct NormArgs {
   int out_bf16;
 };
 cudaError_t launch_norm(const NormArgs& a, cudaStream_t st);
+
+// Adapter up-projection plus the block-closing epilogue, for the adapter rows:
+// y[m, :] = W_2 ah[m, :] (rank d_r = 64 contraction), then LayerOutArgs on token
+// idx[m] with scale[m] = 1 - g.  SIMT: the contraction is 2 d_r FLOP per output
+// element, so the kernel is bound by the epilogue's HBM traffic.
+struct AdapterUpArgs {
+  const int* m_dev;     // number of adapter rows (device)
+  int m_max;
+  int d, d_r;
+  const void* ah;       // [rows, d_r] SiLU(W_1 u), bf16 or fp32
+  const void* w2;       // [d, d_r] bf16 or fp32
+  int bf16;
+  int slot_cols;        // columns per partial-sum slot (64 or 256)
+  LayerOutArgs lo;
+};
+cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st);
 
 // Weight conversion: dst[map(r)] = convert(src[r]) for rows of `cols` elements.
 // map(r) = (r / grp) * grp_stride + (r % grp) + offset.
