@@ -143,6 +143,39 @@ hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, const float* 
                                   uint8_t* mask_out, int32_t* ffn_count_out,
                                   void* cuda_stream);
 
+/* ---- one routed block at a time ----------------------------------------------
+ * Per-token router state carried from one routed block to the next within a
+ * forward pass (Sec. 3.2).  DEVICE pointers, caller-owned, T tokens.  Lets the
+ * caller run its own attention sublayer between routed blocks (Eq. 1) instead of
+ * the additive stand-in of hero_routed_ffn_stack. */
+typedef struct {
+  float* S;           /* [T, d_m, d_m] memory matrix S (Eqs. 11-12), key index first */
+  float* zeta;        /* [T, d_m] normaliser zeta (Eqs. 11-12)                          */
+  float* p_hist;      /* [T] history score of the previous block (Eqs. 4, 14)           */
+  float* m_hist;      /* [T] cumulative history score (Eqs. 4, 15)                      */
+  float* d_prev;      /* [T] ||delta|| of the previous block (Eqs. 7-8)                 */
+  float* h_bar_prev;  /* [T, d] h_bar of the previous routed block (Eq. 7)              */
+  float* delta_prev;  /* [T, d] delta of the previous routed block (Eq. 8)              */
+} hero_router_state;
+
+/* Start of a forward pass: S = 0, zeta = 0, p_hist = m_hist = 1, d_prev = 0
+ * (Sec. 3.2; Eq. 4 initial scores).  h_bar_prev / delta_prev need no reset: block
+ * 1 does not read them. */
+hero_status hero_router_state_reset(hero_model* m, int64_t n_tokens, const hero_router_state* state,
+                                    void* cuda_stream);
+
+/* Routed block `block` (j = 1..n_layers) on post-attention hidden states
+ * h_bar [T,d] fp32 (Eq. 1).  Reads then updates `state` (read before write,
+ * Eqs. 11-12) and writes h_out [T,d] = h_bar + g FFN(u) or h_bar + (1-g)
+ * Adapter(u) (Eq. 3).  flags: HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK (mask_in [T]).
+ * gate_out [T], mask_out [T], ffn_count_out [1] may be NULL.  h_out must not
+ * alias h_bar.  Same error and stream conventions as hero_routed_ffn_stack;
+ * host pointers are not accepted here. */
+hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n_tokens, const float* h_bar,
+                              const hero_router_state* state, float tau_exec, uint32_t flags,
+                              const uint8_t* mask_in, float* h_out, float* gate_out,
+                              uint8_t* mask_out, int32_t* ffn_count_out, void* cuda_stream);
+
 /* Release every resource of the model (NULL-safe).  Synchronizes the device. */
 void hero_free(hero_model* m);
 

@@ -38,10 +38,14 @@ Readings where the paper is silent (each listed in the design notes):
   * decisions: g >= tau_exec -> FFN (ties go to the FFN).
   * precision contract for bf16 workloads: values are rounded to bf16 (nearest,
     ties to even) exactly at (i) every parameter (done by the input generator),
-    (ii) the operands of the router's d-wide contraction: bf16(h_bar) and
+    (ii) the operands of the router's d-wide contraction: the weight
     bf16(W_hd diag(gain_r)) for the encoder (the row scale 1/rms is applied after
-    the contraction, exact in real arithmetic), bf16(h_bar) for f_psi's first
-    layer, (iii) u = LN_ffn(h_bar), the FFN and adapter input, (iv) the SwiGLU
+    the contraction, exact in real arithmetic) and f_psi's first-layer weight;
+    the activation h_bar enters both as a pair of bf16 numbers,
+    hi = bf16(h_bar), lo = bf16(h_bar - hi) (16 significant bits), because a
+    single bf16 rounding of the router input makes the gates of a deep stack
+    drift by ~1e-3 under perturbations of 1e-7 (rounding flips cascade through
+    depth), (iii) u = LN_ffn(h_bar), the FFN and adapter input, (iv) the SwiGLU
     product entering W_down, (v) the adapter hidden SiLU(W_1 u) entering W_2.
     Everything else is float64 here.  f32 workloads round nowhere.
 
@@ -79,6 +83,12 @@ def bf16_round(x: np.ndarray) -> np.ndarray:
 
 def _identity(x: np.ndarray) -> np.ndarray:
     return x
+
+
+def bf16_pair(x: np.ndarray) -> np.ndarray:
+    """x carried as two bf16 numbers, hi = bf16(x) and lo = bf16(x - hi): 16 significant bits."""
+    hi = bf16_round(x)
+    return hi + bf16_round(x - hi)
 
 
 def sigmoid(x: np.ndarray) -> np.ndarray:
@@ -171,16 +181,16 @@ def path_vector(j: int, L: int, d, gamma, p_prev, m_prev):
     return np.stack([r, q_rem, d, gamma, p_prev, m_prev], axis=1)
 
 
-def hidden_encoder(h_bar, w, cfg: OracleConfig, R):
+def hidden_encoder(h_bar, w, cfg: OracleConfig, R, Rx):
     """Eq. 5: z_h = W_hu SiLU(W_hd RMSNorm(h_bar)).
 
     RMSNorm(h) = (h * gain_r) / rms(h); the contraction is written as
-    (1/rms) * (W_hd diag(gain_r)) h so that the bf16 operand rounding of the
-    precision contract applies to bf16(h_bar) and bf16(W_hd diag(gain_r)).
+    (1/rms) * (W_hd diag(gain_r)) h so that the precision contract applies to
+    the operands Rx(h_bar) and R(W_hd diag(gain_r)).
     """
     rinv = 1.0 / np.sqrt(np.mean(h_bar * h_bar, axis=1) + cfg.rms_eps)
     w_enc = R(w["w_hd"] * w["r_norm_g"][None, :])
-    pre = rinv[:, None] * (R(h_bar) @ w_enc.T)
+    pre = rinv[:, None] * (Rx(h_bar) @ w_enc.T)
     return silu(pre) @ w["w_hu"].T
 
 
@@ -219,9 +229,9 @@ def history_head(s, c, nu, w):
     return _mlp2(x, w["th_w1"], w["th_b1"], w["th_w2"], w["th_b2"])[:, 0]
 
 
-def local_head(h_bar, w, R):
-    """Eq. 16, first part: b = f_psi(h_bar); its first layer reads bf16(h_bar) in bf16."""
-    return _mlp2(R(h_bar), w["ps_w1"], w["ps_b1"], w["ps_w2"], w["ps_b2"])[:, 0]
+def local_head(h_bar, w, Rx):
+    """Eq. 16, first part: b = f_psi(h_bar); its first layer reads the operand Rx(h_bar)."""
+    return _mlp2(Rx(h_bar), w["ps_w1"], w["ps_b1"], w["ps_w2"], w["ps_b2"])[:, 0]
 
 
 def swiglu_ffn(u, wl, R):
@@ -262,6 +272,7 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     if mode == "force" and mask_in is None:
         raise ValueError("force mode needs mask_in")
     R = bf16_round if cfg.dtype == "bf16" else _identity
+    Rx = bf16_pair if cfg.dtype == "bf16" else _identity   # router activation operand
     hk = hooks or {}
     L = cfg.n_layers
     h = _f64(h_in)
@@ -293,7 +304,7 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             delta, d, gamma = transition_features(j, h_bar, h_bar_prev, delta_prev,
                                                   d_prev, cfg.eps)
             x_path = path_vector(j, L, d, gamma, p_prev, m_prev)
-            z_h = hidden_encoder(h_bar, w, cfg, R)
+            z_h = hidden_encoder(h_bar, w, cfg, R, Rx)
             z_a = path_encoder(x_path, w)
             s = np.concatenate([z_h, z_a], axis=1)                 # Eq. 9
             q = s @ w["w_q"].T                                      # Eq. 10
@@ -306,7 +317,7 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             a = history_head(s, c, nu, w)                           # Eq. 14
             p = sigmoid(a / cfg.t_hist)
             m = m_prev * p                                          # Eq. 15
-            b = local_head(h_bar, w, R)                             # Eq. 16
+            b = local_head(h_bar, w, Rx)                            # Eq. 16
             g = sigmoid(a + b)
             rho = sigmoid(eta[j - 1])
             S, zeta = memory_write(S, zeta, fk, v, rho)             # Eq. 12

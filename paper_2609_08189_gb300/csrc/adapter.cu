@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
       for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(x[i], w[j], acc[i][j]);
   }
 
-  constexpr int spt = AU_COLS / SLOT;   // partial slots per tile: 1 or 4
+  constexpr int spt = AU_COLS / SLOT;   // partial slots per tile
 #pragma unroll 1
   for (int i = 0; i < 4; ++i) {
     const int m = m0 + warp * 4 + i;
@@ -145,8 +145,6 @@ cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st) {
   if (a.d_r > AU_DR) return cudaErrorInvalidValue;
   if (a.bf16 && a.slot_cols == 256) return launch_au<256, uint16_t>(a, st);
   if (!a.bf16 && a.slot_cols == 64) return launch_au<64, float>(a, st);
-  if (a.bf16 && a.slot_cols == 64) return launch_au<64, uint16_t>(a, st);
-  if (!a.bf16 && a.slot_cols == 256) return launch_au<256, float>(a, st);
   return cudaErrorInvalidValue;
 }
 

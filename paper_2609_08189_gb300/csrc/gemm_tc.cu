@@ -21,7 +21,7 @@ constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int kGroupM = 16;   // raster: 16 M-tiles share each wave of N-tiles (L2 reuse)
 
-template <int BN>
+template <int BN, int EPI>
 struct TcCfg {
   static constexpr int STAGES = BN == 256 ? 4 : 6;
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -32,9 +32,14 @@ struct TcCfg {
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                     ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-  // ring | barriers (256 B) | per-epilogue-warp staging tiles (4 x 32 x 32 fp32)
+  // One epilogue warp per TMEM lane quadrant.  (Two per quadrant, each taking half
+  // of the columns, measured within 1% for the block-closing epilogue.)
+  static constexpr int EPI_WARPS = 4;
+  static constexpr int THREADS = 64 + 32 * EPI_WARPS;
+  static constexpr int EPI_COLS = BN / (EPI_WARPS / 4);
+  // ring | barriers (256 B) | per-epilogue-warp staging tiles (32 x 32 fp32 each)
   static constexpr uint32_t EPI_STAGE_OFF = STAGES * STAGE_BYTES + 256;
-  static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + 4 * 32 * 32 * 4 + 1024;
+  static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + EPI_WARPS * 32 * 32 * 4 + 1024;
 };
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
@@ -133,12 +138,15 @@ __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int 
   }
 }
 
-// Block-closing epilogue, row-contiguous through the staging tile.  Each lane
-// keeps the partial sums of its 8 rows and reduces them over the 8 lanes that
-// share a row at the end of the tile.
-template <int BN>
+// Block-closing epilogue over columns [c_begin, c_begin + NCOLS) of the tile,
+// row-contiguous through the staging tile.  Each lane keeps the partial sums of
+// its 8 rows and reduces them over the 8 lanes that share a row at the end; the
+// partial-sum slot covers kPartCols columns.
+constexpr int kPartCols = kTcPartCols;
+
+template <int BN, int NCOLS>
 __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase, int row0, int M,
-                                              int nb, float4* st) {
+                                              int nb, int c_begin, float4* st) {
   const int lane = threadIdx.x & 31;
   const int sub = lane >> 3, slot = lane & 7;
   const LayerOutArgs& p = a.lo;
@@ -154,7 +162,7 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
 #pragma unroll
   for (int k = 0; k < 8; ++k) ss[k] = dd[k] = dp[k] = 0.f;
 #pragma unroll 1
-  for (int c0 = 0; c0 < BN; c0 += 32) {
+  for (int c0 = c_begin; c0 < c_begin + NCOLS; c0 += 32) {
     uint32_t r[32];
     tmem_ld32(tbase + c0, r);
     stage_rows(st, r, lane);
@@ -184,18 +192,20 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
         dd[k] += __shfl_xor_sync(0xffffffffu, dd[k], o);
         dp[k] += __shfl_xor_sync(0xffffffffu, dp[k], o);
       }
+      static_assert(NCOLS == kPartCols, "one partial slot per warp and tile");
       if (slot == 0 && tok[k] >= 0)
-        *reinterpret_cast<float4*>(p.part + ((size_t)tok[k] * p.np + nb) * 4) =
+        *reinterpret_cast<float4*>(
+            p.part + ((size_t)tok[k] * p.np + (nb * BN + c_begin) / kPartCols) * 4) =
             make_float4(ss[k], dd[k], dp[k], 0.f);
     }
   }
 }
 
 template <int BN, int EPI>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const GemmArgs args) {
-  using C = TcCfg<BN>;
+  using C = TcCfg<BN, EPI>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -232,7 +242,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull_bar(a), 1);
-      mbar_init(tempty_bar(a), 4);
+      mbar_init(tempty_bar(a), C::EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
     misc[1] = 0;  // abort flag
@@ -332,26 +342,14 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     // ------------------------------ epilogue ------------------------------
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int ew = warp - 2;  // epilogue warp index
+    const int c_begin = (ew >> 2) * C::EPI_COLS;  // second warp of a quadrant: upper columns
     const int row = q * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       int mb, nb;
       tile_coords(tile, m_tiles, n_tiles, mb, nb);
-      if constexpr (EPI == EPI_LAYER_OUT) {
-        // pull this row's h_bar / delta / P_{j+1} segment into L2 while the tile accumulates
-        const LayerOutArgs& p = args.lo;
-        const int mr = mb * BM + row;
-        if (mr < M) {
-          const size_t off = (size_t)p.idx[mr] * p.d + (size_t)nb * BN;
-          prefetch_l2(p.hbar + off, BN * 4);
-          if (!p.last) {
-            if (p.router && !p.first) prefetch_l2(p.delta + off, BN * 4);
-            const int pes = p.p_bf16 ? 2 : 4;
-            if (p.p_next) prefetch_l2(static_cast<const char*>(p.p_next) + off * pes, BN * pes);
-          }
-        }
-      }
       bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);
@@ -366,7 +364,7 @@ __global__ void __launch_bounds__(192, 1)
       const int m = mb * BM + row;
       const bool valid = m < M;
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + q * (32 * 8);
+      float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + ew * (32 * 8);
       if constexpr (EPI == EPI_STORE_F32) {
         epi_store_f32<BN>(args, tbase, mb * BM + q * 32, M, nb, stg);
       } else if constexpr (EPI == EPI_SWIGLU) {
@@ -374,7 +372,7 @@ __global__ void __launch_bounds__(192, 1)
       } else if constexpr (EPI == EPI_SILU) {
         epi_silu<BN>(args, tbase, m, valid, nb);
       } else {
-        epi_layer_out<BN>(args, tbase, mb * BM + q * 32, M, nb, stg);
+        epi_layer_out<BN, C::EPI_COLS>(args, tbase, mb * BM + q * 32, M, nb, c_begin, stg);
       }
       tc_fence_before();
       __syncwarp();
@@ -395,7 +393,7 @@ __global__ void __launch_bounds__(192, 1)
 template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& args,
                        int num_sms, cudaStream_t st) {
-  using C = TcCfg<BN>;
+  using C = TcCfg<BN, EPI>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI>,
@@ -406,7 +404,7 @@ cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const Gem
   const long max_tiles = (long)((args.m_max + BM - 1) / BM) * ((args.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
   const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
-  k_gemm_tc<BN, EPI><<<grid, 192, C::SMEM, st>>>(tmA, tmB, args);
+  k_gemm_tc<BN, EPI><<<grid, C::THREADS, C::SMEM, st>>>(tmA, tmB, args);
   return cudaGetLastError();
 }
 

@@ -119,9 +119,15 @@ struct hero_model {
   int *idx_f, *idx_a, *counts;
   uint32_t* err;
 
-  // host-IO staging (lazily grown)
+  // host-IO staging (lazily grown) and the attention stand-in's upload pipeline
   void* io = nullptr;
   size_t io_bytes = 0;
+  cudaStream_t copy_stream = nullptr;
+  std::vector<cudaEvent_t> ev_ready, ev_consumed;  // per routed block
+  cudaEvent_t ev_start = nullptr;
+  // the adapter branch runs on a side stream, concurrently with the FFN branch
+  cudaStream_t side_stream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
@@ -222,6 +228,13 @@ void free_model(hero_model* m) {
     cudaEventDestroy(p.e1);
   }
   for (auto e : m->event_pool) cudaEventDestroy(e);
+  for (auto e : m->ev_ready) cudaEventDestroy(e);
+  for (auto e : m->ev_consumed) cudaEventDestroy(e);
+  if (m->ev_start) cudaEventDestroy(m->ev_start);
+  if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
+  if (m->ev_fork) cudaEventDestroy(m->ev_fork);
+  if (m->ev_join) cudaEventDestroy(m->ev_join);
+  if (m->side_stream) cudaStreamDestroy(m->side_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io};
   for (void* p : ptrs)
@@ -278,7 +291,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
   const hero_config& c = *cfg;
   const long L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r, dm = c.d_m;
   const long ds = c.d_h + c.d_a, nY = c.d_enc + c.d_head;
-  m->np = bf16 ? (int)(d / 256) : (int)((d + kSimtTileN - 1) / kSimtTileN);
+  m->np = bf16 ? (int)(d / kTcPartCols) : (int)((d + kSimtTileN - 1) / kSimtTileN);
   const hero_dtype hd = w->host_dtype;
   const size_t hes = hd == HERO_BF16 ? 2 : 4;
 
@@ -310,7 +323,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
   CUDA_M(cudaMalloc(&m->wdown, (size_t)L * d * I * es));
   CUDA_M(cudaMalloc(&m->w1, (size_t)L * r * d * es));
   CUDA_M(cudaMalloc(&m->w2, (size_t)L * d * r * es));
-  CUDA_M(cudaMalloc(&m->wr, (size_t)nY * d * es));
+  CUDA_M(cudaMalloc(&m->wr, (size_t)nY * d * es * (bf16 ? 2 : 1)));  // bf16: [W | W] for hi | lo
 
   size_t stage_elems = (size_t)1 << 25;  // 32 Mi elements
   void* stage = nullptr;
@@ -358,10 +371,23 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     if (cudaMalloc(&gain_r, d * sizeof(float)) != cudaSuccess ||
         cudaMemcpy(gain_r, gr.data(), d * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess)
       st = fail(HERO_ERR_CUDA, "router gain upload failed");
-    if (st == HERO_OK) st = up(w->w_hd, m->wr, c.d_enc, d, 1, 1, 0, gain_r);
+    // bf16 models contract it against the operand pair [hi | lo] of h_bar, so the
+    // weight is stored twice along K: wr = [W | W], [nY, 2d].
+    void* wr1 = m->wr;
+    if (st == HERO_OK && bf16 && cudaMalloc(&wr1, (size_t)nY * d * es) != cudaSuccess)
+      st = fail(HERO_ERR_NOMEM, "router weight staging allocation failed");
+    if (st == HERO_OK) st = up(w->w_hd, wr1, c.d_enc, d, 1, 1, 0, gain_r);
     if (st == HERO_OK)
-      st = up(w->ps_w1, static_cast<char*>(m->wr) + (size_t)c.d_enc * d * es, c.d_head, d, 1, 1, 0,
+      st = up(w->ps_w1, static_cast<char*>(wr1) + (size_t)c.d_enc * d * es, c.d_head, d, 1, 1, 0,
               nullptr);
+    if (st == HERO_OK && bf16) {
+      const size_t wb = (size_t)d * es;
+      if (cudaMemcpy2D(m->wr, 2 * wb, wr1, wb, wb, nY, cudaMemcpyDeviceToDevice) != cudaSuccess ||
+          cudaMemcpy2D(static_cast<char*>(m->wr) + wb, 2 * wb, wr1, wb, wb, nY,
+                       cudaMemcpyDeviceToDevice) != cudaSuccess)
+        st = fail(HERO_ERR_CUDA, "router weight duplication failed");
+    }
+    if (bf16 && wr1 && wr1 != m->wr) cudaFree(wr1);
   }
   if (st == HERO_OK && cudaDeviceSynchronize() != cudaSuccess)
     st = fail(HERO_ERR_CUDA, "weight conversion failed: %s", cudaGetErrorString(cudaGetLastError()));
@@ -445,7 +471,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         {(void**)&m->pst, Tm * 4},             {(void**)&m->mst, Tm * 4},
         {(void**)&m->dprev, Tm * 4},           {(void**)&m->gate, Tm * 4},
         {(void**)&m->scale_f, Tm * 4},         {(void**)&m->scale_a, Tm * 4},
-        {(void**)&m->xl, Tm * d * es},         {(void**)&m->u_f, Tm * d * es},
+        {(void**)&m->xl, Tm * d * es * (bf16 ? 2 : 1)},         {(void**)&m->u_f, Tm * d * es},
         {(void**)&m->u_a, Tm * d * es},        {(void**)&m->act, Tm * I * es},
         {(void**)&m->ah, Tm * r * es},         {(void**)&m->mask, Tm},
         {(void**)&m->idx_f, Tm * 4},           {(void**)&m->idx_a, Tm * 4},
@@ -465,12 +491,12 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
   // ---- tensor maps ----
   if (bf16) {
     const uint64_t Tm = (uint64_t)c.max_tokens;
-    bool ok = encode_bf16_2d(&m->tm_xl, m->xl, d, Tm, 128) &&
+    bool ok = encode_bf16_2d(&m->tm_xl, m->xl, 2 * d, Tm, 128) &&
               encode_bf16_2d(&m->tm_uf, m->u_f, d, Tm, 128) &&
               encode_bf16_2d(&m->tm_ua, m->u_a, d, Tm, 128) &&
               encode_bf16_2d(&m->tm_act, m->act, I, Tm, 128) &&
               encode_bf16_2d(&m->tm_ah, m->ah, r, Tm, 128) &&
-              encode_bf16_2d(&m->tm_wr, m->wr, d, nY, 256);
+              encode_bf16_2d(&m->tm_wr, m->wr, 2 * d, nY, 256);
     m->tm_wgu.resize(L);
     m->tm_wd.resize(L);
     m->tm_w1.resize(L);
@@ -487,6 +513,9 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     }
     if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
   }
+  CUDA_M(cudaStreamCreateWithFlags(&m->side_stream, cudaStreamNonBlocking));
+  CUDA_M(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming));
+  CUDA_M(cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming));
   *out = m;
   return HERO_OK;
 #undef TRY_M
@@ -507,86 +536,231 @@ hero_status ensure_io(hero_model* m, size_t bytes) {
   return HERO_OK;
 }
 
-// The per-block launch sequence on device pointers.
-hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, float tau,
-                      uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
-                      uint8_t* mask_out, int32_t* count_out, cudaStream_t st) {
+// Router state of one forward pass (workspace for the fused stack, the caller's
+// for hero_routed_block).
+struct BlockState {
+  float *S, *zeta, *pst, *mst, *dprev;
+};
+
+// Everything of routed block jj after its entry (h_bar, its operand copy and the
+// partial sums are in place): router contraction and router, compaction, LN_ffn,
+// FFN and adapter branches with the block-closing epilogue `lo`.
+hero_status block_body(hero_model* m, int jj, int T, const BlockState& bs, const float* hbar,
+                       const LayerOutArgs& lo, float tau, uint32_t flags, const uint8_t* mask_in_j,
+                       float* gate_out_j, uint8_t* mask_out_j, int32_t* count_out_j,
+                       cudaStream_t st) {
   const hero_config& c = m->cfg;
   const int L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r;
   const int nY = c.d_enc + c.d_head;
+  const int j = jj + 1;
+  const bool dense = flags & HERO_FLAG_DENSE;
+  const size_t es = m->esz;
+  if (!dense) {
+    GemmArgs g{};
+    g.m_dev = nullptr;
+    g.m_static = T;
+    g.m_max = T;
+    g.N = nY;
+    g.K = m->bf16 ? 2 * d : d;   // bf16: K runs over the operand pair [hi | lo]
+    g.out_f32 = m->Y;
+    g.ldo = nY;
+    g.err = m->err;
+    g.A = m->xl;
+    g.B = m->wr;
+    g.lda = d;
+    g.ldb = d;
+    CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
+      return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
+                     : launch_gemm_simt(EPI_STORE_F32, g, st);
+    }));
+    RouterArgs ra{};
+    ra.T = T;
+    ra.j = j;
+    ra.L = L;
+    ra.np = m->np;
+    ra.d = d;
+    ra.d_h = c.d_h;
+    ra.d_a = c.d_a;
+    ra.d_enc = c.d_enc;
+    ra.d_head = c.d_head;
+    ra.d_path = c.d_path;
+    ra.Y = m->Y;
+    ra.part = m->part;
+    ra.dprev = bs.dprev;
+    ra.pst = bs.pst;
+    ra.mst = bs.mst;
+    ra.S = bs.S;
+    ra.zeta = bs.zeta;
+    ra.rho = m->rho[jj];
+    ra.w = m->rw;
+    ra.rms_eps = c.rms_eps;
+    ra.eps = c.eps;
+    ra.t_hist = c.t_hist;
+    ra.tau = tau;
+    ra.mask_in = mask_in_j;
+    ra.gate = m->gate;
+    ra.mask = m->mask;
+    ra.gate_out = gate_out_j;
+    ra.mask_out = mask_out_j;
+    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, st); }));
+  }
+  CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
+                 m->counts, count_out_j, dense ? gate_out_j : nullptr,
+                 dense ? mask_out_j : nullptr};
+  CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
+  NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, hbar, m->part,
+              m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
+  CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, st); }));
+
+  // FFN branch: gate/up + SwiGLU, then down + scaled scatter
+  {
+    GemmArgs g{};
+    g.m_dev = m->counts;
+    g.m_max = T;
+    g.N = m->bf16 ? 2 * I : I;
+    g.K = d;
+    g.out = m->act;
+    g.ldo = I;
+    g.err = m->err;
+    g.A = m->u_f;
+    g.lda = d;
+    g.B = static_cast<const char*>(m->wgu) + (size_t)jj * (m->bf16 ? 2 : 1) * I * d * es;
+    g.B2 = m->bf16 ? nullptr : static_cast<const char*>(m->wup) + (size_t)jj * I * d * es;
+    g.ldb = d;
+    CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] {
+      return m->bf16 ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], g, m->num_sms, st)
+                     : launch_gemm_simt(EPI_SWIGLU, g, st);
+    }));
+    // The adapter branch (disjoint token rows) may start now on the side stream and
+    // fill the SMs the FFN-down GEMM leaves idle in its last wave.
+    if (!dense && m->side_stream) {
+      CUDA_TRY(cudaEventRecord(m->ev_fork, st));
+      CUDA_TRY(cudaStreamWaitEvent(m->side_stream, m->ev_fork, 0));
+    }
+    GemmArgs g2{};
+    g2.m_dev = m->counts;
+    g2.m_max = T;
+    g2.N = d;
+    g2.K = I;
+    g2.err = m->err;
+    g2.lo = lo;
+    g2.lo.idx = m->idx_f;
+    g2.lo.scale = m->scale_f;
+    g2.A = m->act;
+    g2.lda = I;
+    g2.B = static_cast<const char*>(m->wdown) + (size_t)jj * d * I * es;
+    g2.ldb = I;
+    CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
+      return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], g2, m->num_sms, st)
+                     : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
+    }));
+  }
+  // adapter branch
+  if (!dense) {
+    cudaStream_t sa = m->side_stream ? m->side_stream : st;
+    GemmArgs g{};
+    g.m_dev = m->counts + 1;
+    g.m_max = T;
+    g.N = r;
+    g.K = d;
+    g.out = m->ah;
+    g.ldo = r;
+    g.err = m->err;
+    g.A = m->u_a;
+    g.lda = d;
+    g.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
+    g.ldb = d;
+    CUDA_TRY(timed(m, HERO_K_ADAPTER_DOWN, sa, [&] {
+      return m->bf16 ? launch_gemm_tc(64, EPI_SILU, m->tm_ua, m->tm_w1[jj], g, m->num_sms, sa)
+                     : launch_gemm_simt(EPI_SILU, g, sa);
+    }));
+    AdapterUpArgs au{};
+    au.m_dev = m->counts + 1;
+    au.m_max = T;
+    au.d = d;
+    au.d_r = r;
+    au.ah = m->ah;
+    au.w2 = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
+    au.bf16 = m->bf16;
+    au.slot_cols = m->bf16 ? kTcPartCols : kSimtTileN;
+    au.lo = lo;
+    au.lo.idx = m->idx_a;
+    au.lo.scale = m->scale_a;
+    CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, sa, [&] { return launch_adapter_up(au, sa); }));
+    if (m->side_stream) {   // join: the next block reads every token's rows
+      CUDA_TRY(cudaEventRecord(m->ev_join, m->side_stream));
+      CUDA_TRY(cudaStreamWaitEvent(st, m->ev_join, 0));
+    }
+  }
+  return HERO_OK;
+}
+
+// Host-resident attention stand-in fed to the stack block by block: P_k is copied
+// on the model's copy stream into device slot k % 3 and the compute stream waits
+// for it just before its first reader; slot k % 3 is refilled with P_{k+3} once the
+// reader of P_k has run, so uploads overlap the compute of earlier blocks.
+struct PFeed {
+  const char* host;     // [L, T, d] in the model's operand type
+  char* slots;          // 3 device slots of one block each
+  size_t layer_bytes;
+};
+constexpr int kPSlots = 3;
+
+hero_status feed_copy(hero_model* m, const PFeed& f, int k, cudaStream_t st, bool after_consume) {
+  if (after_consume) CUDA_TRY(cudaStreamWaitEvent(m->copy_stream, m->ev_consumed[k - kPSlots], 0));
+  CUDA_TRY(cudaMemcpyAsync(f.slots + (size_t)(k % kPSlots) * f.layer_bytes,
+                           f.host + (size_t)k * f.layer_bytes, f.layer_bytes,
+                           cudaMemcpyHostToDevice, m->copy_stream));
+  CUDA_TRY(cudaEventRecord(m->ev_ready[k], m->copy_stream));
+  (void)st;
+  return HERO_OK;
+}
+
+// The per-block launch sequence on device pointers (P device-resident, or fed
+// from the host through `feed`).
+hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, float tau,
+                      uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
+                      uint8_t* mask_out, int32_t* count_out, cudaStream_t st,
+                      const PFeed* feed = nullptr) {
+  const hero_config& c = m->cfg;
+  const int L = c.n_layers, d = c.d_model;
   const bool dense = flags & HERO_FLAG_DENSE;
   const bool force = flags & HERO_FLAG_FORCE_MASK;
   const size_t es = m->esz;
   const size_t layer_elems = (size_t)T * d;
+  auto p_layer = [&](int k) -> const void* {
+    if (k >= L) return nullptr;
+    if (feed) return feed->slots + (size_t)(k % kPSlots) * feed->layer_bytes;
+    return P ? static_cast<const char*>(P) + (size_t)k * layer_elems * es : nullptr;
+  };
+  if (feed) {
+    // the slots may still be read by the previous call's kernels on `st`
+    CUDA_TRY(cudaEventRecord(m->ev_start, st));
+    CUDA_TRY(cudaStreamWaitEvent(m->copy_stream, m->ev_start, 0));
+    for (int k = 0; k < L && k < kPSlots; ++k) {
+      hero_status s = feed_copy(m, *feed, k, st, false);
+      if (s != HERO_OK) return s;
+    }
+  }
 
   for (int jj = 0; jj < L; ++jj) {
-    const int j = jj + 1;
-    const void* Pj = P ? static_cast<const char*>(P) + (size_t)jj * layer_elems * es : nullptr;
-    const void* Pn = (P && jj + 1 < L) ? static_cast<const char*>(P) + (size_t)(jj + 1) * layer_elems * es
-                                       : nullptr;
+    const void* Pj = p_layer(jj);
+    const void* Pn = p_layer(jj + 1);
     if (jj == 0) {
+      if (feed) CUDA_TRY(cudaStreamWaitEvent(st, m->ev_ready[0], 0));
       InitArgs ia{T, d, m->np, c.d_m, h_in, Pj, (int)m->bf16, m->hbar, m->xl, (int)m->bf16,
                   m->part, m->S, m->zeta, m->pst, m->mst, m->dprev, dense ? 0 : 1};
       CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_init(ia, st); }));
+      if (feed) {
+        CUDA_TRY(cudaEventRecord(m->ev_consumed[0], st));
+        if (kPSlots < L) {
+          hero_status s = feed_copy(m, *feed, kPSlots, st, true);
+          if (s != HERO_OK) return s;
+        }
+      }
     }
-    if (!dense) {
-      GemmArgs g{};
-      g.m_dev = nullptr;
-      g.m_static = T;
-      g.m_max = T;
-      g.N = nY;
-      g.K = d;
-      g.out_f32 = m->Y;
-      g.ldo = nY;
-      g.err = m->err;
-      g.A = m->xl;
-      g.B = m->wr;
-      g.lda = d;
-      g.ldb = d;
-      CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
-        return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
-                       : launch_gemm_simt(EPI_STORE_F32, g, st);
-      }));
-      RouterArgs ra{};
-      ra.T = T;
-      ra.j = j;
-      ra.L = L;
-      ra.np = m->np;
-      ra.d = d;
-      ra.d_h = c.d_h;
-      ra.d_a = c.d_a;
-      ra.d_enc = c.d_enc;
-      ra.d_head = c.d_head;
-      ra.d_path = c.d_path;
-      ra.Y = m->Y;
-      ra.part = m->part;
-      ra.dprev = m->dprev;
-      ra.pst = m->pst;
-      ra.mst = m->mst;
-      ra.S = m->S;
-      ra.zeta = m->zeta;
-      ra.rho = m->rho[jj];
-      ra.w = m->rw;
-      ra.rms_eps = c.rms_eps;
-      ra.eps = c.eps;
-      ra.t_hist = c.t_hist;
-      ra.tau = tau;
-      ra.mask_in = force ? mask_in + (size_t)jj * T : nullptr;
-      ra.gate = m->gate;
-      ra.mask = m->mask;
-      ra.gate_out = gate_out ? gate_out + (size_t)jj * T : nullptr;
-      ra.mask_out = mask_out ? mask_out + (size_t)jj * T : nullptr;
-      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, st); }));
-    }
-    CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
-                   m->counts, count_out ? count_out + jj : nullptr,
-                   dense && gate_out ? gate_out + (size_t)jj * T : nullptr,
-                   dense && mask_out ? mask_out + (size_t)jj * T : nullptr};
-    CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
-    NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, m->hbar, m->part,
-                m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
-    CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, st); }));
-
+    if (feed && jj + 1 < L) CUDA_TRY(cudaStreamWaitEvent(st, m->ev_ready[jj + 1], 0));
+    BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
     LayerOutArgs lo{};
     lo.hbar = m->hbar;
     lo.delta = m->delta;
@@ -596,81 +770,24 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
     lo.h_out = h_out;
     lo.d = d;
     lo.np = m->np;
-    lo.tile_n = m->bf16 ? 256 : kSimtTileN;
+    lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
     lo.last = jj == L - 1;
     lo.first = jj == 0;
     lo.p_bf16 = m->bf16;
     lo.xl_bf16 = m->bf16;
     lo.router = dense ? 0 : 1;
-
-    // FFN branch: gate/up + SwiGLU, then down + scaled scatter
-    {
-      GemmArgs g{};
-      g.m_dev = m->counts;
-      g.m_max = T;
-      g.N = m->bf16 ? 2 * I : I;
-      g.K = d;
-      g.out = m->act;
-      g.ldo = I;
-      g.err = m->err;
-      g.A = m->u_f;
-      g.lda = d;
-      g.B = static_cast<const char*>(m->wgu) + (size_t)jj * (m->bf16 ? 2 : 1) * I * d * es;
-      g.B2 = m->bf16 ? nullptr : static_cast<const char*>(m->wup) + (size_t)jj * I * d * es;
-      g.ldb = d;
-      CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] {
-        return m->bf16 ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], g, m->num_sms, st)
-                       : launch_gemm_simt(EPI_SWIGLU, g, st);
-      }));
-      GemmArgs g2{};
-      g2.m_dev = m->counts;
-      g2.m_max = T;
-      g2.N = d;
-      g2.K = I;
-      g2.err = m->err;
-      g2.lo = lo;
-      g2.lo.idx = m->idx_f;
-      g2.lo.scale = m->scale_f;
-      g2.A = m->act;
-      g2.lda = I;
-      g2.B = static_cast<const char*>(m->wdown) + (size_t)jj * d * I * es;
-      g2.ldb = I;
-      CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
-        return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], g2, m->num_sms, st)
-                       : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
-      }));
-    }
-    // adapter branch
-    if (!dense) {
-      GemmArgs g{};
-      g.m_dev = m->counts + 1;
-      g.m_max = T;
-      g.N = r;
-      g.K = d;
-      g.out = m->ah;
-      g.ldo = r;
-      g.err = m->err;
-      g.A = m->u_a;
-      g.lda = d;
-      g.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
-      g.ldb = d;
-      CUDA_TRY(timed(m, HERO_K_ADAPTER_DOWN, st, [&] {
-        return m->bf16 ? launch_gemm_tc(64, EPI_SILU, m->tm_ua, m->tm_w1[jj], g, m->num_sms, st)
-                       : launch_gemm_simt(EPI_SILU, g, st);
-      }));
-      AdapterUpArgs au{};
-      au.m_dev = m->counts + 1;
-      au.m_max = T;
-      au.d = d;
-      au.d_r = r;
-      au.ah = m->ah;
-      au.w2 = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
-      au.bf16 = m->bf16;
-      au.slot_cols = m->bf16 ? 256 : kSimtTileN;
-      au.lo = lo;
-      au.lo.idx = m->idx_a;
-      au.lo.scale = m->scale_a;
-      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] { return launch_adapter_up(au, st); }));
+    hero_status sb = block_body(m, jj, T, bs, m->hbar, lo, tau, flags,
+                                force ? mask_in + (size_t)jj * T : nullptr,
+                                gate_out ? gate_out + (size_t)jj * T : nullptr,
+                                mask_out ? mask_out + (size_t)jj * T : nullptr,
+                                count_out ? count_out + jj : nullptr, st);
+    if (sb != HERO_OK) return sb;
+    if (feed && jj + 1 < L) {  // P_{jj+1} has been read: refill its slot with P_{jj+4}
+      CUDA_TRY(cudaEventRecord(m->ev_consumed[jj + 1], st));
+      if (jj + 1 + kPSlots < L) {
+        hero_status s = feed_copy(m, *feed, jj + 1 + kPSlots, st, true);
+        if (s != HERO_OK) return s;
+      }
     }
   }
   return HERO_OK;
@@ -721,8 +838,20 @@ extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, co
 
   // Host I/O: stage inputs on the device, run, copy outputs back on the stream.
   const size_t esz = m->esz;
-  const size_t p_bytes = attn_delta ? (size_t)L * T * d * esz : 0;
+  const size_t p_layer_bytes = (size_t)T * d * esz;
+  const size_t p_bytes = attn_delta ? (size_t)kPSlots * p_layer_bytes : 0;   // upload ring
   const size_t lt = (size_t)L * T;
+  if (attn_delta && !m->copy_stream) {
+    CUDA_TRY(cudaStreamCreateWithFlags(&m->copy_stream, cudaStreamNonBlocking));
+    CUDA_TRY(cudaEventCreateWithFlags(&m->ev_start, cudaEventDisableTiming));
+  }
+  while (attn_delta && (int)m->ev_ready.size() < L) {
+    cudaEvent_t a = nullptr, b = nullptr;
+    CUDA_TRY(cudaEventCreateWithFlags(&a, cudaEventDisableTiming));
+    CUDA_TRY(cudaEventCreateWithFlags(&b, cudaEventDisableTiming));
+    m->ev_ready.push_back(a);
+    m->ev_consumed.push_back(b);
+  }
   const size_t need = (size_t)T * d * 4 /*h_out*/ + p_bytes + lt /*mask_in*/ + lt * 4 /*gate*/ +
                       lt /*mask*/ + (size_t)L * 4 + 4096;
   hero_status s = ensure_io(m, need);
@@ -741,15 +870,88 @@ extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, co
   int32_t* d_cnt = ffn_count_out ? reinterpret_cast<int32_t*>(carve((size_t)L * 4)) : nullptr;
   // h_0 goes straight into the h_bar buffer; k_init adds P_1 in place.
   CUDA_TRY(cudaMemcpyAsync(m->hbar, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
-  if (d_P) CUDA_TRY(cudaMemcpyAsync(d_P, attn_delta, p_bytes, cudaMemcpyHostToDevice, st));
   if (d_mask_in) CUDA_TRY(cudaMemcpyAsync(d_mask_in, mask_in, lt, cudaMemcpyHostToDevice, st));
-  s = run_stack(m, T, m->hbar, d_P, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask, d_cnt, st);
+  PFeed feed{static_cast<const char*>(attn_delta), static_cast<char*>(d_P), p_layer_bytes};
+  s = run_stack(m, T, m->hbar, nullptr, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask, d_cnt,
+                st, attn_delta ? &feed : nullptr);
   if (s != HERO_OK) return s;
   CUDA_TRY(cudaMemcpyAsync(h_out, d_hout, (size_t)T * d * 4, cudaMemcpyDeviceToHost, st));
   if (d_gate) CUDA_TRY(cudaMemcpyAsync(gate_out, d_gate, lt * 4, cudaMemcpyDeviceToHost, st));
   if (d_mask) CUDA_TRY(cudaMemcpyAsync(mask_out, d_mask, lt, cudaMemcpyDeviceToHost, st));
   if (d_cnt) CUDA_TRY(cudaMemcpyAsync(ffn_count_out, d_cnt, (size_t)L * 4, cudaMemcpyDeviceToHost, st));
   return HERO_OK;
+}
+
+extern "C" hero_status hero_router_state_reset(hero_model* m, int64_t n_tokens,
+                                               const hero_router_state* s, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m || !s) return fail(HERO_ERR_ARG, "model or state is NULL");
+  if (n_tokens < 0 || n_tokens > m->cfg.max_tokens)
+    return fail(HERO_ERR_ARG, "n_tokens %lld outside [0, max_tokens=%d]", (long long)n_tokens,
+                m->cfg.max_tokens);
+  if (n_tokens > 0 && (!s->S || !s->zeta || !s->p_hist || !s->m_hist || !s->d_prev))
+    return fail(HERO_ERR_ARG, "state pointers S, zeta, p_hist, m_hist and d_prev are required");
+  CUDA_TRY(cudaSetDevice(m->device));
+  CUDA_TRY(launch_state_reset(s->S, s->zeta, s->p_hist, s->m_hist, s->d_prev, (int)n_tokens,
+                              m->cfg.d_m, static_cast<cudaStream_t>(cuda_stream)));
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n_tokens,
+                                         const float* h_bar, const hero_router_state* s,
+                                         float tau_exec, uint32_t flags, const uint8_t* mask_in,
+                                         float* h_out, float* gate_out, uint8_t* mask_out,
+                                         int32_t* ffn_count_out, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  const hero_config& c = m->cfg;
+  if (block < 1 || block > c.n_layers)
+    return fail(HERO_ERR_ARG, "block %d outside [1, %d]", block, c.n_layers);
+  if (n_tokens < 0 || n_tokens > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_tokens %lld outside [0, max_tokens=%d]", (long long)n_tokens,
+                c.max_tokens);
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK))
+    return fail(HERO_ERR_ARG, "hero_routed_block takes only HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK");
+  if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
+    return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
+  const bool dense = flags & HERO_FLAG_DENSE;
+  if (!std::isfinite(tau_exec)) return fail(HERO_ERR_ARG, "tau_exec is not finite");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (n_tokens == 0) {
+    CUDA_TRY(cudaSetDevice(m->device));
+    if (ffn_count_out) CUDA_TRY(cudaMemsetAsync(ffn_count_out, 0, 4, st));
+    return HERO_OK;
+  }
+  if (!h_bar || !h_out) return fail(HERO_ERR_ARG, "h_bar and h_out are required");
+  if ((const void*)h_bar == (const void*)h_out) return fail(HERO_ERR_ARG, "h_out must not alias h_bar");
+  if ((flags & HERO_FLAG_FORCE_MASK) && !mask_in)
+    return fail(HERO_ERR_ARG, "HERO_FLAG_FORCE_MASK needs mask_in");
+  if (!dense && (!s || !s->S || !s->zeta || !s->p_hist || !s->m_hist || !s->d_prev ||
+                 !s->h_bar_prev || !s->delta_prev))
+    return fail(HERO_ERR_ARG, "the router state needs all seven pointers");
+  CUDA_TRY(cudaSetDevice(m->device));
+  const int T = (int)n_tokens, jj = block - 1;
+  BlockEntryArgs be{T, c.d_model, m->np, block, dense ? 0 : 1, h_bar,
+                    dense ? nullptr : s->h_bar_prev, dense ? nullptr : s->delta_prev,
+                    m->xl, (int)m->bf16, m->part};
+  CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
+  BlockState bs{dense ? nullptr : s->S, dense ? nullptr : s->zeta, dense ? nullptr : s->p_hist,
+                dense ? nullptr : s->m_hist, dense ? nullptr : s->d_prev};
+  LayerOutArgs lo{};
+  lo.hbar = const_cast<float*>(h_bar);  // read only: the block writes h_out
+  lo.h_out = h_out;
+  lo.part = m->part;
+  lo.d = c.d_model;
+  lo.np = m->np;
+  lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
+  lo.last = 1;
+  lo.first = jj == 0;
+  lo.p_bf16 = m->bf16;
+  lo.xl_bf16 = m->bf16;
+  lo.router = 0;
+  return block_body(m, jj, T, bs, h_bar, lo, tau_exec, flags,
+                    (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr, gate_out, mask_out,
+                    ffn_count_out, st);
 }
 
 extern "C" hero_status hero_check_device_status(hero_model* m, void* cuda_stream) {

@@ -50,6 +50,38 @@ __device__ __forceinline__ void store4(void* base, size_t idx, float4 v, int is_
   }
 }
 
+// Operand copy of h_bar for the router contraction.  bf16 models keep it as a
+// pair per element, hi = bf16(x) and lo = bf16(x - hi) (16 significant bits), in
+// a [T, 2d] row: hi in columns [0, d), lo in [d, 2d).  f32 models: [T, d] fp32.
+__device__ __forceinline__ void store_xl4(void* xl, int xl_bf16, int d, int t, int n, float4 v) {
+  if (xl_bf16) {
+    const __nv_bfloat162 h01 = __floats2bfloat162_rn(v.x, v.y);
+    const __nv_bfloat162 h23 = __floats2bfloat162_rn(v.z, v.w);
+    const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+    const __nv_bfloat162 l01 = __floats2bfloat162_rn(v.x - f01.x, v.y - f01.y);
+    const __nv_bfloat162 l23 = __floats2bfloat162_rn(v.z - f23.x, v.w - f23.y);
+    uint16_t* row = static_cast<uint16_t*>(xl) + (size_t)t * 2 * d;
+    *reinterpret_cast<uint2*>(row + n) = make_uint2(*reinterpret_cast<const uint32_t*>(&h01),
+                                                    *reinterpret_cast<const uint32_t*>(&h23));
+    *reinterpret_cast<uint2*>(row + d + n) = make_uint2(*reinterpret_cast<const uint32_t*>(&l01),
+                                                        *reinterpret_cast<const uint32_t*>(&l23));
+  } else {
+    *reinterpret_cast<float4*>(static_cast<float*>(xl) + (size_t)t * d + n) = v;
+  }
+}
+
+__device__ __forceinline__ void store_xl1(void* xl, int xl_bf16, int d, int t, int n, float v) {
+  if (xl_bf16) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(v);
+    const __nv_bfloat16 l = __float2bfloat16_rn(v - __bfloat162float(h));
+    __nv_bfloat16* row = static_cast<__nv_bfloat16*>(xl) + (size_t)t * 2 * d;
+    row[n] = h;
+    row[d + n] = l;
+  } else {
+    static_cast<float*>(xl)[(size_t)t * d + n] = v;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Block-closing epilogue on 4 consecutive columns n..n+3 of token t.
 // y: GEMM outputs, s: branch scale.  Accumulates the partial sums.
@@ -79,7 +111,7 @@ __device__ __forceinline__ void layer_out4(const LayerOutArgs& p, int t, int n, 
     float4 dn;
     dn.x = s * y.x + pn.x; dn.y = s * y.y + pn.y; dn.z = s * y.z + pn.z; dn.w = s * y.w + pn.w;
     *reinterpret_cast<float4*>(p.delta + off) = dn;
-    store4(p.xl, off, hn, p.xl_bf16);
+    store_xl4(p.xl, p.xl_bf16, p.d, t, n, hn);
     dd += dn.x * dn.x + dn.y * dn.y + dn.z * dn.z + dn.w * dn.w;
     dp += dn.x * dprev.x + dn.y * dprev.y + dn.z * dprev.z + dn.w * dprev.w;
   }
@@ -126,7 +158,7 @@ __device__ __forceinline__ void layer_out_store(const LayerOutArgs& p, int t, in
     float4 dn;
     dn.x = s * y.x + pn.x; dn.y = s * y.y + pn.y; dn.z = s * y.z + pn.z; dn.w = s * y.w + pn.w;
     *reinterpret_cast<float4*>(p.delta + off) = dn;
-    store4(p.xl, off, hn, p.xl_bf16);
+    store_xl4(p.xl, p.xl_bf16, p.d, t, n, hn);
     const float4 dv = in.dprev;
     dd += dn.x * dn.x + dn.y * dn.y + dn.z * dn.z + dn.w * dn.w;
     dp += dn.x * dv.x + dn.y * dv.y + dn.z * dv.z + dn.w * dv.w;
@@ -168,10 +200,7 @@ __device__ __forceinline__ void layer_out_store1(const LayerOutArgs& p, int t, i
   if (p.router) {
     const float dn = s * y + in.pn;
     p.delta[off] = dn;
-    if (p.xl_bf16)
-      static_cast<__nv_bfloat16*>(p.xl)[off] = __float2bfloat16_rn(hn);
-    else
-      static_cast<float*>(p.xl)[off] = hn;
+    store_xl1(p.xl, p.xl_bf16, p.d, t, n, hn);
     dd += dn * dn;
     dp += dn * in.dprev;
   }

@@ -90,6 +90,10 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
 cudaError_t launch_gemm_simt(EpiKind epi, const GemmArgs& args, cudaStream_t st);
 constexpr int kSimtTileN = 64;
 
+// Columns per partial-sum slot of the block-closing epilogues: bf16 models (tensor
+// core path) use the 256-column tile, f32 models the SIMT tile width.
+constexpr int kTcPartCols = 256;
+
 // Router and bookkeeping kernels ------------------------------------------------
 
 struct RouterWeights {   // shared router parameters, fp32, transposed to [in][out]
@@ -149,6 +153,21 @@ struct InitArgs {
   int reset_router;      // 0 in dense mode
 };
 cudaError_t launch_init(const InitArgs& a, cudaStream_t st);
+
+// Entry of one routed block run on its own (hero_routed_block).
+struct BlockEntryArgs {
+  int T, d, np, j;       // j is 1-based
+  int router;            // 0 in dense mode: only the sum of squares is needed
+  const float* h_bar;    // [T, d] post-attention hidden states of this block
+  float* h_bar_prev;     // [T, d] in: previous block's h_bar; out: this block's
+  float* delta_prev;     // [T, d] in: previous block's delta; out: this block's
+  void* xl;              // router operand copy of h_bar
+  int xl_bf16;
+  float* part;           // [T, np, 4]
+};
+cudaError_t launch_block_entry(const BlockEntryArgs& a, cudaStream_t st);
+cudaError_t launch_state_reset(float* S, float* zeta, float* pst, float* mst, float* dprev, int T,
+                               int dm, cudaStream_t st);
 
 struct CompactArgs {
   int T;

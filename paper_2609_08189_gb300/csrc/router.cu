@@ -33,7 +33,7 @@ __global__ void __launch_bounds__(256) k_init(const InitArgs a) {
       h.x += p.x; h.y += p.y; h.z += p.z; h.w += p.w;
     }
     *reinterpret_cast<float4*>(a.hbar + row + n) = h;
-    store4(a.xl, row + n, h, a.xl_bf16);
+    store_xl4(a.xl, a.xl_bf16, a.d, t, n, h);
     ss += h.x * h.x + h.y * h.y + h.z * h.z + h.w * h.w;
   }
   ss = warp_sum(ss);
@@ -50,6 +50,62 @@ __global__ void __launch_bounds__(256) k_init(const InitArgs a) {
       a.pst[t] = 1.f;   // p_hist_{l_0} = 1
       a.mst[t] = 1.f;   // m_hist_{l_0} = 1
       a.dprev[t] = 0.f;
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------
+// k_block_entry: one warp per token, for one routed block run on its own.
+// delta_j = h_bar_j - h_bar_{j-1} (Eq. 7, zero for j = 1); partial sums
+// (sum h_bar^2, sum delta^2, sum delta . delta_{j-1}) into slot 0; the router's
+// operand copy of h_bar; then the carried h_bar_prev / delta_prev become this
+// block's (each element is read before it is overwritten by the same lane).
+// ------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_block_entry(const BlockEntryArgs a) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= a.T) return;
+  const int t = warp;
+  const size_t row = (size_t)t * a.d;
+  float ss = 0.f, dd = 0.f, dp = 0.f;
+  for (int n = lane * 4; n < a.d; n += 128) {
+    const float4 h = *reinterpret_cast<const float4*>(a.h_bar + row + n);
+    float4 dl = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (a.router) {
+      if (a.j > 1) {
+        const float4 hp = *reinterpret_cast<const float4*>(a.h_bar_prev + row + n);
+        dl = make_float4(h.x - hp.x, h.y - hp.y, h.z - hp.z, h.w - hp.w);
+      }
+      if (a.j > 2) {
+        const float4 dv = *reinterpret_cast<const float4*>(a.delta_prev + row + n);
+        dp += dl.x * dv.x + dl.y * dv.y + dl.z * dv.z + dl.w * dv.w;
+      }
+      dd += dl.x * dl.x + dl.y * dl.y + dl.z * dl.z + dl.w * dl.w;
+      *reinterpret_cast<float4*>(a.h_bar_prev + row + n) = h;
+      *reinterpret_cast<float4*>(a.delta_prev + row + n) = dl;
+      store_xl4(a.xl, a.xl_bf16, a.d, t, n, h);
+    }
+    ss += h.x * h.x + h.y * h.y + h.z * h.z + h.w * h.w;
+  }
+  ss = warp_sum(ss);
+  dd = warp_sum(dd);
+  dp = warp_sum(dp);
+  for (int s = lane; s < a.np; s += 32)
+    *reinterpret_cast<float4*>(a.part + ((size_t)t * a.np + s) * 4) =
+        s == 0 ? make_float4(ss, dd, dp, 0.f) : make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+// Router state reset for a new forward pass (S = 0, zeta = 0, p = m = 1, d_prev = 0).
+__global__ void __launch_bounds__(256) k_state_reset(float* S, float* zeta, float* pst, float* mst,
+                                                     float* dprev, int T, int dm) {
+  const long n_s = (long)T * dm * dm;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n_s; i += (long)gridDim.x * blockDim.x) {
+    S[i] = 0.f;
+    if (i < (long)T * dm) zeta[i] = 0.f;
+    if (i < T) {
+      pst[i] = 1.f;
+      mst[i] = 1.f;
+      dprev[i] = 0.f;
     }
   }
 }
@@ -547,6 +603,22 @@ cudaError_t launch_init(const InitArgs& a, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
   const int warps_per_block = 8;
   k_init<<<(a.T + warps_per_block - 1) / warps_per_block, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_block_entry(const BlockEntryArgs& a, cudaStream_t st) {
+  if (a.T <= 0) return cudaSuccess;
+  k_block_entry<<<(a.T + 7) / 8, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_state_reset(float* S, float* zeta, float* pst, float* mst, float* dprev, int T,
+                               int dm, cudaStream_t st) {
+  if (T <= 0) return cudaSuccess;
+  long n = (long)T * dm * dm;
+  long blocks = (n + 255) / 256;
+  if (blocks > 8192) blocks = 8192;
+  k_state_reset<<<(unsigned)blocks, 256, 0, st>>>(S, zeta, pst, mst, dprev, T, dm);
   return cudaGetLastError();
 }
 

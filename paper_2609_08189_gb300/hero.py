@@ -44,6 +44,13 @@ class hero_weights_host(ctypes.Structure):
     _fields_ = [("host_dtype", ctypes.c_int)] + [(n, ctypes.c_void_p) for n in WEIGHT_FIELDS]
 
 
+STATE_FIELDS = ("S", "zeta", "p_hist", "m_hist", "d_prev", "h_bar_prev", "delta_prev")
+
+
+class hero_router_state(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in STATE_FIELDS]
+
+
 class HeroError(RuntimeError):
     def __init__(self, status: int, msg: str):
         super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
@@ -80,6 +87,11 @@ def load(path: Optional[str] = None) -> ctypes.CDLL:
     lib.hero_get_profile.restype = ctypes.c_int
     lib.hero_gemm_bf16_check.argtypes = [vp, vp, vp, i32, i32, i32, vp]
     lib.hero_gemm_bf16_check.restype = ctypes.c_int
+    lib.hero_router_state_reset.argtypes = [vp, i64, ctypes.POINTER(hero_router_state), vp]
+    lib.hero_router_state_reset.restype = ctypes.c_int
+    lib.hero_routed_block.argtypes = [vp, i32, i64, vp, ctypes.POINTER(hero_router_state), f32, u32,
+                                      vp, vp, vp, vp, vp, vp]
+    lib.hero_routed_block.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -133,6 +145,26 @@ def hero_routed_ffn_stack(model: int, n_tokens: int, h_in: int, attn_delta: int,
                                         cuda_stream or None))
 
 
+def make_state(ptrs: Dict[str, int]) -> hero_router_state:
+    """hero_router_state from raw device addresses keyed by STATE_FIELDS (missing = NULL)."""
+    return hero_router_state(*[ptrs.get(n) or None for n in STATE_FIELDS])
+
+
+def hero_router_state_reset(model: int, n_tokens: int, state: hero_router_state,
+                            cuda_stream: int = 0) -> None:
+    _check(load().hero_router_state_reset(model, n_tokens, ctypes.byref(state), cuda_stream or None))
+
+
+def hero_routed_block(model: int, block: int, n_tokens: int, h_bar: int, state: hero_router_state,
+                      tau_exec: float, flags: int, mask_in: int, h_out: int, gate_out: int,
+                      mask_out: int, ffn_count_out: int, cuda_stream: int) -> None:
+    """One routed block on post-attention hidden states (pointer-level call)."""
+    _check(load().hero_routed_block(model, block, n_tokens, h_bar or None, ctypes.byref(state),
+                                    float(tau_exec), flags, mask_in or None, h_out or None,
+                                    gate_out or None, mask_out or None, ffn_count_out or None,
+                                    cuda_stream or None))
+
+
 def hero_free(model: int) -> None:
     if model:
         load().hero_free(model)
@@ -155,6 +187,7 @@ def hero_get_profile(model: int, reset: bool = True):
 
 def hero_gemm_bf16_check(A: int, B: int, C: int, M: int, N: int, K: int, cuda_stream: int = 0) -> None:
     _check(load().hero_gemm_bf16_check(A, B, C, M, N, K, cuda_stream or None))
+
 
 
 # ---------------------------------------------------------------------------

@@ -11,6 +11,8 @@ Tolerances (fixed by the workload definition):
 
 from __future__ import annotations
 
+import json
+import os
 from dataclasses import dataclass, field
 from typing import Dict, List, Optional
 
@@ -22,6 +24,32 @@ from synth import hero_inputs as hi
 BOUNDARY = 1e-3
 GATE_TOL = 1e-3
 H_TOL = {"f32": 1e-5, "bf16": 2e-2}
+
+_SENS = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "gate_sensitivity.json")
+
+
+def free_run_gate_bound(name: str) -> float:
+    """Gate bound for a free-running bf16 stack compared over its full depth.
+
+    The gate bound GATE_TOL holds block by block (teacher-forced tests).  Over the
+    full depth of a bf16 stack the float64 oracle itself moves its gates by more
+    than that when h_0 is perturbed at the size of fp32 rounding: a bf16 rounding
+    that flips feeds every later block (tests/golden/gate_sensitivity.json, written
+    by tests/golden/gate_sensitivity.py from the oracle alone).  No fp32
+    implementation can agree with the oracle below that floor, so the free-running
+    bound is twice the oracle's own largest drift under 1e-7, 3e-7 and 1e-6
+    relative perturbations of the same token sample (the drift is chaotic, not
+    monotone in the perturbation), and never less than GATE_TOL.
+    """
+    try:
+        with open(_SENS) as f:
+            rec = json.load(f).get(name)
+    except OSError:
+        rec = None
+    if not rec:
+        return GATE_TOL
+    drift = max(v["gate_max"] for k, v in rec.items() if isinstance(v, dict))
+    return max(GATE_TOL, 2.0 * drift)
 
 
 def rel_err_rows(x: np.ndarray, y: np.ndarray) -> np.ndarray:

@@ -1,0 +1,166 @@
+"""GPU parity of single routed blocks (hero_routed_block).
+
+Teacher-forced parity: block j of the CUDA path is fed the oracle's own state
+before block j (memory S, zeta, p_hist, m_hist, d_{j-1}, h_bar_{j-1}, delta_{j-1})
+and its post-attention input h_bar_j, runs once, and is compared with the oracle's
+block j: gates, decisions, h_j and the updated state.  Each block is compared in
+isolation, so the bf16 rounding cascade through depth (see the free-running
+tests) does not enter and the stated bounds apply block by block at full size.
+Also: chaining hero_routed_block over all blocks reproduces hero_routed_ffn_stack.
+"""
+
+import numpy as np
+import pytest
+
+from oracle import hero_oracle as ho
+from synth import hero_inputs as hi
+from tests import parity as pr
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hero():
+    import torch
+    assert torch.cuda.is_available()
+    from paper_2609_08189_gb300 import build, hero as H
+    build.build()
+    H.load()
+    return H
+
+
+def _state_tensors(T, d, dm):
+    import torch
+    f = dict(device="cuda", dtype=torch.float32)
+    return {"S": torch.zeros((T, dm, dm), **f), "zeta": torch.zeros((T, dm), **f),
+            "p_hist": torch.ones((T,), **f), "m_hist": torch.ones((T,), **f),
+            "d_prev": torch.zeros((T,), **f), "h_bar_prev": torch.zeros((T, d), **f),
+            "delta_prev": torch.zeros((T, d), **f)}
+
+
+def _ptrs(ts):
+    return {k: v.data_ptr() for k, v in ts.items()}
+
+
+TF = [("tiny_f32", None, None), ("small_bf16", None, None), ("llama2_7b_prefill", None, 32),
+      ("llama31_8b_prefill", None, 32), ("llama31_8b_decode", None, 32),
+      ("llama2_13b_prefill", 0.27, 16)]
+
+
+@pytest.mark.parametrize("name,bypass,n_sample", TF)
+def test_teacher_forced_blocks(hero, name, bypass, n_sample):
+    import torch
+    inp = pr.inputs(name, bypass=bypass)
+    cfg = inp.cfg
+    rows = np.arange(cfg.n_tokens) if n_sample is None else hi.sample_tokens(cfg.n_tokens, n_sample)
+    T, d, dm, L = len(rows), cfg.d_model, cfg.d_m, cfg.n_layers
+    ref = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), inp.weights, inp.h[rows],
+                              inp.P[:, rows], inp.tau, record=True)
+    lay = ref["layers"]
+    st = hero.HeroStack(cfg, inp.weights, max_tokens=T)
+    ts = _state_tensors(T, d, dm)
+    state = hero.make_state(_ptrs(ts))
+    g = torch.empty(T, device="cuda")
+    m = torch.empty(T, device="cuda", dtype=torch.uint8)
+    h_out = torch.empty((T, d), device="cuda")
+    cnt = torch.empty(1, device="cuda", dtype=torch.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    tol_h = pr.H_TOL[cfg.dtype]
+    worst_g = worst_h = worst_S = 0.0
+    far = 0
+    f32 = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.float32), device="cuda")
+    for j in range(1, L + 1):
+        if j == 1:
+            hero.hero_router_state_reset(st.model, T, state, stream)
+        else:
+            prev = lay[j - 2]
+            ts["S"].copy_(f32(prev["S"]))
+            ts["zeta"].copy_(f32(prev["zeta"]))
+            ts["p_hist"].copy_(f32(prev["p"]))
+            ts["m_hist"].copy_(f32(prev["m"]))
+            ts["d_prev"].copy_(f32(prev["d"]))
+            ts["h_bar_prev"].copy_(f32(prev["h_bar"]))
+            ts["delta_prev"].copy_(f32(prev["delta"]))
+        cur = lay[j - 1]
+        hb = f32(cur["h_bar"])
+        mask_in = torch.as_tensor(cur["mask"].astype(np.uint8), device="cuda")
+        hero.hero_routed_block(st.model, j, T, hb.data_ptr(), state, inp.tau,
+                               hero.HERO_FLAG_FORCE_MASK, mask_in.data_ptr(), h_out.data_ptr(),
+                               g.data_ptr(), m.data_ptr(), cnt.data_ptr(), stream)
+        torch.cuda.synchronize()
+        st.check()
+        gg = g.cpu().numpy().astype(np.float64)
+        worst_g = max(worst_g, float(np.max(np.abs(gg - cur["g"]))))
+        worst_h = max(worst_h, float(np.max(pr.rel_err_rows(h_out.cpu().numpy().astype(np.float64),
+                                                            cur["h"]))))
+        # the free decision the GPU would take agrees with the oracle's away from the boundary
+        dec = gg >= inp.tau
+        far += int(np.sum((dec != cur["mask"]) & (np.abs(cur["g"] - inp.tau) >= pr.BOUNDARY)))
+        assert int(cnt.item()) == int(cur["mask"].sum())
+        Sg = ts["S"].cpu().numpy().astype(np.float64)
+        worst_S = max(worst_S, float(np.max(np.abs(Sg - cur["S"])) / (np.max(np.abs(cur["S"])) + 1e-30)))
+    print(name, "teacher-forced: gate", worst_g, "h", worst_h, "S", worst_S)
+    assert far == 0
+    assert worst_g < pr.GATE_TOL
+    assert worst_h < tol_h
+    assert worst_S < (1e-5 if cfg.dtype == "f32" else 1e-3)
+    st.close()
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+def test_block_chain_equals_fused_stack(hero, name):
+    """Blocks run one by one (attention stand-in added by the caller) == the fused stack."""
+    import torch
+    inp = pr.inputs(name)
+    cfg = inp.cfg
+    T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
+    st = hero.HeroStack(cfg, inp.weights)
+    fused = pr.run_gpu(st, inp)
+    ts = _state_tensors(T, d, cfg.d_m)
+    state = hero.make_state(_ptrs(ts))
+    stream = torch.cuda.current_stream().cuda_stream
+    h = torch.from_numpy(inp.h).cuda()
+    if inp.P.dtype == np.uint16:
+        P = torch.from_numpy(inp.P.astype(np.int32) << 16).cuda().view(torch.float32)
+    else:
+        P = torch.from_numpy(inp.P).cuda()
+    g = torch.empty((L, T), device="cuda")
+    m = torch.empty((L, T), device="cuda", dtype=torch.uint8)
+    hero.hero_router_state_reset(st.model, T, state, stream)
+    for j in range(1, L + 1):
+        hb = h + P[j - 1]                    # the caller's "attention" output
+        h = torch.empty_like(hb)
+        hero.hero_routed_block(st.model, j, T, hb.data_ptr(), state, inp.tau, 0, 0, h.data_ptr(),
+                               g[j - 1].data_ptr(), m[j - 1].data_ptr(), 0, stream)
+    torch.cuda.synchronize()
+    st.check()
+    np.testing.assert_array_equal(m.cpu().numpy(), fused.mask)
+    assert np.max(np.abs(g.cpu().numpy() - fused.gate)) < 1e-5
+    assert np.max(pr.rel_err_rows(h.cpu().numpy().astype(np.float64), fused.h_out)) < 1e-4
+    st.close()
+
+
+def test_block_argument_errors(hero):
+    import torch
+    inp = pr.inputs("tiny_f32")
+    st = hero.HeroStack(inp.cfg, inp.weights)
+    state = hero.make_state({})
+    x = torch.zeros((4, inp.cfg.d_model), device="cuda")
+    y = torch.zeros_like(x)
+    for block in (0, inp.cfg.n_layers + 1):
+        with pytest.raises(hero.HeroError) as e:
+            hero.hero_routed_block(st.model, block, 4, x.data_ptr(), state, 0.5, 0, 0, y.data_ptr(),
+                                   0, 0, 0, 0)
+        assert e.value.status == hero.HERO_ERR_ARG
+    with pytest.raises(hero.HeroError) as e:   # routed mode needs the state
+        hero.hero_routed_block(st.model, 1, 4, x.data_ptr(), state, 0.5, 0, 0, y.data_ptr(), 0, 0, 0, 0)
+    assert e.value.status == hero.HERO_ERR_ARG
+    with pytest.raises(hero.HeroError):        # host I/O is not accepted per block
+        hero.hero_routed_block(st.model, 1, 4, x.data_ptr(), state, 0.5, hero.HERO_FLAG_HOST_IO, 0,
+                               y.data_ptr(), 0, 0, 0, 0)
+    # dense mode needs no state
+    hero.hero_routed_block(st.model, 1, 4, x.data_ptr(), state, 0.5, hero.HERO_FLAG_DENSE, 0,
+                           y.data_ptr(), 0, 0, 0, 0)
+    torch.cuda.synchronize()
+    st.check()
+    st.close()

@@ -61,6 +61,18 @@ def test_bf16_round_matches_torch():
         np.testing.assert_array_equal(ho.bf16_round(v), ref)
 
 
+def test_bf16_pair_is_a_16_bit_split():
+    """hi = bf16(x), lo = bf16(x - hi): both bf16 (torch agrees), |x - (hi + lo)| <= 2^-16 |x|."""
+    rng = np.random.default_rng(7)
+    x = (rng.standard_normal(100000) * 10.0 ** rng.integers(-5, 5, 100000)).astype(np.float32)
+    x = x.astype(np.float64)
+    pair = ho.bf16_pair(x)
+    hi = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).to(torch.float64)
+    lo = (torch.tensor(x) - hi).to(torch.float32).to(torch.bfloat16).to(torch.float64)
+    np.testing.assert_array_equal(pair, (hi + lo).numpy())
+    assert np.all(np.abs(x - pair) <= 2.0 ** -16 * np.abs(x))
+
+
 def test_elementwise_functions_match_torch():
     x = np.linspace(-30, 30, 10001)
     np.testing.assert_allclose(ho.sigmoid(x), torch.sigmoid(_t(x)).numpy(), rtol=1e-15, atol=1e-300)
