@@ -217,6 +217,33 @@ hero_status hero_get_profile(hero_model* m, double* ms_out, int64_t* launches_ou
 hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B, float* C, int32_t M,
                                  int32_t N, int32_t K, void* cuda_stream);
 
+/* ---- allocation-free variant ------------------------------------------------
+ * The paper has no counterpart of this entry point; it exists for callers that
+ * must not allocate device memory at call time, such as a host framework that
+ * owns every device allocation through its own pool, or a latency-critical loop
+ * where a cudaMalloc would synchronise the device.
+ *
+ * C[M,N] (fp32) = A[M,K] B[N,K]^T with A, B bf16 (uint16 bit patterns), DEVICE
+ * pointers owned by the caller, row-major, computed as `splits` slices of K (whole
+ * 64-wide blocks) on the tensor-core GEMM kernel and added in slice order.  The
+ * partial sums (splits * M * N fp32, at most 4,194,304 values = 16 MiB) and the
+ * kernel's error word live in static device arrays that every GPU loading this
+ * library holds until process exit.  Nothing is allocated: no cudaMalloc, no
+ * cudaFree, no allocating library call.
+ *   - Requires M >= 1, N % 8 == 0, K % 64 == 0, 1 <= splits <= K / 64 and
+ *     splits * M * N <= 4,194,304; otherwise HERO_ERR_ARG (hero_last_error()
+ *     says which limit) and nothing is enqueued.
+ *   - The first call on a device resolves the static arrays' device addresses
+ *     for that device (with it current); make that first call before any stream
+ *     capture.
+ *   - Every call shares the static arrays and the arrays keep the last call's
+ *     contents; calls that overlap on the GPU (other streams, other host
+ *     threads) race on them.  Serialise calls on one stream.
+ *   - Asynchronous on cuda_stream like the other entry points. */
+hero_status hero_gemm_bf16_splitk_noalloc(const uint16_t* A, const uint16_t* B, float* C,
+                                          int32_t M, int32_t N, int32_t K, int32_t splits,
+                                          void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -92,6 +92,8 @@ def load(path: Optional[str] = None) -> ctypes.CDLL:
     lib.hero_routed_block.argtypes = [vp, i32, i64, vp, ctypes.POINTER(hero_router_state), f32, u32,
                                       vp, vp, vp, vp, vp, vp]
     lib.hero_routed_block.restype = ctypes.c_int
+    lib.hero_gemm_bf16_splitk_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
+    lib.hero_gemm_bf16_splitk_noalloc.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -188,6 +190,11 @@ def hero_get_profile(model: int, reset: bool = True):
 def hero_gemm_bf16_check(A: int, B: int, C: int, M: int, N: int, K: int, cuda_stream: int = 0) -> None:
     _check(load().hero_gemm_bf16_check(A, B, C, M, N, K, cuda_stream or None))
 
+
+def hero_gemm_bf16_splitk_noalloc(A: int, B: int, C: int, M: int, N: int, K: int, splits: int,
+                                  cuda_stream: int = 0) -> None:
+    """Split-K bf16 GEMM whose scratch lives in static device memory (no allocation)."""
+    _check(load().hero_gemm_bf16_splitk_noalloc(A, B, C, M, N, K, splits, cuda_stream or None))
 
 
 # ---------------------------------------------------------------------------
