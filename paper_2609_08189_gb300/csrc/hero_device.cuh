@@ -118,7 +118,8 @@ __device__ __forceinline__ void layer_out4(const LayerOutArgs& p, int t, int n, 
 }
 
 // The same epilogue split into a load phase and a compute/store phase so that a
-// caller can keep several rows' loads in flight.
+// caller can keep several rows' loads in flight.  (Streaming cache hints on these
+// accesses measured 7% slower for the FFN down GEMM, so none are used.)
 struct LayerOutIn {
   float4 hb, pn, dprev;
 };

@@ -138,7 +138,7 @@ struct RouterLayout {
     x = aux + naux;
     ph = x + 8 * TB;
     red = ph + d_path * TB;
-    sc = red + 2 * 16 * TB;
+    sc = red + 3 * NTHR;
     ab = sc + TB * 16;
     floats = ab + 2 * TB;
   }
@@ -251,18 +251,36 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
                    : "memory");
   }
 
+  // Thread tid serves token tl = tid % TB as part pt = tid / TB of 16 in the two
+  // input phases; the 16 parts of a token are added in a fixed order.
+  const int tl0 = tid % TB, pt0 = tid / TB;
+  const int tok0 = t0 + tl0;
+
   // 1. per-token scalars from the partial sums of the previous block's epilogue;
   //    transition features (Eqs. 7-8) and the path vector (Eqs. 4, 6)
-  if (tid < TB) {
-    const int t = t0 + tid;
-    float ss = 0.f, dd = 0.f, dp = 0.f, dprev = 0.f, pp = 1.f, mp = 1.f;
-    if (t < a.T) {
-      for (int s = 0; s < a.np; ++s) {
-        const float4 v = *reinterpret_cast<const float4*>(a.part + ((size_t)t * a.np + s) * 4);
+  {
+    float ss = 0.f, dd = 0.f, dp = 0.f;
+    if (tok0 < a.T)
+      for (int s = pt0; s < a.np; s += NTHR / TB) {
+        const float4 v = *reinterpret_cast<const float4*>(a.part + ((size_t)tok0 * a.np + s) * 4);
         ss += v.x;
         dd += v.y;
         dp += v.z;
       }
+    red[tid] = ss;
+    red[NTHR + tid] = dd;
+    red[2 * NTHR + tid] = dp;
+  }
+  __syncthreads();
+  if (tid < TB) {
+    const int t = t0 + tid;
+    float ss = 0.f, dd = 0.f, dp = 0.f, dprev = 0.f, pp = 1.f, mp = 1.f;
+    for (int p = 0; p < NTHR / TB; ++p) {
+      ss += red[p * TB + tid];
+      dd += red[NTHR + p * TB + tid];
+      dp += red[2 * NTHR + p * TB + tid];
+    }
+    if (t < a.T) {
       dprev = a.dprev[t];
       pp = a.pst[t];
       mp = a.mst[t];
@@ -284,19 +302,38 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
 
   // 2. encoder hidden SiLU(rinv (W_hd diag(g_r)) h_bar), transposed; f_psi's
   //    second layer reduced on the fly (b = w_ps2 . SiLU(W_ps1 h_bar + b_ps1), Eq. 16).
-  //    Thread tid always serves token tid % TB (the stride is a multiple of TB).
+  //    Part pt reads float4 column groups pt, pt + 16, ... of its token's Y row; a
+  //    warp instruction covers 16 rows x 32 contiguous bytes, and up to eight
+  //    loads per thread are in flight.  d_enc is a multiple of 4, so no group
+  //    straddles the encoder / f_psi boundary.
   {
+    constexpr int YB = 8;
     float bpart = 0.f;
-    const int tl = tid % TB;
-    const int t = t0 + tl;
-    for (int i = tid; i < TB * nY; i += NTHR) {
-      const int c = i / TB;
-      const float y = t < a.T ? __ldg(a.Y + (size_t)t * nY + c) : 0.f;
-      if (c < a.d_enc) {
-        bigT[c * TB + tl] = siluf_(y * sc[tl * 16]);
-      } else {
-        const int e = c - a.d_enc;
-        bpart = fmaf(__ldg(a.w.ps_w2 + e), siluf_(y + __ldg(a.w.ps_b1 + e)), bpart);
+    const int ng = nY >> 2;
+    const float rinv = sc[tl0 * 16];
+    const float4* yrow = reinterpret_cast<const float4*>(a.Y + (size_t)tok0 * nY);
+    for (int g0 = pt0; g0 < ng; g0 += YB * (NTHR / TB)) {
+      float4 yv[YB];
+#pragma unroll
+      for (int k = 0; k < YB; ++k) {
+        const int g = g0 + k * (NTHR / TB);
+        yv[k] = (tok0 < a.T && g < ng) ? __ldg(yrow + g) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < YB; ++k) {
+        const int g = g0 + k * (NTHR / TB);
+        if (g >= ng) break;
+        const int c = 4 * g;
+        const float y4[4] = {yv[k].x, yv[k].y, yv[k].z, yv[k].w};
+        if (c < a.d_enc) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) bigT[(c + i) * TB + tl0] = siluf_(y4[i] * rinv);
+        } else {
+          const int e = c - a.d_enc;
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            bpart = fmaf(__ldg(a.w.ps_w2 + e + i), siluf_(y4[i] + __ldg(a.w.ps_b1 + e + i)), bpart);
+        }
       }
     }
     reduce16(red, bpart, ab + TB);   // also orders step 2's writes before step 3
@@ -537,15 +574,15 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
 }
 
 // ------------------------------------------------------------------------------
-// k_norm: 8 consecutive elements per thread; slot s < n_f is FFN row s (token
-// idx_f[s]), slot s >= n_f is adapter row s - n_f.
+// k_norm: one warp per branch row; slot s < n_f is FFN row s (token idx_f[s]),
+// slot s >= n_f is adapter row s - n_f.  The row's 1/rms comes from the
+// epilogue's partial sums (lane-parallel loads, fixed-order warp reduction); the
+// row is then streamed with up to eight float4 loads per lane in flight.
 // ------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_norm(const NormArgs a) {
-  const int per_row = a.d / 8;
-  const long gid = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  const long slot = gid / per_row;
+  const long slot = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
   if (slot >= a.T) return;
-  const int c = (int)(gid % per_row) * 8;
   const int nf = a.counts[0];
   int t;
   void* dst;
@@ -560,20 +597,31 @@ __global__ void __launch_bounds__(256) k_norm(const NormArgs a) {
     r = slot - nf;
   }
   float ss = 0.f;
-  for (int s = 0; s < a.np; ++s) ss += a.part[((size_t)t * a.np + s) * 4];
+  for (int s = lane; s < a.np; s += 32) ss += a.part[((size_t)t * a.np + s) * 4];
+  ss = warp_sum(ss);
   const float rinv = rsqrtf(ss / (float)a.d + a.rms_eps);
-  const float* h = a.hbar + (size_t)t * a.d + c;
-  const float4 h0 = *reinterpret_cast<const float4*>(h);
-  const float4 h1 = *reinterpret_cast<const float4*>(h + 4);
-  const float4 g0 = *reinterpret_cast<const float4*>(a.gain + c);
-  const float4 g1 = *reinterpret_cast<const float4*>(a.gain + c + 4);
-  const float4 u0 = make_float4(h0.x * rinv * g0.x, h0.y * rinv * g0.y, h0.z * rinv * g0.z,
-                                h0.w * rinv * g0.w);
-  const float4 u1 = make_float4(h1.x * rinv * g1.x, h1.y * rinv * g1.y, h1.z * rinv * g1.z,
-                                h1.w * rinv * g1.w);
-  const size_t off = (size_t)r * a.d + c;
-  store4(dst, off, u0, a.out_bf16);
-  store4(dst, off + 4, u1, a.out_bf16);
+  const float* h = a.hbar + (size_t)t * a.d;
+  const size_t ro = (size_t)r * a.d;
+  constexpr int NB = 8;
+  for (int c0 = lane * 4; c0 < a.d; c0 += 128 * NB) {
+    float4 hv[NB];
+#pragma unroll
+    for (int k = 0; k < NB; ++k) {
+      const int c = c0 + 128 * k;
+      if (c < a.d) hv[k] = *reinterpret_cast<const float4*>(h + c);
+    }
+#pragma unroll
+    for (int k = 0; k < NB; ++k) {
+      const int c = c0 + 128 * k;
+      if (c < a.d) {
+        const float4 g = __ldg(reinterpret_cast<const float4*>(a.gain + c));
+        store4(dst, ro + c,
+               make_float4(hv[k].x * rinv * g.x, hv[k].y * rinv * g.y, hv[k].z * rinv * g.z,
+                           hv[k].w * rinv * g.w),
+               a.out_bf16);
+      }
+    }
+  }
 }
 
 // ------------------------------------------------------------------------------
@@ -655,8 +703,7 @@ cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st) {
 
 cudaError_t launch_norm(const NormArgs& a, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
-  const long threads = (long)a.T * (a.d / 8);
-  k_norm<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(a);
+  k_norm<<<(unsigned)((a.T + 7) / 8), 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 
