@@ -112,19 +112,25 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def algorithmic_work(cfg, counts_per_step, steps):
-    """Executed FLOPs per kernel class over the timed steps (counts: FFN tokens per block)."""
+def algorithmic_work(cfg, counts_per_step, steps, routed=True):
+    """Algorithmic FLOPs per kernel class over the timed steps (counts: FFN tokens per
+    block).  bf16 models run the adapter's down projection inside the FFN gate/up
+    launch of the same block (grouped), so that class carries its FLOPs too."""
     T, d, I, r = cfg.n_tokens, cfg.d_model, cfg.d_ff, cfg.d_r
     nY = cfg.d_enc + cfg.d_head
+    k_r = 2 * d if cfg.dtype == "bf16" else d   # bf16: the operand pair [hi | lo]
     nf = np.asarray(counts_per_step, dtype=np.float64)
     na = T - nf
-    return {
+    work = {
         "ffn_gate_up": steps * float(np.sum(2.0 * nf * 2 * I * d)),
         "ffn_down": steps * float(np.sum(2.0 * nf * I * d)),
-        "router_gemm": steps * float(cfg.n_layers * 2.0 * T * nY * d),
+        "router_gemm": steps * float(cfg.n_layers * 2.0 * T * nY * k_r) if routed else 0.0,
         "adapter_down": steps * float(np.sum(2.0 * na * r * d)),
         "adapter_up": steps * float(np.sum(2.0 * na * d * r)),
     }
+    if cfg.dtype == "bf16":
+        work["ffn_gate_up"] += work.pop("adapter_down")
+    return work
 
 
 def reference_arm(args, rank, world):

@@ -67,7 +67,7 @@ typedef enum { HERO_F32 = 0, HERO_BF16 = 1 } hero_dtype;
  *   t_hist     history temperature T_hist (Eq. 14)
  * Supported: d_m in {16, 32, 64, 128}; d_s <= 128; d_enc, d_head <= 256;
  * d_path <= 64.  bf16 additionally needs d % 256 == 0, d_ff % 128 == 0 and
- * d_r == 64; f32 needs d % 4 == 0. */
+ * d_r % 32 == 0 (d_r <= 4096); f32 needs d % 4 == 0 and d_r <= 64. */
 typedef struct {
   int32_t n_layers, d_model, d_ff, d_r, d_m;
   int32_t d_h, d_a, d_enc, d_head, d_path;
@@ -195,9 +195,10 @@ enum {
   HERO_K_ROUTER = 2,      /* memory read/update, heads, gate, decision        */
   HERO_K_COMPACT = 3,     /* stable scan of the decisions into index lists    */
   HERO_K_NORM = 4,        /* LN^ffn of each token into its branch's rows      */
-  HERO_K_FFN_GATE_UP = 5, /* gathered gate/up GEMM with the SwiGLU epilogue   */
+  HERO_K_FFN_GATE_UP = 5, /* gathered gate/up GEMM with the SwiGLU epilogue;
+                             bf16 models: also the adapter W_1 GEMM (grouped) */
   HERO_K_FFN_DOWN = 6,    /* down GEMM with the scaled scatter epilogue       */
-  HERO_K_ADAPTER_DOWN = 7,/* adapter W_1 GEMM with the SiLU epilogue          */
+  HERO_K_ADAPTER_DOWN = 7,/* f32 models: adapter W_1 GEMM with the SiLU epilogue */
   HERO_K_ADAPTER_UP = 8,  /* adapter W_2 GEMM with the scaled scatter epilogue */
   HERO_K_COUNT = 9
 };

@@ -3,6 +3,11 @@
 //
 //   C[M, N] = A[M, K] * B[N, K]^T        (bf16 operands, fp32 accumulation)
 //
+// A launch may carry a second, independent problem (grouped launch): the FFN and
+// the adapter branch of a routed block touch disjoint token rows, so the adapter's
+// GEMM tiles are spread evenly among the FFN's tiles of the same launch and their
+// epilogues overlap the FFN's tensor-core work.
+//
 // One CTA per SM, 6 warps:
 //   warp 0      TMA producer (one elected lane) - A and B tiles into a STAGES-deep ring
 //   warp 1      TMEM allocator and MMA issuer (one elected lane)
@@ -21,7 +26,9 @@ constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int kGroupM = 16;   // raster: 16 M-tiles share each wave of N-tiles (L2 reuse)
 
-template <int BN, int EPI>
+constexpr int EPI_NONE = -1;   // no second problem
+
+template <int BN, int EPIW>
 struct TcCfg {
   static constexpr int STAGES = BN == 256 ? 4 : 6;
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -32,15 +39,18 @@ struct TcCfg {
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                     ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-  // One epilogue warp per TMEM lane quadrant.  (Two per quadrant, each taking half
-  // of the columns, measured within 1% for the block-closing epilogue.)
-  static constexpr int EPI_WARPS = 4;
+  // EPIW epilogue warps: one (4 warps) or two (8 warps, each taking half of the
+  // tile's columns) per TMEM lane quadrant.
+  static constexpr int EPI_WARPS = EPIW;
+  static constexpr int EPI_COLS = BN / (EPIW / 4);
   static constexpr int THREADS = 64 + 32 * EPI_WARPS;
-  static constexpr int EPI_COLS = BN / (EPI_WARPS / 4);
   // ring | barriers (256 B) | per-epilogue-warp staging tiles (32 x 32 fp32 each)
   static constexpr uint32_t EPI_STAGE_OFF = STAGES * STAGE_BYTES + 256;
   static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + EPI_WARPS * 32 * 32 * 4 + 1024;
 };
+
+template <int EPI>
+constexpr int epi_warps() { return EPI == EPI_LAYER_OUT_WIDE ? 8 : 4; }
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
   const int group = kGroupM * n_tiles;
@@ -118,11 +128,14 @@ __device__ __forceinline__ void epi_swiglu(const GemmArgs& a, uint32_t tbase, in
   }
 }
 
+// Columns past N (a multiple of 32) are not written: the adapter's rank can be
+// narrower than the tile.
 template <int BN>
 __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int m, bool valid,
                                          int nb) {
+  const int ncols = min(BN, a.N - nb * BN);
 #pragma unroll 1
-  for (int c0 = 0; c0 < BN; c0 += 32) {
+  for (int c0 = 0; c0 < ncols; c0 += 32) {
     uint32_t r[32];
     tmem_ld32(tbase + c0, r);
     if (valid) {
@@ -140,13 +153,31 @@ __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int 
 
 // Block-closing epilogue over columns [c_begin, c_begin + NCOLS) of the tile,
 // row-contiguous through the staging tile.  Each lane keeps the partial sums of
-// its 8 rows and reduces them over the 8 lanes that share a row at the end; the
-// partial-sum slot covers kPartCols columns.
-constexpr int kPartCols = kTcPartCols;
+// its 8 rows; every kTcPartCols columns they are reduced over the 8 lanes that
+// share a row and stored as one partial-sum slot.
+template <int BN, int NCOLS>
+__device__ __forceinline__ void flush_partials(const LayerOutArgs& p, const int (&tok)[8],
+                                               float (&ss)[8], float (&dd)[8], float (&dp)[8],
+                                               int slot_lane, int pslot) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+      ss[k] += __shfl_xor_sync(0xffffffffu, ss[k], o);
+      dd[k] += __shfl_xor_sync(0xffffffffu, dd[k], o);
+      dp[k] += __shfl_xor_sync(0xffffffffu, dp[k], o);
+    }
+    if (slot_lane == 0 && tok[k] >= 0)
+      *reinterpret_cast<float4*>(p.part + ((size_t)tok[k] * p.np + pslot) * 4) =
+          make_float4(ss[k], dd[k], dp[k], 0.f);
+    ss[k] = dd[k] = dp[k] = 0.f;
+  }
+}
 
 template <int BN, int NCOLS>
 __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase, int row0, int M,
                                               int nb, int c_begin, float4* st) {
+  static_assert(NCOLS % kTcPartCols == 0, "whole partial-sum slots per warp");
   const int lane = threadIdx.x & 31;
   const int sub = lane >> 3, slot = lane & 7;
   const LayerOutArgs& p = a.lo;
@@ -182,30 +213,76 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
                           scl[k0 + k], ss[k0 + k], dd[k0 + k], dp[k0 + k]);
     }
     __syncwarp();
-  }
-  if (!p.last) {
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-#pragma unroll
-      for (int o = 1; o < 8; o <<= 1) {
-        ss[k] += __shfl_xor_sync(0xffffffffu, ss[k], o);
-        dd[k] += __shfl_xor_sync(0xffffffffu, dd[k], o);
-        dp[k] += __shfl_xor_sync(0xffffffffu, dp[k], o);
-      }
-      static_assert(NCOLS == kPartCols, "one partial slot per warp and tile");
-      if (slot == 0 && tok[k] >= 0)
-        *reinterpret_cast<float4*>(
-            p.part + ((size_t)tok[k] * p.np + (nb * BN + c_begin) / kPartCols) * 4) =
-            make_float4(ss[k], dd[k], dp[k], 0.f);
-    }
+    if (!p.last && (c0 + 32) % kTcPartCols == 0)
+      flush_partials<BN, NCOLS>(p, tok, ss, dd, dp, slot, (nb * BN + c0 + 32) / kTcPartCols - 1);
   }
 }
 
+// Sizes of one problem of a launch (the row count may be device-resident).
+struct ProbSize {
+  int M, m_tiles, n_tiles, kblocks, tiles;
+};
+
+template <int BN>
+__device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
+  ProbSize p;
+  int M = a.m_dev ? *a.m_dev : a.m_static;
+  if (M < 0 || M > a.m_max) {
+    if (threadIdx.x == 0) atomicOr(a.err, ERR_BAD_INDEX);
+    M = 0;
+  }
+  p.M = M;
+  p.m_tiles = (M + BM - 1) / BM;
+  p.n_tiles = (a.N + BN - 1) / BN;
+  p.kblocks = (a.K + BK - 1) / BK;
+  p.tiles = p.m_tiles * p.n_tiles;
+  return p;
+}
+
+// Tile g of a grouped launch -> (problem, tile within it): the second problem's
+// t1 tiles are spread evenly among all `total` tiles (Bresenham), so every
+// persistent CTA gets its share of both.
+__device__ __forceinline__ int split_tile(int g, int t1, int total, int& local) {
+  if (t1 == 0) {
+    local = g;
+    return 0;
+  }
+  const int before = (int)(((long long)g * t1) / total);
+  const int upto = (int)(((long long)(g + 1) * t1) / total);
+  if (upto > before) {
+    local = before;
+    return 1;
+  }
+  local = g - before;
+  return 0;
+}
+
+// Epilogue warp ew serves TMEM lane quadrant q = ew % 4; with 8 epilogue warps the
+// second warp of a quadrant takes the upper half of the columns.
 template <int BN, int EPI>
-__global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const GemmArgs args) {
-  using C = TcCfg<BN, EPI>;
+__device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, int q, int ew,
+                                             int lane, int mb, int nb, int M, float4* stg) {
+  const int row0 = mb * BM + q * 32;
+  if constexpr (EPI == EPI_STORE_F32) {
+    epi_store_f32<BN>(a, tbase, row0, M, nb, stg);
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    epi_swiglu(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_SILU) {
+    epi_silu<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_LAYER_OUT) {
+    epi_layer_out<BN, BN>(a, tbase, row0, M, nb, 0, stg);
+  } else {
+    epi_layer_out<BN, BN / 2>(a, tbase, row0, M, nb, (ew >> 2) * (BN / 2), stg);
+  }
+}
+
+template <int BN, int EPI0, int EPI1>
+__global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+              const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+              const GemmArgs a0, const GemmArgs a1) {
+  using C = TcCfg<BN, epi_warps<EPI0>()>;
+  constexpr bool kGrouped = EPI1 != EPI_NONE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -221,19 +298,15 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
   const uint32_t smem_base = smem_u32(smem);
   auto sA = [&](int s) { return smem_base + s * C::STAGE_BYTES; };
   auto sB = [&](int s) { return smem_base + s * C::STAGE_BYTES + C::A_BYTES; };
+  uint32_t* err = a0.err;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  int M = args.m_dev ? *args.m_dev : args.m_static;
-  if (M < 0 || M > args.m_max) {
-    if (threadIdx.x == 0) atomicOr(args.err, ERR_BAD_INDEX);
-    M = 0;
-  }
-  const int m_tiles = (M + BM - 1) / BM;
-  const int n_tiles = (args.N + BN - 1) / BN;
-  const int total = m_tiles * n_tiles;
-  const int kblocks = (args.K + BK - 1) / BK;
+  const ProbSize P0 = prob_size<BN>(a0);
+  ProbSize P1{0, 0, 0, 0, 0};
+  if constexpr (kGrouped) P1 = prob_size<BN>(a1);
+  const int total = P0.tiles + P1.tiles;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -260,23 +333,32 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
     if (lane == 0 && total > 0) {
-      tma_prefetch_desc(&tmA);
-      tma_prefetch_desc(&tmB);
+      tma_prefetch_desc(&tmA0);
+      tma_prefetch_desc(&tmB0);
+      if constexpr (kGrouped) {
+        tma_prefetch_desc(&tmA1);
+        tma_prefetch_desc(&tmB1);
+      }
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, last_par = 0;  // per-stage bit masks for the drain
       bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
+        int local;
+        const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb;
-        tile_coords(tile, m_tiles, n_tiles, mb, nb);
+        tile_coords(local, pr ? P1.m_tiles : P0.m_tiles, pr ? P1.n_tiles : P0.n_tiles, mb, nb);
+        const CUtensorMap* tA = pr ? &tmA1 : &tmA0;
+        const CUtensorMap* tB = pr ? &tmB1 : &tmB0;
+        const int kblocks = pr ? P1.kblocks : P0.kblocks;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitLimitNs) || misc[1]) {
             ok = false;
             break;
           }
           mbar_arrive_expect_tx(full_bar(stage), C::STAGE_BYTES);
-          tma_load_2d(sA(stage), &tmA, kb * BK, mb * BM, full_bar(stage));
-          tma_load_2d(sB(stage), &tmB, kb * BK, nb * BN, full_bar(stage));
+          tma_load_2d(sA(stage), tA, kb * BK, mb * BM, full_bar(stage));
+          tma_load_2d(sB(stage), tB, kb * BK, nb * BN, full_bar(stage));
           issued |= 1u << stage;
           last_par = (last_par & ~(1u << stage)) | (phase << stage);
           if (++stage == C::STAGES) {
@@ -287,7 +369,7 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
       }
       if (!ok) {
         misc[1] = 1;
-        atomicOr(args.err, ERR_WAIT_PRODUCER);
+        atomicOr(err, ERR_WAIT_PRODUCER);
         // let copies still in flight land before the CTA can exit
         for (int s = 0; s < C::STAGES; ++s)
           if (issued & (1u << s)) mbar_wait(full_bar(s), (last_par >> s) & 1u, 100000000ull);
@@ -301,7 +383,10 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
+        int local;
+        const int pr = split_tile(g, P1.tiles, total, local);
+        const int kblocks = pr ? P1.kblocks : P0.kblocks;
         if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, kWaitLimitNs) || misc[1]) {
           ok = false;
           break;
@@ -334,45 +419,42 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
       }
       if (!ok) {
         misc[1] = 1;
-        atomicOr(args.err, ERR_WAIT_MMA);
+        atomicOr(err, ERR_WAIT_MMA);
         umma_commit(drain_bar);  // completes once every issued MMA has finished
-        if (!mbar_wait(drain_bar, 0, 100000000ull)) atomicOr(args.err, ERR_WAIT_DRAIN);
+        if (!mbar_wait(drain_bar, 0, 100000000ull)) atomicOr(err, ERR_WAIT_DRAIN);
       }
     }
   } else {
     // ------------------------------ epilogue ------------------------------
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
     const int ew = warp - 2;  // epilogue warp index
-    const int c_begin = (ew >> 2) * C::EPI_COLS;  // second warp of a quadrant: upper columns
-    const int row = q * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    for (int g = blockIdx.x; g < total; g += gridDim.x) {
+      int local;
+      const int pr = split_tile(g, P1.tiles, total, local);
       int mb, nb;
-      tile_coords(tile, m_tiles, n_tiles, mb, nb);
+      tile_coords(local, pr ? P1.m_tiles : P0.m_tiles, pr ? P1.n_tiles : P0.n_tiles, mb, nb);
       bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) {
         if (lane == 0) {
           misc[1] = 1;
-          atomicOr(args.err, ERR_WAIT_EPILOGUE);
+          atomicOr(err, ERR_WAIT_EPILOGUE);
         }
         break;
       }
       tc_fence_after();
-      const int m = mb * BM + row;
-      const bool valid = m < M;
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + ew * (32 * 8);
-      if constexpr (EPI == EPI_STORE_F32) {
-        epi_store_f32<BN>(args, tbase, mb * BM + q * 32, M, nb, stg);
-      } else if constexpr (EPI == EPI_SWIGLU) {
-        epi_swiglu(args, tbase, m, valid, nb);
-      } else if constexpr (EPI == EPI_SILU) {
-        epi_silu<BN>(args, tbase, m, valid, nb);
+      if constexpr (kGrouped) {
+        if (pr)
+          run_epilogue<BN, EPI1>(a1, tbase, q, ew, lane, mb, nb, P1.M, stg);
+        else
+          run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, stg);
       } else {
-        epi_layer_out<BN, C::EPI_COLS>(args, tbase, mb * BM + q * 32, M, nb, c_begin, stg);
+        run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, stg);
       }
       tc_fence_before();
       __syncwarp();
@@ -390,21 +472,23 @@ __global__ void __launch_bounds__(TcCfg<BN, EPI>::THREADS, 1)
   }
 }
 
-template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& args,
-                       int num_sms, cudaStream_t st) {
-  using C = TcCfg<BN, EPI>;
+template <int BN, int EPI0, int EPI1>
+cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const GemmArgs& a0,
+                      const CUtensorMap& tmA1, const CUtensorMap& tmB1, const GemmArgs& a1,
+                      int num_sms, cudaStream_t st) {
+  using C = TcCfg<BN, epi_warps<EPI0>()>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI>,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI0, EPI1>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const long max_tiles = (long)((args.m_max + BM - 1) / BM) * ((args.N + BN - 1) / BN);
+  long max_tiles = (long)((a0.m_max + BM - 1) / BM) * ((a0.N + BN - 1) / BN);
+  if (EPI1 != EPI_NONE) max_tiles += (long)((a1.m_max + BM - 1) / BM) * ((a1.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
   const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
-  k_gemm_tc<BN, EPI><<<grid, C::THREADS, C::SMEM, st>>>(tmA, tmB, args);
+  k_gemm_tc<BN, EPI0, EPI1><<<grid, C::THREADS, C::SMEM, st>>>(tmA0, tmB0, tmA1, tmB1, a0, a1);
   return cudaGetLastError();
 }
 
@@ -412,16 +496,29 @@ cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const Gem
 
 cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
                            const GemmArgs& args, int num_sms, cudaStream_t st) {
-  if (bn == 256) {
-    switch (epi) {
-      case EPI_STORE_F32: return launch_one<256, EPI_STORE_F32>(tmA, tmB, args, num_sms, st);
-      case EPI_SWIGLU: return launch_one<256, EPI_SWIGLU>(tmA, tmB, args, num_sms, st);
-      case EPI_LAYER_OUT: return launch_one<256, EPI_LAYER_OUT>(tmA, tmB, args, num_sms, st);
-      default: break;
-    }
-  } else if (bn == 64 && epi == EPI_SILU) {
-    return launch_one<64, EPI_SILU>(tmA, tmB, args, num_sms, st);
+  if (bn != 256) return cudaErrorInvalidValue;
+  const GemmArgs none{};
+  switch (epi) {
+    case EPI_STORE_F32:
+      return launch_tc<256, EPI_STORE_F32, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_SWIGLU:
+      return launch_tc<256, EPI_SWIGLU, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_LAYER_OUT:
+      return launch_tc<256, EPI_LAYER_OUT, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_LAYER_OUT_WIDE:
+      return launch_tc<256, EPI_LAYER_OUT_WIDE, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms,
+                                                          st);
+    default:
+      return cudaErrorInvalidValue;
   }
+}
+
+cudaError_t launch_gemm_tc_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUtensorMap& tmB0,
+                                const GemmArgs& a0, EpiKind epi1, const CUtensorMap& tmA1,
+                                const CUtensorMap& tmB1, const GemmArgs& a1, int num_sms,
+                                cudaStream_t st) {
+  if (epi0 == EPI_SWIGLU && epi1 == EPI_SILU)
+    return launch_tc<256, EPI_SWIGLU, EPI_SILU>(tmA0, tmB0, a0, tmA1, tmB1, a1, num_sms, st);
   return cudaErrorInvalidValue;
 }
 

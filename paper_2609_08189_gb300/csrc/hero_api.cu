@@ -125,9 +125,6 @@ struct hero_model {
   cudaStream_t copy_stream = nullptr;
   std::vector<cudaEvent_t> ev_ready, ev_consumed;  // per routed block
   cudaEvent_t ev_start = nullptr;
-  // the adapter branch runs on a side stream, concurrently with the FFN branch
-  cudaStream_t side_stream = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
@@ -187,11 +184,12 @@ hero_status validate_config(const hero_config* c) {
   if (c->d_h % 4 || c->d_a % 4 || c->d_enc % 4 || c->d_head % 4 || c->d_path % 4)
     return fail(HERO_ERR_UNSUPPORTED, "router widths d_h, d_a, d_enc, d_head, d_path must be multiples of 4");
   if (c->d_model % 8 != 0) return fail(HERO_ERR_UNSUPPORTED, "d_model must be a multiple of 8");
-  if (c->d_r > 64) return fail(HERO_ERR_UNSUPPORTED, "d_r must be at most 64");
+  if (c->dtype == HERO_F32 && c->d_r > 64)
+    return fail(HERO_ERR_UNSUPPORTED, "f32 models need d_r <= 64");
   if (c->dtype == HERO_BF16) {
-    if (c->d_model % 256 != 0 || c->d_ff % 128 != 0 || c->d_r != 64)
+    if (c->d_model % 256 != 0 || c->d_ff % 128 != 0 || c->d_r % 32 != 0 || c->d_r > 4096)
       return fail(HERO_ERR_UNSUPPORTED,
-                  "bf16 needs d_model %% 256 == 0, d_ff %% 128 == 0 and d_r == 64");
+                  "bf16 needs d_model %% 256 == 0, d_ff %% 128 == 0 and d_r %% 32 == 0 (<= 4096)");
     if ((c->d_enc + c->d_head) % 8 != 0)
       return fail(HERO_ERR_UNSUPPORTED, "bf16 needs d_enc + d_head to be a multiple of 8");
   }
@@ -232,9 +230,6 @@ void free_model(hero_model* m) {
   for (auto e : m->ev_consumed) cudaEventDestroy(e);
   if (m->ev_start) cudaEventDestroy(m->ev_start);
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
-  if (m->ev_fork) cudaEventDestroy(m->ev_fork);
-  if (m->ev_join) cudaEventDestroy(m->ev_join);
-  if (m->side_stream) cudaStreamDestroy(m->side_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io};
   for (void* p : ptrs)
@@ -507,15 +502,12 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
            encode_bf16_2d(&m->tm_wd[j], static_cast<char*>(m->wdown) + (size_t)j * d * I * 2, I, d,
                           256) &&
            encode_bf16_2d(&m->tm_w1[j], static_cast<char*>(m->w1) + (size_t)j * r * d * 2, d, r,
-                          64) &&
+                          256) &&
            encode_bf16_2d(&m->tm_w2[j], static_cast<char*>(m->w2) + (size_t)j * d * r * 2, r, d,
                           256);
     }
     if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
   }
-  CUDA_M(cudaStreamCreateWithFlags(&m->side_stream, cudaStreamNonBlocking));
-  CUDA_M(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming));
-  CUDA_M(cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming));
   *out = m;
   return HERO_OK;
 #undef TRY_M
@@ -612,68 +604,75 @@ hero_status block_body(hero_model* m, int jj, int T, const BlockState& bs, const
               m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
   CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, st); }));
 
-  // FFN branch: gate/up + SwiGLU, then down + scaled scatter
-  {
-    GemmArgs g{};
-    g.m_dev = m->counts;
-    g.m_max = T;
-    g.N = m->bf16 ? 2 * I : I;
-    g.K = d;
-    g.out = m->act;
-    g.ldo = I;
-    g.err = m->err;
-    g.A = m->u_f;
-    g.lda = d;
-    g.B = static_cast<const char*>(m->wgu) + (size_t)jj * (m->bf16 ? 2 : 1) * I * d * es;
-    g.B2 = m->bf16 ? nullptr : static_cast<const char*>(m->wup) + (size_t)jj * I * d * es;
-    g.ldb = d;
+  // FFN branch: gate/up + SwiGLU, then down + scaled scatter.  The adapter branch
+  // (the other token rows): W_1 with SiLU, then W_2 + scaled scatter; on bf16
+  // models each adapter GEMM rides in the FFN GEMM's launch as a second problem.
+  GemmArgs gu{};
+  gu.m_dev = m->counts;
+  gu.m_max = T;
+  gu.N = m->bf16 ? 2 * I : I;
+  gu.K = d;
+  gu.out = m->act;
+  gu.ldo = I;
+  gu.err = m->err;
+  gu.A = m->u_f;
+  gu.lda = d;
+  gu.B = static_cast<const char*>(m->wgu) + (size_t)jj * (m->bf16 ? 2 : 1) * I * d * es;
+  gu.B2 = m->bf16 ? nullptr : static_cast<const char*>(m->wup) + (size_t)jj * I * d * es;
+  gu.ldb = d;
+  GemmArgs ad{};
+  ad.m_dev = m->counts + 1;
+  ad.m_max = T;
+  ad.N = r;
+  ad.K = d;
+  ad.out = m->ah;
+  ad.ldo = r;
+  ad.err = m->err;
+  ad.A = m->u_a;
+  ad.lda = d;
+  ad.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
+  ad.ldb = d;
+  GemmArgs dn{};
+  dn.m_dev = m->counts;
+  dn.m_max = T;
+  dn.N = d;
+  dn.K = I;
+  dn.err = m->err;
+  dn.lo = lo;
+  dn.lo.idx = m->idx_f;
+  dn.lo.scale = m->scale_f;
+  dn.A = m->act;
+  dn.lda = I;
+  dn.B = static_cast<const char*>(m->wdown) + (size_t)jj * d * I * es;
+  dn.ldb = I;
+  if (m->bf16) {
+    GemmArgs au{};   // adapter W_2: [n_a, d_r] x [d_r, d] with the closing epilogue
+    au.m_dev = m->counts + 1;
+    au.m_max = T;
+    au.N = d;
+    au.K = r;
+    au.err = m->err;
+    au.lo = lo;
+    au.lo.idx = m->idx_a;
+    au.lo.scale = m->scale_a;
     CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] {
-      return m->bf16 ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], g, m->num_sms, st)
-                     : launch_gemm_simt(EPI_SWIGLU, g, st);
+      return dense ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st)
+                   : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU, m->tm_ua,
+                                         m->tm_w1[jj], ad, m->num_sms, st);
     }));
-    // The adapter branch (disjoint token rows) may start now on the side stream and
-    // fill the SMs the FFN-down GEMM leaves idle in its last wave.
-    if (!dense && m->side_stream) {
-      CUDA_TRY(cudaEventRecord(m->ev_fork, st));
-      CUDA_TRY(cudaStreamWaitEvent(m->side_stream, m->ev_fork, 0));
-    }
-    GemmArgs g2{};
-    g2.m_dev = m->counts;
-    g2.m_max = T;
-    g2.N = d;
-    g2.K = I;
-    g2.err = m->err;
-    g2.lo = lo;
-    g2.lo.idx = m->idx_f;
-    g2.lo.scale = m->scale_f;
-    g2.A = m->act;
-    g2.lda = I;
-    g2.B = static_cast<const char*>(m->wdown) + (size_t)jj * d * I * es;
-    g2.ldb = I;
+    if (!dense)   // epilogue-bound (rank-d_r contraction): the wide-epilogue variant
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
+        return launch_gemm_tc(256, EPI_LAYER_OUT_WIDE, m->tm_ah, m->tm_w2[jj], au, m->num_sms, st);
+      }));
     CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
-      return m->bf16 ? launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], g2, m->num_sms, st)
-                     : launch_gemm_simt(EPI_LAYER_OUT, g2, st);
+      return launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dn, m->num_sms, st);
     }));
+    return HERO_OK;
   }
-  // adapter branch
+  CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] { return launch_gemm_simt(EPI_SWIGLU, gu, st); }));
+  CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] { return launch_gemm_simt(EPI_LAYER_OUT, dn, st); }));
   if (!dense) {
-    cudaStream_t sa = m->side_stream ? m->side_stream : st;
-    GemmArgs g{};
-    g.m_dev = m->counts + 1;
-    g.m_max = T;
-    g.N = r;
-    g.K = d;
-    g.out = m->ah;
-    g.ldo = r;
-    g.err = m->err;
-    g.A = m->u_a;
-    g.lda = d;
-    g.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
-    g.ldb = d;
-    CUDA_TRY(timed(m, HERO_K_ADAPTER_DOWN, sa, [&] {
-      return m->bf16 ? launch_gemm_tc(64, EPI_SILU, m->tm_ua, m->tm_w1[jj], g, m->num_sms, sa)
-                     : launch_gemm_simt(EPI_SILU, g, sa);
-    }));
+    CUDA_TRY(timed(m, HERO_K_ADAPTER_DOWN, st, [&] { return launch_gemm_simt(EPI_SILU, ad, st); }));
     AdapterUpArgs au{};
     au.m_dev = m->counts + 1;
     au.m_max = T;
@@ -681,16 +680,12 @@ hero_status block_body(hero_model* m, int jj, int T, const BlockState& bs, const
     au.d_r = r;
     au.ah = m->ah;
     au.w2 = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
-    au.bf16 = m->bf16;
-    au.slot_cols = m->bf16 ? kTcPartCols : kSimtTileN;
+    au.bf16 = 0;
+    au.slot_cols = kSimtTileN;
     au.lo = lo;
     au.lo.idx = m->idx_a;
     au.lo.scale = m->scale_a;
-    CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, sa, [&] { return launch_adapter_up(au, sa); }));
-    if (m->side_stream) {   // join: the next block reads every token's rows
-      CUDA_TRY(cudaEventRecord(m->ev_join, m->side_stream));
-      CUDA_TRY(cudaStreamWaitEvent(st, m->ev_join, 0));
-    }
+    CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] { return launch_adapter_up(au, st); }));
   }
   return HERO_OK;
 }

@@ -60,6 +60,8 @@ enum EpiKind : int {
   EPI_SWIGLU = 1,      // out[m, n] = SiLU(gate) * up   (gate/up column pairs)
   EPI_SILU = 2,        // out[m, n] = SiLU(acc)
   EPI_LAYER_OUT = 3,   // LayerOutArgs
+  EPI_LAYER_OUT_WIDE = 4,  // the same with twice the epilogue warps, for launches whose
+                           // time is the epilogue's (the adapter's rank-d_r up projection)
 };
 
 struct GemmArgs {
@@ -81,18 +83,29 @@ struct GemmArgs {
 };
 
 // Tensor-core GEMM (tcgen05 + TMA + TMEM), bf16 operands, fp32 accumulation.
-// A: [rows, K] K-major; B: [N, K] K-major.  BN = 256 (STORE/SWIGLU/LAYER_OUT) or
-// 64 (SILU, the adapter's rank-64 projection).
+// A: [rows, K] K-major; B: [N, K] K-major; 128 x 256 tiles (bn must be 256).
 cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
                            const GemmArgs& args, int num_sms, cudaStream_t st);
+
+// Grouped launch of two independent problems in one persistent kernel, the second
+// problem's tiles spread evenly among the first's: (SWIGLU, SILU) = FFN gate/up
+// with the adapter's down projection (disjoint rows).  The SILU problem's N (the
+// adapter rank) must be a multiple of 32; a narrower-than-tile B is zero-filled
+// by TMA.  (The block-closing pair, FFN down with the adapter's up projection, is
+// not grouped: an adapter tile holds one of the two TMEM accumulators for a whole
+// epilogue while its MMA takes under a microsecond, which stalls the FFN's MMA.)
+cudaError_t launch_gemm_tc_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUtensorMap& tmB0,
+                                const GemmArgs& a0, EpiKind epi1, const CUtensorMap& tmA1,
+                                const CUtensorMap& tmB1, const GemmArgs& a1, int num_sms,
+                                cudaStream_t st);
 
 // SIMT fp32 GEMM with the same epilogues (f32 models).
 cudaError_t launch_gemm_simt(EpiKind epi, const GemmArgs& args, cudaStream_t st);
 constexpr int kSimtTileN = 64;
 
 // Columns per partial-sum slot of the block-closing epilogues: bf16 models (tensor
-// core path) use the 256-column tile, f32 models the SIMT tile width.
-constexpr int kTcPartCols = 256;
+// core path) use half a 256-column tile, f32 models the SIMT tile width.
+constexpr int kTcPartCols = 128;
 
 // Router and bookkeeping kernels ------------------------------------------------
 
