@@ -48,7 +48,9 @@ def load_peaks():
 
 
 def workload_desc(cfg, bypass):
-    return (f"{cfg.name}: {cfg.n_layers} routed blocks, d={cfg.d_model}, I={cfg.d_ff}, "
+    blocks = (f"{cfg.n_layers} routed blocks" if not cfg.n_dense else
+              f"{cfg.n_dense} dense + {cfg.n_layers - cfg.n_dense} routed blocks")
+    return (f"{cfg.name}: {blocks}, d={cfg.d_model}, I={cfg.d_ff}, "
             f"d_r={cfg.d_r}, d_m={cfg.d_m}, T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len}), "
             f"{cfg.dtype}, bypass target {bypass:.2%}, random-init weights, seeded inputs")
 
@@ -124,7 +126,8 @@ def algorithmic_work(cfg, counts_per_step, steps, routed=True):
     work = {
         "ffn_gate_up": steps * float(np.sum(2.0 * nf * 2 * I * d)),
         "ffn_down": steps * float(np.sum(2.0 * nf * I * d)),
-        "router_gemm": steps * float(cfg.n_layers * 2.0 * T * nY * k_r) if routed else 0.0,
+        "router_gemm": steps * float((cfg.n_layers - cfg.n_dense) * 2.0 * T * nY * k_r)
+        if routed else 0.0,
         "adapter_down": steps * float(np.sum(2.0 * na * r * d)),
         "adapter_up": steps * float(np.sum(2.0 * na * d * r)),
     }
@@ -265,7 +268,7 @@ def main():
     prof = hero.hero_get_profile(stack.model, reset=True)
     stack.check()
     counts = c.cpu().numpy().astype(np.int64)
-    bypass = 1.0 - counts.sum() / (L * T)
+    bypass = 1.0 - counts[cfg.n_dense:].sum() / ((L - cfg.n_dense) * T)   # routed blocks
     value = world * T * args.steps / (ms / 1e3)
 
     # ---- dense stack, same kernels ----

@@ -52,7 +52,8 @@ typedef enum {
 typedef enum { HERO_F32 = 0, HERO_BF16 = 1 } hero_dtype;
 
 /* Shapes and constants of one routed FFN stack.
- *   n_layers   L_R, routed blocks (Sec. 3.1)
+ *   n_layers   FFN layers of the stack; the last n_layers - n_dense are the routed
+ *              blocks j = 1..L_R (Sec. 3.1)
  *   d_model    d, hidden width; d_ff = I, SwiGLU intermediate width
  *   d_r        adapter rank (W_1: d_r x d, W_2: d x d_r; Eq. 2)
  *   d_m        memory width (q, k, v in R^{d_m}; S is d_m x d_m per token; Sec. 3.2)
@@ -74,6 +75,9 @@ typedef struct {
   int32_t max_tokens;
   hero_dtype dtype;
   float rms_eps, eps, t_hist;
+  int32_t n_dense;   /* leading layers outside the routing candidate set (Sec. 4.1
+                        placement): plain FFN blocks, scale 1, router untouched;
+                        0 <= n_dense < n_layers, L_R = n_layers - n_dense */
 } hero_config;
 
 /* HOST pointers to the parameters, canonical [out, in] layouts, stacked over
@@ -164,8 +168,9 @@ typedef struct {
 hero_status hero_router_state_reset(hero_model* m, int64_t n_tokens, const hero_router_state* state,
                                     void* cuda_stream);
 
-/* Routed block `block` (j = 1..n_layers) on post-attention hidden states
- * h_bar [T,d] fp32 (Eq. 1).  Reads then updates `state` (read before write,
+/* Block `block` (1..n_layers) on post-attention hidden states h_bar [T,d] fp32
+ * (Eq. 1); blocks 1..n_dense are plain FFN blocks (state unused, may be NULL),
+ * block n_dense + j is routed block j.  Reads then updates `state` (read before write,
  * Eqs. 11-12) and writes h_out [T,d] = h_bar + g FFN(u) or h_bar + (1-g)
  * Adapter(u) (Eq. 3).  flags: HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK (mask_in [T]).
  * gate_out [T], mask_out [T], ffn_count_out [1] may be NULL.  h_out must not

@@ -52,6 +52,12 @@ Readings where the paper is silent (each listed in the design notes):
 Modes: "route" (the method), "force" (decisions taken from mask_in, g still
 computed and used as branch scale), "dense" (router skipped, every token through
 the FFN with scale 1: the dense SwiGLU stack).
+
+Placement (Sec. 4.1): only a candidate set of FFN layers is routed; the others
+stay dense.  With n_dense > 0 the first n_dense layers of the stack run the plain
+FFN block (scale 1, no router, router state untouched) and layers
+n_dense+1 .. n_layers are the routed blocks j = 1 .. L_R, L_R = n_layers - n_dense
+(the routed index j and L_R enter the path features, Eqs. 4 and 6).
 """
 
 from __future__ import annotations
@@ -139,11 +145,13 @@ class OracleConfig:
     eps: float = 1e-6
     t_hist: float = 0.9
     dtype: str = "f32"
+    n_dense: int = 0          # leading FFN layers outside the candidate set (dense)
 
     @staticmethod
     def from_stack(c) -> "OracleConfig":
         return OracleConfig(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a,
-                            c.d_enc, c.d_head, c.d_path, c.rms_eps, c.eps, c.t_hist, c.dtype)
+                            c.d_enc, c.d_head, c.d_path, c.rms_eps, c.eps, c.t_hist, c.dtype,
+                            getattr(c, "n_dense", 0))
 
 
 def _f64(a) -> np.ndarray:
@@ -262,7 +270,8 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     """Run the routed FFN stack on tokens h_in [T, d].
 
     attn_delta: [L, T, d] attention stand-in (None = zero).
-    mode: "route" | "force" (mask_in [L, T] gives decisions) | "dense".
+    mode: "route" | "force" (mask_in [L, T] gives decisions; rows of the dense
+    prefix are ignored) | "dense".
     branch_scale: "gate" (Eq. 3: g and 1 - g) or "one" (unscaled branches).
     Returns h_out [T, d], gate [L, T], mask [L, T] (uint8), counts [L] (FFN tokens)
     and, if record, per-layer intermediates under "layers".
@@ -275,6 +284,10 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     Rx = bf16_pair if cfg.dtype == "bf16" else _identity   # router activation operand
     hk = hooks or {}
     L = cfg.n_layers
+    n_dense = cfg.n_dense
+    if not 0 <= n_dense < L:
+        raise ValueError("need 0 <= n_dense < n_layers")
+    L_R = L - n_dense                                               # routed blocks
     h = _f64(h_in)
     T = h.shape[0]
     w = {k: _f64(weights[k]) for k in _SHARED_KEYS}
@@ -292,18 +305,20 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     counts = np.zeros(L, dtype=np.int64)
     layers: List[Dict[str, np.ndarray]] = []
 
-    for j in range(1, L + 1):
-        wl = {k: _f64(weights[k][j - 1]) for k in _LAYER_KEYS}
-        P = 0.0 if attn_delta is None else _f64(attn_delta[j - 1])
+    for layer in range(1, L + 1):
+        wl = {k: _f64(weights[k][layer - 1]) for k in _LAYER_KEYS}
+        P = 0.0 if attn_delta is None else _f64(attn_delta[layer - 1])
         h_bar = h + P                                               # Eq. 1 stand-in
         rec: Dict[str, np.ndarray] = {"h_bar": h_bar}
-        if mode == "dense":
+        j = layer - n_dense                                         # routed index (Sec. 4.1)
+        dense_layer = mode == "dense" or j < 1
+        if dense_layer:
             g = np.ones(T)
             decide = np.ones(T, dtype=bool)
         else:
             delta, d, gamma = transition_features(j, h_bar, h_bar_prev, delta_prev,
                                                   d_prev, cfg.eps)
-            x_path = path_vector(j, L, d, gamma, p_prev, m_prev)
+            x_path = path_vector(j, L_R, d, gamma, p_prev, m_prev)
             z_h = hidden_encoder(h_bar, w, cfg, R, Rx)
             z_a = path_encoder(x_path, w)
             s = np.concatenate([z_h, z_a], axis=1)                 # Eq. 9
@@ -319,12 +334,12 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             m = m_prev * p                                          # Eq. 15
             b = local_head(h_bar, w, Rx)                            # Eq. 16
             g = sigmoid(a + b)
-            rho = sigmoid(eta[j - 1])
+            rho = sigmoid(eta[layer - 1])
             S, zeta = memory_write(S, zeta, fk, v, rho)             # Eq. 12
             if mode == "route":
                 decide = g >= tau                                   # Eq. 3 threshold
             else:
-                decide = np.asarray(mask_in[j - 1]).astype(bool)
+                decide = np.asarray(mask_in[layer - 1]).astype(bool)
             if record:
                 rec.update(delta=delta, d=d, gamma=gamma, x_path=x_path, z_h=z_h, z_a=z_a,
                            s=s, q=q, k=k, v=v, c=c, nu=nu, a=a, b=b, p=p, m=m,
@@ -333,7 +348,7 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             p_prev, m_prev = p, m
 
         u = R(rms_norm(h_bar, wl["ffn_norm_g"], cfg.rms_eps))       # Eq. 1, u = LN_ffn(h_bar)
-        if mode == "dense" or branch_scale == "one":
+        if dense_layer or branch_scale == "one":
             sf = np.ones(T)
             sa = np.ones(T)
         else:
@@ -345,9 +360,9 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             h_new[F] += sf[F, None] * swiglu_ffn(u[F], wl, R)       # Eq. 3, g >= tau
         if A.size:
             h_new[A] += sa[A, None] * adapter(u[A], wl, R)          # Eq. 3, g < tau
-        gates[j - 1] = g
-        masks[j - 1] = decide.astype(np.uint8)
-        counts[j - 1] = F.size
+        gates[layer - 1] = g
+        masks[layer - 1] = decide.astype(np.uint8)
+        counts[layer - 1] = F.size
         if record:
             rec.update(g=g, mask=decide.copy(), u=u, h=h_new)
             layers.append(rec)
@@ -359,7 +374,8 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     return out
 
 
-def bypass_fraction(masks: np.ndarray) -> float:
-    """Share of FFN executions replaced by the adapter: sum_j n_a,j / (L_R T)."""
-    m = np.asarray(masks)
+def bypass_fraction(masks: np.ndarray, n_dense: int = 0) -> float:
+    """Share of the routed blocks' FFN executions replaced by the adapter:
+    sum_j n_a,j / (L_R T), over the routed blocks only (rows n_dense.. of masks)."""
+    m = np.asarray(masks)[n_dense:]
     return float(1.0 - m.mean()) if m.size else 0.0

@@ -175,6 +175,8 @@ hero_status validate_config(const hero_config* c) {
       c->d_a < 1 || c->d_enc < 1 || c->d_head < 1 || c->d_path < 1 || c->max_tokens < 1)
     return fail(HERO_ERR_ARG, "config has a non-positive dimension");
   if (c->dtype != HERO_F32 && c->dtype != HERO_BF16) return fail(HERO_ERR_ARG, "unknown dtype");
+  if (c->n_dense < 0 || c->n_dense >= c->n_layers)
+    return fail(HERO_ERR_ARG, "need 0 <= n_dense < n_layers (got %d)", c->n_dense);
   if (!(c->rms_eps >= 0.f) || !(c->eps >= 0.f) || !(c->t_hist > 0.f))
     return fail(HERO_ERR_ARG, "eps must be >= 0 and t_hist > 0");
   if (c->d_m != 16 && c->d_m != 32 && c->d_m != 64 && c->d_m != 128)
@@ -534,17 +536,18 @@ struct BlockState {
   float *S, *zeta, *pst, *mst, *dprev;
 };
 
-// Everything of routed block jj after its entry (h_bar, its operand copy and the
-// partial sums are in place): router contraction and router, compaction, LN_ffn,
-// FFN and adapter branches with the block-closing epilogue `lo`.
-hero_status block_body(hero_model* m, int jj, int T, const BlockState& bs, const float* hbar,
+// Everything of block jj (layer index; routed index jr = jj - n_dense) after its
+// entry (h_bar, its operand copy and the partial sums are in place): router
+// contraction and router, compaction, LN_ffn, FFN and adapter branches with the
+// block-closing epilogue `lo`.  HERO_FLAG_DENSE in flags runs the plain FFN block.
+hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& bs, const float* hbar,
                        const LayerOutArgs& lo, float tau, uint32_t flags, const uint8_t* mask_in_j,
                        float* gate_out_j, uint8_t* mask_out_j, int32_t* count_out_j,
                        cudaStream_t st) {
   const hero_config& c = m->cfg;
   const int L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r;
   const int nY = c.d_enc + c.d_head;
-  const int j = jj + 1;
+  const int j = jr + 1;                 // routed index (layer jj = n_dense + jr)
   const bool dense = flags & HERO_FLAG_DENSE;
   const size_t es = m->esz;
   if (!dense) {
@@ -568,7 +571,7 @@ hero_status block_body(hero_model* m, int jj, int T, const BlockState& bs, const
     RouterArgs ra{};
     ra.T = T;
     ra.j = j;
-    ra.L = L;
+    ra.L = L - c.n_dense;               // L_R
     ra.np = m->np;
     ra.d = d;
     ra.d_h = c.d_h;
@@ -756,6 +759,9 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
     }
     if (feed && jj + 1 < L) CUDA_TRY(cudaStreamWaitEvent(st, m->ev_ready[jj + 1], 0));
     BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
+    // layers before the routing candidate set run the plain FFN block
+    const int jr = jj - c.n_dense;
+    const bool dense_blk = dense || jr < 0;
     LayerOutArgs lo{};
     lo.hbar = m->hbar;
     lo.delta = m->delta;
@@ -767,11 +773,13 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
     lo.np = m->np;
     lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
     lo.last = jj == L - 1;
-    lo.first = jj == 0;
+    lo.first = jr <= 0;                       // delta_1 = 0; no delta before routing starts
     lo.p_bf16 = m->bf16;
     lo.xl_bf16 = m->bf16;
-    lo.router = dense ? 0 : 1;
-    hero_status sb = block_body(m, jj, T, bs, m->hbar, lo, tau, flags,
+    lo.router = (!dense && jr + 1 >= 0) ? 1 : 0;   // the next block is routed
+    hero_status sb = block_body(m, jj, jr, T, bs, m->hbar, lo, tau,
+                                dense_blk ? (flags & ~(uint32_t)HERO_FLAG_FORCE_MASK) | HERO_FLAG_DENSE
+                                          : flags,
                                 force ? mask_in + (size_t)jj * T : nullptr,
                                 gate_out ? gate_out + (size_t)jj * T : nullptr,
                                 mask_out ? mask_out + (size_t)jj * T : nullptr,
@@ -909,7 +917,7 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
     return fail(HERO_ERR_ARG, "hero_routed_block takes only HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK");
   if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
     return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
-  const bool dense = flags & HERO_FLAG_DENSE;
+  bool dense = (flags & HERO_FLAG_DENSE) || block <= c.n_dense;
   if (!std::isfinite(tau_exec)) return fail(HERO_ERR_ARG, "tau_exec is not finite");
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   if (n_tokens == 0) {
@@ -925,8 +933,12 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
                  !s->h_bar_prev || !s->delta_prev))
     return fail(HERO_ERR_ARG, "the router state needs all seven pointers");
   CUDA_TRY(cudaSetDevice(m->device));
-  const int T = (int)n_tokens, jj = block - 1;
-  BlockEntryArgs be{T, c.d_model, m->np, block, dense ? 0 : 1, h_bar,
+  const int T = (int)n_tokens, jj = block - 1, jr = jj - c.n_dense;
+  if (jr < 0) {   // outside the routing candidate set: the plain FFN block
+    dense = true;
+    flags = (flags & ~(uint32_t)HERO_FLAG_FORCE_MASK) | HERO_FLAG_DENSE;
+  }
+  BlockEntryArgs be{T, c.d_model, m->np, jr + 1, dense ? 0 : 1, h_bar,
                     dense ? nullptr : s->h_bar_prev, dense ? nullptr : s->delta_prev,
                     m->xl, (int)m->bf16, m->part};
   CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
@@ -940,11 +952,11 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
   lo.np = m->np;
   lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
   lo.last = 1;
-  lo.first = jj == 0;
+  lo.first = jr <= 0;
   lo.p_bf16 = m->bf16;
   lo.xl_bf16 = m->bf16;
   lo.router = 0;
-  return block_body(m, jj, T, bs, h_bar, lo, tau_exec, flags,
+  return block_body(m, jj, jr, T, bs, h_bar, lo, tau_exec, flags,
                     (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr, gate_out, mask_out,
                     ffn_count_out, st);
 }

@@ -493,42 +493,33 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
 }
 
 // ------------------------------------------------------------------------------
-// k_compact: one CTA; stable exclusive scan of the decisions, chunks of 16384.
+// k_compact: one CTA; stable exclusive scan of the decisions in chunks of
+// CT * SEGS tokens.  A warp owns SEGS consecutive 32-token segments: one ballot
+// per segment gives its FFN count (pass 1, then a block scan of the warp totals)
+// and each lane's rank inside the segment (pass 2), so every load and every
+// index write of a segment is one coalesced warp access.
 // ------------------------------------------------------------------------------
-constexpr int CT = 1024, CPT = 16;
+constexpr int CT = 1024, SEGS = 16;
 
 __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
   __shared__ int wsum[CT / 32];
   __shared__ int carry_s;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t lt_mask = (1u << lane) - 1u;
   if (tid == 0) carry_s = 0;
   __syncthreads();
-  for (int base = 0; base < a.T; base += CT * CPT) {
-    uint8_t f[CPT];
-    int cnt = 0;
-    const int tb = base + tid * CPT;
-    if (!a.dense && tb + CPT <= a.T) {   // 16 flags in one 16-byte load (tb is 16-aligned)
-      const uint4 u = *reinterpret_cast<const uint4*>(a.mask + tb);
-      const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+  for (int base = 0; base < a.T; base += CT * SEGS) {
+    const int wbase = base + warp * 32 * SEGS;
+    uint32_t bal[SEGS];
+    int wtot = 0;
 #pragma unroll
-      for (int i = 0; i < CPT; ++i) f[i] = ((w4[i >> 2] >> (8 * (i & 3))) & 0xffu) ? 1 : 0;
-    } else {
-#pragma unroll
-      for (int i = 0; i < CPT; ++i) {
-        const int t = tb + i;
-        f[i] = (t < a.T) ? (a.dense ? 1 : (a.mask[t] ? 1 : 0)) : 2;
-      }
+    for (int sg = 0; sg < SEGS; ++sg) {
+      const int t = wbase + sg * 32 + lane;
+      const bool f = t < a.T && (a.dense || a.mask[t] != 0);
+      bal[sg] = __ballot_sync(0xffffffffu, f);
+      wtot += __popc(bal[sg]);
     }
-#pragma unroll
-    for (int i = 0; i < CPT; ++i) cnt += f[i] == 1;
-    // inclusive warp scan of the per-thread counts
-    int x = cnt;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, x, o);
-      if (lane >= o) x += y;
-    }
-    if (lane == 31) wsum[warp] = x;
+    if (lane == 0) wsum[warp] = wtot;
     __syncthreads();
     if (warp == 0) {
       int w = wsum[lane];
@@ -541,25 +532,27 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
     }
     __syncthreads();
     const int carry = carry_s;
-    int pos_f = carry + (warp ? wsum[warp - 1] : 0) + x - cnt;  // exclusive
-    int t = tb;
-    int pos_a = t - pos_f;  // tokens before t that went to the adapter
+    int pos0 = carry + (warp ? wsum[warp - 1] : 0);   // FFN tokens before this warp's tokens
 #pragma unroll
-    for (int i = 0; i < CPT; ++i, ++t) {
-      if (f[i] == 2) break;
-      if (f[i]) {
-        a.idx_f[pos_f] = t;
-        a.scale_f[pos_f] = a.dense ? 1.f : a.gate[t];
-        ++pos_f;
-      } else {
-        a.idx_a[pos_a] = t;
-        a.scale_a[pos_a] = 1.f - a.gate[t];
-        ++pos_a;
+    for (int sg = 0; sg < SEGS; ++sg) {
+      const int t = wbase + sg * 32 + lane;
+      if (t < a.T) {
+        const bool f = (bal[sg] >> lane) & 1u;
+        const int pf = pos0 + __popc(bal[sg] & lt_mask);
+        if (f) {
+          a.idx_f[pf] = t;
+          a.scale_f[pf] = a.dense ? 1.f : a.gate[t];
+        } else {
+          const int pa = t - pf;   // tokens before t that went to the adapter
+          a.idx_a[pa] = t;
+          a.scale_a[pa] = 1.f - a.gate[t];
+        }
+        if (a.dense) {
+          if (a.gate_out) a.gate_out[t] = 1.f;
+          if (a.mask_out) a.mask_out[t] = 1;
+        }
       }
-      if (a.dense) {
-        if (a.gate_out) a.gate_out[t] = 1.f;
-        if (a.mask_out) a.mask_out[t] = 1;
-      }
+      pos0 += __popc(bal[sg]);
     }
     __syncthreads();
     if (tid == 0) carry_s = carry + wsum[CT / 32 - 1];

@@ -37,7 +37,7 @@ class hero_config(ctypes.Structure):
                 ("n_layers", "d_model", "d_ff", "d_r", "d_m", "d_h", "d_a", "d_enc", "d_head",
                  "d_path", "max_tokens")] + \
                [("dtype", ctypes.c_int), ("rms_eps", ctypes.c_float), ("eps", ctypes.c_float),
-                ("t_hist", ctypes.c_float)]
+                ("t_hist", ctypes.c_float), ("n_dense", ctypes.c_int32)]
 
 
 class hero_weights_host(ctypes.Structure):
@@ -112,7 +112,8 @@ def make_config(stack_cfg, max_tokens: Optional[int] = None) -> hero_config:
     c = stack_cfg
     return hero_config(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a, c.d_enc,
                        c.d_head, c.d_path, max_tokens or c.n_tokens,
-                       HERO_BF16 if c.dtype == "bf16" else HERO_F32, c.rms_eps, c.eps, c.t_hist)
+                       HERO_BF16 if c.dtype == "bf16" else HERO_F32, c.rms_eps, c.eps, c.t_hist,
+                       getattr(c, "n_dense", 0))
 
 
 def make_weights(weights: Dict[str, np.ndarray]):

@@ -30,7 +30,7 @@ TAU_FILE = os.path.join(os.path.dirname(os.path.abspath(__file__)), "tau.json")
 
 def _bypass(cfg, w, h, P, tau):
     r = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, tau)
-    return ho.bypass_fraction(r["mask"]), r
+    return ho.bypass_fraction(r["mask"], cfg.n_dense), r
 
 
 def calibrate(cfg, target, sample, iters=14):
@@ -39,7 +39,7 @@ def calibrate(cfg, target, sample, iters=14):
     idx = hi.sample_tokens(cfg.n_tokens, sample)
     h = hi.generate_h_in(cfg)[idx]
     P = hi.generate_attn_delta(cfg)[:, idx]
-    n_dec = cfg.n_layers * len(idx)
+    n_dec = (cfg.n_layers - cfg.n_dense) * len(idx)     # routed decisions
     if target <= 0.0:
         return {"tau": 0.0, "bypass": 0.0, "sample": int(len(idx)), "decisions": n_dec}
     lo, hi_ = 0.0, 1.0        # bypass(lo) = 0 (every g >= 0), bypass(hi) = 1

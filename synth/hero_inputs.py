@@ -63,6 +63,7 @@ class StackConfig:
     seed: int = 0
     batch: int = 1         # sequences (for reporting only; tokens are independent)
     seq_len: int = 0
+    n_dense: int = 0       # leading FFN layers outside the routing candidate set (Sec. 4.1)
 
     @property
     def d_s(self) -> int:
@@ -89,6 +90,17 @@ CONFIGS: Dict[str, StackConfig] = {
     # plus ragged tails, small enough that the oracle covers every token in seconds.
     "small_bf16": StackConfig("small_bf16", 4, 512, 1024, 64, 64, 333, "bf16", 0.27,
                               batch=1, seq_len=333),
+    # The paper's placement (Sec. 4.1): candidates are the latter half of the layers,
+    # the adapter has d_r = 896, and the 25% budget is of all parameters of
+    # Llama-3.1-8B (8.03e9): 0.25 * 8.03e9 / (16 * (3 d I - 2 d d_r)) = 74.3% of the
+    # routed blocks' executions take the adapter.
+    "llama31_8b_paper": StackConfig("llama31_8b_paper", 32, 4096, 14336, 896, 64, 16384, "bf16",
+                                    0.7432, batch=4, seq_len=4096, n_dense=16),
+    # The same placement at small shapes for full-token parity: a dense prefix, and an
+    # adapter rank that is not a multiple of 64 (a ragged K tail in the tensor-core
+    # up projection, a partial N tile in the down projection).
+    "small_bf16_placed": StackConfig("small_bf16_placed", 4, 512, 1024, 96, 64, 333, "bf16",
+                                     0.5, batch=1, seq_len=333, n_dense=2),
 }
 
 # The 13B workload is swept over these bypass targets.

@@ -31,7 +31,7 @@ from synth import hero_inputs as hi  # noqa: E402
 OUT = os.path.join(os.path.dirname(os.path.abspath(__file__)), "gate_sensitivity.json")
 # tokens per workload: the sample sizes of the full-size sampled GPU tests
 SAMPLE = {"small_bf16": 32, "llama2_7b_prefill": 64, "llama31_8b_prefill": 64,
-          "llama31_8b_decode": 64, "llama2_13b_prefill": 32}
+          "llama31_8b_decode": 64, "llama2_13b_prefill": 32, "llama31_8b_paper": 32}
 EPS = (1e-7, 3e-7, 1e-6)
 
 

@@ -61,7 +61,7 @@ def test_gemm_building_block(hero, M, N, K):
 # full-token parity on small workloads
 # ------------------------------------------------------------------------------
 
-@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16", "small_bf16_placed"])
 def test_free_running(hero, name):
     inp = pr.inputs(name)
     st = _stack(hero, inp)
@@ -71,12 +71,12 @@ def test_free_running(hero, name):
     print(name, rep)
     _assert_free(rep, pr.H_TOL[inp.cfg.dtype])
     np.testing.assert_array_equal(gpu.counts, gpu.mask.sum(axis=1))
-    bypass = 1 - gpu.mask.mean()
+    bypass = 1 - gpu.mask[inp.cfg.n_dense:].mean()          # routed blocks only
     assert abs(bypass - inp.cfg.bypass) < 0.03
     st.close()
 
 
-@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16", "small_bf16_placed"])
 def test_forced_mask(hero, name):
     inp = pr.inputs(name)
     st = _stack(hero, inp)
@@ -90,7 +90,7 @@ def test_forced_mask(hero, name):
     st.close()
 
 
-@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16"])
+@pytest.mark.parametrize("name", ["tiny_f32", "small_bf16", "small_bf16_placed"])
 def test_dense(hero, name):
     inp = pr.inputs(name)
     st = _stack(hero, inp)
@@ -180,7 +180,8 @@ def test_host_io_matches_device_path(hero):
 # ------------------------------------------------------------------------------
 
 FULL = [("llama2_7b_prefill", None, 64), ("llama31_8b_prefill", None, 64),
-        ("llama31_8b_decode", None, 64), ("llama2_13b_prefill", 0.27, 32)]
+        ("llama31_8b_decode", None, 64), ("llama2_13b_prefill", 0.27, 32),
+        ("llama31_8b_paper", None, 32)]
 
 
 @pytest.mark.parametrize("name,bypass,n_sample", FULL)
@@ -199,7 +200,8 @@ def test_full_size_sampled(hero, name, bypass, n_sample):
     # whole-workload properties: counts agree with decisions, bypass near the budget
     np.testing.assert_array_equal(gpu_all.counts, gpu_all.mask.sum(axis=1))
     target = cfg.bypass if bypass is None else bypass
-    assert abs((1 - gpu_all.mask.mean()) - target) < 0.05
+    assert (gpu_all.mask[:cfg.n_dense] == 1).all()           # dense prefix (placement)
+    assert abs((1 - gpu_all.mask[cfg.n_dense:].mean()) - target) < 0.05
     # forced mode on the sample: the GPU follows the oracle's decisions
     mask_in = gpu_all.mask.copy()
     mask_in[:, rows] = ref["mask"]

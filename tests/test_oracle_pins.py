@@ -411,9 +411,12 @@ def test_p7_budget_tiny():
 # P8: independent per-token, per-element pure-Python restatement (tiny shapes)
 # ---------------------------------------------------------------------------
 
-def _py_stack(cfg, W, h_in, P, tau):
-    """Per-token loops over scalars, written from Sec. 3 without numpy linear algebra."""
+def _py_stack(cfg, W, h_in, P, tau, n_dense=0):
+    """Per-token loops over scalars, written from Sec. 3 without numpy linear algebra.
+    The first n_dense layers are plain FFN blocks (Sec. 4.1 placement); the rest are
+    routed blocks j = 1 .. L - n_dense."""
     L, d = cfg.n_layers, cfg.d_model
+    LR = L - n_dense
 
     def mv(M, x):
         return [sum(M[o][i] * x[i] for i in range(len(x))) for o in range(len(M))]
@@ -437,8 +440,17 @@ def _py_stack(cfg, W, h_in, P, tau):
         hb_prev = dl_prev = None
         d_prev = 0.0
         gs = []
-        for j in range(1, L + 1):
-            hb = [h[i] + P[j - 1][t][i] for i in range(d)]
+        for layer in range(1, L + 1):
+            hb = [h[i] + P[layer - 1][t][i] for i in range(d)]
+            if layer <= n_dense:
+                rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+                u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
+                gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
+                y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
+                h = [hb[i] + y[i] for i in range(d)]
+                gs.append(1.0)
+                continue
+            j = layer - n_dense
             if j == 1:
                 dl = [0.0] * d
             else:
@@ -450,7 +462,7 @@ def _py_stack(cfg, W, h_in, P, tau):
             rms = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
             nr = [hb[i] / rms * W["r_norm_g"][i] for i in range(d)]
             zh = mv(W["w_hu"], [sl(x) for x in mv(W["w_hd"], nr)])
-            xp = [j / L, (L - j) / L, dd, gam, p_prev, m_prev]
+            xp = [j / LR, (LR - j) / LR, dd, gam, p_prev, m_prev]
             hid = [sl(x + b) for x, b in zip(mv(W["path_w1"], xp), W["path_b1"])]
             za = [x + b for x, b in zip(mv(W["path_w2"], hid), W["path_b2"])]
             s = zh + za
@@ -472,19 +484,19 @@ def _py_stack(cfg, W, h_in, P, tau):
             hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], hb), W["ps_b1"])]
             bb = sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0]
             g = sg(a + bb)
-            rho = sg(W["eta"][j - 1])
+            rho = sg(W["eta"][layer - 1])
             for mm in range(dm):
                 for n in range(dm):
                     S[mm][n] = rho * S[mm][n] + fk[mm] * v[n]
                 Z[mm] = rho * Z[mm] + fk[mm]
             rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
-            u = [hb[i] / rf * W["ffn_norm_g"][j - 1][i] for i in range(d)]
+            u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
             if g >= tau:
-                gt, up = mv(W["w_gate"][j - 1], u), mv(W["w_up"][j - 1], u)
-                y = mv(W["w_down"][j - 1], [sl(x) * z for x, z in zip(gt, up)])
+                gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
+                y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
                 h = [hb[i] + g * y[i] for i in range(d)]
             else:
-                y = mv(W["ad_w2"][j - 1], [sl(x) for x in mv(W["ad_w1"][j - 1], u)])
+                y = mv(W["ad_w2"][layer - 1], [sl(x) for x in mv(W["ad_w1"][layer - 1], u)])
                 h = [hb[i] + (1 - g) * y[i] for i in range(d)]
             gs.append(g)
             hb_prev, dl_prev, d_prev, p_prev, m_prev = hb, dl, dd, p, m
@@ -506,6 +518,25 @@ def test_p8_loop_restatement_tiny_shapes():
     np.testing.assert_allclose(got["gate"], ref_g, rtol=0, atol=1e-12)
     np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
     assert 0 < got["mask"].sum() < got["mask"].size
+
+
+def test_p8_placement_dense_prefix_restatement():
+    """Sec. 4.1 placement: the first n_dense FFN layers stay dense, the candidate
+    layers after them are routed blocks j = 1 .. L_R with their own L_R."""
+    cfg = hi.StackConfig("micro", 5, 8, 12, 4, 4, 6, "f32", 0.3, d_h=3, d_a=2, d_enc=5,
+                         d_head=6, d_path=3, seed=12)
+    w, h, P = _inputs(cfg)
+    W = {k: hi.to_f64(v).tolist() for k, v in w.items()}
+    oc = ho.OracleConfig.from_stack(cfg)
+    oc.n_dense = 2
+    base = ho.routed_ffn_stack(oc, w, h, P, 0.0)
+    tau = float(np.median(base["gate"][2:]))
+    got = ho.routed_ffn_stack(oc, w, h, P, tau)
+    ref_h, ref_g = _py_stack(cfg, W, hi.to_f64(h).tolist(), hi.to_f64(P).tolist(), tau, n_dense=2)
+    np.testing.assert_allclose(got["gate"], ref_g, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
+    assert (got["mask"][:2] == 1).all() and 0 < got["mask"][2:].sum() < got["mask"][2:].size
+    assert ho.bypass_fraction(got["mask"], n_dense=2) == 1.0 - got["mask"][2:].mean()
 
 
 # ---------------------------------------------------------------------------
