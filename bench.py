@@ -50,9 +50,10 @@ def load_peaks():
 def workload_desc(cfg, bypass):
     blocks = (f"{cfg.n_layers} routed blocks" if not cfg.n_dense else
               f"{cfg.n_dense} dense + {cfg.n_layers - cfg.n_dense} routed blocks")
+    variant = f", router ablation bits {cfg.router_variant}" if cfg.router_variant else ""
     return (f"{cfg.name}: {blocks}, d={cfg.d_model}, I={cfg.d_ff}, "
             f"d_r={cfg.d_r}, d_m={cfg.d_m}, T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len}), "
-            f"{cfg.dtype}, bypass target {bypass:.2%}, random-init weights, seeded inputs")
+            f"{cfg.dtype}, bypass target {bypass:.2%}{variant}, random-init weights, seeded inputs")
 
 
 class ClockSampler:
@@ -182,6 +183,9 @@ def main():
     ap.add_argument("--tau", type=float, default=None)
     ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--layers", type=int, default=None)
+    ap.add_argument("--router-variant", type=int, default=0,
+                    help="Sec. 4.4 router ablation bits (1 history, 2 memread, 4 aux, 8 pos)")
+    ap.add_argument("--d-m", type=int, default=None, help="memory width override (ablation)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -209,6 +213,8 @@ def main():
     tau = hi.calibrated_tau(cfg.name) if args.tau is None else args.tau
     if args.tokens or args.layers:
         cfg = cfg.replace(n_tokens=args.tokens or cfg.n_tokens, n_layers=args.layers or cfg.n_layers)
+    if args.router_variant or args.d_m:   # ablations run with the workload's tau
+        cfg = cfg.replace(router_variant=args.router_variant, d_m=args.d_m or cfg.d_m)
     T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
     t_gen = time.time()
     w = hi.generate_weights(cfg)

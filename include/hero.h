@@ -66,7 +66,7 @@ typedef enum { HERO_F32 = 0, HERO_BF16 = 1 } hero_dtype;
  *              fp32 residual; HERO_F32: fp32 everywhere
  *   rms_eps    RMSNorm epsilon; eps: the epsilon of Eqs. 8, 11 and 13's cosine
  *   t_hist     history temperature T_hist (Eq. 14)
- * Supported: d_m in {16, 32, 64, 128}; d_s <= 128; d_enc, d_head <= 256;
+ * Supported: d_m in {16, 32, 64, 128, 256}; d_s <= 128; d_enc, d_head <= 256;
  * d_path <= 64.  bf16 additionally needs d % 256 == 0, d_ff % 128 == 0 and
  * d_r % 32 == 0 (d_r <= 4096); f32 needs d % 4 == 0 and d_r <= 64. */
 typedef struct {
@@ -78,7 +78,24 @@ typedef struct {
   int32_t n_dense;   /* leading layers outside the routing candidate set (Sec. 4.1
                         placement): plain FFN blocks, scale 1, router untouched;
                         0 <= n_dense < n_layers, L_R = n_layers - n_dense */
+  uint32_t router_variant;  /* 0 = HeRo; else HERO_ROUTER_* ablation bits */
 } hero_config;
+
+/* Router ablations of Sec. 4.4 (bits of hero_config.router_variant):
+ *   NO_HISTORY  g = sigma(b), the local logit alone (Eq. 16 without a); memory,
+ *               path features and f_theta are skipped and the router state is
+ *               left untouched
+ *   NO_MEMREAD  f_theta keeps s but sees c = 0 and nu = 0 (Eqs. 11, 13); the
+ *               memory S, zeta is neither read nor written
+ *   NO_AUX      no auxiliary path encoder: z_a = 0 in s (Eq. 9)
+ *   NO_POS      routing progress r, q_rem and transition d, gamma are zeroed in
+ *               x_path (Eqs. 4, 6); p_hist, m_hist remain */
+enum {
+  HERO_ROUTER_NO_HISTORY = 1u,
+  HERO_ROUTER_NO_MEMREAD = 2u,
+  HERO_ROUTER_NO_AUX = 4u,
+  HERO_ROUTER_NO_POS = 8u
+};
 
 /* HOST pointers to the parameters, canonical [out, in] layouts, stacked over
  * layers where marked [L, ...].  All arrays have element type host_dtype

@@ -53,6 +53,15 @@ Modes: "route" (the method), "force" (decisions taken from mask_in, g still
 computed and used as branch scale), "dense" (router skipped, every token through
 the FFN with scale 1: the dense SwiGLU stack).
 
+Router ablations (Sec. 4.4, component ablations), bits of `variant`:
+  NO_HISTORY  the history branch is removed: g = sigma(b), the local logit alone;
+              memory, path features and f_theta are not evaluated.
+  NO_MEMREAD  the history head keeps its inputs s but loses the memory: c = 0 and
+              nu = 0 enter f_theta; the memory is neither read nor written.
+  NO_AUX      the auxiliary path encoder is removed: z_a = 0, s = [z_h; 0].
+  NO_POS      the routing progress (r, q_rem) and residual transition (d, gamma)
+              features are removed from x_path (zeroed); p_hist, m_hist remain.
+
 Placement (Sec. 4.1): only a candidate set of FFN layers is routed; the others
 stay dense.  With n_dense > 0 the first n_dense layers of the stack run the plain
 FFN block (scale 1, no router, router state untouched) and layers
@@ -129,6 +138,10 @@ def _mlp2(x, w1, b1, w2, b2):
 # Configuration and parameters
 # ---------------------------------------------------------------------------
 
+# Router ablation bits (Sec. 4.4); the same values as the C ABI's HERO_ROUTER_*.
+NO_HISTORY, NO_MEMREAD, NO_AUX, NO_POS = 1, 2, 4, 8
+
+
 @dataclass
 class OracleConfig:
     n_layers: int
@@ -146,12 +159,13 @@ class OracleConfig:
     t_hist: float = 0.9
     dtype: str = "f32"
     n_dense: int = 0          # leading FFN layers outside the candidate set (dense)
+    variant: int = 0          # router ablation bits (NO_HISTORY | NO_MEMREAD | ...)
 
     @staticmethod
     def from_stack(c) -> "OracleConfig":
         return OracleConfig(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a,
                             c.d_enc, c.d_head, c.d_path, c.rms_eps, c.eps, c.t_hist, c.dtype,
-                            getattr(c, "n_dense", 0))
+                            getattr(c, "n_dense", 0), getattr(c, "router_variant", 0))
 
 
 def _f64(a) -> np.ndarray:
@@ -315,27 +329,45 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
         if dense_layer:
             g = np.ones(T)
             decide = np.ones(T, dtype=bool)
+        elif cfg.variant & NO_HISTORY:                              # ablation: local logit
+            b = local_head(h_bar, w, Rx)                            # Eq. 16
+            g = sigmoid(b)
+            if mode == "route":
+                decide = g >= tau
+            else:
+                decide = np.asarray(mask_in[layer - 1]).astype(bool)
+            if record:
+                rec.update(b=b)
         else:
             delta, d, gamma = transition_features(j, h_bar, h_bar_prev, delta_prev,
                                                   d_prev, cfg.eps)
             x_path = path_vector(j, L_R, d, gamma, p_prev, m_prev)
+            if cfg.variant & NO_POS:                                # ablation: no progress /
+                x_path[:, :4] = 0.0                                 # transition features
             z_h = hidden_encoder(h_bar, w, cfg, R, Rx)
             z_a = path_encoder(x_path, w)
+            if cfg.variant & NO_AUX:                                # ablation: no path encoder
+                z_a = np.zeros_like(z_a)
             s = np.concatenate([z_h, z_a], axis=1)                 # Eq. 9
             q = s @ w["w_q"].T                                      # Eq. 10
             k = s @ w["w_k"].T
             v = s @ w["w_v"].T
             fq = hk.get("phi", phi)(q)
             fk = hk.get("phi", phi)(k)
-            c = memory_read(fq, S, zeta, cfg.eps)                   # Eq. 11 (before write)
-            nu = history_dissimilarity(j, s, c, w, cfg.eps)         # Eq. 13
+            if cfg.variant & NO_MEMREAD:                            # ablation: no memory access
+                c = np.zeros((T, cfg.d_m))
+                nu = np.zeros(T)
+            else:
+                c = memory_read(fq, S, zeta, cfg.eps)               # Eq. 11 (before write)
+                nu = history_dissimilarity(j, s, c, w, cfg.eps)     # Eq. 13
             a = history_head(s, c, nu, w)                           # Eq. 14
             p = sigmoid(a / cfg.t_hist)
             m = m_prev * p                                          # Eq. 15
             b = local_head(h_bar, w, Rx)                            # Eq. 16
             g = sigmoid(a + b)
             rho = sigmoid(eta[layer - 1])
-            S, zeta = memory_write(S, zeta, fk, v, rho)             # Eq. 12
+            if not cfg.variant & NO_MEMREAD:
+                S, zeta = memory_write(S, zeta, fk, v, rho)         # Eq. 12
             if mode == "route":
                 decide = g >= tau                                   # Eq. 3 threshold
             else:

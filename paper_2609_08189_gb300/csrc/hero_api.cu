@@ -179,8 +179,11 @@ hero_status validate_config(const hero_config* c) {
     return fail(HERO_ERR_ARG, "need 0 <= n_dense < n_layers (got %d)", c->n_dense);
   if (!(c->rms_eps >= 0.f) || !(c->eps >= 0.f) || !(c->t_hist > 0.f))
     return fail(HERO_ERR_ARG, "eps must be >= 0 and t_hist > 0");
-  if (c->d_m != 16 && c->d_m != 32 && c->d_m != 64 && c->d_m != 128)
-    return fail(HERO_ERR_UNSUPPORTED, "d_m must be 16, 32, 64 or 128 (got %d)", c->d_m);
+  if (c->d_m != 16 && c->d_m != 32 && c->d_m != 64 && c->d_m != 128 && c->d_m != 256)
+    return fail(HERO_ERR_UNSUPPORTED, "d_m must be 16, 32, 64, 128 or 256 (got %d)", c->d_m);
+  if (c->router_variant & ~(uint32_t)(HERO_ROUTER_NO_HISTORY | HERO_ROUTER_NO_MEMREAD |
+                                      HERO_ROUTER_NO_AUX | HERO_ROUTER_NO_POS))
+    return fail(HERO_ERR_ARG, "unknown router_variant bits 0x%x", c->router_variant);
   if (c->d_h + c->d_a > 128 || c->d_enc > 256 || c->d_head > 256 || c->d_path > 64)
     return fail(HERO_ERR_UNSUPPORTED, "router widths exceed d_s<=128, d_enc,d_head<=256, d_path<=64");
   if (c->d_h % 4 || c->d_a % 4 || c->d_enc % 4 || c->d_head % 4 || c->d_path % 4)
@@ -597,6 +600,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.mask = m->mask;
     ra.gate_out = gate_out_j;
     ra.mask_out = mask_out_j;
+    ra.variant = c.router_variant;
     CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, st); }));
   }
   CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,

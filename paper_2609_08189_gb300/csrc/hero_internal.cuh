@@ -145,7 +145,11 @@ struct RouterArgs {
   uint8_t* mask;         // [T]
   float* gate_out;       // [T] caller slice or nullptr
   uint8_t* mask_out;     // [T] caller slice or nullptr
+  uint32_t variant;      // router ablation bits (RV_*)
 };
+
+// Router ablation bits (the values of the ABI's HERO_ROUTER_*).
+enum : uint32_t { RV_NO_HISTORY = 1u, RV_NO_MEMREAD = 2u, RV_NO_AUX = 4u, RV_NO_POS = 8u };
 
 cudaError_t launch_router(int d_m, const RouterArgs& a, cudaStream_t st);
 

@@ -221,8 +221,117 @@ __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
   __syncthreads();
 }
 
+// Memory read (Eq. 11) fused with the write (Eq. 12) for the CTA's TB tokens, one
+// warp per token: c[n] = sum_m phi(q)_m S[m][n] / (phi(q) . zeta + eps), then
+// S = rho S + phi(k) v^T and zeta = rho zeta + phi(k); S is read once and written
+// once.  c goes to cT ([DM][TB], transposed).  DM <= 128: lane owns a 4-column
+// group and every (32 / (DM/4))-th row, partial c summed over the lanes of a
+// column group; DM = 256: lane owns column groups lane and lane + 32 over all
+// rows (a warp instruction covers 512 contiguous bytes of one row).
 template <int DM>
-__global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
+__device__ __forceinline__ void memory_read_write(const RouterArgs& a, const float* qkv, float* cT,
+                                                  int t0, int warp, int lane) {
+  for (int tl = warp; tl < TB; tl += NTHR / 32) {
+    const int t = t0 + tl;
+    if (t >= a.T) continue;
+    const float* q = qkv + tl * 3 * DM;
+    const float* k = q + DM;
+    const float* v = q + 2 * DM;
+    float* S = a.S + (size_t)t * DM * DM;
+    float* z = a.zeta + (size_t)t * DM;
+    float den = 0.f;
+    for (int m = lane; m < DM; m += 32) {
+      const float zo = z[m];
+      den += phif_(q[m]) * zo;
+      z[m] = a.rho * zo + phif_(k[m]);
+    }
+    den = warp_sum(den);
+    const float inv = 1.0f / (den + a.eps);
+    if constexpr (DM <= 128) {
+      constexpr int LPR = DM / 4;          // lanes per S row
+      constexpr int RPI = 32 / LPR;        // rows per iteration
+      constexpr int NIT = DM / RPI;        // S rows handled by this lane
+      constexpr int BATCH = NIT < 8 ? NIT : 8;  // loads kept in flight
+      const int cq = lane % LPR;
+      const int r0 = lane / LPR;
+      float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
+      const float4 vv = *reinterpret_cast<const float4*>(v + 4 * cq);
+#pragma unroll 1
+      for (int i0 = 0; i0 < NIT; i0 += BATCH) {
+        float4 so[BATCH];
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i)
+          so[i] = *reinterpret_cast<const float4*>(S + (r0 + (i0 + i) * RPI) * DM + 4 * cq);
+#pragma unroll
+        for (int i = 0; i < BATCH; ++i) {
+          const int r = r0 + (i0 + i) * RPI;
+          const float fq = phif_(q[r]);
+          const float fk = phif_(k[r]);
+          c.x += fq * so[i].x; c.y += fq * so[i].y; c.z += fq * so[i].z; c.w += fq * so[i].w;
+          *reinterpret_cast<float4*>(S + r * DM + 4 * cq) =
+              make_float4(a.rho * so[i].x + fk * vv.x, a.rho * so[i].y + fk * vv.y,
+                          a.rho * so[i].z + fk * vv.z, a.rho * so[i].w + fk * vv.w);
+        }
+      }
+#pragma unroll
+      for (int o = LPR; o < 32; o <<= 1) {
+        c.x += __shfl_xor_sync(0xffffffffu, c.x, o);
+        c.y += __shfl_xor_sync(0xffffffffu, c.y, o);
+        c.z += __shfl_xor_sync(0xffffffffu, c.z, o);
+        c.w += __shfl_xor_sync(0xffffffffu, c.w, o);
+      }
+      if (r0 == 0) {
+        float* cdst = cT + (4 * cq) * TB + tl;
+        cdst[0 * TB] = c.x * inv;
+        cdst[1 * TB] = c.y * inv;
+        cdst[2 * TB] = c.z * inv;
+        cdst[3 * TB] = c.w * inv;
+      }
+    } else {
+      constexpr int NCG = DM / 128;        // column groups per lane
+      constexpr int RB = 8;                // rows per batch: 64 KB of S in flight per CTA
+      float4 c[NCG], vv[NCG];
+#pragma unroll
+      for (int i = 0; i < NCG; ++i) {
+        c[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        vv[i] = *reinterpret_cast<const float4*>(v + 4 * (lane + 32 * i));
+      }
+#pragma unroll 1
+      for (int r0 = 0; r0 < DM; r0 += RB) {
+        float4 so[RB][NCG];
+#pragma unroll
+        for (int rr = 0; rr < RB; ++rr)
+#pragma unroll
+          for (int i = 0; i < NCG; ++i)
+            so[rr][i] = *reinterpret_cast<const float4*>(S + (r0 + rr) * DM + 4 * (lane + 32 * i));
+#pragma unroll
+        for (int rr = 0; rr < RB; ++rr) {
+          const float fq = phif_(q[r0 + rr]);
+          const float fk = phif_(k[r0 + rr]);
+#pragma unroll
+          for (int i = 0; i < NCG; ++i) {
+            const float4 x = so[rr][i];
+            c[i].x += fq * x.x; c[i].y += fq * x.y; c[i].z += fq * x.z; c[i].w += fq * x.w;
+            *reinterpret_cast<float4*>(S + (r0 + rr) * DM + 4 * (lane + 32 * i)) =
+                make_float4(a.rho * x.x + fk * vv[i].x, a.rho * x.y + fk * vv[i].y,
+                            a.rho * x.z + fk * vv[i].z, a.rho * x.w + fk * vv[i].w);
+          }
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < NCG; ++i) {
+        float* cdst = cT + (4 * (lane + 32 * i)) * TB + tl;
+        cdst[0 * TB] = c[i].x * inv;
+        cdst[1 * TB] = c[i].y * inv;
+        cdst[2 * TB] = c[i].z * inv;
+        cdst[3 * TB] = c[i].w * inv;
+      }
+    }
+  }
+}
+
+template <int DM>
+__global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const RouterArgs a) {
   extern __shared__ __align__(16) float sm[];
   const int ds = a.d_h + a.d_a;
   const RouterLayout lay(a.d_enc, a.d_head, ds, DM, a.d_path);
@@ -241,8 +350,11 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
   const int warp = tid >> 5, lane = tid & 31;
   const int nvalid = min(TB, a.T - t0);
 
+  const bool no_history = a.variant & RV_NO_HISTORY;
+  const bool no_memread = a.variant & RV_NO_MEMREAD;
+
   // 0. pull this CTA's memory block into L2 while the heads run (read in step 5)
-  if (tid == 0) {
+  if (tid == 0 && !no_history && !no_memread) {
     const char* Sb = reinterpret_cast<const char*>(a.S + (size_t)t0 * DM * DM);
     const uint32_t bytes = (uint32_t)(DM * DM * sizeof(float));
     for (int i = 0; i < nvalid; ++i)
@@ -291,10 +403,11 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
     sc[tid * 16 + 0] = rinv;
     sc[tid * 16 + 1] = dj;
     sc[tid * 16 + 4] = mp;
-    xT[0 * TB + tid] = (float)a.j / (float)a.L;
-    xT[1 * TB + tid] = (float)(a.L - a.j) / (float)a.L;
-    xT[2 * TB + tid] = dj;
-    xT[3 * TB + tid] = gam;
+    const bool pos = !(a.variant & RV_NO_POS);   // ablation: no progress / transition
+    xT[0 * TB + tid] = pos ? (float)a.j / (float)a.L : 0.f;
+    xT[1 * TB + tid] = pos ? (float)(a.L - a.j) / (float)a.L : 0.f;
+    xT[2 * TB + tid] = pos ? dj : 0.f;
+    xT[3 * TB + tid] = pos ? gam : 0.f;
     xT[4 * TB + tid] = pp;
     xT[5 * TB + tid] = mp;
   }
@@ -339,79 +452,45 @@ __global__ void __launch_bounds__(NTHR, 4) k_router(const RouterArgs a) {
     reduce16(red, bpart, ab + TB);   // also orders step 2's writes before step 3
   }
 
+  if (no_history) {   // ablation: g = sigma(b), the local logit alone; state untouched
+    if (tid < TB) {
+      const int t = t0 + tid;
+      if (t < a.T) {
+        const float g = sigmoidf_(ab[TB + tid] + __ldg(a.w.ps_b2));
+        const uint8_t dec = a.mask_in ? (a.mask_in[t] ? 1 : 0) : (g >= a.tau ? 1 : 0);
+        a.gate[t] = g;
+        a.mask[t] = dec;
+        if (a.gate_out) a.gate_out[t] = g;
+        if (a.mask_out) a.mask_out[t] = dec;
+      }
+    }
+    return;
+  }
+
   // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s)
   bmm4(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
-  bmm4(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
-  bmm4(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
+  if (a.variant & RV_NO_AUX) {   // ablation: no auxiliary path encoder, z_a = 0
+    for (int e = tid; e < a.d_a * TB; e += NTHR) sT[a.d_h * TB + e] = 0.f;
+    __syncthreads();
+  } else {
+    bmm4(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
+    bmm4(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
+  }
 
   // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step
   bmm4(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false);
 
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
-  //    Lane owns a 4-column group and every (32/LPR)-th row of S.
-  {
-    constexpr int LPR = DM / 4;          // lanes per S row
-    constexpr int RPI = 32 / LPR;        // rows per iteration
-    constexpr int NIT = DM / RPI;        // S rows handled by this lane
-    constexpr int BATCH = NIT < 8 ? NIT : 8;  // loads kept in flight
-    const int cq = lane % LPR;
-    const int r0 = lane / LPR;
-    for (int tl = warp; tl < TB; tl += NTHR / 32) {
-      const int t = t0 + tl;
-      if (t >= a.T) continue;
-      const float* q = qkv + tl * 3 * DM;
-      const float* k = q + DM;
-      const float* v = q + 2 * DM;
-      float* S = a.S + (size_t)t * DM * DM;
-      float* z = a.zeta + (size_t)t * DM;
-      float den = 0.f;
-      for (int m = lane; m < DM; m += 32) {
-        const float zo = z[m];
-        den += phif_(q[m]) * zo;
-        z[m] = a.rho * zo + phif_(k[m]);
-      }
-      den = warp_sum(den);
-      float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
-      const float4 vv = *reinterpret_cast<const float4*>(v + 4 * cq);
-#pragma unroll 1
-      for (int i0 = 0; i0 < NIT; i0 += BATCH) {
-        float4 so[BATCH];
-#pragma unroll
-        for (int i = 0; i < BATCH; ++i)
-          so[i] = *reinterpret_cast<const float4*>(S + (r0 + (i0 + i) * RPI) * DM + 4 * cq);
-#pragma unroll
-        for (int i = 0; i < BATCH; ++i) {
-          const int r = r0 + (i0 + i) * RPI;
-          const float fq = phif_(q[r]);
-          const float fk = phif_(k[r]);
-          c.x += fq * so[i].x; c.y += fq * so[i].y; c.z += fq * so[i].z; c.w += fq * so[i].w;
-          *reinterpret_cast<float4*>(S + r * DM + 4 * cq) =
-              make_float4(a.rho * so[i].x + fk * vv.x, a.rho * so[i].y + fk * vv.y,
-                          a.rho * so[i].z + fk * vv.z, a.rho * so[i].w + fk * vv.w);
-        }
-      }
-#pragma unroll
-      for (int o = LPR; o < 32; o <<= 1) {
-        c.x += __shfl_xor_sync(0xffffffffu, c.x, o);
-        c.y += __shfl_xor_sync(0xffffffffu, c.y, o);
-        c.z += __shfl_xor_sync(0xffffffffu, c.z, o);
-        c.w += __shfl_xor_sync(0xffffffffu, c.w, o);
-      }
-      if (r0 == 0) {
-        const float inv = 1.0f / (den + a.eps);
-        float* cdst = sT + (ds + 4 * cq) * TB + tl;
-        cdst[0 * TB] = c.x * inv;
-        cdst[1 * TB] = c.y * inv;
-        cdst[2 * TB] = c.z * inv;
-        cdst[3 * TB] = c.w * inv;
-      }
-    }
+  if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
+    for (int e = tid; e < DM * TB; e += NTHR) sT[ds * TB + e] = 0.f;
+  } else {
+    memory_read_write<DM>(a, qkv, sT + ds * TB, t0, warp, lane);
   }
   __syncthreads();
 
   // 6. nu = 1 - cos(W_n s, W_c c) for j > 1 (Eq. 13); nu_1 = 0
   float* nuT = sT + (ds + DM) * TB;
-  if (a.j > 1) {
+  if (a.j > 1 && !no_memread) {   // the ablation without memory access sees nu = 0
     const int cap = (a.d_enc > a.d_head ? a.d_enc : a.d_head) * TB;
     float* nv = aux;               // [DM][TB]
     float* cv = aux + DM * TB;     // [DM][TB]
@@ -685,6 +764,7 @@ cudaError_t launch_router(int d_m, const RouterArgs& a, cudaStream_t st) {
     case 32: return launch_router_dm<32>(a, st);
     case 64: return launch_router_dm<64>(a, st);
     case 128: return launch_router_dm<128>(a, st);
+    case 256: return launch_router_dm<256>(a, st);
     default: return cudaErrorInvalidValue;
   }
 }

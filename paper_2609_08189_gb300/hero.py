@@ -22,6 +22,7 @@ STATUS_NAMES = {0: "HERO_OK", 1: "HERO_ERR_ARG", 2: "HERO_ERR_CUDA", 3: "HERO_ER
                 4: "HERO_ERR_UNSUPPORTED", 5: "HERO_ERR_TIMEOUT"}
 HERO_F32, HERO_BF16 = 0, 1
 HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO = 1, 2, 4
+HERO_ROUTER_NO_HISTORY, HERO_ROUTER_NO_MEMREAD, HERO_ROUTER_NO_AUX, HERO_ROUTER_NO_POS = 1, 2, 4, 8
 KERNEL_CLASSES = ("init", "router_gemm", "router", "compact", "norm", "ffn_gate_up", "ffn_down",
                   "adapter_down", "adapter_up")
 HERO_K_COUNT = len(KERNEL_CLASSES)
@@ -37,7 +38,8 @@ class hero_config(ctypes.Structure):
                 ("n_layers", "d_model", "d_ff", "d_r", "d_m", "d_h", "d_a", "d_enc", "d_head",
                  "d_path", "max_tokens")] + \
                [("dtype", ctypes.c_int), ("rms_eps", ctypes.c_float), ("eps", ctypes.c_float),
-                ("t_hist", ctypes.c_float), ("n_dense", ctypes.c_int32)]
+                ("t_hist", ctypes.c_float), ("n_dense", ctypes.c_int32),
+                ("router_variant", ctypes.c_uint32)]
 
 
 class hero_weights_host(ctypes.Structure):
@@ -113,7 +115,7 @@ def make_config(stack_cfg, max_tokens: Optional[int] = None) -> hero_config:
     return hero_config(c.n_layers, c.d_model, c.d_ff, c.d_r, c.d_m, c.d_h, c.d_a, c.d_enc,
                        c.d_head, c.d_path, max_tokens or c.n_tokens,
                        HERO_BF16 if c.dtype == "bf16" else HERO_F32, c.rms_eps, c.eps, c.t_hist,
-                       getattr(c, "n_dense", 0))
+                       getattr(c, "n_dense", 0), getattr(c, "router_variant", 0))
 
 
 def make_weights(weights: Dict[str, np.ndarray]):

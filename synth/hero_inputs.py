@@ -64,6 +64,7 @@ class StackConfig:
     batch: int = 1         # sequences (for reporting only; tokens are independent)
     seq_len: int = 0
     n_dense: int = 0       # leading FFN layers outside the routing candidate set (Sec. 4.1)
+    router_variant: int = 0  # Sec. 4.4 router ablation bits (1 history, 2 memread, 4 aux, 8 pos)
 
     @property
     def d_s(self) -> int:

@@ -411,10 +411,12 @@ def test_p7_budget_tiny():
 # P8: independent per-token, per-element pure-Python restatement (tiny shapes)
 # ---------------------------------------------------------------------------
 
-def _py_stack(cfg, W, h_in, P, tau, n_dense=0):
+def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
     """Per-token loops over scalars, written from Sec. 3 without numpy linear algebra.
     The first n_dense layers are plain FFN blocks (Sec. 4.1 placement); the rest are
-    routed blocks j = 1 .. L - n_dense."""
+    routed blocks j = 1 .. L - n_dense.  variant: the Sec. 4.4 ablations, bits
+    1 = w/o History (g from the local logit), 2 = w/o MemRead (c = 0, nu = 0, no
+    memory), 4 = w/o Aux State (z_a = 0), 8 = w/o Pos State (r, q_rem, d, gamma = 0)."""
     L, d = cfg.n_layers, cfg.d_model
     LR = L - n_dense
 
@@ -451,6 +453,20 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0):
                 gs.append(1.0)
                 continue
             j = layer - n_dense
+            if variant & 1:                                    # w/o History
+                hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], hb), W["ps_b1"])]
+                g = sg(sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0])
+                rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+                u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
+                if g >= tau:
+                    gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
+                    y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
+                    h = [hb[i] + g * y[i] for i in range(d)]
+                else:
+                    y = mv(W["ad_w2"][layer - 1], [sl(x) for x in mv(W["ad_w1"][layer - 1], u)])
+                    h = [hb[i] + (1 - g) * y[i] for i in range(d)]
+                gs.append(g)
+                continue
             if j == 1:
                 dl = [0.0] * d
             else:
@@ -463,14 +479,21 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0):
             nr = [hb[i] / rms * W["r_norm_g"][i] for i in range(d)]
             zh = mv(W["w_hu"], [sl(x) for x in mv(W["w_hd"], nr)])
             xp = [j / LR, (LR - j) / LR, dd, gam, p_prev, m_prev]
+            if variant & 8:                                    # w/o Pos State
+                xp = [0.0, 0.0, 0.0, 0.0, p_prev, m_prev]
             hid = [sl(x + b) for x, b in zip(mv(W["path_w1"], xp), W["path_b1"])]
             za = [x + b for x, b in zip(mv(W["path_w2"], hid), W["path_b2"])]
+            if variant & 4:                                    # w/o Aux State
+                za = [0.0] * len(za)
             s = zh + za
             q, k, v = mv(W["w_q"], s), mv(W["w_k"], s), mv(W["w_v"], s)
             fq, fk = [ph(x) for x in q], [ph(x) for x in k]
             den = sum(fq[m] * Z[m] for m in range(dm)) + cfg.eps
             c = [sum(fq[m] * S[m][n] for m in range(dm)) / den for n in range(dm)]
-            if j == 1:
+            if variant & 2:                                    # w/o MemRead
+                c = [0.0] * dm
+                nu = 0.0
+            elif j == 1:
                 nu = 0.0
             else:
                 a1, b1 = mv(W["w_n"], s), mv(W["w_c"], c)
@@ -489,6 +512,9 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0):
                 for n in range(dm):
                     S[mm][n] = rho * S[mm][n] + fk[mm] * v[n]
                 Z[mm] = rho * Z[mm] + fk[mm]
+            if variant & 2:                                    # the memory stays empty
+                S = [[0.0] * dm for _ in range(dm)]
+                Z = [0.0] * dm
             rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
             u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
             if g >= tau:
@@ -518,6 +544,29 @@ def test_p8_loop_restatement_tiny_shapes():
     np.testing.assert_allclose(got["gate"], ref_g, rtol=0, atol=1e-12)
     np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
     assert 0 < got["mask"].sum() < got["mask"].size
+
+
+@pytest.mark.parametrize("variant", [1, 2, 4, 8, 4 | 8, 2 | 4 | 8])
+def test_p8_router_ablations_restatement(variant):
+    """Sec. 4.4 component ablations against the independent loop restatement."""
+    cfg = hi.StackConfig("micro", 4, 8, 12, 4, 4, 6, "f32", 0.3, d_h=3, d_a=2, d_enc=5,
+                         d_head=6, d_path=3, seed=13)
+    w, h, P = _inputs(cfg)
+    W = {k: hi.to_f64(v).tolist() for k, v in w.items()}
+    oc = ho.OracleConfig.from_stack(cfg)
+    oc.variant = variant
+    base = ho.routed_ffn_stack(oc, w, h, P, 0.0)
+    tau = float(np.median(base["gate"]))
+    got = ho.routed_ffn_stack(oc, w, h, P, tau, record=True)
+    ref_h, ref_g = _py_stack(cfg, W, hi.to_f64(h).tolist(), hi.to_f64(P).tolist(), tau,
+                             variant=variant)
+    np.testing.assert_allclose(got["gate"], ref_g, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
+    full = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, tau)
+    assert np.max(np.abs(full["gate"] - got["gate"])) > 1e-6   # the ablation changes g
+    if variant & 2:                                           # no memory read or write
+        for rec in got["layers"]:
+            assert not rec["S"].any() and not rec["c"].any() and not rec["nu"].any()
 
 
 def test_p8_placement_dense_prefix_restatement():
