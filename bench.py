@@ -191,6 +191,8 @@ def main():
     ap.add_argument("--router-variant", type=int, default=0,
                     help="Sec. 4.4 router ablation bits (1 history, 2 memread, 4 aux, 8 pos)")
     ap.add_argument("--d-m", type=int, default=None, help="memory width override (ablation)")
+    ap.add_argument("--graph", action="store_true",
+                    help="time CUDA-graph replays of one captured step (launch-bound decode)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -248,8 +250,9 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         return float(t.item())
 
-    def run(flags):
-        stack(h, P, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m, counts_out=c, stream=stream)
+    def run(flags, st=None):
+        stack(h, P, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m, counts_out=c,
+              stream=st or stream)
 
     def timed(fn, K, sampler=None):
         barrier()
@@ -279,6 +282,21 @@ def main():
     hero.hero_set_profiling(stack.model, False)
     prof = hero.hero_get_profile(stack.model, reset=True)
     stack.check()
+    ms_eager = ms / args.steps
+    if args.graph:
+        # the stack enqueues with no host synchronisation, so one step captures into a
+        # CUDA graph whose replays remove the per-launch CPU cost
+        graph = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        with torch.cuda.graph(graph, stream=cap):
+            run(0, cap)
+        stream.wait_stream(cap)
+        for _ in range(args.warmup):
+            graph.replay()
+        torch.cuda.synchronize()
+        ms, clocks = timed(graph.replay, args.steps, ClockSampler(local_rank))
+        stack.check()
     counts = c.cpu().numpy().astype(np.int64)
     bypass = 1.0 - counts[cfg.n_dense:].sum() / ((L - cfg.n_dense) * T)   # routed blocks
     value = world * T * args.steps / (ms / 1e3)
@@ -351,7 +369,8 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
         "config": {"workload": workload_desc(cfg, cfg.bypass),
                    "l2": "inputs larger than L2 (no flush): weights and P_j stream from HBM each step",
-                   "parallelism": f"token shards, {world} rank(s), no collective"},
+                   "parallelism": f"token shards, {world} rank(s), no collective",
+                   **({"cuda_graph": True, "eager_ms_per_step": ms_eager} if args.graph else {})},
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": e2e,

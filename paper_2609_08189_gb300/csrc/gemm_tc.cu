@@ -82,7 +82,8 @@ __device__ __forceinline__ float4 staged(const float4* st, int row, int slot) {
 
 template <int BN>
 __device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase, int row0, int M,
-                                              int nb, float4* st) {
+                                              int nb, int split, float4* st) {
+  float* out = a.out_f32 + (size_t)split * a.split_stride;
   const int lane = threadIdx.x & 31;
   const int sub = lane >> 3, slot = lane & 7;
 #pragma unroll 1
@@ -97,7 +98,7 @@ __device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase,
       const int rr = sub + 4 * k;
       const int m = row0 + rr;
       if (m < M && n < a.N)
-        *reinterpret_cast<float4*>(a.out_f32 + (size_t)m * a.ldo + n) = staged(st, rr, slot);
+        *reinterpret_cast<float4*>(out + (size_t)m * a.ldo + n) = staged(st, rr, slot);
     }
     __syncwarp();
   }
@@ -218,10 +219,16 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
   }
 }
 
-// Sizes of one problem of a launch (the row count may be device-resident).
+// Sizes of one problem of a launch (the row count may be device-resident).  With
+// split-K the tile index runs over splits x M-tiles x N-tiles and split s covers
+// K-blocks [s * kpb, min((s + 1) * kpb, kblocks)).
 struct ProbSize {
-  int M, m_tiles, n_tiles, kblocks, tiles;
+  int M, m_tiles, n_tiles, kblocks, tiles, kpb;
 };
+
+// Tile `local` of a problem -> coordinates and K-block range.
+__device__ __forceinline__ void tile_work(const ProbSize& p, int local, int& mb, int& nb, int& s,
+                                          int& kb0, int& kb1);
 
 template <int BN>
 __device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
@@ -235,8 +242,19 @@ __device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
   p.m_tiles = (M + BM - 1) / BM;
   p.n_tiles = (a.N + BN - 1) / BN;
   p.kblocks = (a.K + BK - 1) / BK;
-  p.tiles = p.m_tiles * p.n_tiles;
+  const int splits = a.k_splits > 1 ? a.k_splits : 1;
+  p.kpb = (p.kblocks + splits - 1) / splits;
+  p.tiles = p.m_tiles * p.n_tiles * splits;
   return p;
+}
+
+__device__ __forceinline__ void tile_work(const ProbSize& p, int local, int& mb, int& nb, int& s,
+                                          int& kb0, int& kb1) {
+  const int per_split = p.m_tiles * p.n_tiles;
+  s = local / per_split;
+  tile_coords(local - s * per_split, p.m_tiles, p.n_tiles, mb, nb);
+  kb0 = s * p.kpb;
+  kb1 = min(p.kblocks, kb0 + p.kpb);
 }
 
 // Tile g of a grouped launch -> (problem, tile within it): the second problem's
@@ -261,10 +279,11 @@ __device__ __forceinline__ int split_tile(int g, int t1, int total, int& local) 
 // second warp of a quadrant takes the upper half of the columns.
 template <int BN, int EPI>
 __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, int q, int ew,
-                                             int lane, int mb, int nb, int M, float4* stg) {
+                                             int lane, int mb, int nb, int M, int split,
+                                             float4* stg) {
   const int row0 = mb * BM + q * 32;
   if constexpr (EPI == EPI_STORE_F32) {
-    epi_store_f32<BN>(a, tbase, row0, M, nb, stg);
+    epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
   } else if constexpr (EPI == EPI_SWIGLU) {
     epi_swiglu(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_SILU) {
@@ -346,12 +365,11 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
-        int mb, nb;
-        tile_coords(local, pr ? P1.m_tiles : P0.m_tiles, pr ? P1.n_tiles : P0.n_tiles, mb, nb);
+        int mb, nb, sp, kb0, kb1;
+        tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         const CUtensorMap* tA = pr ? &tmA1 : &tmA0;
         const CUtensorMap* tB = pr ? &tmB1 : &tmB0;
-        const int kblocks = pr ? P1.kblocks : P0.kblocks;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitLimitNs) || misc[1]) {
             ok = false;
             break;
@@ -386,14 +404,15 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
-        const int kblocks = pr ? P1.kblocks : P0.kblocks;
+        int mb, nb, sp, kb0, kb1;
+        tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, kWaitLimitNs) || misc[1]) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(full_bar(stage), phase, kWaitLimitNs) || misc[1]) {
             ok = false;
             break;
@@ -404,7 +423,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             // +32 bytes per K step of 16 bf16 inside the 128-byte swizzle row
-            umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb | k) != 0);
+            umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb != kb0) || k != 0);
           }
           umma_commit(empty_bar(stage));
           if (++stage == C::STAGES) {
@@ -433,8 +452,8 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     for (int g = blockIdx.x; g < total; g += gridDim.x) {
       int local;
       const int pr = split_tile(g, P1.tiles, total, local);
-      int mb, nb;
-      tile_coords(local, pr ? P1.m_tiles : P0.m_tiles, pr ? P1.n_tiles : P0.n_tiles, mb, nb);
+      int mb, nb, sp, kb0, kb1;
+      tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
       bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);
@@ -450,11 +469,11 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + ew * (32 * 8);
       if constexpr (kGrouped) {
         if (pr)
-          run_epilogue<BN, EPI1>(a1, tbase, q, ew, lane, mb, nb, P1.M, stg);
+          run_epilogue<BN, EPI1>(a1, tbase, q, ew, lane, mb, nb, P1.M, sp, stg);
         else
-          run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, stg);
+          run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg);
       } else {
-        run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, stg);
+        run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg);
       }
       tc_fence_before();
       __syncwarp();
@@ -484,7 +503,13 @@ cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const Ge
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  long max_tiles = (long)((a0.m_max + BM - 1) / BM) * ((a0.N + BN - 1) / BN);
+  if (a0.k_splits > 1 && EPI0 != EPI_STORE_F32) return cudaErrorInvalidValue;
+  const long kb0 = (a0.K + BK - 1) / BK;
+  if (a0.k_splits > 1 && (a0.k_splits > kb0 || (long)(a0.k_splits - 1) *
+                                                 ((kb0 + a0.k_splits - 1) / a0.k_splits) >= kb0))
+    return cudaErrorInvalidValue;   // every split must own at least one K-block
+  long max_tiles = (long)((a0.m_max + BM - 1) / BM) * ((a0.N + BN - 1) / BN) *
+                   (a0.k_splits > 1 ? a0.k_splits : 1);
   if (EPI1 != EPI_NONE) max_tiles += (long)((a1.m_max + BM - 1) / BM) * ((a1.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
   const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);

@@ -2,6 +2,7 @@
 // per-block launch sequence of the routed FFN stack, profiling and the C ABI.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -114,6 +115,7 @@ struct hero_model {
   void* ws = nullptr;
   size_t ws_bytes = 0;
   float *hbar, *delta, *part, *Y, *S, *zeta, *pst, *mst, *dprev, *gate, *scale_f, *scale_a;
+  float* splitk_ws = nullptr;   // bf16: partial slices of split-K GEMMs (few-tile launches)
   void *xl, *u_f, *u_a, *act, *ah;
   uint8_t* mask;
   int *idx_f, *idx_a, *counts;
@@ -199,6 +201,48 @@ hero_status validate_config(const hero_config* c) {
       return fail(HERO_ERR_UNSUPPORTED, "bf16 needs d_enc + d_head to be a multiple of 8");
   }
   return HERO_OK;
+}
+
+// K splits for a tensor-core launch of `tiles` 128x256 output tiles over `kblocks`
+// 64-wide K-blocks (`rows` x `n` outputs), from a wave-quantisation cost model: the
+// GEMM takes ceil(tiles * s / num_sms) waves of ceil(kblocks / s) K-block steps
+// (~0.4 us each on one SM) plus the last tile's epilogue (~50 us for the block-closing
+// epilogue, ~10 us for a plain store), and s > 1 adds a finishing pass that moves
+// rows * n * (4 s + epi_bytes) bytes at ~5 TB/s.  rows is the launch's upper bound
+// (the routed count is device-resident).  Every split keeps >= 1 K-block.
+int choose_splits(int tiles, int kblocks, int num_sms, long rows, long n, int epi_bytes) {
+  if (tiles <= 0 || kblocks <= 1) return 1;
+  double best_t = 0.0;
+  int best = 1;
+  for (int s = 1; s <= 16 && s <= kblocks; ++s) {
+    const int kpb = (kblocks + s - 1) / s;
+    const int eff = (kblocks + kpb - 1) / kpb;   // splits that own K-blocks
+    if (eff != s) continue;
+    const long waves = ((long)tiles * s + num_sms - 1) / num_sms;
+    double t = (double)waves * kpb * 0.4;
+    if (s > 1)
+      t += 10.0 + (double)rows * n * (4.0 * s + epi_bytes) / 5.0e6;
+    else
+      t += epi_bytes > 4 ? 50.0 : 10.0;
+    if (s == 1 || t < best_t * 0.97) {   // a split must win by 3%
+      best_t = t;
+      best = s;
+    }
+  }
+  return best;
+}
+
+// Largest split-K partial buffer (floats) any token count up to T may ask for.
+size_t splitk_ws_floats(int T, int num_sms, int nY, int K_router, int d, int I) {
+  size_t most = 0;
+  for (int m_t = 1; m_t <= (T + 127) / 128; ++m_t) {
+    const long rows = (long)m_t * 128;
+    const int rs = choose_splits(m_t * ((nY + 255) / 256), (K_router + 63) / 64, num_sms, rows, nY, 4);
+    const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, num_sms, rows, d, 22);
+    if (rs > 1) most = std::max(most, (size_t)rs * rows * nY);
+    if (ds > 1) most = std::max(most, (size_t)ds * rows * d);
+  }
+  return most;
 }
 
 // Upload a host matrix [rows, cols] (element type src_dt) through a device staging
@@ -476,6 +520,9 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         {(void**)&m->ah, Tm * r * es},         {(void**)&m->mask, Tm},
         {(void**)&m->idx_f, Tm * 4},           {(void**)&m->idx_a, Tm * 4},
         {(void**)&m->counts, 64},              {(void**)&m->err, 64},
+        // split-K partials of the few-wave launches (router contraction, FFN down)
+        {(void**)&m->splitk_ws, bf16 ? splitk_ws_floats(c.max_tokens, m->num_sms, (int)nY,
+                                                        (int)(2 * d), (int)d, (int)I) * 4 : 0},
     };
     for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
     CUDA_M(cudaMalloc(&m->ws, off));
@@ -539,6 +586,8 @@ struct BlockState {
   float *S, *zeta, *pst, *mst, *dprev;
 };
 
+
+
 // Everything of block jj (layer index; routed index jr = jj - n_dense) after its
 // entry (h_bar, its operand copy and the partial sums are in place): router
 // contraction and router, compaction, LN_ffn, FFN and adapter branches with the
@@ -567,10 +616,22 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     g.B = m->wr;
     g.lda = d;
     g.ldb = d;
+    const int m_t = (T + 127) / 128;
+    const int rs = m->bf16 ? choose_splits(m_t * ((nY + 255) / 256), (g.K + 63) / 64, m->num_sms,
+                                           (long)m_t * 128, nY, 4) : 1;
+    if (rs > 1) {   // few tiles (small T): split K, then add the slices in order into Y
+      g.out_f32 = m->splitk_ws;
+      g.k_splits = rs;
+      g.split_stride = (long)m_t * 128 * nY;
+    }
     CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
       return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
                      : launch_gemm_simt(EPI_STORE_F32, g, st);
     }));
+    if (rs > 1)
+      CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
+        return launch_splitk_sum(m->splitk_ws, rs, g.split_stride, T, nY, m->Y, st);
+      }));
     RouterArgs ra{};
     ra.T = T;
     ra.j = j;
@@ -601,7 +662,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.gate_out = gate_out_j;
     ra.mask_out = mask_out_j;
     ra.variant = c.router_variant;
-    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, st); }));
+    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, m->num_sms, st); }));
   }
   CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
                  m->counts, count_out_j, dense ? gate_out_j : nullptr,
@@ -671,6 +732,22 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
         return launch_gemm_tc(256, EPI_LAYER_OUT_WIDE, m->tm_ah, m->tm_w2[jj], au, m->num_sms, st);
       }));
+    const int m_t = (T + 127) / 128;
+    const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
+    if (ds > 1) {   // few tiles (small T): split K into partials, then the closing epilogue
+      GemmArgs sk = dn;
+      sk.out_f32 = m->splitk_ws;
+      sk.ldo = d;
+      sk.k_splits = ds;
+      sk.split_stride = (long)m_t * 128 * d;
+      CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
+        return launch_gemm_tc(256, EPI_STORE_F32, m->tm_act, m->tm_wd[jj], sk, m->num_sms, st);
+      }));
+      CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
+        return launch_splitk_close(m->splitk_ws, ds, sk.split_stride, d, m->counts, T, dn.lo, st);
+      }));
+      return HERO_OK;
+    }
     CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
       return launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dn, m->num_sms, st);
     }));

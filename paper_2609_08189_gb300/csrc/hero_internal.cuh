@@ -75,6 +75,10 @@ struct GemmArgs {
   int ldo;             // leading dimension of out / out_f32 in elements
   LayerOutArgs lo;     // EPI_LAYER_OUT
   uint32_t* err;
+  // split-K (EPI_STORE_F32 only): K-blocks are cut into k_splits contiguous ranges;
+  // range s stores its partial sums at out_f32 + s * split_stride
+  int k_splits;        // 0 or 1: no split
+  long split_stride;
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
@@ -151,7 +155,7 @@ struct RouterArgs {
 // Router ablation bits (the values of the ABI's HERO_ROUTER_*).
 enum : uint32_t { RV_NO_HISTORY = 1u, RV_NO_MEMREAD = 2u, RV_NO_AUX = 4u, RV_NO_POS = 8u };
 
-cudaError_t launch_router(int d_m, const RouterArgs& a, cudaStream_t st);
+cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st);
 
 struct InitArgs {
   int T, d, np, d_m;
@@ -232,6 +236,17 @@ struct AdapterUpArgs {
   LayerOutArgs lo;
 };
 cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st);
+
+// Split-K finishing kernels (few-tile launches, e.g. decode): fixed-order sums of
+// the k_splits partial slices [s][rows][ld] written by a split tensor-core GEMM.
+//   sum:   out[m, n] = sum_s part[s, m, n]                     (m < M, n < N)
+//   close: y = sum_s part[s, m, n], then the block-closing epilogue (LayerOutArgs)
+//          on token idx[m] for m < *m_dev, with kTcPartCols-column partial sums
+cudaError_t launch_splitk_sum(const float* part, int splits, long split_stride, int M, int N,
+                              float* out, cudaStream_t st);
+cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
+                                const int* m_dev, int m_max, const LayerOutArgs& lo,
+                                cudaStream_t st);
 
 // Weight conversion: dst[map(r)] = convert(src[r]) for rows of `cols` elements.
 // map(r) = (r / grp) * grp_stride + (r % grp) + offset.

@@ -115,7 +115,10 @@ __global__ void __launch_bounds__(256) k_state_reset(float* S, float* zeta, floa
 // [feature][TB], so a block matmul loads one float4 of weights (four outputs) and
 // one float4 of activations (four tokens) per 16 FMAs.
 // ------------------------------------------------------------------------------
-constexpr int TB = 16;        // tokens per CTA
+// Tokens per CTA: 16 for large token counts, 4 when T/16 CTAs would not fill the
+// GPU twice over (decode and short prefill), where the per-CTA chain of dependent
+// phases is the critical path and the head matmuls split K more widely.
+constexpr int TB_LARGE = 16, TB_SMALL = 4;
 constexpr int NTHR = 256;
 
 // Shared-memory layout (floats), computed from the model's widths on host and
@@ -125,8 +128,12 @@ constexpr int NTHR = 256;
 //   s     [d_s + d_m + 1][TB]: s | c | nu
 //   qkv   [TB][3 d_m] token-major
 //   aux   [max(3072, 2 d_m TB)]: split-K scratch of W_hu (step 3), W_n s | W_c c (step 6)
+template <int TB>
 struct RouterLayout {
-  int big, s, qkv, aux, x, ph, red, sc, ab, floats;
+  int big, s, qkv, aux, x, ph, red, sc, ab, sk, floats;
+  // sk: split-K scratch of q/k/v and f_theta (small TB only; with TB = 16 those
+  // products have enough output tiles to occupy every thread without a split)
+  static constexpr int kSplitScratch = TB < 16 ? 4096 : 0;
   __host__ __device__ RouterLayout(int d_enc, int d_head, int ds, int dm, int d_path) {
     const int nbig = (d_enc > d_head ? d_enc : d_head) * TB;
     const int ns = ((ds + dm + 1 + 3) & ~3) * TB;
@@ -140,7 +147,8 @@ struct RouterLayout {
     red = ph + d_path * TB;
     sc = red + 3 * NTHR;
     ab = sc + TB * 16;
-    floats = ab + 2 * TB;
+    sk = ab + 2 * TB;
+    floats = sk + kSplitScratch;
   }
 };
 
@@ -150,6 +158,7 @@ struct RouterLayout {
 // `scratch` ([ks][NO][TB], at most scratch_cap floats) and are added in a fixed
 // order, so results are bitwise reproducible.  NO must be a multiple of 4;
 // contains __syncthreads.
+template <int TB>
 __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int NO,
                      const float* __restrict__ bias, float* out, int out_tok_ld, bool silu_act,
                      float* scratch = nullptr, int scratch_cap = 0) {
@@ -210,6 +219,7 @@ __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int 
 
 // Sum the 16 per-thread partials of each token (thread t + 16 p holds partial p of
 // token t) in a fixed order; contains __syncthreads.
+template <int TB>
 __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
   red[threadIdx.x] = v;
   __syncthreads();
@@ -228,7 +238,7 @@ __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
 // group and every (32 / (DM/4))-th row, partial c summed over the lanes of a
 // column group; DM = 256: lane owns column groups lane and lane + 32 over all
 // rows (a warp instruction covers 512 contiguous bytes of one row).
-template <int DM>
+template <int DM, int TB>
 __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const float* qkv, float* cT,
                                                   int t0, int warp, int lane) {
   for (int tl = warp; tl < TB; tl += NTHR / 32) {
@@ -330,11 +340,12 @@ __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const flo
   }
 }
 
-template <int DM>
+template <int DM, int TB>
 __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const RouterArgs a) {
   extern __shared__ __align__(16) float sm[];
   const int ds = a.d_h + a.d_a;
-  const RouterLayout lay(a.d_enc, a.d_head, ds, DM, a.d_path);
+  const RouterLayout<TB> lay(a.d_enc, a.d_head, ds, DM, a.d_path);
+  float* skT = RouterLayout<TB>::kSplitScratch ? sm + lay.sk : nullptr;
   float* bigT = sm + lay.big;
   float* sT = sm + lay.s;      // rows [0, d_s) s, [d_s, d_s + DM) c, d_s + DM nu
   float* qkv = sm + lay.qkv;   // [TB][3 DM]
@@ -449,7 +460,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
         }
       }
     }
-    reduce16(red, bpart, ab + TB);   // also orders step 2's writes before step 3
+    reduce16<TB>(red, bpart, ab + TB);   // also orders step 2's writes before step 3
   }
 
   if (no_history) {   // ablation: g = sigma(b), the local logit alone; state untouched
@@ -468,23 +479,24 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
   }
 
   // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s)
-  bmm4(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
+  bmm4<TB>(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
   if (a.variant & RV_NO_AUX) {   // ablation: no auxiliary path encoder, z_a = 0
     for (int e = tid; e < a.d_a * TB; e += NTHR) sT[a.d_h * TB + e] = 0.f;
     __syncthreads();
   } else {
-    bmm4(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
-    bmm4(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
+    bmm4<TB>(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
+    bmm4<TB>(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
   }
 
   // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step
-  bmm4(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false);
+  bmm4<TB>(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false, skT,
+           RouterLayout<TB>::kSplitScratch);
 
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
     for (int e = tid; e < DM * TB; e += NTHR) sT[ds * TB + e] = 0.f;
   } else {
-    memory_read_write<DM>(a, qkv, sT + ds * TB, t0, warp, lane);
+    memory_read_write<DM, TB>(a, qkv, sT + ds * TB, t0, warp, lane);
   }
   __syncthreads();
 
@@ -494,8 +506,8 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
     const int cap = (a.d_enc > a.d_head ? a.d_enc : a.d_head) * TB;
     float* nv = aux;               // [DM][TB]
     float* cv = aux + DM * TB;     // [DM][TB]
-    bmm4(sT, ds, a.w.w_n_t, DM, nullptr, nv, 0, false, bigT, cap);
-    bmm4(sT + ds * TB, DM, a.w.w_c_t, DM, nullptr, cv, 0, false, bigT, cap);
+    bmm4<TB>(sT, ds, a.w.w_n_t, DM, nullptr, nv, 0, false, bigT, cap);
+    bmm4<TB>(sT + ds * TB, DM, a.w.w_c_t, DM, nullptr, cv, 0, false, bigT, cap);
     // thread (part, t) sums DM/16 products; fixed-order reduction per token
     const int tl = tid % TB, part = tid / TB;
     float xy = 0.f, xx = 0.f, yy = 0.f;
@@ -505,30 +517,18 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
       xx += u * u;
       yy += w * w;
     }
-    float* r3 = sc;  // reuse columns 8..10 of the scalar rows for the three sums
-    red[tid] = xy;
+    red[tid] = xy;                 // the three sums reduced in one pass (red holds 3 x NTHR)
+    red[NTHR + tid] = xx;
+    red[2 * NTHR + tid] = yy;
     __syncthreads();
     if (tid < TB) {
-      float s = 0.f;
-      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
-      r3[tid * 16 + 8] = s;
-    }
-    __syncthreads();
-    red[tid] = xx;
-    __syncthreads();
-    if (tid < TB) {
-      float s = 0.f;
-      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
-      r3[tid * 16 + 9] = s;
-    }
-    __syncthreads();
-    red[tid] = yy;
-    __syncthreads();
-    if (tid < TB) {
-      float s = 0.f;
-      for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + tid];
-      const float sxy = r3[tid * 16 + 8], sxx = r3[tid * 16 + 9];
-      nuT[tid] = 1.f - sxy / (sqrtf(sxx) * sqrtf(s) + a.eps);
+      float sxy = 0.f, sxx = 0.f, syy = 0.f;
+      for (int p = 0; p < NTHR / TB; ++p) {
+        sxy += red[p * TB + tid];
+        sxx += red[NTHR + p * TB + tid];
+        syy += red[2 * NTHR + p * TB + tid];
+      }
+      nuT[tid] = 1.f - sxy / (sqrtf(sxx) * sqrtf(syy) + a.eps);
     }
   } else {
     if (tid < TB) nuT[tid] = 0.f;
@@ -536,14 +536,15 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
   __syncthreads();
 
   // 7. f_theta hidden = SiLU(W_th1 [s; c; nu] + b) -> big region
-  bmm4(sT, ds + DM + 1, a.w.th_w1_t, a.d_head, a.w.th_b1, bigT, 0, true);
+  bmm4<TB>(sT, ds + DM + 1, a.w.th_w1_t, a.d_head, a.w.th_b1, bigT, 0, true, skT,
+           RouterLayout<TB>::kSplitScratch);
 
   // 8. a = w_th2 . hidden + b (Eq. 14)
   {
     const int tl = tid % TB, part = tid / TB;
     float sa = 0.f;
     for (int i = part; i < a.d_head; i += NTHR / TB) sa = fmaf(__ldg(a.w.th_w2 + i), bigT[i * TB + tl], sa);
-    reduce16(red, sa, ab);
+    reduce16<TB>(red, sa, ab);
   }
 
   // 9. history score, cumulative score, gate and decision
@@ -742,29 +743,35 @@ cudaError_t launch_state_reset(float* S, float* zeta, float* pst, float* mst, fl
   return cudaGetLastError();
 }
 
-template <int DM>
-static cudaError_t launch_router_dm(const RouterArgs& a, cudaStream_t st) {
-  const RouterLayout lay(a.d_enc, a.d_head, a.d_h + a.d_a, DM, a.d_path);
+template <int DM, int TB>
+static cudaError_t launch_router_tb(const RouterArgs& a, cudaStream_t st) {
+  const RouterLayout<TB> lay(a.d_enc, a.d_head, a.d_h + a.d_a, DM, a.d_path);
   const size_t smem = sizeof(float) * (size_t)lay.floats;
   static size_t attr = 0;
   if (smem > attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_router<DM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(k_router<DM, TB>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr = smem;
   }
-  k_router<DM><<<(a.T + TB - 1) / TB, NTHR, smem, st>>>(a);
+  k_router<DM, TB><<<(a.T + TB - 1) / TB, NTHR, smem, st>>>(a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_router(int d_m, const RouterArgs& a, cudaStream_t st) {
+template <int DM>
+static cudaError_t launch_router_dm(const RouterArgs& a, int num_sms, cudaStream_t st) {
+  if ((a.T + TB_LARGE - 1) / TB_LARGE < 2 * num_sms) return launch_router_tb<DM, TB_SMALL>(a, st);
+  return launch_router_tb<DM, TB_LARGE>(a, st);
+}
+
+cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
   switch (d_m) {
-    case 16: return launch_router_dm<16>(a, st);
-    case 32: return launch_router_dm<32>(a, st);
-    case 64: return launch_router_dm<64>(a, st);
-    case 128: return launch_router_dm<128>(a, st);
-    case 256: return launch_router_dm<256>(a, st);
+    case 16: return launch_router_dm<16>(a, num_sms, st);
+    case 32: return launch_router_dm<32>(a, num_sms, st);
+    case 64: return launch_router_dm<64>(a, num_sms, st);
+    case 128: return launch_router_dm<128>(a, num_sms, st);
+    case 256: return launch_router_dm<256>(a, num_sms, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -212,3 +212,41 @@ def test_full_size_sampled(hero, name, bypass, n_sample):
     st.close()
     del gpu_all
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name", ["small_bf16", "llama31_8b_decode"])
+def test_cuda_graph_replay_matches_eager(hero, name):
+    """One stack call captured into a CUDA graph replays to the eager result, bit for bit
+    (no host synchronisation inside the call; the decode shape runs the split-K GEMMs)."""
+    import torch
+    inp = pr.inputs(name)
+    cfg = inp.cfg
+    T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
+    st = _stack(hero, inp)
+    dev = torch.device("cuda")
+    h = torch.from_numpy(np.ascontiguousarray(inp.h)).to(dev)
+    P = torch.from_numpy(np.ascontiguousarray(inp.P)).to(dev)
+    outs = [torch.empty((T, d), device=dev), torch.empty((L, T), device=dev),
+            torch.empty((L, T), dtype=torch.uint8, device=dev),
+            torch.empty((L,), dtype=torch.int32, device=dev)]
+    st(h, P, inp.tau, h_out=outs[0], gate_out=outs[1], mask_out=outs[2], counts_out=outs[3])
+    torch.cuda.synchronize()
+    eager = [o.clone() for o in outs]
+    for o in outs:
+        o.zero_()
+    graph = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.graph(graph, stream=cap):
+        st(h, P, inp.tau, h_out=outs[0], gate_out=outs[1], mask_out=outs[2], counts_out=outs[3],
+           stream=cap)
+    torch.cuda.current_stream().wait_stream(cap)
+    for o in outs:
+        o.zero_()
+    graph.replay()
+    graph.replay()
+    torch.cuda.synchronize()
+    st.check()
+    for a, b in zip(outs, eager):
+        assert torch.equal(a, b)
+    st.close()
