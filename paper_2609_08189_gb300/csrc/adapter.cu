@@ -33,6 +33,7 @@ __device__ __forceinline__ float to_f32(float v) { return v; }
 // partial-sum slot of the model (64 or 256).
 template <int SLOT, typename WT>
 __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
+  pdl_enter();
   extern __shared__ __align__(16) float smem_au[];
   float* ahs = smem_au;                                         // [AU_ROWS][AU_DR] fp32
   WT* w2s = reinterpret_cast<WT*>(smem_au + AU_ROWS * AU_DR);   // [AU_COLS][AU_WLD]
@@ -135,8 +136,7 @@ cudaError_t launch_au(const AdapterUpArgs& a, cudaStream_t st) {
     attr = true;
   }
   dim3 grid((a.d + AU_COLS - 1) / AU_COLS, (a.m_max + AU_ROWS - 1) / AU_ROWS);
-  k_adapter_up<SLOT, WT><<<grid, 256, au_smem<WT>(), st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_adapter_up<SLOT, WT>, grid, dim3(256), au_smem<WT>(), st, a);
 }
 
 }  // namespace

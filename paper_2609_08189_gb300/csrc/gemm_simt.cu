@@ -15,6 +15,7 @@ constexpr int TM = 64, TN = kSimtTileN, TK = 16;
 
 template <int EPI>
 __global__ void __launch_bounds__(256) k_gemm_simt(const GemmArgs a) {
+  pdl_enter();
   constexpr bool DUAL = EPI == EPI_SWIGLU;
   __shared__ float As[TK][TM + 4];
   __shared__ float Bs[TK][TN + 4];
@@ -123,13 +124,15 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const GemmArgs a) {
 cudaError_t launch_gemm_simt(EpiKind epi, const GemmArgs& a, cudaStream_t st) {
   if (a.m_max <= 0) return cudaSuccess;
   dim3 grid((a.N + TN - 1) / TN, (a.m_max + TM - 1) / TM);
+  cudaError_t e = cudaErrorInvalidValue;
   switch (epi) {
-    case EPI_STORE_F32: k_gemm_simt<EPI_STORE_F32><<<grid, 256, 0, st>>>(a); break;
-    case EPI_SWIGLU: k_gemm_simt<EPI_SWIGLU><<<grid, 256, 0, st>>>(a); break;
-    case EPI_SILU: k_gemm_simt<EPI_SILU><<<grid, 256, 0, st>>>(a); break;
-    case EPI_LAYER_OUT: k_gemm_simt<EPI_LAYER_OUT><<<grid, 256, 0, st>>>(a); break;
+    case EPI_STORE_F32: e = launch_pdl(k_gemm_simt<EPI_STORE_F32>, grid, dim3(256), 0, st, a); break;
+    case EPI_SWIGLU: e = launch_pdl(k_gemm_simt<EPI_SWIGLU>, grid, dim3(256), 0, st, a); break;
+    case EPI_SILU: e = launch_pdl(k_gemm_simt<EPI_SILU>, grid, dim3(256), 0, st, a); break;
+    case EPI_LAYER_OUT: e = launch_pdl(k_gemm_simt<EPI_LAYER_OUT>, grid, dim3(256), 0, st, a); break;
+    default: break;
   }
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace hero

@@ -300,6 +300,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
               const GemmArgs a0, const GemmArgs a1) {
+  pdl_enter();
   using C = TcCfg<BN, epi_warps<EPI0>()>;
   constexpr bool kGrouped = EPI1 != EPI_NONE;
   extern __shared__ uint8_t smem_raw[];
@@ -513,8 +514,8 @@ cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const Ge
   if (EPI1 != EPI_NONE) max_tiles += (long)((a1.m_max + BM - 1) / BM) * ((a1.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
   const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
-  k_gemm_tc<BN, EPI0, EPI1><<<grid, C::THREADS, C::SMEM, st>>>(tmA0, tmB0, tmA1, tmB1, a0, a1);
-  return cudaGetLastError();
+  return launch_pdl(k_gemm_tc<BN, EPI0, EPI1>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tmA0, tmB0,
+                    tmA1, tmB1, a0, a1);
 }
 
 }  // namespace

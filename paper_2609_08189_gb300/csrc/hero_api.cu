@@ -126,7 +126,10 @@ struct hero_model {
   size_t io_bytes = 0;
   cudaStream_t copy_stream = nullptr;
   std::vector<cudaEvent_t> ev_ready, ev_consumed;  // per routed block
-  cudaEvent_t ev_start = nullptr;
+  // recorded on the compute stream after the last kernel of every call: the next
+  // host-IO call's uploads into the workspace wait for it, not for the previous
+  // call's result downloads, so both directions overlap
+  cudaEvent_t ev_kernels_done = nullptr;
 
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
@@ -277,7 +280,7 @@ void free_model(hero_model* m) {
   for (auto e : m->event_pool) cudaEventDestroy(e);
   for (auto e : m->ev_ready) cudaEventDestroy(e);
   for (auto e : m->ev_consumed) cudaEventDestroy(e);
-  if (m->ev_start) cudaEventDestroy(m->ev_start);
+  if (m->ev_kernels_done) cudaEventDestroy(m->ev_kernels_done);
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io};
@@ -560,6 +563,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     }
     if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
   }
+  CUDA_M(cudaEventCreateWithFlags(&m->ev_kernels_done, cudaEventDisableTiming));
   *out = m;
   return HERO_OK;
 #undef TRY_M
@@ -782,6 +786,9 @@ struct PFeed {
   const char* host;     // [L, T, d] in the model's operand type
   char* slots;          // 3 device slots of one block each
   size_t layer_bytes;
+  const void* h0;       // host h_0, uploaded on the copy stream ahead of P_1
+  void* h0_dst;
+  size_t h0_bytes;
 };
 constexpr int kPSlots = 3;
 
@@ -813,9 +820,11 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
     return P ? static_cast<const char*>(P) + (size_t)k * layer_elems * es : nullptr;
   };
   if (feed) {
-    // the slots may still be read by the previous call's kernels on `st`
-    CUDA_TRY(cudaEventRecord(m->ev_start, st));
-    CUDA_TRY(cudaStreamWaitEvent(m->copy_stream, m->ev_start, 0));
+    // h_bar and the slots may still be read by the previous call's kernels
+    CUDA_TRY(cudaStreamWaitEvent(m->copy_stream, m->ev_kernels_done, 0));
+    if (feed->h0)
+      CUDA_TRY(cudaMemcpyAsync(feed->h0_dst, feed->h0, feed->h0_bytes, cudaMemcpyHostToDevice,
+                               m->copy_stream));
     for (int k = 0; k < L && k < kPSlots; ++k) {
       hero_status s = feed_copy(m, *feed, k, st, false);
       if (s != HERO_OK) return s;
@@ -874,6 +883,7 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
       }
     }
   }
+  CUDA_TRY(cudaEventRecord(m->ev_kernels_done, st));
   return HERO_OK;
 }
 
@@ -925,10 +935,8 @@ extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, co
   const size_t p_layer_bytes = (size_t)T * d * esz;
   const size_t p_bytes = attn_delta ? (size_t)kPSlots * p_layer_bytes : 0;   // upload ring
   const size_t lt = (size_t)L * T;
-  if (attn_delta && !m->copy_stream) {
+  if (attn_delta && !m->copy_stream)
     CUDA_TRY(cudaStreamCreateWithFlags(&m->copy_stream, cudaStreamNonBlocking));
-    CUDA_TRY(cudaEventCreateWithFlags(&m->ev_start, cudaEventDisableTiming));
-  }
   while (attn_delta && (int)m->ev_ready.size() < L) {
     cudaEvent_t a = nullptr, b = nullptr;
     CUDA_TRY(cudaEventCreateWithFlags(&a, cudaEventDisableTiming));
@@ -952,10 +960,12 @@ extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, co
   float* d_gate = gate_out ? reinterpret_cast<float*>(carve(lt * 4)) : nullptr;
   uint8_t* d_mask = mask_out ? reinterpret_cast<uint8_t*>(carve(lt)) : nullptr;
   int32_t* d_cnt = ffn_count_out ? reinterpret_cast<int32_t*>(carve((size_t)L * 4)) : nullptr;
-  // h_0 goes straight into the h_bar buffer; k_init adds P_1 in place.
-  CUDA_TRY(cudaMemcpyAsync(m->hbar, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
+  // h_0 goes straight into the h_bar buffer (k_init adds P_1 in place): on the copy
+  // stream ahead of P_1 when P is streamed, else on the compute stream.
+  if (!attn_delta) CUDA_TRY(cudaMemcpyAsync(m->hbar, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
   if (d_mask_in) CUDA_TRY(cudaMemcpyAsync(d_mask_in, mask_in, lt, cudaMemcpyHostToDevice, st));
-  PFeed feed{static_cast<const char*>(attn_delta), static_cast<char*>(d_P), p_layer_bytes};
+  PFeed feed{static_cast<const char*>(attn_delta), static_cast<char*>(d_P), p_layer_bytes,
+             h_in, m->hbar, (size_t)T * d * 4};
   s = run_stack(m, T, m->hbar, nullptr, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask, d_cnt,
                 st, attn_delta ? &feed : nullptr);
   if (s != HERO_OK) return s;
@@ -1037,9 +1047,12 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
   lo.p_bf16 = m->bf16;
   lo.xl_bf16 = m->bf16;
   lo.router = 0;
-  return block_body(m, jj, jr, T, bs, h_bar, lo, tau_exec, flags,
-                    (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr, gate_out, mask_out,
-                    ffn_count_out, st);
+  const hero_status sb = block_body(m, jj, jr, T, bs, h_bar, lo, tau_exec, flags,
+                                    (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr, gate_out,
+                                    mask_out, ffn_count_out, st);
+  if (sb != HERO_OK) return sb;
+  CUDA_TRY(cudaEventRecord(m->ev_kernels_done, st));
+  return HERO_OK;
 }
 
 extern "C" hero_status hero_check_device_status(hero_model* m, void* cuda_stream) {

@@ -8,6 +8,25 @@
 
 namespace hero {
 
+// Launch `kernel` on `st` with programmatic stream serialisation: its launch may
+// overlap the tail of the previous kernel on the stream; the kernel itself waits
+// (pdl_enter) for that kernel's completion before touching memory.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // Device error word bits (set by kernels, read by hero_check_device_status).
 enum : uint32_t {
   ERR_WAIT_PRODUCER = 1u,

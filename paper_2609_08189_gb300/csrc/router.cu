@@ -20,6 +20,7 @@ namespace {
 // k_init: one warp per token.
 // ------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_init(const InitArgs a) {
+  pdl_enter();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= a.T) return;
@@ -62,6 +63,7 @@ __global__ void __launch_bounds__(256) k_init(const InitArgs a) {
 // block's (each element is read before it is overwritten by the same lane).
 // ------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_block_entry(const BlockEntryArgs a) {
+  pdl_enter();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= a.T) return;
@@ -98,6 +100,7 @@ __global__ void __launch_bounds__(256) k_block_entry(const BlockEntryArgs a) {
 // Router state reset for a new forward pass (S = 0, zeta = 0, p = m = 1, d_prev = 0).
 __global__ void __launch_bounds__(256) k_state_reset(float* S, float* zeta, float* pst, float* mst,
                                                      float* dprev, int T, int dm) {
+  pdl_enter();
   const long n_s = (long)T * dm * dm;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n_s; i += (long)gridDim.x * blockDim.x) {
     S[i] = 0.f;
@@ -342,6 +345,7 @@ __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const flo
 
 template <int DM, int TB>
 __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const RouterArgs a) {
+  pdl_enter();
   extern __shared__ __align__(16) float sm[];
   const int ds = a.d_h + a.d_a;
   const RouterLayout<TB> lay(a.d_enc, a.d_head, ds, DM, a.d_path);
@@ -582,6 +586,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
 constexpr int CT = 1024, SEGS = 16;
 
 __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
+  pdl_enter();
   __shared__ int wsum[CT / 32];
   __shared__ int carry_s;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -653,6 +658,7 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
 // row is then streamed with up to eight float4 loads per lane in flight.
 // ------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_norm(const NormArgs a) {
+  pdl_enter();
   const long slot = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (slot >= a.T) return;
@@ -723,14 +729,12 @@ __global__ void k_convert(const void* src, int src_bf16, void* dst, int dst_bf16
 cudaError_t launch_init(const InitArgs& a, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
   const int warps_per_block = 8;
-  k_init<<<(a.T + warps_per_block - 1) / warps_per_block, 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_init, dim3((a.T + warps_per_block - 1) / warps_per_block), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_block_entry(const BlockEntryArgs& a, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
-  k_block_entry<<<(a.T + 7) / 8, 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_block_entry, dim3((a.T + 7) / 8), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_state_reset(float* S, float* zeta, float* pst, float* mst, float* dprev, int T,
@@ -739,8 +743,8 @@ cudaError_t launch_state_reset(float* S, float* zeta, float* pst, float* mst, fl
   long n = (long)T * dm * dm;
   long blocks = (n + 255) / 256;
   if (blocks > 8192) blocks = 8192;
-  k_state_reset<<<(unsigned)blocks, 256, 0, st>>>(S, zeta, pst, mst, dprev, T, dm);
-  return cudaGetLastError();
+  return launch_pdl(k_state_reset, dim3((unsigned)blocks), dim3(256), 0, st, S, zeta, pst, mst, dprev,
+                    T, dm);
 }
 
 template <int DM, int TB>
@@ -754,8 +758,7 @@ static cudaError_t launch_router_tb(const RouterArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr = smem;
   }
-  k_router<DM, TB><<<(a.T + TB - 1) / TB, NTHR, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_router<DM, TB>, dim3((a.T + TB - 1) / TB), dim3(NTHR), smem, st, a);
 }
 
 template <int DM>
@@ -777,14 +780,12 @@ cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_
 }
 
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st) {
-  k_compact<<<1, CT, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_compact, dim3(1), dim3(CT), 0, st, a);
 }
 
 cudaError_t launch_norm(const NormArgs& a, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
-  k_norm<<<(unsigned)((a.T + 7) / 8), 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_norm, dim3((unsigned)((a.T + 7) / 8)), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_convert_rows(const void* src, int src_bf16, void* dst, int dst_bf16, long rows,

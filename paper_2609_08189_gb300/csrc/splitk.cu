@@ -11,6 +11,7 @@ namespace {
 __global__ void __launch_bounds__(256) k_splitk_sum(const float* __restrict__ part, int splits,
                                                     long split_stride, int M, int N,
                                                     float* __restrict__ out) {
+  pdl_enter();
   const int n4 = N >> 2;
   const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (long)M * n4) return;
@@ -31,6 +32,7 @@ __global__ void __launch_bounds__(256) k_splitk_sum(const float* __restrict__ pa
 __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ part, int splits,
                                                       long split_stride, int ld, const int* m_dev,
                                                       int m_max, const LayerOutArgs lo) {
+  pdl_enter();
   static_assert(kTcPartCols == 128, "one warp covers one 128-column slot with float4 lanes");
   int M = *m_dev;
   if (M < 0 || M > m_max) M = 0;
@@ -69,9 +71,8 @@ cudaError_t launch_splitk_sum(const float* part, int splits, long split_stride, 
   if (M <= 0) return cudaSuccess;
   if (N % 4) return cudaErrorInvalidValue;
   const long threads = (long)M * (N / 4);
-  k_splitk_sum<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(part, splits, split_stride, M, N,
-                                                                  out);
-  return cudaGetLastError();
+  return launch_pdl(k_splitk_sum, dim3((unsigned)((threads + 255) / 256)), dim3(256), 0, st, part,
+                    splits, split_stride, M, N, out);
 }
 
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
@@ -80,9 +81,8 @@ cudaError_t launch_splitk_close(const float* part, int splits, long split_stride
   if (m_max <= 0) return cudaSuccess;
   if (lo.d % kTcPartCols) return cudaErrorInvalidValue;
   const long warps = (long)m_max * (lo.d / kTcPartCols);
-  k_splitk_close<<<(unsigned)((warps + 7) / 8), 256, 0, st>>>(part, splits, split_stride, ld, m_dev,
-                                                              m_max, lo);
-  return cudaGetLastError();
+  return launch_pdl(k_splitk_close, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, part, splits,
+                    split_stride, ld, m_dev, m_max, lo);
 }
 
 }  // namespace hero
