@@ -2,10 +2,11 @@
 // tokens routed to the adapter):
 //   y = W_2 SiLU(W_1 u)   (the SiLU(W_1 u) rows come from the adapter-down GEMM)
 //   h = h_bar + (1 - g) y, then the next block's h_bar, delta and partial sums.
-// f32 models only (bf16 models run the adapter's up projection on the tensor
-// cores, grouped into the FFN down GEMM's launch).  The contraction has depth d_r
-// (<= 64), i.e. 2 d_r FLOP per output element against 20 bytes of epilogue
-// traffic, so it runs on the FMA pipes with row-contiguous global access.
+// Used by f32 models, and by bf16 models when the token count is small (decode),
+// where the tensor-core launch's fixed latency dominates; large bf16 batches run
+// the up projection as a tensor-core GEMM.  The contraction has depth d_r (<= 64),
+// i.e. 2 d_r FLOP per output element against 22 bytes of epilogue traffic, so it
+// runs on the FMA pipes with row-contiguous global access.
 //
 // CTA: 32 adapter rows x 256 output columns, 256 threads.  Warp w owns rows
 // 4w..4w+3; lane x owns columns x + 32 j (j < 8), so every warp instruction of
@@ -144,6 +145,7 @@ cudaError_t launch_au(const AdapterUpArgs& a, cudaStream_t st) {
 cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st) {
   if (a.m_max <= 0) return cudaSuccess;
   if (a.d_r > AU_DR) return cudaErrorInvalidValue;
+  if (a.bf16 && a.slot_cols == 128) return launch_au<128, uint16_t>(a, st);
   if (!a.bf16 && a.slot_cols == 64) return launch_au<64, float>(a, st);
   return cudaErrorInvalidValue;
 }

@@ -632,10 +632,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
                      : launch_gemm_simt(EPI_STORE_F32, g, st);
     }));
-    if (rs > 1)
-      CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
-        return launch_splitk_sum(m->splitk_ws, rs, g.split_stride, T, nY, m->Y, st);
-      }));
+
     RouterArgs ra{};
     ra.T = T;
     ra.j = j;
@@ -647,7 +644,9 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.d_enc = c.d_enc;
     ra.d_head = c.d_head;
     ra.d_path = c.d_path;
-    ra.Y = m->Y;
+    ra.Y = rs > 1 ? m->splitk_ws : m->Y;   // the router adds split-K slices as it reads
+    ra.y_splits = rs > 1 ? rs : 1;
+    ra.y_split_stride = rs > 1 ? g.split_stride : 0;
     ra.part = m->part;
     ra.dprev = bs.dprev;
     ra.pst = bs.pst;
@@ -674,7 +673,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
   CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
   NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, hbar, m->part,
               m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
-  CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, st); }));
+  CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, m->num_sms, st); }));
 
   // FFN branch: gate/up + SwiGLU, then down + scaled scatter.  The adapter branch
   // (the other token rows): W_1 with SiLU, then W_2 + scaled scatter; on bf16
@@ -732,10 +731,23 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
                    : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU, m->tm_ua,
                                          m->tm_w1[jj], ad, m->num_sms, st);
     }));
-    if (!dense)   // epilogue-bound (rank-d_r contraction): the wide-epilogue variant
+    if (!dense && T <= 256 && r <= 64) {   // few rows: the latency-light FMA-pipe kernel
+      AdapterUpArgs ua{};
+      ua.m_dev = m->counts + 1;
+      ua.m_max = T;
+      ua.d = d;
+      ua.d_r = r;
+      ua.ah = m->ah;
+      ua.w2 = static_cast<const char*>(m->w2) + (size_t)jj * d * r * es;
+      ua.bf16 = 1;
+      ua.slot_cols = kTcPartCols;
+      ua.lo = au.lo;
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] { return launch_adapter_up(ua, st); }));
+    } else if (!dense) {   // epilogue-bound (rank-d_r contraction): the wide-epilogue variant
       CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
         return launch_gemm_tc(256, EPI_LAYER_OUT_WIDE, m->tm_ah, m->tm_w2[jj], au, m->num_sms, st);
       }));
+    }
     const int m_t = (T + 127) / 128;
     const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
     if (ds > 1) {   // few tiles (small T): split K into partials, then the closing epilogue

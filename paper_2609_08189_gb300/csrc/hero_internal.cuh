@@ -153,7 +153,11 @@ struct RouterWeights {   // shared router parameters, fp32, transposed to [in][o
 struct RouterArgs {
   int T, j, L, np;       // j is 1-based
   int d, d_h, d_a, d_enc, d_head, d_path;
-  const float* Y;        // [T, d_enc + d_head] router contraction output
+  const float* Y;        // [T, d_enc + d_head] router contraction output, or its y_splits
+                         // split-K partial slices y_split_stride floats apart (summed in
+                         // slice order as they are read)
+  int y_splits;
+  long y_split_stride;
   const float* part;     // [T, np, 4]
   float* dprev;          // [T] in: d_{j-1}; out: d_j
   float* pst;            // [T] p_hist
@@ -238,7 +242,8 @@ struct NormArgs {
   void* u_a;             // [T, d]
   int out_bf16;
 };
-cudaError_t launch_norm(const NormArgs& a, cudaStream_t st);
+// wpr: warps per row (each takes a contiguous d / wpr column range; wpr divides d / 4)
+cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st);
 
 // Adapter up-projection plus the block-closing epilogue, for the adapter rows:
 // y[m, :] = W_2 ah[m, :] (rank d_r = 64 contraction), then LayerOutArgs on token
@@ -256,13 +261,9 @@ struct AdapterUpArgs {
 };
 cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st);
 
-// Split-K finishing kernels (few-tile launches, e.g. decode): fixed-order sums of
-// the k_splits partial slices [s][rows][ld] written by a split tensor-core GEMM.
-//   sum:   out[m, n] = sum_s part[s, m, n]                     (m < M, n < N)
-//   close: y = sum_s part[s, m, n], then the block-closing epilogue (LayerOutArgs)
-//          on token idx[m] for m < *m_dev, with kTcPartCols-column partial sums
-cudaError_t launch_splitk_sum(const float* part, int splits, long split_stride, int M, int N,
-                              float* out, cudaStream_t st);
+// Split-K finishing kernel (few-tile launches, e.g. decode): y = sum_s part[s, m, n]
+// over the k_splits partial slices in slice order, then the block-closing epilogue
+// (LayerOutArgs) on token idx[m] for m < *m_dev, with kTcPartCols-column partial sums.
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
                                 cudaStream_t st);

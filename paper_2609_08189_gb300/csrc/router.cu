@@ -445,7 +445,14 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
 #pragma unroll
       for (int k = 0; k < YB; ++k) {
         const int g = g0 + k * (NTHR / TB);
-        yv[k] = (tok0 < a.T && g < ng) ? __ldg(yrow + g) : make_float4(0.f, 0.f, 0.f, 0.f);
+        yv[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (tok0 < a.T && g < ng) {
+          yv[k] = __ldg(yrow + g);
+          for (int sp = 1; sp < a.y_splits; ++sp) {   // split-K slices, in slice order
+            const float4 v = __ldg(yrow + (size_t)sp * (a.y_split_stride / 4) + g);
+            yv[k].x += v.x; yv[k].y += v.y; yv[k].z += v.z; yv[k].w += v.w;
+          }
+        }
       }
 #pragma unroll
       for (int k = 0; k < YB; ++k) {
@@ -652,14 +659,18 @@ __global__ void __launch_bounds__(CT) k_compact(const CompactArgs a) {
 }
 
 // ------------------------------------------------------------------------------
-// k_norm: one warp per branch row; slot s < n_f is FFN row s (token idx_f[s]),
-// slot s >= n_f is adapter row s - n_f.  The row's 1/rms comes from the
-// epilogue's partial sums (lane-parallel loads, fixed-order warp reduction); the
-// row is then streamed with up to eight float4 loads per lane in flight.
+// k_norm: wpr warps per branch row (1 for large T; more when few rows would leave
+// the GPU idle), each over a contiguous column range; slot s < n_f is FFN row s
+// (token idx_f[s]), slot s >= n_f is adapter row s - n_f.  The row's 1/rms comes
+// from the epilogue's partial sums (lane-parallel loads, fixed-order warp
+// reduction); the columns are streamed with up to eight float4 loads per lane in
+// flight.
 // ------------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_norm(const NormArgs a) {
+__global__ void __launch_bounds__(256) k_norm(const NormArgs a, int wpr) {
   pdl_enter();
-  const long slot = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const long gw = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const long slot = gw / wpr;
+  const int part = (int)(gw - slot * wpr);
   const int lane = threadIdx.x & 31;
   if (slot >= a.T) return;
   const int nf = a.counts[0];
@@ -679,20 +690,22 @@ __global__ void __launch_bounds__(256) k_norm(const NormArgs a) {
   for (int s = lane; s < a.np; s += 32) ss += a.part[((size_t)t * a.np + s) * 4];
   ss = warp_sum(ss);
   const float rinv = rsqrtf(ss / (float)a.d + a.rms_eps);
+  const int cols = a.d / wpr;
+  const int c_lo = part * cols, c_hi = c_lo + cols;
   const float* h = a.hbar + (size_t)t * a.d;
   const size_t ro = (size_t)r * a.d;
   constexpr int NB = 8;
-  for (int c0 = lane * 4; c0 < a.d; c0 += 128 * NB) {
+  for (int c0 = c_lo + lane * 4; c0 < c_hi; c0 += 128 * NB) {
     float4 hv[NB];
 #pragma unroll
     for (int k = 0; k < NB; ++k) {
       const int c = c0 + 128 * k;
-      if (c < a.d) hv[k] = *reinterpret_cast<const float4*>(h + c);
+      if (c < c_hi) hv[k] = *reinterpret_cast<const float4*>(h + c);
     }
 #pragma unroll
     for (int k = 0; k < NB; ++k) {
       const int c = c0 + 128 * k;
-      if (c < a.d) {
+      if (c < c_hi) {
         const float4 g = __ldg(reinterpret_cast<const float4*>(a.gain + c));
         store4(dst, ro + c,
                make_float4(hv[k].x * rinv * g.x, hv[k].y * rinv * g.y, hv[k].z * rinv * g.z,
@@ -783,9 +796,15 @@ cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st) {
   return launch_pdl(k_compact, dim3(1), dim3(CT), 0, st, a);
 }
 
-cudaError_t launch_norm(const NormArgs& a, cudaStream_t st) {
+cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
-  return launch_pdl(k_norm, dim3((unsigned)((a.T + 7) / 8)), dim3(256), 0, st, a);
+  // split rows across warps until there are ~16 warps per SM (column ranges stay
+  // whole multiples of 4 elements)
+  int wpr = 1;
+  while ((long)a.T * wpr * 2 <= 16L * num_sms && (a.d / (wpr * 2)) % 4 == 0 && a.d / (wpr * 2) >= 128)
+    wpr *= 2;
+  const long warps = (long)a.T * wpr;
+  return launch_pdl(k_norm, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, a, wpr);
 }
 
 cudaError_t launch_convert_rows(const void* src, int src_bf16, void* dst, int dst_bf16, long rows,

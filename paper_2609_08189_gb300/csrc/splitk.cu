@@ -1,30 +1,12 @@
-// Finishing kernels of split-K tensor-core GEMMs.  Launches with few output tiles
+// Finishing kernel of the split-K FFN down GEMM.  Launches with few output tiles
 // (a decode step: 64 tokens give the router contraction 2 tiles and the FFN down
 // GEMM 16) split K so that every SM streams weights; the k_splits fp32 partial
-// slices are added here in a fixed order, so results do not depend on scheduling.
+// slices are added in a fixed order, so results do not depend on scheduling (the
+// router kernel adds the router contraction's slices the same way as it reads them).
 #include "hero_device.cuh"
 
 namespace hero {
 namespace {
-
-// out[m, n] = sum_s part[s][m][n]; one thread per 4 consecutive columns.
-__global__ void __launch_bounds__(256) k_splitk_sum(const float* __restrict__ part, int splits,
-                                                    long split_stride, int M, int N,
-                                                    float* __restrict__ out) {
-  pdl_enter();
-  const int n4 = N >> 2;
-  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (long)M * n4) return;
-  const long m = i / n4;
-  const int n = (int)(i - m * n4) * 4;
-  const size_t off = (size_t)m * N + n;
-  float4 acc = *reinterpret_cast<const float4*>(part + off);
-  for (int s = 1; s < splits; ++s) {
-    const float4 v = *reinterpret_cast<const float4*>(part + (size_t)s * split_stride + off);
-    acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
-  }
-  *reinterpret_cast<float4*>(out + off) = acc;
-}
 
 // Block-closing epilogue over the summed partials: one warp per (row, partial-sum
 // slot of kTcPartCols columns); lane owns 4 consecutive columns and the slot's
@@ -65,15 +47,6 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
 }
 
 }  // namespace
-
-cudaError_t launch_splitk_sum(const float* part, int splits, long split_stride, int M, int N,
-                              float* out, cudaStream_t st) {
-  if (M <= 0) return cudaSuccess;
-  if (N % 4) return cudaErrorInvalidValue;
-  const long threads = (long)M * (N / 4);
-  return launch_pdl(k_splitk_sum, dim3((unsigned)((threads + 255) / 256)), dim3(256), 0, st, part,
-                    splits, split_stride, M, N, out);
-}
 
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
