@@ -220,15 +220,27 @@ __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int 
   }
 }
 
-// Sum the 16 per-thread partials of each token (thread t + 16 p holds partial p of
-// token t) in a fixed order; contains __syncthreads.
+// Within a warp, add the partials of the lanes that serve the same token (lane %
+// TB) with a fixed shuffle tree; lanes < TB then hold the warp's sum per token.
+template <int TB>
+__device__ __forceinline__ float warp_part_sum(float v) {
+#pragma unroll
+  for (int o = TB; o < 32; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum the NTHR / TB per-thread partials of each token (thread tid holds a partial of
+// token tid % TB): a shuffle tree inside each warp, then the warps' sums in warp
+// order (fixed, so bitwise reproducible); contains __syncthreads.
 template <int TB>
 __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
-  red[threadIdx.x] = v;
+  v = warp_part_sum<TB>(v);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane < TB) red[warp * TB + lane] = v;
   __syncthreads();
   if (threadIdx.x < TB) {
     float s = 0.f;
-    for (int p = 0; p < NTHR / TB; ++p) s += red[p * TB + threadIdx.x];
+    for (int w = 0; w < NTHR / 32; ++w) s += red[w * TB + threadIdx.x];
     out[threadIdx.x] = s;
   }
   __syncthreads();
@@ -394,18 +406,23 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
         dd += v.y;
         dp += v.z;
       }
-    red[tid] = ss;
-    red[NTHR + tid] = dd;
-    red[2 * NTHR + tid] = dp;
+    ss = warp_part_sum<TB>(ss);
+    dd = warp_part_sum<TB>(dd);
+    dp = warp_part_sum<TB>(dp);
+    if (lane < TB) {
+      red[warp * TB + lane] = ss;
+      red[NTHR + warp * TB + lane] = dd;
+      red[2 * NTHR + warp * TB + lane] = dp;
+    }
   }
   __syncthreads();
   if (tid < TB) {
     const int t = t0 + tid;
     float ss = 0.f, dd = 0.f, dp = 0.f, dprev = 0.f, pp = 1.f, mp = 1.f;
-    for (int p = 0; p < NTHR / TB; ++p) {
-      ss += red[p * TB + tid];
-      dd += red[NTHR + p * TB + tid];
-      dp += red[2 * NTHR + p * TB + tid];
+    for (int w = 0; w < NTHR / 32; ++w) {
+      ss += red[w * TB + tid];
+      dd += red[NTHR + w * TB + tid];
+      dp += red[2 * NTHR + w * TB + tid];
     }
     if (t < a.T) {
       dprev = a.dprev[t];
@@ -528,16 +545,21 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
       xx += u * u;
       yy += w * w;
     }
-    red[tid] = xy;                 // the three sums reduced in one pass (red holds 3 x NTHR)
-    red[NTHR + tid] = xx;
-    red[2 * NTHR + tid] = yy;
+    xy = warp_part_sum<TB>(xy);    // the three sums reduced in one pass
+    xx = warp_part_sum<TB>(xx);
+    yy = warp_part_sum<TB>(yy);
+    if (lane < TB) {
+      red[warp * TB + lane] = xy;
+      red[NTHR + warp * TB + lane] = xx;
+      red[2 * NTHR + warp * TB + lane] = yy;
+    }
     __syncthreads();
     if (tid < TB) {
       float sxy = 0.f, sxx = 0.f, syy = 0.f;
-      for (int p = 0; p < NTHR / TB; ++p) {
-        sxy += red[p * TB + tid];
-        sxx += red[NTHR + p * TB + tid];
-        syy += red[2 * NTHR + p * TB + tid];
+      for (int w = 0; w < NTHR / 32; ++w) {
+        sxy += red[w * TB + tid];
+        sxx += red[NTHR + w * TB + tid];
+        syy += red[2 * NTHR + w * TB + tid];
       }
       nuT[tid] = 1.f - sxy / (sqrtf(sxx) * sqrtf(syy) + a.eps);
     }
