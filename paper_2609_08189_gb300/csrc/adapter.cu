@@ -63,15 +63,40 @@ __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
     }
   }
 
-  for (int e = tid; e < AU_ROWS * dr; e += 256) {
-    const int r = e / dr, k = e % dr;
-    const int m = m0 + r;
-    ahs[r * AU_DR + k] = m < M ? to_f32(ah[(size_t)m * dr + k]) : 0.f;
-  }
-  for (int e = tid; e < AU_COLS * dr; e += 256) {
-    const int c = e / dr, k = e % dr;
-    const int n = n0 + c;
-    w2s[c * AU_WLD + k] = n < a.d ? w2[(size_t)n * dr + k] : WT(0);
+  constexpr int V = 16 / (int)sizeof(WT);   // elements per 16-byte vector
+  if (dr % V == 0) {   // 16-byte loads, several per thread in flight
+    const int vr = dr / V;
+#pragma unroll 4
+    for (int e = tid; e < AU_ROWS * vr; e += 256) {
+      const int r = e / vr, kv = (e - r * vr) * V;
+      const int m = m0 + r;
+      uint4 u = make_uint4(0u, 0u, 0u, 0u);
+      if (m < M) u = __ldg(reinterpret_cast<const uint4*>(ah + (size_t)m * dr + kv));
+      const WT* x = reinterpret_cast<const WT*>(&u);
+#pragma unroll
+      for (int i = 0; i < V; ++i) ahs[r * AU_DR + kv + i] = to_f32(x[i]);
+    }
+#pragma unroll 4
+    for (int e = tid; e < AU_COLS * vr; e += 256) {
+      const int c = e / vr, kv = (e - c * vr) * V;
+      const int n = n0 + c;
+      uint4 u = make_uint4(0u, 0u, 0u, 0u);
+      if (n < a.d) u = __ldg(reinterpret_cast<const uint4*>(w2 + (size_t)n * dr + kv));
+      const WT* x = reinterpret_cast<const WT*>(&u);
+#pragma unroll
+      for (int i = 0; i < V; ++i) w2s[c * AU_WLD + kv + i] = x[i];
+    }
+  } else {
+    for (int e = tid; e < AU_ROWS * dr; e += 256) {
+      const int r = e / dr, k = e % dr;
+      const int m = m0 + r;
+      ahs[r * AU_DR + k] = m < M ? to_f32(ah[(size_t)m * dr + k]) : 0.f;
+    }
+    for (int e = tid; e < AU_COLS * dr; e += 256) {
+      const int c = e / dr, k = e % dr;
+      const int n = n0 + c;
+      w2s[c * AU_WLD + k] = n < a.d ? w2[(size_t)n * dr + k] : WT(0);
+    }
   }
   __syncthreads();
 

@@ -873,7 +873,6 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
     lo.h_out = h_out;
     lo.d = d;
     lo.np = m->np;
-    lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
     lo.last = jj == L - 1;
     lo.first = jr <= 0;                       // delta_1 = 0; no delta before routing starts
     lo.p_bf16 = m->bf16;
@@ -1053,7 +1052,6 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
   lo.part = m->part;
   lo.d = c.d_model;
   lo.np = m->np;
-  lo.tile_n = m->bf16 ? kTcPartCols : kSimtTileN;
   lo.last = 1;
   lo.first = jr <= 0;
   lo.p_bf16 = m->bf16;

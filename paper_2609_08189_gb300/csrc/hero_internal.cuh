@@ -64,8 +64,7 @@ struct LayerOutArgs {
   float* part;           // [T, np, 4] out: partial sums per column tile
   float* h_out;          // [T, d] out (last block only)
   int d;
-  int np;                // partial slots per token
-  int tile_n;            // columns per partial slot
+  int np;                // partial slots per token (kTcPartCols or kSimtTileN columns each)
   int last;              // 1: write h_out only
   int first;             // 1: delta_j = 0 (do not read it)
   int p_bf16;            // P_{j+1} element type
