@@ -268,6 +268,59 @@ def adapter(u, wl, R):
 
 
 # ---------------------------------------------------------------------------
+# The attention sublayer of Eq. 1 (the full decoder forward)
+# ---------------------------------------------------------------------------
+# Readings (the paper keeps the backbone's attention, Sec. 3.1, and names Llama
+# backbones, Sec. 4.1): Llama attention without biases; LN_attn is RMSNorm with
+# its own gain; RoPE in the rotate-half form, inverse frequencies
+# theta^(-2i/hd); causal softmax(q k^T / sqrt(hd)) per sequence; grouped-query
+# heads (query head h reads key/value head h // (H / H_kv)).  Precision points
+# for bf16 workloads: x = LN_attn(h), q and k after RoPE, v, the softmax
+# probabilities entering P V, and the attention output entering W_o.
+
+def rope_cos_sin(seq_len: int, hd: int, theta: float):
+    """cos and sin tables [S, hd/2] of RoPE (position p, frequency theta^(-2i/hd))."""
+    inv = theta ** (-np.arange(0, hd, 2, dtype=np.float64) / hd)
+    ang = np.arange(seq_len, dtype=np.float64)[:, None] * inv[None, :]
+    return np.cos(ang), np.sin(ang)
+
+
+def apply_rope(x, cos, sin):
+    """Rotate-half RoPE on x [..., S, hd]: each pair (x_i, x_{i+hd/2}) is rotated by
+    position p times frequency i."""
+    h = x.shape[-1] // 2
+    x1, x2 = x[..., :h], x[..., h:]
+    return np.concatenate([x1 * cos - x2 * sin, x2 * cos + x1 * sin], axis=-1)
+
+
+def attention_sublayer(h, wa, n_heads: int, n_kv_heads: int, theta: float, n_seqs: int,
+                       seq_len: int, rms_eps: float, R=None):
+    """Eq. 1, first line: h_bar = h + Attn(LN_attn(h)) on n_seqs sequences of seq_len
+    tokens (rows of h in sequence order).  wa: attn_norm_g [d], w_q [H hd, d],
+    w_k / w_v [H_kv hd, d], w_o [d, H hd] (float64)."""
+    R = R or _identity
+    T, d = h.shape
+    hd = d // n_heads
+    x = R(rms_norm(h, wa["attn_norm_g"], rms_eps))
+    shape = lambda a, nh: a.reshape(n_seqs, seq_len, nh, hd).transpose(0, 2, 1, 3)
+    q = shape(x @ wa["w_q"].T, n_heads)
+    k = shape(x @ wa["w_k"].T, n_kv_heads)
+    v = shape(x @ wa["w_v"].T, n_kv_heads)
+    cos, sin = rope_cos_sin(seq_len, hd, theta)
+    q, k, v = R(apply_rope(q, cos, sin)), R(apply_rope(k, cos, sin)), R(v)
+    group = n_heads // n_kv_heads
+    k = np.repeat(k, group, axis=1)
+    v = np.repeat(v, group, axis=1)
+    scores = q @ k.transpose(0, 1, 3, 2) / np.sqrt(hd)                   # [B, H, S, S]
+    scores = np.where(np.tril(np.ones((seq_len, seq_len), dtype=bool)), scores, -np.inf)
+    scores = scores - scores.max(axis=-1, keepdims=True)
+    p = np.exp(scores)
+    p = R(p / p.sum(axis=-1, keepdims=True))
+    o = R(p @ v).transpose(0, 2, 1, 3).reshape(T, n_heads * hd)
+    return h + o @ wa["w_o"].T
+
+
+# ---------------------------------------------------------------------------
 # The stack
 # ---------------------------------------------------------------------------
 
@@ -280,10 +333,13 @@ _SHARED_KEYS = ("r_norm_g", "w_hd", "w_hu", "path_w1", "path_b1", "path_w2", "pa
 def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, attn_delta,
                      tau: float, mode: str = "route", mask_in=None,
                      branch_scale: str = "gate", record: bool = False,
-                     hooks: Optional[Dict[str, Callable]] = None) -> Dict[str, object]:
+                     hooks: Optional[Dict[str, Callable]] = None,
+                     attn: Optional[Callable] = None) -> Dict[str, object]:
     """Run the routed FFN stack on tokens h_in [T, d].
 
     attn_delta: [L, T, d] attention stand-in (None = zero).
+    attn: optional callable (layer index from 0, h) -> h_bar that replaces the stand-in
+    with a real attention sublayer (the full decoder forward; attn_delta is ignored).
     mode: "route" | "force" (mask_in [L, T] gives decisions; rows of the dense
     prefix are ignored) | "dense".
     branch_scale: "gate" (Eq. 3: g and 1 - g) or "one" (unscaled branches).
@@ -321,8 +377,11 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
 
     for layer in range(1, L + 1):
         wl = {k: _f64(weights[k][layer - 1]) for k in _LAYER_KEYS}
-        P = 0.0 if attn_delta is None else _f64(attn_delta[layer - 1])
-        h_bar = h + P                                               # Eq. 1 stand-in
+        if attn is not None:
+            h_bar = attn(layer - 1, h)                              # Eq. 1
+        else:
+            P = 0.0 if attn_delta is None else _f64(attn_delta[layer - 1])
+            h_bar = h + P                                           # Eq. 1 stand-in
         rec: Dict[str, np.ndarray] = {"h_bar": h_bar}
         j = layer - n_dense                                         # routed index (Sec. 4.1)
         dense_layer = mode == "dense" or j < 1
@@ -404,6 +463,21 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
     if record:
         out["layers"] = layers
     return out
+
+
+def decoder_forward(cfg: OracleConfig, weights, attn_weights, h_in, tau: float, n_heads: int,
+                    n_kv_heads: int, theta: float, n_seqs: int, seq_len: int, **kw):
+    """The full decoder forward: each block's h_bar comes from the attention sublayer
+    (Eq. 1) instead of the stand-in; everything else as routed_ffn_stack."""
+    R = bf16_round if cfg.dtype == "bf16" else _identity
+    wa_all = {k: _f64(v) for k, v in attn_weights.items()}
+
+    def attn(j, h):
+        wa = {k: v[j] for k, v in wa_all.items()}
+        return attention_sublayer(h, wa, n_heads, n_kv_heads, theta, n_seqs, seq_len,
+                                  cfg.rms_eps, R)
+
+    return routed_ffn_stack(cfg, weights, h_in, None, tau, attn=attn, **kw)
 
 
 def bypass_fraction(masks: np.ndarray, n_dense: int = 0) -> float:

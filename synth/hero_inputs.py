@@ -65,6 +65,10 @@ class StackConfig:
     seq_len: int = 0
     n_dense: int = 0       # leading FFN layers outside the routing candidate set (Sec. 4.1)
     router_variant: int = 0  # Sec. 4.4 router ablation bits (1 history, 2 memread, 4 aux, 8 pos)
+    # attention sublayer of the full decoder forward (Eq. 1; 0 heads: the additive stand-in)
+    n_heads: int = 0
+    n_kv_heads: int = 0
+    rope_theta: float = 10000.0
 
     @property
     def d_s(self) -> int:
@@ -102,6 +106,15 @@ CONFIGS: Dict[str, StackConfig] = {
     # up projection, a partial N tile in the down projection).
     "small_bf16_placed": StackConfig("small_bf16_placed", 4, 512, 1024, 96, 64, 333, "bf16",
                                      0.5, batch=1, seq_len=333, n_dense=2),
+    # Full decoder forward (Eq. 1 with real attention): small shapes for full-token parity
+    # (2 sequences of 160 tokens, 4 heads sharing 2 KV heads, head_dim 128) and
+    # Llama-3.1-8B prefill shapes (32 heads, 8 KV heads, head_dim 128, RoPE base 5e5).
+    "small_bf16_decoder": StackConfig("small_bf16_decoder", 4, 512, 1024, 64, 64, 320, "bf16",
+                                      0.27, batch=2, seq_len=160, n_heads=4, n_kv_heads=2,
+                                      rope_theta=500000.0),
+    "llama31_8b_decoder": StackConfig("llama31_8b_decoder", 32, 4096, 14336, 64, 64, 16384,
+                                      "bf16", 0.2687, batch=4, seq_len=4096, n_heads=32,
+                                      n_kv_heads=8, rope_theta=500000.0),
 }
 
 # The 13B workload is swept over these bypass targets.
@@ -149,6 +162,8 @@ WEIGHT_NAMES = tuple(n for n, *_ in _shapes(CONFIGS["tiny_f32"]))
 _TAG = {n: i + 1 for i, n in enumerate(WEIGHT_NAMES)}
 _TAG_H = 101
 _TAG_P = 102
+_TAG_ATTN = {"attn_norm_g": 201, "w_q": 202, "w_k": 203, "w_v": 204, "w_o": 205}
+ATTN_WEIGHT_NAMES = tuple(_TAG_ATTN)
 
 
 def round_to_bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -231,6 +246,30 @@ def generate_weights(cfg: StackConfig, threads: Optional[int] = None,
         if is_bf16 and not bf16_bits:
             arr = bf16_bits_to_f32(round_to_bf16_bits(arr))
         out[name] = arr
+    return out
+
+
+def attn_shapes(cfg: StackConfig):
+    """Attention parameters per layer (Llama layout, no biases): gain of LN_attn,
+    W_q [H hd, d], W_k and W_v [H_kv hd, d], W_o [d, H hd]; hd = d / H."""
+    L, d, H, Hkv = cfg.n_layers, cfg.d_model, cfg.n_heads, cfg.n_kv_heads
+    hd = d // H
+    return [("attn_norm_g", (L, d), "gain", 0.02), ("w_q", (L, H * hd, d), "normal", 0.02),
+            ("w_k", (L, Hkv * hd, d), "normal", 0.02), ("w_v", (L, Hkv * hd, d), "normal", 0.02),
+            ("w_o", (L, d, H * hd), "normal", 0.02 / math.sqrt(2 * L))]
+
+
+def generate_attn_weights(cfg: StackConfig, threads: Optional[int] = None) -> Dict[str, np.ndarray]:
+    """Attention parameters (seed s, own stream tags), encoded like generate_weights."""
+    if not cfg.n_heads:
+        raise ValueError("the workload has no attention sublayer (n_heads = 0)")
+    out: Dict[str, np.ndarray] = {}
+    is_bf16 = cfg.dtype == "bf16"
+    for name, shape, kind, arg in attn_shapes(cfg):
+        mean, std = (1.0, float(arg)) if kind == "gain" else (0.0, float(arg))
+        arr = np.empty(int(np.prod(shape)), dtype=np.uint16 if is_bf16 else np.float32)
+        _fill_normal(arr, (cfg.seed, _TAG_ATTN[name]), mean, std, is_bf16, threads)
+        out[name] = arr.reshape(shape)
     return out
 
 

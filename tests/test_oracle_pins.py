@@ -661,3 +661,81 @@ def test_planted_mistakes_are_caught(monkeypatch):
 
 def silu_swapped(u, wl):
     return ho.silu(u @ wl["w_up"].T) * (u @ wl["w_gate"].T)
+
+
+# ---------------------------------------------------------------------------
+# The attention sublayer of the full decoder forward (Eq. 1)
+# ---------------------------------------------------------------------------
+
+def _attn_inputs(seq_len=24, n_seqs=2, H=4, Hkv=2, d=64, seed=5):
+    cfg = hi.StackConfig("attn_micro", 2, d, 96, 8, 8, n_seqs * seq_len, "f32", 0.3,
+                         d_h=4, d_a=4, d_enc=8, d_head=8, d_path=4, seed=seed, batch=n_seqs,
+                         seq_len=seq_len, n_heads=H, n_kv_heads=Hkv, rope_theta=500000.0)
+    wa = {k: hi.to_f64(v)[0] for k, v in hi.generate_attn_weights(cfg).items()}
+    return cfg, wa, hi.to_f64(hi.generate_h_in(cfg))
+
+
+def test_rope_rotation_properties():
+    """RoPE rotates each (x_i, x_{i+hd/2}) pair: norms are kept, position 0 is the
+    identity, and q.k depends only on the position difference."""
+    rng = np.random.default_rng(0)
+    hd, S = 16, 40
+    cos, sin = ho.rope_cos_sin(S, hd, 10000.0)
+    q, k = rng.standard_normal((S, hd)), rng.standard_normal((S, hd))
+    rq = ho.apply_rope(q, cos, sin)
+    np.testing.assert_allclose(rq[0], q[0], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(np.linalg.norm(rq, axis=1), np.linalg.norm(q, axis=1), rtol=1e-13)
+    qq = np.repeat(q[:1], S, axis=0)
+    kk = np.repeat(k[:1], S, axis=0)
+    dots = np.sum(ho.apply_rope(qq, cos, sin)[5:] * ho.apply_rope(kk, cos, sin)[:-5], axis=1)
+    np.testing.assert_allclose(dots, dots[0], rtol=1e-11)   # positions (m, m-5) for every m
+    # the frequency of pair i is theta^(-2i/hd): pair 0 turns by one radian per position
+    np.testing.assert_allclose(cos[:, 0], np.cos(np.arange(S)), atol=1e-15)
+
+
+def test_attention_matches_torch_sdpa():
+    """Projection, causal softmax attention with grouped KV heads, output projection and
+    residual against torch's scaled_dot_product_attention (float64, no rounding)."""
+    cfg, wa, h = _attn_inputs()
+    B, S, H, Hkv, d = cfg.batch, cfg.seq_len, cfg.n_heads, cfg.n_kv_heads, cfg.d_model
+    hd = d // H
+    got = ho.attention_sublayer(h, wa, H, Hkv, cfg.rope_theta, B, S, cfg.rms_eps)
+    x = F.rms_norm(_t(h), (d,), _t(wa["attn_norm_g"]), cfg.rms_eps)
+    sh = lambda a, nh: a.reshape(B, S, nh, hd).transpose(1, 2)
+    q = sh(x @ _t(wa["w_q"]).T, H)
+    k = sh(x @ _t(wa["w_k"]).T, Hkv)
+    v = sh(x @ _t(wa["w_v"]).T, Hkv)
+    cos, sin = ho.rope_cos_sin(S, hd, cfg.rope_theta)
+    q = _t(ho.apply_rope(q.numpy(), cos, sin))
+    k = _t(ho.apply_rope(k.numpy(), cos, sin))
+    k = k.repeat_interleave(H // Hkv, dim=1)
+    v = v.repeat_interleave(H // Hkv, dim=1)
+    o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+    ref = _t(h) + o.transpose(1, 2).reshape(B * S, H * hd) @ _t(wa["w_o"]).T
+    np.testing.assert_allclose(got, ref.numpy(), rtol=0, atol=1e-12)
+
+
+def test_attention_is_causal_and_per_sequence():
+    cfg, wa, h = _attn_inputs()
+    B, S = cfg.batch, cfg.seq_len
+    run = lambda x: ho.attention_sublayer(x, wa, cfg.n_heads, cfg.n_kv_heads, cfg.rope_theta, B, S,
+                                          cfg.rms_eps)
+    base = run(h)
+    h2 = h.copy()
+    h2[S + 10] += 1.0                     # token 10 of the second sequence
+    out = run(h2)
+    changed = np.nonzero(np.abs(out - base).max(axis=1) > 1e-12)[0]
+    assert changed.min() == S + 10 and changed.max() < 2 * S   # itself and later tokens only
+    assert (changed >= S + 10).all()
+
+
+def test_attention_single_token_is_value_path():
+    """A one-token sequence attends only to itself: h_bar = h + W_o [v of its KV head]."""
+    cfg, wa, h = _attn_inputs(seq_len=1, n_seqs=6)
+    H, Hkv, d = cfg.n_heads, cfg.n_kv_heads, cfg.d_model
+    hd = d // H
+    got = ho.attention_sublayer(h, wa, H, Hkv, cfg.rope_theta, 6, 1, cfg.rms_eps)
+    x = F.rms_norm(_t(h), (d,), _t(wa["attn_norm_g"]), cfg.rms_eps).numpy()
+    v = (x @ wa["w_v"].T).reshape(6, Hkv, hd)
+    o = np.repeat(v, H // Hkv, axis=1).reshape(6, H * hd)
+    np.testing.assert_allclose(got, h + o @ wa["w_o"].T, rtol=0, atol=1e-12)
