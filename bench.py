@@ -11,8 +11,14 @@ needed between steps.  With N > 1 ranks (torchrun), every rank runs its own
 token shard of the same size on its own GPU (weak scaling, no collective on the
 data path); value = all ranks' tokens / the slowest rank's time.
 
+Decoder workloads (--workload llama31_8b_decoder, small_bf16_decoder) run the full
+decoder forward instead: every block's h_bar comes from the real attention
+sublayer (Eq. 1) rather than the stand-in; a step is all blocks' attention plus
+routed FFN over B sequences of S tokens.
+
 --impl reference times the CPU oracle (the only reference this method has) on a
-bounded token sample per step, on rank 0 only.
+bounded token sample per step, on rank 0 only (decoder workloads: a causal prefix
+of one sequence, which the oracle computes exactly without the rest).
 """
 
 from __future__ import annotations
@@ -34,6 +40,12 @@ sys.path.insert(0, ROOT)
 from synth import hero_inputs as hi  # noqa: E402
 
 METRIC = "routed-FFN-stack tokens/s at Llama-3.1-8B shapes; % of bf16 tensor peak"
+# decoder workloads: the same tokens/s, with the attention sublayers inside the step
+METRIC_DECODER = "decoder-forward (attention + routed FFN) tokens/s at Llama-3.1-8B shapes"
+
+
+def metric_for(cfg):
+    return METRIC_DECODER if cfg.n_heads else METRIC
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # DRAM bytes (read + write) per launch of the dominant kernel, from one ncu capture of the
@@ -56,6 +68,9 @@ def workload_desc(cfg, bypass):
     blocks = (f"{cfg.n_layers} routed blocks" if not cfg.n_dense else
               f"{cfg.n_dense} dense + {cfg.n_layers - cfg.n_dense} routed blocks")
     variant = f", router ablation bits {cfg.router_variant}" if cfg.router_variant else ""
+    if cfg.n_heads:
+        variant += (f", causal attention H={cfg.n_heads}, H_kv={cfg.n_kv_heads}, hd=128, "
+                    f"RoPE theta={cfg.rope_theta:g}")
     return (f"{cfg.name}: {blocks}, d={cfg.d_model}, I={cfg.d_ff}, "
             f"d_r={cfg.d_r}, d_m={cfg.d_m}, T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len}), "
             f"{cfg.dtype}, bypass target {bypass:.2%}{variant}, random-init weights, seeded inputs")
@@ -139,7 +154,39 @@ def algorithmic_work(cfg, counts_per_step, steps, routed=True):
     }
     if cfg.dtype == "bf16":
         work["ffn_gate_up"] += work.pop("adapter_down")
+    if cfg.n_heads:   # decoder: projections and causal attention of every block
+        hd = cfg.d_model // cfg.n_heads
+        nqkv = (cfg.n_heads + 2 * cfg.n_kv_heads) * hd
+        B, S = cfg.batch, cfg.seq_len
+        work["attn_proj"] = steps * cfg.n_layers * 2.0 * T * d * (nqkv + cfg.n_heads * hd)
+        # q k^T and p v over the causal triangle (S (S + 1) / 2 scores per head)
+        work["attn_core"] = steps * cfg.n_layers * B * cfg.n_heads * 4.0 * hd * S * (S + 1) / 2
     return work
+
+
+def oracle_step(ho, cfg, w, h_np, tau, n_sample, P_np=None):
+    """One oracle pass over a bounded sample of the workload: evenly spread tokens of
+    the stack (tokens are independent), or the first n_sample positions of sequence 1
+    of a decoder workload (a causal prefix needs nothing after it)."""
+    oc = ho.OracleConfig.from_stack(cfg)
+    if cfg.n_heads:
+        wa = hi.generate_attn_weights(cfg)
+        n = min(n_sample, cfg.seq_len)
+        rows = np.arange(n)
+        h = h_np[rows]
+
+        def step():
+            ho.decoder_forward(oc, w, wa, h, tau, cfg.n_heads, cfg.n_kv_heads, cfg.rope_theta, 1, n)
+        return step, rows, (f"positions 0..{n - 1} of sequence 1 (of {cfg.batch}x{cfg.seq_len}) "
+                            f"through all {cfg.n_layers} blocks with attention, float64 numpy")
+    rows = hi.sample_tokens(cfg.n_tokens, n_sample)
+    h = h_np[rows]
+    P = (hi.generate_attn_delta(cfg) if P_np is None else P_np)[:, rows]
+
+    def step():
+        ho.routed_ffn_stack(oc, w, h, P, tau)
+    return step, rows, (f"{len(rows)} evenly spread tokens of T={cfg.n_tokens} through all "
+                        f"{cfg.n_layers} blocks, float64 numpy")
 
 
 def reference_arm(args, rank, world):
@@ -149,24 +196,20 @@ def reference_arm(args, rank, world):
     cfg = hi.CONFIGS[args.workload]
     tau = hi.calibrated_tau(cfg.name)
     w = hi.generate_weights(cfg)
-    rows = hi.sample_tokens(cfg.n_tokens, args.cpu_sample)
-    h = hi.generate_h_in(cfg)[rows]
-    P = hi.generate_attn_delta(cfg)[:, rows]
-    oc = ho.OracleConfig.from_stack(cfg)
+    step, rows, sample = oracle_step(ho, cfg, w, hi.generate_h_in(cfg), tau, args.cpu_sample)
     for _ in range(args.warmup):
-        ho.routed_ffn_stack(oc, w, h, P, tau)
+        step()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        ho.routed_ffn_stack(oc, w, h, P, tau)
+        step()
     dt = time.perf_counter() - t0
     v = len(rows) * args.steps / dt
     cores = len(os.sched_getaffinity(0))
-    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+    line = {"metric": metric_for(cfg), "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": workload_desc(cfg, cfg.bypass),
-                       "sample": f"{len(rows)} evenly spread tokens of T={cfg.n_tokens} per step"},
+            "config": {"workload": workload_desc(cfg, cfg.bypass), "sample": sample},
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"{len(rows)} tokens x {cfg.n_layers} blocks per step"},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -224,16 +267,22 @@ def main():
         cfg = cfg.replace(router_variant=args.router_variant, d_m=args.d_m or cfg.d_m)
     default_shape = cfg == hi.CONFIGS[args.workload] and args.tau is None
     T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
+    decoder = bool(cfg.n_heads)
+    if decoder and args.tokens:
+        cfg = cfg.replace(batch=max(1, cfg.n_tokens // cfg.seq_len))
+    B, S = cfg.batch, cfg.seq_len
+    if decoder and B * S != T:
+        raise SystemExit(f"decoder workload needs T = batch x seq_len ({B}x{S} != {T})")
     t_gen = time.time()
     w = hi.generate_weights(cfg)
     h_np = hi.generate_h_in(cfg)
-    P_np = hi.generate_attn_delta(cfg)
+    P_np = None if decoder else hi.generate_attn_delta(cfg)
     t_gen = time.time() - t_gen
-    stack = hero.HeroStack(cfg, w)
+    stack = hero.HeroDecoder(cfg, w, hi.generate_attn_weights(cfg)) if decoder else hero.HeroStack(cfg, w)
     dev = torch.device("cuda", local_rank)
     stream = torch.cuda.current_stream(dev)
     h = torch.from_numpy(h_np).to(dev)
-    P = torch.from_numpy(P_np).to(dev)
+    P = None if decoder else torch.from_numpy(P_np).to(dev)
     h_out = torch.empty((T, d), dtype=torch.float32, device=dev)
     g = torch.empty((L, T), dtype=torch.float32, device=dev)
     m = torch.empty((L, T), dtype=torch.uint8, device=dev)
@@ -251,8 +300,12 @@ def main():
         return float(t.item())
 
     def run(flags, st=None):
-        stack(h, P, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m, counts_out=c,
-              stream=st or stream)
+        if decoder:
+            stack.forward(h, tau, B, S, flags=flags, h_out=h_out, gate_out=g, mask_out=m,
+                          counts_out=c, stream=st or stream)
+        else:
+            stack(h, P, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m, counts_out=c,
+                  stream=st or stream)
 
     def timed(fn, K, sampler=None):
         barrier()
@@ -318,20 +371,25 @@ def main():
     e2e = None
     if not args.no_e2e:
         hp = torch.from_numpy(h_np).pin_memory()
-        Pp = torch.from_numpy(P_np).pin_memory()
+        Pp = None if decoder else torch.from_numpy(P_np).pin_memory()
         ho_ = torch.empty((T, d), dtype=torch.float32).pin_memory()
         cp = torch.empty((L,), dtype=torch.int32).pin_memory()
 
         def run_host():
-            hero.hero_routed_ffn_stack(stack.model, T, hp.data_ptr(), Pp.data_ptr(), tau,
-                                       hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
-                                       cp.data_ptr(), stream.cuda_stream)
+            if decoder:
+                hero.hero_decoder_forward(stack.model, B, S, hp.data_ptr(), tau,
+                                          hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                          cp.data_ptr(), stream.cuda_stream)
+            else:
+                hero.hero_routed_ffn_stack(stack.model, T, hp.data_ptr(), Pp.data_ptr(), tau,
+                                           hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                           cp.data_ptr(), stream.cuda_stream)
         run_host()
         torch.cuda.synchronize()
         ms_e2e, _ = timed(run_host, args.steps)
         stack.check()
         e2e = {"value": world * T * args.steps / (ms_e2e / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": int(hp.numel() * 4 + Pp.numel() * 2),
+               "h2d_bytes_per_step": int(hp.numel() * 4 + (0 if decoder else Pp.numel() * 2)),
                "d2h_bytes_per_step": int(ho_.numel() * 4 + cp.numel() * 4)}
         assert np.array_equal(cp.numpy(), counts), "host-IO path routed differently"
 
@@ -356,23 +414,21 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         from oracle import hero_oracle as ho
-        rows = hi.sample_tokens(T, args.cpu_sample)
-        oc = ho.OracleConfig.from_stack(cfg)
+        step, rows, sample = oracle_step(ho, cfg, w, h_np, tau, args.cpu_sample, P_np)
         t0 = time.perf_counter()
-        ho.routed_ffn_stack(oc, w, h_np[rows], P_np[:, rows], tau)
+        step()
         dt = time.perf_counter() - t0
         cpu = {"value": len(rows) / dt, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
-               "kind": "oracle",
-               "sample": f"{len(rows)} evenly spread tokens of T={T} through all {L} blocks, "
-                         f"float64 numpy ({dt:.1f} s; BLAS threads = cores)"}
+               "kind": "oracle", "sample": f"{sample} ({dt:.1f} s; BLAS threads = cores)"}
 
     launches = int(sum(n for _, n in prof.values()))
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "metric": metric_for(cfg), "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
         "config": {"workload": workload_desc(cfg, cfg.bypass),
-                   "l2": "inputs larger than L2 (no flush): weights and P_j stream from HBM each step",
+                   "l2": ("inputs larger than L2 (no flush): weights stream from HBM each step"
+                          + ("" if decoder else ", and so does P_j")),
                    "parallelism": f"token shards, {world} rank(s), no collective",
                    **({"cuda_graph": True, "eager_ms_per_step": ms_eager} if args.graph else {})},
         "roofline": roof,

@@ -209,6 +209,57 @@ const char* hero_last_error(void);
  * HERO_ERR_CUDA if the stream holds a CUDA error. */
 hero_status hero_check_device_status(hero_model* m, void* cuda_stream);
 
+/* ---- the full decoder forward: real attention in Eq. 1 -----------------------
+ * Eq. 1 gives each routed block the representation after attention,
+ * h_bar = h + Attn(LN_attn(h)), and keeps attention dense (Sec. 3.1).  The fused
+ * stack above stands in an additive perturbation for Attn; these calls attach the
+ * backbone's attention (Llama form, Sec. 4.1: RMSNorm with its own gain,
+ * bias-free projections, rotate-half RoPE with inverse frequencies
+ * theta^(-2i/hd), causal softmax(q k^T / sqrt(hd)) per sequence, grouped-query
+ * heads: query head h reads key/value head h / (H / H_kv)) and run the whole
+ * decoder.  bf16 models only; head dimension 128 (d = H * 128). */
+typedef struct {
+  int32_t n_heads;       /* H; d_model = 128 H                                      */
+  int32_t n_kv_heads;    /* H_kv; divides H                                         */
+  float rope_theta;      /* RoPE base theta                                         */
+} hero_attn_config;
+
+/* HOST pointers, canonical layouts, stacked over the model's n_layers:
+ *   attn_norm_g [L,d], w_q [L,H hd,d], w_k [L,H_kv hd,d], w_v [L,H_kv hd,d],
+ *   w_o [L,d,H hd]; element type host_dtype.  Copied (converted to bf16). */
+typedef struct {
+  hero_dtype host_dtype;
+  const void *attn_norm_g, *w_q, *w_k, *w_v, *w_o;
+} hero_attn_weights_host;
+
+/* Attach the attention parameters to a bf16 model and size its attention
+ * workspace for max_tokens.  HERO_ERR_UNSUPPORTED for f32 models or
+ * d != 128 H; HERO_ERR_ARG for bad counts or NULL pointers.  Call once. */
+hero_status hero_attn_init(hero_model* m, const hero_attn_config* c, const hero_attn_weights_host* w);
+
+/* Eq. 1, first line, for layer `layer` (1..n_layers) on n_seqs sequences of
+ * seq_len tokens, rows of h in sequence order (T = n_seqs * seq_len <=
+ * max_tokens, n_seqs <= 65535): h_bar [T,d] = h + Attn(LN_attn(h)).  DEVICE pointers, fp32, must
+ * not alias.  Precision: bf16 operands (LN_attn(h), q and k after RoPE, v, the
+ * softmax probabilities entering P V, the attention output), fp32 accumulation
+ * and softmax.  Asynchronous on cuda_stream. */
+hero_status hero_attention_block(hero_model* m, int32_t layer, int32_t n_seqs, int32_t seq_len,
+                                 const float* h, float* h_bar, void* cuda_stream);
+
+/* The full decoder forward over all n_layers blocks: h_bar = h + Attn(LN_attn(h))
+ * (Eq. 1), then the block's FFN routing exactly as hero_routed_block (Eqs. 2-16;
+ * blocks 1..n_dense are plain FFN blocks), the router state carried in the model's
+ * workspace and reset at the start.  h_in [T,d] -> h_out [T,d] fp32; tau_exec,
+ * flags (HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK with mask_in [L,T], optionally
+ * HERO_FLAG_HOST_IO), gate_out [L,T], mask_out [L,T], ffn_count_out [L] as
+ * hero_routed_ffn_stack (NULL allowed).  DEVICE pointers, or HOST pointers with
+ * HERO_FLAG_HOST_IO (copied on the stream); h_out must not alias h_in.
+ * n_seqs <= 65535. */
+hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len, const float* h_in,
+                                 float tau_exec, uint32_t flags, const uint8_t* mask_in,
+                                 float* h_out, float* gate_out, uint8_t* mask_out,
+                                 int32_t* ffn_count_out, void* cuda_stream);
+
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes of one block, for per-kernel timing. */
 enum {
@@ -222,7 +273,9 @@ enum {
   HERO_K_FFN_DOWN = 6,    /* down GEMM with the scaled scatter epilogue       */
   HERO_K_ADAPTER_DOWN = 7,/* f32 models: adapter W_1 GEMM with the SiLU epilogue */
   HERO_K_ADAPTER_UP = 8,  /* adapter W_2 GEMM with the scaled scatter epilogue */
-  HERO_K_COUNT = 9
+  HERO_K_ATTN_PROJ = 9,   /* LN_attn, q/k/v projection, RoPE, output projection */
+  HERO_K_ATTN_CORE = 10,  /* causal softmax attention                           */
+  HERO_K_COUNT = 11
 };
 
 /* When enabled, every later launch of the model is bracketed by CUDA events on

@@ -320,6 +320,35 @@ def attention_sublayer(h, wa, n_heads: int, n_kv_heads: int, theta: float, n_seq
     return h + o @ wa["w_o"].T
 
 
+def attention_rows(h_seq, rows, wa, n_heads: int, n_kv_heads: int, theta: float,
+                   rms_eps: float, R=None):
+    """attention_sublayer restricted to query positions `rows` of ONE sequence h_seq
+    [S, d] (keys and values of all its positions): h_bar[rows].  The same steps in
+    the same order, for checking long sequences on a sample of positions."""
+    R = R or _identity
+    S, d = h_seq.shape
+    hd = d // n_heads
+    rows = np.asarray(rows)
+    last = int(rows.max()) + 1                                   # causal: keys < last suffice
+    x = R(rms_norm(h_seq[:last], wa["attn_norm_g"], rms_eps))
+    cos, sin = rope_cos_sin(last, hd, theta)
+    q = (x[rows] @ wa["w_q"].T).reshape(len(rows), n_heads, hd).transpose(1, 0, 2)
+    k = (x @ wa["w_k"].T).reshape(last, n_kv_heads, hd).transpose(1, 0, 2)
+    v = (x @ wa["w_v"].T).reshape(last, n_kv_heads, hd).transpose(1, 0, 2)
+    q = R(apply_rope(q, cos[rows], sin[rows]))
+    k, v = R(apply_rope(k, cos, sin)), R(v)
+    group = n_heads // n_kv_heads
+    k = np.repeat(k, group, axis=0)
+    v = np.repeat(v, group, axis=0)
+    scores = q @ k.transpose(0, 2, 1) / np.sqrt(hd)                   # [H, rows, last]
+    scores = np.where(np.arange(last)[None, None, :] <= rows[None, :, None], scores, -np.inf)
+    scores = scores - scores.max(axis=-1, keepdims=True)
+    p = np.exp(scores)
+    p = R(p / p.sum(axis=-1, keepdims=True))
+    o = R(p @ v).transpose(1, 0, 2).reshape(len(rows), n_heads * hd)
+    return h_seq[rows] + o @ wa["w_o"].T
+
+
 # ---------------------------------------------------------------------------
 # The stack
 # ---------------------------------------------------------------------------

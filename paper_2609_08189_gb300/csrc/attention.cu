@@ -1,0 +1,334 @@
+// The attention sublayer of Eq. 1 (the full decoder forward), bf16 models:
+//   x = LN_attn(h)                      k_attn_norm (bf16 rows, the projection operand)
+//   qkv = x [W_q; W_k; W_v]^T           tensor-core GEMM (gemm_tc.cu)
+//   q, k <- RoPE(q), RoPE(k)            k_rope (bf16, [sequence][head][position][128])
+//   o = softmax(q k^T / sqrt(hd)) v     k_flash_attn (causal, grouped-query heads)
+//   h_bar = h + o W_o^T                 tensor-core GEMM with the residual epilogue
+#include "hero_device.cuh"
+
+namespace hero {
+namespace {
+
+constexpr int HD = 128;       // head dimension
+constexpr int FA_BM = 64;     // query rows per CTA (16 per warp)
+constexpr int FA_BN = 64;     // keys per tile
+constexpr int FA_THREADS = 128;
+
+// ---------------------------------------------------------------------------------
+// x = bf16(h * rsqrt(mean(h^2) + eps) * g), one warp per row.
+// ---------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_attn_norm(const float* __restrict__ h,
+                                                   const float* __restrict__ g, int T, int d,
+                                                   float eps, uint16_t* __restrict__ x) {
+  pdl_enter();
+  const long row = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const float* hr = h + (size_t)row * d;
+  float ss = 0.f;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(hr + c);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  const float rinv = rsqrtf(ss / (float)d + eps);
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(hr + c);
+    const float4 gv = __ldg(reinterpret_cast<const float4*>(g + c));
+    store4(x, (size_t)row * d + c,
+           make_float4(v.x * rinv * gv.x, v.y * rinv * gv.y, v.z * rinv * gv.z, v.w * rinv * gv.w),
+           1);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// RoPE and layout: qkv fp32 [T][(H + 2 H_kv) 128] (q heads | k heads | v heads) ->
+// Q [B][H][S][128], K and V [B][H_kv][S][128], bf16.  Pair (i, i + 64) of a q or
+// k head at position s turns by s * theta^(-2i/128).  One thread per (token, head,
+// pair).
+// ---------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_rope(const float* __restrict__ qkv, int B, int S, int H,
+                                              int Hkv, float log2_theta, uint16_t* __restrict__ Q,
+                                              uint16_t* __restrict__ K, uint16_t* __restrict__ V) {
+  pdl_enter();
+  const int heads = H + 2 * Hkv;
+  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (long)B * S * heads * (HD / 2)) return;
+  const int pair = (int)(i % (HD / 2));
+  const long rest = i / (HD / 2);
+  const int hh = (int)(rest % heads);
+  const long t = rest / heads;
+  const int b = (int)(t / S), s = (int)(t - (long)b * S);
+  const float* src = qkv + (size_t)t * heads * HD + (size_t)hh * HD;
+  const float x1 = src[pair], x2 = src[pair + HD / 2];
+  uint16_t* dst;
+  float y1 = x1, y2 = x2;
+  if (hh < H + Hkv) {   // q or k head: rotate
+    const float inv_freq = exp2f(-(2.0f * pair / HD) * log2_theta);
+    float sn, cs;
+    sincosf((float)s * inv_freq, &sn, &cs);
+    y1 = x1 * cs - x2 * sn;
+    y2 = x2 * cs + x1 * sn;
+  }
+  if (hh < H)
+    dst = Q + (((size_t)b * H + hh) * S + s) * HD;
+  else if (hh < H + Hkv)
+    dst = K + (((size_t)b * Hkv + (hh - H)) * S + s) * HD;
+  else
+    dst = V + (((size_t)b * Hkv + (hh - H - Hkv)) * S + s) * HD;
+  dst[pair] = (uint16_t)(pack_bf16x2(y1, 0.f) & 0xffffu);
+  dst[pair + HD / 2] = (uint16_t)(pack_bf16x2(y2, 0.f) & 0xffffu);
+}
+
+// ---------------------------------------------------------------------------------
+// Causal attention, FlashAttention-2 schedule on the mma.sync bf16 tensor path:
+// CTA = 64 query rows of one (sequence, head), 4 warps of 16 rows; key/value tiles
+// of 64 rows double-buffered in shared memory (cp.async); S = Q K^T and O += P V
+// with m16n8k16 MMAs, fp32 accumulators in registers; online softmax in fp32 with
+// exp2; P is rounded to bf16 as the A operand of P V (the FlashAttention rounding
+// of exp(s - running max)); O / l is rounded to bf16 on store.
+// Shared tiles are [row][128] bf16 with 16-byte chunks XOR-swizzled by row % 8.
+// ---------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t swz(int r, int c) {   // element offset (c multiple of 8)
+  return (uint32_t)(r * HD + (((c >> 3) ^ (r & 7)) << 3));
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Load rows [row0, row0 + 64) of a [S][128] bf16 matrix into a swizzled tile;
+// rows at or past S are zero-filled (their source address is clamped to row 0).
+__device__ __forceinline__ void load_tile(uint32_t tile, const uint16_t* src, int row0, int S,
+                                          int tid) {
+#pragma unroll
+  for (int i = 0; i < (FA_BM * HD / 8) / FA_THREADS; ++i) {
+    const int chunk = tid + i * FA_THREADS;
+    const int r = chunk >> 4, c = (chunk & 15) << 3;
+    const bool valid = row0 + r < S;
+    const uint16_t* g = src + (size_t)(valid ? row0 + r : 0) * HD + c;
+    cp_async16(tile + 2u * swz(r, c), g, valid);
+  }
+}
+
+__global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __restrict__ Q,
+                                                           const uint16_t* __restrict__ K,
+                                                           const uint16_t* __restrict__ V, int H,
+                                                           int Hkv, int S, float scale_log2,
+                                                           uint16_t* __restrict__ O) {
+  pdl_enter();
+  extern __shared__ __align__(128) uint16_t fa_smem[];
+  const uint32_t sQ = smem_u32(fa_smem);
+  const uint32_t sK = sQ + 2u * FA_BM * HD;            // 2 buffers
+  const uint32_t sV = sK + 2u * 2 * FA_BN * HD;        // 2 buffers
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int qt = gridDim.x - 1 - blockIdx.x;           // long rows first
+  const int hh = blockIdx.y, b = blockIdx.z;
+  const int kvh = hh / (H / Hkv);
+  const int q0 = qt * FA_BM;
+  const uint16_t* Qg = Q + ((size_t)b * H + hh) * S * HD;
+  const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * S * HD;
+  const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * S * HD;
+  const int n_tiles = qt + 1;                          // causal: key tiles 0..qt
+
+  load_tile(sQ, Qg, q0, S, tid);
+  load_tile(sK, Kg, 0, S, tid);
+  load_tile(sV, Vg, 0, S, tid);
+  cp_async_commit();
+
+  uint32_t qa[HD / 16][4];
+  float o[HD / 8][4];
+#pragma unroll
+  for (int j = 0; j < HD / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;   // rows lane/4 and lane/4 + 8
+  const int qrow0 = q0 + warp * 16 + (lane >> 2);
+
+  for (int it = 0; it < n_tiles; ++it) {
+    const int buf = it & 1;
+    if (it + 1 < n_tiles) {   // prefetch the next key/value tile
+      load_tile(sK + 2u * (buf ^ 1) * FA_BN * HD, Kg, (it + 1) * FA_BN, S, tid);
+      load_tile(sV + 2u * (buf ^ 1) * FA_BN * HD, Vg, (it + 1) * FA_BN, S, tid);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    if (it == 0) {   // the warp's 16 query rows as A fragments, once
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const int r = warp * 16 + (lane & 15), c = kk * 16 + ((lane >> 4) << 3);
+        ldsm_x4(sQ + 2u * swz(r, c), qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
+      }
+    }
+    const uint32_t kt = sK + 2u * buf * FA_BN * HD;
+    const uint32_t vt = sV + 2u * buf * FA_BN * HD;
+
+    // S = Q K^T for 16 rows x 64 keys
+    float sc[FA_BN / 8][4];
+#pragma unroll
+    for (int j = 0; j < FA_BN / 8; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+#pragma unroll
+      for (int j = 0; j < FA_BN / 8; j += 2) {
+        const int r = j * 8 + (lane & 7) + ((lane >> 4) << 3);
+        const int c = kk * 16 + (((lane >> 3) & 1) << 3);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(kt + 2u * swz(r, c), b0, b1, b2, b3);
+        mma_bf16(sc[j], qa[kk], b0, b1);
+        mma_bf16(sc[j + 1], qa[kk], b2, b3);
+      }
+    }
+    // causal / length mask, then the online softmax (scores in log2 units)
+    const int k0 = it * FA_BN;
+    float tmax0 = -INFINITY, tmax1 = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < FA_BN / 8; ++j) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int kpos = k0 + j * 8 + ((lane & 3) << 1) + (e & 1);
+        const int qpos = qrow0 + ((e >> 1) << 3);
+        float v = sc[j][e] * scale_log2;
+        if (kpos > qpos || kpos >= S) v = -INFINITY;
+        sc[j][e] = v;
+      }
+      tmax0 = fmaxf(tmax0, fmaxf(sc[j][0], sc[j][1]));
+      tmax1 = fmaxf(tmax1, fmaxf(sc[j][2], sc[j][3]));
+    }
+#pragma unroll
+    for (int off = 1; off < 4; off <<= 1) {
+      tmax0 = fmaxf(tmax0, __shfl_xor_sync(0xffffffffu, tmax0, off));
+      tmax1 = fmaxf(tmax1, __shfl_xor_sync(0xffffffffu, tmax1, off));
+    }
+    const float mn0 = fmaxf(m0, tmax0), mn1 = fmaxf(m1, tmax1);   // finite: key 0 is in tile 0
+    const float al0 = exp2f(m0 - mn0), al1 = exp2f(m1 - mn1);
+    m0 = mn0;
+    m1 = mn1;
+    float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+    for (int j = 0; j < FA_BN / 8; ++j) {
+      sc[j][0] = exp2f(sc[j][0] - mn0);
+      sc[j][1] = exp2f(sc[j][1] - mn0);
+      sc[j][2] = exp2f(sc[j][2] - mn1);
+      sc[j][3] = exp2f(sc[j][3] - mn1);
+      ps0 += sc[j][0] + sc[j][1];
+      ps1 += sc[j][2] + sc[j][3];
+    }
+    l0 = l0 * al0 + ps0;
+    l1 = l1 * al1 + ps1;
+#pragma unroll
+    for (int j = 0; j < HD / 8; ++j) {
+      o[j][0] *= al0;
+      o[j][1] *= al0;
+      o[j][2] *= al1;
+      o[j][3] *= al1;
+    }
+    // O += P V: P (bf16) as A fragments straight from the score accumulators
+#pragma unroll
+    for (int kk = 0; kk < FA_BN / 16; ++kk) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
+      pa[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
+      pa[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      pa[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int j = 0; j < HD / 8; j += 2) {
+        const int r = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
+        const int c = j * 8 + ((lane >> 4) << 3);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(vt + 2u * swz(r, c), b0, b1, b2, b3);
+        mma_bf16(o[j], pa, b0, b1);
+        mma_bf16(o[j + 1], pa, b2, b3);
+      }
+    }
+    __syncthreads();   // this buffer is refilled by the next iteration's prefetch
+  }
+  // rows' sums over the four lanes of a row, then O / l in bf16
+#pragma unroll
+  for (int off = 1; off < 4; off <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+  }
+  const float inv0 = 1.f / l0, inv1 = 1.f / l1;
+  const int dcol = hh * HD + ((lane & 3) << 1);
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    const int qpos = qrow0 + half * 8;
+    if (qpos >= S) continue;
+    uint32_t* orow = reinterpret_cast<uint32_t*>(O + ((size_t)b * S + qpos) * H * HD + dcol);
+    const float inv = half ? inv1 : inv0;
+#pragma unroll
+    for (int j = 0; j < HD / 8; ++j)
+      orow[j * 4] = pack_bf16x2(o[j][2 * half] * inv, o[j][2 * half + 1] * inv);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float eps, void* x,
+                             cudaStream_t st) {
+  if (T <= 0) return cudaSuccess;
+  if (d % 128) return cudaErrorInvalidValue;
+  return launch_pdl(k_attn_norm, dim3((unsigned)((T + 7) / 8)), dim3(256), 0, st, h, g, T, d, eps,
+                    static_cast<uint16_t*>(x));
+}
+
+cudaError_t launch_rope(const float* qkv, int B, int S, int H, int Hkv, float theta, void* Q, void* K,
+                        void* V, cudaStream_t st) {
+  const long n = (long)B * S * (H + 2 * Hkv) * (HD / 2);
+  if (n <= 0) return cudaSuccess;
+  return launch_pdl(k_rope, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, qkv, B, S, H, Hkv,
+                    log2f(theta), static_cast<uint16_t*>(Q), static_cast<uint16_t*>(K),
+                    static_cast<uint16_t*>(V));
+}
+
+cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
+                              int Hkv, void* O, cudaStream_t st) {
+  if (B <= 0 || S <= 0) return cudaSuccess;
+  if (H % Hkv || H > 65535 || B > 65535) return cudaErrorInvalidValue;   // grid y and z limits
+  constexpr size_t smem = 2u * (FA_BM * HD + 2 * 2 * FA_BN * HD);   // 80 KB
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_flash_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
+  dim3 grid((unsigned)((S + FA_BM - 1) / FA_BM), (unsigned)H, (unsigned)B);
+  return launch_pdl(k_flash_attn, grid, dim3(FA_THREADS), smem, st,
+                    static_cast<const uint16_t*>(Q), static_cast<const uint16_t*>(K),
+                    static_cast<const uint16_t*>(V), H, Hkv, S, scale_log2,
+                    static_cast<uint16_t*>(O));
+}
+
+}  // namespace hero

@@ -80,7 +80,7 @@ __device__ __forceinline__ float4 staged(const float4* st, int row, int slot) {
   return st[row * 8 + (slot ^ (row & 7))];
 }
 
-template <int BN>
+template <int BN, bool RESID = false>
 __device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase, int row0, int M,
                                               int nb, int split, float4* st) {
   float* out = a.out_f32 + (size_t)split * a.split_stride;
@@ -97,8 +97,14 @@ __device__ __forceinline__ void epi_store_f32(const GemmArgs& a, uint32_t tbase,
     for (int k = 0; k < 8; ++k) {
       const int rr = sub + 4 * k;
       const int m = row0 + rr;
-      if (m < M && n < a.N)
-        *reinterpret_cast<float4*>(out + (size_t)m * a.ldo + n) = staged(st, rr, slot);
+      if (m < M && n < a.N) {
+        float4 v = staged(st, rr, slot);
+        if constexpr (RESID) {
+          const float4 r = *reinterpret_cast<const float4*>(a.resid + (size_t)m * a.ldo + n);
+          v.x += r.x; v.y += r.y; v.z += r.z; v.w += r.w;
+        }
+        *reinterpret_cast<float4*>(out + (size_t)m * a.ldo + n) = v;
+      }
     }
     __syncwarp();
   }
@@ -284,6 +290,8 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
   const int row0 = mb * BM + q * 32;
   if constexpr (EPI == EPI_STORE_F32) {
     epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
+  } else if constexpr (EPI == EPI_RESIDUAL) {
+    epi_store_f32<BN, true>(a, tbase, row0, M, nb, split, stg);
   } else if constexpr (EPI == EPI_SWIGLU) {
     epi_swiglu(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_SILU) {
@@ -534,6 +542,8 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
     case EPI_LAYER_OUT_WIDE:
       return launch_tc<256, EPI_LAYER_OUT_WIDE, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms,
                                                           st);
+    case EPI_RESIDUAL:
+      return launch_tc<256, EPI_RESIDUAL, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

@@ -135,6 +135,19 @@ struct hero_model {
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
   std::vector<CUtensorMap> tm_wgu, tm_wd, tm_w1, tm_w2;
 
+  // attention sublayer of the full decoder forward (hero_attn_init; bf16 models)
+  bool attn = false;
+  int n_heads = 0, n_kv_heads = 0;
+  float rope_theta = 0.f;
+  void* wqkv = nullptr;        // [L][(H + 2 H_kv) 128][d]: W_q | W_k | W_v rows
+  void* wo = nullptr;          // [L][d][H 128]
+  float* attn_gain = nullptr;  // [L][d]
+  void* aws = nullptr;         // attention workspace
+  void *ax = nullptr, *aq = nullptr, *ak = nullptr, *av = nullptr, *ao = nullptr;
+  float *aqkv = nullptr, *hcur = nullptr, *hbprev = nullptr, *dlprev = nullptr;
+  CUtensorMap tm_ax, tm_ao;
+  std::vector<CUtensorMap> tm_wqkv, tm_wo;
+
   // measurement
   bool profiling = false;
   std::vector<ProfEvent> pending;
@@ -283,7 +296,7 @@ void free_model(hero_model* m) {
   if (m->ev_kernels_done) cudaEventDestroy(m->ev_kernels_done);
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
-                  m->ws, m->io};
+                  m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -1002,6 +1015,85 @@ extern "C" hero_status hero_router_state_reset(hero_model* m, int64_t n_tokens,
   return HERO_OK;
 }
 
+namespace {
+
+// One block on post-attention states h_bar (layer jj, the caller's router state
+// and carried h_bar_prev / delta_prev): block entry (delta, partial sums, router
+// operand), then block_body writing h_out.  Arguments already validated.
+hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, const BlockState& bs,
+                             float* h_bar_prev, float* delta_prev, float tau, uint32_t flags,
+                             const uint8_t* mask_in, float* h_out, float* gate_out,
+                             uint8_t* mask_out, int32_t* count_out, cudaStream_t st) {
+  const hero_config& c = m->cfg;
+  const int jr = jj - c.n_dense;
+  bool dense = flags & HERO_FLAG_DENSE;
+  if (jr < 0) {   // outside the routing candidate set: the plain FFN block
+    dense = true;
+    flags = (flags & ~(uint32_t)HERO_FLAG_FORCE_MASK) | HERO_FLAG_DENSE;
+  }
+  BlockEntryArgs be{T, c.d_model, m->np, jr + 1, dense ? 0 : 1, h_bar,
+                    dense ? nullptr : h_bar_prev, dense ? nullptr : delta_prev,
+                    m->xl, (int)m->bf16, m->part};
+  CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
+  LayerOutArgs lo{};
+  lo.hbar = const_cast<float*>(h_bar);  // read only: the block writes h_out
+  lo.h_out = h_out;
+  lo.part = m->part;
+  lo.d = c.d_model;
+  lo.np = m->np;
+  lo.last = 1;
+  lo.first = jr <= 0;
+  lo.p_bf16 = m->bf16;
+  lo.xl_bf16 = m->bf16;
+  lo.router = 0;
+  return block_body(m, jj, jr, T, dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr} : bs,
+                    h_bar, lo, tau, flags, (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr,
+                    gate_out, mask_out, count_out, st);
+}
+
+// Eq. 1, first line, for layer jj on B sequences of S tokens: h_bar = h + Attn(LN_attn(h)).
+hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, float* h_bar,
+                          cudaStream_t st) {
+  const hero_config& c = m->cfg;
+  const int T = B * S, d = c.d_model, H = m->n_heads, Hkv = m->n_kv_heads;
+  const int nqkv = (H + 2 * Hkv) * 128;
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_attn_norm(h, m->attn_gain + (size_t)jj * d, T, d, c.rms_eps, m->ax, st);
+  }));
+  GemmArgs g{};
+  g.m_static = T;
+  g.m_max = T;
+  g.N = nqkv;
+  g.K = d;
+  g.out_f32 = m->aqkv;
+  g.ldo = nqkv;
+  g.err = m->err;
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_gemm_tc(256, EPI_STORE_F32, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
+  }));
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_rope(m->aqkv, B, S, H, Hkv, m->rope_theta, m->aq, m->ak, m->av, st);
+  }));
+  CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
+    return launch_flash_attn(m->aq, m->ak, m->av, B, S, H, Hkv, m->ao, st);
+  }));
+  GemmArgs o{};
+  o.m_static = T;
+  o.m_max = T;
+  o.N = d;
+  o.K = H * 128;
+  o.out_f32 = h_bar;
+  o.ldo = d;
+  o.resid = h;
+  o.err = m->err;
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_gemm_tc(256, EPI_RESIDUAL, m->tm_ao, m->tm_wo[jj], o, m->num_sms, st);
+  }));
+  return HERO_OK;
+}
+
+}  // namespace
+
 extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n_tokens,
                                          const float* h_bar, const hero_router_state* s,
                                          float tau_exec, uint32_t flags, const uint8_t* mask_in,
@@ -1035,33 +1127,217 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
                  !s->h_bar_prev || !s->delta_prev))
     return fail(HERO_ERR_ARG, "the router state needs all seven pointers");
   CUDA_TRY(cudaSetDevice(m->device));
-  const int T = (int)n_tokens, jj = block - 1, jr = jj - c.n_dense;
-  if (jr < 0) {   // outside the routing candidate set: the plain FFN block
-    dense = true;
-    flags = (flags & ~(uint32_t)HERO_FLAG_FORCE_MASK) | HERO_FLAG_DENSE;
-  }
-  BlockEntryArgs be{T, c.d_model, m->np, jr + 1, dense ? 0 : 1, h_bar,
-                    dense ? nullptr : s->h_bar_prev, dense ? nullptr : s->delta_prev,
-                    m->xl, (int)m->bf16, m->part};
-  CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
-  BlockState bs{dense ? nullptr : s->S, dense ? nullptr : s->zeta, dense ? nullptr : s->p_hist,
-                dense ? nullptr : s->m_hist, dense ? nullptr : s->d_prev};
-  LayerOutArgs lo{};
-  lo.hbar = const_cast<float*>(h_bar);  // read only: the block writes h_out
-  lo.h_out = h_out;
-  lo.part = m->part;
-  lo.d = c.d_model;
-  lo.np = m->np;
-  lo.last = 1;
-  lo.first = jr <= 0;
-  lo.p_bf16 = m->bf16;
-  lo.xl_bf16 = m->bf16;
-  lo.router = 0;
-  const hero_status sb = block_body(m, jj, jr, T, bs, h_bar, lo, tau_exec, flags,
-                                    (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr, gate_out,
-                                    mask_out, ffn_count_out, st);
+  const BlockState bs = dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr}
+                              : BlockState{s->S, s->zeta, s->p_hist, s->m_hist, s->d_prev};
+  const hero_status sb =
+      routed_block_run(m, block - 1, (int)n_tokens, h_bar, bs, dense ? nullptr : s->h_bar_prev,
+                       dense ? nullptr : s->delta_prev, tau_exec, flags, mask_in, h_out, gate_out,
+                       mask_out, ffn_count_out, st);
   if (sb != HERO_OK) return sb;
   CUDA_TRY(cudaEventRecord(m->ev_kernels_done, st));
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
+                                      const hero_attn_weights_host* w) {
+  g_last_error.clear();
+  if (!m || !ac || !w) return fail(HERO_ERR_ARG, "model, config and weights are required");
+  if (m->attn) return fail(HERO_ERR_ARG, "the model already has its attention parameters");
+  if (!m->bf16) return fail(HERO_ERR_UNSUPPORTED, "the attention sublayer needs a bf16 model");
+  const hero_config& c = m->cfg;
+  const long L = c.n_layers, d = c.d_model, H = ac->n_heads, Hkv = ac->n_kv_heads;
+  if (H < 1 || Hkv < 1 || H % Hkv) return fail(HERO_ERR_ARG, "need H >= 1, H_kv >= 1, H_kv | H");
+  if (d != 128 * H) return fail(HERO_ERR_UNSUPPORTED, "head dimension must be 128 (d = 128 H)");
+  if (!(ac->rope_theta > 1.f)) return fail(HERO_ERR_ARG, "rope_theta must be > 1");
+  if (!w->attn_norm_g || !w->w_q || !w->w_k || !w->w_v || !w->w_o)
+    return fail(HERO_ERR_ARG, "an attention weight pointer is NULL");
+  if (w->host_dtype != HERO_F32 && w->host_dtype != HERO_BF16)
+    return fail(HERO_ERR_ARG, "unknown host_dtype");
+  CUDA_TRY(cudaSetDevice(m->device));
+  const long nqkv = (H + 2 * Hkv) * 128, Tm = c.max_tokens;
+  const size_t hes = w->host_dtype == HERO_BF16 ? 2 : 4;
+  CUDA_TRY(cudaMalloc(&m->wqkv, (size_t)L * nqkv * d * 2));
+  CUDA_TRY(cudaMalloc(&m->wo, (size_t)L * d * d * 2));
+  CUDA_TRY(cudaMalloc(&m->attn_gain, (size_t)L * d * 4));
+  const size_t stage_elems = (size_t)16 << 20;
+  void* stage = nullptr;
+  CUDA_TRY(cudaMalloc(&stage, stage_elems * 4));
+  hero_status st = HERO_OK;
+  for (long j = 0; j < L && st == HERO_OK; ++j) {
+    char* q = static_cast<char*>(m->wqkv) + (size_t)j * nqkv * d * 2;
+    st = upload_rows(m, static_cast<const char*>(w->w_q) + (size_t)j * H * 128 * d * hes,
+                     w->host_dtype, q, H * 128, d, 1, 1, 0, nullptr, stage, stage_elems);
+    if (st == HERO_OK)
+      st = upload_rows(m, static_cast<const char*>(w->w_k) + (size_t)j * Hkv * 128 * d * hes,
+                       w->host_dtype, q, Hkv * 128, d, 1, 1, H * 128, nullptr, stage, stage_elems);
+    if (st == HERO_OK)
+      st = upload_rows(m, static_cast<const char*>(w->w_v) + (size_t)j * Hkv * 128 * d * hes,
+                       w->host_dtype, q, Hkv * 128, d, 1, 1, (H + Hkv) * 128, nullptr, stage,
+                       stage_elems);
+    if (st == HERO_OK)
+      st = upload_rows(m, static_cast<const char*>(w->w_o) + (size_t)j * d * d * hes, w->host_dtype,
+                       static_cast<char*>(m->wo) + (size_t)j * d * d * 2, d, d, 1, 1, 0, nullptr,
+                       stage, stage_elems);
+  }
+  cudaFree(stage);
+  if (st != HERO_OK) return st;
+  std::vector<float> gains = host_f32(w->attn_norm_g, (size_t)L * d, w->host_dtype);
+  CUDA_TRY(cudaMemcpy(m->attn_gain, gains.data(), gains.size() * 4, cudaMemcpyHostToDevice));
+  // workspace: x and o (bf16 [T,d]), qkv (fp32), Q/K/V (bf16), the decoder's current
+  // h and its carried h_bar_prev / delta_prev (fp32 [T,d])
+  struct Item {
+    void** p;
+    size_t bytes;
+  };
+  std::vector<Item> items = {
+      {&m->ax, (size_t)Tm * d * 2},          {&m->ao, (size_t)Tm * d * 2},
+      {(void**)&m->aqkv, (size_t)Tm * nqkv * 4}, {&m->aq, (size_t)Tm * H * 128 * 2},
+      {&m->ak, (size_t)Tm * Hkv * 128 * 2},  {&m->av, (size_t)Tm * Hkv * 128 * 2},
+      {(void**)&m->hcur, (size_t)Tm * d * 4}, {(void**)&m->hbprev, (size_t)Tm * d * 4},
+      {(void**)&m->dlprev, (size_t)Tm * d * 4}};
+  size_t off = 0;
+  for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
+  CUDA_TRY(cudaMalloc(&m->aws, off));
+  off = 0;
+  for (auto& it : items) {
+    *it.p = static_cast<char*>(m->aws) + off;
+    off += (it.bytes + 1023) & ~(size_t)1023;
+  }
+  bool ok = encode_bf16_2d(&m->tm_ax, m->ax, d, Tm, 128) && encode_bf16_2d(&m->tm_ao, m->ao, d, Tm, 128);
+  m->tm_wqkv.resize(L);
+  m->tm_wo.resize(L);
+  for (long j = 0; j < L && ok; ++j)
+    ok = encode_bf16_2d(&m->tm_wqkv[j], static_cast<char*>(m->wqkv) + (size_t)j * nqkv * d * 2, d,
+                        nqkv, 256) &&
+         encode_bf16_2d(&m->tm_wo[j], static_cast<char*>(m->wo) + (size_t)j * d * d * 2, d, d, 256);
+  if (!ok) return fail(HERO_ERR_CUDA, "tensor map encoding failed");
+  m->n_heads = (int)H;
+  m->n_kv_heads = (int)Hkv;
+  m->rope_theta = ac->rope_theta;
+  m->attn = true;
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_attention_block(hero_model* m, int32_t layer, int32_t n_seqs,
+                                            int32_t seq_len, const float* h, float* h_bar,
+                                            void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->attn) return fail(HERO_ERR_ARG, "hero_attn_init has not been called");
+  const hero_config& c = m->cfg;
+  if (layer < 1 || layer > c.n_layers)
+    return fail(HERO_ERR_ARG, "layer %d outside [1, %d]", layer, c.n_layers);
+  if (n_seqs < 0 || n_seqs > 65535 || seq_len < 1 || (long)n_seqs * seq_len > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_seqs x seq_len outside [0, max_tokens=%d] (n_seqs <= 65535)",
+                c.max_tokens);
+  if (n_seqs == 0) return HERO_OK;
+  if (!h || !h_bar) return fail(HERO_ERR_ARG, "h and h_bar are required");
+  if ((const void*)h == (const void*)h_bar) return fail(HERO_ERR_ARG, "h_bar must not alias h");
+  CUDA_TRY(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const hero_status s = attention_run(m, layer - 1, n_seqs, seq_len, h, h_bar, st);
+  if (s != HERO_OK) return s;
+  CUDA_TRY(cudaEventRecord(m->ev_kernels_done, st));
+  return HERO_OK;
+}
+
+namespace {
+
+// The decoder forward on device buffers (h_in may be m->hcur: layer 1 reads it into
+// h_bar before anything writes hcur).
+hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_in, float tau_exec,
+                        uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
+                        uint8_t* mask_out, int32_t* ffn_count_out, cudaStream_t st) {
+  const hero_config& c = m->cfg;
+  const int L = c.n_layers, T = n_seqs * seq_len;
+  if (!(flags & HERO_FLAG_DENSE))
+    CUDA_TRY(launch_state_reset(m->S, m->zeta, m->pst, m->mst, m->dprev, T, c.d_m, st));
+  const BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
+  const float* h = h_in;
+  for (int jj = 0; jj < L; ++jj) {
+    hero_status s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st);   // Eq. 1
+    if (s != HERO_OK) return s;
+    float* out = jj == L - 1 ? h_out : m->hcur;
+    s = routed_block_run(m, jj, T, m->hbar, bs, m->hbprev, m->dlprev, tau_exec, flags,
+                         mask_in ? mask_in + (size_t)jj * T : nullptr, out,
+                         gate_out ? gate_out + (size_t)jj * T : nullptr,
+                         mask_out ? mask_out + (size_t)jj * T : nullptr,
+                         ffn_count_out ? ffn_count_out + jj : nullptr, st);
+    if (s != HERO_OK) return s;
+    h = out;
+  }
+  CUDA_TRY(cudaEventRecord(m->ev_kernels_done, st));
+  return HERO_OK;
+}
+
+}  // namespace
+
+extern "C" hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len,
+                                            const float* h_in, float tau_exec, uint32_t flags,
+                                            const uint8_t* mask_in, float* h_out, float* gate_out,
+                                            uint8_t* mask_out, int32_t* ffn_count_out,
+                                            void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->attn) return fail(HERO_ERR_ARG, "hero_attn_init has not been called");
+  const hero_config& c = m->cfg;
+  const int L = c.n_layers, d = c.d_model;
+  if (n_seqs < 0 || n_seqs > 65535 || seq_len < 1 || (long)n_seqs * seq_len > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_seqs x seq_len outside [0, max_tokens=%d] (n_seqs <= 65535)",
+                c.max_tokens);
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO))
+    return fail(HERO_ERR_ARG, "unknown flag bits 0x%x", flags);
+  if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
+    return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
+  if (!std::isfinite(tau_exec)) return fail(HERO_ERR_ARG, "tau_exec is not finite");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const int T = n_seqs * seq_len;
+  const bool host = flags & HERO_FLAG_HOST_IO;
+  CUDA_TRY(cudaSetDevice(m->device));
+  if (T == 0) {
+    if (ffn_count_out) {
+      if (host)
+        memset(ffn_count_out, 0, (size_t)L * 4);
+      else
+        CUDA_TRY(cudaMemsetAsync(ffn_count_out, 0, (size_t)L * 4, st));
+    }
+    return HERO_OK;
+  }
+  if (!h_in || !h_out) return fail(HERO_ERR_ARG, "h_in and h_out are required");
+  if ((const void*)h_in == (const void*)h_out) return fail(HERO_ERR_ARG, "h_out must not alias h_in");
+  if ((flags & HERO_FLAG_FORCE_MASK) && !mask_in)
+    return fail(HERO_ERR_ARG, "HERO_FLAG_FORCE_MASK needs mask_in");
+  flags &= ~(uint32_t)HERO_FLAG_HOST_IO;
+  if (!host)
+    return decoder_run(m, n_seqs, seq_len, h_in, tau_exec, flags, mask_in, h_out, gate_out,
+                       mask_out, ffn_count_out, st);
+
+  // Host I/O: h_0 straight into the decoder's running-h buffer, outputs staged in the
+  // I/O area and copied back on the stream.
+  const size_t lt = (size_t)L * T;
+  const size_t need = (size_t)T * d * 4 + lt /*mask_in*/ + lt * 4 + lt + (size_t)L * 4 + 4096;
+  hero_status s = ensure_io(m, need);
+  if (s != HERO_OK) return s;
+  char* p = static_cast<char*>(m->io);
+  auto carve = [&](size_t bytes) {
+    char* q = p;
+    p += (bytes + 255) & ~(size_t)255;
+    return q;
+  };
+  float* d_hout = reinterpret_cast<float*>(carve((size_t)T * d * 4));
+  uint8_t* d_mask_in = (flags & HERO_FLAG_FORCE_MASK) ? reinterpret_cast<uint8_t*>(carve(lt)) : nullptr;
+  float* d_gate = gate_out ? reinterpret_cast<float*>(carve(lt * 4)) : nullptr;
+  uint8_t* d_mask = mask_out ? reinterpret_cast<uint8_t*>(carve(lt)) : nullptr;
+  int32_t* d_cnt = ffn_count_out ? reinterpret_cast<int32_t*>(carve((size_t)L * 4)) : nullptr;
+  CUDA_TRY(cudaMemcpyAsync(m->hcur, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
+  if (d_mask_in) CUDA_TRY(cudaMemcpyAsync(d_mask_in, mask_in, lt, cudaMemcpyHostToDevice, st));
+  s = decoder_run(m, n_seqs, seq_len, m->hcur, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask,
+                  d_cnt, st);
+  if (s != HERO_OK) return s;
+  CUDA_TRY(cudaMemcpyAsync(h_out, d_hout, (size_t)T * d * 4, cudaMemcpyDeviceToHost, st));
+  if (d_gate) CUDA_TRY(cudaMemcpyAsync(gate_out, d_gate, lt * 4, cudaMemcpyDeviceToHost, st));
+  if (d_mask) CUDA_TRY(cudaMemcpyAsync(mask_out, d_mask, lt, cudaMemcpyDeviceToHost, st));
+  if (d_cnt) CUDA_TRY(cudaMemcpyAsync(ffn_count_out, d_cnt, (size_t)L * 4, cudaMemcpyDeviceToHost, st));
   return HERO_OK;
 }
 

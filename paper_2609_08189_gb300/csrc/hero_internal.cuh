@@ -80,6 +80,7 @@ enum EpiKind : int {
   EPI_LAYER_OUT = 3,   // LayerOutArgs
   EPI_LAYER_OUT_WIDE = 4,  // the same with twice the epilogue warps, for launches whose
                            // time is the epilogue's (the adapter's rank-d_r up projection)
+  EPI_RESIDUAL = 5,    // out_f32[m, n] = acc + resid[m, n]  (attention output projection)
 };
 
 struct GemmArgs {
@@ -97,6 +98,7 @@ struct GemmArgs {
   // range s stores its partial sums at out_f32 + s * split_stride
   int k_splits;        // 0 or 1: no split
   long split_stride;
+  const float* resid;  // EPI_RESIDUAL: [rows, N] fp32 added to the product (ld = ldo)
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
@@ -128,6 +130,14 @@ constexpr int kSimtTileN = 64;
 // Columns per partial-sum slot of the block-closing epilogues: bf16 models (tensor
 // core path) use half a 256-column tile, f32 models the SIMT tile width.
 constexpr int kTcPartCols = 128;
+
+// Attention sublayer kernels (attention.cu), head dimension 128 --------------------
+cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float eps, void* x,
+                             cudaStream_t st);
+cudaError_t launch_rope(const float* qkv, int B, int S, int H, int Hkv, float theta, void* Q, void* K,
+                        void* V, cudaStream_t st);
+cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
+                              int Hkv, void* O, cudaStream_t st);
 
 // Router and bookkeeping kernels ------------------------------------------------
 

@@ -24,7 +24,8 @@ HERO_F32, HERO_BF16 = 0, 1
 HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO = 1, 2, 4
 HERO_ROUTER_NO_HISTORY, HERO_ROUTER_NO_MEMREAD, HERO_ROUTER_NO_AUX, HERO_ROUTER_NO_POS = 1, 2, 4, 8
 KERNEL_CLASSES = ("init", "router_gemm", "router", "compact", "norm", "ffn_gate_up", "ffn_down",
-                  "adapter_down", "adapter_up")
+                  "adapter_down", "adapter_up", "attn_proj", "attn_core")
+ATTN_WEIGHT_FIELDS = ("attn_norm_g", "w_q", "w_k", "w_v", "w_o")
 HERO_K_COUNT = len(KERNEL_CLASSES)
 
 WEIGHT_FIELDS = ("ffn_norm_g", "w_gate", "w_up", "w_down", "ad_w1", "ad_w2", "eta",
@@ -44,6 +45,15 @@ class hero_config(ctypes.Structure):
 
 class hero_weights_host(ctypes.Structure):
     _fields_ = [("host_dtype", ctypes.c_int)] + [(n, ctypes.c_void_p) for n in WEIGHT_FIELDS]
+
+
+class hero_attn_config(ctypes.Structure):
+    _fields_ = [("n_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("rope_theta", ctypes.c_float)]
+
+
+class hero_attn_weights_host(ctypes.Structure):
+    _fields_ = [("host_dtype", ctypes.c_int)] + [(n, ctypes.c_void_p) for n in ATTN_WEIGHT_FIELDS]
 
 
 STATE_FIELDS = ("S", "zeta", "p_hist", "m_hist", "d_prev", "h_bar_prev", "delta_prev")
@@ -94,6 +104,13 @@ def load(path: Optional[str] = None) -> ctypes.CDLL:
     lib.hero_routed_block.argtypes = [vp, i32, i64, vp, ctypes.POINTER(hero_router_state), f32, u32,
                                       vp, vp, vp, vp, vp, vp]
     lib.hero_routed_block.restype = ctypes.c_int
+    lib.hero_attn_init.argtypes = [vp, ctypes.POINTER(hero_attn_config),
+                                   ctypes.POINTER(hero_attn_weights_host)]
+    lib.hero_attn_init.restype = ctypes.c_int
+    lib.hero_attention_block.argtypes = [vp, i32, i32, i32, vp, vp, vp]
+    lib.hero_attention_block.restype = ctypes.c_int
+    lib.hero_decoder_forward.argtypes = [vp, i32, i32, vp, f32, u32, vp, vp, vp, vp, vp, vp]
+    lib.hero_decoder_forward.restype = ctypes.c_int
     lib.hero_gemm_bf16_splitk_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     lib.hero_gemm_bf16_splitk_noalloc.restype = ctypes.c_int
     _lib = lib
@@ -200,6 +217,37 @@ def hero_gemm_bf16_splitk_noalloc(A: int, B: int, C: int, M: int, N: int, K: int
     _check(load().hero_gemm_bf16_splitk_noalloc(A, B, C, M, N, K, splits, cuda_stream or None))
 
 
+def hero_attn_init(model: int, stack_cfg, attn_weights: Dict[str, np.ndarray]) -> None:
+    """Attach the attention parameters (canonical layouts, stacked over layers)."""
+    arrs = {k: np.ascontiguousarray(attn_weights[k]) for k in ATTN_WEIGHT_FIELDS}
+    dts = {a.dtype for a in arrs.values()}
+    if dts == {np.dtype(np.uint16)}:
+        hd = HERO_BF16
+    elif dts == {np.dtype(np.float32)}:
+        hd = HERO_F32
+    else:
+        raise ValueError(f"attention weights must all be uint16 (bf16 bits) or float32, got {dts}")
+    w = hero_attn_weights_host(hd, *[a.ctypes.data for a in arrs.values()])
+    c = hero_attn_config(stack_cfg.n_heads, stack_cfg.n_kv_heads, stack_cfg.rope_theta)
+    _check(load().hero_attn_init(model, ctypes.byref(c), ctypes.byref(w)))
+
+
+def hero_attention_block(model: int, layer: int, n_seqs: int, seq_len: int, h: int, h_bar: int,
+                         cuda_stream: int) -> None:
+    """Eq. 1, first line, for one layer (pointer-level call)."""
+    _check(load().hero_attention_block(model, layer, n_seqs, seq_len, h or None, h_bar or None,
+                                       cuda_stream or None))
+
+
+def hero_decoder_forward(model: int, n_seqs: int, seq_len: int, h_in: int, tau_exec: float,
+                         flags: int, mask_in: int, h_out: int, gate_out: int, mask_out: int,
+                         ffn_count_out: int, cuda_stream: int) -> None:
+    """The full decoder forward (pointer-level call)."""
+    _check(load().hero_decoder_forward(model, n_seqs, seq_len, h_in or None, float(tau_exec), flags,
+                                       mask_in or None, h_out or None, gate_out or None,
+                                       mask_out or None, ffn_count_out or None, cuda_stream or None))
+
+
 # ---------------------------------------------------------------------------
 # PyTorch convenience layer (device tensors, current stream)
 # ---------------------------------------------------------------------------
@@ -254,3 +302,42 @@ class HeroStack:
         import torch
         st = stream if stream is not None else torch.cuda.current_stream()
         hero_check_device_status(self.model, st.cuda_stream)
+
+
+class HeroDecoder(HeroStack):
+    """A routed stack with its attention sublayers: the full decoder forward."""
+
+    def __init__(self, stack_cfg, weights: Dict[str, np.ndarray],
+                 attn_weights: Dict[str, np.ndarray], max_tokens: Optional[int] = None):
+        super().__init__(stack_cfg, weights, max_tokens)
+        hero_attn_init(self.model, stack_cfg, attn_weights)
+
+    def attention(self, layer: int, h, n_seqs: int, seq_len: int, h_bar=None, stream=None):
+        """h_bar = h + Attn(LN_attn(h)) of one layer (1-based), device tensors."""
+        import torch
+        T, d = h.shape
+        assert T == n_seqs * seq_len and h.is_contiguous()
+        h_bar = h_bar if h_bar is not None else torch.empty_like(h)
+        st = stream if stream is not None else torch.cuda.current_stream(h.device)
+        hero_attention_block(self.model, layer, n_seqs, seq_len, h.data_ptr(), h_bar.data_ptr(),
+                             st.cuda_stream)
+        return h_bar
+
+    def forward(self, h_in, tau: float, n_seqs: int, seq_len: int, flags: int = 0, mask_in=None,
+                h_out=None, gate_out=None, mask_out=None, counts_out=None, stream=None):
+        """Device tensors in and out.  Returns (h_out, gate, mask, counts)."""
+        import torch
+        T, d = h_in.shape
+        assert T == n_seqs * seq_len and h_in.is_contiguous()
+        L = self.cfg.n_layers
+        dev = h_in.device
+        h_out = h_out if h_out is not None else torch.empty((T, d), dtype=torch.float32, device=dev)
+        gate_out = gate_out if gate_out is not None else torch.empty((L, T), dtype=torch.float32, device=dev)
+        mask_out = mask_out if mask_out is not None else torch.empty((L, T), dtype=torch.uint8, device=dev)
+        counts_out = counts_out if counts_out is not None else torch.empty((L,), dtype=torch.int32, device=dev)
+        st = stream if stream is not None else torch.cuda.current_stream(dev)
+        hero_decoder_forward(self.model, n_seqs, seq_len, h_in.data_ptr(), tau, flags,
+                             mask_in.data_ptr() if mask_in is not None else 0, h_out.data_ptr(),
+                             gate_out.data_ptr(), mask_out.data_ptr(), counts_out.data_ptr(),
+                             st.cuda_stream)
+        return h_out, gate_out, mask_out, counts_out

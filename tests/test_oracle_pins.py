@@ -739,3 +739,14 @@ def test_attention_single_token_is_value_path():
     v = (x @ wa["w_v"].T).reshape(6, Hkv, hd)
     o = np.repeat(v, H // Hkv, axis=1).reshape(6, H * hd)
     np.testing.assert_allclose(got, h + o @ wa["w_o"].T, rtol=0, atol=1e-12)
+
+
+def test_attention_rows_equals_full_sublayer():
+    """The sampled-position form (used to check long sequences) equals the full one."""
+    cfg, wa, h = _attn_inputs(seq_len=40, n_seqs=1)
+    full = ho.attention_sublayer(h, wa, cfg.n_heads, cfg.n_kv_heads, cfg.rope_theta, 1, 40,
+                                 cfg.rms_eps, ho.bf16_round)
+    rows = np.array([0, 7, 19, 39])
+    got = ho.attention_rows(h, rows, wa, cfg.n_heads, cfg.n_kv_heads, cfg.rope_theta, cfg.rms_eps,
+                            ho.bf16_round)
+    np.testing.assert_allclose(got, full[rows], rtol=0, atol=1e-12)
