@@ -1,7 +1,7 @@
 // The attention sublayer of Eq. 1 (the full decoder forward), bf16 models:
 //   x = LN_attn(h)                      k_attn_norm (bf16 rows, the projection operand)
-//   qkv = x [W_q; W_k; W_v]^T           tensor-core GEMM (gemm_tc.cu)
-//   q, k <- RoPE(q), RoPE(k)            k_rope (bf16, [sequence][head][position][128])
+//   q, k, v = x [W_q; W_k; W_v]^T,      tensor-core GEMM (gemm_tc.cu) whose epilogue
+//   q, k <- RoPE(q), RoPE(k)            rotates and stores bf16 [sequence][head][position][128]
 //   o = softmax(q k^T / sqrt(hd)) v     k_flash_attn (causal, grouped-query heads)
 //   h_bar = h + o W_o^T                 tensor-core GEMM with the residual epilogue
 #include "hero_device.cuh"
@@ -39,45 +39,6 @@ __global__ void __launch_bounds__(256) k_attn_norm(const float* __restrict__ h,
            make_float4(v.x * rinv * gv.x, v.y * rinv * gv.y, v.z * rinv * gv.z, v.w * rinv * gv.w),
            1);
   }
-}
-
-// ---------------------------------------------------------------------------------
-// RoPE and layout: qkv fp32 [T][(H + 2 H_kv) 128] (q heads | k heads | v heads) ->
-// Q [B][H][S][128], K and V [B][H_kv][S][128], bf16.  Pair (i, i + 64) of a q or
-// k head at position s turns by s * theta^(-2i/128).  One thread per (token, head,
-// pair).
-// ---------------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_rope(const float* __restrict__ qkv, int B, int S, int H,
-                                              int Hkv, float log2_theta, uint16_t* __restrict__ Q,
-                                              uint16_t* __restrict__ K, uint16_t* __restrict__ V) {
-  pdl_enter();
-  const int heads = H + 2 * Hkv;
-  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (long)B * S * heads * (HD / 2)) return;
-  const int pair = (int)(i % (HD / 2));
-  const long rest = i / (HD / 2);
-  const int hh = (int)(rest % heads);
-  const long t = rest / heads;
-  const int b = (int)(t / S), s = (int)(t - (long)b * S);
-  const float* src = qkv + (size_t)t * heads * HD + (size_t)hh * HD;
-  const float x1 = src[pair], x2 = src[pair + HD / 2];
-  uint16_t* dst;
-  float y1 = x1, y2 = x2;
-  if (hh < H + Hkv) {   // q or k head: rotate
-    const float inv_freq = exp2f(-(2.0f * pair / HD) * log2_theta);
-    float sn, cs;
-    sincosf((float)s * inv_freq, &sn, &cs);
-    y1 = x1 * cs - x2 * sn;
-    y2 = x2 * cs + x1 * sn;
-  }
-  if (hh < H)
-    dst = Q + (((size_t)b * H + hh) * S + s) * HD;
-  else if (hh < H + Hkv)
-    dst = K + (((size_t)b * Hkv + (hh - H)) * S + s) * HD;
-  else
-    dst = V + (((size_t)b * Hkv + (hh - H - Hkv)) * S + s) * HD;
-  dst[pair] = (uint16_t)(pack_bf16x2(y1, 0.f) & 0xffffu);
-  dst[pair + HD / 2] = (uint16_t)(pack_bf16x2(y2, 0.f) & 0xffffu);
 }
 
 // ---------------------------------------------------------------------------------
@@ -300,15 +261,6 @@ cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float
   if (d % 128) return cudaErrorInvalidValue;
   return launch_pdl(k_attn_norm, dim3((unsigned)((T + 7) / 8)), dim3(256), 0, st, h, g, T, d, eps,
                     static_cast<uint16_t*>(x));
-}
-
-cudaError_t launch_rope(const float* qkv, int B, int S, int H, int Hkv, float theta, void* Q, void* K,
-                        void* V, cudaStream_t st) {
-  const long n = (long)B * S * (H + 2 * Hkv) * (HD / 2);
-  if (n <= 0) return cudaSuccess;
-  return launch_pdl(k_rope, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, qkv, B, S, H, Hkv,
-                    log2f(theta), static_cast<uint16_t*>(Q), static_cast<uint16_t*>(K),
-                    static_cast<uint16_t*>(V));
 }
 
 cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,

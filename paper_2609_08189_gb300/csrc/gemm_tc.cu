@@ -50,7 +50,7 @@ struct TcCfg {
 };
 
 template <int EPI>
-constexpr int epi_warps() { return EPI == EPI_LAYER_OUT_WIDE ? 8 : 4; }
+constexpr int epi_warps() { return EPI == EPI_LAYER_OUT_WIDE || EPI == EPI_ATTN_ENTRY ? 8 : 4; }
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
   const int group = kGroupM * n_tiles;
@@ -158,6 +158,63 @@ __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int 
   }
 }
 
+// Fused q/k/v projection epilogue: one thread = one token row; the two halves of a
+// head (columns i and i + 64) are read from TMEM together, q and k heads are
+// rotated (RoPE, fp32), and each head's 128 values are stored as bf16 into its
+// [sequence][head][position][128] array (64 contiguous bytes per store group).
+template <int BN>
+__device__ __forceinline__ void epi_qkv_rope(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                             int nb) {
+  static_assert(BN % 128 == 0, "whole heads per tile");
+  const RopeArgs& r = a.rope;
+  const int heads = r.H + 2 * r.Hkv;
+  const int bq = valid ? m / r.S : 0;
+  const int s = valid ? m - bq * r.S : 0;
+#pragma unroll 1
+  for (int hb = 0; hb < BN; hb += 128) {
+    const int head = (nb * BN + hb) >> 7;
+    if (head >= heads) break;                      // uniform over the warp
+#pragma unroll 1
+    for (int c0 = 0; c0 < 64; c0 += 32) {
+      uint32_t x1[32], x2[32];
+      tmem_ld32(tbase + hb + c0, x1);
+      tmem_ld32(tbase + hb + c0 + 64, x2);
+      if (!valid) continue;
+      uint16_t* dst;
+      const bool rot = head < r.H + r.Hkv;
+      if (head < r.H)
+        dst = static_cast<uint16_t*>(r.q) + (((size_t)bq * r.H + head) * r.S + s) * 128;
+      else if (rot)
+        dst = static_cast<uint16_t*>(r.k) + (((size_t)bq * r.Hkv + head - r.H) * r.S + s) * 128;
+      else
+        dst = static_cast<uint16_t*>(r.v) +
+              (((size_t)bq * r.Hkv + head - r.H - r.Hkv) * r.S + s) * 128;
+      uint32_t p1[16], p2[16];
+      const float4* cs = reinterpret_cast<const float4*>(r.cs + ((size_t)s * 64 + c0) * 2);
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        float a0 = __uint_as_float(x1[e]), a1 = __uint_as_float(x1[e + 1]);
+        float b0 = __uint_as_float(x2[e]), b1 = __uint_as_float(x2[e + 1]);
+        if (rot) {
+          const float4 t = __ldg(cs + (e >> 1));   // (cos, sin) of pairs e and e + 1
+          const float y0 = a0 * t.x - b0 * t.y, z0 = b0 * t.x + a0 * t.y;
+          const float y1 = a1 * t.z - b1 * t.w, z1 = b1 * t.z + a1 * t.w;
+          a0 = y0; b0 = z0; a1 = y1; b1 = z1;
+        }
+        p1[e >> 1] = pack_bf16x2(a0, a1);
+        p2[e >> 1] = pack_bf16x2(b0, b1);
+      }
+      uint4* d1 = reinterpret_cast<uint4*>(dst + c0);
+      uint4* d2 = reinterpret_cast<uint4*>(dst + c0 + 64);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        d1[i] = make_uint4(p1[4 * i], p1[4 * i + 1], p1[4 * i + 2], p1[4 * i + 3]);
+        d2[i] = make_uint4(p2[4 * i], p2[4 * i + 1], p2[4 * i + 2], p2[4 * i + 3]);
+      }
+    }
+  }
+}
+
 // Block-closing epilogue over columns [c_begin, c_begin + NCOLS) of the tile,
 // row-contiguous through the staging tile.  Each lane keeps the partial sums of
 // its 8 rows; every kTcPartCols columns they are reduced over the 8 lanes that
@@ -221,6 +278,75 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
     }
     __syncwarp();
     if (!p.last && (c0 + 32) % kTcPartCols == 0)
+      flush_partials<BN, NCOLS>(p, tok, ss, dd, dp, slot, (nb * BN + c0 + 32) / kTcPartCols - 1);
+  }
+}
+
+// Attention output projection closing into the block entry (Eq. 7): per element
+// h_bar_j = h_{j-1} + acc, delta_j = h_bar_j - h_bar_{j-1} (zero in the first routed
+// block); h_bar_j and delta_j overwrite the carried h_bar_{j-1} and delta_{j-1}
+// after the same thread has read them; partial sums of h_bar_j^2, delta_j^2 and
+// delta_j . delta_{j-1} per 128-column slot.  Rows are tokens.
+template <int BN, int NCOLS>
+__device__ __forceinline__ void epi_attn_entry(const GemmArgs& a, uint32_t tbase, int row0, int M,
+                                               int nb, int c_begin, float4* st) {
+  static_assert(NCOLS % kTcPartCols == 0, "whole partial-sum slots per warp");
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> 3, slot = lane & 7;
+  const LayerOutArgs& p = a.lo;
+  const bool rt = p.router, carry = p.router && !p.first;
+  int tok[8];
+  float ss[8], dd[8], dp[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int m = row0 + sub + 4 * k;
+    tok[k] = m < M ? m : -1;
+    ss[k] = dd[k] = dp[k] = 0.f;
+  }
+#pragma unroll 1
+  for (int c0 = c_begin; c0 < c_begin + NCOLS; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    stage_rows(st, r, lane);
+    __syncwarp();
+    const int n = nb * BN + c0 + 4 * slot;
+#pragma unroll
+    for (int k0 = 0; k0 < 8; k0 += 4) {
+      float4 hr[4], hp[4], dv[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = tok[k0 + k];
+        if (t < 0) continue;
+        const size_t off = (size_t)t * p.d + n;
+        hr[k] = *reinterpret_cast<const float4*>(a.resid + off);
+        if (carry) {
+          hp[k] = *reinterpret_cast<const float4*>(p.hbar + off);
+          dv[k] = *reinterpret_cast<const float4*>(p.delta + off);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = tok[k0 + k];
+        if (t < 0) continue;
+        const size_t off = (size_t)t * p.d + n;
+        const float4 y = staged(st, sub + 4 * (k0 + k), slot);
+        const float4 hn = make_float4(hr[k].x + y.x, hr[k].y + y.y, hr[k].z + y.z, hr[k].w + y.w);
+        *reinterpret_cast<float4*>(p.hbar + off) = hn;
+        ss[k0 + k] += hn.x * hn.x + hn.y * hn.y + hn.z * hn.z + hn.w * hn.w;
+        if (rt) {
+          float4 dl = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (carry) {
+            dl = make_float4(hn.x - hp[k].x, hn.y - hp[k].y, hn.z - hp[k].z, hn.w - hp[k].w);
+            dp[k0 + k] += dl.x * dv[k].x + dl.y * dv[k].y + dl.z * dv[k].z + dl.w * dv[k].w;
+          }
+          dd[k0 + k] += dl.x * dl.x + dl.y * dl.y + dl.z * dl.z + dl.w * dl.w;
+          *reinterpret_cast<float4*>(p.delta + off) = dl;
+          store_xl4(p.xl, p.xl_bf16, p.d, t, n, hn);
+        }
+      }
+    }
+    __syncwarp();
+    if ((c0 + 32) % kTcPartCols == 0)
       flush_partials<BN, NCOLS>(p, tok, ss, dd, dp, slot, (nb * BN + c0 + 32) / kTcPartCols - 1);
   }
 }
@@ -292,6 +418,10 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
     epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
   } else if constexpr (EPI == EPI_RESIDUAL) {
     epi_store_f32<BN, true>(a, tbase, row0, M, nb, split, stg);
+  } else if constexpr (EPI == EPI_ATTN_ENTRY) {
+    epi_attn_entry<BN, BN / 2>(a, tbase, row0, M, nb, (ew >> 2) * (BN / 2), stg);
+  } else if constexpr (EPI == EPI_QKV_ROPE) {
+    epi_qkv_rope<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_SWIGLU) {
     epi_swiglu(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_SILU) {
@@ -544,6 +674,13 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
                                                           st);
     case EPI_RESIDUAL:
       return launch_tc<256, EPI_RESIDUAL, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_QKV_ROPE:
+      if (args.N != (args.rope.H + 2 * args.rope.Hkv) * 128 || args.rope.S <= 0)
+        return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_QKV_ROPE, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_ATTN_ENTRY:
+      if (args.lo.d != args.N || args.ldo != args.N) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_ATTN_ENTRY, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

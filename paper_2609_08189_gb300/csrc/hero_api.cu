@@ -144,7 +144,7 @@ struct hero_model {
   float* attn_gain = nullptr;  // [L][d]
   void* aws = nullptr;         // attention workspace
   void *ax = nullptr, *aq = nullptr, *ak = nullptr, *av = nullptr, *ao = nullptr;
-  float *aqkv = nullptr, *hcur = nullptr, *hbprev = nullptr, *dlprev = nullptr;
+  float *rope_cs = nullptr, *hcur = nullptr, *dlprev = nullptr;
   CUtensorMap tm_ax, tm_ao;
   std::vector<CUtensorMap> tm_wqkv, tm_wo;
 
@@ -1023,7 +1023,8 @@ namespace {
 hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, const BlockState& bs,
                              float* h_bar_prev, float* delta_prev, float tau, uint32_t flags,
                              const uint8_t* mask_in, float* h_out, float* gate_out,
-                             uint8_t* mask_out, int32_t* count_out, cudaStream_t st) {
+                             uint8_t* mask_out, int32_t* count_out, cudaStream_t st,
+                             bool entry_done = false) {
   const hero_config& c = m->cfg;
   const int jr = jj - c.n_dense;
   bool dense = flags & HERO_FLAG_DENSE;
@@ -1034,7 +1035,8 @@ hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, c
   BlockEntryArgs be{T, c.d_model, m->np, jr + 1, dense ? 0 : 1, h_bar,
                     dense ? nullptr : h_bar_prev, dense ? nullptr : delta_prev,
                     m->xl, (int)m->bf16, m->part};
-  CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
+  if (!entry_done)   // else the producer of h_bar closed into the entry (EPI_ATTN_ENTRY)
+    CUDA_TRY(timed(m, HERO_K_INIT, st, [&] { return launch_block_entry(be, st); }));
   LayerOutArgs lo{};
   lo.hbar = const_cast<float*>(h_bar);  // read only: the block writes h_out
   lo.h_out = h_out;
@@ -1052,8 +1054,10 @@ hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, c
 }
 
 // Eq. 1, first line, for layer jj on B sequences of S tokens: h_bar = h + Attn(LN_attn(h)).
+// With `entry`, the output projection also closes into the routed block's entry
+// (h_bar written over entry->hbar = h_bar_{j-1}, delta, router operand, partials).
 hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, float* h_bar,
-                          cudaStream_t st) {
+                          cudaStream_t st, const LayerOutArgs* entry = nullptr) {
   const hero_config& c = m->cfg;
   const int T = B * S, d = c.d_model, H = m->n_heads, Hkv = m->n_kv_heads;
   const int nqkv = (H + 2 * Hkv) * 128;
@@ -1065,14 +1069,11 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   g.m_max = T;
   g.N = nqkv;
   g.K = d;
-  g.out_f32 = m->aqkv;
   g.ldo = nqkv;
   g.err = m->err;
-  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
-    return launch_gemm_tc(256, EPI_STORE_F32, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
-  }));
-  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
-    return launch_rope(m->aqkv, B, S, H, Hkv, m->rope_theta, m->aq, m->ak, m->av, st);
+  g.rope = RopeArgs{m->aq, m->ak, m->av, m->rope_cs, H, Hkv, S};
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q, k, v with RoPE, attention layout
+    return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
   }));
   CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
     return launch_flash_attn(m->aq, m->ak, m->av, B, S, H, Hkv, m->ao, st);
@@ -1086,8 +1087,10 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   o.ldo = d;
   o.resid = h;
   o.err = m->err;
+  if (entry) o.lo = *entry;
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
-    return launch_gemm_tc(256, EPI_RESIDUAL, m->tm_ao, m->tm_wo[jj], o, m->num_sms, st);
+    return launch_gemm_tc(256, entry ? EPI_ATTN_ENTRY : EPI_RESIDUAL, m->tm_ao, m->tm_wo[jj], o,
+                          m->num_sms, st);
   }));
   return HERO_OK;
 }
@@ -1183,17 +1186,17 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   if (st != HERO_OK) return st;
   std::vector<float> gains = host_f32(w->attn_norm_g, (size_t)L * d, w->host_dtype);
   CUDA_TRY(cudaMemcpy(m->attn_gain, gains.data(), gains.size() * 4, cudaMemcpyHostToDevice));
-  // workspace: x and o (bf16 [T,d]), qkv (fp32), Q/K/V (bf16), the decoder's current
-  // h and its carried h_bar_prev / delta_prev (fp32 [T,d])
+  // workspace: x and o (bf16 [T,d]), the RoPE table, Q/K/V (bf16), the decoder's current
+  // h and its carried delta (fp32 [T,d]; h_bar_{j-1} is carried in the model's h_bar)
   struct Item {
     void** p;
     size_t bytes;
   };
   std::vector<Item> items = {
       {&m->ax, (size_t)Tm * d * 2},          {&m->ao, (size_t)Tm * d * 2},
-      {(void**)&m->aqkv, (size_t)Tm * nqkv * 4}, {&m->aq, (size_t)Tm * H * 128 * 2},
+      {(void**)&m->rope_cs, (size_t)Tm * 64 * 2 * 4}, {&m->aq, (size_t)Tm * H * 128 * 2},
       {&m->ak, (size_t)Tm * Hkv * 128 * 2},  {&m->av, (size_t)Tm * Hkv * 128 * 2},
-      {(void**)&m->hcur, (size_t)Tm * d * 4}, {(void**)&m->hbprev, (size_t)Tm * d * 4},
+      {(void**)&m->hcur, (size_t)Tm * d * 4},
       {(void**)&m->dlprev, (size_t)Tm * d * 4}};
   size_t off = 0;
   for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
@@ -1202,6 +1205,16 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   for (auto& it : items) {
     *it.p = static_cast<char*>(m->aws) + off;
     off += (it.bytes + 1023) & ~(size_t)1023;
+  }
+  {   // RoPE (cos, sin) of s * theta^(-2i/128) for positions s < max_tokens, in double
+    std::vector<float> cs((size_t)Tm * 64 * 2);
+    for (long p = 0; p < Tm; ++p)
+      for (int i = 0; i < 64; ++i) {
+        const double ang = (double)p * std::pow((double)ac->rope_theta, -2.0 * i / 128.0);
+        cs[((size_t)p * 64 + i) * 2] = (float)std::cos(ang);
+        cs[((size_t)p * 64 + i) * 2 + 1] = (float)std::sin(ang);
+      }
+    CUDA_TRY(cudaMemcpy(m->rope_cs, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice));
   }
   bool ok = encode_bf16_2d(&m->tm_ax, m->ax, d, Tm, 128) && encode_bf16_2d(&m->tm_ao, m->ao, d, Tm, 128);
   m->tm_wqkv.resize(L);
@@ -1255,14 +1268,28 @@ hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_i
   const BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
   const float* h = h_in;
   for (int jj = 0; jj < L; ++jj) {
-    hero_status s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st);   // Eq. 1
+    // Eq. 1 with the block entry fused into the output projection: m->hbar carries
+    // h_bar_{j-1} into the launch and h_bar_j out of it, m->dlprev likewise delta
+    const int jr = jj - c.n_dense;
+    const bool dense = (flags & HERO_FLAG_DENSE) || jr < 0;
+    LayerOutArgs entry{};
+    entry.hbar = m->hbar;
+    entry.delta = m->dlprev;
+    entry.xl = m->xl;
+    entry.part = m->part;
+    entry.d = c.d_model;
+    entry.np = m->np;
+    entry.first = jr <= 0;
+    entry.xl_bf16 = 1;
+    entry.router = dense ? 0 : 1;
+    hero_status s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st, &entry);
     if (s != HERO_OK) return s;
     float* out = jj == L - 1 ? h_out : m->hcur;
-    s = routed_block_run(m, jj, T, m->hbar, bs, m->hbprev, m->dlprev, tau_exec, flags,
+    s = routed_block_run(m, jj, T, m->hbar, bs, nullptr, m->dlprev, tau_exec, flags,
                          mask_in ? mask_in + (size_t)jj * T : nullptr, out,
                          gate_out ? gate_out + (size_t)jj * T : nullptr,
                          mask_out ? mask_out + (size_t)jj * T : nullptr,
-                         ffn_count_out ? ffn_count_out + jj : nullptr, st);
+                         ffn_count_out ? ffn_count_out + jj : nullptr, st, true);
     if (s != HERO_OK) return s;
     h = out;
   }

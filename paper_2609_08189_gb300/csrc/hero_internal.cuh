@@ -81,6 +81,23 @@ enum EpiKind : int {
   EPI_LAYER_OUT_WIDE = 4,  // the same with twice the epilogue warps, for launches whose
                            // time is the epilogue's (the adapter's rank-d_r up projection)
   EPI_RESIDUAL = 5,    // out_f32[m, n] = acc + resid[m, n]  (attention output projection)
+  EPI_ATTN_ENTRY = 6,  // the same, closing into the next routed block's entry: h_bar_j =
+                       // resid + acc written over lo.hbar (= h_bar_{j-1}, read first),
+                       // delta_j over lo.delta, the router operand copy lo.xl and the
+                       // partial sums lo.part (lo.router, lo.first as in LayerOutArgs)
+  EPI_QKV_ROPE = 7,    // fused q/k/v projection: RoPE on the q and k heads, bf16 out in
+                       // the attention layout (RopeArgs)
+};
+
+// EPI_QKV_ROPE: columns are heads of 128 (q heads | k heads | v heads); row t is
+// position t % S of sequence t / S.  Pair (i, i + 64) of a q or k head at position s
+// turns by the angle s * theta^(-2i/128), whose (cos, sin) come from cs.
+struct RopeArgs {
+  void* q;             // bf16 [B][H][S][128]
+  void* k;             // bf16 [B][H_kv][S][128]
+  void* v;             // bf16 [B][H_kv][S][128]
+  const float* cs;     // [positions >= S][64][2]: cos, sin
+  int H, Hkv, S;
 };
 
 struct GemmArgs {
@@ -99,6 +116,7 @@ struct GemmArgs {
   int k_splits;        // 0 or 1: no split
   long split_stride;
   const float* resid;  // EPI_RESIDUAL: [rows, N] fp32 added to the product (ld = ldo)
+  RopeArgs rope;       // EPI_QKV_ROPE
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
@@ -134,8 +152,6 @@ constexpr int kTcPartCols = 128;
 // Attention sublayer kernels (attention.cu), head dimension 128 --------------------
 cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float eps, void* x,
                              cudaStream_t st);
-cudaError_t launch_rope(const float* qkv, int B, int S, int H, int Hkv, float theta, void* Q, void* K,
-                        void* V, cudaStream_t st);
 cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
                               int Hkv, void* O, cudaStream_t st);
 

@@ -224,8 +224,10 @@ def test_decoder_forward_parity(small_decoder, hero):
 
 def test_decoder_matches_caller_driven_blocks(small_decoder, hero):
     """hero_decoder_forward equals the caller-driven form: hero_attention_block, then
-    hero_routed_block with a caller-held router state (the same kernels; tolerances
-    of the fused-versus-blockwise stack test)."""
+    hero_routed_block with a caller-held router state.  The same arithmetic except
+    the order of the fp32 sums behind the block entry's norms (the decoder's output
+    projection sums per 128-column slot, k_block_entry per row), so decisions agree
+    exactly and gates and states to 1e-4, ten times inside the oracle bound."""
     import torch
     cfg, w, wa, dec = small_decoder
     B, S = cfg.batch, cfg.seq_len
@@ -251,10 +253,12 @@ def test_decoder_matches_caller_driven_blocks(small_decoder, hero):
                                gs[j - 1].data_ptr(), ms[j - 1].data_ptr(), 0, stream)
     torch.cuda.synchronize()
     dec.check()
+    gerr = float((gs - g).abs().max())
+    err = float(np.max(pr.rel_err_rows(x.cpu().numpy().astype(np.float64),
+                                       h_out.cpu().numpy().astype(np.float64))))
+    print("caller-driven vs fused: mask equal", bool((ms == m).all()), "gate", gerr, "h", err)
     np.testing.assert_array_equal(ms.cpu().numpy(), m.cpu().numpy())
-    assert float((gs - g).abs().max()) < 1e-5
-    err = pr.rel_err_rows(x.cpu().numpy().astype(np.float64), h_out.cpu().numpy().astype(np.float64))
-    assert float(np.max(err)) < 1e-4
+    assert gerr < 1e-4 and err < 1e-4, (gerr, err)
 
 
 def test_decoder_full_size_prefix(hero):
