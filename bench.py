@@ -14,7 +14,10 @@ data path); value = all ranks' tokens / the slowest rank's time.
 Decoder workloads (--workload llama31_8b_decoder, small_bf16_decoder) run the full
 decoder forward instead: every block's h_bar comes from the real attention
 sublayer (Eq. 1) rather than the stand-in; a step is all blocks' attention plus
-routed FFN over B sequences of S tokens.
+routed FFN over B sequences of S tokens.  The KV-cache decoding workload
+(llama31_8b_kvdecode) first fills the cache of 64 sequences with 4096-token
+prefills (untimed); a step is then one new token for each sequence at position
+4096 (every step decodes the same position: the context stays 4096).
 
 --impl reference times the CPU oracle (the only reference this method has) on a
 bounded token sample per step, on rank 0 only (decoder workloads: a causal prefix
@@ -42,9 +45,12 @@ from synth import hero_inputs as hi  # noqa: E402
 METRIC = "routed-FFN-stack tokens/s at Llama-3.1-8B shapes; % of bf16 tensor peak"
 # decoder workloads: the same tokens/s, with the attention sublayers inside the step
 METRIC_DECODER = "decoder-forward (attention + routed FFN) tokens/s at Llama-3.1-8B shapes"
+METRIC_KVDECODE = "KV-cache decoding tokens/s (attention over the cache + routed FFN) at Llama-3.1-8B shapes"
 
 
 def metric_for(cfg):
+    if cfg.kv_decode_of:
+        return METRIC_KVDECODE
     return METRIC_DECODER if cfg.n_heads else METRIC
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
@@ -71,8 +77,11 @@ def workload_desc(cfg, bypass):
     if cfg.n_heads:
         variant += (f", causal attention H={cfg.n_heads}, H_kv={cfg.n_kv_heads}, hd=128, "
                     f"RoPE theta={cfg.rope_theta:g}")
+    shape = (f"T={cfg.n_tokens} per step ({cfg.batch} sequences, one new token each at position "
+             f"{cfg.seq_len} after a {cfg.seq_len}-token cached prefix)" if cfg.kv_decode_of else
+             f"T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len})")
     return (f"{cfg.name}: {blocks}, d={cfg.d_model}, I={cfg.d_ff}, "
-            f"d_r={cfg.d_r}, d_m={cfg.d_m}, T={cfg.n_tokens} ({cfg.batch}x{cfg.seq_len}), "
+            f"d_r={cfg.d_r}, d_m={cfg.d_m}, {shape}, "
             f"{cfg.dtype}, bypass target {bypass:.2%}{variant}, random-init weights, seeded inputs")
 
 
@@ -159,9 +168,36 @@ def algorithmic_work(cfg, counts_per_step, steps, routed=True):
         nqkv = (cfg.n_heads + 2 * cfg.n_kv_heads) * hd
         B, S = cfg.batch, cfg.seq_len
         work["attn_proj"] = steps * cfg.n_layers * 2.0 * T * d * (nqkv + cfg.n_heads * hd)
-        # q k^T and p v over the causal triangle (S (S + 1) / 2 scores per head)
-        work["attn_core"] = steps * cfg.n_layers * B * cfg.n_heads * 4.0 * hd * S * (S + 1) / 2
+        if cfg.kv_decode_of:   # one query per sequence over S + 1 keys
+            work["attn_core"] = steps * cfg.n_layers * B * cfg.n_heads * 4.0 * hd * (S + 1)
+        else:   # q k^T and p v over the causal triangle (S (S + 1) / 2 scores per head)
+            work["attn_core"] = steps * cfg.n_layers * B * cfg.n_heads * 4.0 * hd * S * (S + 1) / 2
     return work
+
+
+def algorithmic_bytes(cfg, counts_per_step, steps):
+    """Algorithmic HBM bytes per kernel class over the timed steps: every weight a
+    class multiplies is read once per block that runs it (bf16), and decoding
+    attention reads the cached keys and values once.  Activations are left out
+    (a lower bound; they matter only where the tensor bound wins anyway)."""
+    d, I, r, L = cfg.d_model, cfg.d_ff, cfg.d_r, cfg.n_layers
+    nf = np.asarray(counts_per_step)
+    T = cfg.n_tokens
+    nY = cfg.d_enc + cfg.d_head
+    wb = 2.0
+    out = {
+        "ffn_gate_up": steps * wb * float(np.sum((nf > 0) * 2 * I * d + (nf < T) * r * d)),
+        "ffn_down": steps * wb * float(np.sum((nf > 0) * I * d)),
+        "router_gemm": steps * wb * (L - cfg.n_dense) * nY * 2 * d,
+        "adapter_up": steps * wb * float(np.sum((nf < T) * d * r)),
+    }
+    if cfg.n_heads:
+        hd = d // cfg.n_heads
+        nqkv = (cfg.n_heads + 2 * cfg.n_kv_heads) * hd
+        out["attn_proj"] = steps * wb * L * (nqkv + cfg.n_heads * hd) * d
+        if cfg.kv_decode_of:
+            out["attn_core"] = steps * wb * L * cfg.batch * cfg.n_kv_heads * (cfg.seq_len + 1) * hd * 2
+    return out
 
 
 def oracle_step(ho, cfg, w, h_np, tau, n_sample, P_np=None):
@@ -268,19 +304,42 @@ def main():
     default_shape = cfg == hi.CONFIGS[args.workload] and args.tau is None
     T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
     decoder = bool(cfg.n_heads)
-    if decoder and args.tokens:
+    kvdec = bool(cfg.kv_decode_of)
+    if decoder and not kvdec and args.tokens:
         cfg = cfg.replace(batch=max(1, cfg.n_tokens // cfg.seq_len))
     B, S = cfg.batch, cfg.seq_len
-    if decoder and B * S != T:
+    if kvdec and B != T:
+        raise SystemExit(f"KV decoding workload needs T = batch ({B} != {T})")
+    if decoder and not kvdec and B * S != T:
         raise SystemExit(f"decoder workload needs T = batch x seq_len ({B}x{S} != {T})")
     t_gen = time.time()
     w = hi.generate_weights(cfg)
     h_np = hi.generate_h_in(cfg)
     P_np = None if decoder else hi.generate_attn_delta(cfg)
     t_gen = time.time() - t_gen
-    stack = hero.HeroDecoder(cfg, w, hi.generate_attn_weights(cfg)) if decoder else hero.HeroStack(cfg, w)
     dev = torch.device("cuda", local_rank)
     stream = torch.cuda.current_stream(dev)
+    t_prefill = None
+    if kvdec:
+        # the cache: every sequence's S-token prefix, prefilled in chunks of the prefill
+        # workload's shape (untimed)
+        pcfg = hi.CONFIGS[cfg.kv_decode_of]
+        stack = hero.HeroDecoder(cfg, w, hi.generate_attn_weights(cfg), max_tokens=pcfg.n_tokens)
+        stack.init_cache(B, S + 1)
+        hp_dev = torch.from_numpy(hi.generate_h_in(pcfg)).to(dev)
+        t_prefill = time.time()
+        for seq0 in range(0, B, pcfg.batch):
+            nb = min(pcfg.batch, B - seq0)
+            stack.prefill(hp_dev[:nb * S], tau, seq0, nb, S)
+        torch.cuda.synchronize()
+        t_prefill = time.time() - t_prefill
+        stack.check()
+        del hp_dev
+        pos = torch.full((B,), S, dtype=torch.int32, device=dev)
+    elif decoder:
+        stack = hero.HeroDecoder(cfg, w, hi.generate_attn_weights(cfg))
+    else:
+        stack = hero.HeroStack(cfg, w)
     h = torch.from_numpy(h_np).to(dev)
     P = None if decoder else torch.from_numpy(P_np).to(dev)
     h_out = torch.empty((T, d), dtype=torch.float32, device=dev)
@@ -300,7 +359,10 @@ def main():
         return float(t.item())
 
     def run(flags, st=None):
-        if decoder:
+        if kvdec:
+            stack.decode(h, pos, S, tau, flags=flags, h_out=h_out, gate_out=g, mask_out=m,
+                         counts_out=c, stream=st or stream)
+        elif decoder:
             stack.forward(h, tau, B, S, flags=flags, h_out=h_out, gate_out=g, mask_out=m,
                           counts_out=c, stream=st or stream)
         else:
@@ -375,8 +437,14 @@ def main():
         ho_ = torch.empty((T, d), dtype=torch.float32).pin_memory()
         cp = torch.empty((L,), dtype=torch.int32).pin_memory()
 
+        pos_h = torch.full((B,), S, dtype=torch.int32).pin_memory() if kvdec else None
+
         def run_host():
-            if decoder:
+            if kvdec:
+                hero.hero_decode_step(stack.model, B, pos_h.data_ptr(), S, hp.data_ptr(), tau,
+                                      hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                      cp.data_ptr(), stream.cuda_stream)
+            elif decoder:
                 hero.hero_decoder_forward(stack.model, B, S, hp.data_ptr(), tau,
                                           hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
                                           cp.data_ptr(), stream.cuda_stream)
@@ -389,7 +457,8 @@ def main():
         ms_e2e, _ = timed(run_host, args.steps)
         stack.check()
         e2e = {"value": world * T * args.steps / (ms_e2e / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": int(hp.numel() * 4 + (0 if decoder else Pp.numel() * 2)),
+               "h2d_bytes_per_step": int(hp.numel() * 4 + (0 if decoder else Pp.numel() * 2)
+                                         + (B * 4 if kvdec else 0)),
                "d2h_bytes_per_step": int(ho_.numel() * 4 + cp.numel() * 4)}
         assert np.array_equal(cp.numpy(), counts), "host-IO path routed differently"
 
@@ -399,14 +468,25 @@ def main():
     dom = max(prof, key=lambda k: prof[k][0])
     dom_ms, dom_n = prof[dom]
     roof = None
+    nbytes = algorithmic_bytes(cfg, counts, args.steps)
     if dom in work and dom_ms > 0:
-        achieved = work[dom] / (dom_ms / 1e3) / 1e12
-        peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": DOMINANT_TRAFFIC.get((cfg.name, dom)) if default_shape else None,
-                "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)",
-                "avg_launch_ms": dom_ms / max(dom_n, 1)}
+        peak_tf = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        peak_bw = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+        # the bound is whichever floor is higher: FLOPs at the tensor peak or bytes at HBM
+        hbm = nbytes.get(dom, 0.0) / (peak_bw * 1e9) > work[dom] / (peak_tf * 1e12)
+        traffic = DOMINANT_TRAFFIC.get((cfg.name, dom)) if default_shape else None
+        if hbm:
+            achieved = nbytes[dom] / (dom_ms / 1e3) / 1e9
+            roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peak_bw,
+                    "unit": "GB/s", "frac": achieved / peak_bw, "traffic": traffic,
+                    "peak_source": f"{peak_src} hbm_gbs",
+                    "algorithmic": "weights read once per block (bf16) plus cached keys/values"}
+        else:
+            achieved = work[dom] / (dom_ms / 1e3) / 1e12
+            roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak_tf,
+                    "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": traffic,
+                    "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
+        roof["avg_launch_ms"] = dom_ms / max(dom_n, 1)
     ffn_ms = prof["ffn_gate_up"][0] + prof["ffn_down"][0]
     ffn_tflops = (work["ffn_gate_up"] + work["ffn_down"]) / (ffn_ms / 1e3) / 1e12 if ffn_ms else None
 
@@ -415,6 +495,9 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         from oracle import hero_oracle as ho
         step, rows, sample = oracle_step(ho, cfg, w, h_np, tau, args.cpu_sample, P_np)
+        if kvdec:
+            sample = ("the oracle has no incremental form (it recomputes a sequence's prefix); "
+                      + sample)
         t0 = time.perf_counter()
         step()
         dt = time.perf_counter() - t0
@@ -444,7 +527,7 @@ def main():
         "ffn_gemm_frac_of_sustained": (ffn_tflops / float(peaks.get("bf16_tflops_sustained", 1700.0)))
         if ffn_tflops else None,
         "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items()},
-        "setup_s": {"generate": t_gen},
+        "setup_s": {"generate": t_gen, **({"prefill_cache": t_prefill} if kvdec else {})},
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

@@ -260,6 +260,45 @@ hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len,
                                  float* h_out, float* gate_out, uint8_t* mask_out,
                                  int32_t* ffn_count_out, void* cuda_stream);
 
+/* ---- KV-cache decoding: the decoder's incremental form ------------------------
+ * Causal attention lets a sequence grow one token at a time: a new token's
+ * h_bar (Eq. 1) needs the rotated keys and values of every earlier position,
+ * which the model keeps in a cache, and its routing (Eqs. 2-16) runs on that
+ * token alone with a fresh router state, as every token's does.
+ *
+ * Allocate the cache for max_seqs sequence slots of max_len positions, all
+ * layers: 2 * n_layers * max_seqs * H_kv * max_len * 128 bf16, plus the
+ * split-KV partial results of the decode attention.  Needs hero_attn_init;
+ * once per model (HERO_ERR_ARG on a second call).  Synchronous. */
+hero_status hero_kv_cache_init(hero_model* m, int32_t max_seqs, int32_t max_len);
+
+/* hero_decoder_forward on n_seqs sequences of seq_len tokens that are cache slots
+ * seq0 .. seq0 + n_seqs - 1 (seq0 + n_seqs <= max_seqs, seq_len <= max_len);
+ * every layer's rotated keys and values of positions 0 .. seq_len - 1 are also
+ * stored in those slots.  Arguments and outputs as hero_decoder_forward. */
+hero_status hero_decoder_prefill(hero_model* m, int32_t seq0, int32_t n_seqs, int32_t seq_len,
+                                 const float* h_in, float tau_exec, uint32_t flags,
+                                 const uint8_t* mask_in, float* h_out, float* gate_out,
+                                 uint8_t* mask_out, int32_t* ffn_count_out, void* cuda_stream);
+
+/* One decoding step: a new token for each cache slot b < n_seqs (n_seqs <=
+ * max_seqs and <= max_tokens), at position positions[b] (int32 [n_seqs]); it
+ * attends to positions 0 .. positions[b] - 1 of its slot (which must hold that
+ * sequence's earlier keys and values) and to itself, and its key and value are
+ * stored at positions[b].  max_position (host) bounds every positions[b] and
+ * sizes the launch; a position outside [0, min(max_position, max_len - 1)]
+ * sets the device error word (the token's cache writes are skipped; reported
+ * by hero_check_device_status).  h_in [n_seqs,d] are the new tokens' inputs;
+ * tau_exec, flags (HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK with mask_in
+ * [L,n_seqs], HERO_FLAG_HOST_IO: h_in, positions, mask_in and the outputs are
+ * host pointers) and the outputs as hero_decoder_forward with T = n_seqs.
+ * Precision: as hero_attention_block, except that the softmax probabilities
+ * enter P V in fp32. */
+hero_status hero_decode_step(hero_model* m, int32_t n_seqs, const int32_t* positions,
+                             int32_t max_position, const float* h_in, float tau_exec,
+                             uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
+                             uint8_t* mask_out, int32_t* ffn_count_out, void* cuda_stream);
+
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes of one block, for per-kernel timing. */
 enum {

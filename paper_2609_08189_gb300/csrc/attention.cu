@@ -103,7 +103,8 @@ __device__ __forceinline__ void load_tile(uint32_t tile, const uint16_t* src, in
 __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __restrict__ Q,
                                                            const uint16_t* __restrict__ K,
                                                            const uint16_t* __restrict__ V, int H,
-                                                           int Hkv, int S, float scale_log2,
+                                                           int Hkv, int S, int kv_stride,
+                                                           float scale_log2,
                                                            uint16_t* __restrict__ O) {
   pdl_enter();
   extern __shared__ __align__(128) uint16_t fa_smem[];
@@ -116,8 +117,8 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
   const int kvh = hh / (H / Hkv);
   const int q0 = qt * FA_BM;
   const uint16_t* Qg = Q + ((size_t)b * H + hh) * S * HD;
-  const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * S * HD;
-  const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * S * HD;
+  const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * kv_stride * HD;
+  const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * kv_stride * HD;
   const int n_tiles = qt + 1;                          // causal: key tiles 0..qt
 
   load_tile(sQ, Qg, q0, S, tid);
@@ -253,6 +254,163 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
   }
 }
 
+// ---------------------------------------------------------------------------------
+// Decoding step attention (flash-decoding): one query per sequence, the G = H / H_kv
+// query heads of a key/value head together, keys split into chunks of DC positions
+// so that every SM streams the cache.  CTA = (chunk, kv head, sequence), 128 threads:
+//   1. scores: thread t takes keys t, t + 128 of the chunk, one 256-byte key row
+//      each (16 x 16-byte loads), against the G queries (fp32, from shared memory);
+//   2. per query head (one warp each): chunk max m, p = 2^(s - m), l = sum p;
+//   3. P V: thread t owns value columns 2 (t % 64), +1 for half of the keys
+//      (4-byte loads, 128 contiguous bytes per warp), halves added in shared memory.
+// Partial (m, l, o[128]) per (sequence, head, chunk) are merged by k_attn_combine.
+// ---------------------------------------------------------------------------------
+constexpr int DC = 256;          // keys per chunk
+constexpr int DEC_THREADS = 128;
+constexpr int DEC_GMAX = 8;      // query heads per key/value head
+
+template <int G>
+__global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __restrict__ Q,
+                                                             const uint16_t* __restrict__ K,
+                                                             const uint16_t* __restrict__ V,
+                                                             const int* __restrict__ pos, int H,
+                                                             int Hkv, int kv_stride, int max_pos,
+                                                             float scale_log2, float* __restrict__ pm,
+                                                             float* __restrict__ pl,
+                                                             float* __restrict__ po, int n_chunks,
+                                                             uint32_t* err) {
+  pdl_enter();
+  __shared__ float qs[G][HD];
+  __shared__ float sc[G][DC];
+  __shared__ float ored[G][HD];
+  const int c = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int len = pos[b] + 1;
+  if (len < 1 || len > kv_stride || len > max_pos + 1) {   // bad position: no keys, reported
+    if (c == 0 && kvh == 0 && threadIdx.x == 0) atomicOr(err, ERR_BAD_INDEX);
+    len = 0;
+  }
+  const int j0 = c * DC, j1 = min(j0 + DC, len);
+  const size_t part = ((size_t)b * H + (size_t)kvh * G) * n_chunks + c;   // + g * n_chunks
+  if (j0 >= j1) {   // chunk past the sequence (or a bad position): an empty partial
+    if (tid < G) {
+      pm[part + (size_t)tid * n_chunks] = -INFINITY;
+      pl[part + (size_t)tid * n_chunks] = 0.f;
+    }
+    return;
+  }
+  for (int i = tid; i < G * HD; i += DEC_THREADS) {
+    const int g = i / HD, e = i - g * HD;
+    const uint16_t u = Q[((size_t)b * H + kvh * G + g) * HD + e];
+    qs[g][e] = __uint_as_float((uint32_t)u << 16) * scale_log2;
+  }
+  __syncthreads();
+  const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * kv_stride * HD;
+  const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * kv_stride * HD;
+#pragma unroll 1
+  for (int j = j0 + tid; j < j0 + DC; j += DEC_THREADS) {
+    float acc[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) acc[g] = 0.f;
+    if (j < j1) {
+      const uint4* kr = reinterpret_cast<const uint4*>(Kg + (size_t)j * HD);
+      uint4 kv[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) kv[i] = __ldg(kr + i);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const uint32_t w[4] = {kv[i].x, kv[i].y, kv[i].z, kv[i].w};
+#pragma unroll
+        for (int h2 = 0; h2 < 4; ++h2) {
+          float k0, k1;
+          unpack_bf16x2(w[h2], k0, k1);
+          const int e = i * 8 + h2 * 2;
+#pragma unroll
+          for (int g = 0; g < G; ++g) acc[g] += qs[g][e] * k0 + qs[g][e + 1] * k1;
+        }
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) sc[g][j - j0] = j < j1 ? acc[g] : -INFINITY;
+  }
+  __syncthreads();
+  for (int g = warp; g < G; g += DEC_THREADS / 32) {
+    float mx = -INFINITY;
+    for (int i = lane; i < DC; i += 32) mx = fmaxf(mx, sc[g][i]);
+    mx = warp_max(mx);
+    float l = 0.f;
+    for (int i = lane; i < DC; i += 32) {
+      const float p = exp2f(sc[g][i] - mx);   // 0 past the sequence
+      sc[g][i] = p;
+      l += p;
+    }
+    l = warp_sum(l);
+    if (lane == 0) {
+      pm[part + (size_t)g * n_chunks] = mx;
+      pl[part + (size_t)g * n_chunks] = l;
+    }
+  }
+  __syncthreads();
+  const int col = 2 * (tid & 63), half = tid >> 6;
+  float o0[G], o1[G];
+#pragma unroll
+  for (int g = 0; g < G; ++g) o0[g] = o1[g] = 0.f;
+#pragma unroll 4
+  for (int j = j0 + half; j < j1; j += 2) {
+    float v0, v1;
+    unpack_bf16x2(__ldg(reinterpret_cast<const uint32_t*>(Vg + (size_t)j * HD + col)), v0, v1);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const float p = sc[g][j - j0];
+      o0[g] += p * v0;
+      o1[g] += p * v1;
+    }
+  }
+  if (half) {
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      ored[g][col] = o0[g];
+      ored[g][col + 1] = o1[g];
+    }
+  }
+  __syncthreads();
+  if (!half) {
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float* dst = po + (part + (size_t)g * n_chunks) * HD + col;
+      *reinterpret_cast<float2*>(dst) = make_float2(o0[g] + ored[g][col], o1[g] + ored[g][col + 1]);
+    }
+  }
+}
+
+// Merge of the chunk partials: one warp per (sequence, head), lane owns 4 columns;
+// o = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c, stored bf16 into O [B][H 128].
+__global__ void __launch_bounds__(256) k_attn_combine(const float* __restrict__ pm,
+                                                      const float* __restrict__ pl,
+                                                      const float* __restrict__ po, int BH,
+                                                      int n_chunks, uint16_t* __restrict__ O) {
+  pdl_enter();
+  const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (w >= BH) return;
+  const size_t base = (size_t)w * n_chunks;
+  float M = -INFINITY;
+  for (int c = 0; c < n_chunks; ++c) M = fmaxf(M, pm[base + c]);
+  float L = 0.f;
+  float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (M > -INFINITY) {
+    for (int c = 0; c < n_chunks; ++c) {
+      const float mc = pm[base + c];
+      if (mc == -INFINITY) continue;
+      const float f = exp2f(mc - M);
+      L += f * pl[base + c];
+      const float4 v = *reinterpret_cast<const float4*>(po + (base + c) * HD + 4 * lane);
+      o.x += f * v.x; o.y += f * v.y; o.z += f * v.z; o.w += f * v.w;
+    }
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  store4(O, (size_t)w * HD + 4 * lane, make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv), 1);
+}
+
 }  // namespace
 
 cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float eps, void* x,
@@ -264,9 +422,9 @@ cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float
 }
 
 cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
-                              int Hkv, void* O, cudaStream_t st) {
+                              int Hkv, int kv_stride, void* O, cudaStream_t st) {
   if (B <= 0 || S <= 0) return cudaSuccess;
-  if (H % Hkv || H > 65535 || B > 65535) return cudaErrorInvalidValue;   // grid y and z limits
+  if (H % Hkv || H > 65535 || B > 65535 || kv_stride < S) return cudaErrorInvalidValue;
   constexpr size_t smem = 2u * (FA_BM * HD + 2 * 2 * FA_BN * HD);   // 80 KB
   static bool attr = false;
   if (!attr) {
@@ -279,8 +437,40 @@ cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B
   dim3 grid((unsigned)((S + FA_BM - 1) / FA_BM), (unsigned)H, (unsigned)B);
   return launch_pdl(k_flash_attn, grid, dim3(FA_THREADS), smem, st,
                     static_cast<const uint16_t*>(Q), static_cast<const uint16_t*>(K),
-                    static_cast<const uint16_t*>(V), H, Hkv, S, scale_log2,
+                    static_cast<const uint16_t*>(V), H, Hkv, S, kv_stride, scale_log2,
                     static_cast<uint16_t*>(O));
+}
+
+}  // namespace hero
+
+namespace hero {
+
+int attn_decode_chunks(int max_pos) { return (max_pos + 1 + DC - 1) / DC; }
+
+cudaError_t launch_attn_decode(const void* Q, const void* K, const void* V, const int* pos, int B,
+                               int H, int Hkv, int kv_stride, int max_pos, float* pm, float* pl,
+                               float* po, void* O, uint32_t* err, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  if (H % Hkv || Hkv > 65535 || B > 65535 || max_pos < 0 || max_pos >= kv_stride)
+    return cudaErrorInvalidValue;
+  const int G = H / Hkv, nc = attn_decode_chunks(max_pos);
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
+  const dim3 grid((unsigned)nc, (unsigned)Hkv, (unsigned)B);
+  cudaError_t e;
+  const uint16_t *q = static_cast<const uint16_t*>(Q), *k = static_cast<const uint16_t*>(K),
+                 *v = static_cast<const uint16_t*>(V);
+  switch (G) {
+    case 1: e = launch_pdl(k_attn_decode<1>, grid, dim3(DEC_THREADS), 0, st, q, k, v, pos, H, Hkv, kv_stride, max_pos, scale_log2, pm, pl, po, nc, err); break;
+    case 2: e = launch_pdl(k_attn_decode<2>, grid, dim3(DEC_THREADS), 0, st, q, k, v, pos, H, Hkv, kv_stride, max_pos, scale_log2, pm, pl, po, nc, err); break;
+    case 4: e = launch_pdl(k_attn_decode<4>, grid, dim3(DEC_THREADS), 0, st, q, k, v, pos, H, Hkv, kv_stride, max_pos, scale_log2, pm, pl, po, nc, err); break;
+    case 8: e = launch_pdl(k_attn_decode<8>, grid, dim3(DEC_THREADS), 0, st, q, k, v, pos, H, Hkv, kv_stride, max_pos, scale_log2, pm, pl, po, nc, err); break;
+    default: return cudaErrorInvalidValue;
+  }
+  if (e != cudaSuccess) return e;
+  const int BH = B * H;
+  return launch_pdl(k_attn_combine, dim3((unsigned)((BH + 7) / 8)), dim3(256), 0, st,
+                    static_cast<const float*>(pm), static_cast<const float*>(pl),
+                    static_cast<const float*>(po), BH, nc, static_cast<uint16_t*>(O));
 }
 
 }  // namespace hero

@@ -168,8 +168,21 @@ __device__ __forceinline__ void epi_qkv_rope(const GemmArgs& a, uint32_t tbase, 
   static_assert(BN % 128 == 0, "whole heads per tile");
   const RopeArgs& r = a.rope;
   const int heads = r.H + 2 * r.Hkv;
-  const int bq = valid ? m / r.S : 0;
-  const int s = valid ? m - bq * r.S : 0;
+  int bq = 0, s = 0, sq = 0;
+  if (valid) {
+    if (r.pos) {   // decoding step: row = sequence, its position from memory
+      bq = m;
+      s = r.pos[m];
+      if (s < 0 || s >= r.S_kv) {   // outside the cache: report, store nothing
+        if (nb == 0) atomicOr(a.err, ERR_BAD_INDEX);
+        valid = false;
+      }
+    } else {
+      bq = m / r.S;
+      s = m - bq * r.S;
+      sq = s;
+    }
+  }
 #pragma unroll 1
   for (int hb = 0; hb < BN; hb += 128) {
     const int head = (nb * BN + hb) >> 7;
@@ -183,12 +196,12 @@ __device__ __forceinline__ void epi_qkv_rope(const GemmArgs& a, uint32_t tbase, 
       uint16_t* dst;
       const bool rot = head < r.H + r.Hkv;
       if (head < r.H)
-        dst = static_cast<uint16_t*>(r.q) + (((size_t)bq * r.H + head) * r.S + s) * 128;
+        dst = static_cast<uint16_t*>(r.q) + (((size_t)bq * r.H + head) * r.S_q + sq) * 128;
       else if (rot)
-        dst = static_cast<uint16_t*>(r.k) + (((size_t)bq * r.Hkv + head - r.H) * r.S + s) * 128;
+        dst = static_cast<uint16_t*>(r.k) + (((size_t)bq * r.Hkv + head - r.H) * r.S_kv + s) * 128;
       else
         dst = static_cast<uint16_t*>(r.v) +
-              (((size_t)bq * r.Hkv + head - r.H - r.Hkv) * r.S + s) * 128;
+              (((size_t)bq * r.Hkv + head - r.H - r.Hkv) * r.S_kv + s) * 128;
       uint32_t p1[16], p2[16];
       const float4* cs = reinterpret_cast<const float4*>(r.cs + ((size_t)s * 64 + c0) * 2);
 #pragma unroll
@@ -675,7 +688,8 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
     case EPI_RESIDUAL:
       return launch_tc<256, EPI_RESIDUAL, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_QKV_ROPE:
-      if (args.N != (args.rope.H + 2 * args.rope.Hkv) * 128 || args.rope.S <= 0)
+      if (args.N != (args.rope.H + 2 * args.rope.Hkv) * 128 || args.rope.S <= 0 ||
+          args.rope.S_q <= 0 || args.rope.S_kv <= 0 || (!args.rope.pos && args.rope.S_kv < args.rope.S))
         return cudaErrorInvalidValue;
       return launch_tc<256, EPI_QKV_ROPE, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_ATTN_ENTRY:

@@ -144,7 +144,17 @@ struct hero_model {
   float* attn_gain = nullptr;  // [L][d]
   void* aws = nullptr;         // attention workspace
   void *ax = nullptr, *aq = nullptr, *ak = nullptr, *av = nullptr, *ao = nullptr;
-  float *rope_cs = nullptr, *hcur = nullptr, *dlprev = nullptr;
+  float *hcur = nullptr, *dlprev = nullptr;
+  float* rope_cs = nullptr;    // [rope_rows][64][2] RoPE cos, sin (own allocation)
+  long rope_rows = 0;
+  // KV cache (hero_kv_cache_init): per layer [max_seqs][H_kv][max_len][128] bf16, K then V
+  void* kv = nullptr;
+  int kv_seqs = 0, kv_len = 0;
+  float *dec_pm = nullptr, *dec_pl = nullptr, *dec_po = nullptr;   // decode attention partials
+  int* dec_pos = nullptr;      // positions staged for HERO_FLAG_HOST_IO
+  size_t kv_layer_elems() const { return (size_t)kv_seqs * n_kv_heads * kv_len * 128; }
+  uint16_t* kv_k(int jj) { return static_cast<uint16_t*>(kv) + (size_t)jj * 2 * kv_layer_elems(); }
+  uint16_t* kv_v(int jj) { return kv_k(jj) + kv_layer_elems(); }
   CUtensorMap tm_ax, tm_ao;
   std::vector<CUtensorMap> tm_wqkv, tm_wo;
 
@@ -296,7 +306,8 @@ void free_model(hero_model* m) {
   if (m->ev_kernels_done) cudaEventDestroy(m->ev_kernels_done);
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
-                  m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws};
+                  m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
+                  m->dec_pm, m->dec_pos};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -1053,11 +1064,39 @@ hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, c
                     gate_out, mask_out, count_out, st);
 }
 
+// RoPE (cos, sin) of s * theta^(-2i/128) for positions s < rows, computed in double.
+hero_status build_rope_table(hero_model* m, long rows) {
+  if (rows <= m->rope_rows) return HERO_OK;
+  std::vector<float> cs((size_t)rows * 64 * 2);
+  for (long p = 0; p < rows; ++p)
+    for (int i = 0; i < 64; ++i) {
+      const double ang = (double)p * std::pow((double)m->rope_theta, -2.0 * i / 128.0);
+      cs[((size_t)p * 64 + i) * 2] = (float)std::cos(ang);
+      cs[((size_t)p * 64 + i) * 2 + 1] = (float)std::sin(ang);
+    }
+  CUDA_TRY(cudaDeviceSynchronize());   // the old table may be in use
+  if (m->rope_cs) cudaFree(m->rope_cs);
+  m->rope_cs = nullptr;
+  m->rope_rows = 0;
+  CUDA_TRY(cudaMalloc(&m->rope_cs, cs.size() * 4));
+  CUDA_TRY(cudaMemcpy(m->rope_cs, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice));
+  m->rope_rows = rows;
+  return HERO_OK;
+}
+
+// Where a sublayer's keys and values go: the workspace (nullptr) or a cache range.
+struct KvTarget {
+  void* k;
+  void* v;
+  int stride;   // positions per (sequence, head) slab
+};
+
 // Eq. 1, first line, for layer jj on B sequences of S tokens: h_bar = h + Attn(LN_attn(h)).
 // With `entry`, the output projection also closes into the routed block's entry
 // (h_bar written over entry->hbar = h_bar_{j-1}, delta, router operand, partials).
 hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, float* h_bar,
-                          cudaStream_t st, const LayerOutArgs* entry = nullptr) {
+                          cudaStream_t st, const LayerOutArgs* entry = nullptr,
+                          const KvTarget* kv = nullptr) {
   const hero_config& c = m->cfg;
   const int T = B * S, d = c.d_model, H = m->n_heads, Hkv = m->n_kv_heads;
   const int nqkv = (H + 2 * Hkv) * 128;
@@ -1071,12 +1110,13 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   g.K = d;
   g.ldo = nqkv;
   g.err = m->err;
-  g.rope = RopeArgs{m->aq, m->ak, m->av, m->rope_cs, H, Hkv, S};
+  const KvTarget kt = kv ? *kv : KvTarget{m->ak, m->av, S};
+  g.rope = RopeArgs{m->aq, kt.k, kt.v, m->rope_cs, nullptr, H, Hkv, S, S, kt.stride};
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q, k, v with RoPE, attention layout
     return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
   }));
   CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
-    return launch_flash_attn(m->aq, m->ak, m->av, B, S, H, Hkv, m->ao, st);
+    return launch_flash_attn(m->aq, kt.k, kt.v, B, S, H, Hkv, kt.stride, m->ao, st);
   }));
   GemmArgs o{};
   o.m_static = T;
@@ -1194,7 +1234,7 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   };
   std::vector<Item> items = {
       {&m->ax, (size_t)Tm * d * 2},          {&m->ao, (size_t)Tm * d * 2},
-      {(void**)&m->rope_cs, (size_t)Tm * 64 * 2 * 4}, {&m->aq, (size_t)Tm * H * 128 * 2},
+      {&m->aq, (size_t)Tm * H * 128 * 2},
       {&m->ak, (size_t)Tm * Hkv * 128 * 2},  {&m->av, (size_t)Tm * Hkv * 128 * 2},
       {(void**)&m->hcur, (size_t)Tm * d * 4},
       {(void**)&m->dlprev, (size_t)Tm * d * 4}};
@@ -1206,16 +1246,8 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
     *it.p = static_cast<char*>(m->aws) + off;
     off += (it.bytes + 1023) & ~(size_t)1023;
   }
-  {   // RoPE (cos, sin) of s * theta^(-2i/128) for positions s < max_tokens, in double
-    std::vector<float> cs((size_t)Tm * 64 * 2);
-    for (long p = 0; p < Tm; ++p)
-      for (int i = 0; i < 64; ++i) {
-        const double ang = (double)p * std::pow((double)ac->rope_theta, -2.0 * i / 128.0);
-        cs[((size_t)p * 64 + i) * 2] = (float)std::cos(ang);
-        cs[((size_t)p * 64 + i) * 2 + 1] = (float)std::sin(ang);
-      }
-    CUDA_TRY(cudaMemcpy(m->rope_cs, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice));
-  }
+  m->rope_theta = ac->rope_theta;
+  if (hero_status rs = build_rope_table(m, Tm); rs != HERO_OK) return rs;
   bool ok = encode_bf16_2d(&m->tm_ax, m->ax, d, Tm, 128) && encode_bf16_2d(&m->tm_ao, m->ao, d, Tm, 128);
   m->tm_wqkv.resize(L);
   m->tm_wo.resize(L);
@@ -1226,7 +1258,6 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   if (!ok) return fail(HERO_ERR_CUDA, "tensor map encoding failed");
   m->n_heads = (int)H;
   m->n_kv_heads = (int)Hkv;
-  m->rope_theta = ac->rope_theta;
   m->attn = true;
   return HERO_OK;
 }
@@ -1256,11 +1287,68 @@ extern "C" hero_status hero_attention_block(hero_model* m, int32_t layer, int32_
 
 namespace {
 
+// The block entry that the output projection closes into (Eq. 7 bookkeeping).
+LayerOutArgs entry_args(hero_model* m, int jj, uint32_t flags) {
+  const int jr = jj - m->cfg.n_dense;
+  LayerOutArgs entry{};
+  entry.hbar = m->hbar;
+  entry.delta = m->dlprev;
+  entry.xl = m->xl;
+  entry.part = m->part;
+  entry.d = m->cfg.d_model;
+  entry.np = m->np;
+  entry.first = jr <= 0;
+  entry.xl_bf16 = 1;
+  entry.router = ((flags & HERO_FLAG_DENSE) || jr < 0) ? 0 : 1;
+  return entry;
+}
+
+// Eq. 1 for one new token per cache slot b < B at position pos[b] (decoding step).
+hero_status attention_decode_run(hero_model* m, int jj, int B, const int* pos, int max_pos,
+                                 const float* h, cudaStream_t st, const LayerOutArgs& entry) {
+  const hero_config& c = m->cfg;
+  const int d = c.d_model, H = m->n_heads, Hkv = m->n_kv_heads;
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_attn_norm(h, m->attn_gain + (size_t)jj * d, B, d, c.rms_eps, m->ax, st);
+  }));
+  GemmArgs g{};
+  g.m_static = B;
+  g.m_max = B;
+  g.N = (H + 2 * Hkv) * 128;
+  g.K = d;
+  g.ldo = g.N;
+  g.err = m->err;
+  g.rope = RopeArgs{m->aq, m->kv_k(jj), m->kv_v(jj), m->rope_cs, pos, H, Hkv, 1, 1, m->kv_len};
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q; k and v into the cache
+    return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
+  }));
+  CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
+    return launch_attn_decode(m->aq, m->kv_k(jj), m->kv_v(jj), pos, B, H, Hkv, m->kv_len, max_pos,
+                              m->dec_pm, m->dec_pl, m->dec_po, m->ao, m->err, st);
+  }));
+  GemmArgs o{};
+  o.m_static = B;
+  o.m_max = B;
+  o.N = d;
+  o.K = H * 128;
+  o.ldo = d;
+  o.resid = h;
+  o.err = m->err;
+  o.lo = entry;
+  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+    return launch_gemm_tc(256, EPI_ATTN_ENTRY, m->tm_ao, m->tm_wo[jj], o, m->num_sms, st);
+  }));
+  return HERO_OK;
+}
+
 // The decoder forward on device buffers (h_in may be m->hcur: layer 1 reads it into
-// h_bar before anything writes hcur).
+// h_bar before anything writes hcur).  seq0 >= 0: the sequences are cache slots
+// seq0.. and every layer's keys and values go there.  pos != nullptr: a decoding
+// step (one token per cache slot, n_seqs tokens at positions pos, seq_len 1).
 hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_in, float tau_exec,
                         uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
-                        uint8_t* mask_out, int32_t* ffn_count_out, cudaStream_t st) {
+                        uint8_t* mask_out, int32_t* ffn_count_out, cudaStream_t st, int seq0 = -1,
+                        const int* pos = nullptr, int max_pos = 0) {
   const hero_config& c = m->cfg;
   const int L = c.n_layers, T = n_seqs * seq_len;
   if (!(flags & HERO_FLAG_DENSE))
@@ -1270,19 +1358,17 @@ hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_i
   for (int jj = 0; jj < L; ++jj) {
     // Eq. 1 with the block entry fused into the output projection: m->hbar carries
     // h_bar_{j-1} into the launch and h_bar_j out of it, m->dlprev likewise delta
-    const int jr = jj - c.n_dense;
-    const bool dense = (flags & HERO_FLAG_DENSE) || jr < 0;
-    LayerOutArgs entry{};
-    entry.hbar = m->hbar;
-    entry.delta = m->dlprev;
-    entry.xl = m->xl;
-    entry.part = m->part;
-    entry.d = c.d_model;
-    entry.np = m->np;
-    entry.first = jr <= 0;
-    entry.xl_bf16 = 1;
-    entry.router = dense ? 0 : 1;
-    hero_status s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st, &entry);
+    const LayerOutArgs entry = entry_args(m, jj, flags);
+    hero_status s;
+    if (pos) {
+      s = attention_decode_run(m, jj, n_seqs, pos, max_pos, h, st, entry);
+    } else if (seq0 >= 0) {
+      const size_t off = (size_t)seq0 * m->n_kv_heads * m->kv_len * 128;
+      const KvTarget kt{m->kv_k(jj) + off, m->kv_v(jj) + off, m->kv_len};
+      s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st, &entry, &kt);
+    } else {
+      s = attention_run(m, jj, n_seqs, seq_len, h, m->hbar, st, &entry);
+    }
     if (s != HERO_OK) return s;
     float* out = jj == L - 1 ? h_out : m->hcur;
     s = routed_block_run(m, jj, T, m->hbar, bs, nullptr, m->dlprev, tau_exec, flags,
@@ -1297,36 +1383,25 @@ hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_i
   return HERO_OK;
 }
 
-}  // namespace
-
-extern "C" hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len,
-                                            const float* h_in, float tau_exec, uint32_t flags,
-                                            const uint8_t* mask_in, float* h_out, float* gate_out,
-                                            uint8_t* mask_out, int32_t* ffn_count_out,
-                                            void* cuda_stream) {
-  g_last_error.clear();
-  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
-  if (!m->attn) return fail(HERO_ERR_ARG, "hero_attn_init has not been called");
-  const hero_config& c = m->cfg;
-  const int L = c.n_layers, d = c.d_model;
-  if (n_seqs < 0 || n_seqs > 65535 || seq_len < 1 || (long)n_seqs * seq_len > c.max_tokens)
-    return fail(HERO_ERR_ARG, "n_seqs x seq_len outside [0, max_tokens=%d] (n_seqs <= 65535)",
-                c.max_tokens);
+// Argument checks shared by the decoder entry points (T tokens).  T == 0 is
+// handled here: ffn_count_out is zeroed and nothing else happens.
+hero_status check_decoder_args(hero_model* m, int T, const float* h_in, float tau_exec,
+                               uint32_t flags, const uint8_t* mask_in, const float* h_out,
+                               int32_t* ffn_count_out, void* cuda_stream) {
+  const int L = m->cfg.n_layers;
   if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO))
     return fail(HERO_ERR_ARG, "unknown flag bits 0x%x", flags);
   if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
     return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
   if (!std::isfinite(tau_exec)) return fail(HERO_ERR_ARG, "tau_exec is not finite");
-  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  const int T = n_seqs * seq_len;
-  const bool host = flags & HERO_FLAG_HOST_IO;
   CUDA_TRY(cudaSetDevice(m->device));
   if (T == 0) {
     if (ffn_count_out) {
-      if (host)
+      if (flags & HERO_FLAG_HOST_IO)
         memset(ffn_count_out, 0, (size_t)L * 4);
       else
-        CUDA_TRY(cudaMemsetAsync(ffn_count_out, 0, (size_t)L * 4, st));
+        CUDA_TRY(cudaMemsetAsync(ffn_count_out, 0, (size_t)L * 4,
+                                 static_cast<cudaStream_t>(cuda_stream)));
     }
     return HERO_OK;
   }
@@ -1334,13 +1409,22 @@ extern "C" hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32
   if ((const void*)h_in == (const void*)h_out) return fail(HERO_ERR_ARG, "h_out must not alias h_in");
   if ((flags & HERO_FLAG_FORCE_MASK) && !mask_in)
     return fail(HERO_ERR_ARG, "HERO_FLAG_FORCE_MASK needs mask_in");
+  return HERO_OK;
+}
+
+// Run decoder_run on device buffers, staging host buffers first with HERO_FLAG_HOST_IO
+// (h_0 straight into the decoder's running-h buffer, the decoding step's positions
+// into the model's position buffer, outputs through the I/O area).
+hero_status decoder_io(hero_model* m, int n_seqs, int seq_len, int seq0, const int* pos, int max_pos,
+                       const float* h_in, float tau_exec, uint32_t flags, const uint8_t* mask_in,
+                       float* h_out, float* gate_out, uint8_t* mask_out, int32_t* ffn_count_out,
+                       cudaStream_t st) {
+  const int L = m->cfg.n_layers, d = m->cfg.d_model, T = n_seqs * seq_len;
+  const bool host = flags & HERO_FLAG_HOST_IO;
   flags &= ~(uint32_t)HERO_FLAG_HOST_IO;
   if (!host)
     return decoder_run(m, n_seqs, seq_len, h_in, tau_exec, flags, mask_in, h_out, gate_out,
-                       mask_out, ffn_count_out, st);
-
-  // Host I/O: h_0 straight into the decoder's running-h buffer, outputs staged in the
-  // I/O area and copied back on the stream.
+                       mask_out, ffn_count_out, st, seq0, pos, max_pos);
   const size_t lt = (size_t)L * T;
   const size_t need = (size_t)T * d * 4 + lt /*mask_in*/ + lt * 4 + lt + (size_t)L * 4 + 4096;
   hero_status s = ensure_io(m, need);
@@ -1358,14 +1442,110 @@ extern "C" hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32
   int32_t* d_cnt = ffn_count_out ? reinterpret_cast<int32_t*>(carve((size_t)L * 4)) : nullptr;
   CUDA_TRY(cudaMemcpyAsync(m->hcur, h_in, (size_t)T * d * 4, cudaMemcpyHostToDevice, st));
   if (d_mask_in) CUDA_TRY(cudaMemcpyAsync(d_mask_in, mask_in, lt, cudaMemcpyHostToDevice, st));
+  if (pos) {
+    CUDA_TRY(cudaMemcpyAsync(m->dec_pos, pos, (size_t)n_seqs * 4, cudaMemcpyHostToDevice, st));
+    pos = m->dec_pos;
+  }
   s = decoder_run(m, n_seqs, seq_len, m->hcur, tau_exec, flags, d_mask_in, d_hout, d_gate, d_mask,
-                  d_cnt, st);
+                  d_cnt, st, seq0, pos, max_pos);
   if (s != HERO_OK) return s;
   CUDA_TRY(cudaMemcpyAsync(h_out, d_hout, (size_t)T * d * 4, cudaMemcpyDeviceToHost, st));
   if (d_gate) CUDA_TRY(cudaMemcpyAsync(gate_out, d_gate, lt * 4, cudaMemcpyDeviceToHost, st));
   if (d_mask) CUDA_TRY(cudaMemcpyAsync(mask_out, d_mask, lt, cudaMemcpyDeviceToHost, st));
   if (d_cnt) CUDA_TRY(cudaMemcpyAsync(ffn_count_out, d_cnt, (size_t)L * 4, cudaMemcpyDeviceToHost, st));
   return HERO_OK;
+}
+
+}  // namespace
+
+extern "C" hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len,
+                                            const float* h_in, float tau_exec, uint32_t flags,
+                                            const uint8_t* mask_in, float* h_out, float* gate_out,
+                                            uint8_t* mask_out, int32_t* ffn_count_out,
+                                            void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->attn) return fail(HERO_ERR_ARG, "hero_attn_init has not been called");
+  const hero_config& c = m->cfg;
+  if (n_seqs < 0 || n_seqs > 65535 || seq_len < 1 || (long)n_seqs * seq_len > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_seqs x seq_len outside [0, max_tokens=%d] (n_seqs <= 65535)",
+                c.max_tokens);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  hero_status s = check_decoder_args(m, n_seqs * seq_len, h_in, tau_exec, flags, mask_in, h_out,
+                                     ffn_count_out, cuda_stream);
+  if (s != HERO_OK || n_seqs == 0) return s;
+  return decoder_io(m, n_seqs, seq_len, -1, nullptr, 0, h_in, tau_exec, flags, mask_in, h_out,
+                    gate_out, mask_out, ffn_count_out, st);
+}
+
+extern "C" hero_status hero_kv_cache_init(hero_model* m, int32_t max_seqs, int32_t max_len) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->attn) return fail(HERO_ERR_ARG, "hero_attn_init has not been called");
+  if (m->kv) return fail(HERO_ERR_ARG, "the model already has a KV cache");
+  if (max_seqs < 1 || max_seqs > 65535 || max_len < 1)
+    return fail(HERO_ERR_ARG, "need 1 <= max_seqs <= 65535 and max_len >= 1");
+  CUDA_TRY(cudaSetDevice(m->device));
+  const hero_config& c = m->cfg;
+  const size_t layer = (size_t)max_seqs * m->n_kv_heads * max_len * 128;
+  const size_t bytes = (size_t)c.n_layers * 2 * layer * 2;
+  cudaError_t e = cudaMalloc(&m->kv, bytes);
+  if (e != cudaSuccess) {
+    m->kv = nullptr;
+    return fail(HERO_ERR_NOMEM, "KV cache of %zu bytes: %s", bytes, cudaGetErrorString(e));
+  }
+  CUDA_TRY(cudaMemset(m->kv, 0, bytes));   // never-written positions read as zeros, not NaN
+  const size_t pr = (size_t)max_seqs * m->n_heads * attn_decode_chunks(max_len - 1);
+  CUDA_TRY(cudaMalloc(&m->dec_pm, pr * (2 + 128) * 4));
+  m->dec_pl = m->dec_pm + pr;
+  m->dec_po = m->dec_pl + pr;
+  CUDA_TRY(cudaMalloc(&m->dec_pos, (size_t)max_seqs * 4));
+  if (hero_status rs = build_rope_table(m, max_len); rs != HERO_OK) return rs;
+  m->kv_seqs = max_seqs;
+  m->kv_len = max_len;
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_decoder_prefill(hero_model* m, int32_t seq0, int32_t n_seqs,
+                                            int32_t seq_len, const float* h_in, float tau_exec,
+                                            uint32_t flags, const uint8_t* mask_in, float* h_out,
+                                            float* gate_out, uint8_t* mask_out,
+                                            int32_t* ffn_count_out, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->kv) return fail(HERO_ERR_ARG, "hero_kv_cache_init has not been called");
+  const hero_config& c = m->cfg;
+  if (seq0 < 0 || n_seqs < 0 || (long)seq0 + n_seqs > m->kv_seqs)
+    return fail(HERO_ERR_ARG, "cache slots [%d, %d) outside [0, %d)", seq0, seq0 + n_seqs, m->kv_seqs);
+  if (seq_len < 1 || seq_len > m->kv_len || (long)n_seqs * seq_len > c.max_tokens)
+    return fail(HERO_ERR_ARG, "seq_len %d outside [1, max_len=%d] or n_seqs x seq_len > max_tokens",
+                seq_len, m->kv_len);
+  hero_status s = check_decoder_args(m, n_seqs * seq_len, h_in, tau_exec, flags, mask_in, h_out,
+                                     ffn_count_out, cuda_stream);
+  if (s != HERO_OK || n_seqs == 0) return s;
+  return decoder_io(m, n_seqs, seq_len, seq0, nullptr, 0, h_in, tau_exec, flags, mask_in, h_out,
+                    gate_out, mask_out, ffn_count_out, static_cast<cudaStream_t>(cuda_stream));
+}
+
+extern "C" hero_status hero_decode_step(hero_model* m, int32_t n_seqs, const int32_t* positions,
+                                        int32_t max_position, const float* h_in, float tau_exec,
+                                        uint32_t flags, const uint8_t* mask_in, float* h_out,
+                                        float* gate_out, uint8_t* mask_out, int32_t* ffn_count_out,
+                                        void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->kv) return fail(HERO_ERR_ARG, "hero_kv_cache_init has not been called");
+  const hero_config& c = m->cfg;
+  if (n_seqs < 0 || n_seqs > m->kv_seqs || n_seqs > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_seqs %d outside [0, min(max_seqs, max_tokens)]", n_seqs);
+  if (max_position < 0 || max_position >= m->kv_len)
+    return fail(HERO_ERR_ARG, "max_position %d outside [0, max_len=%d)", max_position, m->kv_len);
+  if (n_seqs > 0 && !positions) return fail(HERO_ERR_ARG, "positions is required");
+  hero_status s = check_decoder_args(m, n_seqs, h_in, tau_exec, flags, mask_in, h_out,
+                                     ffn_count_out, cuda_stream);
+  if (s != HERO_OK || n_seqs == 0) return s;
+  return decoder_io(m, n_seqs, 1, -1, positions, max_position, h_in, tau_exec, flags, mask_in,
+                    h_out, gate_out, mask_out, ffn_count_out, static_cast<cudaStream_t>(cuda_stream));
 }
 
 extern "C" hero_status hero_check_device_status(hero_model* m, void* cuda_stream) {

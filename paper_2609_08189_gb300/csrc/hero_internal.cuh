@@ -89,15 +89,17 @@ enum EpiKind : int {
                        // the attention layout (RopeArgs)
 };
 
-// EPI_QKV_ROPE: columns are heads of 128 (q heads | k heads | v heads); row t is
-// position t % S of sequence t / S.  Pair (i, i + 64) of a q or k head at position s
-// turns by the angle s * theta^(-2i/128), whose (cos, sin) come from cs.
+// EPI_QKV_ROPE: columns are heads of 128 (q heads | k heads | v heads).  Row t is
+// position t % S of sequence t / S, or (pos != nullptr, a decoding step) position
+// pos[t] of sequence t.  Pair (i, i + 64) of a q or k head at position s turns by
+// the angle s * theta^(-2i/128), whose (cos, sin) come from cs.
 struct RopeArgs {
-  void* q;             // bf16 [B][H][S][128]
-  void* k;             // bf16 [B][H_kv][S][128]
-  void* v;             // bf16 [B][H_kv][S][128]
-  const float* cs;     // [positions >= S][64][2]: cos, sin
-  int H, Hkv, S;
+  void* q;             // bf16 [B][H][S_q][128]; a decoding step stores at index 0 (S_q = 1)
+  void* k;             // bf16 [B][H_kv][S_kv][128] at the token's position
+  void* v;             // bf16 [B][H_kv][S_kv][128]
+  const float* cs;     // [positions >= S_kv][64][2]: cos, sin
+  const int* pos;      // [B] positions of a decoding step, or nullptr
+  int H, Hkv, S, S_q, S_kv;
 };
 
 struct GemmArgs {
@@ -152,8 +154,16 @@ constexpr int kTcPartCols = 128;
 // Attention sublayer kernels (attention.cu), head dimension 128 --------------------
 cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float eps, void* x,
                              cudaStream_t st);
+// K and V hold kv_stride positions per (sequence, head) slab (>= S; the cache's max_len).
 cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
-                              int Hkv, void* O, cudaStream_t st);
+                              int Hkv, int kv_stride, void* O, cudaStream_t st);
+// Decoding step: Q [B][H][128], K/V slabs of kv_stride positions, pos [B] (each <=
+// max_pos < kv_stride); partials pm, pl [B][H][chunks], po [B][H][chunks][128] with
+// chunks = attn_decode_chunks(max_pos); O [B][H 128] bf16.
+int attn_decode_chunks(int max_pos);
+cudaError_t launch_attn_decode(const void* Q, const void* K, const void* V, const int* pos, int B,
+                               int H, int Hkv, int kv_stride, int max_pos, float* pm, float* pl,
+                               float* po, void* O, uint32_t* err, cudaStream_t st);
 
 // Router and bookkeeping kernels ------------------------------------------------
 

@@ -111,6 +111,12 @@ def load(path: Optional[str] = None) -> ctypes.CDLL:
     lib.hero_attention_block.restype = ctypes.c_int
     lib.hero_decoder_forward.argtypes = [vp, i32, i32, vp, f32, u32, vp, vp, vp, vp, vp, vp]
     lib.hero_decoder_forward.restype = ctypes.c_int
+    lib.hero_kv_cache_init.argtypes = [vp, i32, i32]
+    lib.hero_kv_cache_init.restype = ctypes.c_int
+    lib.hero_decoder_prefill.argtypes = [vp, i32, i32, i32, vp, f32, u32, vp, vp, vp, vp, vp, vp]
+    lib.hero_decoder_prefill.restype = ctypes.c_int
+    lib.hero_decode_step.argtypes = [vp, i32, vp, i32, vp, f32, u32, vp, vp, vp, vp, vp, vp]
+    lib.hero_decode_step.restype = ctypes.c_int
     lib.hero_gemm_bf16_splitk_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     lib.hero_gemm_bf16_splitk_noalloc.restype = ctypes.c_int
     _lib = lib
@@ -248,6 +254,30 @@ def hero_decoder_forward(model: int, n_seqs: int, seq_len: int, h_in: int, tau_e
                                        mask_out or None, ffn_count_out or None, cuda_stream or None))
 
 
+def hero_kv_cache_init(model: int, max_seqs: int, max_len: int) -> None:
+    """Allocate the model's KV cache (max_seqs slots of max_len positions, all layers)."""
+    _check(load().hero_kv_cache_init(model, max_seqs, max_len))
+
+
+def hero_decoder_prefill(model: int, seq0: int, n_seqs: int, seq_len: int, h_in: int,
+                         tau_exec: float, flags: int, mask_in: int, h_out: int, gate_out: int,
+                         mask_out: int, ffn_count_out: int, cuda_stream: int) -> None:
+    """The decoder forward on cache slots seq0.., storing their keys and values."""
+    _check(load().hero_decoder_prefill(model, seq0, n_seqs, seq_len, h_in or None, float(tau_exec),
+                                       flags, mask_in or None, h_out or None, gate_out or None,
+                                       mask_out or None, ffn_count_out or None, cuda_stream or None))
+
+
+def hero_decode_step(model: int, n_seqs: int, positions: int, max_position: int, h_in: int,
+                     tau_exec: float, flags: int, mask_in: int, h_out: int, gate_out: int,
+                     mask_out: int, ffn_count_out: int, cuda_stream: int) -> None:
+    """One decoding step: a token per cache slot b < n_seqs at positions[b]."""
+    _check(load().hero_decode_step(model, n_seqs, positions or None, max_position, h_in or None,
+                                   float(tau_exec), flags, mask_in or None, h_out or None,
+                                   gate_out or None, mask_out or None, ffn_count_out or None,
+                                   cuda_stream or None))
+
+
 # ---------------------------------------------------------------------------
 # PyTorch convenience layer (device tensors, current stream)
 # ---------------------------------------------------------------------------
@@ -322,6 +352,43 @@ class HeroDecoder(HeroStack):
         hero_attention_block(self.model, layer, n_seqs, seq_len, h.data_ptr(), h_bar.data_ptr(),
                              st.cuda_stream)
         return h_bar
+
+    def init_cache(self, max_seqs: int, max_len: int) -> None:
+        hero_kv_cache_init(self.model, max_seqs, max_len)
+
+    def _outs(self, T, dev, h_out, gate_out, mask_out, counts_out):
+        import torch
+        L, d = self.cfg.n_layers, self.cfg.d_model
+        return (h_out if h_out is not None else torch.empty((T, d), dtype=torch.float32, device=dev),
+                gate_out if gate_out is not None else torch.empty((L, T), dtype=torch.float32, device=dev),
+                mask_out if mask_out is not None else torch.empty((L, T), dtype=torch.uint8, device=dev),
+                counts_out if counts_out is not None else torch.empty((L,), dtype=torch.int32, device=dev))
+
+    def prefill(self, h_in, tau: float, seq0: int, n_seqs: int, seq_len: int, flags: int = 0,
+                mask_in=None, h_out=None, gate_out=None, mask_out=None, counts_out=None, stream=None):
+        """Decoder forward on cache slots seq0 .. seq0 + n_seqs - 1, filling their cache."""
+        import torch
+        T = h_in.shape[0]
+        assert T == n_seqs * seq_len and h_in.is_contiguous()
+        outs = self._outs(T, h_in.device, h_out, gate_out, mask_out, counts_out)
+        st = stream if stream is not None else torch.cuda.current_stream(h_in.device)
+        hero_decoder_prefill(self.model, seq0, n_seqs, seq_len, h_in.data_ptr(), tau, flags,
+                             mask_in.data_ptr() if mask_in is not None else 0,
+                             *[o.data_ptr() for o in outs], st.cuda_stream)
+        return outs
+
+    def decode(self, h_in, positions, max_position: int, tau: float, flags: int = 0, mask_in=None,
+               h_out=None, gate_out=None, mask_out=None, counts_out=None, stream=None):
+        """One decoding step for cache slots 0 .. n - 1 (positions: device int32 [n])."""
+        import torch
+        n = h_in.shape[0]
+        assert positions.dtype == torch.int32 and positions.numel() == n and h_in.is_contiguous()
+        outs = self._outs(n, h_in.device, h_out, gate_out, mask_out, counts_out)
+        st = stream if stream is not None else torch.cuda.current_stream(h_in.device)
+        hero_decode_step(self.model, n, positions.data_ptr(), max_position, h_in.data_ptr(), tau,
+                         flags, mask_in.data_ptr() if mask_in is not None else 0,
+                         *[o.data_ptr() for o in outs], st.cuda_stream)
+        return outs
 
     def forward(self, h_in, tau: float, n_seqs: int, seq_len: int, flags: int = 0, mask_in=None,
                 h_out=None, gate_out=None, mask_out=None, counts_out=None, stream=None):

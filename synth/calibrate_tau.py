@@ -99,6 +99,8 @@ def main():
             table = json.load(f)
     for name in names:
         cfg = hi.CONFIGS[name]
+        if cfg.kv_decode_of:   # uses its prefill workload's tau
+            continue
         targets = hi.BYPASS_SWEEP_13B if name == "llama2_13b_prefill" else (cfg.bypass,)
         for tgt in targets:
             res = calibrate(cfg, tgt, args.sample)

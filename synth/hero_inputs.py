@@ -69,6 +69,9 @@ class StackConfig:
     n_heads: int = 0
     n_kv_heads: int = 0
     rope_theta: float = 10000.0
+    # KV-cache decoding: a step is one new token for each of `batch` sequences at
+    # position seq_len (n_tokens = batch); tau comes from the workload named here
+    kv_decode_of: str = ""
 
     @property
     def d_s(self) -> int:
@@ -115,6 +118,12 @@ CONFIGS: Dict[str, StackConfig] = {
     "llama31_8b_decoder": StackConfig("llama31_8b_decoder", 32, 4096, 14336, 64, 64, 16384,
                                       "bf16", 0.2687, batch=4, seq_len=4096, n_heads=32,
                                       n_kv_heads=8, rope_theta=500000.0),
+    # KV-cache decoding with the same model: 64 sequences whose 4096-token prefixes are
+    # in the cache, one new token each per step (T = 64 per step)
+    "llama31_8b_kvdecode": StackConfig("llama31_8b_kvdecode", 32, 4096, 14336, 64, 64, 64,
+                                       "bf16", 0.2687, batch=64, seq_len=4096, n_heads=32,
+                                       n_kv_heads=8, rope_theta=500000.0,
+                                       kv_decode_of="llama31_8b_decoder"),
 }
 
 # The 13B workload is swept over these bypass targets.
@@ -318,6 +327,8 @@ def calibrated_tau(name: str, bypass: Optional[float] = None) -> float:
     with open(_TAU_FILE) as f:
         table = json.load(f)
     cfg = CONFIGS[name]
+    if cfg.kv_decode_of:   # the decoding workload runs the model of its prefill workload
+        return calibrated_tau(cfg.kv_decode_of, bypass)
     b = cfg.bypass if bypass is None else bypass
     key = f"{name}@{b:.4f}"
     if key not in table["tau"]:
