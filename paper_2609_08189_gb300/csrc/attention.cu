@@ -258,16 +258,19 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
 // Decoding step attention (flash-decoding): one query per sequence, the G = H / H_kv
 // query heads of a key/value head together, keys split into chunks of DC positions
 // so that every SM streams the cache.  CTA = (chunk, kv head, sequence), 128 threads:
-//   1. scores: thread t takes keys t, t + 128 of the chunk, one 256-byte key row
-//      each (16 x 16-byte loads), against the G queries (fp32, from shared memory);
+//   1. scores: warp w takes keys 64 w .. 64 w + 63; each load instruction covers two
+//      whole 256-byte key rows (lane: row 2 i + lane / 16, 16-byte chunk lane % 16,
+//      16 loads in flight), lanes multiply by the G queries' matching 8 elements (held
+//      in registers) and the 16 lanes of a row add up by shuffles;
 //   2. per query head (one warp each): chunk max m, p = 2^(s - m), l = sum p;
-//   3. P V: thread t owns value columns 2 (t % 64), +1 for half of the keys
-//      (4-byte loads, 128 contiguous bytes per warp), halves added in shared memory.
+//   3. P V: thread t owns value columns 8 (t % 16) .. +7 of keys t / 16 + 8 i
+//      (16-byte loads, 16 in flight), the 8 key groups added in shared memory.
 // Partial (m, l, o[128]) per (sequence, head, chunk) are merged by k_attn_combine.
 // ---------------------------------------------------------------------------------
 constexpr int DC = 256;          // keys per chunk
 constexpr int DEC_THREADS = 128;
-constexpr int DEC_GMAX = 8;      // query heads per key/value head
+constexpr int DEC_KPW = DC / (DEC_THREADS / 32);   // keys per warp in the score phase
+constexpr int DEC_KG = 8;                          // key groups in the P V phase
 
 template <int G>
 __global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __restrict__ Q,
@@ -280,9 +283,8 @@ __global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __r
                                                              float* __restrict__ po, int n_chunks,
                                                              uint32_t* err) {
   pdl_enter();
-  __shared__ float qs[G][HD];
   __shared__ float sc[G][DC];
-  __shared__ float ored[G][HD];
+  __shared__ __align__(16) float ored[DEC_KG][G][HD];
   const int c = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int len = pos[b] + 1;
@@ -299,39 +301,53 @@ __global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __r
     }
     return;
   }
-  for (int i = tid; i < G * HD; i += DEC_THREADS) {
-    const int g = i / HD, e = i - g * HD;
-    const uint16_t u = Q[((size_t)b * H + kvh * G + g) * HD + e];
-    qs[g][e] = __uint_as_float((uint32_t)u << 16) * scale_log2;
-  }
-  __syncthreads();
   const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * kv_stride * HD;
   const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * kv_stride * HD;
+  const int ch = lane & 15;   // this lane's 16-byte chunk (elements 8 ch .. 8 ch + 7)
+  float qr[G][8];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const uint4 u = *reinterpret_cast<const uint4*>(Q + ((size_t)b * H + kvh * G + g) * HD + ch * 8);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int h2 = 0; h2 < 4; ++h2) {
+      unpack_bf16x2(w[h2], qr[g][2 * h2], qr[g][2 * h2 + 1]);
+      qr[g][2 * h2] *= scale_log2;
+      qr[g][2 * h2 + 1] *= scale_log2;
+    }
+  }
+  const int kw0 = warp * DEC_KPW;   // the warp's first key (offset in the chunk)
 #pragma unroll 1
-  for (int j = j0 + tid; j < j0 + DC; j += DEC_THREADS) {
-    float acc[G];
+  for (int half = 0; half < DEC_KPW / 32; ++half) {
+    uint4 kr[16];
 #pragma unroll
-    for (int g = 0; g < G; ++g) acc[g] = 0.f;
-    if (j < j1) {
-      const uint4* kr = reinterpret_cast<const uint4*>(Kg + (size_t)j * HD);
-      uint4 kv[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) kv[i] = __ldg(kr + i);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const uint32_t w[4] = {kv[i].x, kv[i].y, kv[i].z, kv[i].w};
-#pragma unroll
-        for (int h2 = 0; h2 < 4; ++h2) {
-          float k0, k1;
-          unpack_bf16x2(w[h2], k0, k1);
-          const int e = i * 8 + h2 * 2;
-#pragma unroll
-          for (int g = 0; g < G; ++g) acc[g] += qs[g][e] * k0 + qs[g][e + 1] * k1;
-        }
-      }
+    for (int i = 0; i < 16; ++i) {
+      const int j = j0 + kw0 + half * 32 + 2 * i + (lane >> 4);
+      kr[i] = j < j1 ? __ldg(reinterpret_cast<const uint4*>(Kg + (size_t)j * HD + ch * 8))
+                     : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
-    for (int g = 0; g < G; ++g) sc[g][j - j0] = j < j1 ? acc[g] : -INFINITY;
+    for (int i = 0; i < 16; ++i) {
+      float k8[8];
+      const uint32_t w[4] = {kr[i].x, kr[i].y, kr[i].z, kr[i].w};
+#pragma unroll
+      for (int h2 = 0; h2 < 4; ++h2) unpack_bf16x2(w[h2], k8[2 * h2], k8[2 * h2 + 1]);
+      float acc[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float a = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a += qr[g][e] * k8[e];
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+        acc[g] = a;
+      }
+      if (ch == 0) {
+        const int r = kw0 + half * 32 + 2 * i + (lane >> 4);
+#pragma unroll
+        for (int g = 0; g < G; ++g) sc[g][r] = j0 + r < j1 ? acc[g] : -INFINITY;
+      }
+    }
   }
   __syncthreads();
   for (int g = warp; g < G; g += DEC_THREADS / 32) {
@@ -351,35 +367,51 @@ __global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __r
     }
   }
   __syncthreads();
-  const int col = 2 * (tid & 63), half = tid >> 6;
-  float o0[G], o1[G];
+  const int cg = tid & 15, kg = tid >> 4;
+  float o[G][8];
 #pragma unroll
-  for (int g = 0; g < G; ++g) o0[g] = o1[g] = 0.f;
-#pragma unroll 4
-  for (int j = j0 + half; j < j1; j += 2) {
-    float v0, v1;
-    unpack_bf16x2(__ldg(reinterpret_cast<const uint32_t*>(Vg + (size_t)j * HD + col)), v0, v1);
+  for (int g = 0; g < G; ++g)
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const float p = sc[g][j - j0];
-      o0[g] += p * v0;
-      o1[g] += p * v1;
+    for (int e = 0; e < 8; ++e) o[g][e] = 0.f;
+#pragma unroll
+  for (int h16 = 0; h16 < DC / DEC_KG; h16 += 16) {
+    uint4 vr[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int j = j0 + kg + DEC_KG * (h16 + i);
+      vr[i] = j < j1 ? __ldg(reinterpret_cast<const uint4*>(Vg + (size_t)j * HD + cg * 8))
+                     : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int jj = kg + DEC_KG * (h16 + i);   // p is 0 past the sequence
+      const uint32_t w[4] = {vr[i].x, vr[i].y, vr[i].z, vr[i].w};
+#pragma unroll
+      for (int h2 = 0; h2 < 4; ++h2) {
+        float v0, v1;
+        unpack_bf16x2(w[h2], v0, v1);
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          const float p = sc[g][jj];
+          o[g][2 * h2] += p * v0;
+          o[g][2 * h2 + 1] += p * v1;
+        }
+      }
     }
   }
-  if (half) {
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      ored[g][col] = o0[g];
-      ored[g][col + 1] = o1[g];
-    }
+  for (int g = 0; g < G; ++g) {
+    float4* dst = reinterpret_cast<float4*>(&ored[kg][g][cg * 8]);
+    dst[0] = make_float4(o[g][0], o[g][1], o[g][2], o[g][3]);
+    dst[1] = make_float4(o[g][4], o[g][5], o[g][6], o[g][7]);
   }
   __syncthreads();
-  if (!half) {
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float* dst = po + (part + (size_t)g * n_chunks) * HD + col;
-      *reinterpret_cast<float2*>(dst) = make_float2(o0[g] + ored[g][col], o1[g] + ored[g][col + 1]);
-    }
+  for (int g = 0; g < G; ++g) {
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < DEC_KG; ++k) acc += ored[k][g][tid];
+    po[(part + (size_t)g * n_chunks) * HD + tid] = acc;
   }
 }
 

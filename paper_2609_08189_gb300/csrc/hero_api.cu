@@ -152,6 +152,8 @@ struct hero_model {
   int kv_seqs = 0, kv_len = 0;
   float *dec_pm = nullptr, *dec_pl = nullptr, *dec_po = nullptr;   // decode attention partials
   int* dec_pos = nullptr;      // positions staged for HERO_FLAG_HOST_IO
+  float* dec_ws = nullptr;     // split-K slices of the decoding step's projections
+  size_t dec_ws_floats = 0;
   size_t kv_layer_elems() const { return (size_t)kv_seqs * n_kv_heads * kv_len * 128; }
   uint16_t* kv_k(int jj) { return static_cast<uint16_t*>(kv) + (size_t)jj * 2 * kv_layer_elems(); }
   uint16_t* kv_v(int jj) { return kv_k(jj) + kv_layer_elems(); }
@@ -307,7 +309,7 @@ void free_model(hero_model* m) {
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
-                  m->dec_pm, m->dec_pos};
+                  m->dec_pm, m->dec_pos, m->dec_ws};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -1319,9 +1321,31 @@ hero_status attention_decode_run(hero_model* m, int jj, int B, const int* pos, i
   g.ldo = g.N;
   g.err = m->err;
   g.rope = RopeArgs{m->aq, m->kv_k(jj), m->kv_v(jj), m->rope_cs, pos, H, Hkv, 1, 1, m->kv_len};
-  CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q; k and v into the cache
-    return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
-  }));
+  // few tiles at decoding sizes: split K so that every SM streams weights
+  const int m_t = (B + 127) / 128;
+  const long rows = (long)m_t * 128;
+  auto splits_for = [&](int n, int epi_bytes) {
+    int sp = choose_splits(m_t * ((n + 255) / 256), (d + 63) / 64, m->num_sms, rows, n, epi_bytes);
+    while (sp > 1 && (size_t)sp * rows * n > m->dec_ws_floats) --sp;
+    return sp;
+  };
+  const int qs = splits_for(g.N, 4);
+  if (qs > 1) {
+    GemmArgs sk = g;
+    sk.out_f32 = m->dec_ws;
+    sk.k_splits = qs;
+    sk.split_stride = rows * g.N;
+    CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+      return launch_gemm_tc(256, EPI_STORE_F32, m->tm_ax, m->tm_wqkv[jj], sk, m->num_sms, st);
+    }));
+    CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // RoPE; q; k and v into the cache
+      return launch_qkv_close(m->dec_ws, qs, sk.split_stride, B, g.rope, m->err, st);
+    }));
+  } else {
+    CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q; k and v into the cache
+      return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
+    }));
+  }
   CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
     return launch_attn_decode(m->aq, m->kv_k(jj), m->kv_v(jj), pos, B, H, Hkv, m->kv_len, max_pos,
                               m->dec_pm, m->dec_pl, m->dec_po, m->ao, m->err, st);
@@ -1335,6 +1359,20 @@ hero_status attention_decode_run(hero_model* m, int jj, int B, const int* pos, i
   o.resid = h;
   o.err = m->err;
   o.lo = entry;
+  const int os = splits_for(d, 22);
+  if (os > 1) {
+    GemmArgs sk = o;
+    sk.out_f32 = m->dec_ws;
+    sk.k_splits = os;
+    sk.split_stride = rows * d;
+    CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+      return launch_gemm_tc(256, EPI_STORE_F32, m->tm_ao, m->tm_wo[jj], sk, m->num_sms, st);
+    }));
+    CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
+      return launch_entry_close(m->dec_ws, os, sk.split_stride, B, h, entry, st);
+    }));
+    return HERO_OK;
+  }
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
     return launch_gemm_tc(256, EPI_ATTN_ENTRY, m->tm_ao, m->tm_wo[jj], o, m->num_sms, st);
   }));
@@ -1500,6 +1538,12 @@ extern "C" hero_status hero_kv_cache_init(hero_model* m, int32_t max_seqs, int32
   m->dec_pl = m->dec_pm + pr;
   m->dec_po = m->dec_pl + pr;
   CUDA_TRY(cudaMalloc(&m->dec_pos, (size_t)max_seqs * 4));
+  {   // split-K slices: at most 16 splits of 128-row tiles of the wider projection
+    const long rows = ((long)std::min(max_seqs, c.max_tokens) + 127) / 128 * 128;
+    const long nmax = std::max((long)(m->n_heads + 2 * m->n_kv_heads) * 128, (long)c.d_model);
+    m->dec_ws_floats = (size_t)16 * rows * nmax;
+    CUDA_TRY(cudaMalloc(&m->dec_ws, m->dec_ws_floats * 4));
+  }
   if (hero_status rs = build_rope_table(m, max_len); rs != HERO_OK) return rs;
   m->kv_seqs = max_seqs;
   m->kv_len = max_len;

