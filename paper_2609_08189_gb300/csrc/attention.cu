@@ -255,6 +255,315 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
 }
 
 // ---------------------------------------------------------------------------------
+// Causal attention on the tcgen05 tensor cores (sequences of 128 tokens or more).
+// CTA = 128 query rows of one (sequence, head), 10 warps:
+//   warp 0     TMA producer: Q once, then K and V^T tiles of 128 keys into a 2-stage ring
+//   warp 1     TMEM allocator and MMA issuer: S_i = Q K_i^T into one of two TMEM score
+//              buffers, O += P_{i-1} V_{i-1} into the TMEM output accumulator
+//   warps 2-9  softmax, two threads per query row (its TMEM lane), each on 64 of the
+//              tile's 128 keys and of O's 128 columns (the two halves exchange their
+//              row maxima through shared memory): online softmax in log2 units whose
+//              running max is raised only when a row's max grows by more than 8 (then
+//              that row's O and l are rescaled; otherwise the stale max keeps every
+//              p <= 2^8), P_i as bf16 into shared memory (the A operand of P V, 128-byte
+//              swizzle; each half writes one 64-key panel), finally O / l in bf16.
+// Issue order S_0, S_1, PV_0, S_2, PV_1, ...: the softmax of tile i overlaps PV_{i-1}
+// and S_{i+1}.  All operands are K-major (V arrives transposed, keys contiguous), 128 x
+// 64 bf16 panels with the 128-byte swizzle as the GEMM's.  Every mbarrier wait is
+// bounded; on expiry the CTA drains its copies and MMAs, reports through err and frees
+// its TMEM.
+// ---------------------------------------------------------------------------------
+namespace fa {
+constexpr int BM = 128, BN = 128, THREADS = 320, HALF = BN / 2;
+constexpr uint32_t PANEL = 128 * 128;   // [128 rows][64 bf16] = 16 KB
+constexpr uint32_t TILE = 2 * PANEL;    // [128 rows][128 bf16]
+constexpr uint32_t OFF_Q = 0, OFF_K = TILE, OFF_V = 3 * TILE, OFF_P = 5 * TILE, OFF_BAR = 6 * TILE;
+enum { Q_FULL = 0, K_FULL = 1, V_FULL = 3, KV_EMPTY = 5, S_FULL = 7, S_FREE = 9, P_FULL = 11,
+       O_DONE = 12, DRAIN = 13, NBAR = 14 };
+constexpr uint32_t OFF_RED = OFF_BAR + 256;   // float [2 tiles][2 halves][128 rows] maxima
+constexpr uint32_t OFF_LSUM = OFF_RED + 2 * 2 * 128 * 4;   // float [2 halves][128 rows]
+constexpr size_t SMEM = OFF_LSUM + 2 * 128 * 4 + 1024;
+constexpr uint32_t TMEM_COLS = 512;     // S0 | S1 | O (128 columns each)
+// kind::f16 instruction descriptor: fp32 D, bf16 A and B, K-major, N = 128, M = 128
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                           ((uint32_t)(BM >> 4) << 24);
+constexpr float RESCALE = 8.f;          // log2 units
+}  // namespace fa
+
+__global__ void __launch_bounds__(fa::THREADS, 1)
+    k_flash_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const __grid_constant__ CUtensorMap tmV, int H, int Hkv, int S, float scale_log2,
+               uint16_t* __restrict__ O, uint32_t* err) {
+  using namespace fa;
+  pdl_enter();
+  extern __shared__ uint8_t fa_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(fa_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sb = smem_u32(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  const uint32_t bar0 = smem_u32(bars);
+  auto bar = [&](int i) { return bar0 + 8u * i; };
+  volatile uint32_t* misc = reinterpret_cast<volatile uint32_t*>(bars + NBAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = gridDim.x - 1 - blockIdx.x;   // long rows first
+  const int hh = blockIdx.y, b = blockIdx.z;
+  const int kvh = hh / (H / Hkv);
+  const int q0 = qt * BM;
+  const int n = qt + 1;                        // causal: key tiles 0 .. qt
+  if (threadIdx.x == 0) {
+    mbar_init(bar(Q_FULL), 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(bar(K_FULL + s), 1);
+      mbar_init(bar(V_FULL + s), 1);
+      mbar_init(bar(KV_EMPTY + s), 1);
+      mbar_init(bar(S_FULL + s), 1);
+      mbar_init(bar(S_FREE + s), 8);
+    }
+    mbar_init(bar(P_FULL), 8);
+    mbar_init(bar(O_DONE), 1);
+    mbar_init(bar(DRAIN), 1);
+    misc[1] = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<uint32_t*>(misc)), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = misc[0];
+  const uint32_t tO = tbase + 256;
+
+  if (warp == 0) {
+    // ------------------------------ TMA producer ------------------------------
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      const int zq = b * H + hh, zk = b * Hkv + kvh;
+      mbar_arrive_expect_tx(bar(Q_FULL), TILE);
+      tma_load_3d(sb + OFF_Q, &tmQ, 0, q0, zq, bar(Q_FULL));
+      tma_load_3d(sb + OFF_Q + PANEL, &tmQ, 64, q0, zq, bar(Q_FULL));
+      bool ok = true, issued[2] = {false, false};
+      uint32_t par[2] = {0, 0};
+      for (int i = 0; i < n; ++i) {
+        const int st = i & 1;
+        const uint32_t ph = (i >> 1) & 1;
+        if (!mbar_wait(bar(KV_EMPTY + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
+          ok = false;
+          break;
+        }
+        const uint32_t sk = sb + OFF_K + st * TILE, sv = sb + OFF_V + st * TILE;
+        mbar_arrive_expect_tx(bar(K_FULL + st), TILE);
+        tma_load_3d(sk, &tmK, 0, i * BN, zk, bar(K_FULL + st));
+        tma_load_3d(sk + PANEL, &tmK, 64, i * BN, zk, bar(K_FULL + st));
+        mbar_arrive_expect_tx(bar(V_FULL + st), TILE);
+        tma_load_3d(sv, &tmV, i * BN, 0, zk, bar(V_FULL + st));
+        tma_load_3d(sv + PANEL, &tmV, i * BN + 64, 0, zk, bar(V_FULL + st));
+        issued[st] = true;
+        par[st] = ph;
+      }
+      if (!ok) {   // let copies still in flight land before the CTA can exit
+        misc[1] = 1;
+        atomicOr(err, ERR_WAIT_PRODUCER);
+        mbar_wait(bar(Q_FULL), 0, 100000000ull);
+        for (int s = 0; s < 2; ++s)
+          if (issued[s]) {
+            mbar_wait(bar(K_FULL + s), par[s], 100000000ull);
+            mbar_wait(bar(V_FULL + s), par[s], 100000000ull);
+          }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer ------------------------------
+    if (lane == 0) {
+      bool ok = mbar_wait(bar(Q_FULL), 0, kWaitLimitNs) && !misc[1];
+      tc_fence_after();
+      auto pv = [&](int j) -> bool {   // O += P_j V_j
+        const int st = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        if (!mbar_wait(bar(V_FULL + st), ph, kWaitLimitNs) ||
+            !mbar_wait(bar(P_FULL), j & 1, kWaitLimitNs) || misc[1])
+          return false;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t ad = sw128_desc(sb + OFF_P + (kk >> 2) * PANEL) + 2u * (kk & 3);
+          const uint64_t bd = sw128_desc(sb + OFF_V + st * TILE + (kk >> 2) * PANEL) + 2u * (kk & 3);
+          umma_bf16(tO, ad, bd, IDESC, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(bar(O_DONE));
+        umma_commit(bar(KV_EMPTY + st));
+        return true;
+      };
+      for (int i = 0; i < n && ok; ++i) {
+        const int st = i & 1;
+        const uint32_t ph = (i >> 1) & 1;
+        if (!mbar_wait(bar(K_FULL + st), ph, kWaitLimitNs) ||
+            !mbar_wait(bar(S_FREE + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tS = tbase + st * 128;
+#pragma unroll
+        for (int kk = 0; kk < 128 / 16; ++kk) {   // S_i = Q K_i^T over the head dimension
+          const uint64_t ad = sw128_desc(sb + OFF_Q + (kk >> 2) * PANEL) + 2u * (kk & 3);
+          const uint64_t bd = sw128_desc(sb + OFF_K + st * TILE + (kk >> 2) * PANEL) + 2u * (kk & 3);
+          umma_bf16(tS, ad, bd, IDESC, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(bar(S_FULL + st));
+        if (i >= 1 && !pv(i - 1)) ok = false;
+      }
+      if (ok) ok = pv(n - 1);
+      if (!ok) {
+        misc[1] = 1;
+        atomicOr(err, ERR_WAIT_MMA);
+        umma_commit(bar(DRAIN));   // completes once every issued MMA has finished
+        if (!mbar_wait(bar(DRAIN), 0, 100000000ull)) atomicOr(err, ERR_WAIT_DRAIN);
+      }
+    }
+  } else {
+    // ------------------------------ softmax ------------------------------
+    const int quad = warp & 3;                  // TMEM lane quadrant of this warp
+    const int half = (warp - 2) >> 2;           // keys / O columns [64 half, 64 half + 64)
+    const int r = quad * 32 + lane;             // query row in the tile
+    const int qpos = q0 + r;
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    float* red = reinterpret_cast<float*>(smem + OFF_RED);     // [2][2][128]
+    float* lsum = reinterpret_cast<float*>(smem + OFF_LSUM);   // [2][128]
+    auto pair_sync = [&]() {   // the two warps of this quadrant (named barrier 1 + quad)
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
+    };
+    float m_used = -INFINITY, l = 0.f;          // m_used in raw score units
+    // The two warps of a quadrant meet at a named barrier once per tile and once at
+    // the end, whatever happens: a warp whose wait expired keeps stepping through the
+    // loop without touching TMEM, so neither can be left waiting at the barrier.
+    bool ok = true;
+    for (int i = 0; i < n; ++i) {
+      const int st = i & 1;
+      const uint32_t ph = (i >> 1) & 1;
+      if (ok) {
+        bool w = mbar_wait(bar(S_FULL + st), ph, kWaitLimitNs);
+        w = __all_sync(0xffffffffu, w) && !misc[1];
+        ok = __all_sync(0xffffffffu, w);
+      }
+      float sv[HALF];
+      if (ok) {
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < HALF / 32; ++c) {
+          uint32_t rr[32];
+          tmem_ld32(tbase + st * 128 + lane_off + half * HALF + c * 32, rr);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) sv[c * 32 + e] = __uint_as_float(rr[e]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(S_FREE + st));   // S_{i+2} may overwrite it
+      } else {
+#pragma unroll
+        for (int c = 0; c < HALF; ++c) sv[c] = 0.f;
+      }
+      if (i == n - 1) {   // the diagonal tile: causal mask and the sequence end
+        const int k0 = i * BN + half * HALF;
+#pragma unroll
+        for (int c = 0; c < HALF; ++c)
+          if (k0 + c > qpos || k0 + c >= S) sv[c] = -INFINITY;
+      }
+      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+      for (int c = 0; c < HALF; ++c) m4[c & 3] = fmaxf(m4[c & 3], sv[c]);
+      red[(st * 2 + half) * 128 + r] = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+      pair_sync();
+      if (!ok) continue;
+      const float mx = fmaxf(red[(st * 2) * 128 + r], red[(st * 2 + 1) * 128 + r]);
+      float alpha = 1.f;
+      if ((mx - m_used) * scale_log2 > RESCALE) {   // raise the running max (first tile: always)
+        alpha = exp2f((m_used - mx) * scale_log2);
+        m_used = mx;
+        l *= alpha;
+      }
+      const float mb = -m_used * scale_log2;
+      uint32_t pk[HALF / 2];
+      float ps[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < HALF / 2; ++c) {
+        const float p0 = exp2f(fmaf(sv[2 * c], scale_log2, mb));
+        const float p1 = exp2f(fmaf(sv[2 * c + 1], scale_log2, mb));
+        ps[c & 3] += p0 + p1;
+        pk[c] = pack_bf16x2(p0, p1);
+      }
+      l += (ps[0] + ps[1]) + (ps[2] + ps[3]);
+      if (i >= 1) {   // the P buffer and O are free once PV_{i-1} has completed
+        const bool w = mbar_wait(bar(O_DONE), (i - 1) & 1, kWaitLimitNs);
+        if (!__all_sync(0xffffffffu, w)) {
+          ok = false;
+          continue;
+        }
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, alpha != 1.f)) {   // rescale this warp's half of O
+#pragma unroll 1
+          for (int c = 0; c < HALF / 32; ++c) {
+            uint32_t rr[32];
+            tmem_ld32(tO + lane_off + half * HALF + c * 32, rr);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
+            tmem_st32(tO + lane_off + half * HALF + c * 32, rr);
+          }
+        }
+      }
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {   // this half's panel of P, 128-byte swizzle
+        const uint32_t off = OFF_P + half * PANEL + r * 128 + ((ch ^ (r & 7)) << 4);
+        *reinterpret_cast<uint4*>(smem + off) =
+            make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(P_FULL));
+    }
+    if (ok) {
+      const bool w = mbar_wait(bar(O_DONE), (n - 1) & 1, kWaitLimitNs);
+      ok = __all_sync(0xffffffffu, w);
+    }
+    // both halves of a row reach this exchange (a warp that gave up passes l = 0)
+    lsum[half * 128 + r] = l;
+    pair_sync();
+    if (ok) {
+      tc_fence_after();
+      const float inv = 1.f / (lsum[r] + lsum[128 + r]);
+      uint16_t* orow = O + ((size_t)b * S + qpos) * H * 128 + hh * 128 + half * HALF;
+#pragma unroll 1
+      for (int c = 0; c < HALF / 32; ++c) {
+        uint32_t rr[32];
+        tmem_ld32(tO + lane_off + half * HALF + c * 32, rr);
+        if (qpos < S) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            dst[q] = make_uint4(pack_bf16x2(__uint_as_float(rr[8 * q]) * inv, __uint_as_float(rr[8 * q + 1]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 2]) * inv, __uint_as_float(rr[8 * q + 3]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 4]) * inv, __uint_as_float(rr[8 * q + 5]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 6]) * inv, __uint_as_float(rr[8 * q + 7]) * inv));
+        }
+      }
+    } else if (lane == 0) {
+      misc[1] = 1;
+      atomicOr(err, ERR_WAIT_EPILOGUE);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tbase, fa::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------------
 // Decoding step attention (flash-decoding): one query per sequence, the G = H / H_kv
 // query heads of a key/value head together, keys split into chunks of DC positions
 // so that every SM streams the cache.  CTA = (chunk, kv head, sequence), 128 threads:
@@ -503,6 +812,27 @@ cudaError_t launch_attn_decode(const void* Q, const void* K, const void* V, cons
   return launch_pdl(k_attn_combine, dim3((unsigned)((BH + 7) / 8)), dim3(256), 0, st,
                     static_cast<const float*>(pm), static_cast<const float*>(pl),
                     static_cast<const float*>(po), BH, nc, static_cast<uint16_t*>(O));
+}
+
+}  // namespace hero
+
+namespace hero {
+
+cudaError_t launch_flash_tc(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                            int B, int S, int H, int Hkv, void* O, uint32_t* err, cudaStream_t st) {
+  if (B <= 0 || S <= 0) return cudaSuccess;
+  if (H % Hkv || H > 65535 || B > 65535) return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_flash_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)fa::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
+  const dim3 grid((unsigned)((S + fa::BM - 1) / fa::BM), (unsigned)H, (unsigned)B);
+  return launch_pdl(k_flash_tc, grid, dim3(fa::THREADS), fa::SMEM, st, tmQ, tmK, tmV, H, Hkv, S,
+                    scale_log2, static_cast<uint16_t*>(O), err);
 }
 
 }  // namespace hero

@@ -195,6 +195,18 @@ __device__ __forceinline__ void epi_qkv_rope(const GemmArgs& a, uint32_t tbase, 
       if (!valid) continue;
       uint16_t* dst;
       const bool rot = head < r.H + r.Hkv;
+      if (!rot && r.vt) {   // v transposed: element e of this token at [e][s]
+        uint16_t* vt = static_cast<uint16_t*>(r.vt) +
+                       ((size_t)bq * r.Hkv + head - r.H - r.Hkv) * 128 * (size_t)r.S_pad + s;
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          vt[(size_t)(c0 + e) * r.S_pad] =
+              (uint16_t)(pack_bf16x2(__uint_as_float(x1[e]), 0.f) & 0xffffu);
+          vt[(size_t)(c0 + 64 + e) * r.S_pad] =
+              (uint16_t)(pack_bf16x2(__uint_as_float(x2[e]), 0.f) & 0xffffu);
+        }
+      }
+      if (!rot && !r.v) continue;
       if (head < r.H)
         dst = static_cast<uint16_t*>(r.q) + (((size_t)bq * r.H + head) * r.S_q + sq) * 128;
       else if (rot)

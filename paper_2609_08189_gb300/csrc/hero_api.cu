@@ -70,6 +70,22 @@ bool encode_bf16_2d(CUtensorMap* tm, const void* ptr, uint64_t inner, uint64_t o
   return r == CUDA_SUCCESS;
 }
 
+// 3-D bf16 map with 64 x 128 x 1 boxes (128-byte swizzle; out-of-range elements read 0):
+// dims d0 (contiguous) x d1 x d2, byte strides s1 (between d1 rows) and s2.
+bool encode_bf16_3d(CUtensorMap* tm, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d2,
+                    uint64_t s1, uint64_t s2) {
+  if (!get_encoder()) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1, s2};
+  cuuint32_t box[3] = {64, 128, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 std::vector<float> host_f32(const void* p, size_t n, hero_dtype dt) {
   std::vector<float> v(n);
   if (dt == HERO_BF16) {
@@ -144,6 +160,8 @@ struct hero_model {
   float* attn_gain = nullptr;  // [L][d]
   void* aws = nullptr;         // attention workspace
   void *ax = nullptr, *aq = nullptr, *ak = nullptr, *av = nullptr, *ao = nullptr;
+  void* avt = nullptr;         // v transposed for the tensor-core attention (S >= 128)
+  size_t avt_elems = 0;
   float *hcur = nullptr, *dlprev = nullptr;
   float* rope_cs = nullptr;    // [rope_rows][64][2] RoPE cos, sin (own allocation)
   long rope_rows = 0;
@@ -1113,11 +1131,24 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   g.ldo = nqkv;
   g.err = m->err;
   const KvTarget kt = kv ? *kv : KvTarget{m->ak, m->av, S};
-  g.rope = RopeArgs{m->aq, kt.k, kt.v, m->rope_cs, nullptr, H, Hkv, S, S, kt.stride};
+  // sequences of 128 or more run the tensor-core attention, which reads v transposed
+  const int S_pad = (S + 63) / 64 * 64;
+  const bool tc = S >= 128 && (size_t)B * Hkv * 128 * S_pad <= m->avt_elems;
+  g.rope = RopeArgs{m->aq, kt.k, (kv || !tc) ? kt.v : nullptr, m->rope_cs, nullptr, H, Hkv, S, S,
+                    kt.stride, tc ? m->avt : nullptr, S_pad};
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q, k, v with RoPE, attention layout
     return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
   }));
   CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
+    if (tc) {
+      CUtensorMap tq, tk, tv;
+      if (!encode_bf16_3d(&tq, m->aq, 128, S, (uint64_t)B * H, 256, (uint64_t)S * 256) ||
+          !encode_bf16_3d(&tk, kt.k, 128, S, (uint64_t)B * Hkv, 256, (uint64_t)kt.stride * 256) ||
+          !encode_bf16_3d(&tv, m->avt, S, 128, (uint64_t)B * Hkv, (uint64_t)S_pad * 2,
+                          (uint64_t)S_pad * 256))
+        return cudaErrorInvalidValue;
+      return launch_flash_tc(tq, tk, tv, B, S, H, Hkv, m->ao, m->err, st);
+    }
     return launch_flash_attn(m->aq, kt.k, kt.v, B, S, H, Hkv, kt.stride, m->ao, st);
   }));
   GemmArgs o{};
@@ -1234,11 +1265,14 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
     void** p;
     size_t bytes;
   };
+  // v transposed: sequences of S >= 128 padded to a multiple of 64 positions
+  const size_t avt_elems = (size_t)Hkv * 128 * (size_t)(Tm + 63 * (Tm / 128) + 64);
   std::vector<Item> items = {
       {&m->ax, (size_t)Tm * d * 2},          {&m->ao, (size_t)Tm * d * 2},
       {&m->aq, (size_t)Tm * H * 128 * 2},
       {&m->ak, (size_t)Tm * Hkv * 128 * 2},  {&m->av, (size_t)Tm * Hkv * 128 * 2},
       {(void**)&m->hcur, (size_t)Tm * d * 4},
+      {&m->avt, avt_elems * 2},
       {(void**)&m->dlprev, (size_t)Tm * d * 4}};
   size_t off = 0;
   for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
@@ -1260,6 +1294,7 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   if (!ok) return fail(HERO_ERR_CUDA, "tensor map encoding failed");
   m->n_heads = (int)H;
   m->n_kv_heads = (int)Hkv;
+  m->avt_elems = avt_elems;
   m->attn = true;
   return HERO_OK;
 }

@@ -96,10 +96,12 @@ enum EpiKind : int {
 struct RopeArgs {
   void* q;             // bf16 [B][H][S_q][128]; a decoding step stores at index 0 (S_q = 1)
   void* k;             // bf16 [B][H_kv][S_kv][128] at the token's position
-  void* v;             // bf16 [B][H_kv][S_kv][128]
+  void* v;             // bf16 [B][H_kv][S_kv][128], or nullptr (v only transposed)
   const float* cs;     // [positions >= S_kv][64][2]: cos, sin
   const int* pos;      // [B] positions of a decoding step, or nullptr
   int H, Hkv, S, S_q, S_kv;
+  void* vt;            // bf16 [B][H_kv][128][S_pad]: v transposed (keys contiguous), or nullptr
+  int S_pad;           // positions per row of vt (a multiple of 8)
 };
 
 struct GemmArgs {
@@ -157,6 +159,11 @@ cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float
 // K and V hold kv_stride positions per (sequence, head) slab (>= S; the cache's max_len).
 cudaError_t launch_flash_attn(const void* Q, const void* K, const void* V, int B, int S, int H,
                               int Hkv, int kv_stride, void* O, cudaStream_t st);
+// Causal attention on the tcgen05 tensor cores: 3-D tensor maps (128-byte swizzle,
+// boxes of 64 x 128 x 1) over Q [B H][S][128], K [B H_kv][S (stride kv_stride)][128]
+// and V^T [B H_kv][128][S (stride S_pad)]; O [B S][H 128] bf16.
+cudaError_t launch_flash_tc(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                            int B, int S, int H, int Hkv, void* O, uint32_t* err, cudaStream_t st);
 // Decoding step: Q [B][H][128], K/V slabs of kv_stride positions, pos [B] (each <=
 // max_pos < kv_stride); partials pm, pl [B][H][chunks], po [B][H][chunks][128] with
 // chunks = attn_decode_chunks(max_pos); O [B][H 128] bf16.

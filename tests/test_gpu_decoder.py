@@ -55,7 +55,10 @@ def _attn_err(x, y, h):
 # the attention sublayer alone
 # ------------------------------------------------------------------------------
 
-SHAPES = [(2, 160), (1, 1), (5, 1), (3, 77), (1, 64), (1, 300), (4, 65), (0, 8)]
+# S >= 128 runs the tensor-core kernel (128-row query tiles, K and transposed V tiles
+# of 128 keys), shorter sequences the mma.sync kernel (64-row tiles)
+SHAPES = [(2, 160), (1, 1), (5, 1), (3, 77), (1, 64), (1, 300), (4, 65), (0, 8), (1, 128),
+          (2, 256), (3, 130), (1, 511)]
 
 
 @pytest.fixture(scope="module")
@@ -69,9 +72,9 @@ def small_decoder(hero):
 
 @pytest.mark.parametrize("n_seqs,seq_len", SHAPES)
 def test_attention_block_parity(small_decoder, n_seqs, seq_len):
-    """Every layer, several sequence shapes: ragged query/key tiles (77, 65, 160,
-    300 = 4 tiles + 44), one tile exactly (64), single-token sequences (the score is
-    the token with itself: o = v), and no sequences."""
+    """Every layer, several sequence shapes: ragged query/key tiles (77, 65, 130, 160,
+    300, 511), whole tiles (64, 128, 256), single-token sequences (the score is the
+    token with itself: o = v), and no sequences."""
     import torch
     cfg, _, wa, dec = small_decoder
     T = n_seqs * seq_len
