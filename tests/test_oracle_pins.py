@@ -750,3 +750,17 @@ def test_attention_rows_equals_full_sublayer():
     got = ho.attention_rows(h, rows, wa, cfg.n_heads, cfg.n_kv_heads, cfg.rope_theta, cfg.rms_eps,
                             ho.bf16_round)
     np.testing.assert_allclose(got, full[rows], rtol=0, atol=1e-12)
+
+
+def test_rope_is_complex_rotation():
+    """RoPE in its complex form (RoFormer): the pair (x_i, x_{i+hd/2}) read as
+    z = x_i + i x_{i+hd/2} is multiplied by exp(i s theta^(-2i/hd)) at position s."""
+    rng = np.random.default_rng(1)
+    hd, S, theta = 16, 12, 500000.0
+    x = rng.standard_normal((S, hd))
+    cos, sin = ho.rope_cos_sin(S, hd, theta)
+    got = ho.apply_rope(x, cos, sin)
+    z = x[:, :hd // 2] + 1j * x[:, hd // 2:]
+    ang = np.arange(S)[:, None] * theta ** (-2.0 * np.arange(hd // 2)[None, :] / hd)
+    w = z * np.exp(1j * ang)
+    np.testing.assert_allclose(got, np.concatenate([w.real, w.imag], axis=1), rtol=0, atol=1e-13)
