@@ -256,44 +256,47 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
 
 // ---------------------------------------------------------------------------------
 // Causal attention on the tcgen05 tensor cores (sequences of 128 tokens or more).
-// CTA = 128 query rows of one (sequence, head), 10 warps:
-//   warp 0     TMA producer: Q once, then K and V^T tiles of 128 keys into a 2-stage ring
-//   warp 1     TMEM allocator and MMA issuer: S_i = Q K_i^T into one of two TMEM score
-//              buffers, O += P_{i-1} V_{i-1} into the TMEM output accumulator
-//   warps 2-9  softmax, two threads per query row (its TMEM lane), each on 64 of the
-//              tile's 128 keys and of O's 128 columns (the two halves exchange their
-//              row maxima through shared memory): online softmax in log2 units whose
-//              running max is raised only when a row's max grows by more than 8 (then
-//              that row's O and l are rescaled; otherwise the stale max keeps every
-//              p <= 2^8), P_i as bf16 into shared memory (the A operand of P V, 128-byte
-//              swizzle; each half writes one 64-key panel), finally O / l in bf16.
-// Issue order S_0, S_1, PV_0, S_2, PV_1, ...: the softmax of tile i overlaps PV_{i-1}
-// and S_{i+1}.  All operands are K-major (V arrives transposed, keys contiguous), 128 x
-// 64 bf16 panels with the 128-byte swizzle as the GEMM's.  Every mbarrier wait is
-// bounded; on expiry the CTA drains its copies and MMAs, reports through err and frees
-// its TMEM.
+// CTA = two query tiles of 128 rows (A = 2p, B = 2p + 1) of one (sequence, head),
+// sharing every K and V^T tile; 10 warps:
+//   warp 0     TMA producer: Q_A, Q_B once, K tiles of 128 keys through a 2-stage ring,
+//              V^T tiles through one stage
+//   warp 1     TMEM allocator and MMA issuer, ping-pong between the tiles:
+//              S_A(0) S_B(0) | PV_A(0) S_A(1) | PV_B(0) S_B(1) | PV_A(1) S_A(2) | ...
+//              so the tensor pipe works on one tile while the other's softmax runs
+//   warps 2-5  softmax of tile A, warps 6-9 of tile B: one thread per query row (its TMEM
+//              lane) reads the row of S from TMEM, runs the online softmax in log2 units
+//              (exp2 of one FMA; the running max is raised only when the row max grows
+//              by more than 8, then that row's O and l are rescaled, otherwise the stale
+//              max keeps every p <= 2^8), writes P as the bf16 A operand of P V (128-byte
+//              swizzle) and finally O / l in bf16.
+// TMEM: S_A | O_A | S_B | O_B, 128 columns each.  A tile's S(i + 1) is issued after its
+// P V(i), and tcgen05.commit signals only when every earlier MMA of the issuing thread has
+// completed, so once S(i + 1) is visible P V(i) has finished: the softmax may then
+// overwrite P and rescale O without another barrier.  All operands are K-major (V^T from
+// the q/k/v epilogue) in 128 x 64 bf16 panels.  Every mbarrier wait is bounded; on expiry
+// the CTA drains its copies and MMAs, reports through err and frees its TMEM.
 // ---------------------------------------------------------------------------------
 namespace fa {
-constexpr int BM = 128, BN = 128, THREADS = 320, HALF = BN / 2;
+constexpr int BM = 128, BN = 128, THREADS = 320;
 constexpr uint32_t PANEL = 128 * 128;   // [128 rows][64 bf16] = 16 KB
 constexpr uint32_t TILE = 2 * PANEL;    // [128 rows][128 bf16]
-constexpr uint32_t OFF_Q = 0, OFF_K = TILE, OFF_V = 3 * TILE, OFF_P = 5 * TILE, OFF_BAR = 6 * TILE;
-enum { Q_FULL = 0, K_FULL = 1, V_FULL = 3, KV_EMPTY = 5, S_FULL = 7, S_FREE = 9, P_FULL = 11,
-       O_DONE = 12, DRAIN = 13, NBAR = 14 };
-constexpr uint32_t OFF_RED = OFF_BAR + 256;   // float [2 tiles][2 halves][128 rows] maxima
-constexpr uint32_t OFF_LSUM = OFF_RED + 2 * 2 * 128 * 4;   // float [2 halves][128 rows]
-constexpr size_t SMEM = OFF_LSUM + 2 * 128 * 4 + 1024;
-constexpr uint32_t TMEM_COLS = 512;     // S0 | S1 | O (128 columns each)
+constexpr uint32_t OFF_Q = 0, OFF_K = 2 * TILE, OFF_V = 4 * TILE, OFF_P = 5 * TILE,
+                   OFF_BAR = 7 * TILE;  // Q_A Q_B | K0 K1 | V | P_A P_B
+enum { Q_FULL = 0, K_FULL = 1, K_EMPTY = 3, V_FULL = 5, V_EMPTY = 6, S_FULL = 7, P_FULL = 9,
+       FINAL = 11, DRAIN = 12, NBAR = 13 };
+constexpr size_t SMEM = OFF_BAR + NBAR * 8 + 16 + 1024;
+constexpr uint32_t TMEM_COLS = 512;
 // kind::f16 instruction descriptor: fp32 D, bf16 A and B, K-major, N = 128, M = 128
 constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                            ((uint32_t)(BM >> 4) << 24);
 constexpr float RESCALE = 8.f;          // log2 units
+static_assert(SMEM <= 232448, "shared memory per CTA");
 }  // namespace fa
 
 __global__ void __launch_bounds__(fa::THREADS, 1)
     k_flash_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-               const __grid_constant__ CUtensorMap tmV, int H, int Hkv, int S, float scale_log2,
-               uint16_t* __restrict__ O, uint32_t* err) {
+               const __grid_constant__ CUtensorMap tmV, int H, int Hkv, int S, int n_qt,
+               float scale_log2, uint16_t* __restrict__ O, uint32_t* err) {
   using namespace fa;
   pdl_enter();
   extern __shared__ uint8_t fa_raw[];
@@ -305,22 +308,24 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
   auto bar = [&](int i) { return bar0 + 8u * i; };
   volatile uint32_t* misc = reinterpret_cast<volatile uint32_t*>(bars + NBAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = gridDim.x - 1 - blockIdx.x;   // long rows first
+  const int pr = gridDim.x - 1 - blockIdx.x;   // long rows first
   const int hh = blockIdx.y, b = blockIdx.z;
   const int kvh = hh / (H / Hkv);
-  const int q0 = qt * BM;
-  const int n = qt + 1;                        // causal: key tiles 0 .. qt
+  const int qtA = 2 * pr;
+  const bool hasB = qtA + 1 < n_qt;
+  const int nA = qtA + 1, nB = hasB ? qtA + 2 : 0;   // causal: key tiles 0 .. qt
+  const int n = hasB ? nB : nA;
   if (threadIdx.x == 0) {
     mbar_init(bar(Q_FULL), 1);
     for (int s = 0; s < 2; ++s) {
       mbar_init(bar(K_FULL + s), 1);
-      mbar_init(bar(V_FULL + s), 1);
-      mbar_init(bar(KV_EMPTY + s), 1);
+      mbar_init(bar(K_EMPTY + s), 1);
       mbar_init(bar(S_FULL + s), 1);
-      mbar_init(bar(S_FREE + s), 8);
+      mbar_init(bar(P_FULL + s), 4);
     }
-    mbar_init(bar(P_FULL), 8);
-    mbar_init(bar(O_DONE), 1);
+    mbar_init(bar(V_FULL), 1);
+    mbar_init(bar(V_EMPTY), 1);
+    mbar_init(bar(FINAL), 1);
     mbar_init(bar(DRAIN), 1);
     misc[1] = 0;
     fence_mbar_init();
@@ -333,7 +338,8 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tbase = misc[0];
-  const uint32_t tO = tbase + 256;
+  auto tS = [&](int x) { return tbase + 256u * x; };
+  auto tO = [&](int x) { return tbase + 256u * x + 128u; };
 
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
@@ -342,143 +348,141 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
       const int zq = b * H + hh, zk = b * Hkv + kvh;
-      mbar_arrive_expect_tx(bar(Q_FULL), TILE);
-      tma_load_3d(sb + OFF_Q, &tmQ, 0, q0, zq, bar(Q_FULL));
-      tma_load_3d(sb + OFF_Q + PANEL, &tmQ, 64, q0, zq, bar(Q_FULL));
-      bool ok = true, issued[2] = {false, false};
-      uint32_t par[2] = {0, 0};
-      for (int i = 0; i < n; ++i) {
+      mbar_arrive_expect_tx(bar(Q_FULL), hasB ? 2 * TILE : TILE);
+      tma_load_3d(sb + OFF_Q, &tmQ, 0, qtA * BM, zq, bar(Q_FULL));
+      tma_load_3d(sb + OFF_Q + PANEL, &tmQ, 64, qtA * BM, zq, bar(Q_FULL));
+      if (hasB) {
+        tma_load_3d(sb + OFF_Q + TILE, &tmQ, 0, (qtA + 1) * BM, zq, bar(Q_FULL));
+        tma_load_3d(sb + OFF_Q + TILE + PANEL, &tmQ, 64, (qtA + 1) * BM, zq, bar(Q_FULL));
+      }
+      bool ok = true, kiss[2] = {false, false}, viss = false;
+      uint32_t kpar[2] = {0, 0}, vpar = 0;
+      for (int i = 0; i < n && ok; ++i) {
         const int st = i & 1;
         const uint32_t ph = (i >> 1) & 1;
-        if (!mbar_wait(bar(KV_EMPTY + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
+        if (!mbar_wait(bar(K_EMPTY + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
           ok = false;
           break;
         }
-        const uint32_t sk = sb + OFF_K + st * TILE, sv = sb + OFF_V + st * TILE;
+        const uint32_t sk = sb + OFF_K + st * TILE;
         mbar_arrive_expect_tx(bar(K_FULL + st), TILE);
         tma_load_3d(sk, &tmK, 0, i * BN, zk, bar(K_FULL + st));
         tma_load_3d(sk + PANEL, &tmK, 64, i * BN, zk, bar(K_FULL + st));
-        mbar_arrive_expect_tx(bar(V_FULL + st), TILE);
-        tma_load_3d(sv, &tmV, i * BN, 0, zk, bar(V_FULL + st));
-        tma_load_3d(sv + PANEL, &tmV, i * BN + 64, 0, zk, bar(V_FULL + st));
-        issued[st] = true;
-        par[st] = ph;
+        kiss[st] = true;
+        kpar[st] = ph;
+        if (!mbar_wait(bar(V_EMPTY), (i & 1) ^ 1u, kWaitLimitNs) || misc[1]) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(bar(V_FULL), TILE);
+        tma_load_3d(sb + OFF_V, &tmV, i * BN, 0, zk, bar(V_FULL));
+        tma_load_3d(sb + OFF_V + PANEL, &tmV, i * BN + 64, 0, zk, bar(V_FULL));
+        viss = true;
+        vpar = i & 1;
       }
       if (!ok) {   // let copies still in flight land before the CTA can exit
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_PRODUCER);
         mbar_wait(bar(Q_FULL), 0, 100000000ull);
         for (int s = 0; s < 2; ++s)
-          if (issued[s]) {
-            mbar_wait(bar(K_FULL + s), par[s], 100000000ull);
-            mbar_wait(bar(V_FULL + s), par[s], 100000000ull);
-          }
+          if (kiss[s]) mbar_wait(bar(K_FULL + s), kpar[s], 100000000ull);
+        if (viss) mbar_wait(bar(V_FULL), vpar, 100000000ull);
       }
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
     if (lane == 0) {
       bool ok = mbar_wait(bar(Q_FULL), 0, kWaitLimitNs) && !misc[1];
-      tc_fence_after();
-      auto pv = [&](int j) -> bool {   // O += P_j V_j
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        if (!mbar_wait(bar(V_FULL + st), ph, kWaitLimitNs) ||
-            !mbar_wait(bar(P_FULL), j & 1, kWaitLimitNs) || misc[1])
-          return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t ad = sw128_desc(sb + OFF_P + (kk >> 2) * PANEL) + 2u * (kk & 3);
-          const uint64_t bd = sw128_desc(sb + OFF_V + st * TILE + (kk >> 2) * PANEL) + 2u * (kk & 3);
-          umma_bf16(tO, ad, bd, IDESC, (j > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(bar(O_DONE));
-        umma_commit(bar(KV_EMPTY + st));
-        return true;
+      auto wait = [&](int id, uint32_t par) {
+        ok = ok && mbar_wait(bar(id), par, kWaitLimitNs) && !misc[1];
+        return ok;
       };
-      for (int i = 0; i < n && ok; ++i) {
-        const int st = i & 1;
-        const uint32_t ph = (i >> 1) & 1;
-        if (!mbar_wait(bar(K_FULL + st), ph, kWaitLimitNs) ||
-            !mbar_wait(bar(S_FREE + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
-          ok = false;
-          break;
-        }
+      auto issue_s = [&](int x, int i) {   // S_x(i) = Q_x K_i^T over the head dimension
         tc_fence_after();
-        const uint32_t tS = tbase + st * 128;
+        const uint32_t qx = sb + OFF_Q + x * TILE, kx = sb + OFF_K + (i & 1) * TILE;
 #pragma unroll
-        for (int kk = 0; kk < 128 / 16; ++kk) {   // S_i = Q K_i^T over the head dimension
-          const uint64_t ad = sw128_desc(sb + OFF_Q + (kk >> 2) * PANEL) + 2u * (kk & 3);
-          const uint64_t bd = sw128_desc(sb + OFF_K + st * TILE + (kk >> 2) * PANEL) + 2u * (kk & 3);
-          umma_bf16(tS, ad, bd, IDESC, kk > 0 ? 1u : 0u);
-        }
-        umma_commit(bar(S_FULL + st));
-        if (i >= 1 && !pv(i - 1)) ok = false;
+        for (int kk = 0; kk < 128 / 16; ++kk)
+          umma_bf16(tS(x), sw128_desc(qx + (kk >> 2) * PANEL) + 2u * (kk & 3),
+                    sw128_desc(kx + (kk >> 2) * PANEL) + 2u * (kk & 3), IDESC, kk > 0 ? 1u : 0u);
+        umma_commit(bar(S_FULL + x));
+      };
+      auto issue_pv = [&](int x, int i) {   // O_x += P_x(i) V_i
+        tc_fence_after();
+        const uint32_t px = sb + OFF_P + x * TILE;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk)
+          umma_bf16(tO(x), sw128_desc(px + (kk >> 2) * PANEL) + 2u * (kk & 3),
+                    sw128_desc(sb + OFF_V + (kk >> 2) * PANEL) + 2u * (kk & 3), IDESC,
+                    (i > 0 || kk > 0) ? 1u : 0u);
+      };
+      if (wait(K_FULL, 0)) {
+        issue_s(0, 0);
+        if (hasB) issue_s(1, 0);
+        umma_commit(bar(K_EMPTY));
       }
-      if (ok) ok = pv(n - 1);
+      for (int i = 0; i < n && ok; ++i) {
+        const int nst = (i + 1) & 1;
+        const uint32_t nph = ((i + 1) >> 1) & 1;
+        bool k_next = false;
+        if (!wait(V_FULL, i & 1)) break;
+        if (i < nA) {
+          if (!wait(P_FULL + 0, i & 1)) break;
+          issue_pv(0, i);
+          if (i + 1 < nA) {
+            if (!wait(K_FULL + nst, nph)) break;
+            k_next = true;
+            issue_s(0, i + 1);
+          }
+        }
+        if (i < nB) {
+          if (!wait(P_FULL + 1, i & 1)) break;
+          issue_pv(1, i);
+        }
+        umma_commit(bar(V_EMPTY));   // V_i read by both tiles' P V
+        if (i + 1 < n) {
+          if (!k_next && !wait(K_FULL + nst, nph)) break;
+          if (i + 1 < nB) issue_s(1, i + 1);
+          umma_commit(bar(K_EMPTY + nst));
+        }
+      }
+      if (ok) umma_commit(bar(FINAL));   // every MMA of the CTA has completed
       if (!ok) {
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_MMA);
-        umma_commit(bar(DRAIN));   // completes once every issued MMA has finished
+        umma_commit(bar(DRAIN));
         if (!mbar_wait(bar(DRAIN), 0, 100000000ull)) atomicOr(err, ERR_WAIT_DRAIN);
       }
     }
   } else {
     // ------------------------------ softmax ------------------------------
+    const int x = (warp - 2) >> 2;              // 0: tile A, 1: tile B
     const int quad = warp & 3;                  // TMEM lane quadrant of this warp
-    const int half = (warp - 2) >> 2;           // keys / O columns [64 half, 64 half + 64)
     const int r = quad * 32 + lane;             // query row in the tile
-    const int qpos = q0 + r;
+    const int nx = x ? nB : nA;
+    const int qpos = (qtA + x) * BM + r;
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    float* red = reinterpret_cast<float*>(smem + OFF_RED);     // [2][2][128]
-    float* lsum = reinterpret_cast<float*>(smem + OFF_LSUM);   // [2][128]
-    auto pair_sync = [&]() {   // the two warps of this quadrant (named barrier 1 + quad)
-      asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
-    };
     float m_used = -INFINITY, l = 0.f;          // m_used in raw score units
-    // The two warps of a quadrant meet at a named barrier once per tile and once at
-    // the end, whatever happens: a warp whose wait expired keeps stepping through the
-    // loop without touching TMEM, so neither can be left waiting at the barrier.
     bool ok = true;
-    for (int i = 0; i < n; ++i) {
-      const int st = i & 1;
-      const uint32_t ph = (i >> 1) & 1;
-      if (ok) {
-        bool w = mbar_wait(bar(S_FULL + st), ph, kWaitLimitNs);
-        w = __all_sync(0xffffffffu, w) && !misc[1];
-        ok = __all_sync(0xffffffffu, w);
+    for (int i = 0; i < nx; ++i) {
+      bool w = mbar_wait(bar(S_FULL + x), i & 1, kWaitLimitNs);
+      w = __all_sync(0xffffffffu, w) && !misc[1];
+      if (!__all_sync(0xffffffffu, w)) {
+        ok = false;
+        break;
       }
-      float sv[HALF];
-      if (ok) {
-        tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < HALF / 32; ++c) {
-          uint32_t rr[32];
-          tmem_ld32(tbase + st * 128 + lane_off + half * HALF + c * 32, rr);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) sv[c * 32 + e] = __uint_as_float(rr[e]);
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(S_FREE + st));   // S_{i+2} may overwrite it
-      } else {
-#pragma unroll
-        for (int c = 0; c < HALF; ++c) sv[c] = 0.f;
-      }
-      if (i == n - 1) {   // the diagonal tile: causal mask and the sequence end
-        const int k0 = i * BN + half * HALF;
-#pragma unroll
-        for (int c = 0; c < HALF; ++c)
-          if (k0 + c > qpos || k0 + c >= S) sv[c] = -INFINITY;
-      }
+      tc_fence_after();
+      // the row of S in one TMEM load; p = 2^(s scale - m) streamed into the P tile
+      const bool diag = i == nx - 1;   // the diagonal tile: causal mask and the sequence end
+      const int kvalid = min(qpos + 1, S) - i * BN;   // keys c < kvalid are visible
+      uint32_t rr[BN];
+      tmem_ld128(tS(x) + lane_off, rr);
       float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int c = 0; c < HALF; ++c) m4[c & 3] = fmaxf(m4[c & 3], sv[c]);
-      red[(st * 2 + half) * 128 + r] = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-      pair_sync();
-      if (!ok) continue;
-      const float mx = fmaxf(red[(st * 2) * 128 + r], red[(st * 2 + 1) * 128 + r]);
+      for (int c = 0; c < BN; ++c) {
+        if (diag && c >= kvalid) rr[c] = 0xff800000u;   // -inf
+        m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(rr[c]));
+      }
+      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       float alpha = 1.f;
       if ((mx - m_used) * scale_log2 > RESCALE) {   // raise the running max (first tile: always)
         alpha = exp2f((m_used - mx) * scale_log2);
@@ -486,71 +490,65 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
         l *= alpha;
       }
       const float mb = -m_used * scale_log2;
-      uint32_t pk[HALF / 2];
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
+      // S(i) completing implies P V(i - 1) has: P and O are free
 #pragma unroll
-      for (int c = 0; c < HALF / 2; ++c) {
-        const float p0 = exp2f(fmaf(sv[2 * c], scale_log2, mb));
-        const float p1 = exp2f(fmaf(sv[2 * c + 1], scale_log2, mb));
-        ps[c & 3] += p0 + p1;
-        pk[c] = pack_bf16x2(p0, p1);
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const float p0 = exp2f(fmaf(__uint_as_float(rr[32 * c + 2 * e]), scale_log2, mb));
+          const float p1 = exp2f(fmaf(__uint_as_float(rr[32 * c + 2 * e + 1]), scale_log2, mb));
+          ps[e & 3] += p0 + p1;
+          pk[e] = pack_bf16x2(p0, p1);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {   // 16-byte chunk ch = 4 c + q of the row, 128-byte swizzle
+          const int ch = 4 * c + q;
+          const uint32_t off = OFF_P + x * TILE + (ch >> 3) * PANEL + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+          *reinterpret_cast<uint4*>(smem + off) = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
       }
       l += (ps[0] + ps[1]) + (ps[2] + ps[3]);
-      if (i >= 1) {   // the P buffer and O are free once PV_{i-1} has completed
-        const bool w = mbar_wait(bar(O_DONE), (i - 1) & 1, kWaitLimitNs);
-        if (!__all_sync(0xffffffffu, w)) {
-          ok = false;
-          continue;
-        }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, alpha != 1.f)) {   // rescale this warp's half of O
+      if (i >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {   // rescale this warp's rows of O
 #pragma unroll 1
-          for (int c = 0; c < HALF / 32; ++c) {
-            uint32_t rr[32];
-            tmem_ld32(tO + lane_off + half * HALF + c * 32, rr);
+        for (int c = 0; c < 4; ++c) {
+          uint32_t rr[32];
+          tmem_ld32(tO(x) + lane_off + c * 32, rr);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
-            tmem_st32(tO + lane_off + half * HALF + c * 32, rr);
-          }
+          for (int e = 0; e < 32; ++e) rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
+          tmem_st32(tO(x) + lane_off + c * 32, rr);
         }
-      }
-#pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {   // this half's panel of P, 128-byte swizzle
-        const uint32_t off = OFF_P + half * PANEL + r * 128 + ((ch ^ (r & 7)) << 4);
-        *reinterpret_cast<uint4*>(smem + off) =
-            make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
       }
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(P_FULL));
+      if (lane == 0) mbar_arrive(bar(P_FULL + x));
     }
-    if (ok) {
-      const bool w = mbar_wait(bar(O_DONE), (n - 1) & 1, kWaitLimitNs);
+    if (ok && nx > 0) {
+      const bool w = mbar_wait(bar(FINAL), 0, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, w);
-    }
-    // both halves of a row reach this exchange (a warp that gave up passes l = 0)
-    lsum[half * 128 + r] = l;
-    pair_sync();
-    if (ok) {
-      tc_fence_after();
-      const float inv = 1.f / (lsum[r] + lsum[128 + r]);
-      uint16_t* orow = O + ((size_t)b * S + qpos) * H * 128 + hh * 128 + half * HALF;
+      if (ok) {
+        tc_fence_after();
+        const float inv = 1.f / l;
+        uint16_t* orow = O + ((size_t)b * S + qpos) * H * 128 + hh * 128;
 #pragma unroll 1
-      for (int c = 0; c < HALF / 32; ++c) {
-        uint32_t rr[32];
-        tmem_ld32(tO + lane_off + half * HALF + c * 32, rr);
-        if (qpos < S) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+        for (int c = 0; c < 4; ++c) {
+          uint32_t rr[32];
+          tmem_ld32(tO(x) + lane_off + c * 32, rr);
+          if (qpos < S) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            dst[q] = make_uint4(pack_bf16x2(__uint_as_float(rr[8 * q]) * inv, __uint_as_float(rr[8 * q + 1]) * inv),
-                                pack_bf16x2(__uint_as_float(rr[8 * q + 2]) * inv, __uint_as_float(rr[8 * q + 3]) * inv),
-                                pack_bf16x2(__uint_as_float(rr[8 * q + 4]) * inv, __uint_as_float(rr[8 * q + 5]) * inv),
-                                pack_bf16x2(__uint_as_float(rr[8 * q + 6]) * inv, __uint_as_float(rr[8 * q + 7]) * inv));
+            for (int q = 0; q < 4; ++q)
+              dst[q] = make_uint4(pack_bf16x2(__uint_as_float(rr[8 * q]) * inv, __uint_as_float(rr[8 * q + 1]) * inv),
+                                  pack_bf16x2(__uint_as_float(rr[8 * q + 2]) * inv, __uint_as_float(rr[8 * q + 3]) * inv),
+                                  pack_bf16x2(__uint_as_float(rr[8 * q + 4]) * inv, __uint_as_float(rr[8 * q + 5]) * inv),
+                                  pack_bf16x2(__uint_as_float(rr[8 * q + 6]) * inv, __uint_as_float(rr[8 * q + 7]) * inv));
+          }
         }
       }
-    } else if (lane == 0) {
+    }
+    if (!ok && lane == 0) {
       misc[1] = 1;
       atomicOr(err, ERR_WAIT_EPILOGUE);
     }
@@ -830,9 +828,10 @@ cudaError_t launch_flash_tc(const CUtensorMap& tmQ, const CUtensorMap& tmK, cons
     attr = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
-  const dim3 grid((unsigned)((S + fa::BM - 1) / fa::BM), (unsigned)H, (unsigned)B);
+  const int n_qt = (S + fa::BM - 1) / fa::BM;
+  const dim3 grid((unsigned)((n_qt + 1) / 2), (unsigned)H, (unsigned)B);   // query tile pairs
   return launch_pdl(k_flash_tc, grid, dim3(fa::THREADS), fa::SMEM, st, tmQ, tmK, tmV, H, Hkv, S,
-                    scale_log2, static_cast<uint16_t*>(O), err);
+                    n_qt, scale_log2, static_cast<uint16_t*>(O), err);
 }
 
 }  // namespace hero
