@@ -532,19 +532,16 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
         tc_fence_after();
         const float inv = 1.f / l;
         uint16_t* orow = O + ((size_t)b * S + qpos) * H * 128 + hh * 128;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t rr[32];
-          tmem_ld32(tO(x) + lane_off + c * 32, rr);
-          if (qpos < S) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+        uint32_t rr[128];
+        tmem_ld128(tO(x) + lane_off, rr);
+        if (qpos < S) {
+          uint4* dst = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-              dst[q] = make_uint4(pack_bf16x2(__uint_as_float(rr[8 * q]) * inv, __uint_as_float(rr[8 * q + 1]) * inv),
-                                  pack_bf16x2(__uint_as_float(rr[8 * q + 2]) * inv, __uint_as_float(rr[8 * q + 3]) * inv),
-                                  pack_bf16x2(__uint_as_float(rr[8 * q + 4]) * inv, __uint_as_float(rr[8 * q + 5]) * inv),
-                                  pack_bf16x2(__uint_as_float(rr[8 * q + 6]) * inv, __uint_as_float(rr[8 * q + 7]) * inv));
-          }
+          for (int q = 0; q < 16; ++q)
+            dst[q] = make_uint4(pack_bf16x2(__uint_as_float(rr[8 * q]) * inv, __uint_as_float(rr[8 * q + 1]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 2]) * inv, __uint_as_float(rr[8 * q + 3]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 4]) * inv, __uint_as_float(rr[8 * q + 5]) * inv),
+                                pack_bf16x2(__uint_as_float(rr[8 * q + 6]) * inv, __uint_as_float(rr[8 * q + 7]) * inv));
         }
       }
     }
