@@ -562,10 +562,10 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
 // Decoding step attention (flash-decoding): one query per sequence, the G = H / H_kv
 // query heads of a key/value head together, keys split into chunks of DC positions
 // so that every SM streams the cache.  CTA = (chunk, kv head, sequence), 128 threads:
-//   1. scores: warp w takes keys 64 w .. 64 w + 63; each load instruction covers two
-//      whole 256-byte key rows (lane: row 2 i + lane / 16, 16-byte chunk lane % 16,
-//      16 loads in flight), lanes multiply by the G queries' matching 8 elements (held
-//      in registers) and the 16 lanes of a row add up by shuffles;
+//   1. scores: warp w takes keys 64 w .. 64 w + 63; eight lanes share a 256-byte key
+//      row (lane: row 4 i + lane / 8, 16-byte chunks lane % 8 and lane % 8 + 8; 16 loads
+//      in flight), multiply by the G queries' matching 16 elements (held in registers)
+//      and add up over the eight lanes by shuffles;
 //   2. per query head (one warp each): chunk max m, p = 2^(s - m), l = sum p;
 //   3. P V: thread t owns value columns 8 (t % 16) .. +7 of keys t / 16 + 8 i
 //      (16-byte loads, 16 in flight), the 8 key groups added in shared memory.
@@ -607,47 +607,61 @@ __global__ void __launch_bounds__(DEC_THREADS) k_attn_decode(const uint16_t* __r
   }
   const uint16_t* Kg = K + ((size_t)b * Hkv + kvh) * kv_stride * HD;
   const uint16_t* Vg = V + ((size_t)b * Hkv + kvh) * kv_stride * HD;
-  const int ch = lane & 15;   // this lane's 16-byte chunk (elements 8 ch .. 8 ch + 7)
-  float qr[G][8];
+  const int ch = lane & 7;   // this lane's 16-byte chunks ch and ch + 8 (elements 8 ch.., 64 + 8 ch..)
+  float qr[G][16];
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    const uint4 u = *reinterpret_cast<const uint4*>(Q + ((size_t)b * H + kvh * G + g) * HD + ch * 8);
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  for (int g = 0; g < G; ++g)
 #pragma unroll
-    for (int h2 = 0; h2 < 4; ++h2) {
-      unpack_bf16x2(w[h2], qr[g][2 * h2], qr[g][2 * h2 + 1]);
-      qr[g][2 * h2] *= scale_log2;
-      qr[g][2 * h2 + 1] *= scale_log2;
+    for (int hlf = 0; hlf < 2; ++hlf) {
+      const uint4 u = *reinterpret_cast<const uint4*>(Q + ((size_t)b * H + kvh * G + g) * HD +
+                                                      (ch + 8 * hlf) * 8);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int h2 = 0; h2 < 4; ++h2) {
+        unpack_bf16x2(w[h2], qr[g][8 * hlf + 2 * h2], qr[g][8 * hlf + 2 * h2 + 1]);
+        qr[g][8 * hlf + 2 * h2] *= scale_log2;
+        qr[g][8 * hlf + 2 * h2 + 1] *= scale_log2;
+      }
     }
-  }
   const int kw0 = warp * DEC_KPW;   // the warp's first key (offset in the chunk)
 #pragma unroll 1
-  for (int half = 0; half < DEC_KPW / 32; ++half) {
-    uint4 kr[16];
+  for (int blk = 0; blk < DEC_KPW / 32; ++blk) {
+    // 8 lanes per key row, 4 rows per instruction pair; 16 loads of 16 bytes in flight
+    uint4 kr[8][2];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const int j = j0 + kw0 + half * 32 + 2 * i + (lane >> 4);
-      kr[i] = j < j1 ? __ldg(reinterpret_cast<const uint4*>(Kg + (size_t)j * HD + ch * 8))
-                     : make_uint4(0u, 0u, 0u, 0u);
+    for (int i = 0; i < 8; ++i) {
+      const int j = j0 + kw0 + blk * 32 + 4 * i + (lane >> 3);
+#pragma unroll
+      for (int hlf = 0; hlf < 2; ++hlf)
+        kr[i][hlf] = j < j1 ? __ldg(reinterpret_cast<const uint4*>(Kg + (size_t)j * HD + (ch + 8 * hlf) * 8))
+                            : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      float k8[8];
-      const uint32_t w[4] = {kr[i].x, kr[i].y, kr[i].z, kr[i].w};
+    for (int i = 0; i < 8; ++i) {
+      float k16[16];
 #pragma unroll
-      for (int h2 = 0; h2 < 4; ++h2) unpack_bf16x2(w[h2], k8[2 * h2], k8[2 * h2 + 1]);
+      for (int hlf = 0; hlf < 2; ++hlf) {
+        const uint32_t w[4] = {kr[i][hlf].x, kr[i][hlf].y, kr[i][hlf].z, kr[i][hlf].w};
+#pragma unroll
+        for (int h2 = 0; h2 < 4; ++h2)
+          unpack_bf16x2(w[h2], k16[8 * hlf + 2 * h2], k16[8 * hlf + 2 * h2 + 1]);
+      }
       float acc[G];
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float a = 0.f;
+        float a0 = 0.f, a1 = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) a += qr[g][e] * k8[e];
+        for (int e = 0; e < 16; e += 2) {
+          a0 = fmaf(qr[g][e], k16[e], a0);
+          a1 = fmaf(qr[g][e + 1], k16[e + 1], a1);
+        }
+        float a = a0 + a1;
 #pragma unroll
-        for (int o = 8; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+        for (int o = 4; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
         acc[g] = a;
       }
       if (ch == 0) {
-        const int r = kw0 + half * 32 + 2 * i + (lane >> 4);
+        const int r = kw0 + blk * 32 + 4 * i + (lane >> 3);
 #pragma unroll
         for (int g = 0; g < G; ++g) sc[g][r] = j0 + r < j1 ? acc[g] : -INFINITY;
       }
