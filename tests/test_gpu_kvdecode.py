@@ -247,3 +247,62 @@ def test_decode_full_size(hero):
     assert gerr < pr.free_run_gate_bound("llama31_8b_prefill") and herr < H_TOL
     dec.close()
     torch.cuda.empty_cache()
+
+
+def test_host_io_and_graph_capture(small, hero):
+    """The decoder forward and a decoding step through host buffers (HERO_FLAG_HOST_IO)
+    equal the device-buffer calls bit for bit, and a decoding step captured in a CUDA
+    graph replays to the eager result (device-resident positions: no host sync)."""
+    import torch
+    cfg, w, wa, dec = small
+    B, S, d, L = 3, 40, cfg.d_model, cfg.n_layers
+    tau = hi.calibrated_tau(cfg.name)
+    h0 = hi.generate_h_in(cfg.replace(n_tokens=B * S, seed=9))
+    ref = dec.forward(_dev(h0), tau, B, S)
+    torch.cuda.synchronize()
+    hp = torch.from_numpy(h0).pin_memory()
+    ho_ = torch.empty((B * S, d)).pin_memory()
+    gp = torch.empty((L, B * S)).pin_memory()
+    mp = torch.empty((L, B * S), dtype=torch.uint8).pin_memory()
+    cp = torch.empty((L,), dtype=torch.int32).pin_memory()
+    stream = torch.cuda.current_stream().cuda_stream
+    hero.hero_decoder_forward(dec.model, B, S, hp.data_ptr(), tau, hero.HERO_FLAG_HOST_IO, 0,
+                              ho_.data_ptr(), gp.data_ptr(), mp.data_ptr(), cp.data_ptr(), stream)
+    torch.cuda.synchronize()
+    dec.check()
+    assert torch.equal(ho_, ref[0].cpu()) and torch.equal(gp, ref[1].cpu()) and torch.equal(mp, ref[2].cpu())
+    assert torch.equal(cp, ref[3].cpu())
+    # a prefill, then the same step through device buffers, host buffers and a graph
+    dec.prefill(_dev(h0), tau, 0, B, S)
+    hn = hi.generate_h_in(cfg.replace(n_tokens=B, seed=31))
+    pos = np.array([40, 12, 39], dtype=np.int32)
+    outs = [torch.empty((B, d), device="cuda"), torch.empty((L, B), device="cuda"),
+            torch.empty((L, B), dtype=torch.uint8, device="cuda"),
+            torch.empty((L,), dtype=torch.int32, device="cuda")]
+    hn_d, pos_d = _dev(hn), _dev(pos)
+    dec.decode(hn_d, pos_d, 40, tau, h_out=outs[0], gate_out=outs[1], mask_out=outs[2],
+               counts_out=outs[3])
+    torch.cuda.synchronize()
+    eager = [o.clone() for o in outs]
+    hp2 = torch.from_numpy(hn).pin_memory()
+    pp = torch.from_numpy(pos).pin_memory()
+    ho2 = torch.empty((B, d)).pin_memory()
+    cp2 = torch.empty((L,), dtype=torch.int32).pin_memory()
+    hero.hero_decode_step(dec.model, B, pp.data_ptr(), 40, hp2.data_ptr(), tau, hero.HERO_FLAG_HOST_IO,
+                          0, ho2.data_ptr(), 0, 0, cp2.data_ptr(), stream)
+    torch.cuda.synchronize()
+    assert torch.equal(ho2, eager[0].cpu()) and torch.equal(cp2, eager[3].cpu())
+    for o in outs:
+        o.zero_()
+    graph = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.graph(graph, stream=cap):
+        dec.decode(hn_d, pos_d, 40, tau, h_out=outs[0], gate_out=outs[1], mask_out=outs[2],
+                   counts_out=outs[3], stream=cap)
+    torch.cuda.current_stream().wait_stream(cap)
+    graph.replay()
+    torch.cuda.synchronize()
+    dec.check()
+    for a_, b_ in zip(outs, eager):
+        assert torch.equal(a_, b_)
