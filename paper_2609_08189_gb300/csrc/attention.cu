@@ -276,6 +276,12 @@ __global__ void __launch_bounds__(FA_THREADS) k_flash_attn(const uint16_t* __res
 // the q/k/v epilogue) in 128 x 64 bf16 panels.  Every mbarrier wait is bounded; on expiry
 // the CTA drains its copies and MMAs, reports through err and frees its TMEM.
 // ---------------------------------------------------------------------------------
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 namespace fa {
 constexpr int BM = 128, BN = 128, THREADS = 320;
 constexpr uint32_t PANEL = 128 * 128;   // [128 rows][64 bf16] = 16 KB
@@ -476,12 +482,17 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
       const int kvalid = min(qpos + 1, S) - i * BN;   // keys c < kvalid are visible
       uint32_t rr[BN];
       tmem_ld128(tS(x) + lane_off, rr);
+      if (diag) {
+#pragma unroll
+        for (int c = 0; c < BN; ++c)
+          if (c >= kvalid) rr[c] = 0xff800000u;   // -inf
+      }
       float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int c = 0; c < BN; ++c) {
-        if (diag && c >= kvalid) rr[c] = 0xff800000u;   // -inf
-        m4[c & 3] = fmaxf(m4[c & 3], __uint_as_float(rr[c]));
-      }
+      for (int c = 0; c < BN; c += 8)   // three-input max: two new values per instruction
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          m4[k] = fmax3(m4[k], __uint_as_float(rr[c + 2 * k]), __uint_as_float(rr[c + 2 * k + 1]));
       const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       float alpha = 1.f;
       if ((mx - m_used) * scale_log2 > RESCALE) {   // raise the running max (first tile: always)
