@@ -122,7 +122,10 @@ __global__ void __launch_bounds__(256) k_state_reset(float* S, float* zeta, floa
 // GPU twice over (decode and short prefill), where the per-CTA chain of dependent
 // phases is the critical path and the head matmuls split K more widely.
 constexpr int TB_LARGE = 16, TB_SMALL = 4;
-constexpr int NTHR = 256;
+// Threads per CTA: 256 with 16 tokens; 1024 with 4 tokens, where each phase's split-K
+// and per-token reductions spread over four times the threads to shorten the chain.
+template <int TB>
+constexpr int nthr() { return TB < 16 ? 1024 : 256; }
 
 // Shared-memory layout (floats), computed from the model's widths on host and
 // device alike.  Regions are reused once their contents are dead:
@@ -136,7 +139,7 @@ struct RouterLayout {
   int big, s, qkv, aux, x, ph, red, sc, ab, sk, floats;
   // sk: split-K scratch of q/k/v and f_theta (small TB only; with TB = 16 those
   // products have enough output tiles to occupy every thread without a split)
-  static constexpr int kSplitScratch = TB < 16 ? 4096 : 0;
+  static constexpr int kSplitScratch = TB < 16 ? 16384 : 0;
   __host__ __device__ RouterLayout(int d_enc, int d_head, int ds, int dm, int d_path) {
     const int nbig = (d_enc > d_head ? d_enc : d_head) * TB;
     const int ns = ((ds + dm + 1 + 3) & ~3) * TB;
@@ -148,7 +151,7 @@ struct RouterLayout {
     x = aux + naux;
     ph = x + 8 * TB;
     red = ph + d_path * TB;
-    sc = red + 3 * NTHR;
+    sc = red + 3 * nthr<TB>();
     ab = sc + TB * 16;
     sk = ab + 2 * TB;
     floats = sk + kSplitScratch;
@@ -169,10 +172,12 @@ __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int 
   const int base = no4 * (TB / 4);
   int ks = 1;
   if (scratch)
-    while (base * ks * 2 <= NTHR && NI / (ks * 2) >= 16 && (ks * 2) * NO * TB <= scratch_cap) ks <<= 1;
+    while (base * ks * 2 <= nthr<TB>() && NI / (ks * 2) >= (TB < 16 ? 8 : 16) &&
+           (ks * 2) * NO * TB <= scratch_cap)
+      ks <<= 1;
   const int kchunk = (NI + ks - 1) / ks;
   auto oidx = [&](int o, int t) { return out_tok_ld > 0 ? t * out_tok_ld + o : o * TB + t; };
-  for (int w = threadIdx.x; w < base * ks; w += NTHR) {
+  for (int w = threadIdx.x; w < base * ks; w += nthr<TB>()) {
     const int o4 = (w % no4) * 4;
     const int rest = w / no4;
     const int t4 = (rest % (TB / 4)) * 4;
@@ -209,7 +214,7 @@ __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int 
   }
   __syncthreads();
   if (ks > 1) {
-    for (int e = threadIdx.x; e < NO * TB; e += NTHR) {
+    for (int e = threadIdx.x; e < NO * TB; e += nthr<TB>()) {
       const int o = e / TB, t = e % TB;
       float v = 0.f;
       for (int kk = 0; kk < ks; ++kk) v += scratch[(kk * NO + o) * TB + t];
@@ -229,7 +234,7 @@ __device__ __forceinline__ float warp_part_sum(float v) {
   return v;
 }
 
-// Sum the NTHR / TB per-thread partials of each token (thread tid holds a partial of
+// Sum the nthr<TB>() / TB per-thread partials of each token (thread tid holds a partial of
 // token tid % TB): a shuffle tree inside each warp, then the warps' sums in warp
 // order (fixed, so bitwise reproducible); contains __syncthreads.
 template <int TB>
@@ -240,7 +245,7 @@ __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
   __syncthreads();
   if (threadIdx.x < TB) {
     float s = 0.f;
-    for (int w = 0; w < NTHR / 32; ++w) s += red[w * TB + threadIdx.x];
+    for (int w = 0; w < nthr<TB>() / 32; ++w) s += red[w * TB + threadIdx.x];
     out[threadIdx.x] = s;
   }
   __syncthreads();
@@ -256,7 +261,7 @@ __device__ __forceinline__ void reduce16(float* red, float v, float* out) {
 template <int DM, int TB>
 __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const float* qkv, float* cT,
                                                   int t0, int warp, int lane) {
-  for (int tl = warp; tl < TB; tl += NTHR / 32) {
+  for (int tl = warp; tl < TB; tl += nthr<TB>() / 32) {
     const int t = t0 + tl;
     if (t >= a.T) continue;
     const float* q = qkv + tl * 3 * DM;
@@ -356,7 +361,7 @@ __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const flo
 }
 
 template <int DM, int TB>
-__global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const RouterArgs a) {
+__global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_router(const RouterArgs a) {
   pdl_enter();
   extern __shared__ __align__(16) float sm[];
   const int ds = a.d_h + a.d_a;
@@ -390,8 +395,8 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
                    : "memory");
   }
 
-  // Thread tid serves token tl = tid % TB as part pt = tid / TB of 16 in the two
-  // input phases; the 16 parts of a token are added in a fixed order.
+  // Thread tid serves token tl = tid % TB as part pt = tid / TB of nthr / TB in the
+  // two input phases; the parts of a token are added in a fixed order.
   const int tl0 = tid % TB, pt0 = tid / TB;
   const int tok0 = t0 + tl0;
 
@@ -400,7 +405,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
   {
     float ss = 0.f, dd = 0.f, dp = 0.f;
     if (tok0 < a.T)
-      for (int s = pt0; s < a.np; s += NTHR / TB) {
+      for (int s = pt0; s < a.np; s += nthr<TB>() / TB) {
         const float4 v = *reinterpret_cast<const float4*>(a.part + ((size_t)tok0 * a.np + s) * 4);
         ss += v.x;
         dd += v.y;
@@ -411,18 +416,18 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
     dp = warp_part_sum<TB>(dp);
     if (lane < TB) {
       red[warp * TB + lane] = ss;
-      red[NTHR + warp * TB + lane] = dd;
-      red[2 * NTHR + warp * TB + lane] = dp;
+      red[nthr<TB>() + warp * TB + lane] = dd;
+      red[2 * nthr<TB>() + warp * TB + lane] = dp;
     }
   }
   __syncthreads();
   if (tid < TB) {
     const int t = t0 + tid;
     float ss = 0.f, dd = 0.f, dp = 0.f, dprev = 0.f, pp = 1.f, mp = 1.f;
-    for (int w = 0; w < NTHR / 32; ++w) {
+    for (int w = 0; w < nthr<TB>() / 32; ++w) {
       ss += red[w * TB + tid];
-      dd += red[NTHR + w * TB + tid];
-      dp += red[2 * NTHR + w * TB + tid];
+      dd += red[nthr<TB>() + w * TB + tid];
+      dp += red[2 * nthr<TB>() + w * TB + tid];
     }
     if (t < a.T) {
       dprev = a.dprev[t];
@@ -457,11 +462,11 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
     const int ng = nY >> 2;
     const float rinv = sc[tl0 * 16];
     const float4* yrow = reinterpret_cast<const float4*>(a.Y + (size_t)tok0 * nY);
-    for (int g0 = pt0; g0 < ng; g0 += YB * (NTHR / TB)) {
+    for (int g0 = pt0; g0 < ng; g0 += YB * (nthr<TB>() / TB)) {
       float4 yv[YB];
 #pragma unroll
       for (int k = 0; k < YB; ++k) {
-        const int g = g0 + k * (NTHR / TB);
+        const int g = g0 + k * (nthr<TB>() / TB);
         yv[k] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (tok0 < a.T && g < ng) {
           yv[k] = __ldg(yrow + g);
@@ -473,7 +478,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
       }
 #pragma unroll
       for (int k = 0; k < YB; ++k) {
-        const int g = g0 + k * (NTHR / TB);
+        const int g = g0 + k * (nthr<TB>() / TB);
         if (g >= ng) break;
         const int c = 4 * g;
         const float y4[4] = {yv[k].x, yv[k].y, yv[k].z, yv[k].w};
@@ -509,7 +514,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
   // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s)
   bmm4<TB>(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
   if (a.variant & RV_NO_AUX) {   // ablation: no auxiliary path encoder, z_a = 0
-    for (int e = tid; e < a.d_a * TB; e += NTHR) sT[a.d_h * TB + e] = 0.f;
+    for (int e = tid; e < a.d_a * TB; e += nthr<TB>()) sT[a.d_h * TB + e] = 0.f;
     __syncthreads();
   } else {
     bmm4<TB>(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
@@ -522,7 +527,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
 
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
-    for (int e = tid; e < DM * TB; e += NTHR) sT[ds * TB + e] = 0.f;
+    for (int e = tid; e < DM * TB; e += nthr<TB>()) sT[ds * TB + e] = 0.f;
   } else {
     memory_read_write<DM, TB>(a, qkv, sT + ds * TB, t0, warp, lane);
   }
@@ -539,7 +544,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
     // thread (part, t) sums DM/16 products; fixed-order reduction per token
     const int tl = tid % TB, part = tid / TB;
     float xy = 0.f, xx = 0.f, yy = 0.f;
-    for (int i = part; i < DM; i += NTHR / TB) {
+    for (int i = part; i < DM; i += nthr<TB>() / TB) {
       const float u = nv[i * TB + tl], w = cv[i * TB + tl];
       xy += u * w;
       xx += u * u;
@@ -550,16 +555,16 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
     yy = warp_part_sum<TB>(yy);
     if (lane < TB) {
       red[warp * TB + lane] = xy;
-      red[NTHR + warp * TB + lane] = xx;
-      red[2 * NTHR + warp * TB + lane] = yy;
+      red[nthr<TB>() + warp * TB + lane] = xx;
+      red[2 * nthr<TB>() + warp * TB + lane] = yy;
     }
     __syncthreads();
     if (tid < TB) {
       float sxy = 0.f, sxx = 0.f, syy = 0.f;
-      for (int w = 0; w < NTHR / 32; ++w) {
+      for (int w = 0; w < nthr<TB>() / 32; ++w) {
         sxy += red[w * TB + tid];
-        sxx += red[NTHR + w * TB + tid];
-        syy += red[2 * NTHR + w * TB + tid];
+        sxx += red[nthr<TB>() + w * TB + tid];
+        syy += red[2 * nthr<TB>() + w * TB + tid];
       }
       nuT[tid] = 1.f - sxy / (sqrtf(sxx) * sqrtf(syy) + a.eps);
     }
@@ -576,7 +581,7 @@ __global__ void __launch_bounds__(NTHR, DM >= 256 ? 1 : 4) k_router(const Router
   {
     const int tl = tid % TB, part = tid / TB;
     float sa = 0.f;
-    for (int i = part; i < a.d_head; i += NTHR / TB) sa = fmaf(__ldg(a.w.th_w2 + i), bigT[i * TB + tl], sa);
+    for (int i = part; i < a.d_head; i += nthr<TB>() / TB) sa = fmaf(__ldg(a.w.th_w2 + i), bigT[i * TB + tl], sa);
     reduce16<TB>(red, sa, ab);
   }
 
@@ -793,7 +798,7 @@ static cudaError_t launch_router_tb(const RouterArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr = smem;
   }
-  return launch_pdl(k_router<DM, TB>, dim3((a.T + TB - 1) / TB), dim3(NTHR), smem, st, a);
+  return launch_pdl(k_router<DM, TB>, dim3((a.T + TB - 1) / TB), dim3(nthr<TB>()), smem, st, a);
 }
 
 template <int DM>
