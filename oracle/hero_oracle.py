@@ -453,6 +453,8 @@ def routed_ffn_stack(cfg: OracleConfig, weights: Dict[str, np.ndarray], h_in, at
             m = m_prev * p                                          # Eq. 15
             b = local_head(h_bar, w, Rx)                            # Eq. 16
             g = sigmoid(a + b)
+            if "gate" in hk:                                        # test hook: g override
+                g = hk["gate"](layer, g)
             rho = sigmoid(eta[layer - 1])
             if not cfg.variant & NO_MEMREAD:
                 S, zeta = memory_write(S, zeta, fk, v, rho)         # Eq. 12
@@ -514,3 +516,42 @@ def bypass_fraction(masks: np.ndarray, n_dense: int = 0) -> float:
     sum_j n_a,j / (L_R T), over the routed blocks only (rows n_dense.. of masks)."""
     m = np.asarray(masks)[n_dense:]
     return float(1.0 - m.mean()) if m.size else 0.0
+
+
+# ---------------------------------------------------------------------------
+# Training objective (Sec. 3.3), for gradient checks of the training path
+# ---------------------------------------------------------------------------
+
+# Parameters the training path optimises (Sec. 3.3: the backbone - FFN, its norm gain
+# and attention - is frozen; adapters, state encoders, depth memory and router heads
+# are trained).
+TRAINABLE = ("ad_w1", "ad_w2", "eta", "r_norm_g", "w_hd", "w_hu", "path_w1", "path_b1",
+             "path_w2", "path_b2", "w_q", "w_k", "w_v", "w_n", "w_c", "th_w1", "th_b1",
+             "th_w2", "th_b2", "ps_w1", "ps_b1", "ps_w2", "ps_b2")
+
+
+def skip_penalty(gates, n_seqs: int, seq_len: int, n_dense: int = 0) -> float:
+    """L_skip (Sec. 3.3): for each sequence and each of its seq_len - 1 next-token
+    positions, the square of the token's summed gates over the routed blocks, averaged
+    over B (T - 1).  gates [L, n_seqs seq_len], tokens in sequence order; rows of the
+    dense prefix carry no gate."""
+    g = np.asarray(gates, dtype=np.float64)[n_dense:]
+    g = g.reshape(g.shape[0], n_seqs, seq_len)[:, :, :seq_len - 1]
+    return float(np.sum(np.sum(g, axis=0) ** 2) / (n_seqs * (seq_len - 1)))
+
+
+def training_loss(cfg: OracleConfig, weights, h_in, attn_delta, mask, G, alpha: float,
+                  n_seqs: int, seq_len: int, hooks=None) -> float:
+    """L = <G, h_out> + alpha L_skip with the decisions fixed to mask [L, T]: the
+    threshold of Eq. 3 is not differentiated, the selected branch's scale g or 1 - g
+    carries the gradient to the router (Sec. 3.1).  G [T, d] is a synthetic upstream
+    gradient standing in for dL_LM / dh_out (no language-model head or data)."""
+    out = routed_ffn_stack(cfg, weights, h_in, attn_delta, 0.0, mode="force", mask_in=mask,
+                           hooks=hooks)
+    return float(np.sum(np.asarray(G, dtype=np.float64) * out["h_out"])) + \
+        alpha * skip_penalty(out["gate"], n_seqs, seq_len, cfg.n_dense)
+
+
+def directional_derivative(f: Callable[[float], float], h: float) -> float:
+    """Central difference (f(h) - f(-h)) / 2h of a function of the step along a direction."""
+    return (f(h) - f(-h)) / (2.0 * h)

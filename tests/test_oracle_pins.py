@@ -764,3 +764,92 @@ def test_rope_is_complex_rotation():
     ang = np.arange(S)[:, None] * theta ** (-2.0 * np.arange(hd // 2)[None, :] / hd)
     w = z * np.exp(1j * ang)
     np.testing.assert_allclose(got, np.concatenate([w.real, w.imag], axis=1), rtol=0, atol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# Training objective (Sec. 3.3): the pins a training path's gradients are checked with
+# ---------------------------------------------------------------------------
+
+def test_skip_penalty_gradient_closed_form():
+    """d L_skip / d g_{j,b,t} = 2 / (B (T - 1)) sum_j' g_{j',b,t} for the T - 1
+    next-token positions, 0 at a sequence's last position and for dense-prefix rows."""
+    rng = np.random.default_rng(3)
+    n_dense, L, B, S = 1, 4, 2, 5
+    g = rng.uniform(0.05, 0.95, size=(L, B * S))
+    base = ho.skip_penalty(g, B, S, n_dense)
+    for j in range(L):
+        for t in range(B * S):
+            e = np.zeros_like(g)
+            e[j, t] = 1.0
+            fd = ho.directional_derivative(lambda hh: ho.skip_penalty(g + hh * e, B, S, n_dense), 1e-6)
+            pos = t % S
+            want = 0.0 if (j < n_dense or pos == S - 1) else \
+                2.0 / (B * (S - 1)) * g[n_dense:, t].sum()
+            assert abs(fd - want) < 1e-8, (j, t, fd, want)
+    assert base == pytest.approx(np.sum(g[n_dense:].reshape(L - n_dense, B, S)[:, :, :S - 1].sum(0) ** 2)
+                                 / (B * (S - 1)), rel=1e-15)
+
+
+def _training_inputs():
+    cfg = hi.CONFIGS["tiny_f32"]
+    oc = ho.OracleConfig.from_stack(cfg)
+    w, h, P = hi.generate_weights(cfg), hi.generate_h_in(cfg), hi.generate_attn_delta(cfg)
+    free = ho.routed_ffn_stack(oc, w, h, P, hi.calibrated_tau(cfg.name))
+    G = np.random.default_rng(5).standard_normal(h.shape)
+    return cfg, oc, w, h, P, free["mask"], G
+
+
+def test_last_block_gate_gradient_closed_form():
+    """Eq. 3 with the decision fixed: in the last block g scales only the selected
+    branch, so dL/dg_{L,t} = <G_t, FFN(u_t)> (FFN token) or -<G_t, Adapter(u_t)>
+    (adapter token), plus alpha times L_skip's term - checked against central
+    differences of the whole objective with g_{L,t} perturbed."""
+    cfg, oc, w, h, P, mask, G = _training_inputs()
+    B, S, alpha = 2, 32, 0.3
+    rec = ho.routed_ffn_stack(oc, w, h, P, 0.0, mode="force", mask_in=mask, record=True)
+    u = rec["layers"][-1]["u"]
+    wl = {k: ho._f64(w[k][-1]) for k in ("w_gate", "w_up", "w_down", "ad_w1", "ad_w2")}
+    L = cfg.n_layers
+    ffn_t = int(np.nonzero(mask[-1])[0][0])
+    ad_t = int(np.nonzero(mask[-1] == 0)[0][0])
+    for t in sorted({ffn_t, ad_t, S - 1, S}):
+        def f(hh, t=t):
+            def hook(layer, g):
+                if layer != L:
+                    return g
+                g = g.copy()
+                g[t] += hh
+                return g
+            return ho.training_loss(oc, w, h, P, mask, G, alpha, B, S, hooks={"gate": hook})
+        fd = ho.directional_derivative(f, 1e-5)
+        if mask[-1, t]:
+            branch = ho.swiglu_ffn(u[t:t + 1], wl, ho._identity)[0]
+            want = float(G[t] @ branch)
+        else:
+            branch = ho.adapter(u[t:t + 1], wl, ho._identity)[0]
+            want = -float(G[t] @ branch)
+        if t % S != S - 1:
+            want += alpha * 2.0 / (B * (S - 1)) * float(rec["gate"][:, t].sum())
+        assert abs(fd - want) <= 1e-6 * max(1.0, abs(want)), (t, fd, want)
+
+
+@pytest.mark.parametrize("key", ho.TRAINABLE)
+def test_training_loss_is_smooth_along_each_trainable_tensor(key):
+    """With the decisions fixed the objective is differentiable in every trainable
+    tensor: central differences at h and h/2 agree to the O(h^2) truncation, and the
+    derivative is nonzero (every trained tensor reaches the loss)."""
+    cfg, oc, w, h, P, mask, G = _training_inputs()
+    B, S, alpha = 2, 32, 0.3
+    base = w[key].astype(np.float64)
+    V = np.random.default_rng(100 + ho.TRAINABLE.index(key)).standard_normal(base.shape)
+    scale = max(float(np.sqrt(np.mean(base ** 2))), 1e-3)
+
+    def f(hh):
+        w2 = dict(w)
+        w2[key] = base + hh * scale * V
+        return ho.training_loss(oc, w2, h, P, mask, G, alpha, B, S)
+
+    d1 = ho.directional_derivative(f, 1e-4)
+    d2 = ho.directional_derivative(f, 5e-5)
+    assert abs(d1) > 1e-9, key
+    assert abs(d1 - d2) <= 1e-5 * max(1.0, abs(d1)), (key, d1, d2)
