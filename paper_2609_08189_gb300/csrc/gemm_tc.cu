@@ -463,7 +463,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
               const GemmArgs a0, const GemmArgs a1) {
-  pdl_enter();
+  if (a0.pdl_mode != 2) pdl_enter();
   using C = TcCfg<BN, epi_warps<EPI0>()>;
   constexpr bool kGrouped = EPI1 != EPI_NONE;
   extern __shared__ uint8_t smem_raw[];
@@ -533,6 +533,8 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
         tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         const CUtensorMap* tA = pr ? &tmA1 : &tmA0;
         const CUtensorMap* tB = pr ? &tmB1 : &tmB0;
+        if (a0.pdl_mode == 1 && g + (int)gridDim.x >= total)   // this CTA's last tile
+          asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitLimitNs) || misc[1]) {
             ok = false;
@@ -653,6 +655,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
   }
+  if (a0.pdl_mode == 2) pdl_enter();   // complete only after the previous kernel
 }
 
 template <int BN, int EPI0, int EPI1>

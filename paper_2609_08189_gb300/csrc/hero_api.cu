@@ -787,11 +787,19 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       ua.slot_cols = kTcPartCols;
       ua.lo = au.lo;
       CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] { return launch_adapter_up(ua, st); }));
-    } else if (!dense) {   // epilogue-bound (rank-d_r contraction): the wide-epilogue variant
-      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
-        return launch_gemm_tc(256, EPI_LAYER_OUT_WIDE, m->tm_ah, m->tm_w2[jj], au, m->num_sms, st);
-      }));
     }
+    // large batches: the adapter's W_2 GEMM (wide epilogue) runs after FFN down, on the
+    // SMs FFN down's last wave leaves idle (pdl_mode 1 / 2: disjoint rows, inputs from
+    // the gate/up launch)
+    const bool adapter_after = !dense && !(T <= 256 && r <= 64);
+    auto adapter_up_wide = [&](int pdl_mode) -> hero_status {
+      GemmArgs aw = au;
+      aw.pdl_mode = pdl_mode;
+      CUDA_TRY(timed(m, HERO_K_ADAPTER_UP, st, [&] {
+        return launch_gemm_tc(256, EPI_LAYER_OUT_WIDE, m->tm_ah, m->tm_w2[jj], aw, m->num_sms, st);
+      }));
+      return HERO_OK;
+    };
     const int m_t = (T + 127) / 128;
     const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
     if (ds > 1) {   // few tiles (small T): split K into partials, then the closing epilogue
@@ -806,12 +814,14 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
         return launch_splitk_close(m->splitk_ws, ds, sk.split_stride, d, m->counts, T, dn.lo, st);
       }));
-      return HERO_OK;
+      return adapter_after ? adapter_up_wide(0) : HERO_OK;
     }
+    GemmArgs dl = dn;
+    dl.pdl_mode = adapter_after ? 1 : 0;
     CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
-      return launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dn, m->num_sms, st);
+      return launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dl, m->num_sms, st);
     }));
-    return HERO_OK;
+    return adapter_after ? adapter_up_wide(2) : HERO_OK;
   }
   CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] { return launch_gemm_simt(EPI_SWIGLU, gu, st); }));
   CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] { return launch_gemm_simt(EPI_LAYER_OUT, dn, st); }));

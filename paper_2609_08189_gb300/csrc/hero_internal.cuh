@@ -121,6 +121,12 @@ struct GemmArgs {
   long split_stride;
   const float* resid;  // EPI_RESIDUAL: [rows, N] fp32 added to the product (ld = ldo)
   RopeArgs rope;       // EPI_QKV_ROPE
+  // Programmatic dependent launch: 0 waits for the previous kernel at the start;
+  // 1 also lets the next kernel launch once every CTA has taken its last tile;
+  // 2 (a launch whose inputs all come from earlier kernels than the previous one,
+  // writing rows the previous one does not touch) works without waiting and waits
+  // for the previous kernel at its end, so the kernels after it still follow both.
+  int pdl_mode;
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
