@@ -360,6 +360,81 @@ __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const flo
   }
 }
 
+// Memory step at small token counts (every warp of the CTA busy): the nthr / 32 / TB
+// warps of a token each take DM / WPT rows of its S, write them back updated and leave
+// their partial read of c in scratch ([TB][WPT][DM]); warp 0 of a token also reads
+// den = phi(q) . zeta and updates zeta, its den in scratch[TB WPT DM + token].
+// memory_split_finish adds the partials in warp order once the CTA has synchronised.
+template <int DM, int TB>
+constexpr int mem_wpt() { return nthr<TB>() / 32 / TB; }
+
+template <int DM, int TB>
+__device__ __forceinline__ void memory_split(const RouterArgs& a, const float* qkv, float* scratch,
+                                             int t0, int warp, int lane) {
+  constexpr int WPT = mem_wpt<DM, TB>();
+  constexpr int RW = DM / WPT;            // rows of S per warp
+  constexpr int LPR = DM / 4;             // lanes per S row (float4 columns)
+  constexpr int RPI = 32 / LPR;           // rows per iteration
+  static_assert(RW % RPI == 0, "whole iterations per warp");
+  const int tl = warp / WPT, sub = warp - tl * WPT;
+  const int t = t0 + tl;
+  if (tl >= TB || t >= a.T) return;
+  const float* q = qkv + tl * 3 * DM;
+  const float* k = q + DM;
+  const float* v = q + 2 * DM;
+  if (sub == 0) {
+    float* z = a.zeta + (size_t)t * DM;
+    float den = 0.f;
+    for (int m = lane; m < DM; m += 32) {
+      const float zo = z[m];
+      den += phif_(q[m]) * zo;
+      z[m] = a.rho * zo + phif_(k[m]);
+    }
+    den = warp_sum(den);
+    if (lane == 0) scratch[TB * WPT * DM + tl] = den;
+  }
+  float* S = a.S + (size_t)t * DM * DM;
+  const int cq = lane % LPR, r0 = lane / LPR;
+  const float4 vv = *reinterpret_cast<const float4*>(v + 4 * cq);
+  float4 so[RW / RPI];
+#pragma unroll
+  for (int i = 0; i < RW / RPI; ++i)
+    so[i] = *reinterpret_cast<const float4*>(S + (sub * RW + r0 + i * RPI) * DM + 4 * cq);
+  float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int i = 0; i < RW / RPI; ++i) {
+    const int r = sub * RW + r0 + i * RPI;
+    const float fq = phif_(q[r]), fk = phif_(k[r]);
+    c.x += fq * so[i].x; c.y += fq * so[i].y; c.z += fq * so[i].z; c.w += fq * so[i].w;
+    *reinterpret_cast<float4*>(S + r * DM + 4 * cq) =
+        make_float4(a.rho * so[i].x + fk * vv.x, a.rho * so[i].y + fk * vv.y,
+                    a.rho * so[i].z + fk * vv.z, a.rho * so[i].w + fk * vv.w);
+  }
+#pragma unroll
+  for (int o = LPR; o < 32; o <<= 1) {
+    c.x += __shfl_xor_sync(0xffffffffu, c.x, o);
+    c.y += __shfl_xor_sync(0xffffffffu, c.y, o);
+    c.z += __shfl_xor_sync(0xffffffffu, c.z, o);
+    c.w += __shfl_xor_sync(0xffffffffu, c.w, o);
+  }
+  if (r0 == 0)
+    *reinterpret_cast<float4*>(scratch + (tl * WPT + sub) * DM + 4 * cq) = c;
+}
+
+template <int DM, int TB>
+__device__ __forceinline__ void memory_split_finish(const RouterArgs& a, const float* scratch,
+                                                    float* cT, int t0) {
+  constexpr int WPT = mem_wpt<DM, TB>();
+  for (int e = threadIdx.x; e < TB * DM; e += nthr<TB>()) {
+    const int tl = e / DM, col = e - tl * DM;
+    if (t0 + tl >= a.T) continue;
+    float c = 0.f;
+#pragma unroll
+    for (int sub = 0; sub < WPT; ++sub) c += scratch[(tl * WPT + sub) * DM + col];
+    cT[col * TB + tl] = c / (scratch[TB * WPT * DM + tl] + a.eps);
+  }
+}
+
 template <int DM, int TB>
 __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_router(const RouterArgs a) {
   pdl_enter();
@@ -528,6 +603,10 @@ __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
     for (int e = tid; e < DM * TB; e += nthr<TB>()) sT[ds * TB + e] = 0.f;
+  } else if constexpr (TB < 16 && DM <= 128 && DM / mem_wpt<DM, TB>() >= 32 / (DM / 4)) {
+    memory_split<DM, TB>(a, qkv, skT, t0, warp, lane);   // skT is free between steps 4 and 7
+    __syncthreads();
+    memory_split_finish<DM, TB>(a, skT, sT + ds * TB, t0);
   } else {
     memory_read_write<DM, TB>(a, qkv, sT + ds * TB, t0, warp, lane);
   }
