@@ -162,22 +162,32 @@ struct RouterLayout {
 // t < TB; `in` is [NI][TB]; `out` is [NO][TB] or, if out_tok_ld > 0, token-major
 // [TB][out_tok_ld].  Narrow outputs split K across threads; the partial sums go to
 // `scratch` ([ks][NO][TB], at most scratch_cap floats) and are added in a fixed
-// order, so results are bitwise reproducible.  NO must be a multiple of 4;
-// contains __syncthreads.
+// order, so results are bitwise reproducible.  NO must be a multiple of 4.  Run by the
+// gn threads from g0 (default: the whole CTA), which it synchronises: __syncthreads for
+// the whole CTA, else the named barrier `bar` (two groups may run concurrently).
+__device__ __forceinline__ void group_sync(int bar, int gn) {
+  if (bar == 0)
+    __syncthreads();
+  else
+    asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(gn) : "memory");
+}
+
 template <int TB>
 __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int NO,
                      const float* __restrict__ bias, float* out, int out_tok_ld, bool silu_act,
-                     float* scratch = nullptr, int scratch_cap = 0) {
+                     float* scratch = nullptr, int scratch_cap = 0, int g0 = 0,
+                     int gn = nthr<TB>(), int bar = 0) {
   const int no4 = NO >> 2;
   const int base = no4 * (TB / 4);
+  const int gt = threadIdx.x - g0;   // index in the group
   int ks = 1;
   if (scratch)
-    while (base * ks * 2 <= nthr<TB>() && NI / (ks * 2) >= (TB < 16 ? 8 : 16) &&
+    while (base * ks * 2 <= gn && NI / (ks * 2) >= (TB < 16 ? 8 : 16) &&
            (ks * 2) * NO * TB <= scratch_cap)
       ks <<= 1;
   const int kchunk = (NI + ks - 1) / ks;
   auto oidx = [&](int o, int t) { return out_tok_ld > 0 ? t * out_tok_ld + o : o * TB + t; };
-  for (int w = threadIdx.x; w < base * ks; w += nthr<TB>()) {
+  for (int w = gt; w < base * ks; w += gn) {
     const int o4 = (w % no4) * 4;
     const int rest = w / no4;
     const int t4 = (rest % (TB / 4)) * 4;
@@ -212,16 +222,16 @@ __device__ void bmm4(const float* in, int NI, const float* __restrict__ Wt, int 
         }
       }
   }
-  __syncthreads();
+  group_sync(bar, gn);
   if (ks > 1) {
-    for (int e = threadIdx.x; e < NO * TB; e += nthr<TB>()) {
+    for (int e = gt; e < NO * TB; e += gn) {
       const int o = e / TB, t = e % TB;
       float v = 0.f;
       for (int kk = 0; kk < ks; ++kk) v += scratch[(kk * NO + o) * TB + t];
       v += bias ? __ldg(bias + o) : 0.f;
       out[oidx(o, t)] = silu_act ? siluf_(v) : v;
     }
-    __syncthreads();
+    group_sync(bar, gn);
   }
 }
 
@@ -367,6 +377,14 @@ __device__ __forceinline__ void memory_read_write(const RouterArgs& a, const flo
 // memory_split_finish adds the partials in warp order once the CTA has synchronised.
 template <int DM, int TB>
 constexpr int mem_wpt() { return nthr<TB>() / 32 / TB; }
+
+// The split memory step applies when every warp of a token gets whole row iterations.
+template <int DM, int TB>
+constexpr bool mem_split() {
+  if (TB >= 16 || DM > 128) return false;
+  constexpr int wpt = mem_wpt<DM, TB>() > 0 ? mem_wpt<DM, TB>() : 1;
+  return mem_wpt<DM, TB>() > 0 && DM / wpt >= 32 / (DM / 4);
+}
 
 template <int DM, int TB>
 __device__ __forceinline__ void memory_split(const RouterArgs& a, const float* qkv, float* scratch,
@@ -586,14 +604,27 @@ __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_
     return;
   }
 
-  // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s)
-  bmm4<TB>(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
-  if (a.variant & RV_NO_AUX) {   // ablation: no auxiliary path encoder, z_a = 0
-    for (int e = tid; e < a.d_a * TB; e += nthr<TB>()) sT[a.d_h * TB + e] = 0.f;
+  // 3. z_h = W_hu enc (Eq. 5) -> s[0, d_h); FFN_path hidden; z_a (Eq. 9) -> s[d_h, d_s).
+  //    Small token counts: the two are independent and run on the two halves of the CTA.
+  if (TB < 16 && !(a.variant & RV_NO_AUX)) {
+    constexpr int half = nthr<TB>() / 2;
+    if (tid < half) {
+      bmm4<TB>(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072, 0, half, 1);
+    } else {
+      bmm4<TB>(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true, nullptr, 0, half, half, 2);
+      bmm4<TB>(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false,
+               nullptr, 0, half, half, 2);
+    }
     __syncthreads();
   } else {
-    bmm4<TB>(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
-    bmm4<TB>(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
+    bmm4<TB>(bigT, a.d_enc, a.w.w_hu_t, a.d_h, nullptr, sT, 0, false, aux, 3072);
+    if (a.variant & RV_NO_AUX) {   // ablation: no auxiliary path encoder, z_a = 0
+      for (int e = tid; e < a.d_a * TB; e += nthr<TB>()) sT[a.d_h * TB + e] = 0.f;
+      __syncthreads();
+    } else {
+      bmm4<TB>(xT, 6, a.w.path_w1_t, a.d_path, a.w.path_b1, phT, 0, true);
+      bmm4<TB>(phT, a.d_path, a.w.path_w2_t, a.d_a, a.w.path_b2, sT + a.d_h * TB, 0, false);
+    }
   }
 
   // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step
@@ -603,7 +634,7 @@ __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
     for (int e = tid; e < DM * TB; e += nthr<TB>()) sT[ds * TB + e] = 0.f;
-  } else if constexpr (TB < 16 && DM <= 128 && DM / mem_wpt<DM, TB>() >= 32 / (DM / 4)) {
+  } else if constexpr (mem_split<DM, TB>()) {
     memory_split<DM, TB>(a, qkv, skT, t0, warp, lane);   // skT is free between steps 4 and 7
     __syncthreads();
     memory_split_finish<DM, TB>(a, skT, sT + ds * TB, t0);
