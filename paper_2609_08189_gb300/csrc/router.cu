@@ -627,9 +627,23 @@ __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_
     }
   }
 
-  // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step
-  bmm4<TB>(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false, skT,
-           RouterLayout<TB>::kSplitScratch);
+  // 4. q | k | v = W_{q,k,v} s (Eq. 10), token-major for the memory step.  Small token
+  //    counts: W_n s of step 6 (it needs s only) runs beside it on the other half.
+  const bool need_nu = a.j > 1 && !no_memread;
+  const bool nu_early = TB < 16 && need_nu;
+  const int cap_big = (a.d_enc > a.d_head ? a.d_enc : a.d_head) * TB;
+  if (nu_early) {
+    constexpr int half = nthr<TB>() / 2;
+    if (tid < half)
+      bmm4<TB>(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false, skT,
+               RouterLayout<TB>::kSplitScratch, 0, half, 1);
+    else   // W_n s -> aux [DM][TB] (aux and the big region are free after step 3)
+      bmm4<TB>(sT, ds, a.w.w_n_t, DM, nullptr, aux, 0, false, bigT, cap_big, half, half, 2);
+    __syncthreads();
+  } else {
+    bmm4<TB>(sT, ds, a.w.w_qkv_t, 3 * DM, nullptr, qkv, 3 * DM, false, skT,
+             RouterLayout<TB>::kSplitScratch);
+  }
 
   // 5. memory read (Eq. 11) fused with the write (Eq. 12), one warp per token.
   if (no_memread) {   // ablation: c = 0; the memory is neither read nor written
@@ -645,12 +659,11 @@ __global__ void __launch_bounds__(nthr<TB>(), (DM >= 256 || TB < 16) ? 1 : 4) k_
 
   // 6. nu = 1 - cos(W_n s, W_c c) for j > 1 (Eq. 13); nu_1 = 0
   float* nuT = sT + (ds + DM) * TB;
-  if (a.j > 1 && !no_memread) {   // the ablation without memory access sees nu = 0
-    const int cap = (a.d_enc > a.d_head ? a.d_enc : a.d_head) * TB;
+  if (need_nu) {   // the ablation without memory access sees nu = 0
     float* nv = aux;               // [DM][TB]
     float* cv = aux + DM * TB;     // [DM][TB]
-    bmm4<TB>(sT, ds, a.w.w_n_t, DM, nullptr, nv, 0, false, bigT, cap);
-    bmm4<TB>(sT + ds * TB, DM, a.w.w_c_t, DM, nullptr, cv, 0, false, bigT, cap);
+    if (!nu_early) bmm4<TB>(sT, ds, a.w.w_n_t, DM, nullptr, nv, 0, false, bigT, cap_big);
+    bmm4<TB>(sT + ds * TB, DM, a.w.w_c_t, DM, nullptr, cv, 0, false, bigT, cap_big);
     // thread (part, t) sums DM/16 products; fixed-order reduction per token
     const int tl = tid % TB, part = tid / TB;
     float xy = 0.f, xx = 0.f, yy = 0.f;
