@@ -2,8 +2,13 @@
 //   x = LN_attn(h)                      k_attn_norm (bf16 rows, the projection operand)
 //   q, k, v = x [W_q; W_k; W_v]^T,      tensor-core GEMM (gemm_tc.cu) whose epilogue
 //   q, k <- RoPE(q), RoPE(k)            rotates and stores bf16 [sequence][head][position][128]
-//   o = softmax(q k^T / sqrt(hd)) v     k_flash_attn (causal, grouped-query heads)
-//   h_bar = h + o W_o^T                 tensor-core GEMM with the residual epilogue
+//                                       (and v transposed for k_flash_tc)
+//   o = softmax(q k^T / sqrt(hd)) v     causal, grouped-query heads: k_flash_tc (tcgen05,
+//                                       S >= 128), k_flash_attn (mma.sync, shorter), or one
+//                                       query per sequence over the KV cache: k_attn_decode
+//                                       + k_attn_combine
+//   h_bar = h + o W_o^T                 tensor-core GEMM with the residual epilogue, which
+//                                       in the decoder also closes into the block entry
 #include "hero_device.cuh"
 
 namespace hero {
