@@ -8,23 +8,24 @@
 // i.e. 2 d_r FLOP per output element against 22 bytes of epilogue traffic, so it
 // runs on the FMA pipes with row-contiguous global access.
 //
-// CTA: 32 adapter rows x 256 output columns, 256 threads.  Warp w owns rows
-// 4w..4w+3; lane x owns columns x + 32 j (j < 8), so every warp instruction of
-// the epilogue touches 128 contiguous bytes of one row.  The rows the epilogue
+// CTA: 8 RPW adapter rows x 256 output columns, 256 threads.  Warp w owns rows
+// RPW w .. RPW w + RPW - 1; lane x owns columns x + 32 j (j < 8), so every warp
+// instruction of the epilogue touches 128 contiguous bytes of one row.  RPW = 4 for
+// large batches; 1 when the row count is small (decode), so the few rows spread over
+// four times the CTAs.  The rows the epilogue
 // will update are bulk-prefetched into L2 at kernel start.
 #include "hero_device.cuh"
 
 namespace hero {
 namespace {
 
-constexpr int AU_ROWS = 32;
 constexpr int AU_COLS = 256;
 constexpr int AU_DR = 64;          // largest supported rank
 constexpr int AU_WLD = AU_DR + 2;  // row stride of the staged W_2 slice (conflict-free reads)
 
-template <typename WT>
+template <int RPW, typename WT>
 constexpr size_t au_smem() {
-  return sizeof(float) * AU_ROWS * AU_DR + sizeof(WT) * AU_COLS * AU_WLD;
+  return sizeof(float) * 8 * RPW * AU_DR + sizeof(WT) * AU_COLS * AU_WLD;
 }
 
 __device__ __forceinline__ float to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
@@ -32,8 +33,9 @@ __device__ __forceinline__ float to_f32(float v) { return v; }
 
 // WT: operand element type, uint16_t (bf16 bits) or float.  SLOT: columns per
 // partial-sum slot of the model (64 or 256).
-template <int SLOT, typename WT>
+template <int SLOT, int RPW, typename WT>
 __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
+  constexpr int AU_ROWS = 8 * RPW;
   pdl_enter();
   extern __shared__ __align__(16) float smem_au[];
   float* ahs = smem_au;                                         // [AU_ROWS][AU_DR] fp32
@@ -100,28 +102,28 @@ __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
   }
   __syncthreads();
 
-  float acc[4][8];
+  float acc[RPW][8];
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+  for (int i = 0; i < RPW; ++i)
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-  const float* arow = ahs + (warp * 4) * AU_DR;
+  const float* arow = ahs + (warp * RPW) * AU_DR;
   for (int k = 0; k < dr; ++k) {
-    float x[4], w[8];
+    float x[RPW], w[8];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) x[i] = arow[i * AU_DR + k];
+    for (int i = 0; i < RPW; ++i) x[i] = arow[i * AU_DR + k];
 #pragma unroll
     for (int j = 0; j < 8; ++j) w[j] = to_f32(w2s[(lane + 32 * j) * AU_WLD + k]);
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < RPW; ++i)
 #pragma unroll
       for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(x[i], w[j], acc[i][j]);
   }
 
   constexpr int spt = AU_COLS / SLOT;   // partial slots per tile
 #pragma unroll 1
-  for (int i = 0; i < 4; ++i) {
-    const int m = m0 + warp * 4 + i;
+  for (int i = 0; i < RPW; ++i) {
+    const int m = m0 + warp * RPW + i;
     if (m >= M) break;                     // warp-uniform
     const int t = p.idx[m];
     const float s = p.scale[m];
@@ -151,18 +153,18 @@ __global__ void __launch_bounds__(256) k_adapter_up(const AdapterUpArgs a) {
   }
 }
 
-template <int SLOT, typename WT>
+template <int SLOT, int RPW, typename WT>
 cudaError_t launch_au(const AdapterUpArgs& a, cudaStream_t st) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_adapter_up<SLOT, WT>,
+    cudaError_t e = cudaFuncSetAttribute(k_adapter_up<SLOT, RPW, WT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)au_smem<WT>());
+                                         (int)au_smem<RPW, WT>());
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((a.d + AU_COLS - 1) / AU_COLS, (a.m_max + AU_ROWS - 1) / AU_ROWS);
-  return launch_pdl(k_adapter_up<SLOT, WT>, grid, dim3(256), au_smem<WT>(), st, a);
+  dim3 grid((a.d + AU_COLS - 1) / AU_COLS, (a.m_max + 8 * RPW - 1) / (8 * RPW));
+  return launch_pdl(k_adapter_up<SLOT, RPW, WT>, grid, dim3(256), au_smem<RPW, WT>(), st, a);
 }
 
 }  // namespace
@@ -170,8 +172,11 @@ cudaError_t launch_au(const AdapterUpArgs& a, cudaStream_t st) {
 cudaError_t launch_adapter_up(const AdapterUpArgs& a, cudaStream_t st) {
   if (a.m_max <= 0) return cudaSuccess;
   if (a.d_r > AU_DR) return cudaErrorInvalidValue;
-  if (a.bf16 && a.slot_cols == 128) return launch_au<128, uint16_t>(a, st);
-  if (!a.bf16 && a.slot_cols == 64) return launch_au<64, float>(a, st);
+  const bool few = a.m_max <= 256;
+  if (a.bf16 && a.slot_cols == 128)
+    return few ? launch_au<128, 1, uint16_t>(a, st) : launch_au<128, 4, uint16_t>(a, st);
+  if (!a.bf16 && a.slot_cols == 64)
+    return few ? launch_au<64, 1, float>(a, st) : launch_au<64, 4, float>(a, st);
   return cudaErrorInvalidValue;
 }
 
