@@ -46,6 +46,55 @@ __global__ void __launch_bounds__(256) k_attn_norm(const float* __restrict__ h,
   }
 }
 
+// The same with one CTA of 8 warps per row (few rows: decoding steps), each warp
+// 1/8 of the row held in registers; the 8 partial sums of squares are added in warp
+// order.  d must be a multiple of 1024.
+__global__ void __launch_bounds__(256) k_attn_norm_row(const float* __restrict__ h,
+                                                       const float* __restrict__ g, int d,
+                                                       float eps, uint16_t* __restrict__ x) {
+  pdl_enter();
+  __shared__ float part[8];
+  const size_t row = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int seg = d / 8, c0 = warp * seg;
+  const float* hr = h + row * d;
+  constexpr int MAXV = 4;   // float4 per lane for d <= 4096
+  float4 v[MAXV];
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < MAXV; ++i) {
+    const int c = c0 + (i * 32 + lane) * 4;
+    v[i] = (i * 128 < seg) ? *reinterpret_cast<const float4*>(hr + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+  }
+  for (int c = c0 + (MAXV * 32 + lane) * 4; c < c0 + seg; c += 128) {   // d > 4096
+    const float4 w = *reinterpret_cast<const float4*>(hr + c);
+    ss += w.x * w.x + w.y * w.y + w.z * w.z + w.w * w.w;
+  }
+  ss = warp_sum(ss);
+  if (lane == 0) part[warp] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += part[w];
+  const float rinv = rsqrtf(tot / (float)d + eps);
+#pragma unroll
+  for (int i = 0; i < MAXV; ++i) {
+    const int c = c0 + (i * 32 + lane) * 4;
+    if (i * 128 >= seg) break;
+    const float4 gv = __ldg(reinterpret_cast<const float4*>(g + c));
+    store4(x, row * d + c,
+           make_float4(v[i].x * rinv * gv.x, v[i].y * rinv * gv.y, v[i].z * rinv * gv.z,
+                       v[i].w * rinv * gv.w), 1);
+  }
+  for (int c = c0 + (MAXV * 32 + lane) * 4; c < c0 + seg; c += 128) {
+    const float4 w = *reinterpret_cast<const float4*>(hr + c);
+    const float4 gv = __ldg(reinterpret_cast<const float4*>(g + c));
+    store4(x, row * d + c,
+           make_float4(w.x * rinv * gv.x, w.y * rinv * gv.y, w.z * rinv * gv.z, w.w * rinv * gv.w), 1);
+  }
+}
+
 // ---------------------------------------------------------------------------------
 // Causal attention, FlashAttention-2 schedule on the mma.sync bf16 tensor path:
 // CTA = 64 query rows of one (sequence, head), 4 warps of 16 rows; key/value tiles
@@ -783,6 +832,9 @@ cudaError_t launch_attn_norm(const float* h, const float* g, int T, int d, float
                              cudaStream_t st) {
   if (T <= 0) return cudaSuccess;
   if (d % 128) return cudaErrorInvalidValue;
+  if (T <= 512 && d % 1024 == 0)   // few rows: a CTA per row
+    return launch_pdl(k_attn_norm_row, dim3((unsigned)T), dim3(256), 0, st, h, g, d, eps,
+                      static_cast<uint16_t*>(x));
   return launch_pdl(k_attn_norm, dim3((unsigned)((T + 7) / 8)), dim3(256), 0, st, h, g, T, d, eps,
                     static_cast<uint16_t*>(x));
 }
