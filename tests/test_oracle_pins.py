@@ -853,3 +853,27 @@ def test_training_loss_is_smooth_along_each_trainable_tensor(key):
     d2 = ho.directional_derivative(f, 5e-5)
     assert abs(d1) > 1e-9, key
     assert abs(d1 - d2) <= 1e-5 * max(1.0, abs(d1)), (key, d1, d2)
+
+
+@pytest.mark.parametrize("n_dense", [0, 1])
+def test_decoder_forward_is_the_stack_fed_its_attention_updates(n_dense):
+    """decoder_forward wires Eq. 1: replaying routed_ffn_stack with the additive input
+    P_j = h_bar_j - h_{j-1} taken from the decoder run's own records reproduces its
+    outputs, gates and decisions exactly (f32 model, free-running; with and without a
+    dense prefix)."""
+    cfg = hi.StackConfig("dec_micro", 3, 256, 96, 8, 8, 2 * 20, "f32", 0.3, d_h=4, d_a=4,
+                         d_enc=8, d_head=8, d_path=4, seed=7, batch=2, seq_len=20,
+                         n_heads=2, n_kv_heads=1, rope_theta=500000.0, n_dense=n_dense)
+    oc = ho.OracleConfig.from_stack(cfg)
+    w, wa = hi.generate_weights(cfg), hi.generate_attn_weights(cfg)
+    h0 = hi.to_f64(hi.generate_h_in(cfg))
+    first = ho.decoder_forward(oc, w, wa, h0, 0.5, 2, 1, cfg.rope_theta, 2, 20)
+    tau = float(np.median(first["gate"][n_dense]))
+    dec = ho.decoder_forward(oc, w, wa, h0, tau, 2, 1, cfg.rope_theta, 2, 20, record=True)
+    hs = [h0] + [rec["h"] for rec in dec["layers"]]
+    P = np.stack([rec["h_bar"] - hs[j] for j, rec in enumerate(dec["layers"])])
+    stack = ho.routed_ffn_stack(oc, w, h0, P, tau)
+    np.testing.assert_array_equal(stack["mask"], dec["mask"])
+    np.testing.assert_allclose(stack["gate"], dec["gate"], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(stack["h_out"], dec["h_out"], rtol=0, atol=1e-12)
+    assert 0 < dec["mask"][n_dense:].mean() < 1
