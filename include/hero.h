@@ -269,7 +269,8 @@ hero_status hero_decoder_forward(hero_model* m, int32_t n_seqs, int32_t seq_len,
  * Allocate the cache for max_seqs sequence slots of max_len positions, all
  * layers: 2 * n_layers * max_seqs * H_kv * max_len * 128 bf16, plus the
  * split-KV partial results of the decode attention.  Needs hero_attn_init;
- * once per model (HERO_ERR_ARG on a second call).  Synchronous. */
+ * once per model (HERO_ERR_ARG on a second call); HERO_ERR_UNSUPPORTED unless
+ * H / H_kv is 1, 2, 4 or 8.  Synchronous. */
 hero_status hero_kv_cache_init(hero_model* m, int32_t max_seqs, int32_t max_len);
 
 /* hero_decoder_forward on n_seqs sequences of seq_len tokens that are cache slots

@@ -1568,6 +1568,11 @@ extern "C" hero_status hero_kv_cache_init(hero_model* m, int32_t max_seqs, int32
   if (m->kv) return fail(HERO_ERR_ARG, "the model already has a KV cache");
   if (max_seqs < 1 || max_seqs > 65535 || max_len < 1)
     return fail(HERO_ERR_ARG, "need 1 <= max_seqs <= 65535 and max_len >= 1");
+  {
+    const int G = m->n_heads / m->n_kv_heads;   // query heads per key/value head
+    if (G != 1 && G != 2 && G != 4 && G != 8)
+      return fail(HERO_ERR_UNSUPPORTED, "decoding needs 1, 2, 4 or 8 query heads per key/value head");
+  }
   CUDA_TRY(cudaSetDevice(m->device));
   const hero_config& c = m->cfg;
   const size_t layer = (size_t)max_seqs * m->n_kv_heads * max_len * 128;
