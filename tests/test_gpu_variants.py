@@ -1,4 +1,4 @@
-"""GPU parity of the router ablations (Sec. 4.4) and of the memory width d_m = 256.
+"""GPU parity of the router ablations (Sec. 4.4) and of memory widths d_m = 32, 128, 256.
 
 Each ablation bit (HERO_ROUTER_NO_HISTORY, _NO_MEMREAD, _NO_AUX, _NO_POS) and the
 widest memory of the paper's memory-dimension ablation run through the CUDA path
@@ -20,7 +20,10 @@ pytestmark = pytest.mark.gpu
 
 VARIANTS = [ho.NO_HISTORY, ho.NO_MEMREAD, ho.NO_AUX, ho.NO_POS, ho.NO_AUX | ho.NO_POS]
 CASES = ([(name, v, None) for name in ("tiny_f32", "small_bf16") for v in VARIANTS] +
-         [("tiny_f32", 0, 256), ("small_bf16", 0, 256), ("small_bf16", ho.NO_MEMREAD, 256)])
+         [("tiny_f32", 0, 256), ("small_bf16", 0, 256), ("small_bf16", ho.NO_MEMREAD, 256),
+          # the small-token-count router splits a token's memory step over warps; these
+          # widths take whole-row iterations of 4 and 16 rows per warp
+          ("small_bf16", 0, 32), ("small_bf16", 0, 128)])
 
 
 @pytest.fixture(scope="module")
