@@ -555,3 +555,73 @@ def training_loss(cfg: OracleConfig, weights, h_in, attn_delta, mask, G, alpha: 
 def directional_derivative(f: Callable[[float], float], h: float) -> float:
     """Central difference (f(h) - f(-h)) / 2h of a function of the step along a direction."""
     return (f(h) - f(-h)) / (2.0 * h)
+
+
+def silu_grad(x: np.ndarray) -> np.ndarray:
+    """d SiLU / dx = sigma(x) (1 + x (1 - sigma(x)))."""
+    s = sigmoid(x)
+    return s * (1.0 + x * (1.0 - s))
+
+
+def rms_norm_backward(x, gain, eps: float, du):
+    """Gradient of u = RMSNorm(x) gain with respect to x, given du (last axis):
+    r = (mean(x^2) + eps)^(-1/2), u = x r gain, so
+    dx = r (du gain) - x r^3 mean(x (du gain))."""
+    r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)
+    dg = du * gain
+    return r * dg - x * r ** 3 * np.mean(x * dg, axis=-1, keepdims=True)
+
+
+def block_branch_backward(h_bar, g, decide, G, wl, rms_eps: float):
+    """Backward of the branch part of a routed block with its decisions fixed (Eq. 3,
+    Eq. 2, the SwiGLU FFN and LN_ffn), for the training path (Sec. 3.3: the backbone
+    is frozen, the adapter trains, and the selected branch's scale g or 1 - g carries
+    the gradient to the router):
+        h_out = h_bar + s * Branch(u),  u = LN_ffn(h_bar),
+        s = g, Branch = FFN for decide; s = 1 - g, Branch = Adapter otherwise,
+    given G = dL/dh_out [T, d].  Returns dL/dh_bar (residual plus branch path),
+    dL/dg [T], and dL/dW_1 [d_r, d], dL/dW_2 [d, d_r] of the adapter.  float64, no
+    rounding (the f32 model)."""
+    G = np.asarray(G, dtype=np.float64)
+    T, d = h_bar.shape
+    u = rms_norm(h_bar, wl["ffn_norm_g"], rms_eps)
+    du = np.zeros((T, d))
+    dg = np.zeros(T)
+    dW1 = np.zeros_like(wl["ad_w1"])
+    dW2 = np.zeros_like(wl["ad_w2"])
+    F = np.nonzero(decide)[0]
+    A = np.nonzero(~np.asarray(decide, dtype=bool))[0]
+    if F.size:   # h += g W_down (SiLU(W_gate u) * W_up u)
+        uf = u[F]
+        gate, up = uf @ wl["w_gate"].T, uf @ wl["w_up"].T
+        y = (silu(gate) * up) @ wl["w_down"].T
+        dg[F] = np.sum(G[F] * y, axis=1)
+        dy = g[F, None] * G[F]
+        dact = dy @ wl["w_down"]
+        dgate = dact * up * silu_grad(gate)
+        dup = dact * silu(gate)
+        du[F] = dgate @ wl["w_gate"] + dup @ wl["w_up"]
+    if A.size:   # h += (1 - g) W_2 SiLU(W_1 u)
+        ua = u[A]
+        a = ua @ wl["ad_w1"].T
+        hid = silu(a)
+        y = hid @ wl["ad_w2"].T
+        dg[A] = -np.sum(G[A] * y, axis=1)
+        dy = (1.0 - g[A])[:, None] * G[A]
+        dW2 = dy.T @ hid
+        da = (dy @ wl["ad_w2"]) * silu_grad(a)
+        dW1 = da.T @ ua
+        du[A] = da @ wl["ad_w1"]
+    dh_bar = G + rms_norm_backward(h_bar, wl["ffn_norm_g"], rms_eps, du)
+    return {"dh_bar": dh_bar, "dg": dg, "dW1": dW1, "dW2": dW2}
+
+
+def skip_penalty_grad(gates, n_seqs: int, seq_len: int, n_dense: int = 0):
+    """d L_skip / d g [L, T]: 2 / (B (T - 1)) times the token's summed routed gates at its
+    next-token positions, 0 at a sequence's last position and in dense-prefix rows."""
+    g = np.asarray(gates, dtype=np.float64)
+    out = np.zeros_like(g)
+    tot = g[n_dense:].sum(axis=0)
+    pos = np.arange(g.shape[1]) % seq_len
+    out[n_dense:] = np.where(pos < seq_len - 1, 2.0 / (n_seqs * (seq_len - 1)) * tot, 0.0)[None, :]
+    return out

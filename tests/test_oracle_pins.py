@@ -877,3 +877,59 @@ def test_decoder_forward_is_the_stack_fed_its_attention_updates(n_dense):
     np.testing.assert_allclose(stack["gate"], dec["gate"], rtol=0, atol=1e-13)
     np.testing.assert_allclose(stack["h_out"], dec["h_out"], rtol=0, atol=1e-12)
     assert 0 < dec["mask"][n_dense:].mean() < 1
+
+
+def test_block_branch_backward_matches_central_differences():
+    """block_branch_backward against central differences of the forward branch
+    combination (LN_ffn, SwiGLU FFN or adapter, scale g or 1 - g, residual), for every
+    returned gradient: h_bar and g element-wise on a sample, W_1 and W_2 along random
+    directions."""
+    cfg = hi.CONFIGS["tiny_f32"]
+    w = hi.generate_weights(cfg)
+    wl = {k: ho._f64(w[k][1]) for k in ("ffn_norm_g", "w_gate", "w_up", "w_down", "ad_w1", "ad_w2")}
+    rng = np.random.default_rng(11)
+    T, d = 24, cfg.d_model
+    h_bar = rng.standard_normal((T, d))
+    g = rng.uniform(0.1, 0.9, T)
+    decide = rng.random(T) < 0.6
+    G = rng.standard_normal((T, d))
+
+    def loss(hb=h_bar, gg=g, wl_=wl):
+        u = ho.rms_norm(hb, wl_["ffn_norm_g"], cfg.rms_eps)
+        out = hb.copy()
+        F, A = np.nonzero(decide)[0], np.nonzero(~decide)[0]
+        out[F] += gg[F, None] * ho.swiglu_ffn(u[F], wl_, ho._identity)
+        out[A] += (1 - gg[A])[:, None] * ho.adapter(u[A], wl_, ho._identity)
+        return float(np.sum(G * out))
+
+    bw = ho.block_branch_backward(h_bar, g, decide, G, wl, cfg.rms_eps)
+    eps = 1e-6
+    for t, c in [(0, 0), (3, 17), (5, 200), (int(np.nonzero(~decide)[0][0]), 33)]:
+        e = np.zeros_like(h_bar)
+        e[t, c] = 1.0
+        fd = ho.directional_derivative(lambda hh: loss(hb=h_bar + hh * e), eps)
+        assert abs(fd - bw["dh_bar"][t, c]) <= 1e-6 * max(1.0, abs(fd)), (t, c, fd, bw["dh_bar"][t, c])
+    for t in range(T):
+        e = np.zeros(T)
+        e[t] = 1.0
+        fd = ho.directional_derivative(lambda hh: loss(gg=g + hh * e), eps)
+        assert abs(fd - bw["dg"][t]) <= 1e-6 * max(1.0, abs(fd)), t
+    for key, gk in (("ad_w1", "dW1"), ("ad_w2", "dW2")):
+        V = rng.standard_normal(wl[key].shape)
+
+        def f(hh, key=key, V=V):
+            wl2 = dict(wl)
+            wl2[key] = wl[key] + hh * V
+            return loss(wl_=wl2)
+        fd = ho.directional_derivative(f, eps)
+        assert abs(fd - float(np.sum(bw[gk] * V))) <= 1e-6 * max(1.0, abs(fd)), key
+
+
+def test_skip_penalty_grad_matches_differences():
+    rng = np.random.default_rng(4)
+    n_dense, L, B, S = 2, 5, 3, 4
+    g = rng.uniform(0.05, 0.95, size=(L, B * S))
+    grad = ho.skip_penalty_grad(g, B, S, n_dense)
+    V = rng.standard_normal(g.shape)
+    fd = ho.directional_derivative(lambda hh: ho.skip_penalty(g + hh * V, B, S, n_dense), 1e-6)
+    assert abs(fd - float(np.sum(grad * V))) < 1e-8
