@@ -19,6 +19,12 @@
  * sublayer of Eq. 1.  Per-token memory S, zeta and path state are created and
  * zeroed inside every call (one forward pass, Sec. 3.2).
  *
+ * Beyond the stack: hero_routed_block runs one block on a caller's own h_bar;
+ * hero_attn_init / hero_attention_block / hero_decoder_forward add the real
+ * attention sublayer of Eq. 1 (the full decoder forward); hero_kv_cache_init /
+ * hero_decoder_prefill / hero_decode_step run it incrementally over a KV cache;
+ * hero_gemm_bf16_splitk_noalloc is an allocation-free tensor-core GEMM.
+ *
  * Conventions
  *   - Every function returns hero_status; nothing aborts or exits.  On failure
  *     hero_last_error() returns a thread-local message.
