@@ -11,6 +11,7 @@ plausible mistakes in the oracle and shows that a pin catches each one.
 """
 
 import math
+import struct
 
 import numpy as np
 import pytest
@@ -411,17 +412,68 @@ def test_p7_budget_tiny():
 # P8: independent per-token, per-element pure-Python restatement (tiny shapes)
 # ---------------------------------------------------------------------------
 
-def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
+def _bf16_bits(x: float) -> float:
+    """Scalar round-to-nearest-even to bf16 from the float64 bit pattern: keep the sign,
+    the 11 exponent bits and the top 7 of the 52 fraction bits, rounding on the 45
+    dropped bits (ties to an even kept part; a carry moves into the exponent).
+    Independent of the oracle's frexp-based bf16_round; normal bf16 range only."""
+    if x == 0.0:
+        return x
+    b = struct.unpack("<Q", struct.pack("<d", x))[0]
+    sign, mag = b & (1 << 63), b & ((1 << 63) - 1)
+    assert (mag >> 52) >= 1023 - 126, "bf16 subnormals are outside these tests"
+    keep, rest = mag >> 45, mag & ((1 << 45) - 1)
+    if rest > (1 << 44) or (rest == (1 << 44) and keep & 1):
+        keep += 1
+    return struct.unpack("<d", struct.pack("<Q", sign | (keep << 45)))[0]
+
+
+def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0, bf16=False):
     """Per-token loops over scalars, written from Sec. 3 without numpy linear algebra.
     The first n_dense layers are plain FFN blocks (Sec. 4.1 placement); the rest are
     routed blocks j = 1 .. L - n_dense.  variant: the Sec. 4.4 ablations, bits
     1 = w/o History (g from the local logit), 2 = w/o MemRead (c = 0, nu = 0, no
-    memory), 4 = w/o Aux State (z_a = 0), 8 = w/o Pos State (r, q_rem, d, gamma = 0)."""
+    memory), 4 = w/o Aux State (z_a = 0), 8 = w/o Pos State (r, q_rem, d, gamma = 0).
+    bf16: the bf16 models' precision contract (parameters already bf16 values), a
+    bf16 rounding r() at exactly these points: the router contraction's weight
+    r(W_hd[o][i] g_r[i]) with its 1/rms row scale applied after the sum; the router's
+    d-wide activation (encoder and f_psi's first layer) as the pair r(x) + r(x - r(x));
+    u = LN_ffn(h_bar); the SwiGLU product; the adapter hidden SiLU(W_1 u)."""
     L, d = cfg.n_layers, cfg.d_model
     LR = L - n_dense
+    r = _bf16_bits if bf16 else (lambda x: x)
+
+    def pair(x):
+        hi_ = r(x)
+        return hi_ + r(x - hi_)
 
     def mv(M, x):
         return [sum(M[o][i] * x[i] for i in range(len(x))) for o in range(len(M))]
+
+    def ffn(layer, u):
+        gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
+        return mv(W["w_down"][layer - 1], [r(sl(x) * z) for x, z in zip(gt, up)])
+
+    def adp(layer, u):
+        return mv(W["ad_w2"][layer - 1], [r(sl(x)) for x in mv(W["ad_w1"][layer - 1], u)])
+
+    def ln_ffn(layer, hb):
+        rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+        return [r(hb[i] / rf * W["ffn_norm_g"][layer - 1][i]) for i in range(d)]
+
+    def f_psi(hb):
+        xp = [pair(x) for x in hb] if bf16 else hb
+        hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], xp), W["ps_b1"])]
+        return sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0]
+
+    def encoder_pre(hb):
+        rms = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
+        if not bf16:
+            nr = [hb[i] / rms * W["r_norm_g"][i] for i in range(d)]
+            return mv(W["w_hd"], nr)
+        xp = [pair(x) for x in hb]
+        return [sum(r(W["w_hd"][o][i] * W["r_norm_g"][i]) * xp[i] for i in range(d)) / rms
+                for o in range(len(W["w_hd"]))]
 
     def sg(x):
         return 1.0 / (1.0 + math.exp(-x))
@@ -445,25 +497,19 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
         for layer in range(1, L + 1):
             hb = [h[i] + P[layer - 1][t][i] for i in range(d)]
             if layer <= n_dense:
-                rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
-                u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
-                gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
-                y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
+                y = ffn(layer, ln_ffn(layer, hb))
                 h = [hb[i] + y[i] for i in range(d)]
                 gs.append(1.0)
                 continue
             j = layer - n_dense
             if variant & 1:                                    # w/o History
-                hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], hb), W["ps_b1"])]
-                g = sg(sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0])
-                rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
-                u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
+                g = sg(f_psi(hb))
+                u = ln_ffn(layer, hb)
                 if g >= tau:
-                    gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
-                    y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
+                    y = ffn(layer, u)
                     h = [hb[i] + g * y[i] for i in range(d)]
                 else:
-                    y = mv(W["ad_w2"][layer - 1], [sl(x) for x in mv(W["ad_w1"][layer - 1], u)])
+                    y = adp(layer, u)
                     h = [hb[i] + (1 - g) * y[i] for i in range(d)]
                 gs.append(g)
                 continue
@@ -475,9 +521,7 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
             gam = 0.0
             if j > 2:
                 gam = sum(dl[i] * dl_prev[i] for i in range(d)) / (dd * d_prev + cfg.eps)
-            rms = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
-            nr = [hb[i] / rms * W["r_norm_g"][i] for i in range(d)]
-            zh = mv(W["w_hu"], [sl(x) for x in mv(W["w_hd"], nr)])
+            zh = mv(W["w_hu"], [sl(x) for x in encoder_pre(hb)])
             xp = [j / LR, (LR - j) / LR, dd, gam, p_prev, m_prev]
             if variant & 8:                                    # w/o Pos State
                 xp = [0.0, 0.0, 0.0, 0.0, p_prev, m_prev]
@@ -504,9 +548,7 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
             a = sum(x * y for x, y in zip(W["th_w2"][0], hh)) + W["th_b2"][0]
             p = sg(a / cfg.t_hist)
             m = m_prev * p
-            hl = [sl(x + b) for x, b in zip(mv(W["ps_w1"], hb), W["ps_b1"])]
-            bb = sum(x * y for x, y in zip(W["ps_w2"][0], hl)) + W["ps_b2"][0]
-            g = sg(a + bb)
+            g = sg(a + f_psi(hb))
             rho = sg(W["eta"][layer - 1])
             for mm in range(dm):
                 for n in range(dm):
@@ -515,14 +557,12 @@ def _py_stack(cfg, W, h_in, P, tau, n_dense=0, variant=0):
             if variant & 2:                                    # the memory stays empty
                 S = [[0.0] * dm for _ in range(dm)]
                 Z = [0.0] * dm
-            rf = math.sqrt(sum(x * x for x in hb) / d + cfg.rms_eps)
-            u = [hb[i] / rf * W["ffn_norm_g"][layer - 1][i] for i in range(d)]
+            u = ln_ffn(layer, hb)
             if g >= tau:
-                gt, up = mv(W["w_gate"][layer - 1], u), mv(W["w_up"][layer - 1], u)
-                y = mv(W["w_down"][layer - 1], [sl(x) * z for x, z in zip(gt, up)])
+                y = ffn(layer, u)
                 h = [hb[i] + g * y[i] for i in range(d)]
             else:
-                y = mv(W["ad_w2"][layer - 1], [sl(x) for x in mv(W["ad_w1"][layer - 1], u)])
+                y = adp(layer, u)
                 h = [hb[i] + (1 - g) * y[i] for i in range(d)]
             gs.append(g)
             hb_prev, dl_prev, d_prev, p_prev, m_prev = hb, dl, dd, p, m
@@ -586,6 +626,149 @@ def test_p8_placement_dense_prefix_restatement():
     np.testing.assert_allclose(got["h_out"], ref_h, rtol=0, atol=1e-12)
     assert (got["mask"][:2] == 1).all() and 0 < got["mask"][2:].sum() < got["mask"][2:].size
     assert ho.bypass_fraction(got["mask"], n_dense=2) == 1.0 - got["mask"][2:].mean()
+
+
+def test_bf16_bits_rounding_matches_torch():
+    """The restatement's own bf16 rounding against torch's conversion (values that are
+    float32-representable, so torch's path through float32 rounds once) and exact ties."""
+    rng = np.random.default_rng(9)
+    x = (rng.standard_normal(3000) * 10.0 ** rng.integers(-20, 20, 3000)).astype(np.float32)
+    ties = (np.arange(1, 300, dtype=np.float64) * 2.0 + 1.0) * 2.0 ** -8 + 1.0
+    for v in (x.astype(np.float64), ties, -ties):
+        ref = torch.tensor(v, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+        got = np.array([_bf16_bits(float(a)) for a in v])
+        np.testing.assert_array_equal(got, ref)
+
+
+def _micro_bf16(seed=17, n_layers=3):
+    cfg = hi.StackConfig("micro", n_layers, 8, 12, 4, 4, 6, "bf16", 0.3, d_h=3, d_a=2, d_enc=5,
+                         d_head=6, d_path=3, seed=seed)
+    w, h, P = _inputs(cfg)
+    W = {k: hi.to_f64(v).tolist() for k, v in w.items()}
+    oc = ho.OracleConfig.from_stack(cfg)
+    tau = float(np.median(ho.routed_ffn_stack(oc, w, h, P, 0.0)["gate"]))   # both branches
+    return cfg, oc, w, h, P, W, tau
+
+
+def _bf16_restatement_agrees(oc, w, h, P, W, tau, cfg, n_dense=0):
+    got = ho.routed_ffn_stack(oc, w, h, P, tau)
+    ref_h, ref_g = _py_stack(cfg, W, hi.to_f64(h).tolist(), hi.to_f64(P).tolist(), tau,
+                             n_dense=n_dense, bf16=True)
+    return (np.max(np.abs(got["gate"] - ref_g)) <= 1e-12 and
+            np.max(np.abs(got["h_out"] - ref_h)) <= 1e-12, got)
+
+
+@pytest.mark.parametrize("n_dense", [0, 1])
+def test_p8_bf16_precision_contract_restatement(n_dense):
+    """The bf16 models' rounding points (router weight W_hd diag(g_r), the router's
+    activation pair in the encoder and in f_psi, u, the SwiGLU product, the adapter
+    hidden) in the oracle's bf16 mode equal the per-element restatement, which takes
+    them from the contract with its own bf16 rounding; and the rounding matters (the
+    unrounded stack differs)."""
+    cfg, oc, w, h, P, W, tau = _micro_bf16(n_layers=3 + n_dense)
+    oc.n_dense = n_dense
+    ok, got = _bf16_restatement_agrees(oc, w, h, P, W, tau, cfg, n_dense)
+    assert ok
+    m = got["mask"][n_dense:]
+    assert 0 < m.sum() < m.size                      # both branches exercised
+    unrounded = ho.routed_ffn_stack(ho.OracleConfig(**{**oc.__dict__, "dtype": "f32"}), w, h, P, tau,
+                                    mode="force", mask_in=got["mask"])
+    assert np.max(np.abs(unrounded["h_out"] - got["h_out"])) > 1e-7   # far above 1e-12
+
+
+def test_bf16_planted_mistakes_are_caught(monkeypatch):
+    """Each plausible slip in the bf16 contract makes the restatement disagree."""
+    cfg, oc, w, h, P, W, tau = _micro_bf16()
+    assert _bf16_restatement_agrees(oc, w, h, P, W, tau, cfg)[0]
+    plants = {
+        # f_psi reads a single bf16 rounding of h_bar instead of the pair
+        "local_head": lambda f: (lambda hb, ww, Rx: f(hb, ww, ho.bf16_round)),
+        # the encoder weight W_hd diag(g_r) left unrounded
+        "hidden_encoder": lambda f: (lambda hb, ww, c, R, Rx: f(hb, ww, c, ho._identity, Rx)),
+        # the SwiGLU product enters W_down unrounded
+        "swiglu_ffn": lambda f: (lambda u, wl, R: f(u, wl, ho._identity)),
+        # the adapter hidden enters W_2 unrounded
+        "adapter": lambda f: (lambda u, wl, R: f(u, wl, ho._identity)),
+    }
+    for name, make in plants.items():
+        with monkeypatch.context() as mp:
+            mp.setattr(ho, name, make(getattr(ho, name)))
+            assert not _bf16_restatement_agrees(oc, w, h, P, W, tau, cfg)[0], name
+
+
+def _py_attention(h, wa, H, Hkv, theta, n_seqs, S, eps, bf16):
+    """Eq. 1's attention sublayer per element (Llama form), bf16 rounding r() at LN_attn(h),
+    q and k after RoPE, v, the normalised probabilities and the attention output."""
+    r = _bf16_bits if bf16 else (lambda x: x)
+    T, d = len(h), len(h[0])
+    hd = d // H
+    half = hd // 2
+
+    def mv(M, x):
+        return [sum(M[o][i] * x[i] for i in range(len(x))) for o in range(len(M))]
+
+    x = []
+    for t in range(T):
+        rms = math.sqrt(sum(v * v for v in h[t]) / d + eps)
+        x.append([r(h[t][i] / rms * wa["attn_norm_g"][i]) for i in range(d)])
+    Q, K, V = [mv(wa["w_q"], xt) for xt in x], [mv(wa["w_k"], xt) for xt in x], \
+        [mv(wa["w_v"], xt) for xt in x]
+
+    def rope(vec, pos):
+        out = list(vec)
+        for i in range(half):
+            ang = pos * theta ** (-2.0 * i / hd)
+            c, sn = math.cos(ang), math.sin(ang)
+            out[i] = vec[i] * c - vec[i + half] * sn
+            out[i + half] = vec[i + half] * c + vec[i] * sn
+        return out
+
+    out = []
+    for t in range(T):
+        b, pos = divmod(t, S)
+        o = []
+        for hh in range(H):
+            kv = hh // (H // Hkv)
+            q = [r(z) for z in rope(Q[t][hh * hd:(hh + 1) * hd], pos)]
+            sc = []
+            for p2 in range(pos + 1):
+                t2 = b * S + p2
+                k = [r(z) for z in rope(K[t2][kv * hd:(kv + 1) * hd], p2)]
+                sc.append(sum(qi * ki for qi, ki in zip(q, k)) / math.sqrt(hd))
+            mx = max(sc)
+            e = [math.exp(z - mx) for z in sc]
+            tot = sum(e)
+            pr_ = [r(z / tot) for z in e]
+            for c in range(hd):
+                o.append(r(sum(pr_[p2] * r(V[b * S + p2][kv * hd + c]) for p2 in range(pos + 1))))
+        y = mv(wa["w_o"], o)
+        out.append([h[t][i] + y[i] for i in range(d)])
+    return np.array(out)
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_attention_restatement_with_precision_points(bf16, monkeypatch):
+    """attention_sublayer (f32, and bf16 at R28's rounding points) equals the per-element
+    restatement on micro shapes; a planted slip (q and k rounded before RoPE as well) is
+    caught."""
+    rng = np.random.default_rng(21)
+    n_seqs, S, H, Hkv, d, theta = 2, 5, 4, 2, 16, 500000.0
+    h = rng.standard_normal((n_seqs * S, d))
+    wa = {"attn_norm_g": 1 + 0.02 * rng.standard_normal(d),
+          "w_q": 0.3 * rng.standard_normal((d, d)), "w_k": 0.3 * rng.standard_normal((d // 2, d)),
+          "w_v": 0.3 * rng.standard_normal((d // 2, d)), "w_o": 0.3 * rng.standard_normal((d, d))}
+    if bf16:
+        wa = {k: ho.bf16_round(v) for k, v in wa.items()}
+    R = ho.bf16_round if bf16 else None
+    got = ho.attention_sublayer(h, wa, H, Hkv, theta, n_seqs, S, 1e-5, R)
+    ref = _py_attention(h.tolist(), {k: v.tolist() for k, v in wa.items()}, H, Hkv, theta, n_seqs,
+                        S, 1e-5, bf16)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+    if bf16:
+        orig = ho.apply_rope
+        monkeypatch.setattr(ho, "apply_rope", lambda x, c, s_: orig(ho.bf16_round(x), c, s_))
+        planted = ho.attention_sublayer(h, wa, H, Hkv, theta, n_seqs, S, 1e-5, R)
+        assert np.max(np.abs(planted - ref)) > 1e-9
 
 
 # ---------------------------------------------------------------------------
