@@ -1,7 +1,7 @@
 """Throughput of the routed FFN stack on GB300 (one JSON line on rank 0).
 
 python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                [--workload NAME] [--cpu-sample N] [--no-cpu-baseline]
+                [--workload NAME] [--bypass B] [--cpu-sample N] [--no-cpu-baseline]
 
 A step is one pass of the whole routed FFN stack (all routed blocks: memory
 readout, router score, compaction, FFN / adapter, scatter into the residual,
@@ -9,7 +9,8 @@ memory update) over the workload's T tokens.  Inputs (weights 11.3 GB, the
 attention stand-in 4.3 GB) are far larger than the 129 MB L2, so no flush is
 needed between steps.  With N > 1 ranks (torchrun), every rank runs its own
 token shard of the same size on its own GPU (weak scaling, no collective on the
-data path); value = all ranks' tokens / the slowest rank's time.
+data path); value = all ranks' tokens / the slowest rank's time.  Without an outside
+launcher, --gpus N > 1 starts the N ranks itself (torch.distributed.run).
 
 Decoder workloads (--workload llama31_8b_decoder, small_bf16_decoder) run the full
 decoder forward instead: every block's h_bar comes from the real attention
@@ -54,11 +55,11 @@ def metric_for(cfg):
     return METRIC_DECODER if cfg.n_heads else METRIC
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# DRAM bytes (read + write) per launch of the dominant kernel, from one ncu capture of the
-# default workload with the current kernels (profiles/launches_llama31_8b_prefill.md);
-# reported only for that unmodified workload, and to be reset to None whenever the kernel
-# changes before it is captured again.
-DOMINANT_TRAFFIC = {("llama31_8b_prefill", "ffn_gate_up"): 1957.2e6}
+# DRAM bytes (read + write) per launch of the dominant kernel at the default workload,
+# taken from a single-kernel ncu capture of a smaller case of the same kernel and scaled
+# to the full launch by the FFN rows it processes; reported only for the unmodified
+# default workload, and emptied whenever the kernel changes before it is captured again.
+DOMINANT_TRAFFIC = {("llama31_8b_prefill", "ffn_gate_up"): 1901.0e6}
 
 
 def load_peaks():
@@ -230,7 +231,9 @@ def reference_arm(args, rank, world):
         return
     from oracle import hero_oracle as ho
     cfg = hi.CONFIGS[args.workload]
-    tau = hi.calibrated_tau(cfg.name)
+    if args.bypass is not None:
+        cfg = cfg.replace(bypass=args.bypass)
+    tau = hi.calibrated_tau(cfg.name, args.bypass)
     w = hi.generate_weights(cfg)
     step, rows, sample = oracle_step(ho, cfg, w, hi.generate_h_in(cfg), tau, args.cpu_sample)
     for _ in range(args.warmup):
@@ -250,6 +253,97 @@ def reference_arm(args, rank, world):
                              "sample": f"{len(rows)} tokens x {cfg.n_layers} blocks per step"},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def backward_flops(cfg, counts):
+    """Algorithmic FLOPs of the training path's block backwards (decisions fixed): per FFN
+    token the gate/up recomputation (4 I d), e = G W_down (2 I d) and du = [dgate|dup]
+    [W_gate|W_up] (4 I d); per adapter token W_1 u, G W_2, da W_1 and the two weight
+    gradients (2 d d_r each)."""
+    T, d, I, r = cfg.n_tokens, cfg.d_model, cfg.d_ff, cfg.d_r
+    nf = np.asarray(counts, dtype=np.float64)[cfg.n_dense:]
+    return {"backward_gemm": float(np.sum(10.0 * nf * I * d + 6.0 * (T - nf) * d * r)),
+            "wgrad": float(np.sum(4.0 * (T - nf) * d * r))}
+
+
+def backward_arm(args, cfg, stack, hero, h, P, tau, stream, dev, world, rank, timed, sampler, t_gen):
+    """Training-path step: the backward of every routed block's branch part (Sec. 3.1,
+    Sec. 3.3) over the workload's T tokens, with the gates and decisions of one forward
+    pass fixed, a seeded upstream gradient G and h_bar = the stack's input (the cost does
+    not depend on the values).  Metric: tokens per second of one such pass."""
+    import torch
+    T, d, L, r = cfg.n_tokens, cfg.d_model, cfg.n_layers, cfg.d_r
+    _, gate, mask, counts = stack(h, P, tau)
+    torch.cuda.synchronize()
+    stack.backward_init()
+    G = torch.randn((T, d), device=dev, generator=torch.Generator(device=dev).manual_seed(3))
+    gh = torch.empty((T, d), device=dev)
+    gg = torch.empty((L, T), device=dev)
+    g1 = torch.empty((L, r, d), device=dev)
+    g2 = torch.empty((L, d, r), device=dev)
+    blocks = range(cfg.n_dense + 1, L + 1)
+
+    def step():
+        for j in blocks:
+            hero.hero_routed_block_backward(stack.model, j, T, h.data_ptr(), gate[j - 1].data_ptr(),
+                                            mask[j - 1].data_ptr(), G.data_ptr(), 0, gh.data_ptr(),
+                                            gg[j - 1].data_ptr(), g1[j - 1].data_ptr(),
+                                            g2[j - 1].data_ptr(), stream.cuda_stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    stack.check()
+    ms, clocks = timed(step, args.steps, sampler)
+    stack.check()
+    hero.hero_get_profile(stack.model, reset=True)
+    hero.hero_set_profiling(stack.model, True)
+    timed(step, args.steps)
+    hero.hero_set_profiling(stack.model, False)
+    prof = hero.hero_get_profile(stack.model, reset=True)
+    stack.check()
+    cnt = counts.cpu().numpy().astype(np.int64)
+    work = backward_flops(cfg, cnt)
+    peaks, peak_src = load_peaks()
+    peak_tf = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    bms, bn = prof["backward_gemm"]
+    achieved = work["backward_gemm"] * args.steps / (bms / 1e3) / 1e12 if bms else None
+    value = world * T * args.steps / (ms / 1e3)
+    line = {
+        "metric": "routed-block backward (decisions fixed) tokens/s at the workload's shapes",
+        "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+        "config": {"workload": workload_desc(cfg, cfg.bypass) + "; backward of every routed block",
+                   "l2": "inputs larger than L2 (no flush): weights stream from HBM each block"},
+        "roofline": {"kernel": "backward_gemm", "bound": "tensor", "achieved": achieved,
+                     "peak": peak_tf, "unit": "TFLOP/s",
+                     "frac": achieved / peak_tf if achieved else None, "traffic": None,
+                     "peak_source": f"{peak_src} bf16_tflops_sustained",
+                     "avg_launch_ms": bms / max(bn, 1)},
+        "gpu_launches": int(sum(n for _, n in prof.values())),
+        "clocks": clocks, "bypass": 1.0 - cnt[cfg.n_dense:].sum() / ((L - cfg.n_dense) * T),
+        "ffn_counts": cnt.tolist(),
+        "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items() if v[1]},
+        "setup_s": {"generate": t_gen},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    stack.close()
+    return 0
+
+
+def launch_ranks(n: int) -> int:
+    """--gpus N without an outside launcher: run this script again as N ranks of one node
+    under torch.distributed.run (127.0.0.1 rendezvous on a free port); rank 0 prints."""
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr=127.0.0.1", f"--master-port={port}", os.path.abspath(__file__),
+           *sys.argv[1:]]
+    return subprocess.call(cmd)
 
 
 def main():
@@ -272,12 +366,22 @@ def main():
     ap.add_argument("--d-m", type=int, default=None, help="memory width override (ablation)")
     ap.add_argument("--graph", action="store_true",
                     help="time CUDA-graph replays of one captured step (launch-bound decode)")
+    ap.add_argument("--backward", action="store_true",
+                    help="time the training path instead: every routed block's backward with "
+                         "the decisions of one forward pass fixed")
+    ap.add_argument("--bypass", type=float, default=None,
+                    help="bypass target whose committed tau to use (e.g. 0, 0.27, 0.39 for "
+                         "llama2_13b_prefill); default: the workload's own")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
+    if "WORLD_SIZE" not in os.environ and args.gpus > 1 and args.impl == "ours":
+        return launch_ranks(args.gpus)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and args.gpus != world:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={world}")
     if args.impl == "reference":
         return reference_arm(args, rank, world)
 
@@ -296,18 +400,22 @@ def main():
     hero.load()
 
     cfg = hi.CONFIGS[args.workload]
-    tau = hi.calibrated_tau(cfg.name) if args.tau is None else args.tau
+    if args.bypass is not None:
+        cfg = cfg.replace(bypass=args.bypass)
+    tau = hi.calibrated_tau(cfg.name, args.bypass) if args.tau is None else args.tau
     if args.tokens or args.layers:
         cfg = cfg.replace(n_tokens=args.tokens or cfg.n_tokens, n_layers=args.layers or cfg.n_layers)
     if args.router_variant or args.d_m:   # ablations run with the workload's tau
         cfg = cfg.replace(router_variant=args.router_variant, d_m=args.d_m or cfg.d_m)
-    default_shape = cfg == hi.CONFIGS[args.workload] and args.tau is None
+    default_shape = cfg == hi.CONFIGS[args.workload] and args.tau is None and args.bypass is None
     T, d, L = cfg.n_tokens, cfg.d_model, cfg.n_layers
     decoder = bool(cfg.n_heads)
     kvdec = bool(cfg.kv_decode_of)
     if decoder and not kvdec and args.tokens:
         cfg = cfg.replace(batch=max(1, cfg.n_tokens // cfg.seq_len))
     B, S = cfg.batch, cfg.seq_len
+    if args.backward and (decoder or cfg.dtype != "bf16"):
+        raise SystemExit("--backward runs on the bf16 routed-stack workloads")
     if kvdec and B != T:
         raise SystemExit(f"KV decoding workload needs T = batch ({B} != {T})")
     if decoder and not kvdec and B * S != T:
@@ -384,6 +492,10 @@ def main():
         barrier()
         clk = sampler.stop() if sampler else None
         return max_over_ranks(e0.elapsed_time(e1)), clk
+
+    if args.backward:
+        return backward_arm(args, cfg, stack, hero, h, P, tau, stream, dev, world, rank, timed,
+                            ClockSampler(local_rank), t_gen)
 
     # ---- routed stack (the metric) ----
     for _ in range(args.warmup):
@@ -537,4 +649,4 @@ def main():
 
 
 if __name__ == "__main__":
-    main()
+    sys.exit(main() or 0)

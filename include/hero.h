@@ -23,7 +23,9 @@
  * hero_attn_init / hero_attention_block / hero_decoder_forward add the real
  * attention sublayer of Eq. 1 (the full decoder forward); hero_kv_cache_init /
  * hero_decoder_prefill / hero_decode_step run it incrementally over a KV cache;
- * hero_gemm_bf16_splitk_noalloc is an allocation-free tensor-core GEMM.
+ * hero_backward_init / hero_routed_block_backward / hero_skip_penalty_grad give the
+ * training path's gradients (Sec. 3.1, 3.3); hero_gemm_bf16_splitk_noalloc is an
+ * allocation-free tensor-core GEMM.
  *
  * Conventions
  *   - Every function returns hero_status; nothing aborts or exits.  On failure
@@ -33,8 +35,9 @@
  *     HERO_FLAG_HOST_IO); all tensors are dense row-major.
  *   - Execution is asynchronous on the given CUDA stream (cudaStream_t, NULL =
  *     legacy default stream).  Kernels never spin without a bound: a wait that
- *     expires (about 4 s) sets a device error word that hero_check_device_status
- *     reports as HERO_ERR_TIMEOUT.
+ *     expires (4 s by default, hero_set_wait_limit_ns) sets a device error word
+ *     that hero_check_device_status reports as HERO_ERR_TIMEOUT; an out-of-range
+ *     index found on the device is reported as HERO_ERR_BAD_INDEX.
  *   - A model may be used by one host thread at a time.
  */
 #ifndef HERO_H_
@@ -52,7 +55,10 @@ typedef enum {
   HERO_ERR_CUDA = 2,         /* a CUDA runtime call failed                      */
   HERO_ERR_NOMEM = 3,        /* device or host allocation failed                */
   HERO_ERR_UNSUPPORTED = 4,  /* shape or dtype outside what the kernels support */
-  HERO_ERR_TIMEOUT = 5       /* a device-side bounded wait expired              */
+  HERO_ERR_TIMEOUT = 5,      /* a device-side bounded wait expired              */
+  HERO_ERR_BAD_INDEX = 6     /* a kernel met an index outside its bounds (e.g. a
+                                decoding position past the cache); the offending
+                                accesses were skipped                           */
 } hero_status;
 
 typedef enum { HERO_F32 = 0, HERO_BF16 = 1 } hero_dtype;
@@ -210,10 +216,21 @@ void hero_free(hero_model* m);
 /* Message of the last failure on this host thread ("" if none). */
 const char* hero_last_error(void);
 
-/* Synchronize cuda_stream, then report HERO_ERR_TIMEOUT if any kernel of this
- * model hit its wait bound since the last check (and clear the record), or
- * HERO_ERR_CUDA if the stream holds a CUDA error. */
+/* Synchronize cuda_stream, then report what the model's kernels recorded since the
+ * last check (and clear the record): HERO_ERR_TIMEOUT if any wait hit its bound
+ * (the outputs of that call are incomplete), else HERO_ERR_BAD_INDEX if a kernel
+ * met an out-of-range index; HERO_ERR_CUDA if the stream holds a CUDA error. */
 hero_status hero_check_device_status(hero_model* m, void* cuda_stream);
+
+/* Bound, in nanoseconds of the GPU's global timer, on every device-side wait of the
+ * kernels enqueued after this call (process-wide; 0 restores the default of 4 s).
+ * A wait that reaches it gives up: the kernel lets its copies and tensor-core work
+ * in flight finish (a separate 100 ms bound), records the expiry in its error word
+ * (reported as HERO_ERR_TIMEOUT) and returns without completing its outputs.  The
+ * bound is read when a kernel is enqueued, so a captured CUDA graph keeps the bound
+ * of its capture.  Meant for tests of the timeout path; lowering it in production
+ * turns slow waits into failures. */
+void hero_set_wait_limit_ns(uint64_t limit_ns);
 
 /* ---- the full decoder forward: real attention in Eq. 1 -----------------------
  * Eq. 1 gives each routed block the representation after attention,
@@ -306,6 +323,52 @@ hero_status hero_decode_step(hero_model* m, int32_t n_seqs, const int32_t* posit
                              uint32_t flags, const uint8_t* mask_in, float* h_out, float* gate_out,
                              uint8_t* mask_out, int32_t* ffn_count_out, void* cuda_stream);
 
+/* ---- training path: gradients with the decisions fixed -------------------------
+ * Sec. 3.1 keeps the routing threshold out of differentiation: the selected branch's
+ * scale (g for the FFN, 1 - g for the adapter) carries the gradient to the router,
+ * and Sec. 3.3 trains the adapters and the router against the language-model loss
+ * plus alpha L_skip with the backbone (FFN, LN_ffn) frozen.  These calls give the
+ * branch part of a routed block's backward and L_skip's gradient; the router's own
+ * backward (memory recurrence, path features, heads) is not part of them.
+ *
+ * Build the backward's operands for a bf16 model: transposed copies of every block's
+ * W_down, W_gate|W_up and adapter weights (3 d I + 2 d d_r bf16 per block) and a
+ * workspace for max_tokens.  Synchronous; once per model (HERO_ERR_ARG on a second
+ * call); HERO_ERR_UNSUPPORTED for f32 models. */
+hero_status hero_backward_init(hero_model* m);
+
+/* Backward of block `block` (1..n_layers) with its decisions fixed, for
+ *   h = h_bar + s Branch(u),  u = LN_ffn(h_bar)                        (Eqs. 1-3)
+ * s = g and Branch = FFN (SwiGLU) where mask != 0, s = 1 - g and Branch = W_2 SiLU(W_1 u)
+ * (Eq. 2) elsewhere.  DEVICE pointers, fp32, row-major, T = n_tokens <= max_tokens:
+ *   h_bar [T,d], gate [T] (g), mask [T] (the forward's decisions), grad_out [T,d] = dL/dh
+ *   -> grad_h_bar [T,d] = dL/dh_bar (residual plus branch), grad_gate [T] = dL/dg,
+ *      grad_w1 [d_r,d] = dL/dW_1, grad_w2 [d,d_r] = dL/dW_2 of this block's adapter
+ *      (sums over the adapter tokens; zero when there are none).
+ * HERO_FLAG_DENSE (and blocks 1..n_dense): every token through the FFN with scale 1;
+ * gate, mask may be NULL and grad_gate / grad_w1 / grad_w2, if given, are zeroed.
+ * Precision: bf16 GEMM operands (u and the forward's bf16 rounding points, G, the
+ * SwiGLU gradients dgate|dup, da), fp32 accumulation, fp32 row-wise and weight-gradient
+ * arithmetic.  grad_h_bar must not alias h_bar or grad_out.  Needs hero_backward_init.
+ * Asynchronous on cuda_stream (no host synchronisation); uses the model's forward
+ * workspace, so it does not overlap a forward call of the same model. */
+hero_status hero_routed_block_backward(hero_model* m, int32_t block, int64_t n_tokens,
+                                       const float* h_bar, const float* gate, const uint8_t* mask,
+                                       const float* grad_out, uint32_t flags, float* grad_h_bar,
+                                       float* grad_gate, float* grad_w1, float* grad_w2,
+                                       void* cuda_stream);
+
+/* Gradient of the skip penalty (Sec. 3.3) with respect to the gates, times alpha:
+ * L_skip = 1 / (B (S - 1)) sum over sequences b and next-token positions t < S - 1 of
+ * (sum_j g_{j,b,t})^2, the sum over the routed blocks j (rows n_dense.. of gates).
+ * gates [n_layers, B S] (tokens in sequence order) -> grad_gates [n_layers, B S] =
+ * alpha dL_skip/dg: 2 alpha / (B (S - 1)) sum_j g_{j,b,t} for t < S - 1, 0 at each
+ * sequence's last position and in the dense-prefix rows.  DEVICE pointers, not
+ * aliased; seq_len >= 2.  Asynchronous on cuda_stream. */
+hero_status hero_skip_penalty_grad(int32_t n_layers, int32_t n_dense, int32_t n_seqs,
+                                   int32_t seq_len, const float* gates, float alpha,
+                                   float* grad_gates, void* cuda_stream);
+
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes of one block, for per-kernel timing. */
 enum {
@@ -321,7 +384,9 @@ enum {
   HERO_K_ADAPTER_UP = 8,  /* adapter W_2 GEMM with the scaled scatter epilogue */
   HERO_K_ATTN_PROJ = 9,   /* LN_attn, q/k/v projection, RoPE, output projection */
   HERO_K_ATTN_CORE = 10,  /* causal softmax attention                           */
-  HERO_K_COUNT = 11
+  HERO_K_BACKWARD_GEMM = 11, /* training path: the tensor-core GEMMs of a block's backward */
+  HERO_K_BACKWARD = 12,   /* training path: compaction, row and reduction kernels */
+  HERO_K_COUNT = 13
 };
 
 /* When enabled, every later launch of the model is bracketed by CUDA events on
@@ -335,7 +400,9 @@ hero_status hero_get_profile(hero_model* m, double* ms_out, int64_t* launches_ou
 /* Building-block check of the tensor-core GEMM: C[M,N] (fp32) = A[M,K] B[N,K]^T
  * with A, B bf16 (uint16 bit patterns), DEVICE pointers, row-major, K % 64 == 0,
  * K and N multiples of 8 elements.  Not part of the routed stack's contract;
- * exposed so the GEMM core can be tested alone. */
+ * exposed so the GEMM core can be tested alone.  Synchronous: waits for
+ * cuda_stream, then returns HERO_ERR_TIMEOUT if the kernel's wait bound expired
+ * (C incomplete) or HERO_ERR_BAD_INDEX, and clears that record (one per device). */
 hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B, float* C, int32_t M,
                                  int32_t N, int32_t K, void* cuda_stream);
 
@@ -361,10 +428,19 @@ hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B, float* C,
  *   - Every call shares the static arrays and the arrays keep the last call's
  *     contents; calls that overlap on the GPU (other streams, other host
  *     threads) race on them.  Serialise calls on one stream.
- *   - Asynchronous on cuda_stream like the other entry points. */
+ *   - Asynchronous on cuda_stream like the other entry points.  An expired wait
+ *     inside the GEMM (C then incomplete) is recorded in the static error word,
+ *     which keeps it across calls until hero_gemm_bf16_splitk_noalloc_status reads
+ *     and clears it. */
 hero_status hero_gemm_bf16_splitk_noalloc(const uint16_t* A, const uint16_t* B, float* C,
                                           int32_t M, int32_t N, int32_t K, int32_t splits,
                                           void* cuda_stream);
+
+/* Status of the allocation-free GEMM calls on the current device since the last
+ * query: synchronizes cuda_stream, then returns HERO_ERR_TIMEOUT (a wait bound
+ * expired in some call; its C is incomplete), HERO_ERR_BAD_INDEX or HERO_OK, and
+ * clears the static error word.  Allocates nothing. */
+hero_status hero_gemm_bf16_splitk_noalloc_status(void* cuda_stream);
 
 #ifdef __cplusplus
 }

@@ -356,7 +356,7 @@ static_assert(SMEM <= 232448, "shared memory per CTA");
 __global__ void __launch_bounds__(fa::THREADS, 1)
     k_flash_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, int H, int Hkv, int S, int n_qt,
-               float scale_log2, uint16_t* __restrict__ O, uint32_t* err) {
+               float scale_log2, uint16_t* __restrict__ O, uint32_t* err, uint64_t wait_ns) {
   using namespace fa;
   pdl_enter();
   extern __shared__ uint8_t fa_raw[];
@@ -420,7 +420,7 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
       for (int i = 0; i < n && ok; ++i) {
         const int st = i & 1;
         const uint32_t ph = (i >> 1) & 1;
-        if (!mbar_wait(bar(K_EMPTY + st), ph ^ 1u, kWaitLimitNs) || misc[1]) {
+        if (!mbar_wait(bar(K_EMPTY + st), ph ^ 1u, wait_ns) || misc[1]) {
           ok = false;
           break;
         }
@@ -430,7 +430,7 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
         tma_load_3d(sk + PANEL, &tmK, 64, i * BN, zk, bar(K_FULL + st));
         kiss[st] = true;
         kpar[st] = ph;
-        if (!mbar_wait(bar(V_EMPTY), (i & 1) ^ 1u, kWaitLimitNs) || misc[1]) {
+        if (!mbar_wait(bar(V_EMPTY), (i & 1) ^ 1u, wait_ns) || misc[1]) {
           ok = false;
           break;
         }
@@ -440,21 +440,24 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
         viss = true;
         vpar = i & 1;
       }
-      if (!ok) {   // let copies still in flight land before the CTA can exit
+      if (!ok) {
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_PRODUCER);
-        mbar_wait(bar(Q_FULL), 0, 100000000ull);
-        for (int s = 0; s < 2; ++s)
-          if (kiss[s]) mbar_wait(bar(K_FULL + s), kpar[s], 100000000ull);
-        if (viss) mbar_wait(bar(V_FULL), vpar, 100000000ull);
       }
+      // let every copy still in flight land before the CTA can exit, also after a
+      // normal end (another role may have given up before consuming them)
+      bool drained = mbar_wait(bar(Q_FULL), 0, kDrainLimitNs);
+      for (int s = 0; s < 2; ++s)
+        if (kiss[s]) drained = mbar_wait(bar(K_FULL + s), kpar[s], kDrainLimitNs) && drained;
+      if (viss) drained = mbar_wait(bar(V_FULL), vpar, kDrainLimitNs) && drained;
+      if (!drained) atomicOr(err, ERR_WAIT_DRAIN);
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
     if (lane == 0) {
-      bool ok = mbar_wait(bar(Q_FULL), 0, kWaitLimitNs) && !misc[1];
+      bool ok = mbar_wait(bar(Q_FULL), 0, wait_ns) && !misc[1];
       auto wait = [&](int id, uint32_t par) {
-        ok = ok && mbar_wait(bar(id), par, kWaitLimitNs) && !misc[1];
+        ok = ok && mbar_wait(bar(id), par, wait_ns) && !misc[1];
         return ok;
       };
       auto issue_s = [&](int x, int i) {   // S_x(i) = Q_x K_i^T over the head dimension
@@ -509,9 +512,11 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
       if (!ok) {
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_MMA);
-        umma_commit(bar(DRAIN));
-        if (!mbar_wait(bar(DRAIN), 0, 100000000ull)) atomicOr(err, ERR_WAIT_DRAIN);
       }
+      // every issued MMA completes before TMEM is freed, also after a normal end
+      // (a softmax warp may have given up while MMAs were in flight)
+      umma_commit(bar(DRAIN));
+      if (!mbar_wait(bar(DRAIN), 0, kDrainLimitNs)) atomicOr(err, ERR_WAIT_DRAIN);
     }
   } else {
     // ------------------------------ softmax ------------------------------
@@ -524,7 +529,7 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
     float m_used = -INFINITY, l = 0.f;          // m_used in raw score units
     bool ok = true;
     for (int i = 0; i < nx; ++i) {
-      bool w = mbar_wait(bar(S_FULL + x), i & 1, kWaitLimitNs);
+      bool w = mbar_wait(bar(S_FULL + x), i & 1, wait_ns);
       w = __all_sync(0xffffffffu, w) && !misc[1];
       if (!__all_sync(0xffffffffu, w)) {
         ok = false;
@@ -591,7 +596,7 @@ __global__ void __launch_bounds__(fa::THREADS, 1)
       if (lane == 0) mbar_arrive(bar(P_FULL + x));
     }
     if (ok && nx > 0) {
-      const bool w = mbar_wait(bar(FINAL), 0, kWaitLimitNs);
+      const bool w = mbar_wait(bar(FINAL), 0, wait_ns);
       ok = __all_sync(0xffffffffu, w);
       if (ok) {
         tc_fence_after();
@@ -910,7 +915,7 @@ cudaError_t launch_flash_tc(const CUtensorMap& tmQ, const CUtensorMap& tmK, cons
   const int n_qt = (S + fa::BM - 1) / fa::BM;
   const dim3 grid((unsigned)((n_qt + 1) / 2), (unsigned)H, (unsigned)B);   // query tile pairs
   return launch_pdl(k_flash_tc, grid, dim3(fa::THREADS), fa::SMEM, st, tmQ, tmK, tmV, H, Hkv, S,
-                    n_qt, scale_log2, static_cast<uint16_t*>(O), err);
+                    n_qt, scale_log2, static_cast<uint16_t*>(O), err, wait_limit_ns());
 }
 
 }  // namespace hero

@@ -158,6 +158,87 @@ __device__ __forceinline__ void epi_silu(const GemmArgs& a, uint32_t tbase, int 
   }
 }
 
+// Plain bf16 store of the accumulator (columns past N, a multiple of 32, skipped).
+template <int BN>
+__device__ __forceinline__ void epi_store_bf16(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                               int nb) {
+  const int ncols = min(BN, a.N - nb * BN);
+#pragma unroll 1
+  for (int c0 = 0; c0 < ncols; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    if (valid) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) + (size_t)m * a.ldo +
+                                            nb * BN + c0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+    }
+  }
+}
+
+// Backward of act = SiLU(gate) up (training path, decisions fixed).  The accumulator
+// holds e = dL/dy W_down for features f = nb BN + c of compacted FFN row m, where
+// dL/dy = G (the upstream gradient; the branch scale g is applied here):
+//   dact = g e,  dgate = dact up SiLU'(gate),  dup = dact SiLU(gate),
+//   dL/dg contribution: sum_f e_f act_f with act = bf16(SiLU(gate) up), the value the
+//   forward fed to W_down.
+// gate and up (bf16 pre-activations) sit in the interleaved gate/up layout (per 128
+// features: 128 gate columns, then 128 up columns) of row m of a.out and are replaced
+// there by dgate and dup (bf16): the A operand of the input-gradient GEMM.
+template <int BN>
+__device__ __forceinline__ void epi_bw_swiglu(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                              int nb) {
+  const int ncols = min(BN, a.N - nb * BN);
+  uint16_t* row = static_cast<uint16_t*>(a.out) + (size_t)m * a.ldo;
+  const float s = valid ? a.row_scale[m] : 0.f;
+  float dgs = 0.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < ncols; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    if (valid) {
+      const int f = nb * BN + c0;   // 32 features inside one 128-feature group
+      uint4* gp = reinterpret_cast<uint4*>(row + (f >> 7) * 256 + (f & 127));
+      uint4* upp = reinterpret_cast<uint4*>(row + (f >> 7) * 256 + 128 + (f & 127));
+      uint4 gr[4], ur[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        gr[i] = gp[i];
+        ur[i] = upp[i];
+      }
+      const uint32_t* gw = reinterpret_cast<const uint32_t*>(gr);
+      const uint32_t* uw = reinterpret_cast<const uint32_t*>(ur);
+      uint32_t dgw[16], duw[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        float g0, g1, u0, u1;
+        unpack_bf16x2(gw[i], g0, g1);
+        unpack_bf16x2(uw[i], u0, u1);
+        const float e0 = __uint_as_float(r[2 * i]), e1 = __uint_as_float(r[2 * i + 1]);
+        const float s0 = sigmoidf_(g0), s1 = sigmoidf_(g1);
+        const float sl0 = g0 * s0, sl1 = g1 * s1;
+        const float a0 = __bfloat162float(__float2bfloat16_rn(sl0 * u0));
+        const float a1 = __bfloat162float(__float2bfloat16_rn(sl1 * u1));
+        dgs = fmaf(e0, a0, dgs);
+        dgs = fmaf(e1, a1, dgs);
+        const float d0 = s * e0, d1 = s * e1;
+        dgw[i] = pack_bf16x2(d0 * u0 * s0 * (1.f + g0 * (1.f - s0)),
+                             d1 * u1 * s1 * (1.f + g1 * (1.f - s1)));
+        duw[i] = pack_bf16x2(d0 * sl0, d1 * sl1);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        gp[i] = make_uint4(dgw[4 * i], dgw[4 * i + 1], dgw[4 * i + 2], dgw[4 * i + 3]);
+        upp[i] = make_uint4(duw[4 * i], duw[4 * i + 1], duw[4 * i + 2], duw[4 * i + 3]);
+      }
+    }
+  }
+  if (valid) a.row_part[(size_t)m * a.part_ld + nb] = dgs;
+}
+
 // Fused q/k/v projection epilogue: one thread = one token row; the two halves of a
 // head (columns i and i + 64) are read from TMEM together, q and k heads are
 // rotated (RoPE, fp32), and each head's 128 values are stored as bf16 into its
@@ -451,6 +532,10 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
     epi_swiglu(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_SILU) {
     epi_silu<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_STORE_BF16) {
+    epi_store_bf16<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_BW_SWIGLU) {
+    epi_bw_swiglu<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_LAYER_OUT) {
     epi_layer_out<BN, BN>(a, tbase, row0, M, nb, 0, stg);
   } else {
@@ -482,6 +567,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
   auto sA = [&](int s) { return smem_base + s * C::STAGE_BYTES; };
   auto sB = [&](int s) { return smem_base + s * C::STAGE_BYTES + C::A_BYTES; };
   uint32_t* err = a0.err;
+  const uint64_t wait_ns = a0.wait_ns;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -536,7 +622,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
         if (a0.pdl_mode == 1 && g + (int)gridDim.x >= total)   // this CTA's last tile
           asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(empty_bar(stage), phase ^ 1u, kWaitLimitNs) || misc[1]) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, wait_ns) || misc[1]) {
             ok = false;
             break;
           }
@@ -554,10 +640,13 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       if (!ok) {
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_PRODUCER);
-        // let copies still in flight land before the CTA can exit
-        for (int s = 0; s < C::STAGES; ++s)
-          if (issued & (1u << s)) mbar_wait(full_bar(s), (last_par >> s) & 1u, 100000000ull);
       }
+      // Let every copy this thread issued land before the CTA can exit, also when
+      // the loop ended normally: if another role gave up early, stages it never
+      // consumed may still be in flight.  (Normally they have landed already.)
+      for (int s = 0; s < C::STAGES; ++s)
+        if ((issued & (1u << s)) && !mbar_wait(full_bar(s), (last_par >> s) & 1u, kDrainLimitNs))
+          atomicOr(err, ERR_WAIT_DRAIN);
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
@@ -572,14 +661,14 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
         const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb, sp, kb0, kb1;
         tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
-        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, kWaitLimitNs) || misc[1]) {
+        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, wait_ns) || misc[1]) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(full_bar(stage), phase, kWaitLimitNs) || misc[1]) {
+          if (!mbar_wait(full_bar(stage), phase, wait_ns) || misc[1]) {
             ok = false;
             break;
           }
@@ -605,9 +694,11 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       if (!ok) {
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_MMA);
-        umma_commit(drain_bar);  // completes once every issued MMA has finished
-        if (!mbar_wait(drain_bar, 0, 100000000ull)) atomicOr(err, ERR_WAIT_DRAIN);
       }
+      // Every MMA this thread issued completes before TMEM is freed, also when the
+      // loop ended normally but an epilogue warp gave up on a tile still in flight.
+      umma_commit(drain_bar);  // arrives once every issued MMA has finished
+      if (!mbar_wait(drain_bar, 0, kDrainLimitNs)) atomicOr(err, ERR_WAIT_DRAIN);
     }
   } else {
     // ------------------------------ epilogue ------------------------------
@@ -620,7 +711,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       const int pr = split_tile(g, P1.tiles, total, local);
       int mb, nb, sp, kb0, kb1;
       tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
-      bool ok = mbar_wait(tfull_bar(acc), acc_phase, kWaitLimitNs);
+      bool ok = mbar_wait(tfull_bar(acc), acc_phase, wait_ns);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) {
@@ -680,8 +771,10 @@ cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const Ge
   if (EPI1 != EPI_NONE) max_tiles += (long)((a1.m_max + BM - 1) / BM) * ((a1.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
   const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
+  GemmArgs b0 = a0;
+  b0.wait_ns = wait_limit_ns();
   return launch_pdl(k_gemm_tc<BN, EPI0, EPI1>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tmA0, tmB0,
-                    tmA1, tmB1, a0, a1);
+                    tmA1, tmB1, b0, a1);
 }
 
 }  // namespace
@@ -710,6 +803,14 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
     case EPI_ATTN_ENTRY:
       if (args.lo.d != args.N || args.ldo != args.N) return cudaErrorInvalidValue;
       return launch_tc<256, EPI_ATTN_ENTRY, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_STORE_BF16:
+      if (args.N % 32 != 0) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_STORE_BF16, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_BW_SWIGLU:
+      if (args.N % 32 != 0 || args.ldo < 2 * args.N || !args.row_scale || !args.row_part ||
+          args.part_ld < (args.N + 255) / 256)
+        return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_BW_SWIGLU, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

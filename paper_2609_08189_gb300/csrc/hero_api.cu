@@ -7,6 +7,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -178,6 +179,21 @@ struct hero_model {
   CUtensorMap tm_ax, tm_ao;
   std::vector<CUtensorMap> tm_wqkv, tm_wo;
 
+  // training path (hero_backward_init; bf16 models): transposed copies of the frozen
+  // weights, whose rows are the K-major operands of the input-gradient GEMMs, and the
+  // backward workspace
+  bool bw = false;
+  void *wdT = nullptr, *wguT = nullptr, *w1T = nullptr, *w2T = nullptr;
+  void* bws = nullptr;
+  uint16_t *bw_gu = nullptr, *bw_gf = nullptr, *bw_ga = nullptr;
+  __nv_bfloat16* bw_da = nullptr;
+  float *bw_rinv = nullptr, *bw_dgpart = nullptr, *bw_a = nullptr, *bw_gaf = nullptr,
+        *bw_daf = nullptr, *bw_y2 = nullptr, *bw_duf = nullptr, *bw_dua = nullptr,
+        *bw_wpart = nullptr;
+  int bw_part_ld = 0;
+  CUtensorMap tm_bwgf, tm_bwga, tm_bwgu, tm_bwda;
+  std::vector<CUtensorMap> tm_wdT, tm_wguT, tm_w1T, tm_w2T;
+
   // measurement
   bool profiling = false;
   std::vector<ProfEvent> pending;
@@ -327,7 +343,7 @@ void free_model(hero_model* m) {
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
-                  m->dec_pm, m->dec_pos, m->dec_ws};
+                  m->dec_pm, m->dec_pos, m->dec_ws, m->wdT, m->wguT, m->w1T, m->w2T, m->bws};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -340,6 +356,26 @@ void free_model(hero_model* m) {
 // ============================================================================
 
 extern "C" const char* hero_last_error(void) { return g_last_error.c_str(); }
+
+namespace {
+std::atomic<uint64_t> g_wait_limit_ns{0};   // 0: the default bound
+}  // namespace
+
+uint64_t hero::wait_limit_ns() {
+  const uint64_t v = g_wait_limit_ns.load(std::memory_order_relaxed);
+  return v ? v : kWaitLimitNs;
+}
+
+extern "C" void hero_set_wait_limit_ns(uint64_t limit_ns) {
+  g_wait_limit_ns.store(limit_ns, std::memory_order_relaxed);
+}
+
+hero_status hero::status_of_error_word(uint32_t e) {
+  if (!e) return HERO_OK;
+  if (e & (ERR_WAIT_PRODUCER | ERR_WAIT_MMA | ERR_WAIT_EPILOGUE | ERR_WAIT_DRAIN))
+    return fail(HERO_ERR_TIMEOUT, "a device-side wait bound expired (error word 0x%x)", e);
+  return fail(HERO_ERR_BAD_INDEX, "a kernel met an index outside its bounds (error word 0x%x)", e);
+}
 
 void hero::set_last_error(const char* msg) { g_last_error = msg; }
 
@@ -1649,11 +1685,8 @@ extern "C" hero_status hero_check_device_status(hero_model* m, void* cuda_stream
   CUDA_TRY(cudaStreamSynchronize(st));
   uint32_t e = 0;
   CUDA_TRY(cudaMemcpy(&e, m->err, 4, cudaMemcpyDeviceToHost));
-  if (e) {
-    CUDA_TRY(cudaMemset(m->err, 0, 4));
-    return fail(HERO_ERR_TIMEOUT, "device-side wait bound expired or bad index (error word 0x%x)", e);
-  }
-  return HERO_OK;
+  if (e) CUDA_TRY(cudaMemset(m->err, 0, 4));
+  return status_of_error_word(e);
 }
 
 extern "C" hero_status hero_set_profiling(hero_model* m, int enable) {
@@ -1691,10 +1724,21 @@ extern "C" hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B
   g_last_error.clear();
   if (!A || !B || !C || M < 1 || N < 8 || K < 64 || K % 64 != 0 || N % 8 != 0)
     return fail(HERO_ERR_ARG, "need M >= 1, N >= 8 (N %% 8 == 0), K %% 64 == 0 and non-NULL pointers");
-  static uint32_t* err = nullptr;
-  if (!err) CUDA_TRY(cudaMalloc(&err, 64));
+  // one error word per device, allocated with that device current
+  static std::mutex mu;
+  static uint32_t* err_of[64] = {};
   int dev = 0;
   CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) return fail(HERO_ERR_UNSUPPORTED, "device index %d above 63", dev);
+  uint32_t* err = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    if (!err_of[dev]) {
+      CUDA_TRY(cudaMalloc(&err_of[dev], 64));
+      CUDA_TRY(cudaMemset(err_of[dev], 0, 64));
+    }
+    err = err_of[dev];
+  }
   int sms = 0;
   CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   CUtensorMap ta, tb;
@@ -1708,6 +1752,240 @@ extern "C" hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B
   g.out_f32 = C;
   g.ldo = N;
   g.err = err;
-  CUDA_TRY(launch_gemm_tc(256, EPI_STORE_F32, ta, tb, g, sms, static_cast<cudaStream_t>(cuda_stream)));
+  const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  CUDA_TRY(launch_gemm_tc(256, EPI_STORE_F32, ta, tb, g, sms, st));
+  // synchronous: report (and clear) what the kernel recorded in the error word
+  CUDA_TRY(cudaStreamSynchronize(st));
+  uint32_t e = 0;
+  CUDA_TRY(cudaMemcpy(&e, err, 4, cudaMemcpyDeviceToHost));
+  if (e) CUDA_TRY(cudaMemset(err, 0, 4));
+  return status_of_error_word(e);
+}
+
+// ============================================================================
+// Training path: backward of a routed block's branch part, L_skip's gradient
+// ============================================================================
+
+extern "C" hero_status hero_backward_init(hero_model* m) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->bf16) return fail(HERO_ERR_UNSUPPORTED, "the backward runs on bf16 models only");
+  if (m->bw) return fail(HERO_ERR_ARG, "hero_backward_init was already called for this model");
+  const hero_config& c = m->cfg;
+  const size_t L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r, Tm = c.max_tokens;
+  CUDA_TRY(cudaSetDevice(m->device));
+  auto bail = [&](hero_status st) {
+    void* ps[] = {m->wdT, m->wguT, m->w1T, m->w2T, m->bws};
+    for (void* p : ps)
+      if (p) cudaFree(p);
+    m->wdT = m->wguT = m->w1T = m->w2T = m->bws = nullptr;
+    return st;
+  };
+#define BW_CUDA(expr)                                                                        \
+  do {                                                                                       \
+    cudaError_t e_ = (expr);                                                                 \
+    if (e_ != cudaSuccess)                                                                   \
+      return bail(fail(e_ == cudaErrorMemoryAllocation ? HERO_ERR_NOMEM : HERO_ERR_CUDA,     \
+                       "%s failed: %s", #expr, cudaGetErrorString(e_)));                     \
+  } while (0)
+  BW_CUDA(cudaMalloc(&m->wdT, L * I * d * 2));
+  BW_CUDA(cudaMalloc(&m->wguT, L * 2 * I * d * 2));
+  BW_CUDA(cudaMalloc(&m->w1T, L * d * r * 2));
+  BW_CUDA(cudaMalloc(&m->w2T, L * d * r * 2));
+  // W_down [d][I] -> [I][d]; W_gate|W_up interleaved [2I][d] -> [d][2I] (the K order of
+  // the gate/up gradient rows); W_1 [d_r][d] -> [d][d_r]; W_2 [d][d_r] -> [d_r][d]
+  BW_CUDA(launch_transpose_bf16(m->wdown, m->wdT, (int)d, (int)I, (int)L, 0));
+  BW_CUDA(launch_transpose_bf16(m->wgu, m->wguT, (int)(2 * I), (int)d, (int)L, 0));
+  BW_CUDA(launch_transpose_bf16(m->w1, m->w1T, (int)r, (int)d, (int)L, 0));
+  BW_CUDA(launch_transpose_bf16(m->w2, m->w2T, (int)d, (int)r, (int)L, 0));
+  m->bw_part_ld = (int)((I + 255) / 256);
+  const size_t chunks = (Tm + kBwChunk - 1) / kBwChunk;
+  struct Item {
+    void** p;
+    size_t bytes;
+  };
+  std::vector<Item> items = {
+      {(void**)&m->bw_gu, Tm * 2 * I * 2},  {(void**)&m->bw_gf, Tm * d * 2},
+      {(void**)&m->bw_ga, Tm * d * 2},      {(void**)&m->bw_da, Tm * r * 2},
+      {(void**)&m->bw_rinv, Tm * 4},        {(void**)&m->bw_dgpart, Tm * m->bw_part_ld * 4},
+      {(void**)&m->bw_a, Tm * r * 4},       {(void**)&m->bw_gaf, Tm * r * 4},
+      {(void**)&m->bw_daf, Tm * r * 4},     {(void**)&m->bw_y2, Tm * r * 4},
+      {(void**)&m->bw_duf, Tm * d * 4},     {(void**)&m->bw_dua, Tm * d * 4},
+      {(void**)&m->bw_wpart, chunks * d * r * 4},
+  };
+  size_t off = 0;
+  for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
+  BW_CUDA(cudaMalloc(&m->bws, off));
+  BW_CUDA(cudaMemset(m->bws, 0, off));
+  off = 0;
+  for (auto& it : items) {
+    *it.p = static_cast<char*>(m->bws) + off;
+    off += (it.bytes + 1023) & ~(size_t)1023;
+  }
+  bool ok = encode_bf16_2d(&m->tm_bwgf, m->bw_gf, d, Tm, 128) &&
+            encode_bf16_2d(&m->tm_bwga, m->bw_ga, d, Tm, 128) &&
+            encode_bf16_2d(&m->tm_bwgu, m->bw_gu, 2 * I, Tm, 128) &&
+            encode_bf16_2d(&m->tm_bwda, m->bw_da, r, Tm, 128);
+  m->tm_wdT.resize(L);
+  m->tm_wguT.resize(L);
+  m->tm_w1T.resize(L);
+  m->tm_w2T.resize(L);
+  for (size_t j = 0; j < L && ok; ++j) {
+    ok = encode_bf16_2d(&m->tm_wdT[j], static_cast<char*>(m->wdT) + j * I * d * 2, d, I, 256) &&
+         encode_bf16_2d(&m->tm_wguT[j], static_cast<char*>(m->wguT) + j * 2 * I * d * 2, 2 * I, d,
+                        256) &&
+         encode_bf16_2d(&m->tm_w1T[j], static_cast<char*>(m->w1T) + j * d * r * 2, r, d, 256) &&
+         encode_bf16_2d(&m->tm_w2T[j], static_cast<char*>(m->w2T) + j * d * r * 2, d, r, 256);
+  }
+  if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
+  BW_CUDA(cudaDeviceSynchronize());
+#undef BW_CUDA
+  m->bw = true;
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_routed_block_backward(hero_model* m, int32_t block, int64_t n_tokens,
+                                                  const float* h_bar, const float* gate,
+                                                  const uint8_t* mask, const float* grad_out,
+                                                  uint32_t flags, float* grad_h_bar,
+                                                  float* grad_gate, float* grad_w1, float* grad_w2,
+                                                  void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(HERO_ERR_ARG, "model is NULL");
+  if (!m->bw) return fail(HERO_ERR_ARG, "call hero_backward_init first");
+  const hero_config& c = m->cfg;
+  const int L = c.n_layers, d = c.d_model, I = c.d_ff, r = c.d_r;
+  if (block < 1 || block > L) return fail(HERO_ERR_ARG, "block %d outside 1..%d", block, L);
+  if (flags & ~(uint32_t)HERO_FLAG_DENSE) return fail(HERO_ERR_ARG, "flags 0x%x: only HERO_FLAG_DENSE", flags);
+  if (n_tokens < 0 || n_tokens > c.max_tokens)
+    return fail(HERO_ERR_ARG, "n_tokens %lld outside 0..max_tokens", (long long)n_tokens);
+  const bool dense = (flags & HERO_FLAG_DENSE) || block <= c.n_dense;
+  if (n_tokens == 0) return HERO_OK;
+  if (!h_bar || !grad_out || !grad_h_bar) return fail(HERO_ERR_ARG, "h_bar, grad_out and grad_h_bar are required");
+  if (!dense && (!gate || !mask || !grad_gate || !grad_w1 || !grad_w2))
+    return fail(HERO_ERR_ARG, "a routed block needs gate, mask, grad_gate, grad_w1 and grad_w2");
+  if (grad_h_bar == h_bar || grad_h_bar == grad_out)
+    return fail(HERO_ERR_ARG, "grad_h_bar must not alias h_bar or grad_out");
+  const int T = (int)n_tokens;
+  const int jj = block - 1;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const size_t es = 2;
+  CompactArgs ca{T, mask, gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
+                 m->counts, nullptr, nullptr, nullptr};
+  CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_compact(ca, st); }));
+  BwPrepArgs pa{T, d, m->counts, m->idx_f, m->idx_a, h_bar, grad_out,
+                m->ffn_gain + (size_t)jj * d, c.rms_eps,
+                static_cast<uint16_t*>(m->u_f), static_cast<uint16_t*>(m->u_a), m->bw_gf,
+                m->bw_ga, m->bw_rinv};
+  CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_bw_prep(pa, st); }));
+  // FFN rows: gate/up pre-activations (bf16), then e = G W_down with the SwiGLU backward
+  // in the epilogue (in place over the pre-activations), then du = [dgate|dup] [W_g|W_u]
+  GemmArgs gu{};
+  gu.m_dev = m->counts;
+  gu.m_max = T;
+  gu.N = 2 * I;
+  gu.K = d;
+  gu.out = m->bw_gu;
+  gu.ldo = 2 * I;
+  gu.err = m->err;
+  CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+    return launch_gemm_tc(256, EPI_STORE_BF16, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st);
+  }));
+  GemmArgs ge{};
+  ge.m_dev = m->counts;
+  ge.m_max = T;
+  ge.N = I;
+  ge.K = d;
+  ge.out = m->bw_gu;
+  ge.ldo = 2 * I;
+  ge.err = m->err;
+  ge.row_scale = m->scale_f;
+  ge.row_part = m->bw_dgpart;
+  ge.part_ld = m->bw_part_ld;
+  CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+    return launch_gemm_tc(256, EPI_BW_SWIGLU, m->tm_bwgf, m->tm_wdT[jj], ge, m->num_sms, st);
+  }));
+  GemmArgs gx{};
+  gx.m_dev = m->counts;
+  gx.m_max = T;
+  gx.N = d;
+  gx.K = 2 * I;
+  gx.out_f32 = m->bw_duf;
+  gx.ldo = d;
+  gx.err = m->err;
+  CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+    return launch_gemm_tc(256, EPI_STORE_F32, m->tm_bwgu, m->tm_wguT[jj], gx, m->num_sms, st);
+  }));
+  if (!dense) {
+    // adapter rows: a = W_1 u and ga = G W_2 (fp32), the hidden-layer backward per row,
+    // du = da W_1, and the weight gradients
+    GemmArgs g1{};
+    g1.m_dev = m->counts + 1;
+    g1.m_max = T;
+    g1.N = r;
+    g1.K = d;
+    g1.out_f32 = m->bw_a;
+    g1.ldo = r;
+    g1.err = m->err;
+    CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+      return launch_gemm_tc(256, EPI_STORE_F32, m->tm_ua, m->tm_w1[jj], g1, m->num_sms, st);
+    }));
+    GemmArgs g2 = g1;
+    g2.out_f32 = m->bw_gaf;
+    CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+      return launch_gemm_tc(256, EPI_STORE_F32, m->tm_bwga, m->tm_w2T[jj], g2, m->num_sms, st);
+    }));
+  }
+  BwRowsArgs ra{T, r, m->counts, m->idx_f, m->idx_a, m->bw_dgpart, m->bw_part_ld,
+                (I + 255) / 256, m->scale_a, m->bw_a, m->bw_gaf, m->bw_daf, m->bw_da, m->bw_y2,
+                dense ? nullptr : grad_gate};
+  CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_bw_rows(ra, st); }));
+  if (!dense) {
+    GemmArgs g3{};
+    g3.m_dev = m->counts + 1;
+    g3.m_max = T;
+    g3.N = d;
+    g3.K = r;
+    g3.out_f32 = m->bw_dua;
+    g3.ldo = d;
+    g3.err = m->err;
+    CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
+      return launch_gemm_tc(256, EPI_STORE_F32, m->tm_bwda, m->tm_w1T[jj], g3, m->num_sms, st);
+    }));
+    // dL/dW_2 [d, d_r] = sum over adapter rows of G[t] (1 - g) bf16(SiLU(a))^T
+    BwWgradArgs w2{m->counts + 1, grad_out, m->idx_a, m->bw_y2, d, r, m->bw_wpart};
+    CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_bw_wgrad(w2, false, T, st); }));
+    CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] {
+      return launch_bw_wreduce(m->bw_wpart, m->counts + 1, T, d, r, 0, grad_w2, m->num_sms, st);
+    }));
+    // dL/dW_1 [d_r, d] = sum over adapter rows of da u^T (u as the forward's bf16 operand)
+    BwWgradArgs w1{m->counts + 1, m->u_a, nullptr, m->bw_daf, d, r, m->bw_wpart};
+    CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_bw_wgrad(w1, true, T, st); }));
+    CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] {
+      return launch_bw_wreduce(m->bw_wpart, m->counts + 1, T, d, r, 1, grad_w1, m->num_sms, st);
+    }));
+  } else {
+    if (grad_w1) CUDA_TRY(cudaMemsetAsync(grad_w1, 0, (size_t)r * d * 4, st));
+    if (grad_w2) CUDA_TRY(cudaMemsetAsync(grad_w2, 0, (size_t)r * d * 4, st));
+    if (grad_gate) CUDA_TRY(cudaMemsetAsync(grad_gate, 0, (size_t)T * 4, st));
+  }
+  BwOutArgs oa{T, d, m->counts, m->idx_f, m->idx_a, h_bar, grad_out,
+               m->ffn_gain + (size_t)jj * d, m->bw_rinv, m->bw_duf, m->bw_dua, grad_h_bar};
+  CUDA_TRY(timed(m, HERO_K_BACKWARD, st, [&] { return launch_bw_out(oa, st); }));
+  (void)es;
+  return HERO_OK;
+}
+
+extern "C" hero_status hero_skip_penalty_grad(int32_t n_layers, int32_t n_dense, int32_t n_seqs,
+                                              int32_t seq_len, const float* gates, float alpha,
+                                              float* grad_gates, void* cuda_stream) {
+  g_last_error.clear();
+  if (n_layers < 1 || n_dense < 0 || n_dense >= n_layers || n_seqs < 1 || seq_len < 2)
+    return fail(HERO_ERR_ARG, "need n_layers >= 1, 0 <= n_dense < n_layers, n_seqs >= 1, seq_len >= 2");
+  if ((int64_t)n_seqs * seq_len > INT32_MAX) return fail(HERO_ERR_ARG, "too many tokens");
+  if (!gates || !grad_gates) return fail(HERO_ERR_ARG, "gates and grad_gates are required");
+  if (gates == grad_gates) return fail(HERO_ERR_ARG, "grad_gates must not alias gates");
+  CUDA_TRY(launch_skip_grad(gates, n_layers, n_dense, n_seqs, seq_len, alpha, grad_gates,
+                            static_cast<cudaStream_t>(cuda_stream)));
   return HERO_OK;
 }

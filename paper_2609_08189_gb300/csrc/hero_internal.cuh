@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "../../include/hero.h"
+
 namespace hero {
 
 // Launch `kernel` on `st` with programmatic stream serialisation: its launch may
@@ -39,8 +41,19 @@ enum : uint32_t {
 // Record the message hero_last_error() returns on this host thread.
 void set_last_error(const char* msg);
 
-// Bound on every device-side wait (nanoseconds of %globaltimer).
+// Status for a device error word read back by the host: HERO_ERR_TIMEOUT if any
+// wait bit is set, HERO_ERR_BAD_INDEX for a bad index alone, HERO_OK for 0 (sets
+// the thread's message on failure).
+hero_status status_of_error_word(uint32_t e);
+
+// Default bound on every device-side wait (nanoseconds of %globaltimer); the bound a
+// launch uses is wait_limit_ns(), which hero_set_wait_limit_ns may lower (tests of the
+// timeout path).  The drains that follow an expired wait (copies and tensor-core work
+// still in flight must finish before the CTA frees its TMEM and exits) use their own
+// fixed bound, so a tiny wait bound never shortens them.
 constexpr uint64_t kWaitLimitNs = 4000000000ull;
+constexpr uint64_t kDrainLimitNs = 100000000ull;
+uint64_t wait_limit_ns();
 
 // ---------------------------------------------------------------------------
 // Epilogue of the two GEMMs that close a routed block (FFN down, adapter up):
@@ -87,6 +100,12 @@ enum EpiKind : int {
                        // partial sums lo.part (lo.router, lo.first as in LayerOutArgs)
   EPI_QKV_ROPE = 7,    // fused q/k/v projection: RoPE on the q and k heads, bf16 out in
                        // the attention layout (RopeArgs)
+  EPI_STORE_BF16 = 8,  // out[m, n] = bf16(acc) (N a multiple of 32)
+  EPI_BW_SWIGLU = 9,   // backward of the SwiGLU product (training path): acc = e = dL/dy W_down
+                       // for features n of row m; out holds the row's bf16 gate/up
+                       // pre-activations in the interleaved layout and is overwritten in place
+                       // by dL/dgate, dL/dup (scaled by row_scale[m] = g); row_part[m, nb] =
+                       // sum over the tile's features of e * bf16(SiLU(gate) up)
 };
 
 // EPI_QKV_ROPE: columns are heads of 128 (q heads | k heads | v heads).  Row t is
@@ -127,6 +146,10 @@ struct GemmArgs {
   // writing rows the previous one does not touch) works without waiting and waits
   // for the previous kernel at its end, so the kernels after it still follow both.
   int pdl_mode;
+  uint64_t wait_ns;    // bound of every mbarrier wait (set by the launcher: wait_limit_ns())
+  const float* row_scale;  // EPI_BW_SWIGLU: [rows] branch scale g
+  float* row_part;     // EPI_BW_SWIGLU: [rows, part_ld] per-tile sums
+  int part_ld;
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
@@ -322,6 +345,71 @@ cudaError_t launch_entry_close(const float* part, int splits, long split_stride,
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
                                 cudaStream_t st);
+
+// Training path: backward of a routed block's branch part (backward.cu) -------------
+// Compacted rows: FFN rows 0 .. n_f - 1 (idx_f), then adapter rows (idx_a), counts [2].
+struct BwPrepArgs {
+  int T, d;
+  const int* counts;
+  const int* idx_f;
+  const int* idx_a;
+  const float* hbar;     // [T, d] h_bar of the block
+  const float* G;        // [T, d] dL/dh
+  const float* gain;     // [d] LN_ffn gain
+  float rms_eps;
+  uint16_t* u_f;         // [T, d] bf16 u of the FFN rows (compacted)
+  uint16_t* u_a;         // [T, d] bf16 u of the adapter rows
+  uint16_t* g_f;         // [T, d] bf16 G of the FFN rows
+  uint16_t* g_a;         // [T, d] bf16 G of the adapter rows
+  float* rinv;           // [T] 1 / rms(h_bar)
+};
+struct BwRowsArgs {
+  int T, d_r;
+  const int* counts;
+  const int* idx_f;
+  const int* idx_a;
+  const float* dgpart;   // [T, part_ld] FFN rows: per-tile sums of e * act
+  int part_ld, n_parts;
+  const float* scale_a;  // [T] adapter rows: 1 - g
+  const float* pre;      // [T, d_r] adapter rows: a = W_1 u
+  const float* ga;       // [T, d_r] adapter rows: G W_2
+  float* da_f32;         // [T, d_r] out: da
+  __nv_bfloat16* da_bf16;  // [T, d_r] out: bf16(da), the input-gradient GEMM's operand
+  float* y2;             // [T, d_r] out: (1 - g) bf16(SiLU(a)), the W_2 gradient's factor
+  float* grad_gate;      // [T] out: dL/dg by token (nullptr: not wanted)
+};
+constexpr int kBwChunk = 512;   // adapter rows per weight-gradient partial
+struct BwWgradArgs {
+  const int* rows;       // device row count (n_a)
+  const void* X;         // fp32 [tokens, N] gathered through idx, or bf16 [rows, N]
+  const int* idx;
+  const float* Y;        // [rows, R]
+  int N, R;
+  float* part;           // [chunks, N, R]
+};
+struct BwOutArgs {
+  int T, d;
+  const int* counts;
+  const int* idx_f;
+  const int* idx_a;
+  const float* hbar;
+  const float* G;
+  const float* gain;
+  const float* rinv;
+  const float* du_f;     // [T, d] du of the FFN rows (compacted)
+  const float* du_a;     // [T, d] du of the adapter rows
+  float* grad_hbar;      // [T, d] out
+};
+cudaError_t launch_bw_prep(const BwPrepArgs& a, cudaStream_t st);
+cudaError_t launch_bw_rows(const BwRowsArgs& a, cudaStream_t st);
+cudaError_t launch_bw_wgrad(const BwWgradArgs& a, bool x_bf16, int max_rows, cudaStream_t st);
+cudaError_t launch_bw_wreduce(const float* part, const int* rows, int max_rows, int N, int R,
+                              int transposed, float* out, int num_sms, cudaStream_t st);
+cudaError_t launch_bw_out(const BwOutArgs& a, cudaStream_t st);
+cudaError_t launch_skip_grad(const float* gates, int L, int n_dense, int n_seqs, int seq_len,
+                             float alpha, float* out, cudaStream_t st);
+cudaError_t launch_transpose_bf16(const void* in, void* out, int R, int C, int batch,
+                                  cudaStream_t st);
 
 // Weight conversion: dst[map(r)] = convert(src[r]) for rows of `cols` elements.
 // map(r) = (r / grp) * grp_stride + (r % grp) + offset.

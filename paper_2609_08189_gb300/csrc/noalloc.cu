@@ -106,18 +106,18 @@ extern "C" hero_status hero_gemm_bf16_splitk_noalloc(const uint16_t* A, const ui
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   float* scratch = g_scratch_ptr[dev];
   uint32_t* err = g_err_ptr[dev];
-  if (cudaMemsetAsync(err, 0, 64 * sizeof(uint32_t), st) != cudaSuccess)
-    return fail_na(HERO_ERR_CUDA, "clearing the static error word failed");
-  const int kpb = (kblocks + splits - 1) / splits;   // K blocks per slice
+  // A sticky error from earlier work on this thread would otherwise be taken for a
+  // failure of the reduction launch below; report it without enqueueing anything.
+  if (cudaPeekAtLastError() != cudaSuccess)
+    return fail_na(HERO_ERR_CUDA, "a CUDA error from earlier work is pending on this thread");
+  // The error word of the previous call is not cleared here: the status query reports
+  // (and clears) it.  The GEMM only ever sets bits, so one query after a sequence of
+  // calls reports a failure of any of them.
   for (int s = 0; s < splits; ++s) {
-    const int kb0 = s * kpb;
-    const int kb1 = kb0 + kpb < kblocks ? kb0 + kpb : kblocks;
-    if (kb0 >= kb1) {  // empty trailing slice: its partial sums are zero
-      if (cudaMemsetAsync(scratch + (size_t)s * M * N, 0, (size_t)M * N * sizeof(float), st) !=
-          cudaSuccess)
-        return fail_na(HERO_ERR_CUDA, "clearing an empty slice failed");
-      continue;
-    }
+    // slice s owns K blocks [s kblocks / splits, (s + 1) kblocks / splits): never
+    // empty, since splits <= kblocks
+    const int kb0 = (int)((long)s * kblocks / splits);
+    const int kb1 = (int)((long)(s + 1) * kblocks / splits);
     const uint64_t kk = (uint64_t)(kb1 - kb0) * 64;
     CUtensorMap ta, tb;
     if (!encode(&ta, A + (size_t)kb0 * 64, kk, M, (uint64_t)K * 2, 128) ||
@@ -137,7 +137,33 @@ extern "C" hero_status hero_gemm_bf16_splitk_noalloc(const uint16_t* A, const ui
   const long mn = (long)M * N;
   long blocks = (mn + 255) / 256;
   if (blocks > 4096) blocks = 4096;
-  k_splitk_reduce<<<(unsigned)blocks, 256, 0, st>>>(scratch, C, mn, splits);
-  if (cudaGetLastError() != cudaSuccess) return fail_na(HERO_ERR_CUDA, "reduction launch failed");
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3((unsigned)blocks);
+  lc.blockDim = dim3(256);
+  lc.stream = st;
+  if (cudaLaunchKernelEx(&lc, k_splitk_reduce, (const float*)scratch, C, mn, (int)splits) !=
+      cudaSuccess)
+    return fail_na(HERO_ERR_CUDA, "reduction launch failed");
   return HERO_OK;
+}
+
+extern "C" hero_status hero_gemm_bf16_splitk_noalloc_status(void* cuda_stream) {
+  set_last_error("");
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return fail_na(HERO_ERR_CUDA, "no usable current device");
+  uint32_t* err = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_setup_mu);
+    err = g_err_ptr[dev];
+  }
+  if (!err) return HERO_OK;   // no call has run on this device
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(cuda_stream)) != cudaSuccess)
+    return fail_na(HERO_ERR_CUDA, "stream synchronisation failed");
+  uint32_t e = 0;
+  if (cudaMemcpy(&e, err, sizeof(e), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return fail_na(HERO_ERR_CUDA, "reading the static error word failed");
+  if (e && cudaMemset(err, 0, sizeof(e)) != cudaSuccess)
+    return fail_na(HERO_ERR_CUDA, "clearing the static error word failed");
+  return status_of_error_word(e);
 }

@@ -17,14 +17,16 @@ import numpy as np
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libhero.so")
 
-HERO_OK, HERO_ERR_ARG, HERO_ERR_CUDA, HERO_ERR_NOMEM, HERO_ERR_UNSUPPORTED, HERO_ERR_TIMEOUT = range(6)
+(HERO_OK, HERO_ERR_ARG, HERO_ERR_CUDA, HERO_ERR_NOMEM, HERO_ERR_UNSUPPORTED, HERO_ERR_TIMEOUT,
+ HERO_ERR_BAD_INDEX) = range(7)
 STATUS_NAMES = {0: "HERO_OK", 1: "HERO_ERR_ARG", 2: "HERO_ERR_CUDA", 3: "HERO_ERR_NOMEM",
-                4: "HERO_ERR_UNSUPPORTED", 5: "HERO_ERR_TIMEOUT"}
+                4: "HERO_ERR_UNSUPPORTED", 5: "HERO_ERR_TIMEOUT", 6: "HERO_ERR_BAD_INDEX"}
 HERO_F32, HERO_BF16 = 0, 1
 HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO = 1, 2, 4
 HERO_ROUTER_NO_HISTORY, HERO_ROUTER_NO_MEMREAD, HERO_ROUTER_NO_AUX, HERO_ROUTER_NO_POS = 1, 2, 4, 8
 KERNEL_CLASSES = ("init", "router_gemm", "router", "compact", "norm", "ffn_gate_up", "ffn_down",
-                  "adapter_down", "adapter_up", "attn_proj", "attn_core")
+                  "adapter_down", "adapter_up", "attn_proj", "attn_core", "backward_gemm",
+                  "backward")
 ATTN_WEIGHT_FIELDS = ("attn_norm_g", "w_q", "w_k", "w_v", "w_o")
 HERO_K_COUNT = len(KERNEL_CLASSES)
 
@@ -119,6 +121,16 @@ def load(path: Optional[str] = None) -> ctypes.CDLL:
     lib.hero_decode_step.restype = ctypes.c_int
     lib.hero_gemm_bf16_splitk_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     lib.hero_gemm_bf16_splitk_noalloc.restype = ctypes.c_int
+    lib.hero_gemm_bf16_splitk_noalloc_status.argtypes = [vp]
+    lib.hero_gemm_bf16_splitk_noalloc_status.restype = ctypes.c_int
+    lib.hero_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
+    lib.hero_set_wait_limit_ns.restype = None
+    lib.hero_backward_init.argtypes = [vp]
+    lib.hero_backward_init.restype = ctypes.c_int
+    lib.hero_routed_block_backward.argtypes = [vp, i32, i64, vp, vp, vp, vp, u32, vp, vp, vp, vp, vp]
+    lib.hero_routed_block_backward.restype = ctypes.c_int
+    lib.hero_skip_penalty_grad.argtypes = [i32, i32, i32, i32, vp, f32, vp, vp]
+    lib.hero_skip_penalty_grad.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -214,13 +226,46 @@ def hero_get_profile(model: int, reset: bool = True):
 
 
 def hero_gemm_bf16_check(A: int, B: int, C: int, M: int, N: int, K: int, cuda_stream: int = 0) -> None:
+    """Synchronous; raises HeroError(HERO_ERR_TIMEOUT) if the kernel's wait bound expired."""
     _check(load().hero_gemm_bf16_check(A, B, C, M, N, K, cuda_stream or None))
+
+
+def hero_backward_init(model: int) -> None:
+    _check(load().hero_backward_init(model))
+
+
+def hero_routed_block_backward(model: int, block: int, n_tokens: int, h_bar: int, gate: int,
+                               mask: int, grad_out: int, flags: int, grad_h_bar: int,
+                               grad_gate: int, grad_w1: int, grad_w2: int,
+                               cuda_stream: int = 0) -> None:
+    """Backward of one block's branch part with the decisions fixed (pointer-level call)."""
+    _check(load().hero_routed_block_backward(model, block, n_tokens, h_bar or None, gate or None,
+                                             mask or None, grad_out or None, flags,
+                                             grad_h_bar or None, grad_gate or None,
+                                             grad_w1 or None, grad_w2 or None,
+                                             cuda_stream or None))
+
+
+def hero_skip_penalty_grad(n_layers: int, n_dense: int, n_seqs: int, seq_len: int, gates: int,
+                           alpha: float, grad_gates: int, cuda_stream: int = 0) -> None:
+    _check(load().hero_skip_penalty_grad(n_layers, n_dense, n_seqs, seq_len, gates or None,
+                                         float(alpha), grad_gates or None, cuda_stream or None))
+
+
+def hero_set_wait_limit_ns(limit_ns: int) -> None:
+    """Bound on device-side waits of later launches (0 restores the default 4 s)."""
+    load().hero_set_wait_limit_ns(int(limit_ns))
 
 
 def hero_gemm_bf16_splitk_noalloc(A: int, B: int, C: int, M: int, N: int, K: int, splits: int,
                                   cuda_stream: int = 0) -> None:
     """Split-K bf16 GEMM whose scratch lives in static device memory (no allocation)."""
     _check(load().hero_gemm_bf16_splitk_noalloc(A, B, C, M, N, K, splits, cuda_stream or None))
+
+
+def hero_gemm_bf16_splitk_noalloc_status(cuda_stream: int = 0) -> None:
+    """Raises if an allocation-free GEMM call since the last query recorded an error."""
+    _check(load().hero_gemm_bf16_splitk_noalloc_status(cuda_stream or None))
 
 
 def hero_attn_init(model: int, stack_cfg, attn_weights: Dict[str, np.ndarray]) -> None:
@@ -332,6 +377,31 @@ class HeroStack:
         import torch
         st = stream if stream is not None else torch.cuda.current_stream()
         hero_check_device_status(self.model, st.cuda_stream)
+
+    def backward_init(self):
+        """Transposed weight copies and workspace of the training path (hero_backward_init)."""
+        hero_backward_init(self.model)
+
+    def block_backward(self, block: int, h_bar, gate, mask, grad_out, flags: int = 0, stream=None):
+        """Backward of block `block`'s branch part with its decisions fixed (device tensors).
+        Returns (grad_h_bar [T, d], grad_gate [T], grad_w1 [d_r, d], grad_w2 [d, d_r])."""
+        import torch
+        T, d = h_bar.shape
+        dev = h_bar.device
+        r = self.cfg.d_r
+        gh = torch.empty((T, d), dtype=torch.float32, device=dev)
+        gg = torch.empty((T,), dtype=torch.float32, device=dev)
+        g1 = torch.empty((r, d), dtype=torch.float32, device=dev)
+        g2 = torch.empty((d, r), dtype=torch.float32, device=dev)
+        for t in (h_bar, grad_out) + tuple(x for x in (gate, mask) if x is not None):
+            assert t.is_contiguous()
+        st = stream if stream is not None else torch.cuda.current_stream(dev)
+        hero_routed_block_backward(self.model, block, T, h_bar.data_ptr(),
+                                   gate.data_ptr() if gate is not None else 0,
+                                   mask.data_ptr() if mask is not None else 0, grad_out.data_ptr(),
+                                   flags, gh.data_ptr(), gg.data_ptr(), g1.data_ptr(), g2.data_ptr(),
+                                   st.cuda_stream)
+        return gh, gg, g1, g2
 
 
 class HeroDecoder(HeroStack):

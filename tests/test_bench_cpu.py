@@ -69,3 +69,32 @@ def test_workload_descriptions_name_the_shapes():
     assert "4x4096" in bench.workload_desc(hi.CONFIGS["llama31_8b_prefill"], 0.2687)
     desc = bench.workload_desc(hi.CONFIGS["llama31_8b_kvdecode"], 0.2687)
     assert "64 sequences" in desc and "position 4096" in desc and "H_kv=8" in desc
+
+
+def test_gpus_flag_starts_its_own_ranks(monkeypatch):
+    """--gpus N without an outside launcher re-runs bench.py as N ranks of one node under
+    torch.distributed.run on a 127.0.0.1 rendezvous (no GPU is touched here)."""
+    seen = {}
+
+    def fake_call(cmd):
+        seen["cmd"] = cmd
+        return 0
+
+    monkeypatch.setattr(bench.subprocess, "call", fake_call)
+    monkeypatch.delenv("WORLD_SIZE", raising=False)
+    monkeypatch.setattr(sys, "argv", ["bench.py", "--gpus", "4", "--steps", "2"])
+    assert bench.main() == 0
+    cmd = seen["cmd"]
+    assert cmd[1:3] == ["-m", "torch.distributed.run"]
+    assert "--nproc-per-node=4" in cmd and "--master-addr=127.0.0.1" in cmd
+    assert cmd[-4:] == ["--gpus", "4", "--steps", "2"]
+
+
+@pytest.mark.parametrize("bypass", [0.0, 0.27, 0.39])
+def test_bypass_sweep_points_have_a_committed_tau(bypass):
+    """The Llama-2-13B sweep (0 / 27 / 39% bypass) selects a calibrated tau per point;
+    tau grows with the budget (more tokens below it) and 0% admits every token."""
+    tau = hi.calibrated_tau("llama2_13b_prefill", bypass)
+    if bypass == 0.0:
+        assert tau == 0.0
+    assert hi.calibrated_tau("llama2_13b_prefill", 0.39) > hi.calibrated_tau("llama2_13b_prefill", 0.27)

@@ -45,6 +45,7 @@ def _ptrs(ts):
 TF = [("tiny_f32", None, None), ("small_bf16", None, None), ("small_bf16_placed", None, None),
       ("llama2_7b_prefill", None, 32), ("llama31_8b_prefill", None, 32),
       ("llama31_8b_decode", None, 32), ("llama2_13b_prefill", 0.27, 16),
+      ("llama2_13b_prefill", 0.0, 16), ("llama2_13b_prefill", 0.39, 16),
       ("llama31_8b_paper", None, 16)]
 
 

@@ -184,7 +184,7 @@ def test_decode_rejects_and_reports(small, hero):
     dec.decode(h, bad, 5, 0.3)
     with pytest.raises(hero.HeroError) as e:
         dec.check()
-    assert e.value.status == hero.HERO_ERR_TIMEOUT
+    assert e.value.status == hero.HERO_ERR_BAD_INDEX   # not taken for an expired wait
     dec.decode(h, pos, 5, 0.3)        # the model stays usable
     dec.check()
 

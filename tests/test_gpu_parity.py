@@ -181,6 +181,7 @@ def test_host_io_matches_device_path(hero):
 
 FULL = [("llama2_7b_prefill", None, 64), ("llama31_8b_prefill", None, 64),
         ("llama31_8b_decode", None, 64), ("llama2_13b_prefill", 0.27, 32),
+        ("llama2_13b_prefill", 0.0, 32), ("llama2_13b_prefill", 0.39, 32),
         ("llama31_8b_paper", None, 32)]
 
 

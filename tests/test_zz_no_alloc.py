@@ -31,7 +31,8 @@ def _gemm_tol(ref, K):
 
 
 @pytest.mark.parametrize("M,N,K,splits", [(64, 4096, 14336, 8), (333, 512, 1024, 3),
-                                          (1, 256, 320, 5), (128, 264, 4096, 1)])
+                                          (1, 256, 320, 5), (128, 264, 4096, 1),
+                                          (64, 256, 320, 4)])   # 5 K blocks over 4 slices
 def test_noalloc_matches_allocating_gemm_twice(hero, M, N, K, splits):
     import torch
     st = torch.cuda.current_stream().cuda_stream
@@ -50,6 +51,8 @@ def test_noalloc_matches_allocating_gemm_twice(hero, M, N, K, splits):
         assert torch.isfinite(C_na).all()
         assert (C_na.double() - C_ref.double()).abs().max().item() <= 2 * tol
         assert (C_na.double() - exact).abs().max().item() <= tol
+    # the static error word: no wait expired and no bad index in either call
+    hero.hero_gemm_bf16_splitk_noalloc_status(st)
 
 
 def test_noalloc_rejects_requests_beyond_the_static_scratch(hero):
