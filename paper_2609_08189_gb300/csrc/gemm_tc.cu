@@ -28,25 +28,31 @@ constexpr int kGroupM = 16;   // raster: 16 M-tiles share each wave of N-tiles (
 
 constexpr int EPI_NONE = -1;   // no second problem
 
-template <int BN, int EPIW>
+// CG = 1: one CTA computes a 128 x BN tile.  CG = 2: a CTA pair (thread-block cluster
+// of 2) computes a 256 x BN tile with the 2-SM MMA: each CTA holds 128 rows of A, BN / 2
+// rows of B and 128 rows of the accumulator, so per FLOP each SM stages a third less
+// operand data through its shared memory.
+template <int BN, int EPIW, int CG = 1>
 struct TcCfg {
-  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int B_ROWS = BN / CG;   // rows of B staged by this CTA
+  static constexpr int STAGES = CG == 2 ? 6 : (BN == 256 ? 4 : 6);
   static constexpr uint32_t A_BYTES = BM * BK * 2;
-  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  static constexpr uint32_t B_BYTES = B_ROWS * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
   // instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
-  // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+  // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24
+  // (M = 256 for the pair).
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                                    ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+                                    ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((BM * CG) >> 4) << 24);
   // EPIW epilogue warps: one (4 warps) or two (8 warps, each taking half of the
   // tile's columns) per TMEM lane quadrant.
   static constexpr int EPI_WARPS = EPIW;
-  static constexpr int EPI_COLS = BN / (EPIW / 4);
   static constexpr int THREADS = 64 + 32 * EPI_WARPS;
   // ring | barriers (256 B) | per-epilogue-warp staging tiles (32 x 32 fp32 each)
   static constexpr uint32_t EPI_STAGE_OFF = STAGES * STAGE_BYTES + 256;
   static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + EPI_WARPS * 32 * 32 * 4 + 1024;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 template <int EPI>
@@ -468,7 +474,7 @@ struct ProbSize {
 __device__ __forceinline__ void tile_work(const ProbSize& p, int local, int& mb, int& nb, int& s,
                                           int& kb0, int& kb1);
 
-template <int BN>
+template <int BN, int CG = 1>
 __device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
   ProbSize p;
   int M = a.m_dev ? *a.m_dev : a.m_static;
@@ -477,7 +483,7 @@ __device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
     M = 0;
   }
   p.M = M;
-  p.m_tiles = (M + BM - 1) / BM;
+  p.m_tiles = (M + BM * CG - 1) / (BM * CG);   // M-tiles of the CTA or the CTA pair
   p.n_tiles = (a.N + BN - 1) / BN;
   p.kblocks = (a.K + BK - 1) / BK;
   const int splits = a.k_splits > 1 ? a.k_splits : 1;
@@ -515,11 +521,11 @@ __device__ __forceinline__ int split_tile(int g, int t1, int total, int& local) 
 
 // Epilogue warp ew serves TMEM lane quadrant q = ew % 4; with 8 epilogue warps the
 // second warp of a quadrant takes the upper half of the columns.
-template <int BN, int EPI>
+template <int BN, int EPI, int CG>
 __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, int q, int ew,
                                              int lane, int mb, int nb, int M, int split,
-                                             float4* stg) {
-  const int row0 = mb * BM + q * 32;
+                                             float4* stg, int rank) {
+  const int row0 = (mb * CG + rank) * BM + q * 32;
   if constexpr (EPI == EPI_STORE_F32) {
     epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
   } else if constexpr (EPI == EPI_RESIDUAL) {
@@ -543,14 +549,15 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
   }
 }
 
-template <int BN, int EPI0, int EPI1>
-__global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
+template <int BN, int EPI0, int EPI1, int CG>
+__global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
               const GemmArgs a0, const GemmArgs a1) {
   if (a0.pdl_mode != 2) pdl_enter();
-  using C = TcCfg<BN, epi_warps<EPI0>()>;
+  using C = TcCfg<BN, epi_warps<EPI0>(), CG>;
   constexpr bool kGrouped = EPI1 != EPI_NONE;
+  constexpr bool kPair = CG == 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -571,10 +578,18 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // A CTA pair works on one tile: the even CTA (rank 0) issues the MMAs, waits for both
+  // CTAs' operand copies on its full barriers and for both CTAs' epilogues on its
+  // accumulator-empty barriers; its commits arrive on the barriers of both CTAs.
+  const int rank = kPair ? (int)cluster_ctarank() : 0;
+  const bool issuer = rank == 0;
+  const int unit = blockIdx.x / CG, n_units = gridDim.x / CG;
+  // barrier addresses of the pair's even CTA (its own for rank 0)
+  const uint32_t bar0_lead = kPair ? mapa_shared(bar0, 0) : bar0;
 
-  const ProbSize P0 = prob_size<BN>(a0);
+  const ProbSize P0 = prob_size<BN, CG>(a0);
   ProbSize P1{0, 0, 0, 0, 0};
-  if constexpr (kGrouped) P1 = prob_size<BN>(a1);
+  if constexpr (kGrouped) P1 = prob_size<BN, CG>(a1);
   const int total = P0.tiles + P1.tiles;
 
   if (threadIdx.x == 0) {
@@ -584,15 +599,23 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull_bar(a), 1);
-      mbar_init(tempty_bar(a), C::EPI_WARPS);
+      mbar_init(tempty_bar(a), C::EPI_WARPS * CG);
     }
     mbar_init(drain_bar, 1);
     misc[1] = 0;  // abort flag
     fence_mbar_init();
   }
+  // both CTAs' barriers are initialised before either signals the other's (and before
+  // the allocation below, so that no CTA waits on its partner while holding TMEM)
+  if constexpr (kPair) cluster_sync();
   if (warp == 1) {
-    tmem_alloc(smem_u32(const_cast<uint32_t*>(misc)), C::TMEM_COLS);
-    tmem_relinquish();
+    if constexpr (kPair) {   // one warp of each CTA of the pair, collectively
+      tmem_alloc_pair(smem_u32(const_cast<uint32_t*>(misc)), C::TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_u32(const_cast<uint32_t*>(misc)), C::TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -612,23 +635,33 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       uint32_t phase = 0;
       uint32_t issued = 0, last_par = 0;  // per-stage bit masks for the drain
       bool ok = true;
-      for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
+      for (int g = unit; g < total && ok; g += n_units) {
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb, sp, kb0, kb1;
         tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         const CUtensorMap* tA = pr ? &tmA1 : &tmA0;
         const CUtensorMap* tB = pr ? &tmB1 : &tmB0;
-        if (a0.pdl_mode == 1 && g + (int)gridDim.x >= total)   // this CTA's last tile
+        if (a0.pdl_mode == 1 && g + n_units >= total)   // this CTA's last tile
           asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        const int ya = (mb * CG + rank) * BM, yb = nb * BN + rank * C::B_ROWS;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, wait_ns) || misc[1]) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(full_bar(stage), C::STAGE_BYTES);
-          tma_load_2d(sA(stage), tA, kb * BK, mb * BM, full_bar(stage));
-          tma_load_2d(sB(stage), tB, kb * BK, nb * BN, full_bar(stage));
+          if constexpr (kPair) {
+            // both CTAs' copies complete on the even CTA's full barrier, which expects
+            // the bytes of the pair
+            const uint32_t fb = bar0_lead + 8u * stage;
+            if (issuer) mbar_arrive_expect_tx(full_bar(stage), CG * C::STAGE_BYTES);
+            tma_load_2d_pair(sA(stage), tA, kb * BK, ya, fb);
+            tma_load_2d_pair(sB(stage), tB, kb * BK, yb, fb);
+          } else {
+            mbar_arrive_expect_tx(full_bar(stage), C::STAGE_BYTES);
+            tma_load_2d(sA(stage), tA, kb * BK, ya, full_bar(stage));
+            tma_load_2d(sB(stage), tB, kb * BK, yb, full_bar(stage));
+          }
           issued |= 1u << stage;
           last_par = (last_par & ~(1u << stage)) | (phase << stage);
           if (++stage == C::STAGES) {
@@ -641,22 +674,30 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
         misc[1] = 1;
         atomicOr(err, ERR_WAIT_PRODUCER);
       }
-      // Let every copy this thread issued land before the CTA can exit, also when
-      // the loop ended normally: if another role gave up early, stages it never
-      // consumed may still be in flight.  (Normally they have landed already.)
-      for (int s = 0; s < C::STAGES; ++s)
-        if ((issued & (1u << s)) && !mbar_wait(full_bar(s), (last_par >> s) & 1u, kDrainLimitNs))
-          atomicOr(err, ERR_WAIT_DRAIN);
+      if (issuer) {
+        // Let every copy issued into the stages land before the CTA can exit, also when
+        // the loop ended normally: if another role gave up early, stages it never
+        // consumed may still be in flight.  (Normally they have landed already.)
+        for (int s = 0; s < C::STAGES; ++s)
+          if ((issued & (1u << s)) && !mbar_wait(full_bar(s), (last_par >> s) & 1u, kDrainLimitNs))
+            atomicOr(err, ERR_WAIT_DRAIN);
+      } else if (!ok) {
+        // the odd CTA's copies complete on the even CTA's barriers, which it cannot
+        // wait on: after an abort, give copies in flight a fixed grace period
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 2000000ull) {
+        }
+      }
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
-    if (lane == 0 && total > 0) {
+    if (lane == 0 && total > 0 && issuer) {
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int g = blockIdx.x; g < total && ok; g += gridDim.x) {
+      for (int g = unit; g < total && ok; g += n_units) {
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb, sp, kb0, kb1;
@@ -678,16 +719,25 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             // +32 bytes per K step of 16 bf16 inside the 128-byte swizzle row
-            umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb != kb0) || k != 0);
+            if constexpr (kPair)
+              umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb != kb0) || k != 0);
+            else
+              umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, C::IDESC, (kb != kb0) || k != 0);
           }
-          umma_commit(empty_bar(stage));
+          if constexpr (kPair)
+            umma_commit_pair(empty_bar(stage));   // frees the stage in both CTAs
+          else
+            umma_commit(empty_bar(stage));
           if (++stage == C::STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        umma_commit(tfull_bar(acc));
+        if constexpr (kPair)
+          umma_commit_pair(tfull_bar(acc));
+        else
+          umma_commit(tfull_bar(acc));
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1u;
       }
@@ -697,7 +747,10 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       }
       // Every MMA this thread issued completes before TMEM is freed, also when the
       // loop ended normally but an epilogue warp gave up on a tile still in flight.
-      umma_commit(drain_bar);  // arrives once every issued MMA has finished
+      if constexpr (kPair)
+        umma_commit_pair(drain_bar);   // arrives in both CTAs once every MMA has finished
+      else
+        umma_commit(drain_bar);
       if (!mbar_wait(drain_bar, 0, kDrainLimitNs)) atomicOr(err, ERR_WAIT_DRAIN);
     }
   } else {
@@ -706,7 +759,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
     const int ew = warp - 2;  // epilogue warp index
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int g = blockIdx.x; g < total; g += gridDim.x) {
+    for (int g = unit; g < total; g += n_units) {
       int local;
       const int pr = split_tile(g, P1.tiles, total, local);
       int mb, nb, sp, kb0, kb1;
@@ -726,15 +779,20 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
       float4* stg = reinterpret_cast<float4*>(smem + C::EPI_STAGE_OFF) + ew * (32 * 8);
       if constexpr (kGrouped) {
         if (pr)
-          run_epilogue<BN, EPI1>(a1, tbase, q, ew, lane, mb, nb, P1.M, sp, stg);
+          run_epilogue<BN, EPI1, CG>(a1, tbase, q, ew, lane, mb, nb, P1.M, sp, stg, rank);
         else
-          run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg);
+          run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank);
       } else {
-        run_epilogue<BN, EPI0>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg);
+        run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank);
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty_bar(acc));
+      if (lane == 0) {
+        if constexpr (kPair)
+          mbar_arrive_cluster(bar0_lead + 8u * (2 * C::STAGES + 2 + acc));
+        else
+          mbar_arrive(tempty_bar(acc));
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
@@ -743,38 +801,84 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>()>::THREADS, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem_base, C::TMEM_COLS);
+    if constexpr (kPair) {
+      // the odd CTA's accumulator is written by the even CTA's MMAs: wait for their
+      // completion (the even CTA's drain commit) before freeing TMEM
+      if (!issuer && total > 0) {
+        bool w = true;
+        if (lane == 0) w = mbar_wait(drain_bar, 0, kDrainLimitNs);
+        if (!__shfl_sync(0xffffffffu, w ? 1 : 0, 0) && lane == 0) atomicOr(err, ERR_WAIT_DRAIN);
+      }
+      tc_fence_after();
+      tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
+    } else {
+      tc_fence_after();
+      tmem_dealloc(tmem_base, C::TMEM_COLS);
+    }
   }
+  if constexpr (kPair) cluster_sync();   // neither CTA exits while the other may signal it
   if (a0.pdl_mode == 2) pdl_enter();   // complete only after the previous kernel
 }
 
-template <int BN, int EPI0, int EPI1>
+template <int BN, int EPI0, int EPI1, int CG = 1>
 cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const GemmArgs& a0,
                       const CUtensorMap& tmA1, const CUtensorMap& tmB1, const GemmArgs& a1,
                       int num_sms, cudaStream_t st) {
-  using C = TcCfg<BN, epi_warps<EPI0>()>;
+  using C = TcCfg<BN, epi_warps<EPI0>(), CG>;
+  auto kernel = k_gemm_tc<BN, EPI0, EPI1, CG>;
   static bool attr_set = false;  // per process; the attribute is per function
+  static int pair_slots = 0;     // CG = 2: CTA pairs resident at once
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI0, EPI1>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
     if (e != cudaSuccess) return e;
+    if (CG == 2) {
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = CG;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cudaLaunchConfig_t q = {};
+      q.gridDim = dim3(CG * (num_sms / CG));
+      q.blockDim = dim3(C::THREADS);
+      q.dynamicSmemBytes = C::SMEM;
+      q.attrs = at;
+      q.numAttrs = 1;
+      e = cudaOccupancyMaxActiveClusters(&pair_slots, kernel, &q);
+      if (e != cudaSuccess) return e;
+      if (pair_slots < 1) return cudaErrorInvalidConfiguration;
+    }
     attr_set = true;
   }
-  if (a0.k_splits > 1 && EPI0 != EPI_STORE_F32) return cudaErrorInvalidValue;
+  if (a0.k_splits > 1 && (EPI0 != EPI_STORE_F32 || CG != 1)) return cudaErrorInvalidValue;
   const long kb0 = (a0.K + BK - 1) / BK;
   if (a0.k_splits > 1 && (a0.k_splits > kb0 || (long)(a0.k_splits - 1) *
                                                  ((kb0 + a0.k_splits - 1) / a0.k_splits) >= kb0))
     return cudaErrorInvalidValue;   // every split must own at least one K-block
-  long max_tiles = (long)((a0.m_max + BM - 1) / BM) * ((a0.N + BN - 1) / BN) *
+  const long tile_rows = (long)BM * CG;
+  long max_tiles = (long)((a0.m_max + tile_rows - 1) / tile_rows) * ((a0.N + BN - 1) / BN) *
                    (a0.k_splits > 1 ? a0.k_splits : 1);
-  if (EPI1 != EPI_NONE) max_tiles += (long)((a1.m_max + BM - 1) / BM) * ((a1.N + BN - 1) / BN);
+  if (EPI1 != EPI_NONE)
+    max_tiles += (long)((a1.m_max + tile_rows - 1) / tile_rows) * ((a1.N + BN - 1) / BN);
   if (max_tiles <= 0) return cudaSuccess;
-  const int grid = (int)(max_tiles < num_sms ? max_tiles : num_sms);
+  const long slots = CG == 2 ? (long)pair_slots : (long)num_sms;
+  const int units = (int)(max_tiles < slots ? max_tiles : slots);
   GemmArgs b0 = a0;
   b0.wait_ns = wait_limit_ns();
-  return launch_pdl(k_gemm_tc<BN, EPI0, EPI1>, dim3(grid), dim3(C::THREADS), C::SMEM, st, tmA0, tmB0,
-                    tmA1, tmB1, b0, a1);
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = CG;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(units * CG);
+  cfg.blockDim = dim3(C::THREADS);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = CG == 2 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, tmA0, tmB0, tmA1, tmB1, b0, a1);
 }
 
 }  // namespace
@@ -814,6 +918,30 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
     default:
       return cudaErrorInvalidValue;
   }
+}
+
+cudaError_t launch_gemm_tc2(EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                            const GemmArgs& args, int num_sms, cudaStream_t st) {
+  const GemmArgs none{};
+  switch (epi) {
+    case EPI_STORE_F32:
+      return launch_tc<256, EPI_STORE_F32, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_SWIGLU:
+      return launch_tc<256, EPI_SWIGLU, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_LAYER_OUT:
+      return launch_tc<256, EPI_LAYER_OUT, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_gemm_tc2_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUtensorMap& tmB0,
+                                 const GemmArgs& a0, EpiKind epi1, const CUtensorMap& tmA1,
+                                 const CUtensorMap& tmB1, const GemmArgs& a1, int num_sms,
+                                 cudaStream_t st) {
+  if (epi0 == EPI_SWIGLU && epi1 == EPI_SILU)
+    return launch_tc<256, EPI_SWIGLU, EPI_SILU, 2>(tmA0, tmB0, a0, tmA1, tmB1, a1, num_sms, st);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm_tc_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUtensorMap& tmB0,

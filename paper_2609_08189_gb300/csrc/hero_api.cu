@@ -151,6 +151,9 @@ struct hero_model {
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
   std::vector<CUtensorMap> tm_wgu, tm_wd, tm_w1, tm_w2;
+  // the same weights with 128-row boxes: the B operands of the CTA-pair GEMM
+  CUtensorMap tm_wr_p;
+  std::vector<CUtensorMap> tm_wgu_p, tm_wd_p, tm_w1_p;
 
   // attention sublayer of the full decoder forward (hero_attn_init; bf16 models)
   bool attn = false;
@@ -293,6 +296,9 @@ int choose_splits(int tiles, int kblocks, int num_sms, long rows, long n, int ep
   }
   return best;
 }
+
+// Token counts from which the large GEMMs of a block run on CTA pairs (256-row tiles).
+constexpr int kPairMinRows = 1024;
 
 // Largest split-K partial buffer (floats) any token count up to T may ask for.
 size_t splitk_ws_floats(int T, int num_sms, int nY, int K_router, int d, int I) {
@@ -627,19 +633,26 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
               encode_bf16_2d(&m->tm_act, m->act, I, Tm, 128) &&
               encode_bf16_2d(&m->tm_ah, m->ah, r, Tm, 128) &&
               encode_bf16_2d(&m->tm_wr, m->wr, 2 * d, nY, 256);
+    ok = ok && encode_bf16_2d(&m->tm_wr_p, m->wr, 2 * d, nY, 128);
     m->tm_wgu.resize(L);
     m->tm_wd.resize(L);
     m->tm_w1.resize(L);
     m->tm_w2.resize(L);
+    m->tm_wgu_p.resize(L);
+    m->tm_wd_p.resize(L);
+    m->tm_w1_p.resize(L);
     for (long j = 0; j < L && ok; ++j) {
-      ok = encode_bf16_2d(&m->tm_wgu[j], static_cast<char*>(m->wgu) + (size_t)j * 2 * I * d * 2, d,
-                          2 * I, 256) &&
-           encode_bf16_2d(&m->tm_wd[j], static_cast<char*>(m->wdown) + (size_t)j * d * I * 2, I, d,
-                          256) &&
-           encode_bf16_2d(&m->tm_w1[j], static_cast<char*>(m->w1) + (size_t)j * r * d * 2, d, r,
-                          256) &&
+      const char* wgu_j = static_cast<char*>(m->wgu) + (size_t)j * 2 * I * d * 2;
+      const char* wd_j = static_cast<char*>(m->wdown) + (size_t)j * d * I * 2;
+      const char* w1_j = static_cast<char*>(m->w1) + (size_t)j * r * d * 2;
+      ok = encode_bf16_2d(&m->tm_wgu[j], wgu_j, d, 2 * I, 256) &&
+           encode_bf16_2d(&m->tm_wd[j], wd_j, I, d, 256) &&
+           encode_bf16_2d(&m->tm_w1[j], w1_j, d, r, 256) &&
            encode_bf16_2d(&m->tm_w2[j], static_cast<char*>(m->w2) + (size_t)j * d * r * 2, r, d,
-                          256);
+                          256) &&
+           encode_bf16_2d(&m->tm_wgu_p[j], wgu_j, d, 2 * I, 128) &&
+           encode_bf16_2d(&m->tm_wd_p[j], wd_j, I, d, 128) &&
+           encode_bf16_2d(&m->tm_w1_p[j], w1_j, d, r, 128);
     }
     if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
   }
@@ -708,9 +721,11 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       g.k_splits = rs;
       g.split_stride = (long)m_t * 128 * nY;
     }
+    const bool pair = m->bf16 && rs == 1 && T >= kPairMinRows;
     CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
-      return m->bf16 ? launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st)
-                     : launch_gemm_simt(EPI_STORE_F32, g, st);
+      if (!m->bf16) return launch_gemm_simt(EPI_STORE_F32, g, st);
+      return pair ? launch_gemm_tc2(EPI_STORE_F32, m->tm_xl, m->tm_wr_p, g, m->num_sms, st)
+                  : launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st);
     }));
 
     RouterArgs ra{};
@@ -806,7 +821,13 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     au.lo = lo;
     au.lo.idx = m->idx_a;
     au.lo.scale = m->scale_a;
+    // large batches run the FFN GEMMs on CTA pairs (256-row tiles, the 2-SM MMA)
+    const bool pair = T >= kPairMinRows;
     CUDA_TRY(timed(m, HERO_K_FFN_GATE_UP, st, [&] {
+      if (pair)
+        return dense ? launch_gemm_tc2(EPI_SWIGLU, m->tm_uf, m->tm_wgu_p[jj], gu, m->num_sms, st)
+                     : launch_gemm_tc2_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu_p[jj], gu, EPI_SILU,
+                                            m->tm_ua, m->tm_w1_p[jj], ad, m->num_sms, st);
       return dense ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st)
                    : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU, m->tm_ua,
                                          m->tm_w1[jj], ad, m->num_sms, st);
@@ -855,7 +876,8 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     GemmArgs dl = dn;
     dl.pdl_mode = adapter_after ? 1 : 0;
     CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
-      return launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dl, m->num_sms, st);
+      return pair ? launch_gemm_tc2(EPI_LAYER_OUT, m->tm_act, m->tm_wd_p[jj], dl, m->num_sms, st)
+                  : launch_gemm_tc(256, EPI_LAYER_OUT, m->tm_act, m->tm_wd[jj], dl, m->num_sms, st);
     }));
     return adapter_after ? adapter_up_wide(2) : HERO_OK;
   }
@@ -1741,8 +1763,10 @@ extern "C" hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B
   }
   int sms = 0;
   CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  // M >= 1024 runs on CTA pairs (256-row tiles, 128-row B boxes), as the large FFN GEMMs do
+  const bool pair = M >= 1024;
   CUtensorMap ta, tb;
-  if (!encode_bf16_2d(&ta, A, K, M, 128) || !encode_bf16_2d(&tb, B, K, N, 256))
+  if (!encode_bf16_2d(&ta, A, K, M, 128) || !encode_bf16_2d(&tb, B, K, N, pair ? 128 : 256))
     return fail(HERO_ERR_CUDA, "tensor map encoding failed");
   GemmArgs g{};
   g.m_static = M;
@@ -1753,7 +1777,8 @@ extern "C" hero_status hero_gemm_bf16_check(const uint16_t* A, const uint16_t* B
   g.ldo = N;
   g.err = err;
   const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  CUDA_TRY(launch_gemm_tc(256, EPI_STORE_F32, ta, tb, g, sms, st));
+  CUDA_TRY(pair ? launch_gemm_tc2(EPI_STORE_F32, ta, tb, g, sms, st)
+                : launch_gemm_tc(256, EPI_STORE_F32, ta, tb, g, sms, st));
   // synchronous: report (and clear) what the kernel recorded in the error word
   CUDA_TRY(cudaStreamSynchronize(st));
   uint32_t e = 0;

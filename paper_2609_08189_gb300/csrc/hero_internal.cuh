@@ -174,6 +174,17 @@ cudaError_t launch_gemm_tc_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUt
                                 const CUtensorMap& tmB1, const GemmArgs& a1, int num_sms,
                                 cudaStream_t st);
 
+// The same GEMM on CTA pairs (clusters of 2, the 2-SM MMA): 256 x 256 tiles, each CTA
+// staging 128 rows of A and 128 rows of B per K-block.  tmB must use 128-row boxes (the
+// 1-CTA kernel's B maps use 256-row boxes); A maps are the same.  No split-K.  EPI_STORE_F32,
+// EPI_SWIGLU and EPI_LAYER_OUT, and the grouped (SWIGLU, SILU) launch.
+cudaError_t launch_gemm_tc2(EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                            const GemmArgs& args, int num_sms, cudaStream_t st);
+cudaError_t launch_gemm_tc2_pair(EpiKind epi0, const CUtensorMap& tmA0, const CUtensorMap& tmB0,
+                                 const GemmArgs& a0, EpiKind epi1, const CUtensorMap& tmA1,
+                                 const CUtensorMap& tmB1, const GemmArgs& a1, int num_sms,
+                                 cudaStream_t st);
+
 // SIMT fp32 GEMM with the same epilogues (f32 models).
 cudaError_t launch_gemm_simt(EpiKind epi, const GemmArgs& args, cudaStream_t st);
 constexpr int kSimtTileN = 64;
