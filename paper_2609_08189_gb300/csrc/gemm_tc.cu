@@ -881,6 +881,16 @@ cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const Ge
   return cudaLaunchKernelEx(&cfg, kernel, tmA0, tmB0, tmA1, tmB1, b0, a1);
 }
 
+bool qkv_args_ok(const GemmArgs& a) {
+  return a.N == (a.rope.H + 2 * a.rope.Hkv) * 128 && a.rope.S > 0 && a.rope.S_q > 0 &&
+         a.rope.S_kv > 0 && (a.rope.pos || a.rope.S_kv >= a.rope.S);
+}
+
+bool bw_swiglu_args_ok(const GemmArgs& a) {
+  return a.N % 32 == 0 && a.ldo >= 2 * a.N && a.row_scale && a.row_part &&
+         a.part_ld >= (a.N + 255) / 256;
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
@@ -900,9 +910,7 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
     case EPI_RESIDUAL:
       return launch_tc<256, EPI_RESIDUAL, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_QKV_ROPE:
-      if (args.N != (args.rope.H + 2 * args.rope.Hkv) * 128 || args.rope.S <= 0 ||
-          args.rope.S_q <= 0 || args.rope.S_kv <= 0 || (!args.rope.pos && args.rope.S_kv < args.rope.S))
-        return cudaErrorInvalidValue;
+      if (!qkv_args_ok(args)) return cudaErrorInvalidValue;
       return launch_tc<256, EPI_QKV_ROPE, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_ATTN_ENTRY:
       if (args.lo.d != args.N || args.ldo != args.N) return cudaErrorInvalidValue;
@@ -911,9 +919,7 @@ cudaError_t launch_gemm_tc(int bn, EpiKind epi, const CUtensorMap& tmA, const CU
       if (args.N % 32 != 0) return cudaErrorInvalidValue;
       return launch_tc<256, EPI_STORE_BF16, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_BW_SWIGLU:
-      if (args.N % 32 != 0 || args.ldo < 2 * args.N || !args.row_scale || !args.row_part ||
-          args.part_ld < (args.N + 255) / 256)
-        return cudaErrorInvalidValue;
+      if (!bw_swiglu_args_ok(args)) return cudaErrorInvalidValue;
       return launch_tc<256, EPI_BW_SWIGLU, EPI_NONE>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
@@ -930,6 +936,20 @@ cudaError_t launch_gemm_tc2(EpiKind epi, const CUtensorMap& tmA, const CUtensorM
       return launch_tc<256, EPI_SWIGLU, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     case EPI_LAYER_OUT:
       return launch_tc<256, EPI_LAYER_OUT, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_RESIDUAL:
+      return launch_tc<256, EPI_RESIDUAL, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_QKV_ROPE:
+      if (!qkv_args_ok(args)) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_QKV_ROPE, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_ATTN_ENTRY:
+      if (args.lo.d != args.N || args.ldo != args.N) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_ATTN_ENTRY, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_STORE_BF16:
+      if (args.N % 32 != 0) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_STORE_BF16, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_BW_SWIGLU:
+      if (!bw_swiglu_args_ok(args)) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_BW_SWIGLU, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

@@ -180,7 +180,7 @@ struct hero_model {
   uint16_t* kv_k(int jj) { return static_cast<uint16_t*>(kv) + (size_t)jj * 2 * kv_layer_elems(); }
   uint16_t* kv_v(int jj) { return kv_k(jj) + kv_layer_elems(); }
   CUtensorMap tm_ax, tm_ao;
-  std::vector<CUtensorMap> tm_wqkv, tm_wo;
+  std::vector<CUtensorMap> tm_wqkv, tm_wo, tm_wqkv_p, tm_wo_p;   // _p: 128-row boxes (pair GEMM)
 
   // training path (hero_backward_init; bf16 models): transposed copies of the frozen
   // weights, whose rows are the K-major operands of the input-gradient GEMMs, and the
@@ -195,7 +195,7 @@ struct hero_model {
         *bw_wpart = nullptr;
   int bw_part_ld = 0;
   CUtensorMap tm_bwgf, tm_bwga, tm_bwgu, tm_bwda;
-  std::vector<CUtensorMap> tm_wdT, tm_wguT, tm_w1T, tm_w2T;
+  std::vector<CUtensorMap> tm_wdT, tm_wguT, tm_w1T, tm_w2T, tm_wdT_p, tm_wguT_p;
 
   // measurement
   bool profiling = false;
@@ -1204,8 +1204,10 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   const bool tc = S >= 128 && (size_t)B * Hkv * 128 * S_pad <= m->avt_elems;
   g.rope = RopeArgs{m->aq, kt.k, (kv || !tc) ? kt.v : nullptr, m->rope_cs, nullptr, H, Hkv, S, S,
                     kt.stride, tc ? m->avt : nullptr, S_pad};
+  const bool pair = T >= kPairMinRows;   // large token counts: CTA-pair tiles
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {   // q, k, v with RoPE, attention layout
-    return launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
+    return pair ? launch_gemm_tc2(EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv_p[jj], g, m->num_sms, st)
+                : launch_gemm_tc(256, EPI_QKV_ROPE, m->tm_ax, m->tm_wqkv[jj], g, m->num_sms, st);
   }));
   CUDA_TRY(timed(m, HERO_K_ATTN_CORE, st, [&] {
     if (tc) {
@@ -1230,8 +1232,9 @@ hero_status attention_run(hero_model* m, int jj, int B, int S, const float* h, f
   o.err = m->err;
   if (entry) o.lo = *entry;
   CUDA_TRY(timed(m, HERO_K_ATTN_PROJ, st, [&] {
-    return launch_gemm_tc(256, entry ? EPI_ATTN_ENTRY : EPI_RESIDUAL, m->tm_ao, m->tm_wo[jj], o,
-                          m->num_sms, st);
+    const EpiKind e = entry ? EPI_ATTN_ENTRY : EPI_RESIDUAL;
+    return pair ? launch_gemm_tc2(e, m->tm_ao, m->tm_wo_p[jj], o, m->num_sms, st)
+                : launch_gemm_tc(256, e, m->tm_ao, m->tm_wo[jj], o, m->num_sms, st);
   }));
   return HERO_OK;
 }
@@ -1355,10 +1358,16 @@ extern "C" hero_status hero_attn_init(hero_model* m, const hero_attn_config* ac,
   bool ok = encode_bf16_2d(&m->tm_ax, m->ax, d, Tm, 128) && encode_bf16_2d(&m->tm_ao, m->ao, d, Tm, 128);
   m->tm_wqkv.resize(L);
   m->tm_wo.resize(L);
-  for (long j = 0; j < L && ok; ++j)
-    ok = encode_bf16_2d(&m->tm_wqkv[j], static_cast<char*>(m->wqkv) + (size_t)j * nqkv * d * 2, d,
-                        nqkv, 256) &&
-         encode_bf16_2d(&m->tm_wo[j], static_cast<char*>(m->wo) + (size_t)j * d * d * 2, d, d, 256);
+  m->tm_wqkv_p.resize(L);
+  m->tm_wo_p.resize(L);
+  for (long j = 0; j < L && ok; ++j) {
+    const char* wqkv_j = static_cast<char*>(m->wqkv) + (size_t)j * nqkv * d * 2;
+    const char* wo_j = static_cast<char*>(m->wo) + (size_t)j * d * d * 2;
+    ok = encode_bf16_2d(&m->tm_wqkv[j], wqkv_j, d, nqkv, 256) &&
+         encode_bf16_2d(&m->tm_wo[j], wo_j, d, d, 256) &&
+         encode_bf16_2d(&m->tm_wqkv_p[j], wqkv_j, d, nqkv, 128) &&
+         encode_bf16_2d(&m->tm_wo_p[j], wo_j, d, d, 128);
+  }
   if (!ok) return fail(HERO_ERR_CUDA, "tensor map encoding failed");
   m->n_heads = (int)H;
   m->n_kv_heads = (int)Hkv;
@@ -1855,10 +1864,15 @@ extern "C" hero_status hero_backward_init(hero_model* m) {
   m->tm_wguT.resize(L);
   m->tm_w1T.resize(L);
   m->tm_w2T.resize(L);
+  m->tm_wdT_p.resize(L);
+  m->tm_wguT_p.resize(L);
   for (size_t j = 0; j < L && ok; ++j) {
     ok = encode_bf16_2d(&m->tm_wdT[j], static_cast<char*>(m->wdT) + j * I * d * 2, d, I, 256) &&
          encode_bf16_2d(&m->tm_wguT[j], static_cast<char*>(m->wguT) + j * 2 * I * d * 2, 2 * I, d,
                         256) &&
+         encode_bf16_2d(&m->tm_wdT_p[j], static_cast<char*>(m->wdT) + j * I * d * 2, d, I, 128) &&
+         encode_bf16_2d(&m->tm_wguT_p[j], static_cast<char*>(m->wguT) + j * 2 * I * d * 2, 2 * I,
+                        d, 128) &&
          encode_bf16_2d(&m->tm_w1T[j], static_cast<char*>(m->w1T) + j * d * r * 2, r, d, 256) &&
          encode_bf16_2d(&m->tm_w2T[j], static_cast<char*>(m->w2T) + j * d * r * 2, d, r, 256);
   }
@@ -1913,8 +1927,10 @@ extern "C" hero_status hero_routed_block_backward(hero_model* m, int32_t block, 
   gu.out = m->bw_gu;
   gu.ldo = 2 * I;
   gu.err = m->err;
+  const bool pair = T >= kPairMinRows;   // large token counts: CTA-pair tiles
   CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
-    return launch_gemm_tc(256, EPI_STORE_BF16, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st);
+    return pair ? launch_gemm_tc2(EPI_STORE_BF16, m->tm_uf, m->tm_wgu_p[jj], gu, m->num_sms, st)
+                : launch_gemm_tc(256, EPI_STORE_BF16, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st);
   }));
   GemmArgs ge{};
   ge.m_dev = m->counts;
@@ -1928,7 +1944,8 @@ extern "C" hero_status hero_routed_block_backward(hero_model* m, int32_t block, 
   ge.row_part = m->bw_dgpart;
   ge.part_ld = m->bw_part_ld;
   CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
-    return launch_gemm_tc(256, EPI_BW_SWIGLU, m->tm_bwgf, m->tm_wdT[jj], ge, m->num_sms, st);
+    return pair ? launch_gemm_tc2(EPI_BW_SWIGLU, m->tm_bwgf, m->tm_wdT_p[jj], ge, m->num_sms, st)
+                : launch_gemm_tc(256, EPI_BW_SWIGLU, m->tm_bwgf, m->tm_wdT[jj], ge, m->num_sms, st);
   }));
   GemmArgs gx{};
   gx.m_dev = m->counts;
@@ -1939,7 +1956,8 @@ extern "C" hero_status hero_routed_block_backward(hero_model* m, int32_t block, 
   gx.ldo = d;
   gx.err = m->err;
   CUDA_TRY(timed(m, HERO_K_BACKWARD_GEMM, st, [&] {
-    return launch_gemm_tc(256, EPI_STORE_F32, m->tm_bwgu, m->tm_wguT[jj], gx, m->num_sms, st);
+    return pair ? launch_gemm_tc2(EPI_STORE_F32, m->tm_bwgu, m->tm_wguT_p[jj], gx, m->num_sms, st)
+                : launch_gemm_tc(256, EPI_STORE_F32, m->tm_bwgu, m->tm_wguT[jj], gx, m->num_sms, st);
   }));
   if (!dense) {
     // adapter rows: a = W_1 u and ga = G W_2 (fp32), the hidden-layer backward per row,
