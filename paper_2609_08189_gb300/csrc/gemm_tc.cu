@@ -24,7 +24,9 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int kGroupM = 16;   // raster: 16 M-tiles share each wave of N-tiles (L2 reuse)
+// raster: kGroupM M-tiles share each wave of N-tiles (L2 reuse); CTA-pair tiles are twice
+// as tall, so the pair kernel groups half as many (the same rows per group)
+constexpr int kGroupM = 16;
 
 constexpr int EPI_NONE = -1;   // no second problem
 
@@ -58,11 +60,12 @@ struct TcCfg {
 template <int EPI>
 constexpr int epi_warps() { return EPI == EPI_LAYER_OUT_WIDE || EPI == EPI_ATTN_ENTRY ? 8 : 4; }
 
-__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb) {
-  const int group = kGroupM * n_tiles;
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb,
+                                            int group_m) {
+  const int group = group_m * n_tiles;
   const int g = tile / group;
-  const int first_m = g * kGroupM;
-  const int gm = min(kGroupM, m_tiles - first_m);
+  const int first_m = g * group_m;
+  const int gm = min(group_m, m_tiles - first_m);
   const int local = tile - g * group;
   mb = first_m + local % gm;
   nb = local / gm;
@@ -471,6 +474,7 @@ struct ProbSize {
 };
 
 // Tile `local` of a problem -> coordinates and K-block range.
+template <int CG = 1>
 __device__ __forceinline__ void tile_work(const ProbSize& p, int local, int& mb, int& nb, int& s,
                                           int& kb0, int& kb1);
 
@@ -492,11 +496,12 @@ __device__ __forceinline__ ProbSize prob_size(const GemmArgs& a) {
   return p;
 }
 
+template <int CG>
 __device__ __forceinline__ void tile_work(const ProbSize& p, int local, int& mb, int& nb, int& s,
                                           int& kb0, int& kb1) {
   const int per_split = p.m_tiles * p.n_tiles;
   s = local / per_split;
-  tile_coords(local - s * per_split, p.m_tiles, p.n_tiles, mb, nb);
+  tile_coords(local - s * per_split, p.m_tiles, p.n_tiles, mb, nb, kGroupM / CG);
   kb0 = s * p.kpb;
   kb1 = min(p.kblocks, kb0 + p.kpb);
 }
@@ -639,7 +644,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb, sp, kb0, kb1;
-        tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
+        tile_work<CG>(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         const CUtensorMap* tA = pr ? &tmA1 : &tmA0;
         const CUtensorMap* tB = pr ? &tmB1 : &tmB0;
         if (a0.pdl_mode == 1 && g + n_units >= total)   // this CTA's last tile
@@ -701,7 +706,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
         int local;
         const int pr = split_tile(g, P1.tiles, total, local);
         int mb, nb, sp, kb0, kb1;
-        tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
+        tile_work<CG>(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
         if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, wait_ns) || misc[1]) {
           ok = false;
           break;
@@ -763,7 +768,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
       int local;
       const int pr = split_tile(g, P1.tiles, total, local);
       int mb, nb, sp, kb0, kb1;
-      tile_work(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
+      tile_work<CG>(pr ? P1 : P0, local, mb, nb, sp, kb0, kb1);
       bool ok = mbar_wait(tfull_bar(acc), acc_phase, wait_ns);
       ok = __all_sync(0xffffffffu, ok) && !misc[1];
       ok = __all_sync(0xffffffffu, ok);
