@@ -248,6 +248,173 @@ __device__ __forceinline__ void epi_bw_swiglu(const GemmArgs& a, uint32_t tbase,
   if (valid) a.row_part[(size_t)m * a.part_ld + nb] = dgs;
 }
 
+// ---- the router on the tensor cores (RouterTcArgs) ----
+// x = t0 + t1 + t2 exactly, each a bf16 number (8 significant bits per term; the
+// remainders x - t0 and x - t0 - t1 are exact in fp32).
+__device__ __forceinline__ void split3(float x, uint16_t (&t)[3]) {
+  const __nv_bfloat16 h0 = __float2bfloat16_rn(x);
+  const float r0 = x - __bfloat162float(h0);
+  const __nv_bfloat16 h1 = __float2bfloat16_rn(r0);
+  const float r1 = r0 - __bfloat162float(h1);
+  const __nv_bfloat16 h2 = __float2bfloat16_rn(r1);
+  t[0] = *reinterpret_cast<const uint16_t*>(&h0);
+  t[1] = *reinterpret_cast<const uint16_t*>(&h1);
+  t[2] = *reinterpret_cast<const uint16_t*>(&h2);
+}
+
+// Store 32 fp32 values of row `row` (bf16 terms at columns col, col + stride, col + 2 stride).
+__device__ __forceinline__ void store_split32(uint16_t* row, int col, int stride, const float (&x)[32]) {
+  uint32_t w[3][16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    uint16_t a[3], b[3];
+    split3(x[2 * i], a);
+    split3(x[2 * i + 1], b);
+#pragma unroll
+    for (int p = 0; p < 3; ++p) w[p][i] = (uint32_t)a[p] | ((uint32_t)b[p] << 16);
+  }
+#pragma unroll
+  for (int p = 0; p < 3; ++p) {
+    uint4* dst = reinterpret_cast<uint4*>(row + col + p * stride);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) dst[q] = make_uint4(w[p][4 * q], w[p][4 * q + 1], w[p][4 * q + 2], w[p][4 * q + 3]);
+  }
+}
+
+// Step 1 (the router contraction, Eq. 5 and f_psi's first layer, Eq. 16): column tile 0
+// holds (W_hd diag(g_r)) h_bar, tile 1 W_psi1 h_bar.  Tile 0: 1/rms, d_j and gamma
+// (Eqs. 7-8) from the partial sums, and the encoder hidden SiLU(acc / rms) as three bf16
+// terms; tile 1: f_psi's second layer without its bias.  One thread = one token row.
+template <int BN>
+__device__ __forceinline__ void epi_rt_enc(const GemmArgs& a, uint32_t tbase, int m, bool valid, int nb) {
+  static_assert(BN == 256, "one tile per half of the contraction");
+  const RouterTcArgs& r = a.rt;
+  if (nb == 0) {
+    float rinv = 0.f;
+    if (valid) {
+      float ss = 0.f, dd = 0.f, dp = 0.f;
+      const float4* pp = reinterpret_cast<const float4*>(r.part + (size_t)m * r.np * 4);
+      for (int s = 0; s < r.np; ++s) {
+        const float4 v = pp[s];
+        ss += v.x;
+        dd += v.y;
+        dp += v.z;
+      }
+      rinv = rsqrtf(ss / (float)r.d + r.rms_eps);
+      const float dj = r.j == 1 ? 0.f : sqrtf(dd);                       // Eq. 7
+      const float gam = r.j > 2 ? dp / (dj * r.dprev[m] + r.eps) : 0.f;   // Eq. 8
+      r.scal[(size_t)m * 4 + 0] = dj;
+      r.scal[(size_t)m * 4 + 1] = gam;
+    }
+    uint16_t* row = r.enc3 + (size_t)m * 768;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 256; c0 += 32) {
+      uint32_t v[32];
+      tmem_ld32(tbase + c0, v);
+      if (valid) {
+        float x[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) x[i] = siluf_(__uint_as_float(v[i]) * rinv);
+        store_split32(row, c0, 256, x);
+      }
+    }
+  } else {
+    float bsum = 0.f;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 256; c0 += 32) {
+      uint32_t v[32];
+      tmem_ld32(tbase + c0, v);
+      if (valid) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          bsum = fmaf(__ldg(r.w.ps_w2 + c0 + i), siluf_(__uint_as_float(v[i]) + __ldg(r.w.ps_b1 + c0 + i)), bsum);
+      }
+    }
+    if (valid) r.scal[(size_t)m * 4 + 2] = bsum;
+  }
+}
+
+// Step 2: acc = z_h = W_hu enc (Eq. 5); the path vector (Eqs. 4, 6) and its encoder z_a
+// (Eq. 9); s = [z_h; z_a] in fp32 and as three bf16 terms.
+template <int BN>
+__device__ __forceinline__ void epi_rt_s(const GemmArgs& a, uint32_t tbase, int m, bool valid) {
+  const RouterTcArgs& r = a.rt;
+  constexpr int DH = 48, DA = 16, DP = 16;   // d_h, d_a, d_path of this form (checked on host)
+  float s[DH + DA];
+#pragma unroll
+  for (int c0 = 0; c0 < DH; c0 += 16) {
+    uint32_t v[16];
+    tmem_ld16(tbase + c0, v);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) s[c0 + i] = __uint_as_float(v[i]);
+  }
+  if (!valid) return;
+  const float* sc = r.scal + (size_t)m * 4;
+  const float x[6] = {(float)r.j / (float)r.L, (float)(r.L - r.j) / (float)r.L, sc[0], sc[1],
+                      r.pst[m], r.mst[m]};
+  float hid[DP];
+#pragma unroll
+  for (int o = 0; o < DP; ++o) {
+    float acc = __ldg(r.w.path_b1 + o);
+#pragma unroll
+    for (int i = 0; i < 6; ++i) acc = fmaf(__ldg(r.w.path_w1_t + i * DP + o), x[i], acc);
+    hid[o] = siluf_(acc);
+  }
+#pragma unroll
+  for (int o = 0; o < DA; ++o) {
+    float acc = __ldg(r.w.path_b2 + o);
+#pragma unroll
+    for (int i = 0; i < DP; ++i) acc = fmaf(__ldg(r.w.path_w2_t + i * DA + o), hid[i], acc);
+    s[DH + o] = acc;
+  }
+  float4* so = reinterpret_cast<float4*>(r.s + (size_t)m * (DH + DA));
+#pragma unroll
+  for (int i = 0; i < (DH + DA) / 4; ++i) so[i] = make_float4(s[4 * i], s[4 * i + 1], s[4 * i + 2], s[4 * i + 3]);
+  uint16_t* row = r.s3 + (size_t)m * 3 * (DH + DA);
+  float x32[32];
+#pragma unroll
+  for (int h = 0; h < (DH + DA) / 32; ++h) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x32[i] = s[32 * h + i];
+    store_split32(row, 32 * h, DH + DA, x32);
+  }
+}
+
+// Step 5: acc = W_th1 [s; c; nu] (Eq. 14); a = w_th2 . SiLU(acc + b_th1) + b_th2,
+// p_hist = sigma(a / T_hist), m_hist *= p_hist (Eq. 15), g = sigma(a + b) (Eq. 16) and the
+// decision g >= tau (Eq. 3; ties run the FFN) or the caller's.
+template <int BN>
+__device__ __forceinline__ void epi_rt_head(const GemmArgs& a, uint32_t tbase, int m, bool valid) {
+  static_assert(BN == 256, "f_theta's hidden width is one tile");
+  const RouterTcArgs& r = a.rt;
+  float asum = 0.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < 256; c0 += 32) {
+    uint32_t v[32];
+    tmem_ld32(tbase + c0, v);
+    if (valid) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        asum = fmaf(__ldg(r.w.th_w2 + c0 + i), siluf_(__uint_as_float(v[i]) + __ldg(r.w.th_b1 + c0 + i)), asum);
+    }
+  }
+  if (!valid) return;
+  const float* sc = r.scal + (size_t)m * 4;
+  const float av = asum + __ldg(r.w.th_b2);
+  const float bv = sc[2] + __ldg(r.w.ps_b2);
+  const float p = sigmoidf_(av / r.t_hist);
+  const float mm = r.mst[m] * p;
+  const float g = sigmoidf_(av + bv);
+  const uint8_t dec = r.mask_in ? (r.mask_in[m] ? 1 : 0) : (g >= r.tau ? 1 : 0);
+  r.pst[m] = p;
+  r.mst[m] = mm;
+  r.dprev[m] = sc[0];
+  r.gate[m] = g;
+  r.mask[m] = dec;
+  if (r.gate_out) r.gate_out[m] = g;
+  if (r.mask_out) r.mask_out[m] = dec;
+}
+
 // Fused q/k/v projection epilogue: one thread = one token row; the two halves of a
 // head (columns i and i + 64) are read from TMEM together, q and k heads are
 // rotated (RoPE, fp32), and each head's 128 values are stored as bf16 into its
@@ -547,6 +714,12 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
     epi_store_bf16<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
   } else if constexpr (EPI == EPI_BW_SWIGLU) {
     epi_bw_swiglu<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_RT_ENC) {
+    epi_rt_enc<BN>(a, tbase, row0 + lane, row0 + lane < M, nb);
+  } else if constexpr (EPI == EPI_RT_S) {
+    epi_rt_s<BN>(a, tbase, row0 + lane, row0 + lane < M);
+  } else if constexpr (EPI == EPI_RT_HEAD) {
+    epi_rt_head<BN>(a, tbase, row0 + lane, row0 + lane < M);
   } else if constexpr (EPI == EPI_LAYER_OUT) {
     epi_layer_out<BN, BN>(a, tbase, row0, M, nb, 0, stg);
   } else {
@@ -955,6 +1128,16 @@ cudaError_t launch_gemm_tc2(EpiKind epi, const CUtensorMap& tmA, const CUtensorM
     case EPI_BW_SWIGLU:
       if (!bw_swiglu_args_ok(args)) return cudaErrorInvalidValue;
       return launch_tc<256, EPI_BW_SWIGLU, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_RT_ENC:
+      if (args.N != 512) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_RT_ENC, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_RT_S:
+      if (args.N != 48 || args.rt.d_h != 48 || args.rt.d_a != 16 || args.rt.d_path != 16)
+        return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_RT_S, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
+    case EPI_RT_HEAD:
+      if (args.N != 256) return cudaErrorInvalidValue;
+      return launch_tc<256, EPI_RT_HEAD, EPI_NONE, 2>(tmA, tmB, args, tmA, tmB, none, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

@@ -87,6 +87,21 @@ bool encode_bf16_3d(CUtensorMap* tm, const void* ptr, uint64_t d0, uint64_t d1, 
   return r == CUDA_SUCCESS;
 }
 
+// Nearest bf16 (ties to even) of an fp32 value, as its 16-bit pattern.
+uint16_t bf16_bits(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  if ((u & 0x7fffffffu) > 0x7f800000u) return (uint16_t)((u >> 16) | 0x40u);   // NaN stays NaN
+  return (uint16_t)((u + 0x7fffu + ((u >> 16) & 1u)) >> 16);
+}
+
+float bf16_value(float f) {
+  const uint32_t u = (uint32_t)bf16_bits(f) << 16;
+  float r;
+  memcpy(&r, &u, 4);
+  return r;
+}
+
 std::vector<float> host_f32(const void* p, size_t n, hero_dtype dt) {
   std::vector<float> v(n);
   if (dt == HERO_BF16) {
@@ -133,6 +148,13 @@ struct hero_model {
   size_t ws_bytes = 0;
   float *hbar, *delta, *part, *Y, *S, *zeta, *pst, *mst, *dprev, *gate, *scale_f, *scale_a;
   float* splitk_ws = nullptr;   // bf16: partial slices of split-K GEMMs (few-tile launches)
+  // the router on the tensor cores (RouterTcArgs): weights, maps and per-token buffers
+  bool rtc = false;
+  int rt_kf = 0;
+  void* rt_w = nullptr;
+  CUtensorMap tm_whu3, tm_wq3, tm_th3, tm_enc3, tm_s3, tm_fin3;
+  uint16_t *rt_enc3 = nullptr, *rt_s3 = nullptr, *rt_fin3 = nullptr;
+  float *rt_scal = nullptr, *rt_s = nullptr, *rt_qkvn = nullptr;
   void *xl, *u_f, *u_a, *act, *ah;
   uint8_t* mask;
   int *idx_f, *idx_a, *counts;
@@ -349,7 +371,8 @@ void free_model(hero_model* m) {
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
-                  m->dec_pm, m->dec_pos, m->dec_ws, m->wdT, m->wguT, m->w1T, m->w2T, m->bws};
+                  m->dec_pm, m->dec_pos, m->dec_ws, m->wdT, m->wguT, m->w1T, m->w2T, m->bws,
+                  m->rt_w};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -535,10 +558,17 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     m->rho.resize(L);
     for (long j = 0; j < L; ++j) m->rho[j] = (float)(1.0 / (1.0 + std::exp(-(double)eta[j])));
   }
-  {  // shared router parameters, transposed to [in][out]
+  {  // shared router parameters, transposed to [in][out]; bf16 models round every
+     // parameter to bf16 (the precision contract), these included
     std::vector<float> pack;
+    auto params = [&](const void* src, size_t n) {
+      std::vector<float> v = host_f32(src, n, hd);
+      if (bf16)
+        for (float& x : v) x = bf16_value(x);
+      return v;
+    };
     auto add_t = [&](const void* src, long rows, long cols) {  // src [rows][cols] -> [cols][rows]
-      std::vector<float> v = host_f32(src, (size_t)rows * cols, hd);
+      std::vector<float> v = params(src, (size_t)rows * cols);
       pack.resize((pack.size() + 3) & ~(size_t)3);  // 16-byte aligned sub-arrays
       size_t at = pack.size();
       pack.resize(at + (size_t)rows * cols);
@@ -547,7 +577,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
       return at;
     };
     auto add = [&](const void* src, long n) {
-      std::vector<float> v = host_f32(src, n, hd);
+      std::vector<float> v = params(src, n);
       pack.resize((pack.size() + 3) & ~(size_t)3);
       size_t at = pack.size();
       pack.insert(pack.end(), v.begin(), v.end());
@@ -565,7 +595,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     {
       const void* src[3] = {w->w_q, w->w_k, w->w_v};
       for (int p = 0; p < 3; ++p) {
-        std::vector<float> v = host_f32(src[p], (size_t)dm * ds, hd);
+        std::vector<float> v = params(src[p], (size_t)dm * ds);
         for (long i = 0; i < dm; ++i)
           for (long k = 0; k < ds; ++k)
             pack[o_qkv + (size_t)k * 3 * dm + p * dm + i] = v[(size_t)i * ds + k];
@@ -587,6 +617,43 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     m->rw = RouterWeights{b + o_hu, b + o_p1, b + o_pb1, b + o_p2, b + o_pb2, b + o_qkv, b + o_n,
                           b + o_c,  b + o_t1, b + o_tb1, b + o_t2, b + o_tb2, b + o_pb, b + o_p2w,
                           b + o_p2b};
+    // the router on the tensor cores (large token counts): W_hu, [W_q; W_k; W_v; W_n] and
+    // W_th1 as bf16 B operands, each repeated three times along K (one copy per bf16 term
+    // of the activation), f_theta's K zero-padded to a multiple of 64
+    m->rtc = bf16 && c.d_enc == 256 && c.d_head == 256 && c.d_h == 48 && c.d_a == 16 &&
+             c.d_path == 16 && dm <= 128 && c.max_tokens >= kPairMinRows;
+    if (m->rtc) {
+      const long F = ds + dm + 1;
+      m->rt_kf = (int)((3 * F + 63) / 64 * 64);
+      std::vector<uint16_t> whu3((size_t)c.d_h * 768), wq3((size_t)4 * dm * 3 * ds),
+          th3((size_t)c.d_head * m->rt_kf, 0);
+      const std::vector<float> hu = params(w->w_hu, (size_t)c.d_h * c.d_enc);
+      for (long o = 0; o < c.d_h; ++o)
+        for (int pp = 0; pp < 3; ++pp)
+          for (long i = 0; i < 256; ++i) whu3[o * 768 + pp * 256 + i] = bf16_bits(hu[o * 256 + i]);
+      const void* qs[4] = {w->w_q, w->w_k, w->w_v, w->w_n};
+      for (int r4 = 0; r4 < 4; ++r4) {
+        const std::vector<float> v = params(qs[r4], (size_t)dm * ds);
+        for (long o = 0; o < dm; ++o)
+          for (int pp = 0; pp < 3; ++pp)
+            for (long i = 0; i < ds; ++i)
+              wq3[((size_t)r4 * dm + o) * 3 * ds + pp * ds + i] = bf16_bits(v[o * ds + i]);
+      }
+      const std::vector<float> th = params(w->th_w1, (size_t)c.d_head * F);
+      for (long o = 0; o < c.d_head; ++o)
+        for (int pp = 0; pp < 3; ++pp)
+          for (long i = 0; i < F; ++i) th3[(size_t)o * m->rt_kf + pp * F + i] = bf16_bits(th[o * F + i]);
+      const size_t n_hu = whu3.size(), n_q = wq3.size(), n_th = th3.size();
+      CUDA_M(cudaMalloc(&m->rt_w, (n_hu + n_q + n_th) * 2));
+      uint16_t* rb = static_cast<uint16_t*>(m->rt_w);
+      CUDA_M(cudaMemcpy(rb, whu3.data(), n_hu * 2, cudaMemcpyHostToDevice));
+      CUDA_M(cudaMemcpy(rb + n_hu, wq3.data(), n_q * 2, cudaMemcpyHostToDevice));
+      CUDA_M(cudaMemcpy(rb + n_hu + n_q, th3.data(), n_th * 2, cudaMemcpyHostToDevice));
+      if (!encode_bf16_2d(&m->tm_whu3, rb, 768, c.d_h, 128) ||
+          !encode_bf16_2d(&m->tm_wq3, rb + n_hu, 3 * ds, 4 * dm, 128) ||
+          !encode_bf16_2d(&m->tm_th3, rb + n_hu + n_q, m->rt_kf, c.d_head, 128))
+        return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
+    }
   }
 
   // ---- workspace ----
@@ -609,6 +676,12 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         {(void**)&m->ah, Tm * r * es},         {(void**)&m->mask, Tm},
         {(void**)&m->idx_f, Tm * 4},           {(void**)&m->idx_a, Tm * 4},
         {(void**)&m->counts, 64},              {(void**)&m->err, 64},
+        {(void**)&m->rt_enc3, m->rtc ? Tm * 768 * 2 : 0},
+        {(void**)&m->rt_scal, m->rtc ? Tm * 4 * 4 : 0},
+        {(void**)&m->rt_s, m->rtc ? Tm * ds * 4 : 0},
+        {(void**)&m->rt_s3, m->rtc ? Tm * 3 * ds * 2 : 0},
+        {(void**)&m->rt_qkvn, m->rtc ? Tm * 4 * dm * 4 : 0},
+        {(void**)&m->rt_fin3, m->rtc ? Tm * (size_t)m->rt_kf * 2 : 0},
         // split-K partials of the few-wave launches (router contraction, FFN down)
         {(void**)&m->splitk_ws, bf16 ? splitk_ws_floats(c.max_tokens, m->num_sms, (int)nY,
                                                         (int)(2 * d), (int)d, (int)I) * 4 : 0},
@@ -634,6 +707,10 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
               encode_bf16_2d(&m->tm_ah, m->ah, r, Tm, 128) &&
               encode_bf16_2d(&m->tm_wr, m->wr, 2 * d, nY, 256);
     ok = ok && encode_bf16_2d(&m->tm_wr_p, m->wr, 2 * d, nY, 128);
+    if (m->rtc)
+      ok = ok && encode_bf16_2d(&m->tm_enc3, m->rt_enc3, 768, Tm, 128) &&
+           encode_bf16_2d(&m->tm_s3, m->rt_s3, 3 * ds, Tm, 128) &&
+           encode_bf16_2d(&m->tm_fin3, m->rt_fin3, m->rt_kf, Tm, 128);
     m->tm_wgu.resize(L);
     m->tm_wd.resize(L);
     m->tm_w1.resize(L);
@@ -722,6 +799,74 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       g.split_stride = (long)m_t * 128 * nY;
     }
     const bool pair = m->bf16 && rs == 1 && T >= kPairMinRows;
+    if (pair && m->rtc && c.router_variant == 0) {
+      // the router on the tensor cores: five launches (RouterTcArgs)
+      RouterTcArgs rt{};
+      rt.T = T;
+      rt.j = j;
+      rt.L = L - c.n_dense;
+      rt.np = m->np;
+      rt.d = d;
+      rt.d_h = c.d_h;
+      rt.d_a = c.d_a;
+      rt.d_path = c.d_path;
+      rt.dm = c.d_m;
+      rt.rms_eps = c.rms_eps;
+      rt.eps = c.eps;
+      rt.t_hist = c.t_hist;
+      rt.tau = tau;
+      rt.rho = m->rho[jj];
+      rt.part = m->part;
+      rt.dprev = bs.dprev;
+      rt.pst = bs.pst;
+      rt.mst = bs.mst;
+      rt.S = bs.S;
+      rt.zeta = bs.zeta;
+      rt.w = m->rw;
+      rt.enc3 = m->rt_enc3;
+      rt.scal = m->rt_scal;
+      rt.s = m->rt_s;
+      rt.s3 = m->rt_s3;
+      rt.qkvn = m->rt_qkvn;
+      rt.fin3 = m->rt_fin3;
+      rt.kf = m->rt_kf;
+      rt.mask_in = mask_in_j;
+      rt.gate = m->gate;
+      rt.mask = m->mask;
+      rt.gate_out = gate_out_j;
+      rt.mask_out = mask_out_j;
+      const int ds = c.d_h + c.d_a;
+      GemmArgs g1 = g;   // 1. the router contraction, encoder hidden and f_psi in the epilogue
+      g1.rt = rt;
+      CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
+        return launch_gemm_tc2(EPI_RT_ENC, m->tm_xl, m->tm_wr_p, g1, m->num_sms, st);
+      }));
+      auto small = [&](int N, int K) {
+        GemmArgs q{};
+        q.m_static = T;
+        q.m_max = T;
+        q.N = N;
+        q.K = K;
+        q.err = m->err;
+        q.rt = rt;
+        return q;
+      };
+      GemmArgs g2 = small(c.d_h, 3 * 256);   // 2. z_h = W_hu enc; path encoder; s
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
+        return launch_gemm_tc2(EPI_RT_S, m->tm_enc3, m->tm_whu3, g2, m->num_sms, st);
+      }));
+      GemmArgs g3 = small(4 * c.d_m, 3 * ds);   // 3. q | k | v | W_n s
+      g3.out_f32 = m->rt_qkvn;
+      g3.ldo = 4 * c.d_m;
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
+        return launch_gemm_tc2(EPI_STORE_F32, m->tm_s3, m->tm_wq3, g3, m->num_sms, st);
+      }));
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_rt_mem(rt, st); }));   // 4.
+      GemmArgs g5 = small(c.d_head, m->rt_kf);   // 5. f_theta, p_hist, m_hist, g, decision
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
+        return launch_gemm_tc2(EPI_RT_HEAD, m->tm_fin3, m->tm_th3, g5, m->num_sms, st);
+      }));
+    } else {
     CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
       if (!m->bf16) return launch_gemm_simt(EPI_STORE_F32, g, st);
       return pair ? launch_gemm_tc2(EPI_STORE_F32, m->tm_xl, m->tm_wr_p, g, m->num_sms, st)
@@ -761,6 +906,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.mask_out = mask_out_j;
     ra.variant = c.router_variant;
     CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, m->num_sms, st); }));
+    }
   }
   CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
                  m->counts, count_out_j, dense ? gate_out_j : nullptr,

@@ -101,6 +101,12 @@ enum EpiKind : int {
   EPI_QKV_ROPE = 7,    // fused q/k/v projection: RoPE on the q and k heads, bf16 out in
                        // the attention layout (RopeArgs)
   EPI_STORE_BF16 = 8,  // out[m, n] = bf16(acc) (N a multiple of 32)
+  EPI_RT_ENC = 10,     // router on the tensor cores, step 1 (RouterTcArgs): the router
+                       // contraction's columns [0, 256) -> SiLU(rinv acc) as three bf16 terms,
+                       // [256, 512) -> b, plus d_j and gamma from the partial sums
+  EPI_RT_S = 11,       // step 2: acc = z_h = W_hu enc; the path encoder; s = [z_h; z_a]
+  EPI_RT_HEAD = 12,    // step 5: acc = W_th1 [s; c; nu]; f_theta's second layer, p_hist,
+                       // m_hist, g and the decision
   EPI_BW_SWIGLU = 9,   // backward of the SwiGLU product (training path): acc = e = dL/dy W_down
                        // for features n of row m; out holds the row's bf16 gate/up
                        // pre-activations in the interleaved layout and is overwritten in place
@@ -121,6 +127,56 @@ struct RopeArgs {
   int H, Hkv, S, S_q, S_kv;
   void* vt;            // bf16 [B][H_kv][128][S_pad]: v transposed (keys contiguous), or nullptr
   int S_pad;           // positions per row of vt (a multiple of 8)
+};
+
+struct RouterWeights {   // shared router parameters, fp32, transposed to [in][out]
+  const float* w_hu_t;    // [d_enc][d_h]
+  const float* path_w1_t; // [6][d_path]
+  const float* path_b1;   // [d_path]
+  const float* path_w2_t; // [d_path][d_a]
+  const float* path_b2;   // [d_a]
+  const float* w_qkv_t;   // [d_s][3 d_m]  (q | k | v)
+  const float* w_n_t;     // [d_s][d_m]
+  const float* w_c_t;     // [d_m][d_m]
+  const float* th_w1_t;   // [d_s + d_m + 1][d_head]
+  const float* th_b1;     // [d_head]
+  const float* th_w2;     // [d_head]
+  const float* th_b2;     // [1]
+  const float* ps_b1;     // [d_head]
+  const float* ps_w2;     // [d_head]
+  const float* ps_b2;     // [1]
+};
+
+// The HeRo router (no ablation) at large token counts on the tensor cores.  Its small
+// matrices hold bf16 values; an fp32 activation x splits exactly into three bf16 terms
+// x = x_0 + x_1 + x_2 (x_0 = bf16(x), x_1 = bf16(x - x_0), x_2 = bf16(x - x_0 - x_1)), so
+// with the weight matrix repeated three times along K each tensor-core product is exact and
+// the sums accumulate in fp32: the precision of the fp32 FMA router.  Five launches per
+// block: the router contraction with EPI_RT_ENC; W_hu with EPI_RT_S; [W_q; W_k; W_v; W_n]
+// with a plain fp32 store; the memory step (k_rt_mem: memory read and write, W_c c, nu, the
+// f_theta input); W_th1 with EPI_RT_HEAD.  Per-token buffers below (T rows each).
+struct RouterTcArgs {
+  int T, j, L, np, d, d_h, d_a, d_path, dm;
+  float rms_eps, eps, t_hist, tau, rho;
+  const float* part;     // [T, np, 4] partial sums of h_bar (Eqs. 5, 7-8)
+  float* dprev;          // [T] in: d_{j-1} (step 1); out: d_j (step 5)
+  float* pst;            // [T] p_hist
+  float* mst;            // [T] m_hist
+  float* S;              // [T, dm, dm]
+  float* zeta;           // [T, dm]
+  RouterWeights w;
+  uint16_t* enc3;        // [T, 768] bf16: the encoder hidden's three terms
+  float* scal;           // [T, 4]: d_j, gamma, f_psi's second layer without bias
+  float* s;              // [T, d_s] router state s (Eq. 9)
+  uint16_t* s3;          // [T, 3 d_s] bf16: s's three terms
+  float* qkvn;           // [T, 4 dm]: q | k | v | W_n s (Eqs. 10, 13)
+  uint16_t* fin3;        // [T, kf] bf16: [s; c; nu]'s three terms, zero beyond 3 (d_s + dm + 1)
+  int kf;
+  const uint8_t* mask_in;
+  float* gate;
+  uint8_t* mask;
+  float* gate_out;
+  uint8_t* mask_out;
 };
 
 struct GemmArgs {
@@ -150,6 +206,7 @@ struct GemmArgs {
   const float* row_scale;  // EPI_BW_SWIGLU: [rows] branch scale g
   float* row_part;     // EPI_BW_SWIGLU: [rows, part_ld] per-tile sums
   int part_ld;
+  RouterTcArgs rt;     // EPI_RT_*
   // SIMT path only (row-major [rows, K] operands)
   const void* A;
   const void* B;
@@ -214,23 +271,6 @@ cudaError_t launch_attn_decode(const void* Q, const void* K, const void* V, cons
 
 // Router and bookkeeping kernels ------------------------------------------------
 
-struct RouterWeights {   // shared router parameters, fp32, transposed to [in][out]
-  const float* w_hu_t;    // [d_enc][d_h]
-  const float* path_w1_t; // [6][d_path]
-  const float* path_b1;   // [d_path]
-  const float* path_w2_t; // [d_path][d_a]
-  const float* path_b2;   // [d_a]
-  const float* w_qkv_t;   // [d_s][3 d_m]  (q | k | v)
-  const float* w_n_t;     // [d_s][d_m]
-  const float* w_c_t;     // [d_m][d_m]
-  const float* th_w1_t;   // [d_s + d_m + 1][d_head]
-  const float* th_b1;     // [d_head]
-  const float* th_w2;     // [d_head]
-  const float* th_b2;     // [1]
-  const float* ps_b1;     // [d_head]
-  const float* ps_w2;     // [d_head]
-  const float* ps_b2;     // [1]
-};
 
 struct RouterArgs {
   int T, j, L, np;       // j is 1-based
@@ -261,6 +301,8 @@ struct RouterArgs {
 enum : uint32_t { RV_NO_HISTORY = 1u, RV_NO_MEMREAD = 2u, RV_NO_AUX = 4u, RV_NO_POS = 8u };
 
 cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st);
+// Step 4 of the tensor-core router (see RouterTcArgs).
+cudaError_t launch_rt_mem(const RouterTcArgs& a, cudaStream_t st);
 
 struct InitArgs {
   int T, d, np, d_m;

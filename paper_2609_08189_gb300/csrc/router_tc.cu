@@ -1,0 +1,131 @@
+// Step 4 of the router on the tensor cores (RouterTcArgs): the per-token part between the
+// q/k/v product and f_theta's first layer, one warp per token.
+//   c = phi(q)^T S / (phi(q)^T zeta + eps)                Eq. 11 (before the write)
+//   S = rho S + phi(k) v^T, zeta = rho zeta + phi(k)      Eq. 12
+//   nu = 1 - cos(W_n s, W_c c) for j > 1, else 0          Eq. 13
+//   f_theta's input [s; c; nu] as three bf16 terms per value (zero padded to kf columns)
+// S is read once and written once; its lanes and the order in which c's partial sums are
+// added follow the fused router's memory step.
+#include "hero_device.cuh"
+
+namespace hero {
+namespace {
+
+__device__ __forceinline__ uint16_t bf16_term(float x, int term) {
+  __nv_bfloat16 h = __float2bfloat16_rn(x);
+  for (int p = 0; p < term; ++p) {
+    x -= __bfloat162float(h);
+    h = __float2bfloat16_rn(x);
+  }
+  return *reinterpret_cast<const uint16_t*>(&h);
+}
+
+template <int DM>
+__global__ void __launch_bounds__(256) k_rt_mem(const RouterTcArgs a) {
+  pdl_enter();
+  static_assert(DM <= 128, "DM / 4 lanes per S row");
+  __shared__ float cbuf[8][DM];
+  __shared__ float cvbuf[8][DM];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * 8 + w;
+  if (t >= a.T) return;   // whole warps only; nothing below synchronises the CTA
+  const float* q = a.qkvn + (size_t)t * 4 * DM;
+  const float* k = q + DM;
+  const float* v = q + 2 * DM;
+  const float* wn = q + 3 * DM;   // W_n s
+  float* S = a.S + (size_t)t * DM * DM;
+  float* z = a.zeta + (size_t)t * DM;
+  float den = 0.f;
+  for (int m = lane; m < DM; m += 32) {
+    const float zo = z[m];
+    den += phif_(q[m]) * zo;
+    z[m] = a.rho * zo + phif_(k[m]);
+  }
+  den = warp_sum(den);
+  const float inv = 1.0f / (den + a.eps);
+  constexpr int LPR = DM / 4;          // lanes per S row
+  constexpr int RPI = 32 / LPR;        // rows per iteration
+  constexpr int NIT = DM / RPI;        // S rows handled by this lane
+  constexpr int BATCH = NIT < 8 ? NIT : 8;
+  const int cq = lane % LPR;
+  const int r0 = lane / LPR;
+  float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 vv = *reinterpret_cast<const float4*>(v + 4 * cq);
+#pragma unroll 1
+  for (int i0 = 0; i0 < NIT; i0 += BATCH) {
+    float4 so[BATCH];
+#pragma unroll
+    for (int i = 0; i < BATCH; ++i)
+      so[i] = *reinterpret_cast<const float4*>(S + (r0 + (i0 + i) * RPI) * DM + 4 * cq);
+#pragma unroll
+    for (int i = 0; i < BATCH; ++i) {
+      const int r = r0 + (i0 + i) * RPI;
+      const float fq = phif_(q[r]);
+      const float fk = phif_(k[r]);
+      c.x += fq * so[i].x; c.y += fq * so[i].y; c.z += fq * so[i].z; c.w += fq * so[i].w;
+      *reinterpret_cast<float4*>(S + r * DM + 4 * cq) =
+          make_float4(a.rho * so[i].x + fk * vv.x, a.rho * so[i].y + fk * vv.y,
+                      a.rho * so[i].z + fk * vv.z, a.rho * so[i].w + fk * vv.w);
+    }
+  }
+#pragma unroll
+  for (int o = LPR; o < 32; o <<= 1) {
+    c.x += __shfl_xor_sync(0xffffffffu, c.x, o);
+    c.y += __shfl_xor_sync(0xffffffffu, c.y, o);
+    c.z += __shfl_xor_sync(0xffffffffu, c.z, o);
+    c.w += __shfl_xor_sync(0xffffffffu, c.w, o);
+  }
+  if (r0 == 0)
+    *reinterpret_cast<float4*>(&cbuf[w][4 * cq]) = make_float4(c.x * inv, c.y * inv, c.z * inv, c.w * inv);
+  __syncwarp();
+  // W_c c (Eq. 13), w_c_t is [in][out]
+  for (int o = lane; o < DM; o += 32) {
+    float acc = 0.f;
+    for (int i = 0; i < DM; ++i) acc = fmaf(__ldg(a.w.w_c_t + i * DM + o), cbuf[w][i], acc);
+    cvbuf[w][o] = acc;
+  }
+  __syncwarp();
+  float nu = 0.f;
+  if (a.j > 1) {
+    float xy = 0.f, xx = 0.f, yy = 0.f;
+    for (int o = lane; o < DM; o += 32) {
+      const float x = wn[o], y = cvbuf[w][o];
+      xy += x * y;
+      xx += x * x;
+      yy += y * y;
+    }
+    xy = warp_sum(xy);
+    xx = warp_sum(xx);
+    yy = warp_sum(yy);
+    nu = 1.f - xy / (sqrtf(xx) * sqrtf(yy) + a.eps);
+  }
+  // f_theta's input [s; c; nu]: term p of element e at column p * F + e
+  const int ds = a.d_h + a.d_a, F = ds + DM + 1;
+  const float* s = a.s + (size_t)t * ds;
+  uint16_t* fin = a.fin3 + (size_t)t * a.kf;
+  for (int col = lane; col < a.kf; col += 32) {
+    const int p = col / F, e = col - p * F;
+    uint16_t bits = 0;
+    if (p < 3) {
+      const float x = e < ds ? s[e] : (e < ds + DM ? cbuf[w][e - ds] : nu);
+      bits = bf16_term(x, p);
+    }
+    fin[col] = bits;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_rt_mem(const RouterTcArgs& a, cudaStream_t st) {
+  if (a.T <= 0) return cudaSuccess;
+  const dim3 grid((a.T + 7) / 8);
+  switch (a.dm) {
+    case 16: return launch_pdl(k_rt_mem<16>, grid, dim3(256), 0, st, a);
+    case 32: return launch_pdl(k_rt_mem<32>, grid, dim3(256), 0, st, a);
+    case 64: return launch_pdl(k_rt_mem<64>, grid, dim3(256), 0, st, a);
+    case 128: return launch_pdl(k_rt_mem<128>, grid, dim3(256), 0, st, a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace hero

@@ -170,3 +170,59 @@ def test_block_argument_errors(hero):
     torch.cuda.synchronize()
     st.check()
     st.close()
+
+
+def test_teacher_forced_blocks_tensor_core_router(hero):
+    """Blocks with at least 1024 tokens run the router on the tensor cores (five launches;
+    the router's small matrices as bf16 B operands, each fp32 activation split into three
+    bf16 terms, so every product is exact and the sums accumulate in fp32).  Teacher-forced
+    at Llama-3.1-8B shapes (4 blocks, 1024 tokens): the stated bounds block by block."""
+    import torch
+    base = hi.CONFIGS["llama31_8b_prefill"]
+    cfg = base.replace(n_layers=4, n_tokens=1024)
+    w = hi.generate_weights(cfg)
+    h = hi.generate_h_in(cfg)
+    P = hi.generate_attn_delta(cfg)
+    tau = hi.calibrated_tau(base.name)
+    T, d, dm, L = cfg.n_tokens, cfg.d_model, cfg.d_m, cfg.n_layers
+    ref = ho.routed_ffn_stack(ho.OracleConfig.from_stack(cfg), w, h, P, tau, record=True)
+    lay = ref["layers"]
+    st = hero.HeroStack(cfg, w, max_tokens=T)
+    ts = _state_tensors(T, d, dm)
+    state = hero.make_state(_ptrs(ts))
+    g = torch.empty(T, device="cuda")
+    m = torch.empty(T, device="cuda", dtype=torch.uint8)
+    h_out = torch.empty((T, d), device="cuda")
+    cnt = torch.empty(1, device="cuda", dtype=torch.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    f32 = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.float32), device="cuda")
+    worst_g = worst_h = worst_S = 0.0
+    far = 0
+    for j in range(1, L + 1):
+        if j == 1:
+            hero.hero_router_state_reset(st.model, T, state, stream)
+        else:
+            prev = lay[j - 2]
+            for key, src in (("S", "S"), ("zeta", "zeta"), ("p_hist", "p"), ("m_hist", "m"),
+                             ("d_prev", "d"), ("h_bar_prev", "h_bar"), ("delta_prev", "delta")):
+                ts[key].copy_(f32(prev[src]))
+        cur = lay[j - 1]
+        mask_in = torch.as_tensor(cur["mask"].astype(np.uint8), device="cuda")
+        hero.hero_routed_block(st.model, j, T, f32(cur["h_bar"]).data_ptr(), state, tau,
+                               hero.HERO_FLAG_FORCE_MASK, mask_in.data_ptr(), h_out.data_ptr(),
+                               g.data_ptr(), m.data_ptr(), cnt.data_ptr(), stream)
+        torch.cuda.synchronize()
+        st.check()
+        gg = g.cpu().numpy().astype(np.float64)
+        worst_g = max(worst_g, float(np.max(np.abs(gg - cur["g"]))))
+        worst_h = max(worst_h, float(np.max(pr.rel_err_rows(h_out.cpu().numpy().astype(np.float64),
+                                                            cur["h"]))))
+        far += int(np.sum(((gg >= tau) != cur["mask"]) & (np.abs(cur["g"] - tau) >= pr.BOUNDARY)))
+        Sg = ts["S"].cpu().numpy().astype(np.float64)
+        worst_S = max(worst_S, float(np.max(np.abs(Sg - cur["S"])) / np.max(np.abs(cur["S"]))))
+    print("tensor-core router, teacher-forced: gate", worst_g, "h", worst_h, "S", worst_S)
+    assert far == 0
+    assert worst_g < pr.GATE_TOL
+    assert worst_h < pr.H_TOL["bf16"]
+    assert worst_S < 1e-3
+    st.close()
