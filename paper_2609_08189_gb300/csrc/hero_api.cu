@@ -102,6 +102,43 @@ float bf16_value(float f) {
   return r;
 }
 
+// The router's parameters laid out as RsmBlob<DM> from the packed fp32 copy (already
+// rounded to bf16 values on bf16 models, so the bf16 matrices are exact).
+struct RouterPackAt {
+  size_t hu, p1, pb1, p2, pb2, qkv, n, c, t1, tb1, t2, tb2, psb1, psw2, psb2;
+};
+
+template <int DM>
+std::vector<uint8_t> router_sm_blob(const std::vector<float>& pk, const RouterPackAt& o) {
+  using B = RsmBlob<DM>;
+  std::vector<uint8_t> b(B::bytes, 0);
+  auto put16 = [&](int region, size_t i, float v) {
+    const uint16_t h = bf16_bits(v);
+    std::memcpy(&b[region + 2 * i], &h, 2);
+  };
+  auto put32 = [&](int at, size_t src, int n) {
+    std::memcpy(&b[B::f32 + 4 * (size_t)at], &pk[src], 4 * (size_t)n);
+  };
+  for (size_t i = 0; i < (size_t)kRsmEnc * kRsmDh; ++i) put16(B::hu, i, pk[o.hu + i]);
+  for (int k = 0; k < kRsmDs; ++k) {
+    for (int q = 0; q < 3 * DM; ++q) put16(B::q4, (size_t)k * 4 * DM + q, pk[o.qkv + (size_t)k * 3 * DM + q]);
+    for (int q = 0; q < DM; ++q) put16(B::q4, (size_t)k * 4 * DM + 3 * DM + q, pk[o.n + (size_t)k * DM + q]);
+  }
+  for (size_t i = 0; i < (size_t)DM * DM; ++i) put16(B::wc, i, pk[o.c + i]);
+  for (size_t i = 0; i < (size_t)B::F * kRsmHead; ++i) put16(B::t1, i, pk[o.t1 + i]);
+  put32(B::p1, o.p1, 6 * kRsmPath);
+  put32(B::pb1, o.pb1, kRsmPath);
+  put32(B::p2, o.p2, kRsmPath * kRsmDa);
+  put32(B::pb2, o.pb2, kRsmDa);
+  put32(B::tb1, o.tb1, kRsmHead);
+  put32(B::tw2, o.t2, kRsmHead);
+  put32(B::psb1, o.psb1, kRsmHead);
+  put32(B::psw2, o.psw2, kRsmHead);
+  put32(B::tb2, o.tb2, 1);
+  put32(B::psb2, o.psb2, 1);
+  return b;
+}
+
 std::vector<float> host_f32(const void* p, size_t n, hero_dtype dt) {
   std::vector<float> v(n);
   if (dt == HERO_BF16) {
@@ -149,6 +186,9 @@ struct hero_model {
   float *hbar, *delta, *part, *Y, *S, *zeta, *pst, *mst, *dprev, *gate, *scale_f, *scale_a;
   float* splitk_ws = nullptr;   // bf16: partial slices of split-K GEMMs (few-tile launches)
   // the router on the tensor cores (RouterTcArgs): weights, maps and per-token buffers
+  // the router at small and medium token counts (launch_router_sm): its parameters as one
+  // RsmBlob, or nullptr where that kernel does not serve the model
+  void* rsm_w = nullptr;
   bool rtc = false;
   int rt_kf = 0;
   void* rt_w = nullptr;
@@ -372,7 +412,7 @@ void free_model(hero_model* m) {
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
                   m->dec_pm, m->dec_pos, m->dec_ws, m->wdT, m->wguT, m->w1T, m->w2T, m->bws,
-                  m->rt_w};
+                  m->rt_w, m->rsm_w};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -617,6 +657,15 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     m->rw = RouterWeights{b + o_hu, b + o_p1, b + o_pb1, b + o_p2, b + o_pb2, b + o_qkv, b + o_n,
                           b + o_c,  b + o_t1, b + o_tb1, b + o_t2, b + o_tb2, b + o_pb, b + o_p2w,
                           b + o_p2b};
+    if (bf16 && router_sm_supported(c.d_enc, c.d_head, c.d_h, c.d_a, c.d_path, dm)) {
+      const RouterPackAt at{o_hu, o_p1, o_pb1, o_p2, o_pb2, o_qkv, o_n, o_c,
+                            o_t1, o_tb1, o_t2, o_tb2, o_pb, o_p2w, o_p2b};
+      const std::vector<uint8_t> blob = dm == 16   ? router_sm_blob<16>(pack, at)
+                                        : dm == 32 ? router_sm_blob<32>(pack, at)
+                                                   : router_sm_blob<64>(pack, at);
+      CUDA_M(cudaMalloc(&m->rsm_w, blob.size()));
+      CUDA_M(cudaMemcpy(m->rsm_w, blob.data(), blob.size(), cudaMemcpyHostToDevice));
+    }
     // the router on the tensor cores (large token counts): W_hu, [W_q; W_k; W_v; W_n] and
     // W_th1 as bf16 B operands, each repeated three times along K (one copy per bf16 term
     // of the activation), f_theta's K zero-padded to a multiple of 64
@@ -905,16 +954,26 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.gate_out = gate_out_j;
     ra.mask_out = mask_out_j;
     ra.variant = c.router_variant;
-    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_router(c.d_m, ra, m->num_sms, st); }));
+    ra.wsm = c.router_variant == 0 ? m->rsm_w : nullptr;
+    ra.err = m->err;
+    ra.wait_ns = wait_limit_ns();
+    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
+      return ra.wsm ? launch_router_sm(c.d_m, ra, m->num_sms, st)
+                    : launch_router(c.d_m, ra, m->num_sms, st);
+    }));
     }
   }
   CompactArgs ca{T, m->mask, m->gate, dense ? 1 : 0, m->idx_f, m->idx_a, m->scale_f, m->scale_a,
                  m->counts, count_out_j, dense ? gate_out_j : nullptr,
                  dense ? mask_out_j : nullptr};
-  CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
   NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, hbar, m->part,
               m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
-  CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, m->num_sms, st); }));
+  if (T <= kRouteNormMaxT) {   // few tokens: compaction inside the norm's launch
+    CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_route_norm(ca, na, m->num_sms, st); }));
+  } else {
+    CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
+    CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(na, m->num_sms, st); }));
+  }
 
   // FFN branch: gate/up + SwiGLU, then down + scaled scatter.  The adapter branch
   // (the other token rows): W_1 with SiLU, then W_2 + scaled scatter; on bf16

@@ -295,12 +295,53 @@ struct RouterArgs {
   float* gate_out;       // [T] caller slice or nullptr
   uint8_t* mask_out;     // [T] caller slice or nullptr
   uint32_t variant;      // router ablation bits (RV_*)
+  // the router's parameters as one RsmBlob (bf16 models, variant 0) for launch_router_sm,
+  // else nullptr
+  const void* wsm;
+  uint32_t* err;         // device error word (launch_router_sm's bounded waits)
+  uint64_t wait_ns;
+};
+
+// Router at small and medium token counts with all of its parameters staged in shared
+// memory by one bulk copy per CTA (launch_router_sm): the widths of the Llama router
+// (d_enc = d_head = 256, d_h = 48, d_a = 16, d_path = 16, so d_s = 64) and d_m <= 64,
+// on bf16 models, whose router parameters are bf16 values.  Byte offsets of the blob;
+// matrices are bf16, [in][out] (outputs contiguous); the vectors are fp32.
+constexpr int kRsmEnc = 256, kRsmHead = 256, kRsmDh = 48, kRsmDa = 16, kRsmPath = 16,
+              kRsmDs = 64;
+template <int DM>
+struct RsmBlob {
+  static constexpr int F = kRsmDs + DM + 1;               // f_theta's input [s; c; nu]
+  static constexpr int hu = 0;                            // W_hu        [256][48]
+  static constexpr int q4 = hu + kRsmEnc * kRsmDh * 2;    // q|k|v|W_n   [64][4 DM]
+  static constexpr int wc = q4 + kRsmDs * 4 * DM * 2;     // W_c         [DM][DM]
+  static constexpr int t1 = wc + DM * DM * 2;             // W_th1       [F][256]
+  static constexpr int f32 = (t1 + F * kRsmHead * 2 + 15) / 16 * 16;
+  // fp32 vectors, in floats from f32
+  static constexpr int p1 = 0;                            // path W_1    [6][16]
+  static constexpr int pb1 = p1 + 6 * kRsmPath;           // path b_1    [16]
+  static constexpr int p2 = pb1 + kRsmPath;               // path W_2    [16][16]
+  static constexpr int pb2 = p2 + kRsmPath * kRsmDa;      // path b_2    [16]
+  static constexpr int tb1 = pb2 + kRsmDa;                // f_theta b_1 [256]
+  static constexpr int tw2 = tb1 + kRsmHead;              // f_theta w_2 [256]
+  static constexpr int psb1 = tw2 + kRsmHead;             // f_psi b_1   [256]
+  static constexpr int psw2 = psb1 + kRsmHead;            // f_psi w_2   [256]
+  static constexpr int tb2 = psw2 + kRsmHead;             // f_theta b_2
+  static constexpr int psb2 = tb2 + 1;                    // f_psi b_2
+  static constexpr int nf = (psb2 + 1 + 3) / 4 * 4;
+  static constexpr int bytes = f32 + nf * 4;
+  static_assert(q4 % 16 == 0 && wc % 16 == 0 && t1 % 16 == 0 && bytes % 16 == 0,
+                "16-byte bulk-copy regions");
 };
 
 // Router ablation bits (the values of the ABI's HERO_ROUTER_*).
 enum : uint32_t { RV_NO_HISTORY = 1u, RV_NO_MEMREAD = 2u, RV_NO_AUX = 4u, RV_NO_POS = 8u };
 
 cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st);
+// Whether launch_router_sm serves a router of these widths (RsmBlob).
+bool router_sm_supported(int d_enc, int d_head, int d_h, int d_a, int d_path, int d_m);
+size_t router_sm_blob_bytes(int d_m);
+cudaError_t launch_router_sm(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st);
 // Step 4 of the tensor-core router (see RouterTcArgs).
 cudaError_t launch_rt_mem(const RouterTcArgs& a, cudaStream_t st);
 
@@ -368,6 +409,9 @@ struct NormArgs {
 };
 // wpr: warps per row (each takes a contiguous d / wpr column range; wpr divides d / 4)
 cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st);
+// k_compact and k_norm as one launch (T <= kRouteNormMaxT; same outputs).
+constexpr int kRouteNormMaxT = 2048;
+cudaError_t launch_route_norm(const CompactArgs& c, const NormArgs& a, int num_sms, cudaStream_t st);
 
 // Adapter up-projection plus the block-closing epilogue, for the adapter rows:
 // y[m, :] = W_2 ah[m, :] (rank d_r = 64 contraction), then LayerOutArgs on token
