@@ -867,6 +867,88 @@ __global__ void __launch_bounds__(256) k_norm(const NormArgs a, int wpr) {
 }
 
 // ------------------------------------------------------------------------------
+// k_route_norm: k_compact and k_norm in one launch for token counts up to
+// kRouteNormMaxT.  Warp gw serves token t = gw / wpr (column range gw % wpr); it counts
+// the FFN decisions of the tokens before t with one ballot per 32 tokens (every warp
+// repeats that scan, which at these token counts costs less than a launch), so that
+// token t's branch row is its rank among the tokens of its branch, as in k_compact.
+// The column-range-0 warp of a token writes the token's index and scale entries; the
+// warp of the last token writes the counts.  Outputs equal those of the two kernels.
+// ------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_route_norm(const CompactArgs c, const NormArgs a, int wpr) {
+  pdl_enter();
+  const long gw = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int t = (int)(gw / wpr);
+  const int part = (int)(gw - (long)t * wpr);
+  const int lane = threadIdx.x & 31;
+  if (t >= a.T) return;
+  int pf = t;   // FFN tokens before t
+  bool f = true;
+  if (!c.dense) {
+    pf = 0;
+    for (int b = 0; b < t; b += 128) {
+      int n = 0;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int u = b + 32 * q + lane;
+        n += __popc(__ballot_sync(0xffffffffu, u < t && c.mask[u] != 0));
+      }
+      pf += n;
+    }
+    f = c.mask[t] != 0;
+  }
+  if (part == 0 && lane == 0) {
+    if (f) {
+      c.idx_f[pf] = t;
+      c.scale_f[pf] = c.dense ? 1.f : c.gate[t];
+    } else {
+      c.idx_a[t - pf] = t;
+      c.scale_a[t - pf] = 1.f - c.gate[t];
+    }
+    if (c.dense) {
+      if (c.gate_out) c.gate_out[t] = 1.f;
+      if (c.mask_out) c.mask_out[t] = 1;
+    }
+    if (t == a.T - 1) {
+      const int nf = pf + (f ? 1 : 0);
+      c.counts[0] = nf;
+      c.counts[1] = a.T - nf;
+      if (c.count_out) *c.count_out = nf;
+    }
+  }
+  void* dst = f ? a.u_f : a.u_a;
+  const long r = f ? pf : t - pf;
+  float ss = 0.f;
+  for (int s = lane; s < a.np; s += 32) ss += a.part[((size_t)t * a.np + s) * 4];
+  ss = warp_sum(ss);
+  const float rinv = rsqrtf(ss / (float)a.d + a.rms_eps);
+  const int cols = a.d / wpr;
+  const int c_lo = part * cols, c_hi = c_lo + cols;
+  const float* h = a.hbar + (size_t)t * a.d;
+  const size_t ro = (size_t)r * a.d;
+  constexpr int NB = 8;
+  for (int c0 = c_lo + lane * 4; c0 < c_hi; c0 += 128 * NB) {
+    float4 hv[NB];
+#pragma unroll
+    for (int k = 0; k < NB; ++k) {
+      const int cc = c0 + 128 * k;
+      if (cc < c_hi) hv[k] = *reinterpret_cast<const float4*>(h + cc);
+    }
+#pragma unroll
+    for (int k = 0; k < NB; ++k) {
+      const int cc = c0 + 128 * k;
+      if (cc < c_hi) {
+        const float4 g = __ldg(reinterpret_cast<const float4*>(a.gain + cc));
+        store4(dst, ro + cc,
+               make_float4(hv[k].x * rinv * g.x, hv[k].y * rinv * g.y, hv[k].z * rinv * g.z,
+                           hv[k].w * rinv * g.w),
+               a.out_bf16);
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------
 // k_convert: weight conversion / repacking (load time only).
 // ------------------------------------------------------------------------------
 __global__ void k_convert(const void* src, int src_bf16, void* dst, int dst_bf16, long rows,
@@ -946,15 +1028,28 @@ cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st) {
   return launch_pdl(k_compact, dim3(1), dim3(CT), 0, st, a);
 }
 
-cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st) {
-  if (a.T <= 0) return cudaSuccess;
-  // split rows across warps until there are ~16 warps per SM (column ranges stay
-  // whole multiples of 4 elements)
+// Warps per row of the norm: split rows across warps until there are ~16 warps per SM
+// (column ranges stay whole multiples of 4 elements).
+static int norm_wpr(const NormArgs& a, int num_sms) {
   int wpr = 1;
   while ((long)a.T * wpr * 2 <= 16L * num_sms && (a.d / (wpr * 2)) % 4 == 0 && a.d / (wpr * 2) >= 128)
     wpr *= 2;
+  return wpr;
+}
+
+cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st) {
+  if (a.T <= 0) return cudaSuccess;
+  const int wpr = norm_wpr(a, num_sms);
   const long warps = (long)a.T * wpr;
   return launch_pdl(k_norm, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, a, wpr);
+}
+
+cudaError_t launch_route_norm(const CompactArgs& c, const NormArgs& a, int num_sms, cudaStream_t st) {
+  if (a.T <= 0) return cudaSuccess;
+  if (a.T > kRouteNormMaxT || c.T != a.T) return cudaErrorInvalidValue;
+  const int wpr = norm_wpr(a, num_sms);
+  const long warps = (long)a.T * wpr;
+  return launch_pdl(k_route_norm, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, c, a, wpr);
 }
 
 cudaError_t launch_convert_rows(const void* src, int src_bf16, void* dst, int dst_bf16, long rows,
