@@ -1037,7 +1037,11 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
                    : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU, m->tm_ua,
                                          m->tm_w1[jj], ad, m->num_sms, st);
     }));
-    if (!dense && T <= 256 && r <= 64) {   // few rows: the latency-light FMA-pipe kernel
+    const int m_t = (T + 127) / 128;
+    const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
+    // few rows and a split FFN down: the adapter rows close in FFN down's finishing launch
+    const bool adapter_in_close = !dense && T <= 256 && r <= 64 && r % 8 == 0 && ds > 1;
+    if (!dense && T <= 256 && r <= 64 && !adapter_in_close) {   // few rows: the FMA-pipe kernel
       AdapterUpArgs ua{};
       ua.m_dev = m->counts + 1;
       ua.m_max = T;
@@ -1062,8 +1066,6 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       }));
       return HERO_OK;
     };
-    const int m_t = (T + 127) / 128;
-    const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
     if (ds > 1) {   // few tiles (small T): split K into partials, then the closing epilogue
       GemmArgs sk = dn;
       sk.out_f32 = m->splitk_ws;
@@ -1074,7 +1076,10 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
         return launch_gemm_tc(256, EPI_STORE_F32, m->tm_act, m->tm_wd[jj], sk, m->num_sms, st);
       }));
       CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
-        return launch_splitk_close(m->splitk_ws, ds, sk.split_stride, d, m->counts, T, dn.lo, st);
+        SplitkAdapter sa{};
+        if (adapter_in_close)
+          sa = SplitkAdapter{m->ah, static_cast<const char*>(m->w2) + (size_t)jj * d * r * es, r, au.lo};
+        return launch_splitk_close(m->splitk_ws, ds, sk.split_stride, d, m->counts, T, dn.lo, sa, st);
       }));
       return adapter_after ? adapter_up_wide(0) : HERO_OK;
     }

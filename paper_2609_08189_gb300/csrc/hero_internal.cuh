@@ -439,9 +439,20 @@ cudaError_t launch_qkv_close(const float* part, int splits, long split_stride, i
                              const RopeArgs& r, uint32_t* err, cudaStream_t st);
 cudaError_t launch_entry_close(const float* part, int splits, long split_stride, int B,
                                const float* resid, const LayerOutArgs& lo, cudaStream_t st);
+// Adapter rows closed by the same launch (bf16, few tokens): rows m_dev[0] .. m_max - 1 of
+// the launch are adapter rows m - m_dev[0] (the two branches cover every token): y = W_2
+// ah[row] (depth d_r, a multiple of 8, accumulated in k order as k_adapter_up does), then
+// the block-closing epilogue `lo` on token lo.idx[row] with scale lo.scale[row].  ah ==
+// nullptr: no adapter rows.
+struct SplitkAdapter {
+  const void* ah;       // bf16 [rows, d_r] SiLU(W_1 u)
+  const void* w2;       // bf16 [d, d_r]
+  int d_r;
+  LayerOutArgs lo;
+};
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
-                                cudaStream_t st);
+                                const SplitkAdapter& ad, cudaStream_t st);
 
 // Training path: backward of a routed block's branch part (backward.cu) -------------
 // Compacted rows: FFN rows 0 .. n_f - 1 (idx_f), then adapter rows (idx_a), counts [2].

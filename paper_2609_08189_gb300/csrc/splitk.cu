@@ -13,7 +13,8 @@ namespace {
 // sums are reduced over the warp in a fixed order.
 __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ part, int splits,
                                                       long split_stride, int ld, const int* m_dev,
-                                                      int m_max, const LayerOutArgs lo) {
+                                                      int m_max, const LayerOutArgs lo,
+                                                      const SplitkAdapter ad) {
   pdl_enter();
   static_assert(kTcPartCols == 128, "one warp covers one 128-column slot with float4 lanes");
   int M = *m_dev;
@@ -21,27 +22,54 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
   const int slots = lo.d / kTcPartCols;
   const long w = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
-  if (w >= (long)M * slots) return;
+  const long rows = ad.ah ? m_max : M;
+  if (w >= rows * slots) return;
   const int m = (int)(w / slots);
   const int slot = (int)(w - (long)m * slots);
   const int n = slot * kTcPartCols + 4 * lane;
-  const size_t off = (size_t)m * ld + n;
-  float4 y = *reinterpret_cast<const float4*>(part + off);
-  for (int s = 1; s < splits; ++s) {
-    const float4 v = *reinterpret_cast<const float4*>(part + (size_t)s * split_stride + off);
-    y.x += v.x; y.y += v.y; y.z += v.z; y.w += v.w;
+  const bool ffn = m < M;
+  const LayerOutArgs& p = ffn ? lo : ad.lo;
+  const int row = ffn ? m : m - M;
+  float4 y;
+  if (ffn) {
+    const size_t off = (size_t)m * ld + n;
+    y = *reinterpret_cast<const float4*>(part + off);
+    for (int s = 1; s < splits; ++s) {
+      const float4 v = *reinterpret_cast<const float4*>(part + (size_t)s * split_stride + off);
+      y.x += v.x; y.y += v.y; y.z += v.z; y.w += v.w;
+    }
+  } else {   // adapter row: y = W_2 ah[row] over the lane's 4 columns
+    const uint16_t* ar = static_cast<const uint16_t*>(ad.ah) + (size_t)row * ad.d_r;
+    const uint16_t* wr = static_cast<const uint16_t*>(ad.w2) + (size_t)n * ad.d_r;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int k = 0; k < ad.d_r; k += 8) {
+      const uint4 xa = __ldg(reinterpret_cast<const uint4*>(ar + k));
+      const uint32_t xs[4] = {xa.x, xa.y, xa.z, xa.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(wr + (size_t)i * ad.d_r + k));
+        const uint32_t ws[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          acc[i] = fmaf(__uint_as_float(xs[e] << 16), __uint_as_float(ws[e] << 16), acc[i]);
+          acc[i] = fmaf(__uint_as_float(xs[e] & 0xffff0000u), __uint_as_float(ws[e] & 0xffff0000u),
+                        acc[i]);
+        }
+      }
+    }
+    y = make_float4(acc[0], acc[1], acc[2], acc[3]);
   }
-  const int t = lo.idx[m];
-  const float sc = lo.scale[m];
-  const LayerOutIn in = layer_out_load(lo, t, n);
+  const int t = p.idx[row];
+  const float sc = p.scale[row];
+  const LayerOutIn in = layer_out_load(p, t, n);
   float ss = 0.f, dd = 0.f, dp = 0.f;
-  layer_out_store(lo, t, n, in, y, sc, ss, dd, dp);
-  if (!lo.last) {
+  layer_out_store(p, t, n, in, y, sc, ss, dd, dp);
+  if (!p.last) {
     ss = warp_sum(ss);
     dd = warp_sum(dd);
     dp = warp_sum(dp);
     if (lane == 0)
-      *reinterpret_cast<float4*>(lo.part + ((size_t)t * lo.np + slot) * 4) =
+      *reinterpret_cast<float4*>(p.part + ((size_t)t * p.np + slot) * 4) =
           make_float4(ss, dd, dp, 0.f);
   }
 }
@@ -157,12 +185,13 @@ cudaError_t launch_entry_close(const float* part, int splits, long split_stride,
 
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,
-                                cudaStream_t st) {
+                                const SplitkAdapter& ad, cudaStream_t st) {
   if (m_max <= 0) return cudaSuccess;
   if (lo.d % kTcPartCols) return cudaErrorInvalidValue;
+  if (ad.ah && (ad.d_r <= 0 || ad.d_r % 8 || !ad.w2 || ad.lo.d != lo.d)) return cudaErrorInvalidValue;
   const long warps = (long)m_max * (lo.d / kTcPartCols);
   return launch_pdl(k_splitk_close, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, part, splits,
-                    split_stride, ld, m_dev, m_max, lo);
+                    split_stride, ld, m_dev, m_max, lo, ad);
 }
 
 }  // namespace hero
