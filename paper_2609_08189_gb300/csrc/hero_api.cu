@@ -71,6 +71,21 @@ bool encode_bf16_2d(CUtensorMap* tm, const void* ptr, uint64_t inner, uint64_t o
   return r == CUDA_SUCCESS;
 }
 
+// The same with rows ld elements apart (ld >= inner): a view of the first `inner` columns.
+bool encode_bf16_2d_ld(CUtensorMap* tm, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld,
+                       uint32_t box_outer) {
+  if (!get_encoder()) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 // 3-D bf16 map with 64 x 128 x 1 boxes (128-byte swizzle; out-of-range elements read 0):
 // dims d0 (contiguous) x d1 x d2, byte strides s1 (between d1 rows) and s2.
 bool encode_bf16_3d(CUtensorMap* tm, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d2,
@@ -212,6 +227,9 @@ struct hero_model {
 
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
+  // the router operand pair stacked along M: xl viewed as [2T][d] (rows 2t = hi, 2t + 1 = lo
+  // of token t) against the first copy of the router weight, wr viewed as [nY][d]
+  CUtensorMap tm_xl2, tm_wr1;
   std::vector<CUtensorMap> tm_wgu, tm_wd, tm_w1, tm_w2;
   // the same weights with 128-row boxes: the B operands of the CTA-pair GEMM
   CUtensorMap tm_wr_p;
@@ -371,6 +389,12 @@ size_t splitk_ws_floats(int T, int num_sms, int nY, int K_router, int d, int I) 
     const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, num_sms, rows, d, 22);
     if (rs > 1) most = std::max(most, (size_t)rs * rows * nY);
     if (ds > 1) most = std::max(most, (size_t)ds * rows * d);
+  }
+  // the router contraction with the operand pair stacked along M (2T rows, K = K_router / 2)
+  for (int m2 = 1; m2 <= (2 * T + 127) / 128; ++m2) {
+    const long rows = (long)m2 * 128;
+    const int rs2 = choose_splits(m2 * ((nY + 255) / 256), (K_router / 2 + 63) / 64, num_sms, rows, nY, 4);
+    if (rs2 > 1) most = std::max(most, (size_t)rs2 * rows * nY);
   }
   return most;
 }
@@ -715,7 +739,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     };
     std::vector<Item> items = {
         {(void**)&m->hbar, Tm * d * 4},        {(void**)&m->delta, Tm * d * 4},
-        {(void**)&m->part, Tm * m->np * 16},   {(void**)&m->Y, Tm * nY * 4},
+        {(void**)&m->part, Tm * m->np * 16},   {(void**)&m->Y, Tm * nY * 4 * (bf16 ? 2 : 1)},
         {(void**)&m->S, Tm * dm * dm * 4},     {(void**)&m->zeta, Tm * dm * 4},
         {(void**)&m->pst, Tm * 4},             {(void**)&m->mst, Tm * 4},
         {(void**)&m->dprev, Tm * 4},           {(void**)&m->gate, Tm * 4},
@@ -756,6 +780,8 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
               encode_bf16_2d(&m->tm_ah, m->ah, r, Tm, 128) &&
               encode_bf16_2d(&m->tm_wr, m->wr, 2 * d, nY, 256);
     ok = ok && encode_bf16_2d(&m->tm_wr_p, m->wr, 2 * d, nY, 128);
+    ok = ok && encode_bf16_2d_ld(&m->tm_xl2, m->xl, d, 2 * Tm, d, 128) &&
+         encode_bf16_2d_ld(&m->tm_wr1, m->wr, d, nY, 2 * d, 256);
     if (m->rtc)
       ok = ok && encode_bf16_2d(&m->tm_enc3, m->rt_enc3, 768, Tm, 128) &&
            encode_bf16_2d(&m->tm_s3, m->rt_s3, 3 * ds, Tm, 128) &&
@@ -916,7 +942,29 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
         return launch_gemm_tc2(EPI_RT_HEAD, m->tm_fin3, m->tm_th3, g5, m->num_sms, st);
       }));
     } else {
+    // bf16, variant 0: the shared-memory router, with the operand pair stacked along M
+    // (K = d, each router weight element read once per launch); the router adds token t's
+    // rows 2t and 2t + 1 of every slice
+    const bool stacked = m->bf16 && m->rsm_w && c.router_variant == 0;
+    int rs2 = 1;
+    if (stacked) {
+      const int m2 = (2 * T + 127) / 128;
+      rs2 = choose_splits(m2 * ((nY + 255) / 256), (d + 63) / 64, m->num_sms, (long)m2 * 128, nY, 4);
+      g.m_static = 2 * T;
+      g.m_max = 2 * T;
+      g.K = d;
+      g.k_splits = 0;
+      g.split_stride = 0;
+      g.out_f32 = m->Y;
+      g.ldo = nY;
+      if (rs2 > 1) {
+        g.out_f32 = m->splitk_ws;
+        g.k_splits = rs2;
+        g.split_stride = (long)m2 * 128 * nY;
+      }
+    }
     CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
+      if (stacked) return launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl2, m->tm_wr1, g, m->num_sms, st);
       if (!m->bf16) return launch_gemm_simt(EPI_STORE_F32, g, st);
       return pair ? launch_gemm_tc2(EPI_STORE_F32, m->tm_xl, m->tm_wr_p, g, m->num_sms, st)
                   : launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st);
@@ -933,9 +981,10 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.d_enc = c.d_enc;
     ra.d_head = c.d_head;
     ra.d_path = c.d_path;
-    ra.Y = rs > 1 ? m->splitk_ws : m->Y;   // the router adds split-K slices as it reads
-    ra.y_splits = rs > 1 ? rs : 1;
-    ra.y_split_stride = rs > 1 ? g.split_stride : 0;
+    ra.Y = g.k_splits > 1 ? m->splitk_ws : m->Y;   // the router adds split-K slices as it reads
+    ra.y_splits = g.k_splits > 1 ? g.k_splits : 1;
+    ra.y_split_stride = g.k_splits > 1 ? g.split_stride : 0;
+    ra.y_rows = stacked ? 2 : 1;
     ra.part = m->part;
     ra.dprev = bs.dprev;
     ra.pst = bs.pst;

@@ -280,6 +280,8 @@ struct RouterArgs {
                          // slice order as they are read)
   int y_splits;
   long y_split_stride;
+  int y_rows;            // rows of Y per token: 2 when the operand pair is stacked along M
+                         // (rows 2t and 2t + 1 of token t, added; launch_router_sm only)
   const float* part;     // [T, np, 4]
   float* dprev;          // [T] in: d_{j-1}; out: d_j
   float* pst;            // [T] p_hist

@@ -218,29 +218,46 @@ __global__ void __launch_bounds__(kThr, 1) k_router_sm(const RouterArgs a) {
       xf[5 * TB + tl] = mp;
     }
   }
-  wait_part(0);
   __syncthreads();
-  if (aborted()) return;
 
   // 2. thread tid takes columns 2 tid, 2 tid + 1 of the contraction's 512 (split-K slices
   //    added in slice order): encoder input SiLU(rinv y) below 256, f_psi's hidden
-  //    SiLU(y + b_1) dotted with w_2 above (Eq. 16)
+  //    SiLU(y + b_1) dotted with w_2 above (Eq. 16).  The loads are issued before the wait
+  //    on the blob's first part (f_psi's vectors).
   {
     const int c0 = 2 * tid;
     float2 y[TB];
 #pragma unroll
     for (int tl = 0; tl < TB; ++tl) y[tl] = make_float2(0.f, 0.f);
     const long sstride = a.y_split_stride / 2;
-    for (int sp = 0; sp < a.y_splits; ++sp) {
+    const int yr = a.y_rows > 1 ? 2 : 1;   // rows per token (the stacked operand pair)
+    const int parts = a.y_splits * yr;     // part p: slice p / yr, row p % yr of the token
+    // SB parts x TB tokens of loads in flight before they are added (in part order)
+    constexpr int SB = TB >= 8 ? 1 : 8 / TB;
+    for (int p0 = 0; p0 < parts; p0 += SB) {
+      float2 v[SB][TB];
 #pragma unroll
-      for (int tl = 0; tl < TB; ++tl)
-        if (tl < nvalid) {
-          const float2 v = __ldg(reinterpret_cast<const float2*>(a.Y + (size_t)(t0 + tl) * 512) +
-                                 sp * sstride + tid);
-          y[tl].x += v.x;
-          y[tl].y += v.y;
+      for (int i = 0; i < SB; ++i)
+#pragma unroll
+        for (int tl = 0; tl < TB; ++tl) {
+          const int p = p0 + i;
+          v[i][tl] = p < parts && tl < nvalid
+                         ? __ldg(reinterpret_cast<const float2*>(
+                                     a.Y + ((size_t)(t0 + tl) * yr + p % yr) * 512) +
+                                 (p / yr) * sstride + tid)
+                         : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+      for (int i = 0; i < SB; ++i)
+#pragma unroll
+        for (int tl = 0; tl < TB; ++tl) {
+          y[tl].x += v[i][tl].x;
+          y[tl].y += v[i][tl].y;
         }
     }
+    wait_part(0);
+    __syncthreads();
+    if (aborted()) return;
     if (c0 < kRsmEnc) {
 #pragma unroll
       for (int tl = 0; tl < TB; ++tl) {

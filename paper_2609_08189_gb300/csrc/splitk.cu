@@ -34,14 +34,25 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
   if (ffn) {
     const size_t off = (size_t)m * ld + n;
     y = *reinterpret_cast<const float4*>(part + off);
-    for (int s = 1; s < splits; ++s) {
-      const float4 v = *reinterpret_cast<const float4*>(part + (size_t)s * split_stride + off);
-      y.x += v.x; y.y += v.y; y.z += v.z; y.w += v.w;
+    // up to 8 slices' loads in flight, added in slice order
+    for (int s0 = 1; s0 < splits; s0 += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        v[i] = s0 + i < splits
+                   ? *reinterpret_cast<const float4*>(part + (size_t)(s0 + i) * split_stride + off)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        if (s0 + i < splits) {
+          y.x += v[i].x; y.y += v[i].y; y.z += v[i].z; y.w += v[i].w;
+        }
     }
   } else {   // adapter row: y = W_2 ah[row] over the lane's 4 columns
     const uint16_t* ar = static_cast<const uint16_t*>(ad.ah) + (size_t)row * ad.d_r;
     const uint16_t* wr = static_cast<const uint16_t*>(ad.w2) + (size_t)n * ad.d_r;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
     for (int k = 0; k < ad.d_r; k += 8) {
       const uint4 xa = __ldg(reinterpret_cast<const uint4*>(ar + k));
       const uint32_t xs[4] = {xa.x, xa.y, xa.z, xa.w};
