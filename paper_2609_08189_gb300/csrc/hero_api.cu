@@ -210,6 +210,9 @@ struct hero_model {
   CUtensorMap tm_whu3, tm_wq3, tm_th3, tm_enc3, tm_s3, tm_fin3;
   uint16_t *rt_enc3 = nullptr, *rt_s3 = nullptr, *rt_fin3 = nullptr;
   float *rt_scal = nullptr, *rt_s = nullptr, *rt_qkvn = nullptr;
+  // the history form of the memory (d_m = 64 or 128 on the tensor-core router): per token
+  // [L_R][2 d_m] entries phi(k_i) | v_i, and the decay weights [L_R][L_R] (RouterTcArgs)
+  float *hist = nullptr, *hw = nullptr;
   void *xl, *u_f, *u_a, *act, *ah;
   uint8_t* mask;
   int *idx_f, *idx_a, *counts;
@@ -379,6 +382,12 @@ int choose_splits(int tiles, int kblocks, int num_sms, long rows, long n, int ep
 
 // Token counts from which the large GEMMs of a block run on CTA pairs (256-row tiles).
 constexpr int kPairMinRows = 1024;
+
+// Forward passes over every routed block run the tensor-core router's memory step in its
+// history form (k_rt_hist); building with -DHERO_HISTORY_FORM=0 keeps the state form there.
+#ifndef HERO_HISTORY_FORM
+#define HERO_HISTORY_FORM 1
+#endif
 
 // Largest split-K partial buffer (floats) any token count up to T may ask for.
 size_t splitk_ws_floats(int T, int num_sms, int nY, int K_router, int d, int I) {
@@ -732,6 +741,8 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
   // ---- workspace ----
   {
     const size_t Tm = (size_t)c.max_tokens;
+    const long LR = c.n_layers - c.n_dense;   // routed blocks
+    const bool hist_form = HERO_HISTORY_FORM && m->rtc && (dm == 64 || dm == 128) && LR > 0;
     size_t off = 0;
     struct Item {
       void** p;
@@ -755,6 +766,8 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         {(void**)&m->rt_s3, m->rtc ? Tm * 3 * ds * 2 : 0},
         {(void**)&m->rt_qkvn, m->rtc ? Tm * 4 * dm * 4 : 0},
         {(void**)&m->rt_fin3, m->rtc ? Tm * (size_t)m->rt_kf * 2 : 0},
+        {(void**)&m->hist, hist_form ? Tm * (size_t)LR * 2 * dm * 4 : 0},
+        {(void**)&m->hw, hist_form ? (size_t)LR * LR * 4 : 0},
         // split-K partials of the few-wave launches (router contraction, FFN down)
         {(void**)&m->splitk_ws, bf16 ? splitk_ws_floats(c.max_tokens, m->num_sms, (int)nY,
                                                         (int)(2 * d), (int)d, (int)I) * 4 : 0},
@@ -767,6 +780,19 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     for (auto& it : items) {
       *it.p = static_cast<char*>(m->ws) + off;
       off += (it.bytes + 1023) & ~(size_t)1023;
+    }
+    if (hist_form) {   // hw[jb L_R + i] = rho_{i+1} ... rho_{jb-1} (0-based routed blocks)
+      std::vector<float> hw((size_t)LR * LR, 0.f);
+      for (long jb = 0; jb < LR; ++jb) {
+        double wgt = 1.0;
+        for (long i = jb - 1; i >= 0; --i) {
+          hw[(size_t)jb * LR + i] = (float)wgt;
+          wgt *= (double)m->rho[c.n_dense + i];
+        }
+      }
+      CUDA_M(cudaMemcpy(m->hw, hw.data(), hw.size() * 4, cudaMemcpyHostToDevice));
+    } else {
+      m->hist = m->hw = nullptr;
     }
   }
 
@@ -831,8 +857,11 @@ hero_status ensure_io(hero_model* m, size_t bytes) {
 
 // Router state of one forward pass (workspace for the fused stack, the caller's
 // for hero_routed_block).
+// hist: the history form of the memory (k_rt_hist) for a forward pass over every routed
+// block from a fresh state, or nullptr (the state S, zeta).
 struct BlockState {
   float *S, *zeta, *pst, *mst, *dprev;
+  float* hist;
 };
 
 
@@ -897,6 +926,9 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       rt.mst = bs.mst;
       rt.S = bs.S;
       rt.zeta = bs.zeta;
+      rt.hist = bs.hist;
+      rt.hist_ld = (long)rt.L * 2 * c.d_m;
+      rt.hw = m->hw;
       rt.w = m->rw;
       rt.enc3 = m->rt_enc3;
       rt.scal = m->rt_scal;
@@ -936,7 +968,9 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
         return launch_gemm_tc2(EPI_STORE_F32, m->tm_s3, m->tm_wq3, g3, m->num_sms, st);
       }));
-      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] { return launch_rt_mem(rt, st); }));   // 4.
+      CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {   // 4.
+        return rt.hist ? launch_rt_hist(rt, st) : launch_rt_mem(rt, st);
+      }));
       GemmArgs g5 = small(c.d_head, m->rt_kf);   // 5. f_theta, p_hist, m_hist, g, decision
       CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
         return launch_gemm_tc2(EPI_RT_HEAD, m->tm_fin3, m->tm_th3, g5, m->num_sms, st);
@@ -1231,7 +1265,7 @@ hero_status run_stack(hero_model* m, int T, const float* h_in, const void* P, fl
       }
     }
     if (feed && jj + 1 < L) CUDA_TRY(cudaStreamWaitEvent(st, m->ev_ready[jj + 1], 0));
-    BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
+    BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev, m->hist};
     // layers before the routing candidate set run the plain FFN block
     const int jr = jj - c.n_dense;
     const bool dense_blk = dense || jr < 0;
@@ -1406,7 +1440,7 @@ hero_status routed_block_run(hero_model* m, int jj, int T, const float* h_bar, c
   lo.p_bf16 = m->bf16;
   lo.xl_bf16 = m->bf16;
   lo.router = 0;
-  return block_body(m, jj, jr, T, dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr} : bs,
+  return block_body(m, jj, jr, T, dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr} : bs,
                     h_bar, lo, tau, flags, (flags & HERO_FLAG_FORCE_MASK) ? mask_in : nullptr,
                     gate_out, mask_out, count_out, st);
 }
@@ -1533,8 +1567,8 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
                  !s->h_bar_prev || !s->delta_prev))
     return fail(HERO_ERR_ARG, "the router state needs all seven pointers");
   CUDA_TRY(cudaSetDevice(m->device));
-  const BlockState bs = dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr}
-                              : BlockState{s->S, s->zeta, s->p_hist, s->m_hist, s->d_prev};
+  const BlockState bs = dense ? BlockState{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr}
+                              : BlockState{s->S, s->zeta, s->p_hist, s->m_hist, s->d_prev, nullptr};
   const hero_status sb =
       routed_block_run(m, block - 1, (int)n_tokens, h_bar, bs, dense ? nullptr : s->h_bar_prev,
                        dense ? nullptr : s->delta_prev, tau_exec, flags, mask_in, h_out, gate_out,
@@ -1762,7 +1796,7 @@ hero_status decoder_run(hero_model* m, int n_seqs, int seq_len, const float* h_i
   const int L = c.n_layers, T = n_seqs * seq_len;
   if (!(flags & HERO_FLAG_DENSE))
     CUDA_TRY(launch_state_reset(m->S, m->zeta, m->pst, m->mst, m->dprev, T, c.d_m, st));
-  const BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev};
+  const BlockState bs{m->S, m->zeta, m->pst, m->mst, m->dprev, m->hist};
   const float* h = h_in;
   for (int jj = 0; jj < L; ++jj) {
     // Eq. 1 with the block entry fused into the output projection: m->hbar carries

@@ -164,6 +164,12 @@ struct RouterTcArgs {
   float* mst;            // [T] m_hist
   float* S;              // [T, dm, dm]
   float* zeta;           // [T, dm]
+  // history form of the memory (k_rt_hist): per token, L entries of phi(k_i) | v_i
+  // (hist_ld floats per token), and the decay weights hw[(j - 1) L + i] = rho_{i+1} ... rho_{j-1}
+  // of entry i seen from routed block j (1-based blocks, 0-based entries)
+  float* hist;
+  long hist_ld;
+  const float* hw;
   RouterWeights w;
   uint16_t* enc3;        // [T, 768] bf16: the encoder hidden's three terms
   float* scal;           // [T, 4]: d_j, gamma, f_psi's second layer without bias
@@ -344,8 +350,10 @@ cudaError_t launch_router(int d_m, const RouterArgs& a, int num_sms, cudaStream_
 bool router_sm_supported(int d_enc, int d_head, int d_h, int d_a, int d_path, int d_m);
 size_t router_sm_blob_bytes(int d_m);
 cudaError_t launch_router_sm(int d_m, const RouterArgs& a, int num_sms, cudaStream_t st);
-// Step 4 of the tensor-core router (see RouterTcArgs).
+// Step 4 of the tensor-core router (see RouterTcArgs): with the state S, zeta, or in the
+// history form (hist, hw; d_m = 64 or 128).
 cudaError_t launch_rt_mem(const RouterTcArgs& a, cudaStream_t st);
+cudaError_t launch_rt_hist(const RouterTcArgs& a, cudaStream_t st);
 
 struct InitArgs {
   int T, d, np, d_m;

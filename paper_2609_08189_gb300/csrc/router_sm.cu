@@ -233,7 +233,7 @@ __global__ void __launch_bounds__(kThr, 1) k_router_sm(const RouterArgs a) {
     const int yr = a.y_rows > 1 ? 2 : 1;   // rows per token (the stacked operand pair)
     const int parts = a.y_splits * yr;     // part p: slice p / yr, row p % yr of the token
     // SB parts x TB tokens of loads in flight before they are added (in part order)
-    constexpr int SB = TB >= 8 ? 1 : 8 / TB;
+    constexpr int SB = TB >= 8 ? 1 : 16 / TB;
     for (int p0 = 0; p0 < parts; p0 += SB) {
       float2 v[SB][TB];
 #pragma unroll

@@ -5,7 +5,8 @@
 //   nu = 1 - cos(W_n s, W_c c) for j > 1, else 0          Eq. 13
 //   f_theta's input [s; c; nu] as three bf16 terms per value (zero padded to kf columns)
 // S is read once and written once; its lanes and the order in which c's partial sums are
-// added follow the fused router's memory step.
+// added follow the fused router's memory step.  k_rt_hist is the same step in its history
+// form (see there), for a forward pass over all routed blocks.
 #include "hero_device.cuh"
 
 namespace hero {
@@ -18,6 +19,49 @@ __device__ __forceinline__ uint16_t bf16_term(float x, int term) {
     h = __float2bfloat16_rn(x);
   }
   return *reinterpret_cast<const uint16_t*>(&h);
+}
+
+// W_c c and nu = 1 - cos(W_n s, W_c c) (Eq. 13), then f_theta's input [s; c; nu] as three
+// bf16 terms (term p of element e at column p F + e, zero padded to kf): the part of the
+// memory step after c, shared by the two memory kernels.  cb holds c, cvb receives W_c c.
+template <int DM>
+__device__ __forceinline__ void rt_tail(const RouterTcArgs& a, int t, int lane, float* cb, float* cvb,
+                                        const float* wn) {
+  __syncwarp();
+  // W_c c (Eq. 13), w_c_t is [in][out]
+  for (int o = lane; o < DM; o += 32) {
+    float acc = 0.f;
+    for (int i = 0; i < DM; ++i) acc = fmaf(__ldg(a.w.w_c_t + i * DM + o), cb[i], acc);
+    cvb[o] = acc;
+  }
+  __syncwarp();
+  float nu = 0.f;
+  if (a.j > 1) {
+    float xy = 0.f, xx = 0.f, yy = 0.f;
+    for (int o = lane; o < DM; o += 32) {
+      const float x = wn[o], y = cvb[o];
+      xy += x * y;
+      xx += x * x;
+      yy += y * y;
+    }
+    xy = warp_sum(xy);
+    xx = warp_sum(xx);
+    yy = warp_sum(yy);
+    nu = 1.f - xy / (sqrtf(xx) * sqrtf(yy) + a.eps);
+  }
+  // f_theta's input [s; c; nu]: term p of element e at column p * F + e
+  const int ds = a.d_h + a.d_a, F = ds + DM + 1;
+  const float* s = a.s + (size_t)t * ds;
+  uint16_t* fin = a.fin3 + (size_t)t * a.kf;
+  for (int col = lane; col < a.kf; col += 32) {
+    const int p = col / F, e = col - p * F;
+    uint16_t bits = 0;
+    if (p < 3) {
+      const float x = e < ds ? s[e] : (e < ds + DM ? cb[e - ds] : nu);
+      bits = bf16_term(x, p);
+    }
+    fin[col] = bits;
+  }
 }
 
 template <int DM>
@@ -77,41 +121,79 @@ __global__ void __launch_bounds__(256) k_rt_mem(const RouterTcArgs a) {
   }
   if (r0 == 0)
     *reinterpret_cast<float4*>(&cbuf[w][4 * cq]) = make_float4(c.x * inv, c.y * inv, c.z * inv, c.w * inv);
-  __syncwarp();
-  // W_c c (Eq. 13), w_c_t is [in][out]
-  for (int o = lane; o < DM; o += 32) {
-    float acc = 0.f;
-    for (int i = 0; i < DM; ++i) acc = fmaf(__ldg(a.w.w_c_t + i * DM + o), cbuf[w][i], acc);
-    cvbuf[w][o] = acc;
+  rt_tail<DM>(a, t, lane, cbuf[w], cvbuf[w], wn);
+}
+
+// The memory step in its history form, for a forward pass that runs every routed block in
+// order from S_0 = 0, zeta_0 = 0 (the fused stack and the decoder forward).  Unrolling Eq. 12,
+//   S_{j-1} = sum_{i<j} w_ji phi(k_i) v_i^T,  zeta_{j-1} = sum_{i<j} w_ji phi(k_i),
+//   w_ji = rho_{i+1} ... rho_{j-1}  (1 for i = j - 1),
+// so Eq. 11's read is c = sum_i w_ji s_i v_i / (sum_i w_ji s_i + eps) with s_i = phi(q).phi(k_i):
+// the same quantity in exact arithmetic, computed from the token's earlier (phi(k_i), v_i)
+// (2 d_m floats per routed block) instead of its d_m x d_m state.  Block j appends its own
+// pair.  One warp per token; lane owns elements EL lane .. EL lane + EL - 1 of each vector;
+// history entries are taken in order (bitwise reproducible).
+template <int DM>
+__global__ void __launch_bounds__(256) k_rt_hist(const RouterTcArgs a) {
+  pdl_enter();
+  static_assert(DM % 64 == 0 && DM <= 128, "two or four elements per lane");
+  constexpr int EL = DM / 32;
+  __shared__ float cbuf[8][DM];
+  __shared__ float cvbuf[8][DM];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * 8 + w;
+  if (t >= a.T) return;   // whole warps only; nothing below synchronises the CTA
+  const float* q = a.qkvn + (size_t)t * 4 * DM;
+  const float* k = q + DM;
+  const float* v = q + 2 * DM;
+  const float* wn = q + 3 * DM;   // W_n s
+  float fq[EL], fk[EL], vv[EL];
+#pragma unroll
+  for (int e = 0; e < EL; ++e) {
+    const int m = lane * EL + e;
+    fq[e] = phif_(q[m]);
+    fk[e] = phif_(k[m]);
+    vv[e] = v[m];
   }
-  __syncwarp();
-  float nu = 0.f;
-  if (a.j > 1) {
-    float xy = 0.f, xx = 0.f, yy = 0.f;
-    for (int o = lane; o < DM; o += 32) {
-      const float x = wn[o], y = cvbuf[w][o];
-      xy += x * y;
-      xx += x * x;
-      yy += y * y;
+  float* H = a.hist + (size_t)t * a.hist_ld;   // entry i: phi(k_i) [DM] | v_i [DM]
+  const float* wj = a.hw + (size_t)(a.j - 1) * a.L;
+  const int nh = a.j - 1;
+  float c[EL], den = 0.f;
+#pragma unroll
+  for (int e = 0; e < EL; ++e) c[e] = 0.f;
+  constexpr int HB = 8;   // entries per batch of loads
+#pragma unroll 1
+  for (int i0 = 0; i0 < nh; i0 += HB) {
+    float hk[HB][EL], hv[HB][EL];
+#pragma unroll
+    for (int u = 0; u < HB; ++u)
+#pragma unroll
+      for (int e = 0; e < EL; ++e) {
+        const bool in = i0 + u < nh;
+        hk[u][e] = in ? H[(size_t)(i0 + u) * 2 * DM + lane * EL + e] : 0.f;
+        hv[u][e] = in ? H[(size_t)(i0 + u) * 2 * DM + DM + lane * EL + e] : 0.f;
+      }
+#pragma unroll
+    for (int u = 0; u < HB; ++u) {
+      if (i0 + u >= nh) break;   // warp-uniform
+      float sp = 0.f;
+#pragma unroll
+      for (int e = 0; e < EL; ++e) sp = fmaf(fq[e], hk[u][e], sp);
+      const float ws = __ldg(wj + i0 + u) * warp_sum(sp);
+      den += ws;
+#pragma unroll
+      for (int e = 0; e < EL; ++e) c[e] = fmaf(ws, hv[u][e], c[e]);
     }
-    xy = warp_sum(xy);
-    xx = warp_sum(xx);
-    yy = warp_sum(yy);
-    nu = 1.f - xy / (sqrtf(xx) * sqrtf(yy) + a.eps);
   }
-  // f_theta's input [s; c; nu]: term p of element e at column p * F + e
-  const int ds = a.d_h + a.d_a, F = ds + DM + 1;
-  const float* s = a.s + (size_t)t * ds;
-  uint16_t* fin = a.fin3 + (size_t)t * a.kf;
-  for (int col = lane; col < a.kf; col += 32) {
-    const int p = col / F, e = col - p * F;
-    uint16_t bits = 0;
-    if (p < 3) {
-      const float x = e < ds ? s[e] : (e < ds + DM ? cbuf[w][e - ds] : nu);
-      bits = bf16_term(x, p);
-    }
-    fin[col] = bits;
+  const float inv = 1.0f / (den + a.eps);
+  float* Hj = H + (size_t)nh * 2 * DM;   // this block's entry
+#pragma unroll
+  for (int e = 0; e < EL; ++e) {
+    cbuf[w][lane * EL + e] = c[e] * inv;
+    Hj[lane * EL + e] = fk[e];
+    Hj[DM + lane * EL + e] = vv[e];
   }
+  rt_tail<DM>(a, t, lane, cbuf[w], cvbuf[w], wn);
 }
 
 }  // namespace
@@ -124,6 +206,18 @@ cudaError_t launch_rt_mem(const RouterTcArgs& a, cudaStream_t st) {
     case 32: return launch_pdl(k_rt_mem<32>, grid, dim3(256), 0, st, a);
     case 64: return launch_pdl(k_rt_mem<64>, grid, dim3(256), 0, st, a);
     case 128: return launch_pdl(k_rt_mem<128>, grid, dim3(256), 0, st, a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_rt_hist(const RouterTcArgs& a, cudaStream_t st) {
+  if (a.T <= 0) return cudaSuccess;
+  if (!a.hist || !a.hw || a.j < 1 || a.j > a.L || a.hist_ld < (long)a.L * 2 * a.dm)
+    return cudaErrorInvalidValue;
+  const dim3 grid((a.T + 7) / 8);
+  switch (a.dm) {
+    case 64: return launch_pdl(k_rt_hist<64>, grid, dim3(256), 0, st, a);
+    case 128: return launch_pdl(k_rt_hist<128>, grid, dim3(256), 0, st, a);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -132,6 +132,26 @@ def test_ragged_token_counts(hero, T):
     st.close()
 
 
+@pytest.mark.parametrize("T", [200, 700, 1100, 2049, 4096])
+def test_router_paths_by_token_count(hero, T):
+    """The router's kernel follows the token count (bf16, the small_bf16 widths, whose router
+    has the Llama widths); every token against the oracle, free-running:
+      200   the router with its parameters in shared memory, 2 tokens per CTA
+      700   the same, 8 tokens per CTA
+      1100  8 tokens per CTA, compaction inside the norm's launch
+      2049  16 tokens per CTA, the separate compaction (past 2048 tokens)
+      4096  the router contraction no longer splits K: the router on the tensor cores, its
+            memory step in the history form (small_bf16 has d = 512)."""
+    inp = pr.inputs("small_bf16", cfg=hi.CONFIGS["small_bf16"].replace(n_tokens=T))
+    st = _stack(hero, inp)
+    gpu = pr.run_gpu(st, inp)
+    ref = pr.run_oracle(inp)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"])
+    print(T, rep)
+    _assert_free(rep, pr.H_TOL["bf16"])
+    st.close()
+
+
 def test_zero_tokens_and_argument_errors(hero):
     import torch
     inp = pr.inputs("tiny_f32")
