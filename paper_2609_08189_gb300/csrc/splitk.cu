@@ -30,6 +30,9 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
   const bool ffn = m < M;
   const LayerOutArgs& p = ffn ? lo : ad.lo;
   const int row = ffn ? m : m - M;
+  const int t = p.idx[row];
+  const float sc = p.scale[row];
+  const LayerOutIn in = layer_out_load(p, t, n);   // in flight with the loads below
   float4 y;
   if (ffn) {
     const size_t off = (size_t)m * ld + n;
@@ -70,9 +73,6 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
     }
     y = make_float4(acc[0], acc[1], acc[2], acc[3]);
   }
-  const int t = p.idx[row];
-  const float sc = p.scale[row];
-  const LayerOutIn in = layer_out_load(p, t, n);
   float ss = 0.f, dd = 0.f, dp = 0.f;
   layer_out_store(p, t, n, in, y, sc, ss, dd, dp);
   if (!p.last) {
