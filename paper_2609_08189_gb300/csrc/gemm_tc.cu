@@ -58,7 +58,9 @@ struct TcCfg {
 };
 
 template <int EPI>
-constexpr int epi_warps() { return EPI == EPI_LAYER_OUT_WIDE || EPI == EPI_ATTN_ENTRY ? 8 : 4; }
+constexpr int epi_warps() {
+  return EPI == EPI_LAYER_OUT_WIDE || EPI == EPI_ATTN_ENTRY || EPI == EPI_RT_HEAD ? 8 : 4;
+}
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int& mb, int& nb,
                                             int group_m) {
@@ -384,12 +386,17 @@ __device__ __forceinline__ void epi_rt_s(const GemmArgs& a, uint32_t tbase, int 
 // p_hist = sigma(a / T_hist), m_hist *= p_hist (Eq. 15), g = sigma(a + b) (Eq. 16) and the
 // decision g >= tau (Eq. 3; ties run the FFN) or the caller's.
 template <int BN>
-__device__ __forceinline__ void epi_rt_head(const GemmArgs& a, uint32_t tbase, int m, bool valid) {
+__device__ __forceinline__ void epi_rt_head(const GemmArgs& a, uint32_t tbase, int m, bool valid,
+                                            int ew, float4* stg, uint32_t* qcnt, int parity) {
   static_assert(BN == 256, "f_theta's hidden width is one tile");
   const RouterTcArgs& r = a.rt;
+  // two epilogue warps per TMEM lane quadrant (8 warps): warp ew takes hidden units
+  // [128 (ew >> 2), + 128) of its 32 rows
+  const int lane = threadIdx.x & 31;
+  const int c_lo = (ew >> 2) * 128;
   float asum = 0.f;
 #pragma unroll 1
-  for (int c0 = 0; c0 < 256; c0 += 32) {
+  for (int c0 = c_lo; c0 < c_lo + 128; c0 += 32) {
     uint32_t v[32];
     tmem_ld32(tbase + c0, v);
     if (valid) {
@@ -398,6 +405,25 @@ __device__ __forceinline__ void epi_rt_head(const GemmArgs& a, uint32_t tbase, i
         asum = fmaf(__ldg(r.w.th_w2 + c0 + i), siluf_(__uint_as_float(v[i]) + __ldg(r.w.th_b1 + c0 + i)), asum);
     }
   }
+  // The two halves of a row meet in the warps' staging areas, in a slot per tile parity, and
+  // are counted on a counter per tile parity: a warp is at most one tile ahead of its
+  // partner (it cannot reuse an accumulator before the partner released it), so a slot and
+  // a counter only ever see the two arrivals of one tile at a time.  A counter grows by 2 per
+  // use; the warp that finds it odd arrives second, adds the halves (lower half first) and
+  // finishes the row.  No barrier between the warps.
+  float* mine = reinterpret_cast<float*>(stg) + parity * 32;
+  mine[lane] = asum;
+  __syncwarp();
+  __threadfence_block();
+  uint32_t old = 0;
+  if (lane == 0) old = atomicAdd(qcnt + parity, 1u);
+  old = __shfl_sync(0xffffffffu, old, 0);
+  if ((old & 1u) == 0) return;   // first of the two
+  __threadfence_block();
+  const float4* st0 = ew < 4 ? stg : stg - 4 * 256;   // the lower half's warp
+  const float* lo = reinterpret_cast<const float*>(st0) + parity * 32;
+  const float* hi = reinterpret_cast<const float*>(st0 + 4 * 256) + parity * 32;
+  asum = lo[lane] + hi[lane];
   if (!valid) return;
   const float* sc = r.scal + (size_t)m * 4;
   const float av = asum + __ldg(r.w.th_b2);
@@ -696,7 +722,8 @@ __device__ __forceinline__ int split_tile(int g, int t1, int total, int& local) 
 template <int BN, int EPI, int CG>
 __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, int q, int ew,
                                              int lane, int mb, int nb, int M, int split,
-                                             float4* stg, int rank) {
+                                             float4* stg, int rank, uint32_t* qcnt = nullptr,
+                                             int parity = 0) {
   const int row0 = (mb * CG + rank) * BM + q * 32;
   if constexpr (EPI == EPI_STORE_F32) {
     epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
@@ -719,7 +746,7 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
   } else if constexpr (EPI == EPI_RT_S) {
     epi_rt_s<BN>(a, tbase, row0 + lane, row0 + lane < M);
   } else if constexpr (EPI == EPI_RT_HEAD) {
-    epi_rt_head<BN>(a, tbase, row0 + lane, row0 + lane < M);
+    epi_rt_head<BN>(a, tbase, row0 + lane, row0 + lane < M, ew, stg, qcnt + 2 * q, parity);
   } else if constexpr (EPI == EPI_LAYER_OUT) {
     epi_layer_out<BN, BN>(a, tbase, row0, M, nb, 0, stg);
   } else {
@@ -781,6 +808,7 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
     }
     mbar_init(drain_bar, 1);
     misc[1] = 0;  // abort flag
+    for (int i = 4; i < 12; ++i) misc[i] = 0;   // EPI_RT_HEAD: counters per quadrant and parity
     fence_mbar_init();
   }
   // both CTAs' barriers are initialised before either signals the other's (and before
@@ -961,7 +989,8 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
         else
           run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank);
       } else {
-        run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank);
+        run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank,
+                                   const_cast<uint32_t*>(misc) + 4, acc);
       }
       tc_fence_before();
       __syncwarp();

@@ -12,6 +12,8 @@
 namespace hero {
 namespace {
 
+constexpr int kRtMaxF = 64 + 128 + 1;   // [s; c; nu] for d_s = 64, d_m <= 128
+
 __device__ __forceinline__ uint16_t bf16_term(float x, int term) {
   __nv_bfloat16 h = __float2bfloat16_rn(x);
   for (int p = 0; p < term; ++p) {
@@ -23,60 +25,85 @@ __device__ __forceinline__ uint16_t bf16_term(float x, int term) {
 
 // W_c c and nu = 1 - cos(W_n s, W_c c) (Eq. 13), then f_theta's input [s; c; nu] as three
 // bf16 terms (term p of element e at column p F + e, zero padded to kf): the part of the
-// memory step after c, shared by the two memory kernels.  cb holds c, cvb receives W_c c.
+// memory step after c, shared by the two memory kernels.  xin is this warp's [s; c; nu]
+// (s and c stored, nu stored here), wc W_c ([in][out], read through L1), wnr
+// the lane's elements lane + 32 u of W_n s.  The sums run in the order of the plain loops.
 template <int DM>
-__device__ __forceinline__ void rt_tail(const RouterTcArgs& a, int t, int lane, float* cb, float* cvb,
-                                        const float* wn) {
+__device__ __forceinline__ void rt_tail(const RouterTcArgs& a, int t, int lane, float* xin,
+                                        const float* wc, const float (&wnr)[(DM + 31) / 32]) {
+  constexpr int NO = (DM + 31) / 32;
+  const int ds = a.d_h + a.d_a, F = ds + DM + 1;
+  const float* c = xin + ds;
   __syncwarp();
-  // W_c c (Eq. 13), w_c_t is [in][out]
-  for (int o = lane; o < DM; o += 32) {
-    float acc = 0.f;
-    for (int i = 0; i < DM; ++i) acc = fmaf(__ldg(a.w.w_c_t + i * DM + o), cb[i], acc);
-    cvb[o] = acc;
+  float cv[NO];
+#pragma unroll
+  for (int u = 0; u < NO; ++u) cv[u] = 0.f;
+#pragma unroll 8
+  for (int i = 0; i < DM; ++i) {
+    const float ci = c[i];
+#pragma unroll
+    for (int u = 0; u < NO; ++u)
+      if (lane + 32 * u < DM) cv[u] = fmaf(wc[i * DM + lane + 32 * u], ci, cv[u]);
   }
-  __syncwarp();
   float nu = 0.f;
   if (a.j > 1) {
     float xy = 0.f, xx = 0.f, yy = 0.f;
-    for (int o = lane; o < DM; o += 32) {
-      const float x = wn[o], y = cvb[o];
-      xy += x * y;
-      xx += x * x;
-      yy += y * y;
-    }
+#pragma unroll
+    for (int u = 0; u < NO; ++u)
+      if (lane + 32 * u < DM) {
+        const float x = wnr[u], y = cv[u];
+        xy += x * y;
+        xx += x * x;
+        yy += y * y;
+      }
     xy = warp_sum(xy);
     xx = warp_sum(xx);
     yy = warp_sum(yy);
     nu = 1.f - xy / (sqrtf(xx) * sqrtf(yy) + a.eps);
   }
-  // f_theta's input [s; c; nu]: term p of element e at column p * F + e
-  const int ds = a.d_h + a.d_a, F = ds + DM + 1;
-  const float* s = a.s + (size_t)t * ds;
-  uint16_t* fin = a.fin3 + (size_t)t * a.kf;
-  for (int col = lane; col < a.kf; col += 32) {
-    const int p = col / F, e = col - p * F;
-    uint16_t bits = 0;
-    if (p < 3) {
-      const float x = e < ds ? s[e] : (e < ds + DM ? cb[e - ds] : nu);
-      bits = bf16_term(x, p);
+  if (lane == 0) xin[ds + DM] = nu;
+  __syncwarp();
+  // two columns per 32-bit store
+  uint32_t* fin = reinterpret_cast<uint32_t*>(a.fin3 + (size_t)t * a.kf);
+  for (int cp = lane; cp < a.kf / 2; cp += 32) {
+    uint32_t pk = 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int col = 2 * cp + h, p = col / F, e = col - p * F;
+      if (p < 3) pk |= (uint32_t)bf16_term(xin[e], p) << (16 * h);
     }
-    fin[col] = bits;
+    fin[cp] = pk;
   }
+}
+
+// The warp's start: s into its [s; c; nu] row, W_n s into registers.
+template <int DM>
+__device__ __forceinline__ void rt_tail_load(const RouterTcArgs& a, int t, int lane, float* xin,
+                                             const float* wn, float (&wnr)[(DM + 31) / 32]) {
+  const int ds = a.d_h + a.d_a;
+  const float* sr = a.s + (size_t)t * ds;
+  for (int e = lane; e < ds; e += 32) xin[e] = sr[e];
+#pragma unroll
+  for (int u = 0; u < (DM + 31) / 32; ++u) wnr[u] = lane + 32 * u < DM ? wn[lane + 32 * u] : 0.f;
 }
 
 template <int DM>
 __global__ void __launch_bounds__(256) k_rt_mem(const RouterTcArgs a) {
-  pdl_enter();
   static_assert(DM <= 128, "DM / 4 lanes per S row");
-  __shared__ float cbuf[8][DM];
-  __shared__ float cvbuf[8][DM];
+  __shared__ float xin_s[8][kRtMaxF];
+  pdl_enter();
+  const float* wc = a.w.w_c_t;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = blockIdx.x * 8 + w;
   if (t >= a.T) return;   // whole warps only; nothing below synchronises the CTA
+  float* xin = xin_s[w];
   const float* q = a.qkvn + (size_t)t * 4 * DM;
   const float* k = q + DM;
   const float* v = q + 2 * DM;
   const float* wn = q + 3 * DM;   // W_n s
+  float wnr[(DM + 31) / 32];
+  rt_tail_load<DM>(a, t, lane, xin, wn, wnr);
+  const int ds = a.d_h + a.d_a;
   float* S = a.S + (size_t)t * DM * DM;
   float* z = a.zeta + (size_t)t * DM;
   float den = 0.f;
@@ -119,9 +146,13 @@ __global__ void __launch_bounds__(256) k_rt_mem(const RouterTcArgs a) {
     c.z += __shfl_xor_sync(0xffffffffu, c.z, o);
     c.w += __shfl_xor_sync(0xffffffffu, c.w, o);
   }
-  if (r0 == 0)
-    *reinterpret_cast<float4*>(&cbuf[w][4 * cq]) = make_float4(c.x * inv, c.y * inv, c.z * inv, c.w * inv);
-  rt_tail<DM>(a, t, lane, cbuf[w], cvbuf[w], wn);
+  if (r0 == 0) {
+    xin[ds + 4 * cq] = c.x * inv;
+    xin[ds + 4 * cq + 1] = c.y * inv;
+    xin[ds + 4 * cq + 2] = c.z * inv;
+    xin[ds + 4 * cq + 3] = c.w * inv;
+  }
+  rt_tail<DM>(a, t, lane, xin, wc, wnr);
 }
 
 // The memory step in its history form, for a forward pass that runs every routed block in
@@ -135,18 +166,22 @@ __global__ void __launch_bounds__(256) k_rt_mem(const RouterTcArgs a) {
 // history entries are taken in order (bitwise reproducible).
 template <int DM>
 __global__ void __launch_bounds__(256) k_rt_hist(const RouterTcArgs a) {
-  pdl_enter();
   static_assert(DM % 64 == 0 && DM <= 128, "two or four elements per lane");
   constexpr int EL = DM / 32;
-  __shared__ float cbuf[8][DM];
-  __shared__ float cvbuf[8][DM];
+  __shared__ float xin_s[8][kRtMaxF];
+  pdl_enter();
+  const float* wc = a.w.w_c_t;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = blockIdx.x * 8 + w;
   if (t >= a.T) return;   // whole warps only; nothing below synchronises the CTA
+  float* xin = xin_s[w];
   const float* q = a.qkvn + (size_t)t * 4 * DM;
   const float* k = q + DM;
   const float* v = q + 2 * DM;
   const float* wn = q + 3 * DM;   // W_n s
+  float wnr[(DM + 31) / 32];
+  rt_tail_load<DM>(a, t, lane, xin, wn, wnr);
+  const int ds = a.d_h + a.d_a;
   float fq[EL], fk[EL], vv[EL];
 #pragma unroll
   for (int e = 0; e < EL; ++e) {
@@ -189,11 +224,11 @@ __global__ void __launch_bounds__(256) k_rt_hist(const RouterTcArgs a) {
   float* Hj = H + (size_t)nh * 2 * DM;   // this block's entry
 #pragma unroll
   for (int e = 0; e < EL; ++e) {
-    cbuf[w][lane * EL + e] = c[e] * inv;
+    xin[ds + lane * EL + e] = c[e] * inv;
     Hj[lane * EL + e] = fk[e];
     Hj[DM + lane * EL + e] = vv[e];
   }
-  rt_tail<DM>(a, t, lane, cbuf[w], cvbuf[w], wn);
+  rt_tail<DM>(a, t, lane, xin, wc, wnr);
 }
 
 }  // namespace

@@ -128,14 +128,18 @@ class Report:
     compared_h: int = 0
 
 
-def compare_free(gpu: GpuRun, ref: Dict, tol_h: float) -> Report:
-    """Free-running comparison with the near-boundary rule."""
+def compare_free(gpu: GpuRun, ref: Dict, tol_h: float, boundary: float = BOUNDARY) -> Report:
+    """Free-running comparison with the near-boundary rule: a token whose oracle gate lies
+    within `boundary` of tau may take the other decision (it is then dropped from later
+    blocks); any other decision mismatch counts.  Full-depth bf16 stacks pass the
+    free-running gate bound here: gates that may drift by that much may also flip a
+    decision whose gate lies that close to tau."""
     g_ref, m_ref = ref["gate"], ref["mask"]
     L, T = g_ref.shape
     rep = Report(T)
     alive = np.ones(T, dtype=bool)            # token still on the same path as the oracle
     for j in range(L):
-        near = np.abs(g_ref[j] - ref_tau(ref)) < BOUNDARY
+        near = np.abs(g_ref[j] - ref_tau(ref)) < boundary
         mism = gpu.mask[j] != m_ref[j]
         far = alive & mism & ~near
         rep.mask_mismatch_far += int(far.sum())

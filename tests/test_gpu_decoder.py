@@ -147,7 +147,7 @@ def test_attention_full_size_sampled(hero):
 # ------------------------------------------------------------------------------
 
 def compare_decoder_free(gpu: pr.GpuRun, ref, n_seqs: int, seq_len: int,
-                         pos: np.ndarray = None) -> pr.Report:
+                         pos: np.ndarray = None, boundary: float = pr.BOUNDARY) -> pr.Report:
     """compare_free with attention contamination: a near-boundary flip of the token at
     position p of sequence b at block j drops positions >= p of sequence b from
     block j + 1 on (the token itself from block j on).  pos: position of each compared
@@ -159,7 +159,7 @@ def compare_decoder_free(gpu: pr.GpuRun, ref, n_seqs: int, seq_len: int,
     rep = pr.Report(T)
     alive = np.ones(T, dtype=bool)
     for j in range(L):
-        near = np.abs(g_ref[j] - ref["tau"]) < pr.BOUNDARY
+        near = np.abs(g_ref[j] - ref["tau"]) < boundary
         mism = gpu.mask[j] != m_ref[j]
         far = alive & mism & ~near
         rep.mask_mismatch_far += int(far.sum())
@@ -282,10 +282,11 @@ def test_decoder_full_size_prefix(hero):
     assert 0.0 < 1 - gpu_all.mask.mean() < 1.0
     gpu = pr.GpuRun(gpu_all.h_out[rows], gpu_all.gate[:, rows], gpu_all.mask[:, rows], gpu_all.counts)
     ref = _oracle_decoder(cfg, w, wa, h[rows], tau, B, P)
-    rep = compare_decoder_free(gpu, ref, B, P)
+    bound = pr.free_run_gate_bound("llama31_8b_prefill")
+    rep = compare_decoder_free(gpu, ref, B, P, boundary=bound)
     print("full-size prefix", rep, "bypass", 1 - gpu_all.mask.mean())
     assert rep.mask_mismatch_far == 0, rep
-    assert rep.gate_err < pr.free_run_gate_bound("llama31_8b_prefill"), rep
+    assert rep.gate_err < bound, rep
     assert rep.compared_h >= 0.5 * rep.n_tokens, rep
     assert rep.h_err < H_TOL, rep
     dec.close()

@@ -215,9 +215,10 @@ def test_full_size_sampled(hero, name, bypass, n_sample):
     gpu_all = pr.run_gpu(st, inp)          # all T tokens, bench launch configuration
     gpu = pr.GpuRun(gpu_all.h_out[rows], gpu_all.gate[:, rows], gpu_all.mask[:, rows], gpu_all.counts)
     ref = pr.run_oracle(inp, rows=rows)
-    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"])
+    bound = pr.free_run_gate_bound(name)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"], boundary=bound)
     print(name, rep, "bypass", 1 - gpu_all.mask.mean())
-    _assert_free(rep, pr.H_TOL["bf16"], max_boundary_frac=0.1, gate_tol=pr.free_run_gate_bound(name))
+    _assert_free(rep, pr.H_TOL["bf16"], max_boundary_frac=0.1, gate_tol=bound)
     # whole-workload properties: counts agree with decisions, bypass near the budget
     np.testing.assert_array_equal(gpu_all.counts, gpu_all.mask.sum(axis=1))
     target = cfg.bypass if bypass is None else bypass
