@@ -71,7 +71,7 @@ _CACHE: Dict[str, Inputs] = {}
 
 def inputs(name: str, cfg: Optional[hi.StackConfig] = None, bypass: Optional[float] = None) -> Inputs:
     cfg = cfg or hi.CONFIGS[name]
-    key = f"{cfg.name}:{cfg.n_tokens}:{bypass}"
+    key = f"{cfg!r}:{bypass}"   # the whole configuration (a changed width is another input)
     if key not in _CACHE:
         if len(_CACHE) > 1:      # keep host memory bounded across large workloads
             _CACHE.clear()

@@ -152,6 +152,51 @@ def test_router_paths_by_token_count(hero, T):
     st.close()
 
 
+@pytest.mark.parametrize("d_m", [16, 32, 128])
+def test_tensor_core_router_memory_widths(hero, d_m):
+    """The router on the tensor cores at other memory widths (small_bf16 widths, 4096 tokens:
+    the router contraction does not split): the fused stack (state form for d_m = 16 and 32,
+    history form for 128) against the oracle on every token, free-running; and the block
+    chain (hero_routed_block, state form) with the stack's decisions forced against the
+    stack."""
+    import torch
+    T = 4096
+    cfg = hi.CONFIGS["small_bf16"].replace(n_tokens=T, d_m=d_m)
+    inp = pr.inputs("small_bf16", cfg=cfg)
+    st = _stack(hero, inp)
+    gpu = pr.run_gpu(st, inp)
+    ref = pr.run_oracle(inp)
+    rep = pr.compare_free(gpu, ref, pr.H_TOL["bf16"])
+    print(d_m, rep)
+    _assert_free(rep, pr.H_TOL["bf16"])
+    d, L = cfg.d_model, cfg.n_layers
+    f = dict(device="cuda", dtype=torch.float32)
+    ts = {"S": torch.zeros((T, d_m, d_m), **f), "zeta": torch.zeros((T, d_m), **f),
+          "p_hist": torch.ones((T,), **f), "m_hist": torch.ones((T,), **f),
+          "d_prev": torch.zeros((T,), **f), "h_bar_prev": torch.zeros((T, d), **f),
+          "delta_prev": torch.zeros((T, d), **f)}
+    state = hero.make_state({k: v.data_ptr() for k, v in ts.items()})
+    stream = torch.cuda.current_stream().cuda_stream
+    h = torch.from_numpy(inp.h).cuda()
+    P = torch.from_numpy(inp.P.astype(np.int32) << 16).cuda().view(torch.float32)
+    forced = torch.from_numpy(gpu.mask.astype(np.uint8)).cuda()
+    g = torch.empty((L, T), device="cuda")
+    m = torch.empty((L, T), device="cuda", dtype=torch.uint8)
+    hero.hero_router_state_reset(st.model, T, state, stream)
+    for j in range(1, L + 1):
+        hb = h + P[j - 1]
+        h = torch.empty_like(hb)
+        hero.hero_routed_block(st.model, j, T, hb.data_ptr(), state, inp.tau,
+                               hero.HERO_FLAG_FORCE_MASK, forced[j - 1].data_ptr(), h.data_ptr(),
+                               g[j - 1].data_ptr(), m[j - 1].data_ptr(), 0, stream)
+    torch.cuda.synchronize()
+    st.check()
+    gd = np.abs(g.cpu().numpy().astype(np.float64) - gpu.gate)
+    print(d_m, "block chain vs stack: gate max", gd.max(), "mean", gd.mean())
+    assert gd.mean() < 1e-5 and gd.max() < pr.GATE_TOL
+    st.close()
+
+
 def test_zero_tokens_and_argument_errors(hero):
     import torch
     inp = pr.inputs("tiny_f32")
