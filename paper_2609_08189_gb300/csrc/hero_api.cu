@@ -354,7 +354,8 @@ hero_status validate_config(const hero_config* c) {
 // K splits for a tensor-core launch of `tiles` 128x256 output tiles over `kblocks`
 // 64-wide K-blocks (`rows` x `n` outputs), from a wave-quantisation cost model: the
 // GEMM takes ceil(tiles * s / num_sms) waves of ceil(kblocks / s) K-block steps
-// (~0.4 us each on one SM) plus the last tile's epilogue (~50 us for the block-closing
+// (~0.4 us each on one SM when the tensor pipe bounds them; ~0.75 us at 128 rows or fewer,
+// where a step streams its 32 KB weight tile from HBM) plus the last tile's epilogue (~50 us for the block-closing
 // epilogue, ~10 us for a plain store), and s > 1 adds a finishing pass that moves
 // rows * n * (4 s + epi_bytes) bytes at ~5 TB/s.  rows is the launch's upper bound
 // (the routed count is device-resident).  Every split keeps >= 1 K-block.
@@ -367,7 +368,7 @@ int choose_splits(int tiles, int kblocks, int num_sms, long rows, long n, int ep
     const int eff = (kblocks + kpb - 1) / kpb;   // splits that own K-blocks
     if (eff != s) continue;
     const long waves = ((long)tiles * s + num_sms - 1) / num_sms;
-    double t = (double)waves * kpb * 0.4;
+    double t = (double)waves * kpb * (rows <= 128 ? 0.75 : 0.4);
     if (s > 1)
       t += 10.0 + (double)rows * n * (4.0 * s + epi_bytes) / 5.0e6;
     else
