@@ -424,14 +424,21 @@ __device__ __forceinline__ void epi_rt_head(const GemmArgs& a, uint32_t tbase, i
   const float* lo = reinterpret_cast<const float*>(st0) + parity * 32;
   const float* hi = reinterpret_cast<const float*>(st0 + 4 * 256) + parity * 32;
   asum = lo[lane] + hi[lane];
-  if (!valid) return;
+  float p = 0.f, mm = 0.f, g = 0.f;
   const float* sc = r.scal + (size_t)m * 4;
-  const float av = asum + __ldg(r.w.th_b2);
-  const float bv = sc[2] + __ldg(r.w.ps_b2);
-  const float p = sigmoidf_(av / r.t_hist);
-  const float mm = r.mst[m] * p;
-  const float g = sigmoidf_(av + bv);
-  const uint8_t dec = r.mask_in ? (r.mask_in[m] ? 1 : 0) : (g >= r.tau ? 1 : 0);
+  uint8_t dec = 0;
+  if (valid) {
+    const float av = asum + __ldg(r.w.th_b2);
+    const float bv = sc[2] + __ldg(r.w.ps_b2);
+    p = sigmoidf_(av / r.t_hist);
+    mm = r.mst[m] * p;
+    g = sigmoidf_(av + bv);
+    dec = r.mask_in ? (r.mask_in[m] ? 1 : 0) : (g >= r.tau ? 1 : 0);
+  }
+  // the warp's 32 consecutive rows: their FFN count for the compaction
+  const uint32_t bal = __ballot_sync(0xffffffffu, dec != 0);
+  if (r.chunk_cnt && lane == 0 && m - lane < r.T) r.chunk_cnt[(m - lane) >> 5] = __popc(bal);
+  if (!valid) return;
   r.pst[m] = p;
   r.mst[m] = mm;
   r.dprev[m] = sc[0];

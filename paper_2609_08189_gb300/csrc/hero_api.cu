@@ -210,6 +210,7 @@ struct hero_model {
   CUtensorMap tm_whu3, tm_wq3, tm_th3, tm_enc3, tm_s3, tm_fin3;
   uint16_t *rt_enc3 = nullptr, *rt_s3 = nullptr, *rt_fin3 = nullptr;
   float *rt_scal = nullptr, *rt_s = nullptr, *rt_qkvn = nullptr;
+  int* chunk_cnt = nullptr;   // [ceil(T / 32)] FFN decisions per 32 tokens (RouterTcArgs)
   // the history form of the memory (d_m = 64 or 128 on the tensor-core router): per token
   // [L_R][2 d_m] entries phi(k_i) | v_i, and the decay weights [L_R][L_R] (RouterTcArgs)
   float *hist = nullptr, *hw = nullptr;
@@ -767,6 +768,7 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         {(void**)&m->rt_s3, m->rtc ? Tm * 3 * ds * 2 : 0},
         {(void**)&m->rt_qkvn, m->rtc ? Tm * 4 * dm * 4 : 0},
         {(void**)&m->rt_fin3, m->rtc ? Tm * (size_t)m->rt_kf * 2 : 0},
+        {(void**)&m->chunk_cnt, m->rtc ? (Tm + 31) / 32 * 4 : 0},
         {(void**)&m->hist, hist_form ? Tm * (size_t)LR * 2 * dm * 4 : 0},
         {(void**)&m->hw, hist_form ? (size_t)LR * LR * 4 : 0},
         // split-K partials of the few-wave launches (router contraction, FFN down)
@@ -881,6 +883,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
   const int j = jr + 1;                 // routed index (layer jj = n_dense + jr)
   const bool dense = flags & HERO_FLAG_DENSE;
   const size_t es = m->esz;
+  bool chunk_counted = false;   // the router left per-32-token FFN counts (m->chunk_cnt)
   if (!dense) {
     GemmArgs g{};
     g.m_dev = nullptr;
@@ -905,6 +908,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     }
     const bool pair = m->bf16 && rs == 1 && T >= kPairMinRows;
     if (pair && m->rtc && c.router_variant == 0) {
+      chunk_counted = true;
       // the router on the tensor cores: five launches (RouterTcArgs)
       RouterTcArgs rt{};
       rt.T = T;
@@ -943,6 +947,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       rt.mask = m->mask;
       rt.gate_out = gate_out_j;
       rt.mask_out = mask_out_j;
+      rt.chunk_cnt = m->chunk_cnt;
       const int ds = c.d_h + c.d_a;
       GemmArgs g1 = g;   // 1. the router contraction, encoder hidden and f_psi in the epilogue
       g1.rt = rt;
@@ -1052,7 +1057,8 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
                  dense ? mask_out_j : nullptr};
   NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, hbar, m->part,
               m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
-  if (T <= kRouteNormMaxT) {   // few tokens: compaction inside the norm's launch
+  if (chunk_counted) ca.chunk_cnt = m->chunk_cnt;
+  if (T <= kRouteNormMaxT || chunk_counted) {   // compaction inside the norm's launch
     CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_route_norm(ca, na, m->num_sms, st); }));
   } else {
     CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));

@@ -183,6 +183,7 @@ struct RouterTcArgs {
   uint8_t* mask;
   float* gate_out;
   uint8_t* mask_out;
+  int* chunk_cnt;        // [ceil(T / 32)] FFN decisions per 32 consecutive tokens (step 5), or nullptr
 };
 
 struct GemmArgs {
@@ -401,6 +402,9 @@ struct CompactArgs {
   int* count_out;        // caller slot or nullptr
   float* gate_out;       // dense mode: fill with 1 (or nullptr)
   uint8_t* mask_out;     // dense mode: fill with 1 (or nullptr)
+  // launch_route_norm: the FFN decisions of each 32 consecutive tokens, counted by the
+  // router's last launch (RouterTcArgs::chunk_cnt), or nullptr (a ballot scan from token 0)
+  const int* chunk_cnt;
 };
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
 
@@ -419,7 +423,8 @@ struct NormArgs {
 };
 // wpr: warps per row (each takes a contiguous d / wpr column range; wpr divides d / 4)
 cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st);
-// k_compact and k_norm as one launch (T <= kRouteNormMaxT; same outputs).
+// k_compact and k_norm as one launch (same outputs): T <= kRouteNormMaxT, or any T with the
+// per-32-token FFN counts (CompactArgs::chunk_cnt).
 constexpr int kRouteNormMaxT = 2048;
 cudaError_t launch_route_norm(const CompactArgs& c, const NormArgs& a, int num_sms, cudaStream_t st);
 

@@ -868,9 +868,11 @@ __global__ void __launch_bounds__(256) k_norm(const NormArgs a, int wpr) {
 
 // ------------------------------------------------------------------------------
 // k_route_norm: k_compact and k_norm in one launch for token counts up to
-// kRouteNormMaxT.  Warp gw serves token t = gw / wpr (column range gw % wpr); it counts
-// the FFN decisions of the tokens before t with one ballot per 32 tokens (every warp
-// repeats that scan, which at these token counts costs less than a launch), so that
+// kRouteNormMaxT, or any count when the router left per-32-token FFN counts (chunk_cnt).
+// Warp gw serves token t = gw / wpr (column range gw % wpr); it counts the FFN decisions
+// of the tokens before t (the chunks' counts, then one ballot per 32 tokens; without
+// counts every warp repeats the ballot scan, which at those token counts costs less than a
+// launch), so that
 // token t's branch row is its rank among the tokens of its branch, as in k_compact.
 // The column-range-0 warp of a token writes the token's index and scale entries; the
 // warp of the last token writes the counts.  Outputs equal those of the two kernels.
@@ -886,7 +888,16 @@ __global__ void __launch_bounds__(256) k_route_norm(const CompactArgs c, const N
   bool f = true;
   if (!c.dense) {
     pf = 0;
-    for (int b = 0; b < t; b += 128) {
+    int b0 = 0;
+    if (c.chunk_cnt) {   // whole 32-token chunks before t's from their counts
+      const int nc = t >> 5;
+      int sum = 0;
+#pragma unroll 4
+      for (int i = lane; i < nc; i += 32) sum += c.chunk_cnt[i];
+      pf = __reduce_add_sync(0xffffffffu, sum);
+      b0 = nc << 5;
+    }
+    for (int b = b0; b < t; b += 128) {
       int n = 0;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
@@ -1046,7 +1057,7 @@ cudaError_t launch_norm(const NormArgs& a, int num_sms, cudaStream_t st) {
 
 cudaError_t launch_route_norm(const CompactArgs& c, const NormArgs& a, int num_sms, cudaStream_t st) {
   if (a.T <= 0) return cudaSuccess;
-  if (a.T > kRouteNormMaxT || c.T != a.T) return cudaErrorInvalidValue;
+  if ((a.T > kRouteNormMaxT && !c.chunk_cnt) || c.T != a.T) return cudaErrorInvalidValue;
   const int wpr = norm_wpr(a, num_sms);
   const long warps = (long)a.T * wpr;
   return launch_pdl(k_route_norm, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, c, a, wpr);
