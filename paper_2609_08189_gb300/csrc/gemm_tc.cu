@@ -34,10 +34,13 @@ constexpr int EPI_NONE = -1;   // no second problem
 // of 2) computes a 256 x BN tile with the 2-SM MMA: each CTA holds 128 rows of A, BN / 2
 // rows of B and 128 rows of the accumulator, so per FLOP each SM stages a third less
 // operand data through its shared memory.
-template <int BN, int EPIW, int CG = 1>
+// INB = 1 (the wide block-closing epilogue of the adapter's rank-d_r up projection, one
+// K-block per tile): a single ring stage, and per epilogue warp a 12 KB buffer that the
+// epilogue's row inputs (h_bar, delta, P) are copied into with cp.async.
+template <int BN, int EPIW, int CG = 1, int INB = 0>
 struct TcCfg {
   static constexpr int B_ROWS = BN / CG;   // rows of B staged by this CTA
-  static constexpr int STAGES = CG == 2 ? 6 : (BN == 256 ? 4 : 6);
+  static constexpr int STAGES = INB ? 1 : (CG == 2 ? 6 : (BN == 256 ? 4 : 6));
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = B_ROWS * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
@@ -53,9 +56,19 @@ struct TcCfg {
   static constexpr int THREADS = 64 + 32 * EPI_WARPS;
   // ring | barriers (256 B) | per-epilogue-warp staging tiles (32 x 32 fp32 each)
   static constexpr uint32_t EPI_STAGE_OFF = STAGES * STAGE_BYTES + 256;
-  static constexpr size_t SMEM = (size_t)EPI_STAGE_OFF + EPI_WARPS * 32 * 32 * 4 + 1024;
+  static constexpr uint32_t IN_OFF = EPI_STAGE_OFF + EPI_WARPS * 32 * 32 * 4;
+  static constexpr uint32_t IN_BYTES = INB ? 3 * 8 * 32 * 16 : 0;   // per epilogue warp
+  static constexpr size_t SMEM = (size_t)IN_OFF + EPI_WARPS * IN_BYTES + 1024;
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
+
+// The wide block-closing epilogue loads its row inputs with cp.async (epi_layer_out_async);
+// -DHERO_WIDE_INBUF=0 keeps the register-held loads of epi_layer_out.
+#ifndef HERO_WIDE_INBUF
+#define HERO_WIDE_INBUF 1
+#endif
+template <int EPI>
+constexpr int epi_inbuf() { return EPI == EPI_LAYER_OUT_WIDE && HERO_WIDE_INBUF ? 1 : 0; }
 
 template <int EPI>
 constexpr int epi_warps() {
@@ -597,6 +610,87 @@ __device__ __forceinline__ void epi_layer_out(const GemmArgs& a, uint32_t tbase,
   }
 }
 
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async8(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(src) : "memory");
+}
+
+// The block-closing epilogue with its row inputs copied into shared memory (inb: this
+// warp's [3][8][32] 16-byte slots: h_bar, delta, P_{j+1} of the lane's 4 columns of its 8
+// rows) by cp.async, issued for a whole 32-column chunk before the accumulator is read from
+// TMEM, so that a chunk's loads are in flight together without holding registers.  The
+// arithmetic and its order are epi_layer_out's.
+template <int BN, int NCOLS>
+__device__ __forceinline__ void epi_layer_out_async(const GemmArgs& a, uint32_t tbase, int row0,
+                                                    int M, int nb, int c_begin, float4* st,
+                                                    float4* inb) {
+  static_assert(NCOLS % kTcPartCols == 0, "whole partial-sum slots per warp");
+  const int lane = threadIdx.x & 31;
+  const int sub = lane >> 3, slot = lane & 7;
+  const LayerOutArgs& p = a.lo;
+  const bool need_pn = !p.last && p.p_next;
+  const bool need_dv = !p.last && p.router && !p.first;
+  int tok[8];
+  float scl[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int m = row0 + sub + 4 * k;
+    tok[k] = m < M ? p.idx[m] : -1;
+    scl[k] = m < M ? p.scale[m] : 0.f;
+  }
+  float ss[8], dd[8], dp[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) ss[k] = dd[k] = dp[k] = 0.f;
+  const uint32_t ib = smem_u32(inb);
+  auto slot_addr = [&](int arr, int k) { return ib + (uint32_t)(((arr * 8 + k) * 32 + lane) * 16); };
+#pragma unroll 1
+  for (int c0 = c_begin; c0 < c_begin + NCOLS; c0 += 32) {
+    const int n = nb * BN + c0 + 4 * slot;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (tok[k] < 0) continue;
+      const size_t off = (size_t)tok[k] * p.d + n;
+      cp_async16(slot_addr(0, k), p.hbar + off);
+      if (need_dv) cp_async16(slot_addr(1, k), p.delta + off);
+      if (need_pn) {
+        if (p.p_bf16)
+          cp_async8(slot_addr(2, k), static_cast<const uint16_t*>(p.p_next) + off);
+        else
+          cp_async16(slot_addr(2, k), static_cast<const float*>(p.p_next) + off);
+      }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    uint32_t r[32];
+    tmem_ld32(tbase + c0, r);
+    stage_rows(st, r, lane);
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncwarp();
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (tok[k] < 0) continue;
+      LayerOutIn in;
+      in.hb = inb[(0 * 8 + k) * 32 + lane];
+      in.dprev = need_dv ? inb[(1 * 8 + k) * 32 + lane] : make_float4(0.f, 0.f, 0.f, 0.f);
+      in.pn = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (need_pn) {
+        if (p.p_bf16) {
+          const uint2 u = *reinterpret_cast<const uint2*>(&inb[(2 * 8 + k) * 32 + lane]);
+          in.pn = make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                              __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+        } else {
+          in.pn = inb[(2 * 8 + k) * 32 + lane];
+        }
+      }
+      layer_out_store(p, tok[k], n, in, staged(st, sub + 4 * k, slot), scl[k], ss[k], dd[k], dp[k]);
+    }
+    __syncwarp();
+    if (!p.last && (c0 + 32) % kTcPartCols == 0)
+      flush_partials<BN, NCOLS>(p, tok, ss, dd, dp, slot, (nb * BN + c0 + 32) / kTcPartCols - 1);
+  }
+}
+
 // Attention output projection closing into the block entry (Eq. 7): per element
 // h_bar_j = h_{j-1} + acc, delta_j = h_bar_j - h_bar_{j-1} (zero in the first routed
 // block); h_bar_j and delta_j overwrite the carried h_bar_{j-1} and delta_{j-1}
@@ -730,7 +824,7 @@ template <int BN, int EPI, int CG>
 __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, int q, int ew,
                                              int lane, int mb, int nb, int M, int split,
                                              float4* stg, int rank, uint32_t* qcnt = nullptr,
-                                             int parity = 0) {
+                                             int parity = 0, float4* inb = nullptr) {
   const int row0 = (mb * CG + rank) * BM + q * 32;
   if constexpr (EPI == EPI_STORE_F32) {
     epi_store_f32<BN>(a, tbase, row0, M, nb, split, stg);
@@ -756,18 +850,20 @@ __device__ __forceinline__ void run_epilogue(const GemmArgs& a, uint32_t tbase, 
     epi_rt_head<BN>(a, tbase, row0 + lane, row0 + lane < M, ew, stg, qcnt + 2 * q, parity);
   } else if constexpr (EPI == EPI_LAYER_OUT) {
     epi_layer_out<BN, BN>(a, tbase, row0, M, nb, 0, stg);
+  } else if constexpr (EPI == EPI_LAYER_OUT_WIDE && HERO_WIDE_INBUF) {
+    epi_layer_out_async<BN, BN / 2>(a, tbase, row0, M, nb, (ew >> 2) * (BN / 2), stg, inb);
   } else {
     epi_layer_out<BN, BN / 2>(a, tbase, row0, M, nb, (ew >> 2) * (BN / 2), stg);
   }
 }
 
 template <int BN, int EPI0, int EPI1, int CG>
-__global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
+__global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG, epi_inbuf<EPI0>()>::THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
               const GemmArgs a0, const GemmArgs a1) {
   if (a0.pdl_mode != 2) pdl_enter();
-  using C = TcCfg<BN, epi_warps<EPI0>(), CG>;
+  using C = TcCfg<BN, epi_warps<EPI0>(), CG, epi_inbuf<EPI0>()>;
   constexpr bool kGrouped = EPI1 != EPI_NONE;
   constexpr bool kPair = CG == 2;
   extern __shared__ uint8_t smem_raw[];
@@ -997,7 +1093,8 @@ __global__ void __launch_bounds__(TcCfg<BN, epi_warps<EPI0>(), CG>::THREADS, 1)
           run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank);
       } else {
         run_epilogue<BN, EPI0, CG>(a0, tbase, q, ew, lane, mb, nb, P0.M, sp, stg, rank,
-                                   const_cast<uint32_t*>(misc) + 4, acc);
+                                   const_cast<uint32_t*>(misc) + 4, acc,
+                                   reinterpret_cast<float4*>(smem + C::IN_OFF + ew * C::IN_BYTES));
       }
       tc_fence_before();
       __syncwarp();
@@ -1038,7 +1135,7 @@ template <int BN, int EPI0, int EPI1, int CG = 1>
 cudaError_t launch_tc(const CUtensorMap& tmA0, const CUtensorMap& tmB0, const GemmArgs& a0,
                       const CUtensorMap& tmA1, const CUtensorMap& tmB1, const GemmArgs& a1,
                       int num_sms, cudaStream_t st) {
-  using C = TcCfg<BN, epi_warps<EPI0>(), CG>;
+  using C = TcCfg<BN, epi_warps<EPI0>(), CG, epi_inbuf<EPI0>()>;
   auto kernel = k_gemm_tc<BN, EPI0, EPI1, CG>;
   static bool attr_set = false;  // per process; the attribute is per function
   static int pair_slots = 0;     // CG = 2: CTA pairs resident at once
