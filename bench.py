@@ -357,6 +357,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-speculate", action="store_true",
+                    help="batches of one 128-row tile: FFN on the routed tokens only, after the "
+                         "router (default: every token, beside the router)")
     # overrides for profiling small cases (a line produced with them is not the workload's)
     ap.add_argument("--tau", type=float, default=None)
     ap.add_argument("--tokens", type=int, default=None)
@@ -498,18 +501,19 @@ def main():
                             ClockSampler(local_rank), t_gen)
 
     # ---- routed stack (the metric) ----
+    rflags = hero.HERO_FLAG_NO_SPECULATE if args.no_speculate else 0
     for _ in range(args.warmup):
-        run(0)
+        run(rflags)
     torch.cuda.synchronize()
     stack.check()
     sampler = ClockSampler(local_rank)
-    ms, clocks = timed(lambda: run(0), args.steps, sampler)   # the metric: no instrumentation
+    ms, clocks = timed(lambda: run(rflags), args.steps, sampler)   # the metric: no instrumentation
     stack.check()
     # per-kernel breakdown from a separate instrumented pass (events around every launch
     # serialise launches that otherwise overlap their predecessor's tail)
     hero.hero_get_profile(stack.model, reset=True)
     hero.hero_set_profiling(stack.model, True)
-    timed(lambda: run(0), args.steps)
+    timed(lambda: run(rflags), args.steps)
     hero.hero_set_profiling(stack.model, False)
     prof = hero.hero_get_profile(stack.model, reset=True)
     stack.check()
@@ -521,7 +525,7 @@ def main():
         cap = torch.cuda.Stream(dev)
         cap.wait_stream(stream)
         with torch.cuda.graph(graph, stream=cap):
-            run(0, cap)
+            run(rflags, cap)
         stream.wait_stream(cap)
         for _ in range(args.warmup):
             graph.replay()
@@ -554,15 +558,15 @@ def main():
         def run_host():
             if kvdec:
                 hero.hero_decode_step(stack.model, B, pos_h.data_ptr(), S, hp.data_ptr(), tau,
-                                      hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                      hero.HERO_FLAG_HOST_IO | rflags, 0, ho_.data_ptr(), 0, 0,
                                       cp.data_ptr(), stream.cuda_stream)
             elif decoder:
                 hero.hero_decoder_forward(stack.model, B, S, hp.data_ptr(), tau,
-                                          hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                          hero.HERO_FLAG_HOST_IO | rflags, 0, ho_.data_ptr(), 0, 0,
                                           cp.data_ptr(), stream.cuda_stream)
             else:
                 hero.hero_routed_ffn_stack(stack.model, T, hp.data_ptr(), Pp.data_ptr(), tau,
-                                           hero.HERO_FLAG_HOST_IO, 0, ho_.data_ptr(), 0, 0,
+                                           hero.HERO_FLAG_HOST_IO | rflags, 0, ho_.data_ptr(), 0, 0,
                                            cp.data_ptr(), stream.cuda_stream)
         run_host()
         torch.cuda.synchronize()

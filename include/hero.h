@@ -149,7 +149,13 @@ enum {
   /* h_in, attn_delta, mask_in, h_out, gate_out, mask_out and ffn_count_out are
    * HOST pointers; the library copies them to and from the device on the stream
    * (page-locked host memory makes the copies asynchronous). */
-  HERO_FLAG_HOST_IO = 4u
+  HERO_FLAG_HOST_IO = 4u,
+  /* bf16 models, batches of at most 128 tokens (one GEMM tile of rows): by default
+   * the FFN and the adapter branch run on every token while the router runs beside
+   * them on a second stream, and the block-closing step takes each token's branch
+   * from the router's decision (Eq. 3), with the same results.  This flag runs the
+   * FFN on the routed tokens only, after the router. */
+  HERO_FLAG_NO_SPECULATE = 8u
 };
 
 /* Copy, convert and repack the parameters to the current CUDA device and size

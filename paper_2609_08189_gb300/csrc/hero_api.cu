@@ -228,6 +228,12 @@ struct hero_model {
   // host-IO call's uploads into the workspace wait for it, not for the previous
   // call's result downloads, so both directions overlap
   cudaEvent_t ev_kernels_done = nullptr;
+  // batches of one 128-row tile (bf16, shared-memory router): the router's launches run on
+  // side_stream, forked after the block entry (ev_fork) and joined before the block-closing
+  // launch (ev_join); rws holds their split-K router contraction slices
+  cudaStream_t side_stream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  float* rws = nullptr;
 
   // tensor maps (bf16 only)
   CUtensorMap tm_xl, tm_uf, tm_ua, tm_act, tm_ah, tm_wr;
@@ -360,11 +366,12 @@ hero_status validate_config(const hero_config* c) {
 // epilogue, ~10 us for a plain store), and s > 1 adds a finishing pass that moves
 // rows * n * (4 s + epi_bytes) bytes at ~5 TB/s.  rows is the launch's upper bound
 // (the routed count is device-resident).  Every split keeps >= 1 K-block.
+constexpr int kMaxSplits = 16;
 int choose_splits(int tiles, int kblocks, int num_sms, long rows, long n, int epi_bytes) {
   if (tiles <= 0 || kblocks <= 1) return 1;
   double best_t = 0.0;
   int best = 1;
-  for (int s = 1; s <= 16 && s <= kblocks; ++s) {
+  for (int s = 1; s <= kMaxSplits && s <= kblocks; ++s) {
     const int kpb = (kblocks + s - 1) / s;
     const int eff = (kblocks + kpb - 1) / kpb;   // splits that own K-blocks
     if (eff != s) continue;
@@ -443,7 +450,10 @@ void free_model(hero_model* m) {
   for (auto e : m->ev_ready) cudaEventDestroy(e);
   for (auto e : m->ev_consumed) cudaEventDestroy(e);
   if (m->ev_kernels_done) cudaEventDestroy(m->ev_kernels_done);
+  if (m->ev_fork) cudaEventDestroy(m->ev_fork);
+  if (m->ev_join) cudaEventDestroy(m->ev_join);
   if (m->copy_stream) cudaStreamDestroy(m->copy_stream);
+  if (m->side_stream) cudaStreamDestroy(m->side_stream);
   void* ptrs[] = {m->wgu, m->wup, m->wdown, m->w1, m->w2, m->wr, m->ffn_gain, m->router_small,
                   m->ws, m->io, m->wqkv, m->wo, m->attn_gain, m->aws, m->rope_cs, m->kv,
                   m->dec_pm, m->dec_pos, m->dec_ws, m->wdT, m->wguT, m->w1T, m->w2T, m->bws,
@@ -774,6 +784,9 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
         // split-K partials of the few-wave launches (router contraction, FFN down)
         {(void**)&m->splitk_ws, bf16 ? splitk_ws_floats(c.max_tokens, m->num_sms, (int)nY,
                                                         (int)(2 * d), (int)d, (int)I) * 4 : 0},
+        // the router contraction beside the FFN (one 128-row tile of tokens: at most 256
+        // stacked rows, at most kMaxSplits slices)
+        {(void**)&m->rws, m->rsm_w ? (size_t)kMaxSplits * 256 * nY * 4 : 0},
     };
     for (auto& it : items) off += (it.bytes + 1023) & ~(size_t)1023;
     CUDA_M(cudaMalloc(&m->ws, off));
@@ -838,6 +851,11 @@ extern "C" hero_status hero_init_weights(const hero_config* cfg, const hero_weig
     if (!ok) return bail(fail(HERO_ERR_CUDA, "tensor map encoding failed"));
   }
   CUDA_M(cudaEventCreateWithFlags(&m->ev_kernels_done, cudaEventDisableTiming));
+  if (m->rsm_w) {
+    CUDA_M(cudaStreamCreateWithFlags(&m->side_stream, cudaStreamNonBlocking));
+    CUDA_M(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming));
+    CUDA_M(cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming));
+  }
   *out = m;
   return HERO_OK;
 #undef TRY_M
@@ -884,6 +902,30 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
   const bool dense = flags & HERO_FLAG_DENSE;
   const size_t es = m->esz;
   bool chunk_counted = false;   // the router left per-32-token FFN counts (m->chunk_cnt)
+  // One 128-row tile of tokens (a decoding batch): the FFN and the adapter branch run on
+  // every token while the router runs on the model's second stream, on the SMs that the
+  // gate/up launch leaves idle; the block-closing launch then takes each token's branch from
+  // the router's decision (Eq. 3), so every output equals that of the compacted branches.
+  // Bypassed tokens cost FFN FLOPs, but at one tile the FFN GEMMs are bound by their weight
+  // stream, which they read whole either way.
+  const int m_t0 = (T + 127) / 128;
+  const int gu_units = std::min(m_t0 * ((2 * I + 255) / 256 + (r + 255) / 256), m->num_sms);
+  const int side_sms = m->num_sms - gu_units;
+  const int ds0 = m->bf16 ? choose_splits(m_t0 * (d / 256), (I + 63) / 64, m->num_sms,
+                                          (long)m_t0 * 128, d, 22)
+                          : 1;
+  const bool spec_shape = !dense && m->bf16 && m->side_stream && m->rsm_w &&
+                          c.router_variant == 0 && T > 0 && T <= 128 && r <= 64 && r % 8 == 0 &&
+                          ds0 > 1 && side_sms >= 16;
+  const bool spec = spec_shape && !(flags & HERO_FLAG_NO_SPECULATE);
+  const cudaStream_t rst = spec ? m->side_stream : st;   // the router's stream
+  // the router's SMs, which set its split count and tokens per CTA (and with them its fp32
+  // summation order): the same with HERO_FLAG_NO_SPECULATE, so both give the same bits
+  const int r_sms = spec_shape ? side_sms : m->num_sms;
+  if (spec) {
+    CUDA_TRY(cudaEventRecord(m->ev_fork, st));
+    CUDA_TRY(cudaStreamWaitEvent(rst, m->ev_fork, 0));
+  }
   if (!dense) {
     GemmArgs g{};
     g.m_dev = nullptr;
@@ -989,7 +1031,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     int rs2 = 1;
     if (stacked) {
       const int m2 = (2 * T + 127) / 128;
-      rs2 = choose_splits(m2 * ((nY + 255) / 256), (d + 63) / 64, m->num_sms, (long)m2 * 128, nY, 4);
+      rs2 = choose_splits(m2 * ((nY + 255) / 256), (d + 63) / 64, r_sms, (long)m2 * 128, nY, 4);
       g.m_static = 2 * T;
       g.m_max = 2 * T;
       g.K = d;
@@ -998,13 +1040,14 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       g.out_f32 = m->Y;
       g.ldo = nY;
       if (rs2 > 1) {
-        g.out_f32 = m->splitk_ws;
+        // beside the FFN, FFN down's slices take splitk_ws meanwhile; rws holds any split count
+        g.out_f32 = spec_shape ? m->rws : m->splitk_ws;
         g.k_splits = rs2;
         g.split_stride = (long)m2 * 128 * nY;
       }
     }
-    CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, st, [&] {
-      if (stacked) return launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl2, m->tm_wr1, g, m->num_sms, st);
+    CUDA_TRY(timed(m, HERO_K_ROUTER_GEMM, rst, [&] {
+      if (stacked) return launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl2, m->tm_wr1, g, r_sms, rst);
       if (!m->bf16) return launch_gemm_simt(EPI_STORE_F32, g, st);
       return pair ? launch_gemm_tc2(EPI_STORE_F32, m->tm_xl, m->tm_wr_p, g, m->num_sms, st)
                   : launch_gemm_tc(256, EPI_STORE_F32, m->tm_xl, m->tm_wr, g, m->num_sms, st);
@@ -1021,7 +1064,7 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.d_enc = c.d_enc;
     ra.d_head = c.d_head;
     ra.d_path = c.d_path;
-    ra.Y = g.k_splits > 1 ? m->splitk_ws : m->Y;   // the router adds split-K slices as it reads
+    ra.Y = g.k_splits > 1 ? g.out_f32 : m->Y;   // the router adds split-K slices as it reads
     ra.y_splits = g.k_splits > 1 ? g.k_splits : 1;
     ra.y_split_stride = g.k_splits > 1 ? g.split_stride : 0;
     ra.y_rows = stacked ? 2 : 1;
@@ -1046,8 +1089,8 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     ra.wsm = c.router_variant == 0 ? m->rsm_w : nullptr;
     ra.err = m->err;
     ra.wait_ns = wait_limit_ns();
-    CUDA_TRY(timed(m, HERO_K_ROUTER, st, [&] {
-      return ra.wsm ? launch_router_sm(c.d_m, ra, m->num_sms, st)
+    CUDA_TRY(timed(m, HERO_K_ROUTER, rst, [&] {
+      return ra.wsm ? launch_router_sm(c.d_m, ra, r_sms, rst)
                     : launch_router(c.d_m, ra, m->num_sms, st);
     }));
     }
@@ -1058,7 +1101,13 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
   NormArgs na{T, d, m->np, m->counts, m->idx_f, m->idx_a, hbar, m->part,
               m->ffn_gain + (size_t)jj * d, c.rms_eps, m->u_f, m->u_a, (int)m->bf16};
   if (chunk_counted) ca.chunk_cnt = m->chunk_cnt;
-  if (T <= kRouteNormMaxT || chunk_counted) {   // compaction inside the norm's launch
+  if (spec) {   // compaction after the router on its stream; LN_ffn of every token here
+    CUDA_TRY(timed(m, HERO_K_COMPACT, rst, [&] { return launch_compact(ca, rst); }));
+    CUDA_TRY(cudaEventRecord(m->ev_join, rst));
+    NormArgs nall = na;
+    nall.counts = nullptr;
+    CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_norm(nall, m->num_sms, st); }));
+  } else if (T <= kRouteNormMaxT || chunk_counted) {   // compaction inside the norm's launch
     CUDA_TRY(timed(m, HERO_K_NORM, st, [&] { return launch_route_norm(ca, na, m->num_sms, st); }));
   } else {
     CUDA_TRY(timed(m, HERO_K_COMPACT, st, [&] { return launch_compact(ca, st); }));
@@ -1089,8 +1138,14 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
   ad.out = m->ah;
   ad.ldo = r;
   ad.err = m->err;
-  ad.A = m->u_a;
+  ad.A = spec ? m->u_f : m->u_a;
   ad.lda = d;
+  if (spec) {   // every token through both branches, rows in token order
+    gu.m_dev = nullptr;
+    gu.m_static = T;
+    ad.m_dev = nullptr;
+    ad.m_static = T;
+  }
   ad.B = static_cast<const char*>(m->w1) + (size_t)jj * r * d * es;
   ad.ldb = d;
   GemmArgs dn{};
@@ -1124,11 +1179,12 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
                      : launch_gemm_tc2_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu_p[jj], gu, EPI_SILU,
                                             m->tm_ua, m->tm_w1_p[jj], ad, m->num_sms, st);
       return dense ? launch_gemm_tc(256, EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, m->num_sms, st)
-                   : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU, m->tm_ua,
-                                         m->tm_w1[jj], ad, m->num_sms, st);
+                   : launch_gemm_tc_pair(EPI_SWIGLU, m->tm_uf, m->tm_wgu[jj], gu, EPI_SILU,
+                                         spec ? m->tm_uf : m->tm_ua, m->tm_w1[jj], ad, m->num_sms,
+                                         st);
     }));
-    const int m_t = (T + 127) / 128;
-    const int ds = choose_splits(m_t * (d / 256), (I + 63) / 64, m->num_sms, (long)m_t * 128, d, 22);
+    const int m_t = m_t0;
+    const int ds = ds0;
     // few rows and a split FFN down: the adapter rows close in FFN down's finishing launch
     const bool adapter_in_close = !dense && T <= 256 && r <= 64 && r % 8 == 0 && ds > 1;
     if (!dense && T <= 256 && r <= 64 && !adapter_in_close) {   // few rows: the FMA-pipe kernel
@@ -1158,6 +1214,10 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
     };
     if (ds > 1) {   // few tiles (small T): split K into partials, then the closing epilogue
       GemmArgs sk = dn;
+      if (spec) {
+        sk.m_dev = nullptr;
+        sk.m_static = T;
+      }
       sk.out_f32 = m->splitk_ws;
       sk.ldo = d;
       sk.k_splits = ds;
@@ -1165,10 +1225,12 @@ hero_status block_body(hero_model* m, int jj, int jr, int T, const BlockState& b
       CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
         return launch_gemm_tc(256, EPI_STORE_F32, m->tm_act, m->tm_wd[jj], sk, m->num_sms, st);
       }));
+      if (spec) CUDA_TRY(cudaStreamWaitEvent(st, m->ev_join, 0));   // the decisions
       CUDA_TRY(timed(m, HERO_K_FFN_DOWN, st, [&] {
         SplitkAdapter sa{};
         if (adapter_in_close)
-          sa = SplitkAdapter{m->ah, static_cast<const char*>(m->w2) + (size_t)jj * d * r * es, r, au.lo};
+          sa = SplitkAdapter{m->ah, static_cast<const char*>(m->w2) + (size_t)jj * d * r * es, r,
+                             au.lo, spec ? 1 : 0};
         return launch_splitk_close(m->splitk_ws, ds, sk.split_stride, d, m->counts, T, dn.lo, sa, st);
       }));
       return adapter_after ? adapter_up_wide(0) : HERO_OK;
@@ -1323,7 +1385,8 @@ extern "C" hero_status hero_routed_ffn_stack(hero_model* m, int64_t n_tokens, co
   if (n_tokens < 0 || n_tokens > c.max_tokens)
     return fail(HERO_ERR_ARG, "n_tokens %lld outside [0, max_tokens=%d]", (long long)n_tokens,
                 c.max_tokens);
-  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO))
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO |
+                          HERO_FLAG_NO_SPECULATE))
     return fail(HERO_ERR_ARG, "unknown flag bits 0x%x", flags);
   if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
     return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
@@ -1554,8 +1617,9 @@ extern "C" hero_status hero_routed_block(hero_model* m, int32_t block, int64_t n
   if (n_tokens < 0 || n_tokens > c.max_tokens)
     return fail(HERO_ERR_ARG, "n_tokens %lld outside [0, max_tokens=%d]", (long long)n_tokens,
                 c.max_tokens);
-  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK))
-    return fail(HERO_ERR_ARG, "hero_routed_block takes only HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK");
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_NO_SPECULATE))
+    return fail(HERO_ERR_ARG, "hero_routed_block takes only HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK "
+                              "or HERO_FLAG_NO_SPECULATE");
   if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
     return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");
   bool dense = (flags & HERO_FLAG_DENSE) || block <= c.n_dense;
@@ -1839,7 +1903,8 @@ hero_status check_decoder_args(hero_model* m, int T, const float* h_in, float ta
                                uint32_t flags, const uint8_t* mask_in, const float* h_out,
                                int32_t* ffn_count_out, void* cuda_stream) {
   const int L = m->cfg.n_layers;
-  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO))
+  if (flags & ~(uint32_t)(HERO_FLAG_DENSE | HERO_FLAG_FORCE_MASK | HERO_FLAG_HOST_IO |
+                          HERO_FLAG_NO_SPECULATE))
     return fail(HERO_ERR_ARG, "unknown flag bits 0x%x", flags);
   if ((flags & HERO_FLAG_DENSE) && (flags & HERO_FLAG_FORCE_MASK))
     return fail(HERO_ERR_ARG, "HERO_FLAG_DENSE and HERO_FLAG_FORCE_MASK are exclusive");

@@ -410,7 +410,7 @@ cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
 
 struct NormArgs {
   int T, d, np;
-  const int* counts;
+  const int* counts;     // [2] n_f, n_a; nullptr: every token's row into u_f, in token order
   const int* idx_f;
   const int* idx_a;
   const float* hbar;
@@ -464,6 +464,9 @@ struct SplitkAdapter {
   const void* w2;       // bf16 [d, d_r]
   int d_r;
   LayerOutArgs lo;
+  // 1: the FFN partial rows and the rows of ah are tokens (both branches ran on every
+  // token); row m of the FFN branch reads token idx_f[m]'s rows, adapter row m token idx_a[m]'s
+  int by_token;
 };
 cudaError_t launch_splitk_close(const float* part, int splits, long split_stride, int ld,
                                 const int* m_dev, int m_max, const LayerOutArgs& lo,

@@ -823,11 +823,15 @@ __global__ void __launch_bounds__(256) k_norm(const NormArgs a, int wpr) {
   const int part = (int)(gw - slot * wpr);
   const int lane = threadIdx.x & 31;
   if (slot >= a.T) return;
-  const int nf = a.counts[0];
+  const int nf = a.counts ? a.counts[0] : a.T;   // no counts: every token, in token order
   int t;
   void* dst;
   long r;
-  if (slot < nf) {
+  if (!a.counts) {
+    t = (int)slot;
+    dst = a.u_f;
+    r = slot;
+  } else if (slot < nf) {
     t = a.idx_f[slot];
     dst = a.u_f;
     r = slot;

@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
   const LayerOutIn in = layer_out_load(p, t, n);   // in flight with the loads below
   float4 y;
   if (ffn) {
-    const size_t off = (size_t)m * ld + n;
+    const size_t off = (size_t)(ad.by_token ? t : m) * ld + n;
     y = *reinterpret_cast<const float4*>(part + off);
     // up to 8 slices' loads in flight, added in slice order
     for (int s0 = 1; s0 < splits; s0 += 8) {
@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(256) k_splitk_close(const float* __restrict__ 
         }
     }
   } else {   // adapter row: y = W_2 ah[row] over the lane's 4 columns
-    const uint16_t* ar = static_cast<const uint16_t*>(ad.ah) + (size_t)row * ad.d_r;
+    const uint16_t* ar = static_cast<const uint16_t*>(ad.ah) + (size_t)(ad.by_token ? t : row) * ad.d_r;
     const uint16_t* wr = static_cast<const uint16_t*>(ad.w2) + (size_t)n * ad.d_r;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 8
@@ -200,6 +200,7 @@ cudaError_t launch_splitk_close(const float* part, int splits, long split_stride
   if (m_max <= 0) return cudaSuccess;
   if (lo.d % kTcPartCols) return cudaErrorInvalidValue;
   if (ad.ah && (ad.d_r <= 0 || ad.d_r % 8 || !ad.w2 || ad.lo.d != lo.d)) return cudaErrorInvalidValue;
+  if (ad.by_token && !ad.ah) return cudaErrorInvalidValue;
   const long warps = (long)m_max * (lo.d / kTcPartCols);
   return launch_pdl(k_splitk_close, dim3((unsigned)((warps + 7) / 8)), dim3(256), 0, st, part, splits,
                     split_stride, ld, m_dev, m_max, lo, ad);

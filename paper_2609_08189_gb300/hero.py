@@ -22,7 +22,7 @@ LIB_PATH = os.path.join(_PKG, "libhero.so")
 STATUS_NAMES = {0: "HERO_OK", 1: "HERO_ERR_ARG", 2: "HERO_ERR_CUDA", 3: "HERO_ERR_NOMEM",
                 4: "HERO_ERR_UNSUPPORTED", 5: "HERO_ERR_TIMEOUT", 6: "HERO_ERR_BAD_INDEX"}
 HERO_F32, HERO_BF16 = 0, 1
-HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO = 1, 2, 4
+HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK, HERO_FLAG_HOST_IO, HERO_FLAG_NO_SPECULATE = 1, 2, 4, 8
 HERO_ROUTER_NO_HISTORY, HERO_ROUTER_NO_MEMREAD, HERO_ROUTER_NO_AUX, HERO_ROUTER_NO_POS = 1, 2, 4, 8
 KERNEL_CLASSES = ("init", "router_gemm", "router", "compact", "norm", "ffn_gate_up", "ffn_down",
                   "adapter_down", "adapter_up", "attn_proj", "attn_core", "backward_gemm",
