@@ -39,6 +39,18 @@ def test_header_declares_the_boundary():
         assert n in names
 
 
+def test_binding_flags_match_the_header(H):
+    """The binding's HERO_FLAG_* constants are the header's enum values."""
+    src = open(os.path.join(ROOT, "include", "hero.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    flags = {n: int(v) for n, v in re.findall(r"(HERO_FLAG_\w+)\s*=\s*(\d+)u", src)}
+    assert set(flags) == {"HERO_FLAG_DENSE", "HERO_FLAG_FORCE_MASK", "HERO_FLAG_HOST_IO",
+                          "HERO_FLAG_NO_SPECULATE"}
+    for n, v in flags.items():
+        assert getattr(H, n) == v, n
+    assert len(set(flags.values())) == len(flags) and all(v & (v - 1) == 0 for v in flags.values())
+
+
 def test_library_exports_every_declared_symbol(H):
     lib = ctypes.CDLL(H.LIB_PATH)
     missing = [n for n in declared_functions() if not hasattr(lib, n)]
