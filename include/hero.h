@@ -207,7 +207,8 @@ hero_status hero_router_state_reset(hero_model* m, int64_t n_tokens, const hero_
  * (Eq. 1); blocks 1..n_dense are plain FFN blocks (state unused, may be NULL),
  * block n_dense + j is routed block j.  Reads then updates `state` (read before write,
  * Eqs. 11-12) and writes h_out [T,d] = h_bar + g FFN(u) or h_bar + (1-g)
- * Adapter(u) (Eq. 3).  flags: HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK (mask_in [T]).
+ * Adapter(u) (Eq. 3).  flags: HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK (mask_in [T]),
+ * optionally HERO_FLAG_NO_SPECULATE.
  * gate_out [T], mask_out [T], ffn_count_out [1] may be NULL.  h_out must not
  * alias h_bar.  Same error and stream conventions as hero_routed_ffn_stack;
  * host pointers are not accepted here. */
@@ -280,7 +281,7 @@ hero_status hero_attention_block(hero_model* m, int32_t layer, int32_t n_seqs, i
  * blocks 1..n_dense are plain FFN blocks), the router state carried in the model's
  * workspace and reset at the start.  h_in [T,d] -> h_out [T,d] fp32; tau_exec,
  * flags (HERO_FLAG_DENSE or HERO_FLAG_FORCE_MASK with mask_in [L,T], optionally
- * HERO_FLAG_HOST_IO), gate_out [L,T], mask_out [L,T], ffn_count_out [L] as
+ * HERO_FLAG_HOST_IO and HERO_FLAG_NO_SPECULATE), gate_out [L,T], mask_out [L,T], ffn_count_out [L] as
  * hero_routed_ffn_stack (NULL allowed).  DEVICE pointers, or HOST pointers with
  * HERO_FLAG_HOST_IO (copied on the stream); h_out must not alias h_in.
  * n_seqs <= 65535. */
@@ -321,7 +322,7 @@ hero_status hero_decoder_prefill(hero_model* m, int32_t seq0, int32_t n_seqs, in
  * by hero_check_device_status).  h_in [n_seqs,d] are the new tokens' inputs;
  * tau_exec, flags (HERO_FLAG_DENSE, HERO_FLAG_FORCE_MASK with mask_in
  * [L,n_seqs], HERO_FLAG_HOST_IO: h_in, positions, mask_in and the outputs are
- * host pointers) and the outputs as hero_decoder_forward with T = n_seqs.
+ * host pointers; HERO_FLAG_NO_SPECULATE) and the outputs as hero_decoder_forward with T = n_seqs.
  * Precision: as hero_attention_block, except that the softmax probabilities
  * enter P V in fp32. */
 hero_status hero_decode_step(hero_model* m, int32_t n_seqs, const int32_t* positions,
